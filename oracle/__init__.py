@@ -1,0 +1,154 @@
+"""CPU oracle for the UniSVQ linear layer (TEST INFRASTRUCTURE ONLY).
+
+Plain, slow, fp64 NumPy restatement of what the inference-time UniSVQ linear
+layer computes. Only `tests/`, `__graft_entry__.smoke()` and the CPU-baseline
+legs of `bench.py` may import it; the product library never does, and this
+package imports nothing from the product.
+
+Every function cites the passage of the paper it follows:
+
+* Eq. (def:unisvq), Sec. 3.1 -- one length-d weight vector is the affine image
+  A z + B of an integer lattice point z (coordinates in {0,1,2,3} for 2 bits).
+* Eq. (col:dequant), Sec. 3.2.3 -- the dequantised W^T stacks, for each group i
+  of d input columns, the block A W_int,i^T + B 1^T: the vectors run along the
+  input dimension and one (A, B) serves the whole weight matrix.
+* Eq. (col:matmul), Sec. 3.2.3 -- Y = X W^T = sum_i (X_i A) W_int,i^T
+  + sum_i (X_i B) 1^T (the fold of the affine onto the activations).
+* Eq. (def:ptq_loss), Sec. 2.1 -- the layer output is Y = X W^T with X tokens x
+  inputs and W outputs x inputs.
+
+Inputs are exactly widened to fp64 (bf16 activations, fp16 affine). Where the
+paper fixes no rounding, the oracle keeps everything exact in fp64 and rounds
+once at the very end (`dequant_f32`).
+
+Pins (tests/test_oracle_pins.py): exhaustive codebook enumeration with the
+orthogonal initial grid (mean 0, covariance I, App. A.1), the scalar
+quantisation special case (Eq. def:sq), an integer-matrix case checked against
+exact Python integers, the hand-worked example in tests/golden/, linearity in
+x, agreement of Eq. (col:dequant) with Eq. (def:unisvq), and the fold
+identity of Eq. (col:matmul). No function here is "parity unpinned".
+"""
+from __future__ import annotations
+
+import numpy as np
+
+# Tolerances for comparing a layer output against the oracle (per element and
+# over the whole tensor); see `compare`.
+ABS_REL_BOUND = 2.0 ** -7
+ABS_FLOOR = 1e-6
+REL_L2_BOUND = 4e-3
+
+
+def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
+    """Exact widening of bf16 bit patterns (uint16) to float64."""
+    b = np.ascontiguousarray(bits, dtype=np.uint16).astype(np.uint32) << 16
+    return b.view(np.float32).astype(np.float64)
+
+
+def as_f64(a) -> np.ndarray:
+    """Exact widening of fp16 / fp32 / fp64 arrays to float64."""
+    return np.asarray(a).astype(np.float64)
+
+
+def _check(codes: np.ndarray, A: np.ndarray, B: np.ndarray):
+    d = A.shape[0]
+    if A.shape != (d, d) or B.shape != (d,):
+        raise ValueError("A must be d x d and B length d")
+    if codes.ndim != 2 or codes.shape[1] % d:
+        raise ValueError("codes must be [N][K] with K a multiple of d")
+    return d
+
+
+def codeword(z, A, B) -> np.ndarray:
+    """Eq. (def:unisvq): the weight vector A z + B of one lattice point z."""
+    A = as_f64(A)
+    B = as_f64(B)
+    return A @ np.asarray(z, dtype=np.float64) + B
+
+
+def codebook(A, B) -> np.ndarray:
+    """All 4^d codewords, row v = A z(v) + B with z_c(v) = (v >> 2c) & 3.
+
+    Eq. (def:unisvq) evaluated on every point of {0,1,2,3}^d; coordinate c of
+    the lattice point is bit-field [2c+1:2c] of the vector index v.
+    """
+    d = np.asarray(A).shape[0]
+    v = np.arange(4 ** d)
+    Z = np.stack([(v >> (2 * c)) & 3 for c in range(d)], axis=1).astype(np.float64)
+    return Z @ as_f64(A).T + as_f64(B)
+
+
+def dequant(codes: np.ndarray, A, B) -> np.ndarray:
+    """Dequantised weights W_hat [N][K] in fp64.
+
+    Eq. (def:unisvq) applied to every vector: for output row n and input group
+    g (columns g*d .. g*d+d-1), W_hat[n, g*d + r] = sum_c A[r, c] z[n, g*d + c]
+    + B[r], the column-vector form of the blocks of Eq. (col:dequant).
+    """
+    d = _check(codes, np.asarray(A), np.asarray(B))
+    N, K = codes.shape
+    Z = codes.reshape(N, K // d, d).astype(np.float64)
+    W = Z @ as_f64(A).T + as_f64(B)
+    return W.reshape(N, K)
+
+
+def dequant_f32(codes: np.ndarray, A, B) -> np.ndarray:
+    """RN-to-fp32 of the exact fp64 dequantised weights (a single rounding)."""
+    return dequant(codes, A, B).astype(np.float32)
+
+
+def linear(x: np.ndarray, codes: np.ndarray, A, B, row_chunk: int = 4096):
+    """Layer output y = x W_hat^T and the tolerance scale S = |x| |W_hat|^T.
+
+    Eq. (def:ptq_loss): Y = X W^T with X [M][K] and W [N][K]. `x` is either
+    bf16 bits (uint16) or a float array. Rows of W are dequantised in chunks so
+    large layers never hold a full fp64 W.
+    Returns (y, S), both float64 [M][N].
+    """
+    xf = bf16_bits_to_f64(x) if x.dtype == np.uint16 else as_f64(x)
+    M = xf.shape[0]
+    N = codes.shape[0]
+    y = np.empty((M, N))
+    S = np.empty((M, N))
+    ax = np.abs(xf)
+    for r0 in range(0, N, row_chunk):
+        W = dequant(codes[r0:r0 + row_chunk], A, B)
+        y[:, r0:r0 + W.shape[0]] = xf @ W.T
+        S[:, r0:r0 + W.shape[0]] = ax @ np.abs(W).T
+    return y, S
+
+
+def linear_folded(x: np.ndarray, codes: np.ndarray, A, B) -> np.ndarray:
+    """Eq. (col:matmul): y = sum_i (X_i A) W_int,i^T + sum_i (X_i B) 1^T.
+
+    X_i is the [M][d] slice of inputs i*d .. i*d+d-1 and W_int,i the matching
+    [N][d] slice of the integer codes. fp64 throughout.
+    """
+    d = _check(codes, np.asarray(A), np.asarray(B))
+    xf = bf16_bits_to_f64(x) if x.dtype == np.uint16 else as_f64(x)
+    M, K = xf.shape
+    Xi = xf.reshape(M, K // d, d)
+    XA = (Xi @ as_f64(A)).reshape(M, K)          # the row vectors X_i A
+    XB = (Xi @ as_f64(B)).sum(axis=1)            # sum_i X_i B, one scalar per token
+    return XA @ codes.astype(np.float64).T + XB[:, None]
+
+
+def compare(y: np.ndarray, y_ref: np.ndarray, S: np.ndarray) -> dict:
+    """Check a layer output against the oracle.
+
+    Per element |y - y_ref| <= 2^-7 * S + 1e-6 (S = sum_k |W_hat x|), and the
+    relative L2 error over the tensor must not exceed 4e-3.
+    """
+    y = np.asarray(y, dtype=np.float64)
+    err = np.abs(y - y_ref)
+    bound = ABS_REL_BOUND * S + ABS_FLOOR
+    ratio = np.max(err / bound) if err.size else 0.0
+    nref = np.linalg.norm(y_ref)
+    rel_l2 = float(np.linalg.norm(y - y_ref) / nref) if nref > 0 else float(np.linalg.norm(y - y_ref))
+    finite = bool(np.all(np.isfinite(y)))
+    return {
+        "max_err_over_bound": float(ratio),
+        "rel_l2": rel_l2,
+        "finite": finite,
+        "ok": finite and ratio <= 1.0 and rel_l2 <= REL_L2_BOUND,
+    }

@@ -1,0 +1,291 @@
+"""Pins of the CPU oracle to facts the paper and mathematics fix (no GPU).
+
+Each pin is written as a function of the dequantisation / layer routine under
+test, so `test_pins_catch_planted_mistakes` can run the same pins against
+deliberately broken copies of the oracle and show each mistake is caught.
+"""
+import itertools
+import json
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "hand_worked.json")
+
+
+# --------------------------------------------------------------------------
+# pin functions: each returns None on success, raises AssertionError otherwise
+# --------------------------------------------------------------------------
+
+def haar_orthogonal(d, seed):
+    """Haar-distributed orthogonal matrix (QR of a Gaussian with sign fix)."""
+    g = np.random.default_rng(seed)
+    Q, R = np.linalg.qr(g.standard_normal((d, d)))
+    return Q * np.sign(np.diag(R))
+
+
+def pin_enumeration_moments(dequant_fn, d, seed=0):
+    """App. A.1: with A = sG (G orthogonal), B = -sG b 1, b = (2^2-1)/2 and
+    s = sqrt(12/(2^4-1)), the 4^d codewords, each taken once (the uniform law
+    on {0..3}^d), have mean exactly 0 and covariance exactly I."""
+    G = haar_orthogonal(d, seed)
+    bits = 2
+    b = (2 ** bits - 1) / 2
+    s = np.sqrt(12.0 / (2 ** (2 * bits) - 1))
+    A = s * G
+    B = -s * G @ (b * np.ones(d))
+    pts = np.array(list(itertools.product(range(4), repeat=d)), dtype=np.uint8)
+    W = dequant_fn(pts, A, B)            # one codeword per row (K = d)
+    mean = W.mean(axis=0)
+    cov = (W - mean).T @ (W - mean) / W.shape[0]
+    assert np.allclose(mean, 0.0, atol=1e-12), mean
+    assert np.allclose(cov, np.eye(d), atol=1e-12), cov
+
+
+def pin_sq_special_case(dequant_fn, d=4, seed=1):
+    """Eq. (def:sq): with A = s I and B = -s zp 1 the grid is scalar
+    quantisation. Re-quantising W_hat with the SQ rule must give back the
+    codes (clamp inactive), and SQ dequantisation s (q - zp) must equal W_hat."""
+    g = np.random.default_rng(seed)
+    s, zp = 0.0625, 1.5
+    codes = g.integers(0, 4, size=(7, 8 * d), dtype=np.uint8)
+    W = dequant_fn(codes, s * np.eye(d), -s * zp * np.ones(d))
+    q = np.clip(np.rint(W / s + zp), 0, 3)          # Phi_SQ quantiser
+    assert np.array_equal(q.astype(np.uint8), codes)
+    assert np.array_equal(W, s * (q - zp))           # Phi_SQ dequantiser
+
+
+def pin_block_form(dequant_fn, d, seed=2):
+    """Eq. (col:dequant) builds W^T by stacking, for each group i of d input
+    columns, the block A W_int,i^T + B 1^T. Built here with exact rationals
+    and explicit loops; it must equal the per-vector Eq. (def:unisvq) form."""
+    g = np.random.default_rng(seed)
+    N, K = 3, 3 * d
+    A = g.integers(-3, 4, size=(d, d)).astype(np.float64) / 4
+    B = g.integers(-3, 4, size=d).astype(np.float64) / 8
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    Af = [[Fraction(v) for v in row] for row in A]
+    Bf = [Fraction(v) for v in B]
+    WT = []                                            # rows of W^T (K of them)
+    for i in range(K // d):
+        Wi = [[int(codes[n, i * d + c]) for c in range(d)] for n in range(N)]  # W_int,i [N][d]
+        for r in range(d):                             # block row r = (A W_int,i^T + B 1^T)[r]
+            WT.append([sum(Af[r][c] * Wi[n][c] for c in range(d)) + Bf[r] for n in range(N)])
+    Wref = np.array([[float(WT[k][n]) for k in range(K)] for n in range(N)])
+    assert np.array_equal(dequant_fn(codes, A, B), Wref)
+
+
+def pin_integer_layer_exact(linear_fn, seed=3):
+    """The printed D4 generator (App. A.2) is an integer, non-symmetric A:
+    with integer B and small integer x every product is an exact integer, so
+    the layer output must equal exact integer arithmetic done with Python
+    ints on the block form of Eq. (col:dequant)."""
+    d = 4
+    A = np.array([[1, -1, 0, 0], [0, 1, -1, 0], [0, 0, 1, -1], [0, 0, 1, 1]], dtype=np.float64)
+    B = np.array([1, -2, 0, 3], dtype=np.float64)
+    g = np.random.default_rng(seed)
+    N, K, M = 5, 12, 3
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    x = g.integers(-5, 6, size=(M, K)).astype(np.float64)
+    Ai = A.astype(int).tolist()
+    Bi = B.astype(int).tolist()
+    yref = np.zeros((M, N))
+    for m in range(M):
+        for n in range(N):
+            acc = 0
+            for i in range(K // d):
+                for r in range(d):
+                    w = sum(Ai[r][c] * int(codes[n, i * d + c]) for c in range(d)) + Bi[r]
+                    acc += int(x[m, i * d + r]) * w
+            yref[m, n] = acc
+    y = linear_fn(x, codes, A, B)
+    assert np.array_equal(y, yref), (y, yref)
+
+
+def pin_golden(dequant_fn, linear_fn):
+    """Hand-worked examples in tests/golden/hand_worked.json."""
+    with open(GOLDEN) as f:
+        cases = json.load(f)["cases"]
+    for c in cases:
+        A = np.array(c["A"])
+        B = np.array(c["B"])
+        codes = np.array(c["codes"], dtype=np.uint8)
+        x = np.array(c["x"])
+        assert np.array_equal(dequant_fn(codes, A, B), np.array(c["W"])), c["name"]
+        assert np.array_equal(linear_fn(x, codes, A, B), np.array(c["y"])), c["name"]
+
+
+def pin_linearity(linear_fn, seed=4):
+    """The layer is linear in x: y(a x1 + b x2) = a y(x1) + b y(x2)."""
+    g = np.random.default_rng(seed)
+    codes = g.integers(0, 4, size=(9, 16), dtype=np.uint8)
+    A = g.standard_normal((2, 2))
+    B = g.standard_normal(2)
+    x1 = g.standard_normal((3, 16))
+    x2 = g.standard_normal((3, 16))
+    lhs = linear_fn(0.75 * x1 - 1.25 * x2, codes, A, B)
+    rhs = 0.75 * linear_fn(x1, codes, A, B) - 1.25 * linear_fn(x2, codes, A, B)
+    assert np.allclose(lhs, rhs, rtol=1e-12, atol=1e-12)
+
+
+def oracle_linear_y(x, codes, A, B):
+    return oracle.linear(np.asarray(x, dtype=np.float64), codes, A, B)[0]
+
+
+# --------------------------------------------------------------------------
+# the pins, applied to the oracle
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("d", [1, 2, 4, 8])
+def test_enumeration_moments(d):
+    pin_enumeration_moments(oracle.dequant, d)
+
+
+def test_sq_special_case():
+    pin_sq_special_case(oracle.dequant)
+
+
+@pytest.mark.parametrize("d", [1, 2, 4])
+def test_block_form_matches_vector_form(d):
+    pin_block_form(oracle.dequant, d)
+
+
+def test_integer_layer_exact():
+    pin_integer_layer_exact(oracle_linear_y)
+
+
+def test_golden_hand_worked():
+    pin_golden(oracle.dequant, oracle_linear_y)
+    with open(GOLDEN) as f:
+        for c in json.load(f)["cases"]:
+            y, S = oracle.linear(np.array(c["x"]), np.array(c["codes"], dtype=np.uint8),
+                                 np.array(c["A"]), np.array(c["B"]))
+            assert np.array_equal(S, np.array(c["S"]))
+
+
+def test_linearity():
+    pin_linearity(oracle_linear_y)
+
+
+@pytest.mark.parametrize("d", [1, 2, 4])
+def test_fold_identity(d):
+    """Eq. (col:matmul) (fold onto activations) equals the direct form."""
+    g = synth.rng(0, 99, d)
+    codes = synth.gen_codes(g, 33, 64 * d)
+    A, B = synth.gen_affine(g, d)
+    x = synth.gen_activations(g, 5, 64 * d)
+    y, S = oracle.linear(x, codes, A, B)
+    yf = oracle.linear_folded(x, codes, A, B)
+    assert np.allclose(yf, y, rtol=1e-11, atol=1e-11 * np.abs(S).max())
+
+
+def test_codebook_is_dequant_of_every_index():
+    """`codebook` row v is the dequantisation of the lattice point whose
+    coordinate c is bit-field [2c+1:2c] of v."""
+    for d in (1, 2, 4):
+        g = np.random.default_rng(d)
+        A = g.standard_normal((d, d))
+        B = g.standard_normal(d)
+        v = np.arange(4 ** d)
+        pts = np.stack([(v >> (2 * c)) & 3 for c in range(d)], axis=1).astype(np.uint8)
+        cb = oracle.codebook(A, B)
+        assert np.allclose(cb, oracle.dequant(pts, A, B), rtol=0, atol=1e-14 * np.abs(cb).max())
+
+
+def test_dequant_f32_single_rounding():
+    g = np.random.default_rng(5)
+    codes = g.integers(0, 4, size=(4, 8), dtype=np.uint8)
+    A, B = synth.gen_affine(g, 2)
+    W = oracle.dequant(codes, A, B)
+    W32 = oracle.dequant_f32(codes, A, B)
+    assert W32.dtype == np.float32
+    assert np.all(np.abs(W32.astype(np.float64) - W) <= np.abs(W) * 2.0 ** -24)
+
+
+def test_compare_accepts_and_rejects():
+    g = np.random.default_rng(6)
+    y = g.standard_normal((4, 8))
+    S = np.abs(y) + 1.0
+    assert oracle.compare(y, y, S)["ok"]
+    bad = y.copy()
+    bad[1, 3] += 0.1 * S[1, 3]
+    assert not oracle.compare(bad, y, S)["ok"]
+
+
+# --------------------------------------------------------------------------
+# planted mistakes: each broken oracle must fail at least one pin
+# --------------------------------------------------------------------------
+
+def _mut_dequant(kind):
+    def f(codes, A, B):
+        A = np.asarray(A, dtype=np.float64)
+        B = np.asarray(B, dtype=np.float64)
+        d = A.shape[0]
+        N, K = codes.shape
+        if kind == "transpose_A":
+            A = A.T
+        if kind == "drop_B":
+            B = 0 * B
+        if kind == "neg_B":
+            B = -B
+        Z = codes.reshape(N, K // d, d).astype(np.float64)
+        if kind == "reverse_coords":
+            Z = Z[..., ::-1]
+        if kind == "vectors_along_output" and N % d == 0:
+            Z = codes.T.reshape(K, N // d, d).astype(np.float64)
+            W = (Z @ A.T + B).reshape(K, N).T
+            return W
+        W = Z @ A.T + B
+        if kind == "scale_off":
+            W = W * (1 + 2.0 ** -20)
+        return W.reshape(N, K)
+    return f
+
+
+def _linear_from(dequant_fn):
+    def f(x, codes, A, B):
+        return np.asarray(x, dtype=np.float64) @ dequant_fn(codes, A, B).T
+    return f
+
+
+@pytest.mark.parametrize("kind", ["transpose_A", "drop_B", "neg_B", "reverse_coords",
+                                  "vectors_along_output", "scale_off"])
+def test_pins_catch_planted_mistakes(kind):
+    dq = _mut_dequant(kind)
+    lin = _linear_from(dq)
+    checks = [
+        lambda: pin_enumeration_moments(dq, 2),
+        lambda: pin_enumeration_moments(dq, 4),
+        lambda: pin_sq_special_case(dq),
+        lambda: pin_block_form(dq, 2),
+        lambda: pin_block_form(dq, 4),
+        lambda: pin_integer_layer_exact(lin),
+        lambda: pin_golden(dq, lin),
+    ]
+    failed = 0
+    for chk in checks:
+        try:
+            chk()
+        except (AssertionError, ValueError):
+            failed += 1
+    assert failed >= 1, f"planted mistake {kind!r} passed every pin"
+
+
+def test_synth_code_probabilities():
+    c = synth.gen_codes(synth.rng(0, 1), 512, 1024)
+    p = np.bincount(c.ravel(), minlength=4) / c.size
+    assert np.allclose(p, synth.CODE_PROBS, atol=3e-3)
+    assert c.max() <= 3
+
+
+def test_synth_bf16_rounding_matches_torch():
+    torch = pytest.importorskip("torch")
+    v = np.random.default_rng(7).standard_normal(4096).astype(np.float32) * 37
+    ours = synth.f32_to_bf16_bits(v)
+    ref = torch.from_numpy(v).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(ours, ref)
