@@ -1,0 +1,165 @@
+/*
+ * libunisvq -- GB300 (sm_103a) inference kernels for the UniSVQ linear layer.
+ *
+ * The method (UniSVQ, "2-bit Unified Scalar-Vector Quantization"):
+ *   - Eq. (def:unisvq), Sec. 3.1: a length-d weight vector is stored as a
+ *     lattice point z in {0,1,2,3}^d and reconstructed as w = A z + B, with
+ *     A a d x d matrix and B a d-vector.
+ *   - Eq. (col:dequant), Sec. 3.2.3: the vectors run along the INPUT dimension
+ *     of the weight matrix and one (A, B) serves the whole matrix, i.e.
+ *     W_hat[n, g*d + r] = sum_c A[r][c] * z[n, g*d + c] + B[r].
+ *   - Eq. (col:matmul), Sec. 3.2.3: the layer Y = X W_hat^T can be computed as
+ *     sum_i (X_i A) W_int,i^T + sum_i (X_i B) 1^T without a dequantised W.
+ *
+ * Shapes: x [M][K] bf16 (tokens x inputs), codes [N][K] (outputs x inputs),
+ * y [M][N] bf16. d in {1, 2, 4}. No entry point ever writes a dequantised
+ * weight matrix to device memory, except the test hook unisvq_dequant_debug.
+ *
+ * Streams are passed as `void*` holding a cudaStream_t (NULL = legacy default
+ * stream). Device pointers are plain CUDA device addresses.
+ *
+ * Errors: every entry point validates its arguments before touching the GPU
+ * and returns a status; nothing aborts the process. CUDA runtime failures map
+ * to UNISVQ_ERR_CUDA. Kernels bound every wait; a wait that runs out sets a
+ * device error word that unisvq_sync_status reports as UNISVQ_ERR_TIMEOUT.
+ */
+#ifndef UNISVQ_H_
+#define UNISVQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  UNISVQ_OK = 0,
+  UNISVQ_ERR_INVALID_ARG = 1,
+  UNISVQ_ERR_UNSUPPORTED = 2,
+  UNISVQ_ERR_CUDA = 3,
+  UNISVQ_ERR_OOM = 4,
+  UNISVQ_ERR_TIMEOUT = 5
+} unisvq_status;
+
+/* Kernel selectors for unisvq_linear_force and unisvq_info.kernel. */
+enum {
+  UNISVQ_KERNEL_AUTO = 0,    /* pick by M (unisvq_linear does this)            */
+  UNISVQ_KERNEL_DECODE = 1,  /* fold + register-unpack tensor-core GEMV, M<=32 */
+  UNISVQ_KERNEL_PREFILL = 2  /* tcgen05 GEMM, bf16 codeword tiles in smem      */
+};
+
+/*
+ * Packed device layout of the codes (written by unisvq_pack, documented so
+ * that other tools can produce or check it).
+ *
+ * The matrix is padded to Np = roundup(N, 128) rows and Kp = roundup(K, 128)
+ * columns with code 0 and cut into tiles of 16 rows x 128 columns, 512 bytes
+ * each. Tile (rt, kt), rt < Np/16, kt < Kp/128, starts at byte
+ * (rt * (Kp/128) + kt) * 512, so the tiles of one 16-row strip are
+ * consecutive along K.
+ *
+ * Inside a tile, lane l in [0, 32) owns bytes [16 l, 16 l + 16) as four
+ * little-endian 32-bit words W[q], q in [0, 4). With g = l / 4, t = l % 4,
+ * grp = q / 2 and rh = q % 2, word W[q] holds 16 codes of row
+ *   n = 16 rt + g + 8 rh
+ * at 8 positions p in [0, 8): with i = p / 2 and h = p % 2, the column
+ *   k = 128 kt + 64 grp + 16 i + 4 t + 2 h
+ * sits in bits [2p+1 : 2p] and column k + 1 in bits [16+2p+1 : 16+2p].
+ * Every run of 4 columns 4m .. 4m+3 therefore sits in one word, so vectors
+ * of d = 1, 2 or 4 never straddle words.
+ */
+#define UNISVQ_TILE_ROWS 16
+#define UNISVQ_TILE_COLS 128
+#define UNISVQ_TILE_BYTES 512
+
+typedef struct unisvq_layer* unisvq_handle;
+
+typedef struct {
+  int N, K, d;            /* layer shape and vector length                      */
+  int Np, Kp;             /* padded shape of the packed codes                   */
+  int kernel;             /* kernel unisvq_linear runs for this M               */
+  int split_k;            /* CTAs cooperating along K (decode kernel)           */
+  int grid_ctas;          /* CTAs launched                                      */
+  long long code_bytes;   /* packed code bytes resident on the device           */
+  long long meta_bytes;   /* affine parameters: (d*d + d) * 2 bytes (fp16)      */
+  long long algo_bytes;   /* N*K/4 + meta + 2*M*K (x) + 2*M*N (y)               */
+  double flops;           /* 2*M*N*K                                            */
+} unisvq_info;
+
+/*
+ * Pack a quantised weight matrix into a device-resident layer handle.
+ *   codes : host, [N][K] row-major uint8, each 0..3 (lattice coordinates z)
+ *   A_f16 : host, [d][d] row-major IEEE fp16 bit patterns, w = A z + B
+ *   B_f16 : host, [d] fp16 bit patterns
+ *   N, K  : output / input features, N >= 1, K >= d, K % d == 0
+ *   d     : vector length, 1, 2 or 4 (Eq. def:unisvq; the paper uses d = 4)
+ *   stream: stream for the upload; pack synchronises it before returning
+ *   out   : receives the handle
+ * The host buffers are copied before return; the caller keeps ownership.
+ * Errors: INVALID_ARG (null pointer, bad shape, code > 3, non-finite A/B),
+ * UNSUPPORTED (d not in {1,2,4}), OOM, CUDA.
+ * The handle owns all device memory and is immutable afterwards, so
+ * concurrent unisvq_linear calls on different streams are safe.
+ */
+unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
+                          int N, int K, int d, void* stream, unisvq_handle* out);
+
+/*
+ * y = x W_hat^T (Eq. def:ptq_loss with W_hat of Eq. col:dequant).
+ *   x : device, [M][K] row-major bf16, 16-byte aligned
+ *   y : device, [M][N] row-major bf16, 4-byte aligned, must not overlap x
+ *   M : tokens, M >= 0 (M == 0 is a no-op)
+ * Never allocates and never synchronises; enqueues on `stream`. Kernels are
+ * launched with programmatic dependent launch so that, in a stream or a CUDA
+ * graph, a layer starts fetching its codes while the previous kernel finishes;
+ * reads of x and writes of y still wait for the previous kernel to complete.
+ * Errors: INVALID_ARG (null, misaligned, overlap, M < 0), CUDA.
+ */
+unisvq_status unisvq_linear(unisvq_handle h, const void* x, void* y, int M, void* stream);
+
+/* As unisvq_linear but runs the given UNISVQ_KERNEL_* for any M (crossover
+ * sweeps and tests). UNSUPPORTED if that kernel cannot run this shape. */
+unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, void* y, int M,
+                                  void* stream);
+
+/* Test hook: writes W_hat as fp32 [N][K] row-major to device memory W (each
+ * entry RN_fp32 of the exact A z + B), unpacking the device layout with the
+ * same code-extraction helpers the layer kernels use. */
+unisvq_status unisvq_dequant_debug(unisvq_handle h, float* W, void* stream);
+
+/* Describe the launch unisvq_linear would make for M tokens (host only). */
+unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info);
+
+/* Synchronise `stream`, then report and clear the device error word:
+ * UNISVQ_ERR_TIMEOUT if a kernel gave up on a bounded wait since the last
+ * call, UNISVQ_ERR_CUDA on a CUDA error, else UNISVQ_OK. */
+unisvq_status unisvq_sync_status(void* stream);
+
+/* Free the handle and its device memory. NULL is a no-op. The caller must
+ * make sure no work using the handle is still in flight. */
+unisvq_status unisvq_destroy(unisvq_handle h);
+
+/* Device-to-device copy of a packed layer into a new handle. */
+unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out);
+
+const char* unisvq_status_string(unisvq_status s);
+
+/* ---- host-only helpers (no GPU needed) ---------------------------------- */
+
+/* Bytes of the packed code array for an N x K layer (see layout above). */
+size_t unisvq_packed_code_bytes(int N, int K);
+
+/* Write the packed layout of `codes` ([N][K], each 0..3) into the host
+ * buffer `packed` of unisvq_packed_code_bytes(N, K) bytes. */
+unisvq_status unisvq_pack_host(const uint8_t* codes, int N, int K, uint8_t* packed,
+                               size_t packed_bytes);
+
+/* Library version as an integer MAJOR*10000 + MINOR*100 + PATCH. */
+int unisvq_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* UNISVQ_H_ */

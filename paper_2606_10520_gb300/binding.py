@@ -1,0 +1,179 @@
+"""Thin ctypes binding of libunisvq (argument marshalling only).
+
+Every step of the layer runs in the library's CUDA kernels; PyTorch supplies
+device memory (tensors) and the current CUDA stream. If the shared library has
+not been built, `load()` raises instead of falling back to anything else.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libunisvq.so")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM, ERR_TIMEOUT = range(6)
+KERNEL_AUTO, KERNEL_DECODE, KERNEL_PREFILL = 0, 1, 2
+
+# Every function include/unisvq.h declares.
+EXPORTS = [
+    "unisvq_pack", "unisvq_linear", "unisvq_linear_force", "unisvq_dequant_debug",
+    "unisvq_query", "unisvq_sync_status", "unisvq_destroy", "unisvq_clone",
+    "unisvq_status_string", "unisvq_packed_code_bytes", "unisvq_pack_host", "unisvq_version",
+]
+
+
+class UnisvqError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {status_string(status)} (status {status})")
+
+
+class Info(ctypes.Structure):
+    _fields_ = [("N", ctypes.c_int), ("K", ctypes.c_int), ("d", ctypes.c_int),
+                ("Np", ctypes.c_int), ("Kp", ctypes.c_int), ("kernel", ctypes.c_int),
+                ("split_k", ctypes.c_int), ("grid_ctas", ctypes.c_int),
+                ("code_bytes", ctypes.c_longlong), ("meta_bytes", ctypes.c_longlong),
+                ("algo_bytes", ctypes.c_longlong), ("flops", ctypes.c_double)]
+
+
+_lib = None
+
+
+def load():
+    """Load libunisvq.so (built in-tree by `__graft_entry__.build()`)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"libunisvq is not built ({LIB_PATH} missing); run __graft_entry__.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+    lib.unisvq_pack.argtypes = [vp, vp, vp, i, i, i, vp, ctypes.POINTER(vp)]
+    lib.unisvq_linear.argtypes = [vp, vp, vp, i, vp]
+    lib.unisvq_linear_force.argtypes = [vp, i, vp, vp, i, vp]
+    lib.unisvq_dequant_debug.argtypes = [vp, vp, vp]
+    lib.unisvq_query.argtypes = [vp, i, ctypes.POINTER(Info)]
+    lib.unisvq_sync_status.argtypes = [vp]
+    lib.unisvq_destroy.argtypes = [vp]
+    lib.unisvq_clone.argtypes = [vp, vp, ctypes.POINTER(vp)]
+    lib.unisvq_status_string.argtypes = [i]
+    lib.unisvq_status_string.restype = ctypes.c_char_p
+    lib.unisvq_packed_code_bytes.argtypes = [i, i]
+    lib.unisvq_packed_code_bytes.restype = sz
+    lib.unisvq_pack_host.argtypes = [vp, i, i, vp, sz]
+    lib.unisvq_version.argtypes = []
+    _lib = lib
+    return lib
+
+
+def status_string(status: int) -> str:
+    return load().unisvq_status_string(int(status)).decode()
+
+
+def _check(status: int, what: str):
+    if status != OK:
+        raise UnisvqError(status, what)
+
+
+def _stream_ptr(stream=None):
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def packed_code_bytes(N: int, K: int) -> int:
+    return int(load().unisvq_packed_code_bytes(N, K))
+
+
+def pack_host(codes: np.ndarray) -> np.ndarray:
+    """Packed device layout of `codes` ([N][K] uint8), computed on the host."""
+    codes = np.ascontiguousarray(codes, dtype=np.uint8)
+    N, K = codes.shape
+    out = np.zeros(packed_code_bytes(N, K), dtype=np.uint8)
+    _check(load().unisvq_pack_host(codes.ctypes.data, N, K, out.ctypes.data, out.nbytes), "pack_host")
+    return out
+
+
+def _f16_bits(a) -> np.ndarray:
+    a = np.asarray(a)
+    if a.dtype == np.uint16:
+        return np.ascontiguousarray(a)
+    return np.ascontiguousarray(a.astype(np.float16)).view(np.uint16)
+
+
+def sync_status(stream=None) -> int:
+    return int(load().unisvq_sync_status(_stream_ptr(stream)))
+
+
+class UniSVQLinear:
+    """One packed UniSVQ linear layer resident on the current CUDA device."""
+
+    def __init__(self, codes: np.ndarray, A, B, stream=None, _handle=None):
+        lib = load()
+        if _handle is not None:
+            self._h = _handle
+        else:
+            codes = np.ascontiguousarray(codes, dtype=np.uint8)
+            A16 = _f16_bits(A)
+            B16 = _f16_bits(B)
+            d = A16.shape[0]
+            N, K = codes.shape
+            h = ctypes.c_void_p()
+            _check(lib.unisvq_pack(codes.ctypes.data, A16.ctypes.data, B16.ctypes.data, N, K, d,
+                                   _stream_ptr(stream), ctypes.byref(h)), "unisvq_pack")
+            self._h = h
+        info = self.query(1)
+        self.N, self.K, self.d = info["N"], info["K"], info["d"]
+
+    def clone(self, stream=None) -> "UniSVQLinear":
+        h = ctypes.c_void_p()
+        _check(load().unisvq_clone(self._h, _stream_ptr(stream), ctypes.byref(h)), "unisvq_clone")
+        return UniSVQLinear(None, None, None, _handle=h)
+
+    def forward(self, x, out=None, kernel: int = KERNEL_AUTO, stream=None):
+        """y = x W_hat^T for a bf16 CUDA tensor x [M][K]; returns y [M][N] bf16."""
+        import torch
+        if x.dtype != torch.bfloat16 or not x.is_cuda or x.dim() != 2 or x.shape[1] != self.K:
+            raise ValueError("x must be a CUDA bf16 tensor of shape [M, K]")
+        x = x.contiguous()
+        M = x.shape[0]
+        if out is None:
+            out = torch.empty((M, self.N), dtype=torch.bfloat16, device=x.device)
+        elif out.dtype != torch.bfloat16 or not out.is_contiguous() or tuple(out.shape) != (M, self.N):
+            raise ValueError("out must be a contiguous bf16 tensor of shape [M, N]")
+        st = load().unisvq_linear_force(self._h, int(kernel), ctypes.c_void_p(x.data_ptr()),
+                                        ctypes.c_void_p(out.data_ptr()), M, _stream_ptr(stream))
+        _check(st, "unisvq_linear")
+        return out
+
+    __call__ = forward
+
+    def forward_ptr(self, x_ptr: int, y_ptr: int, M: int, stream_ptr: int, kernel: int = KERNEL_AUTO) -> int:
+        """Raw-pointer call (no checks in Python); returns the status."""
+        return load().unisvq_linear_force(self._h, kernel, ctypes.c_void_p(x_ptr), ctypes.c_void_p(y_ptr),
+                                          M, ctypes.c_void_p(stream_ptr))
+
+    def dequant_debug(self, stream=None):
+        import torch
+        W = torch.empty((self.N, self.K), dtype=torch.float32, device="cuda")
+        _check(load().unisvq_dequant_debug(self._h, ctypes.c_void_p(W.data_ptr()), _stream_ptr(stream)),
+               "unisvq_dequant_debug")
+        return W
+
+    def query(self, M: int) -> dict:
+        info = Info()
+        _check(load().unisvq_query(self._h, int(M), ctypes.byref(info)), "unisvq_query")
+        return {f: getattr(info, f) for f, _ in Info._fields_}
+
+    def close(self):
+        if getattr(self, "_h", None) is not None and self._h.value:
+            load().unisvq_destroy(self._h)
+            self._h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,61 @@
+// Internal declarations shared by the libunisvq translation units.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/unisvq.h"
+#include "layout.h"
+
+struct unisvq_layer {
+  int N, K, d;
+  int Np, Kp, KT;          // padded shape; KT = Kp / 128 k-tiles
+  int device;
+  int num_sms;
+  uint8_t* codes;          // device, packed layout (layout.h)
+  size_t code_bytes;
+  float* lut32;            // device, [4^d][d] fp32 codewords RN(A z + B)
+  uint16_t* lut16;         // device, [4^d][d] bf16 codewords RN(A z + B)
+  int lut_entries;         // 4^d
+  float A[16];             // fp32 (exact) copy of A, row-major d x d
+  float B[4];              // fp32 (exact) copy of B
+  float colnorm;           // max_c sum_r |A[r][c]|: |x A|_inf <= |x|_inf * colnorm
+  uint16_t A16[16], B16[4];
+};
+
+namespace unisvq {
+
+struct DecodePlan {
+  int nt;          // n8 token tiles (1, 2, 4)
+  int ks;          // CTAs along K (cluster size)
+  int kt_per_cta;  // k-tiles per CTA
+  int nb;          // row blocks of 128 rows
+  size_t smem;     // dynamic shared memory bytes
+};
+
+struct PrefillPlan {
+  int bn;          // tokens per tile
+  int tiles;
+  int grid;
+  size_t smem;
+};
+
+int* device_error_word();   // device address of the library error word (current device)
+
+DecodePlan plan_decode(const unisvq_layer* L, int M);
+unisvq_status launch_decode(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
+
+bool prefill_supported(const unisvq_layer* L, int M);
+PrefillPlan plan_prefill(const unisvq_layer* L, int M);
+unisvq_status launch_prefill(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
+
+unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s);
+
+// Host packer (pack.cpp).
+void pack_codes_host(const uint8_t* codes, int N, int K, uint8_t* packed);
+// fp64 -> bf16 round-to-nearest-even (single rounding).
+uint16_t f64_to_bf16_rne(double v);
+double f16_bits_to_f64(uint16_t h);
+
+}  // namespace unisvq

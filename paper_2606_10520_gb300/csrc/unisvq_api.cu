@@ -1,0 +1,304 @@
+// C-ABI entry points of libunisvq: argument validation, the layer handle,
+// kernel dispatch and the device error word.
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace unisvq {
+
+namespace {
+__device__ int g_error_word;
+
+// Per-device cache of the error word's device address.
+int* g_err_ptr[64] = {};
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
+  const uintptr_t a0 = reinterpret_cast<uintptr_t>(a), b0 = reinterpret_cast<uintptr_t>(b);
+  return a0 < b0 + nb && b0 < a0 + na;
+}
+
+unisvq_status cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return UNISVQ_OK;
+  if (e == cudaErrorMemoryAllocation) return UNISVQ_ERR_OOM;
+  return UNISVQ_ERR_CUDA;
+}
+
+}  // namespace
+
+int* device_error_word() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  if (!g_err_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
+    g_err_ptr[dev] = static_cast<int*>(p);
+  }
+  return g_err_ptr[dev];
+}
+
+}  // namespace unisvq
+
+using namespace unisvq;
+
+extern "C" {
+
+int unisvq_version(void) { return 100; }
+
+const char* unisvq_status_string(unisvq_status s) {
+  switch (s) {
+    case UNISVQ_OK: return "ok";
+    case UNISVQ_ERR_INVALID_ARG: return "invalid argument";
+    case UNISVQ_ERR_UNSUPPORTED: return "unsupported shape or kernel";
+    case UNISVQ_ERR_CUDA: return "CUDA runtime error";
+    case UNISVQ_ERR_OOM: return "out of device memory";
+    case UNISVQ_ERR_TIMEOUT: return "a kernel gave up on a bounded wait";
+  }
+  return "unknown status";
+}
+
+size_t unisvq_packed_code_bytes(int N, int K) {
+  if (N <= 0 || K <= 0) return 0;
+  return static_cast<size_t>(round_up(N, kRowPad) / kTileRows) *
+         static_cast<size_t>(round_up(K, kColPad) / kTileCols) * kTileBytes;
+}
+
+unisvq_status unisvq_pack_host(const uint8_t* codes, int N, int K, uint8_t* packed,
+                               size_t packed_bytes) {
+  if (!codes || !packed || N <= 0 || K <= 0) return UNISVQ_ERR_INVALID_ARG;
+  if (packed_bytes < unisvq_packed_code_bytes(N, K)) return UNISVQ_ERR_INVALID_ARG;
+  pack_codes_host(codes, N, K, packed);
+  return UNISVQ_OK;
+}
+
+unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
+                          int N, int K, int d, void* stream, unisvq_handle* out) {
+  if (!out) return UNISVQ_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!codes || !A_f16 || !B_f16) return UNISVQ_ERR_INVALID_ARG;
+  if (d != 1 && d != 2 && d != 4) return UNISVQ_ERR_UNSUPPORTED;
+  if (N <= 0 || K <= 0 || K % d != 0) return UNISVQ_ERR_INVALID_ARG;
+  if (static_cast<long long>(round_up(N, kRowPad)) * round_up(K, kColPad) >= (1ll << 40))
+    return UNISVQ_ERR_UNSUPPORTED;
+
+  const size_t total = static_cast<size_t>(N) * K;
+  int bad = 0;
+#pragma omp parallel for reduction(| : bad) schedule(static)
+  for (long long i = 0; i < static_cast<long long>(total); ++i) bad |= codes[i] > 3;
+  if (bad) return UNISVQ_ERR_INVALID_ARG;
+
+  double A[16], B[4];
+  for (int i = 0; i < d * d; ++i) {
+    A[i] = f16_bits_to_f64(A_f16[i]);
+    if (!std::isfinite(A[i])) return UNISVQ_ERR_INVALID_ARG;
+  }
+  for (int i = 0; i < d; ++i) {
+    B[i] = f16_bits_to_f64(B_f16[i]);
+    if (!std::isfinite(B[i])) return UNISVQ_ERR_INVALID_ARG;
+  }
+
+  unisvq_layer* L = new (std::nothrow) unisvq_layer();
+  if (!L) return UNISVQ_ERR_OOM;
+  L->N = N;
+  L->K = K;
+  L->d = d;
+  L->Np = round_up(N, kRowPad);
+  L->Kp = round_up(K, kColPad);
+  L->KT = L->Kp / kTileCols;
+  if (cudaGetDevice(&L->device) != cudaSuccess ||
+      cudaDeviceGetAttribute(&L->num_sms, cudaDevAttrMultiProcessorCount, L->device) != cudaSuccess) {
+    delete L;
+    return UNISVQ_ERR_CUDA;
+  }
+  std::memset(L->A, 0, sizeof(L->A));
+  std::memset(L->B, 0, sizeof(L->B));
+  double colnorm = 0;
+  for (int c = 0; c < d; ++c) {
+    double s = 0;
+    for (int r = 0; r < d; ++r) s += std::fabs(A[r * d + c]);
+    colnorm = s > colnorm ? s : colnorm;
+  }
+  for (int i = 0; i < d * d; ++i) {
+    L->A[i] = static_cast<float>(A[i]);   // exact: fp16 -> fp32
+    L->A16[i] = A_f16[i];
+  }
+  for (int i = 0; i < d; ++i) {
+    L->B[i] = static_cast<float>(B[i]);
+    L->B16[i] = B_f16[i];
+  }
+  // Rounded up so the activation scale never underestimates |x A|.
+  L->colnorm = static_cast<float>(colnorm) * (1.0f + 1e-6f);
+
+  // Codebook of Eq. (def:unisvq): entry v holds A z(v) + B, z_c(v) = (v >> 2c) & 3,
+  // exact in fp64, rounded once to fp32 and to bf16.
+  const int E = 1 << (2 * d);
+  L->lut_entries = E;
+  std::vector<float> lut32(static_cast<size_t>(E) * d);
+  std::vector<uint16_t> lut16(static_cast<size_t>(E) * d);
+  for (int v = 0; v < E; ++v)
+    for (int r = 0; r < d; ++r) {
+      double w = B[r];
+      for (int c = 0; c < d; ++c) w += A[r * d + c] * static_cast<double>((v >> (2 * c)) & 3);
+      lut32[static_cast<size_t>(v) * d + r] = static_cast<float>(w);
+      lut16[static_cast<size_t>(v) * d + r] = f64_to_bf16_rne(w);
+    }
+
+  L->code_bytes = unisvq_packed_code_bytes(N, K);
+  std::vector<uint8_t> packed;
+  try {
+    packed.resize(L->code_bytes);
+  } catch (...) {
+    delete L;
+    return UNISVQ_ERR_OOM;
+  }
+  pack_codes_host(codes, N, K, packed.data());
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMalloc(&L->codes, L->code_bytes);
+  if (e == cudaSuccess) e = cudaMalloc(&L->lut32, lut32.size() * sizeof(float));
+  if (e == cudaSuccess) e = cudaMalloc(&L->lut16, lut16.size() * sizeof(uint16_t));
+  if (e == cudaSuccess) e = cudaMemcpyAsync(L->codes, packed.data(), L->code_bytes, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(L->lut32, lut32.data(), lut32.size() * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(L->lut16, lut16.data(), lut16.size() * sizeof(uint16_t), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess && !device_error_word()) e = cudaErrorUnknown;
+  if (e != cudaSuccess) {
+    cudaFree(L->codes);
+    cudaFree(L->lut32);
+    cudaFree(L->lut16);
+    delete L;
+    return cuda_status(e);
+  }
+  *out = L;
+  return UNISVQ_OK;
+}
+
+unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
+  if (!h || !out) return UNISVQ_ERR_INVALID_ARG;
+  *out = nullptr;
+  unisvq_layer* L = new (std::nothrow) unisvq_layer(*h);
+  if (!L) return UNISVQ_ERR_OOM;
+  L->codes = nullptr;
+  L->lut32 = nullptr;
+  L->lut16 = nullptr;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t n32 = static_cast<size_t>(h->lut_entries) * h->d * sizeof(float);
+  const size_t n16 = static_cast<size_t>(h->lut_entries) * h->d * sizeof(uint16_t);
+  cudaError_t e = cudaMalloc(&L->codes, h->code_bytes);
+  if (e == cudaSuccess) e = cudaMalloc(&L->lut32, n32);
+  if (e == cudaSuccess) e = cudaMalloc(&L->lut16, n16);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(L->codes, h->codes, h->code_bytes, cudaMemcpyDeviceToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(L->lut32, h->lut32, n32, cudaMemcpyDeviceToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(L->lut16, h->lut16, n16, cudaMemcpyDeviceToDevice, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) {
+    cudaFree(L->codes);
+    cudaFree(L->lut32);
+    cudaFree(L->lut16);
+    delete L;
+    return cuda_status(e);
+  }
+  *out = L;
+  return UNISVQ_OK;
+}
+
+unisvq_status unisvq_destroy(unisvq_handle h) {
+  if (!h) return UNISVQ_OK;
+  cudaError_t e1 = cudaFree(h->codes);
+  cudaError_t e2 = cudaFree(h->lut32);
+  cudaError_t e3 = cudaFree(h->lut16);
+  delete h;
+  return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess) ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+}
+
+static int auto_kernel(const unisvq_layer* L, int M) {
+  if (M > 32 && prefill_supported(L, M)) return UNISVQ_KERNEL_PREFILL;
+  return UNISVQ_KERNEL_DECODE;
+}
+
+static unisvq_status check_io(unisvq_handle h, const void* x, void* y, int M) {
+  if (!h || M < 0) return UNISVQ_ERR_INVALID_ARG;
+  if (M == 0) return UNISVQ_OK;
+  if (!x || !y) return UNISVQ_ERR_INVALID_ARG;
+  if (!aligned(x, 16) || !aligned(y, 4)) return UNISVQ_ERR_INVALID_ARG;
+  const size_t nx = static_cast<size_t>(M) * h->K * 2, ny = static_cast<size_t>(M) * h->N * 2;
+  if (overlaps(x, nx, y, ny)) return UNISVQ_ERR_INVALID_ARG;
+  return UNISVQ_OK;
+}
+
+unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, void* y, int M,
+                                  void* stream) {
+  unisvq_status st = check_io(h, x, y, M);
+  if (st != UNISVQ_OK || M == 0) return st;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
+  if (dev != h->device) return UNISVQ_ERR_INVALID_ARG;
+  if (kernel == UNISVQ_KERNEL_AUTO) kernel = auto_kernel(h, M);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (kernel == UNISVQ_KERNEL_DECODE) return launch_decode(h, x, y, M, s);
+  if (kernel == UNISVQ_KERNEL_PREFILL) {
+    if (!prefill_supported(h, M)) return UNISVQ_ERR_UNSUPPORTED;
+    return launch_prefill(h, x, y, M, s);
+  }
+  return UNISVQ_ERR_INVALID_ARG;
+}
+
+unisvq_status unisvq_linear(unisvq_handle h, const void* x, void* y, int M, void* stream) {
+  return unisvq_linear_force(h, UNISVQ_KERNEL_AUTO, x, y, M, stream);
+}
+
+unisvq_status unisvq_dequant_debug(unisvq_handle h, float* W, void* stream) {
+  if (!h || !W || !aligned(W, 4)) return UNISVQ_ERR_INVALID_ARG;
+  return launch_dequant(h, W, static_cast<cudaStream_t>(stream));
+}
+
+unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
+  if (!h || !info || M < 0) return UNISVQ_ERR_INVALID_ARG;
+  std::memset(info, 0, sizeof(*info));
+  info->N = h->N;
+  info->K = h->K;
+  info->d = h->d;
+  info->Np = h->Np;
+  info->Kp = h->Kp;
+  info->code_bytes = static_cast<long long>(h->code_bytes);
+  info->meta_bytes = static_cast<long long>(h->d * h->d + h->d) * 2;
+  info->algo_bytes = static_cast<long long>(h->N) * h->K / 4 + info->meta_bytes +
+                     2ll * M * h->K + 2ll * M * h->N;
+  info->flops = 2.0 * M * static_cast<double>(h->N) * h->K;
+  info->kernel = auto_kernel(h, M > 0 ? M : 1);
+  if (info->kernel == UNISVQ_KERNEL_DECODE) {
+    const DecodePlan p = plan_decode(h, M > 32 ? 32 : (M > 0 ? M : 1));
+    info->split_k = p.ks;
+    info->grid_ctas = p.ks * p.nb * ((M + 31) / 32 > 0 ? (M + 31) / 32 : 1);
+  } else {
+    const PrefillPlan p = plan_prefill(h, M);
+    info->split_k = 1;
+    info->grid_ctas = p.grid;
+  }
+  return UNISVQ_OK;
+}
+
+unisvq_status unisvq_sync_status(void* stream) {
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return UNISVQ_ERR_CUDA;
+  int* ew = device_error_word();
+  if (!ew) return UNISVQ_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpy(&v, ew, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return UNISVQ_ERR_CUDA;
+  if (v != 0) {
+    const int zero = 0;
+    cudaMemcpy(ew, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    return UNISVQ_ERR_TIMEOUT;
+  }
+  return UNISVQ_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,179 @@
+"""GPU parity of libunisvq against the fp64 CPU oracle (needs an sm_103a GPU).
+
+Bars: the fp32 dequantisation hook is bit-exact to RN_fp32 of the exact
+codewords; layer outputs meet |y - y_ref| <= 2^-7 sum|w x| + 1e-6 per element
+and a relative L2 error <= 4e-3 (oracle.compare); integer-valued cases are
+bit-exact.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():
+    pytest.skip("no CUDA device", allow_module_level=True)
+
+from paper_2606_10520_gb300 import binding  # noqa: E402
+
+binding.load()
+
+
+def to_dev(xbits: np.ndarray):
+    return torch.from_numpy(np.ascontiguousarray(xbits).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def run(layer, xbits, kernel=binding.KERNEL_AUTO):
+    y = layer.forward(to_dev(xbits), kernel=kernel)
+    st = binding.sync_status()
+    assert st == binding.OK, binding.status_string(st)
+    return y.float().cpu().numpy().astype(np.float64)
+
+
+def check(yg, xbits, codes, A, B, rows=None):
+    if rows is not None:
+        yr, S = oracle.linear(xbits, codes[rows], A, B)
+        yg = yg[:, rows]
+    else:
+        yr, S = oracle.linear(xbits, codes, A, B)
+    res = oracle.compare(yg, yr, S)
+    assert res["ok"], res
+    return res
+
+
+@pytest.mark.parametrize("d", [1, 2, 4])
+@pytest.mark.parametrize("N,K", [(200, 520), (128, 128), (300, 1024)])
+def test_dequant_debug_bit_exact(d, N, K):
+    codes, A, B = synth.layer_inputs(1, 10, N, K, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    W = layer.dequant_debug().cpu().numpy()
+    assert binding.sync_status() == binding.OK
+    Wref = oracle.dequant_f32(codes, A, B)
+    assert np.array_equal(W.view(np.uint32), Wref.view(np.uint32))
+    layer.close()
+
+
+DECODE_SHAPES = [(256, 1024), (520, 1000), (130, 4096), (1024, 8192)]
+
+
+@pytest.mark.parametrize("d", [1, 2, 4])
+@pytest.mark.parametrize("N,K", DECODE_SHAPES)
+def test_decode_parity_small_M(d, N, K):
+    if K % d:
+        pytest.skip("K % d")
+    codes, A, B = synth.layer_inputs(2, 20, N, K, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    for M in (1, 2, 3, 7, 8, 9, 16, 17, 31, 32):
+        xb = synth.activations(2, 20, 1000 * N + M, M, K)
+        check(run(layer, xb, binding.KERNEL_DECODE), xb, codes, A, B)
+    layer.close()
+
+
+def test_decode_many_token_groups():
+    N, K, d = 384, 768, 2
+    codes, A, B = synth.layer_inputs(3, 30, 0, 0, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    for M in (33, 64, 100):
+        xb = synth.activations(3, 30, M, M, K)
+        check(run(layer, xb, binding.KERNEL_DECODE), xb, codes, A, B)
+    layer.close()
+
+
+def test_integer_case_bit_exact():
+    """Integer A (the printed D4 generator), integer B and small integer x:
+    every intermediate is exact, so the GPU output must equal the oracle's."""
+    d = 4
+    A = np.array([[1, -1, 0, 0], [0, 1, -1, 0], [0, 0, 1, -1], [0, 0, 1, 1]], dtype=np.float16)
+    B = np.array([1, -2, 0, 1], dtype=np.float16)
+    N, K = 256, 512
+    g = np.random.default_rng(11)
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    layer = binding.UniSVQLinear(codes, A, B)
+    for M in (1, 5, 16):
+        x = g.integers(-1, 2, size=(M, K)).astype(np.float32) * (g.random((M, K)) < 0.05)
+        xb = synth.f32_to_bf16_bits(x)
+        yr, _ = oracle.linear(xb, codes, A, B)
+        assert np.abs(yr).max() <= 256
+        yg = run(layer, xb, binding.KERNEL_DECODE)
+        assert np.array_equal(yg, yr), np.abs(yg - yr).max()
+    layer.close()
+
+
+def test_sq_special_case_matches_scalar_dequant():
+    """A = s I (d = 1 and d = 4): the layer is a 2-bit SQ GEMV (Eq. def:sq)."""
+    for d in (1, 4):
+        s, zp = 0.015625, 1.5
+        A = (s * np.eye(d)).astype(np.float16)
+        B = np.full(d, -s * zp).astype(np.float16)
+        N, K = 256, 1024
+        codes = synth.gen_codes(synth.rng(4, d), N, K)
+        layer = binding.UniSVQLinear(codes, A, B)
+        xb = synth.activations(4, 40, d, 4, K)
+        check(run(layer, xb, binding.KERNEL_DECODE), xb, codes, A, B)
+        layer.close()
+
+
+def test_zero_tokens_is_noop_and_bad_pointers_rejected():
+    N, K, d = 128, 256, 2
+    codes, A, B = synth.layer_inputs(5, 50, 0, 0, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    x = torch.zeros((0, K), dtype=torch.bfloat16, device="cuda")
+    y = layer(x)
+    assert y.shape == (0, N)
+    xb = torch.zeros((3, K + 8), dtype=torch.bfloat16, device="cuda")
+    ybuf = torch.zeros((3, N), dtype=torch.bfloat16, device="cuda")
+    st = layer.forward_ptr(xb.data_ptr() + 2, ybuf.data_ptr(), 3, torch.cuda.current_stream().cuda_stream)
+    assert st == binding.ERR_INVALID_ARG
+    st = layer.forward_ptr(ybuf.data_ptr(), ybuf.data_ptr(), 3, torch.cuda.current_stream().cuda_stream)
+    assert st == binding.ERR_INVALID_ARG
+    layer.close()
+
+
+def test_outputs_do_not_touch_guard_bands():
+    N, K, d, M = 130, 384, 2, 5
+    codes, A, B = synth.layer_inputs(6, 60, 0, 0, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    xb = synth.activations(6, 60, 0, M, K)
+    guard = 4096
+    buf = torch.full((guard * 2 + M * N,), 12345.0, dtype=torch.bfloat16, device="cuda")
+    fill = float(buf[0].item())
+    y = buf[guard:guard + M * N].view(M, N)
+    layer.forward(to_dev(xb), out=y)
+    assert binding.sync_status() == binding.OK
+    host = buf.float().cpu().numpy()
+    assert (host[:guard] == fill).all() and (host[guard + M * N:] == fill).all()
+    check(y.float().cpu().numpy().astype(np.float64), xb, codes, A, B)
+    layer.close()
+
+
+def test_clone_matches_original():
+    N, K, d = 256, 512, 4
+    codes, A, B = synth.layer_inputs(7, 70, 0, 0, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    twin = layer.clone()
+    xb = synth.activations(7, 70, 0, 4, K)
+    a = run(layer, xb)
+    b = run(twin, xb)
+    assert np.array_equal(a, b)
+    twin.close()
+    layer.close()
+
+
+FULL_SHAPES = [(4096, 4096), (11008, 4096), (4096, 11008), (28672, 8192), (8192, 28672)]
+
+
+@pytest.mark.parametrize("N,K", FULL_SHAPES)
+def test_full_size_decode_sampled_rows(N, K):
+    """Config-sized layers at the decode batch sizes, checked on sampled rows."""
+    d = 2
+    codes, A, B = synth.layer_inputs(0, 3, 0, N, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    rows = np.sort(synth.rng(0, N, K).choice(N, size=48, replace=False))
+    rows = np.unique(np.concatenate([rows, [0, N - 1]]))
+    for M in (1, 8, 16, 32):
+        xb = synth.activations(0, 3, M, M, K)
+        check(run(layer, xb), xb, codes, A, B, rows=rows)
+    layer.close()

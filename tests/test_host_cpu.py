@@ -1,0 +1,109 @@
+"""Host-side tests of libunisvq that need no GPU: exports, layout, validation."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "unisvq.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(unisvq_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    assert "unisvq_linear" in names and "unisvq_pack" in names
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in include/unisvq.h but not exported"
+    from paper_2606_10520_gb300 import binding
+    assert sorted(binding.EXPORTS) == names
+
+
+def decode_layout(packed: np.ndarray, N: int, K: int) -> np.ndarray:
+    """Independent reader of the packed layout, written from include/unisvq.h."""
+    Np = -(-N // 128) * 128
+    Kp = -(-K // 128) * 128
+    KT = Kp // 128
+    words = packed.view("<u4").reshape(Np // 16, KT, 32, 4)
+    out = np.full((Np, Kp), 255, dtype=np.int64)
+    for rt in range(Np // 16):
+        for kt in range(KT):
+            for lane in range(32):
+                g, t = lane // 4, lane % 4
+                for q in range(4):
+                    grp, rh = q // 2, q % 2
+                    n = 16 * rt + g + 8 * rh
+                    w = int(words[rt, kt, lane, q])
+                    for p in range(8):
+                        i, h = p // 2, p % 2
+                        k = 128 * kt + 64 * grp + 16 * i + 4 * t + 2 * h
+                        out[n, k] = (w >> (2 * p)) & 3
+                        out[n, k + 1] = (w >> (16 + 2 * p)) & 3
+    return out
+
+
+@pytest.mark.parametrize("N,K", [(16, 128), (37, 200), (130, 260), (8, 4)])
+def test_pack_host_layout_roundtrip(lib, N, K):
+    from paper_2606_10520_gb300 import binding
+    g = np.random.default_rng(N * 1000 + K)
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    packed = binding.pack_host(codes)
+    assert packed.nbytes == binding.packed_code_bytes(N, K)
+    assert packed.nbytes == (-(-N // 128) * 8) * (-(-K // 128)) * 512
+    full = decode_layout(packed, N, K)
+    assert not (full == 255).any(), "some (row, col) never written"
+    assert np.array_equal(full[:N, :K], codes)
+    assert (full[N:, :] == 0).all() and (full[:, K:] == 0).all(), "padding must be code 0"
+
+
+def test_packed_bytes_is_quarter_byte_per_weight(lib):
+    from paper_2606_10520_gb300 import binding
+    for N, K in [(4096, 4096), (11008, 4096), (28672, 8192)]:
+        assert binding.packed_code_bytes(N, K) == N * K // 4
+
+
+def test_status_strings(lib):
+    from paper_2606_10520_gb300 import binding
+    for s in range(6):
+        assert isinstance(binding.status_string(s), str) and binding.status_string(s)
+
+
+def _pack_status(lib, codes, A, B, N, K, d):
+    h = ctypes.c_void_p()
+    return lib.unisvq_pack(codes.ctypes.data if codes is not None else None,
+                           A.ctypes.data if A is not None else None,
+                           B.ctypes.data if B is not None else None, N, K, d, None, ctypes.byref(h))
+
+
+def test_pack_rejects_bad_arguments_before_touching_the_gpu(lib):
+    from paper_2606_10520_gb300 import binding
+    codes = np.zeros((4, 8), dtype=np.uint8)
+    A = np.eye(2, dtype=np.float16).view(np.uint16)
+    B = np.zeros(2, dtype=np.float16).view(np.uint16)
+    assert _pack_status(lib, None, A, B, 4, 8, 2) == binding.ERR_INVALID_ARG
+    assert _pack_status(lib, codes, A, B, 4, 8, 3) == binding.ERR_UNSUPPORTED
+    assert _pack_status(lib, codes, A, B, 4, 7, 2) == binding.ERR_INVALID_ARG     # K % d
+    assert _pack_status(lib, codes, A, B, 0, 8, 2) == binding.ERR_INVALID_ARG
+    bad = codes.copy()
+    bad[1, 3] = 4
+    assert _pack_status(lib, bad, A, B, 4, 8, 2) == binding.ERR_INVALID_ARG
+    Anan = np.array([[np.nan, 0], [0, 1]], dtype=np.float16).view(np.uint16)
+    assert _pack_status(lib, codes, Anan, B, 4, 8, 2) == binding.ERR_INVALID_ARG
+
+
+def test_linear_rejects_bad_arguments(lib):
+    from paper_2606_10520_gb300 import binding
+    assert lib.unisvq_linear(None, None, None, 1, None) == binding.ERR_INVALID_ARG
+    assert lib.unisvq_destroy(None) == binding.OK
+    info = binding.Info()
+    assert lib.unisvq_query(None, 1, ctypes.byref(info)) == binding.ERR_INVALID_ARG
+
+
+def test_version(lib):
+    assert lib.unisvq_version() >= 100
