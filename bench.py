@@ -1,0 +1,471 @@
+#!/usr/bin/env python
+"""Benchmark of the UniSVQ linear layer (libunisvq) on GB300.
+
+Workload (the decode sweep of the Llama-2-7B-shaped projection set): 32
+layers x {q, k, v, o: 4096x4096; gate, up: 11008x4096; down: 4096x11008},
+2-bit codes with d = 2 and one fp16 affine per matrix, bf16 activations with
+1% outlier channels, batch M in {1, 2, 4, 8, 16}. One step = one pass of the
+whole layer stack at every M of the sweep (5 x 224 layer calls), replayed from
+CUDA graphs. The 1.62 GB of packed codes per pass is far larger than L2, so
+no flush is needed between steps.
+
+Metric: HBM GB/s = algorithmic bytes (N*K/4 codes + affine + 2*M*K + 2*M*N)
+per step / step time. With --prefill (default on) a second object reports the
+tcgen05 prefill GEMM on the Llama-3-8B-shaped set at M = 2048 in TFLOP/s.
+
+--impl reference times the CPU oracle (the fp64 NumPy restatement of the
+method) on a bounded sample of the same workload, on the host cores.
+
+Multi-GPU (torchrun): the path does not shard, so every rank runs an
+independent replica; value = bytes of all ranks / max time over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "UniSVQ linear: GEMV HBM GB/s (% of ~8 TB/s); prefill TFLOPS (% of bf16 peak)"
+M_SWEEP = (1, 2, 4, 8, 16)
+PREFILL_M = 2048
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def algo_bytes(N, K, M, d=2):
+    return N * K // 4 + (d * d + d) * 2 + 2 * M * K + 2 * M * N
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle baseline (bounded sample)
+# ---------------------------------------------------------------------------
+def cpu_threads():
+    for v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        if os.environ.get(v, "").isdigit():
+            return int(os.environ[v])
+    return os.cpu_count() or 1
+
+
+def oracle_sample(budget_s: float):
+    """Time the oracle on layer-0 projections at M = 1 until `budget_s` passes."""
+    import oracle
+    t0 = time.perf_counter()
+    nbytes = 0
+    done = []
+    i = 0
+    while True:
+        name, N, K = synth.LLAMA2_7B[i % len(synth.LLAMA2_7B)]
+        codes, A, B = synth.layer_inputs(0, 1, 0, i % 7, N, K, 2)
+        xb = synth.activations(0, 1, 1, 1, K)
+        t1 = time.perf_counter()
+        oracle.linear(xb, codes, A, B)
+        dt = time.perf_counter() - t1
+        nbytes += algo_bytes(N, K, 1)
+        done.append((name, dt))
+        i += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    t_oracle = sum(dt for _, dt in done)
+    return nbytes / t_oracle / 1e9, t_oracle, [n for n, _ in done]
+
+
+# ---------------------------------------------------------------------------
+# reference arm: the oracle on the host cores
+# ---------------------------------------------------------------------------
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    import oracle
+    name, N, K = synth.LLAMA2_7B[0]
+    codes, A, B = synth.layer_inputs(0, 1, 0, 0, N, K, 2)
+    xb = synth.activations(0, 1, 1, 1, K)
+    for _ in range(args.warmup):
+        oracle.linear(xb, codes, A, B)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.linear(xb, codes, A, B)
+    dt = time.perf_counter() - t0
+    gbs = args.steps * algo_bytes(N, K, 1) / dt / 1e9
+    sample = f"per step: one {N}x{K} projection (q, layer 0) at M=1 through oracle.linear (fp64 NumPy)"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1000 / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": workload_config(args),
+        "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": cpu_threads(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(args):
+    return {"workload": f"Llama-2-7B-shaped projection set x {args.layers} layers, decode sweep M in "
+                        f"{list(M_SWEEP)}, 2-bit codes d=2, per-matrix fp16 affine",
+            "layers": args.layers, "d": 2, "m_sweep": list(M_SWEEP),
+            "l2": "inputs larger than L2 (1.62 GB of packed codes per pass at 32 layers)",
+            "timing": "CUDA graphs of the full layer stack per M, CUDA events on the capture stream",
+            "parallelism": "replicas"}
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def build_stack(binding, shapes, layers, config_id, d=2):
+    """Distinct random matrices for layer 0; the other layers are device copies."""
+    base = []
+    for pi, (_, N, K) in enumerate(shapes):
+        codes, A, B = synth.layer_inputs(0, config_id, 0, pi, N, K, d)
+        base.append(binding.UniSVQLinear(codes, A, B))
+    stack = [base]
+    for _ in range(layers - 1):
+        stack.append([b.clone() for b in base])
+    return stack
+
+
+def time_graphs(torch, graphs, steps, warmup, stream):
+    for _ in range(warmup):
+        for g in graphs:
+            g.replay()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        for g in graphs:
+            g.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / 1000.0
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+    from paper_2606_10520_gb300 import binding
+
+    torch.cuda.set_device(local_rank)
+    binding.load()
+    peaks, peak_src = load_peaks()
+    shapes = synth.LLAMA2_7B
+    stack = build_stack(binding, shapes, args.layers, 1)
+
+    xs, ys, graphs, step_bytes, launches = {}, {}, [], 0, 0
+    for M in M_SWEEP:
+        for _, N, K in shapes:
+            if (M, K) not in xs:
+                xb = synth.activations(0, 1, 100 + M, M, K)
+                xs[(M, K)] = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).cuda()
+            if (M, N) not in ys:
+                ys[(M, N)] = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    side = torch.cuda.Stream()
+    for M in M_SWEEP:
+        def one_pass(M=M):
+            sp = torch.cuda.current_stream().cuda_stream
+            for layer in stack:
+                for (_, N, K), h in zip(shapes, layer):
+                    st = h.forward_ptr(xs[(M, K)].data_ptr(), ys[(M, N)].data_ptr(), M, sp,
+                                       binding.KERNEL_DECODE)
+                    if st != 0:
+                        raise RuntimeError(f"unisvq_linear failed: {binding.status_string(st)}")
+        with torch.cuda.stream(side):
+            one_pass()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side):
+            one_pass()
+        graphs.append(g)
+        for layer in stack:
+            for (_, N, K), h in zip(shapes, layer):
+                step_bytes += algo_bytes(N, K, M)
+                launches += 1
+    torch.cuda.synchronize()
+    st = binding.sync_status()
+    if st != 0:
+        raise RuntimeError(f"device status {binding.status_string(st)}")
+
+    # ---- timed region: decode sweep ------------------------------------
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clk = ClockSampler(local_rank)
+    clk.start()
+    time.sleep(0.3)
+    t = time_graphs(torch, graphs, args.steps, args.warmup, side)
+    clocks = clk.stop()
+    if world > 1:
+        tt = torch.tensor([t], device="cuda", dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t = float(tt.item())
+    st = binding.sync_status(side)
+    if st != 0:
+        raise RuntimeError(f"device status {binding.status_string(st)}")
+    total_bytes = step_bytes * args.steps * world
+    value = total_bytes / t / 1e9
+    per_rank = step_bytes * args.steps / t / 1e9
+
+    # per-M breakdown (separate short timing of each graph)
+    sweep = []
+    for M, g in zip(M_SWEEP, graphs):
+        tm = time_graphs(torch, [g], max(3, args.steps // 4), 2, side)
+        nb = sum(algo_bytes(N, K, M) for _, N, K in shapes) * args.layers
+        n_calls = len(shapes) * args.layers
+        gbs = nb * max(3, args.steps // 4) / tm / 1e9
+        sweep.append({"M": M, "GB/s": round(gbs, 1), "frac_of_measured_hbm": round(gbs / peaks["hbm_gbs"], 4),
+                      "frac_of_8TBs": round(gbs / 8000.0, 4),
+                      "us_per_layer": round(tm / max(3, args.steps // 4) / n_calls * 1e6, 3),
+                      "kernel": "decode"})
+
+    # ---- e2e: pinned host buffers, H2D + layer + D2H inside the timed graphs ---
+    e2e = None
+    if not args.no_e2e:
+        hx = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True).copy_(v.cpu()) for k, v in xs.items()}
+        hy = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in ys.items()}
+        egraphs, h2d, d2h = [], 0, 0
+        for M in M_SWEEP:
+            def e2e_pass(M=M):
+                sp = torch.cuda.current_stream().cuda_stream
+                for layer in stack:
+                    for (_, N, K), h in zip(shapes, layer):
+                        xs[(M, K)].copy_(hx[(M, K)], non_blocking=True)
+                        st = h.forward_ptr(xs[(M, K)].data_ptr(), ys[(M, N)].data_ptr(), M, sp,
+                                           binding.KERNEL_DECODE)
+                        if st != 0:
+                            raise RuntimeError(binding.status_string(st))
+                        hy[(M, N)].copy_(ys[(M, N)], non_blocking=True)
+            with torch.cuda.stream(side):
+                e2e_pass()
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=side):
+                e2e_pass()
+            egraphs.append(g)
+            for _, N, K in shapes:
+                h2d += 2 * M * K * args.layers
+                d2h += 2 * M * N * args.layers
+        te = time_graphs(torch, egraphs, args.steps, args.warmup, side)
+        e2e = {"value": step_bytes * args.steps * world / te / 1e9, "unit": "GB/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "how": "per layer call: pinned-host x -> device copy, unisvq_linear, device -> pinned-host y; "
+                      "the whole sweep replayed from CUDA graphs"}
+
+    # ---- prefill (tcgen05 GEMM), Llama-3-8B-shaped set at M = 2048 -------
+    prefill = None
+    if not args.no_prefill:
+        prefill = run_prefill(torch, binding, peaks, args, side)
+
+    # ---- CPU oracle baseline (rank 0, N=1 only) --------------------------
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        gbs_cpu, t_cpu, names = oracle_sample(args.cpu_budget)
+        cpu = {"value": gbs_cpu, "unit": "GB/s", "cores": cpu_threads(), "kind": "oracle",
+               "sample": f"oracle.linear (fp64 NumPy) on layer-0 projections {names} at M=1, "
+                         f"{t_cpu:.1f} s of CPU work"}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t * 1000 / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f16 MMA on bf16 I/O, f32 accumulate",
+        "data": "synthetic (seeded codes, affine and activations; layers 1..31 are device copies of layer 0)",
+        "config": workload_config(args),
+        "roofline": {"bound": "hbm", "achieved": per_rank, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": per_rank / peaks["hbm_gbs"], "traffic": None,
+                     "kernel": "decode_kernel (all launches of the timed region)",
+                     "peak_source": f"{peak_src} hbm_gbs (copy, burst)",
+                     "frac_of_8TBs": per_rank / 8000.0},
+        "sweep": sweep,
+        "e2e": e2e,
+        "gpu_launches": launches * args.steps,
+        "clocks": clocks,
+        "cpu_baseline": cpu,
+        "prefill": prefill,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def run_prefill(torch, binding, peaks, args, stream):
+    from paper_2606_10520_gb300 import binding as b
+    shapes = synth.LLAMA3_8B
+    layers = []
+    for pi, (_, N, K) in enumerate(shapes):
+        codes, A, B = synth.layer_inputs(0, 2, 0, pi, N, K, 2)
+        layers.append(b.UniSVQLinear(codes, A, B))
+    q = layers[0].query(PREFILL_M)
+    if q["kernel"] != b.KERNEL_PREFILL:
+        for l in layers:
+            l.close()
+        return {"unavailable": "prefill kernel not supported in this build"}
+    M = PREFILL_M
+    xs = {K: torch.from_numpy(synth.activations(0, 2, K, M, K).view(np.int16)).view(torch.bfloat16).cuda()
+          for K in sorted({K for _, _, K in shapes})}
+    ys = {N: torch.empty((M, N), dtype=torch.bfloat16, device="cuda") for N in sorted({N for _, N, _ in shapes})}
+
+    def one_pass():
+        sp = torch.cuda.current_stream().cuda_stream
+        for (_, N, K), h in zip(shapes, layers):
+            st = h.forward_ptr(xs[K].data_ptr(), ys[N].data_ptr(), M, sp, b.KERNEL_PREFILL)
+            if st != 0:
+                raise RuntimeError(b.status_string(st))
+    with torch.cuda.stream(stream):
+        one_pass()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        one_pass()
+    reps = max(5, args.steps // 2)
+    t = time_graphs(torch, [g], reps, 3, stream)
+    flops = sum(2.0 * M * N * K for _, N, K in shapes)
+    tflops = flops * reps / t / 1e12
+    # per-projection timing
+    per = []
+    for (nm, N, K), h in zip(shapes, layers):
+        def single(h=h, N=N, K=K):
+            sp = torch.cuda.current_stream().cuda_stream
+            h.forward_ptr(xs[K].data_ptr(), ys[N].data_ptr(), M, sp, b.KERNEL_PREFILL)
+        with torch.cuda.stream(stream):
+            single()
+        torch.cuda.synchronize()
+        gs = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gs, stream=stream):
+            single()
+        ts = time_graphs(torch, [gs], reps, 3, stream)
+        per.append({"proj": nm, "N": N, "K": K, "TFLOP/s": round(2.0 * M * N * K * reps / ts / 1e12, 1),
+                    "us": round(ts / reps * 1e6, 1)})
+    # cuBLAS bf16 dense GEMM on the same shapes (speed reference)
+    Wd = {(N, K): torch.randn(N, K, device="cuda").to(torch.bfloat16) for _, N, K in shapes}
+
+    def dense_pass():
+        for _, N, K in shapes:
+            torch.matmul(xs[K], Wd[(N, K)].t(), out=ys[N])
+    with torch.cuda.stream(stream):
+        dense_pass()
+    torch.cuda.synchronize()
+    gd = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gd, stream=stream):
+        dense_pass()
+    td = time_graphs(torch, [gd], reps, 3, stream)
+    for l in layers:
+        l.close()
+    return {"workload": f"Llama-3-8B-shaped projection set (7 GEMMs) at M={M}, d=2",
+            "TFLOP/s": tflops, "frac_of_measured_bf16": tflops / peaks["bf16_tflops"],
+            "frac_of_measured_bf16_sustained": tflops / peaks["bf16_tflops_sustained"],
+            "us_per_layer_set": t / reps * 1e6, "per_projection": per,
+            "cublas_bf16_dense_TFLOP/s": flops * reps / td / 1e12,
+            "kernel": "prefill_kernel (tcgen05)"}
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--layers", type=int, default=32)
+    ap.add_argument("--no-prefill", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    try:
+        run_ours(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

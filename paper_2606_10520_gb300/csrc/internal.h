@@ -16,7 +16,8 @@ struct unisvq_layer {
   uint8_t* codes;          // device, packed layout (layout.h)
   size_t code_bytes;
   float* lut32;            // device, [4^d][d] fp32 codewords RN(A z + B)
-  uint16_t* lut16;         // device, [4^d][d] bf16 codewords RN(A z + B)
+  uint32_t* tlut;          // device, prefill codeword table (bf16 pairs / quads), see pack
+  int tlut_words;
   int lut_entries;         // 4^d
   float A[16];             // fp32 (exact) copy of A, row-major d x d
   float B[4];              // fp32 (exact) copy of B

@@ -1,14 +1,436 @@
-// Prefill GEMM (M >= 64): tcgen05 kernel (not yet built in this revision).
+// Prefill GEMM (M > 32 tokens): tcgen05 tensor cores with the dequantised
+// weight tile built in shared memory and never written to HBM.
+//
+// y[m, n] = sum_k x[m, k] W_hat[n, k] (Eq. def:ptq_loss), W_hat of
+// Eq. (col:dequant). One output tile is 128 weight rows x BN tokens:
+//   D[128 x BN] (fp32, TMEM) = W_tile[128 x K] (bf16, smem) * x_tile[BN x K]^T
+// so the weights are the M=128 operand A and the tokens the N operand B of
+// tcgen05.mma.kind::f16, both K-major in the 128-byte swizzled layout.
+//
+// Roles of the 14 warps of a CTA (persistent over tiles):
+//   warp 0        TMA producer: x tile [BN x 64] per k-block, and TMEM owner
+//   warp 1        MMA issuer (one thread): 4 x tcgen05.mma (K = 16) per k-block
+//   warps 2..9    converters: one 16-row code tile each; every d-vector index
+//                 selects its exact bf16 codeword RN(A z + B) from a pack-time
+//                 table, written straight into the swizzled A tile
+//   warps 10..13  epilogue: tcgen05.ld of the accumulator, bf16, global store
+// The accumulator is double-buffered in TMEM so the epilogue of one tile runs
+// under the main loop of the next.
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
 #include "internal.h"
 
 namespace unisvq {
+namespace {
 
-bool prefill_supported(const unisvq_layer*, int) { return false; }
+constexpr int kPfThreads = 14 * 32;
+constexpr int kBM = 128;
+constexpr int kBK = 64;                  // bf16 columns per stage (one 128B swizzle row)
+constexpr int kATileBytes = kBM * 128;   // 16 KB
+constexpr int kConvWarp0 = 2;
+constexpr int kEpiWarp0 = 10;
 
-PrefillPlan plan_prefill(const unisvq_layer*, int) { return PrefillPlan{}; }
+struct PrefillArgs {
+  const uint8_t* codes;
+  const uint32_t* lut;   // d <= 2: 16 x bf16x2 pair codewords; d == 4: 256 x 4 bf16
+  uint16_t* y;
+  int M, N, K, KT, d;
+  int nkb;               // k-blocks of 64 columns: ceil(K / 64)
+  int mtiles, tiles;
+  int* err;
+};
 
-unisvq_status launch_prefill(const unisvq_layer*, const void*, void*, int, cudaStream_t) {
-  return UNISVQ_ERR_UNSUPPORTED;
+template <int BN, int STAGES>
+struct PfCfg {
+  static constexpr int kBTileBytes = BN * 128;
+  static constexpr int kStageBytes = kATileBytes + kBTileBytes;
+  static constexpr int kOffA = 0;
+  static constexpr int kOffB = STAGES * kATileBytes;
+  static constexpr int kOffLut = STAGES * kStageBytes;            // 2 KB
+  static constexpr int kOffBars = kOffLut + 2048;
+  // bars: bfull[S], afull[S], empty[S], accfull[2], accempty[2]
+  static constexpr int kOffTmemPtr = kOffBars + (3 * STAGES + 5) * 8;   // + drain barrier
+  static constexpr int kOffFlag = kOffTmemPtr + 8;
+  static constexpr int kSmem = kOffFlag + 8 + 1024;                // + alignment slack
+  static constexpr uint32_t kTmemCols = 2 * BN < 32 ? 32 : 2 * BN;
+};
+
+// ---- tcgen05 / TMA wrappers --------------------------------------------------
+
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
+// 128 bytes, 8-row core groups 1024 bytes apart (SBO), version 1 (sm_100+).
+__device__ __forceinline__ uint64_t make_sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);       // start address
+  d |= static_cast<uint64_t>(1) << 16;                       // LBO (unused for swizzled K-major)
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;               // SBO
+  d |= static_cast<uint64_t>(1) << 46;                       // descriptor version
+  d |= static_cast<uint64_t>(2) << 61;                       // SWIZZLE_128B
+  return d;
+}
+
+// Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major, M = 128.
+template <int BN>
+__device__ __forceinline__ uint32_t make_idesc() {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
+         (static_cast<uint32_t>(kBM >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int c0, int c1,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
+        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
+        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void sts64(uint32_t addr, uint32_t a, uint32_t b) {
+  asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
+}
+__device__ __forceinline__ uint32_t lds32(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(addr));
+  return v;
+}
+__device__ __forceinline__ uint2 lds64(uint32_t addr) {
+  uint2 v;
+  asm volatile("ld.shared.v2.b32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+  return v;
+}
+
+template <int BN, int STAGES>
+__global__ void __launch_bounds__(kPfThreads, 1)
+    prefill_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ PrefillArgs a) {
+  using C = PfCfg<BN, STAGES>;
+  extern __shared__ uint8_t smem_raw[];
+  // 1024-byte alignment for the 128B-swizzled tiles.
+  const uint32_t raw_addr = smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + ((1024 - (raw_addr & 1023)) & 1023);
+  const uint32_t sbase = smem_u32(smem);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t bar0 = sbase + C::kOffBars;
+  auto bfull = [&](int s) { return bar0 + 8u * s; };
+  auto afull = [&](int s) { return bar0 + 8u * (STAGES + s); };
+  auto empty = [&](int s) { return bar0 + 8u * (2 * STAGES + s); };
+  auto accfull = [&](int b) { return bar0 + 8u * (3 * STAGES + b); };
+  auto accempty = [&](int b) { return bar0 + 8u * (3 * STAGES + 2 + b); };
+  const uint32_t drain = bar0 + 8u * (3 * STAGES + 4);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffFlag);
+  uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::kOffTmemPtr);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(bfull(s), 1);
+      mbar_init(afull(s), 8);
+      mbar_init(empty(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(accfull(b), 1);
+      mbar_init(accempty(b), 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmap_x)) : "memory");
+  }
+  // Codeword table -> shared memory.
+  {
+    const int words = a.d == 4 ? 512 : 16;
+    uint32_t* lut_s = reinterpret_cast<uint32_t*>(smem + C::kOffLut);
+    for (int i = threadIdx.x; i < words; i += kPfThreads) lut_s[i] = a.lut[i];
+  }
+  if (warp == 0) {
+    tmem_alloc(sbase + C::kOffTmemPtr, C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_ptr;
+
+  if (warp == 0) {
+    // ---------------- TMA producer: activations ----------------
+    if (lane == 0) {
+      int it = 0;
+      for (int tile = blockIdx.x; tile < a.tiles && !*abort_flag; tile += gridDim.x) {
+        const int m0 = (tile % a.mtiles) * BN;
+        for (int kb = 0; kb < a.nkb; ++kb, ++it) {
+          const int s = it % STAGES;
+          if (it >= STAGES && !mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty)) {
+            *abort_flag = 1;
+            break;
+          }
+          mbar_arrive_expect_tx(bfull(s), C::kBTileBytes);
+          tma_load_2d(sbase + C::kOffB + s * C::kBTileBytes, &tmap_x, kb * kBK, m0, bfull(s));
+        }
+      }
+      // After an abort, loads nobody consumed must still land before exit.
+      if (*abort_flag)
+        for (int j = it - STAGES > 0 ? it - STAGES : 0; j < it; ++j)
+          mbar_wait(bfull(j % STAGES), (j / STAGES) & 1, a.err, kErrTimeoutFull);
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      const uint32_t idesc = make_idesc<BN>();
+      int it = 0, lt = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < a.tiles && ok; tile += gridDim.x, ++lt) {
+        const int b = lt & 1;
+        if (lt >= 2) {
+          ok = mbar_wait(accempty(b), ((lt >> 1) - 1) & 1, a.err, kErrTimeoutAcc);
+          if (!ok) break;
+        }
+        tc_fence_after();
+        const uint32_t dcol = tmem_base + static_cast<uint32_t>(b * BN);
+        for (int kb = 0; kb < a.nkb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1;
+          ok = !*abort_flag && mbar_wait(bfull(s), ph, a.err, kErrTimeoutFull) &&
+               mbar_wait(afull(s), ph, a.err, kErrTimeoutFull);
+          if (!ok) break;
+          tc_fence_after();
+          const uint64_t ad = make_sw128_desc(sbase + C::kOffA + s * kATileBytes);
+          const uint64_t bd = make_sw128_desc(sbase + C::kOffB + s * C::kBTileBytes);
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)   // +32 bytes per K=16 step inside the swizzle row
+            mma_bf16(dcol, ad + 2 * k, bd + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          mma_commit(empty(s));
+        }
+        if (!ok) break;
+        mma_commit(accfull(b));
+      }
+      if (!ok) *abort_flag = 1;
+      // Everything issued so far must retire before TMEM is released.
+      mma_commit(drain);
+      mbar_wait(drain, 0, a.err, kErrTimeoutMma);
+    }
+  } else if (warp < kEpiWarp0) {
+    // ---------------- converters: codes -> bf16 codeword tile ----------------
+    const int c = warp - kConvWarp0;            // 16-row code tile of this warp
+    const int g = lane >> 2, t = lane & 3;
+    const uint32_t lut_s = sbase + C::kOffLut;
+    int it = 0;
+    for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
+      const int n_blk = tile / a.mtiles;
+      const uint8_t* tbase =
+          a.codes + (static_cast<size_t>(n_blk * 8 + c) * a.KT) * kTileBytes + lane * 16;
+      uint4 cw = make_uint4(0, 0, 0, 0);
+      bool ok = !*abort_flag;
+      for (int kb = 0; kb < a.nkb; ++kb, ++it) {
+        const int s = it % STAGES;
+        if ((kb & 1) == 0) cw = __ldg(reinterpret_cast<const uint4*>(tbase + (kb >> 1) * kTileBytes));
+        if (ok && it >= STAGES) {
+          ok = !*abort_flag && mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty);
+          if (!ok) *abort_flag = 1;
+        }
+        if (ok) {
+          const uint32_t a_s = sbase + C::kOffA + s * kATileBytes;
+#pragma unroll
+          for (int rh = 0; rh < 2; ++rh) {
+            const uint32_t w = (kb & 1) ? (rh ? cw.w : cw.z) : (rh ? cw.y : cw.x);
+            const int r = c * 16 + g + 8 * rh;          // row within the 128-row tile
+            const uint32_t row_addr = a_s + r * 128 + ((t & 1) << 3);
+            const int sw = r & 7;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              uint32_t e0, e1;
+              if (a.d == 4) {
+                const uint32_t v = (w >> (4 * i)) & 0x000F000Fu;
+                const uint32_t idx = (v & 0xFu) | ((v >> 12) & 0xF0u);
+                const uint2 q = lds64(lut_s + idx * 8);
+                e0 = q.x;
+                e1 = q.y;
+              } else {
+                const uint32_t v0 = (w >> (4 * i)) & 0x00030003u;
+                const uint32_t v1 = (w >> (4 * i + 2)) & 0x00030003u;
+                e0 = lds32(lut_s + (((v0 & 3u) | ((v0 >> 14) & 0xCu)) << 2));
+                e1 = lds32(lut_s + (((v1 & 3u) | ((v1 >> 14) & 0xCu)) << 2));
+              }
+              sts64(row_addr + ((((2 * i) + (t >> 1)) ^ sw) << 4), e0, e1);
+            }
+          }
+          fence_proxy_async_smem();
+        }
+        __syncwarp();
+        if (lane == 0 && ok) mbar_arrive(afull(s));
+      }
+    }
+  } else {
+    // ---------------- epilogue ----------------
+    const int q = warp & 3;                      // TMEM lane quarter of this warp
+    int lt = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < a.tiles && ok; tile += gridDim.x, ++lt) {
+      const int b = lt & 1;
+      const int n0 = (tile / a.mtiles) * kBM;
+      const int m0 = (tile % a.mtiles) * BN;
+      ok = !*abort_flag && mbar_wait(accfull(b), (lt >> 1) & 1, a.err, kErrTimeoutMma);
+      if (!ok) {
+        *abort_flag = 1;
+        break;
+      }
+      tc_fence_after();
+      const int n = n0 + 32 * q + lane;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        uint32_t r[32];
+        tmem_ld32(tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(b * BN + c0), r);
+        if (n < a.N) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const int m = m0 + c0 + j;
+            if (m < a.M) a.y[static_cast<size_t>(m) * a.N + n] = f32_to_bf16_rn(__uint_as_float(r[j]));
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(accempty(b));
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::kTmemCols);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+template <int BN, int STAGES>
+unisvq_status launch_bn(const unisvq_layer* L, const PrefillPlan& p, const void* x, void* y, int M,
+                        cudaStream_t s) {
+  using C = PfCfg<BN, STAGES>;
+  static bool attr_set[64] = {};
+  const int dev = L->device;
+  if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
+  if (!attr_set[dev]) {
+    if (cudaFuncSetAttribute(prefill_kernel<BN, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::kSmem) != cudaSuccess)
+      return UNISVQ_ERR_CUDA;
+    attr_set[dev] = true;
+  }
+  PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode();
+  if (!enc) return UNISVQ_ERR_CUDA;
+  CUtensorMap map;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(L->K), static_cast<cuuint64_t>(M)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(L->K) * 2};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), static_cast<cuuint32_t>(BN)};
+  const cuuint32_t estr[2] = {1, 1};
+  if (enc(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(x), dims, strides, box, estr,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return UNISVQ_ERR_CUDA;
+
+  PrefillArgs a{};
+  a.codes = L->codes;
+  a.lut = L->tlut;
+  a.y = static_cast<uint16_t*>(y);
+  a.M = M;
+  a.N = L->N;
+  a.K = L->K;
+  a.KT = L->KT;
+  a.d = L->d;
+  a.nkb = (L->K + kBK - 1) / kBK;
+  a.mtiles = (M + BN - 1) / BN;
+  a.tiles = p.tiles;
+  a.err = device_error_word();
+  prefill_kernel<BN, STAGES><<<p.grid, kPfThreads, C::kSmem, s>>>(map, a);
+  return cudaGetLastError() == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+}
+
+int pick_bn(int M) { return M <= 64 ? 64 : (M <= 128 ? 128 : 256); }
+
+}  // namespace
+
+bool prefill_supported(const unisvq_layer* L, int M) {
+  return M > 0 && (L->K % 8) == 0 && get_encode() != nullptr;
+}
+
+PrefillPlan plan_prefill(const unisvq_layer* L, int M) {
+  PrefillPlan p{};
+  p.bn = pick_bn(M);
+  const int mtiles = (M + p.bn - 1) / p.bn;
+  p.tiles = (L->Np / kBM) * mtiles;
+  p.grid = p.tiles < L->num_sms ? p.tiles : L->num_sms;
+  if (p.grid < 1) p.grid = 1;
+  p.smem = p.bn == 64 ? PfCfg<64, 8>::kSmem : (p.bn == 128 ? PfCfg<128, 6>::kSmem : PfCfg<256, 4>::kSmem);
+  return p;
+}
+
+unisvq_status launch_prefill(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
+  const PrefillPlan p = plan_prefill(L, M);
+  if (p.bn == 64) return launch_bn<64, 8>(L, p, x, y, M, s);
+  if (p.bn == 128) return launch_bn<128, 6>(L, p, x, y, M, s);
+  return launch_bn<256, 4>(L, p, x, y, M, s);
 }
 
 }  // namespace unisvq

@@ -136,18 +136,43 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
   L->colnorm = static_cast<float>(colnorm) * (1.0f + 1e-6f);
 
   // Codebook of Eq. (def:unisvq): entry v holds A z(v) + B, z_c(v) = (v >> 2c) & 3,
-  // exact in fp64, rounded once to fp32 and to bf16.
+  // exact in fp64 and rounded once (to fp32 here, to bf16 below).
   const int E = 1 << (2 * d);
   L->lut_entries = E;
+  std::vector<double> cb(static_cast<size_t>(E) * d);
   std::vector<float> lut32(static_cast<size_t>(E) * d);
-  std::vector<uint16_t> lut16(static_cast<size_t>(E) * d);
   for (int v = 0; v < E; ++v)
     for (int r = 0; r < d; ++r) {
       double w = B[r];
       for (int c = 0; c < d; ++c) w += A[r * d + c] * static_cast<double>((v >> (2 * c)) & 3);
+      cb[static_cast<size_t>(v) * d + r] = w;
       lut32[static_cast<size_t>(v) * d + r] = static_cast<float>(w);
-      lut16[static_cast<size_t>(v) * d + r] = f64_to_bf16_rne(w);
     }
+  // Prefill tile table, indexed the way the converter warps read a code word:
+  //   d <= 2: 16 bf16 pairs, index lo | hi << 2 for the two columns (k, k+1)
+  //           sharing one word position;
+  //   d == 4: 256 bf16 quads, index z0 | z2 << 2 | z1 << 4 | z3 << 6 (the order
+  //           in which two adjacent positions of a word hold columns 4m..4m+3).
+  auto bf = [](double w) { return static_cast<uint32_t>(f64_to_bf16_rne(w)); };
+  std::vector<uint32_t> tlut;
+  if (d <= 2) {
+    tlut.resize(16);
+    for (int v = 0; v < 16; ++v) {
+      const int lo = v & 3, hi = v >> 2;
+      const double w0 = d == 2 ? cb[static_cast<size_t>(lo | (hi << 2)) * 2 + 0] : cb[lo];
+      const double w1 = d == 2 ? cb[static_cast<size_t>(lo | (hi << 2)) * 2 + 1] : cb[hi];
+      tlut[v] = bf(w0) | (bf(w1) << 16);
+    }
+  } else {
+    tlut.resize(512);
+    for (int idx = 0; idx < 256; ++idx) {
+      const int z0 = idx & 3, z2 = (idx >> 2) & 3, z1 = (idx >> 4) & 3, z3 = (idx >> 6) & 3;
+      const size_t v = static_cast<size_t>(z0 | (z1 << 2) | (z2 << 4) | (z3 << 6));
+      tlut[2 * idx] = bf(cb[v * 4 + 0]) | (bf(cb[v * 4 + 1]) << 16);
+      tlut[2 * idx + 1] = bf(cb[v * 4 + 2]) | (bf(cb[v * 4 + 3]) << 16);
+    }
+  }
+  L->tlut_words = static_cast<int>(tlut.size());
 
   L->code_bytes = unisvq_packed_code_bytes(N, K);
   std::vector<uint8_t> packed;
@@ -162,18 +187,18 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = cudaMalloc(&L->codes, L->code_bytes);
   if (e == cudaSuccess) e = cudaMalloc(&L->lut32, lut32.size() * sizeof(float));
-  if (e == cudaSuccess) e = cudaMalloc(&L->lut16, lut16.size() * sizeof(uint16_t));
+  if (e == cudaSuccess) e = cudaMalloc(&L->tlut, tlut.size() * sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMemcpyAsync(L->codes, packed.data(), L->code_bytes, cudaMemcpyHostToDevice, s);
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(L->lut32, lut32.data(), lut32.size() * sizeof(float), cudaMemcpyHostToDevice, s);
   if (e == cudaSuccess)
-    e = cudaMemcpyAsync(L->lut16, lut16.data(), lut16.size() * sizeof(uint16_t), cudaMemcpyHostToDevice, s);
+    e = cudaMemcpyAsync(L->tlut, tlut.data(), tlut.size() * sizeof(uint32_t), cudaMemcpyHostToDevice, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e == cudaSuccess && !device_error_word()) e = cudaErrorUnknown;
   if (e != cudaSuccess) {
     cudaFree(L->codes);
     cudaFree(L->lut32);
-    cudaFree(L->lut16);
+    cudaFree(L->tlut);
     delete L;
     return cuda_status(e);
   }
@@ -188,21 +213,21 @@ unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
   if (!L) return UNISVQ_ERR_OOM;
   L->codes = nullptr;
   L->lut32 = nullptr;
-  L->lut16 = nullptr;
+  L->tlut = nullptr;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const size_t n32 = static_cast<size_t>(h->lut_entries) * h->d * sizeof(float);
-  const size_t n16 = static_cast<size_t>(h->lut_entries) * h->d * sizeof(uint16_t);
+  const size_t n16 = static_cast<size_t>(h->tlut_words) * sizeof(uint32_t);
   cudaError_t e = cudaMalloc(&L->codes, h->code_bytes);
   if (e == cudaSuccess) e = cudaMalloc(&L->lut32, n32);
-  if (e == cudaSuccess) e = cudaMalloc(&L->lut16, n16);
+  if (e == cudaSuccess) e = cudaMalloc(&L->tlut, n16);
   if (e == cudaSuccess) e = cudaMemcpyAsync(L->codes, h->codes, h->code_bytes, cudaMemcpyDeviceToDevice, s);
   if (e == cudaSuccess) e = cudaMemcpyAsync(L->lut32, h->lut32, n32, cudaMemcpyDeviceToDevice, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(L->lut16, h->lut16, n16, cudaMemcpyDeviceToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(L->tlut, h->tlut, n16, cudaMemcpyDeviceToDevice, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) {
     cudaFree(L->codes);
     cudaFree(L->lut32);
-    cudaFree(L->lut16);
+    cudaFree(L->tlut);
     delete L;
     return cuda_status(e);
   }
@@ -214,7 +239,7 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
   if (!h) return UNISVQ_OK;
   cudaError_t e1 = cudaFree(h->codes);
   cudaError_t e2 = cudaFree(h->lut32);
-  cudaError_t e3 = cudaFree(h->lut16);
+  cudaError_t e3 = cudaFree(h->tlut);
   delete h;
   return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess) ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }

@@ -177,3 +177,66 @@ def test_full_size_decode_sampled_rows(N, K):
         xb = synth.activations(0, 3, M, M, K)
         check(run(layer, xb), xb, codes, A, B, rows=rows)
     layer.close()
+
+
+# ---------------------------------------------------------------------------
+# prefill (tcgen05) kernel
+# ---------------------------------------------------------------------------
+
+PREFILL_SHAPES = [(128, 128), (200, 520), (384, 1024), (1000, 2048)]
+
+
+@pytest.mark.parametrize("d", [1, 2, 4])
+@pytest.mark.parametrize("N,K", PREFILL_SHAPES)
+def test_prefill_parity(d, N, K):
+    codes, A, B = synth.layer_inputs(8, 80, N, K, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    for M in (33, 64, 65, 128, 200, 256, 300, 777):
+        xb = synth.activations(8, 80, 1000 * N + M, M, K)
+        check(run(layer, xb, binding.KERNEL_PREFILL), xb, codes, A, B)
+    layer.close()
+
+
+def test_prefill_integer_case_bit_exact():
+    d = 4
+    A = np.array([[1, -1, 0, 0], [0, 1, -1, 0], [0, 0, 1, -1], [0, 0, 1, 1]], dtype=np.float16)
+    B = np.array([1, -2, 0, 1], dtype=np.float16)
+    N, K = 256, 512
+    g = np.random.default_rng(12)
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    layer = binding.UniSVQLinear(codes, A, B)
+    for M in (40, 300):
+        x = g.integers(-1, 2, size=(M, K)).astype(np.float32) * (g.random((M, K)) < 0.05)
+        xb = synth.f32_to_bf16_bits(x)
+        yr, _ = oracle.linear(xb, codes, A, B)
+        assert np.abs(yr).max() <= 256
+        yg = run(layer, xb, binding.KERNEL_PREFILL)
+        assert np.array_equal(yg, yr), np.abs(yg - yr).max()
+    layer.close()
+
+
+def test_prefill_and_decode_agree_with_auto_dispatch():
+    N, K, d = 512, 1024, 2
+    codes, A, B = synth.layer_inputs(9, 90, 0, 0, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    assert layer.query(1)["kernel"] == binding.KERNEL_DECODE
+    assert layer.query(2048)["kernel"] == binding.KERNEL_PREFILL
+    xb = synth.activations(9, 90, 0, 96, K)
+    check(run(layer, xb), xb, codes, A, B)
+    layer.close()
+
+
+@pytest.mark.parametrize("N,K", [(4096, 4096), (1024, 4096), (14336, 4096), (4096, 14336)])
+def test_full_size_prefill_sampled_rows(N, K):
+    """Llama-3-8B-shaped projections at M = 2048 (the prefill workload)."""
+    d = 2
+    codes, A, B = synth.layer_inputs(0, 2, 0, N + K, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    rows = np.unique(np.concatenate([np.sort(synth.rng(1, N, K).choice(N, size=24, replace=False)), [0, N - 1]]))
+    M = 2048
+    xb = synth.activations(0, 2, K, M, K)
+    yg = run(layer, xb)
+    yr, S = oracle.linear(xb, codes[rows], A, B)
+    res = oracle.compare(yg[:, rows], yr, S)
+    assert res["ok"], res
+    layer.close()
