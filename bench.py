@@ -202,18 +202,21 @@ def build_stack(binding, shapes, layers, config_id, d=2):
 
 
 def time_graphs(torch, graphs, steps, warmup, stream):
-    for _ in range(warmup):
-        for g in graphs:
-            g.replay()
-    torch.cuda.synchronize()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(steps):
-        for g in graphs:
-            g.replay()
-    e1.record(stream)
-    torch.cuda.synchronize()
+    """Replay `graphs` `steps` times on `stream`; seconds between CUDA events
+    recorded on that same stream (graph replays launch on the current stream)."""
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            for g in graphs:
+                g.replay()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            for g in graphs:
+                g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
     return e0.elapsed_time(e1) / 1000.0
 
 
@@ -225,6 +228,12 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     binding.load()
     peaks, peak_src = load_peaks()
+    if args.only == "prefill":
+        side = torch.cuda.Stream()
+        print(json.dumps({"prefill": run_prefill(torch, binding, peaks, args, side)}), flush=True)
+        return
+    if args.only == "decode":
+        args.no_e2e = args.no_cpu = args.no_prefill = True
     shapes = synth.LLAMA2_7B
     stack = build_stack(binding, shapes, args.layers, 1)
 
@@ -444,6 +453,8 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--only", choices=["decode", "prefill"], default=None,
+                    help="profiling aid: run only the decode sweep (no e2e/cpu/prefill) or only the prefill set")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -44,9 +44,11 @@ typedef enum {
 
 /* Kernel selectors for unisvq_linear_force and unisvq_info.kernel. */
 enum {
-  UNISVQ_KERNEL_AUTO = 0,    /* pick by M (unisvq_linear does this)            */
-  UNISVQ_KERNEL_DECODE = 1,  /* fold + register-unpack tensor-core GEMV, M<=32 */
-  UNISVQ_KERNEL_PREFILL = 2  /* tcgen05 GEMM, bf16 codeword tiles in smem      */
+  UNISVQ_KERNEL_AUTO = 0,     /* pick by M (unisvq_linear does this)                   */
+  UNISVQ_KERNEL_DECODE = 1,   /* the decode kernel for this M (GEMV or SKINNY)         */
+  UNISVQ_KERNEL_PREFILL = 2,  /* tcgen05 GEMM, exact bf16 codeword tiles in smem       */
+  UNISVQ_KERNEL_GEMV = 3,     /* fold + register-operand tensor-core GEMV, M <= 16/launch */
+  UNISVQ_KERNEL_SKINNY = 4    /* fold + tcgen05 with codes as 8-bit TMEM operand, M <= 64/launch */
 };
 
 /*
@@ -54,24 +56,22 @@ enum {
  * that other tools can produce or check it).
  *
  * The matrix is padded to Np = roundup(N, 128) rows and Kp = roundup(K, 128)
- * columns with code 0 and cut into tiles of 16 rows x 128 columns, 512 bytes
- * each. Tile (rt, kt), rt < Np/16, kt < Kp/128, starts at byte
- * (rt * (Kp/128) + kt) * 512, so the tiles of one 16-row strip are
+ * columns with code 0 and cut into tiles of 128 rows x 128 columns, 4096
+ * bytes each. Tile (rb, kt), rb < Np/128, kt < Kp/128, starts at byte
+ * (rb * (Kp/128) + kt) * 4096, so the tiles of one 128-row block are
  * consecutive along K.
  *
- * Inside a tile, lane l in [0, 32) owns bytes [16 l, 16 l + 16) as four
- * little-endian 32-bit words W[q], q in [0, 4). With g = l / 4, t = l % 4,
- * grp = q / 2 and rh = q % 2, word W[q] holds 16 codes of row
- *   n = 16 rt + g + 8 rh
- * at 8 positions p in [0, 8): with i = p / 2 and h = p % 2, the column
- *   k = 128 kt + 64 grp + 16 i + 4 t + 2 h
- * sits in bits [2p+1 : 2p] and column k + 1 in bits [16+2p+1 : 16+2p].
- * Every run of 4 columns 4m .. 4m+3 therefore sits in one word, so vectors
- * of d = 1, 2 or 4 never straddle words.
+ * Inside a tile, half h (columns 64h .. 64h+63) fills bytes [2048h, 2048h+2048)
+ * and row r of the tile owns the 16 bytes at 2048h + 16r: four little-endian
+ * 32-bit words w0..w3. Word wi holds the 16 codes of columns
+ *   k = 128 kt + 64 h + 16 wi + 4 s + b,   s, b in 0..3,
+ * the code of column k in bits [8b+2s+1 : 8b+2s]. Shifting a word right by 2s
+ * and masking with 0x03030303 yields the codes of columns 4s..4s+3 one per
+ * byte; a run of 4 columns 4m..4m+3 therefore never spans two words.
  */
-#define UNISVQ_TILE_ROWS 16
+#define UNISVQ_TILE_ROWS 128
 #define UNISVQ_TILE_COLS 128
-#define UNISVQ_TILE_BYTES 512
+#define UNISVQ_TILE_BYTES 4096
 
 typedef struct unisvq_layer* unisvq_handle;
 

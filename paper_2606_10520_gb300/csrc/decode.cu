@@ -1,38 +1,42 @@
-// Decode GEMV / skinny GEMM for M <= 32 tokens (HBM-bound path).
+// Skinny GEMM for decode batches (M <= 64 tokens per launch): tcgen05 tensor cores
+// with the 2-bit codes as an 8-bit operand resident in tensor memory.
 //
 // Computes y = x W_hat^T through the fold of Eq. (col:matmul):
 //   y[m, n] = sum_k x'[m, k] z[n, k] + c[m],
-//   x'[m, g d + c] = sum_r x[m, g d + r] A[r][c]   (the row vectors X_i A),
-//   c[m]          = sum_g x[m, g d .. g d + d - 1] . B  (the X_i B terms),
-// so the 2-bit codes are never turned into weights: they go from the code
-// stream straight into tensor-core A-operand registers.
+//   x'[m, g d + c] = sum_r x[m, g d + r] A[r][c]      (the row vectors X_i A)
+//   c[m]          = sum_g x[m, g d .. g d + d - 1] . B  (the X_i B terms)
+// so the codes are never turned into weights. Each code z becomes the byte z,
+// which is exactly the e4m3 subnormal z * 2^-9; one shift and one AND expand
+// four codes (layout.h) and tcgen05.st writes them as the A operand of
+// tcgen05.mma.kind::f8f6f4 (128 rows in TMEM lanes). The folded activations,
+// scaled per token by 2^P so that |x' 2^P| < 256, are split into three e4m3
+// terms h + m + l (about 12 significant bits, the precision of fp16) that
+// form three B operands in 128B-swizzled shared memory and accumulate into the
+// same fp32 TMEM accumulator; the epilogue multiplies by 2^(9 - P).
 //
-// Per CTA: 128 output rows (8 consumer warps x 16 rows) times a slice of K;
-// the KS CTAs that share the rows form a cluster and add their partial sums
-// through distributed shared memory. A producer warp streams the slice's code
-// tiles into a shared-memory ring with 1-D bulk copies before waiting on the
-// previous kernel (codes never depend on it), so under programmatic dependent
-// launch the code stream of this layer overlaps the tail of the last one.
-//
-// Code -> MMA operand: one AND per fp16x2 register (layout.h). The extracted
-// halves are fp16 subnormals z * 4^s * 2^-24; the folded activations are
-// stored as fp16 x' * 2^P * 4^-s (P per token, chosen so the largest |x'| in
-// the CTA's slice stays below 2^15), so every product is x' z 2^(P-24) and the
-// fp32 accumulator is rescaled by 2^(24-P) once at the end.
+// CTA = 128 output rows x one K slice; the KS CTAs sharing the rows form a
+// thread-block cluster and add their partial sums through distributed shared
+// memory. Warp roles (10 warps):
+//   0      producer: 4 KB code tiles -> shared-memory ring (cp.async.bulk)
+//   1      TMEM owner; one thread issues the MMAs
+//   2..5   converters: shared ring -> TMEM A slots (one row per thread), then
+//          the epilogue (tcgen05.ld of their 32 accumulator rows)
+//   6..9   fold: x -> per-token scale, x' = x_g A, three e4m3 B terms
+// Producer and converters never touch x, so they run before the programmatic-
+// launch wait: while the previous kernel finishes, this layer's codes already
+// stream into shared memory and TMEM.
 #include "common.cuh"
 #include "internal.h"
 
 namespace unisvq {
 namespace {
 
-constexpr int kDecWarps = 8;
-constexpr int kDecThreads = (kDecWarps + 1) * 32;
-constexpr int kDecRows = kDecWarps * kTileRows;   // 128 rows per CTA
-constexpr int kKB = 2;                            // k-tiles per ring stage
-constexpr int kStages = 4;
-constexpr int kMaxTok = 32;
-constexpr int kConsumerThreads = kDecWarps * 32;
-constexpr uint32_t kFoldBarrier = 1;
+constexpr int kThreads = 10 * 32;
+constexpr int kFoldWarp0 = 6;
+constexpr int kTmemCols = 256;
+constexpr int kAColBase = 64;        // A slots start here; the accumulator uses [0, NTOK)
+constexpr int kASlots = (kTmemCols - kAColBase) / 32;
+constexpr int kMaxTokPerLaunch = 64;
 
 struct DecodeArgs {
   const uint8_t* codes;
@@ -42,47 +46,100 @@ struct DecodeArgs {
   int kt_per_cta;
   float A[16];
   float B[4];
-  float colnorm;
+  float colnorm;       // max_c sum_r |A[r][c]|
   int* err;
 };
 
-template <int NT>
-struct DecCfg {
-  static constexpr int CH = NT == 1 ? 8 : (NT == 2 ? 4 : 2);   // k-tiles per fold chunk
-  static constexpr int MP = 8 * NT;                              // padded tokens
-  static constexpr int kStageBytes = kDecWarps * kKB * kTileBytes;
-  static constexpr int kXfragBytes = NT * CH * 8 * 32 * 8;       // one fold buffer
-  static constexpr int kOffBars = 0;
-  static constexpr int kOffTok = 128;
-  static constexpr int kOffRing = 1024;
-  static constexpr int kOffXfrag = kOffRing + kStages * kStageBytes;
-  static constexpr int kOffRed = kOffXfrag + 2 * kXfragBytes;
-  static constexpr int kSmem = kOffRed + kDecRows * MP * 4;
+template <int NTOK>
+struct Cfg {
+  static constexpr int kCodeStages = NTOK == 64 ? 4 : 8;
+  static constexpr int kBStages = NTOK == 16 ? 4 : 2;
+  static constexpr int kTermBytes = NTOK * 128;                  // one e4m3 B tile (128 columns)
+  static constexpr int kBStageBytes = 3 * kTermBytes;
+  static constexpr int kOffCode = 0;
+  static constexpr int kOffB = kOffCode + kCodeStages * kTileBytes;
+  static constexpr int kOffX = kOffB + kBStages * kBStageBytes;
+  static constexpr int kXBytes = NTOK == 64 ? 8192 : 32768;      // staged x slice (bf16)
+  static constexpr int kOffRed = kOffX + kXBytes;
+  static constexpr int kRedBytes = (kTileRows + 8) * NTOK * 4;
+  static constexpr int kOffBars = kOffRed + kRedBytes;
+  static constexpr int kNumBars = 2 * kCodeStages + 2 * kASlots + 2 * kBStages + 4;
+  static constexpr int kOffTok = kOffBars + kNumBars * 8;        // pexp[64], cpart[64]
+  static constexpr int kOffMisc = kOffTok + 512;                 // tmem ptr, abort flag
+  static constexpr int kSmem = kOffMisc + 64 + 1024;             // + alignment slack
+  static constexpr uint32_t kIdesc =
+      (1u << 4) | (0u << 7) | (0u << 10) | (static_cast<uint32_t>(NTOK >> 3) << 17) | ((128u >> 4) << 24);
 };
 
-__device__ __forceinline__ void mma_f16_16816(float (&d)[4], uint32_t a0, uint32_t a1,
-                                              uint32_t a2, uint32_t a3, uint32_t b0,
-                                              uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
-      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+// ---- tcgen05 wrappers ----------------------------------------------------------
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4) | (static_cast<uint64_t>(1) << 16) |
+         (static_cast<uint64_t>(1024 >> 4) << 32) | (static_cast<uint64_t>(1) << 46) |
+         (static_cast<uint64_t>(2) << 61);
 }
 
-// Four consecutive activations x[k .. k+3] of one token (zero past K).
-__device__ __forceinline__ void load4(const uint16_t* xr, int k, int K, float (&v)[4]) {
-  if ((K & 3) == 0 && k + 3 < K) {
-    const uint2 u = __ldg(reinterpret_cast<const uint2*>(xr + k));
-    v[0] = bf16_lo(u.x);
-    v[1] = bf16_hi(u.x);
-    v[2] = bf16_lo(u.y);
-    v[3] = bf16_hi(u.y);
-  } else {
-#pragma unroll
-    for (int e = 0; e < 4; ++e)
-      v[e] = (k + e < K) ? __uint_as_float(static_cast<uint32_t>(xr[k + e]) << 16) : 0.f;
-  }
+__device__ __forceinline__ void mma_f8_tmem_a(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                              uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
+      "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]),
+      "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]),
+      "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
+// e4m3x2 <-> f16x2 (lower byte <-> lower half).
+__device__ __forceinline__ uint16_t f16x2_to_e4m3x2(uint32_t v) {
+  uint16_t r;
+  asm("cvt.rn.satfinite.e4m3x2.f16x2 %0, %1;" : "=h"(r) : "r"(v));
+  return r;
+}
+__device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint16_t v) {
+  uint32_t r;
+  asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(r) : "h"(v));
+  return r;
+}
+__device__ __forceinline__ uint32_t hsub2(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
+// Split an f16 pair into three e4m3 pairs h + m + l (each residual is exact in f16).
+__device__ __forceinline__ void split3(uint32_t v, uint16_t& h, uint16_t& m, uint16_t& l) {
+  h = f16x2_to_e4m3x2(v);
+  const uint32_t r1 = hsub2(v, e4m3x2_to_f16x2(h));
+  m = f16x2_to_e4m3x2(r1);
+  const uint32_t r2 = hsub2(r1, e4m3x2_to_f16x2(m));
+  l = f16x2_to_e4m3x2(r2);
 }
 
 // x'[k+c] for the d-vectors inside x[k .. k+3] (k % 4 == 0): row vector x_g A.
@@ -102,240 +159,354 @@ __device__ __forceinline__ void fold4(const DecodeArgs& a, const float (&v)[4], 
   }
 }
 
-template <int NT>
-__global__ void __launch_bounds__(kDecThreads, 2) decode_kernel(const __grid_constant__ DecodeArgs a) {
-  using C = DecCfg<NT>;
-  extern __shared__ __align__(1024) uint8_t smem[];
-  const int tid = threadIdx.x;
-  const int warp = tid >> 5;
-  const int lane = tid & 31;
+// Activations x[k .. k+3] of one token as packed bf16 (zero at or past kend).
+__device__ __forceinline__ uint2 load_x4(const uint16_t* row, int k, int kend, bool vec) {
+  if (vec && k + 3 < kend) return __ldg(reinterpret_cast<const uint2*>(row + k));
+  uint32_t e[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) e[j] = (k + j < kend) ? static_cast<uint32_t>(row[k + j]) : 0u;
+  return make_uint2(e[0] | (e[1] << 16), e[2] | (e[3] << 16));
+}
+
+template <int NTOK>
+__global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_constant__ DecodeArgs a) {
+  using C = Cfg<NTOK>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + ((1024 - (raw & 1023)) & 1023);
+  const uint32_t sbase = smem_u32(smem);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int KS = gridDim.x;
   const int kt0 = blockIdx.x * a.kt_per_cta;
   const int n_kt = min(a.kt_per_cta, a.KT - kt0);
-  const int n_st = (n_kt + kKB - 1) / kKB;
-  const int rt0 = blockIdx.y * kDecWarps;
+  const int rb = blockIdx.y;
 
-  const uint32_t bar0 = smem_u32(smem + C::kOffBars);
-  auto full_bar = [&](int s) { return bar0 + 8u * s; };
-  auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
-  float* xmax = reinterpret_cast<float*>(smem + C::kOffTok);
-  float* cpart = reinterpret_cast<float*>(smem + C::kOffTok + 128);
-  int* pexp = reinterpret_cast<int*>(smem + C::kOffTok + 256);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffTok + 384);
+  const uint32_t bar0 = sbase + C::kOffBars;
+  auto code_full = [&](int s) { return bar0 + 8u * s; };
+  auto code_empty = [&](int s) { return bar0 + 8u * (C::kCodeStages + s); };
+  auto a_full = [&](int s) { return bar0 + 8u * (2 * C::kCodeStages + s); };
+  auto a_empty = [&](int s) { return bar0 + 8u * (2 * C::kCodeStages + kASlots + s); };
+  auto b_full = [&](int s) { return bar0 + 8u * (2 * C::kCodeStages + 2 * kASlots + s); };
+  auto b_empty = [&](int s) { return bar0 + 8u * (2 * C::kCodeStages + 2 * kASlots + C::kBStages + s); };
+  const uint32_t bar_tail = bar0 + 8u * (2 * C::kCodeStages + 2 * kASlots + 2 * C::kBStages);
+  const uint32_t d_full = bar_tail, tmem_ready = bar_tail + 8, fold_done = bar_tail + 16, drain = bar_tail + 24;
+  int* pexp = reinterpret_cast<int*>(smem + C::kOffTok);
+  float* cpart = reinterpret_cast<float*>(smem + C::kOffTok + 256);
+  uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 8);
   float* red = reinterpret_cast<float*>(smem + C::kOffRed);
 
   if (tid == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), kDecWarps);
+    for (int s = 0; s < C::kCodeStages; ++s) {
+      mbar_init(code_full(s), 1);
+      mbar_init(code_empty(s), 4);
     }
-    *abort_flag = (n_kt <= 0) ? 1 : 0;
+    for (int s = 0; s < kASlots; ++s) {
+      mbar_init(a_full(s), 4);
+      mbar_init(a_empty(s), 1);
+    }
+    for (int s = 0; s < C::kBStages; ++s) {
+      mbar_init(b_full(s), 1);
+      mbar_init(b_empty(s), 1);
+    }
+    mbar_init(d_full, 1);
+    mbar_init(tmem_ready, 1);
+    mbar_init(fold_done, 4);
+    mbar_init(drain, 1);
+    *abort_flag = n_kt <= 0 ? 1 : 0;
     if (n_kt <= 0) record_error(a.err, kErrBadLaunch);
     fence_mbar_init();
-  }
-  if (tid < kMaxTok) {
-    xmax[tid] = 0.f;
-    cpart[tid] = 0.f;
-    pexp[tid] = 0;
-  }
-  {  // zero both fold buffers: tokens >= M stay zero for the whole kernel
-    uint4* xf = reinterpret_cast<uint4*>(smem + C::kOffXfrag);
-    for (int i = tid; i < 2 * C::kXfragBytes / 16; i += kDecThreads) xf[i] = make_uint4(0, 0, 0, 0);
   }
   __syncthreads();
   pdl_launch_dependents();
 
-  int issued = 0;
-  if (warp == kDecWarps) {
-    // ---------------- producer: code tiles -> shared-memory ring ----------------
+  if (warp == 0) {
+    // ---------------- producer: code tiles -> shared ring ----------------
     if (lane == 0 && !*abort_flag) {
       const uint64_t pol = policy_evict_first();
-      for (int st = 0; st < n_st; ++st) {
-        const int slot = st % kStages;
-        if (st >= kStages &&
-            !mbar_wait(empty_bar(slot), ((st / kStages) - 1) & 1, a.err, kErrTimeoutEmpty)) {
+      const uint8_t* src = a.codes + (static_cast<size_t>(rb) * a.KT + kt0) * kTileBytes;
+      int kt = 0;
+      for (; kt < n_kt; ++kt) {
+        const int s = kt % C::kCodeStages;
+        if (kt >= C::kCodeStages &&
+            !mbar_wait(code_empty(s), ((kt / C::kCodeStages) - 1) & 1, a.err, kErrTimeoutEmpty)) {
           *abort_flag = 1;
           break;
         }
         if (*abort_flag) break;
-        const int nk = min(kKB, n_kt - st * kKB);
-        mbar_arrive_expect_tx(full_bar(slot), kDecWarps * nk * kTileBytes);
-        const uint32_t dst = smem_u32(smem + C::kOffRing + slot * C::kStageBytes);
-        for (int r = 0; r < kDecWarps; ++r) {
-          const uint8_t* src =
-              a.codes + (static_cast<size_t>(rt0 + r) * a.KT + kt0 + st * kKB) * kTileBytes;
-          bulk_g2s(dst + r * kKB * kTileBytes, src, nk * kTileBytes, full_bar(slot), pol);
-        }
-        issued = st + 1;
+        mbar_arrive_expect_tx(code_full(s), kTileBytes);
+        bulk_g2s(sbase + C::kOffCode + s * kTileBytes, src + static_cast<size_t>(kt) * kTileBytes, kTileBytes,
+                 code_full(s), pol);
       }
+      if (*abort_flag)   // copies nobody consumed must land before exit
+        for (int j = kt - C::kCodeStages > 0 ? kt - C::kCodeStages : 0; j < kt; ++j)
+          mbar_wait(code_full(j % C::kCodeStages), (j / C::kCodeStages) & 1, a.err, kErrTimeoutFull);
     }
-  } else {
-    // ---------------- consumers ----------------
-    pdl_wait();   // x may be the previous kernel's output
-    const int kend = min(a.K, (kt0 + n_kt) * kTileCols);
-    const int kbeg = kt0 * kTileCols;
-
-    // Per-token max |x| and partial sum_g x_g . B over this CTA's K slice.
-    for (int tok = warp; tok < a.M; tok += kDecWarps) {
-      const uint16_t* xr = a.x + static_cast<size_t>(tok) * a.K;
-      float mx = 0.f, cp = 0.f;
-      for (int k = kbeg + 4 * lane; k < kend; k += 128) {
-        float v[4];
-        load4(xr, k, a.K, v);
+  } else if (warp == 1) {
+    // ---------------- TMEM owner + MMA issuer ----------------
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     sbase + C::kOffMisc),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) {
+      mbar_arrive(tmem_ready);
+      tc_fence_after();
+      const uint32_t tbase = *tmem_ptr;
+      bool ok = !*abort_flag;
+      for (int kt = 0; kt < n_kt && ok; ++kt) {
+        const int sa = kt % kASlots, sb = kt % C::kBStages;
+        ok = !*abort_flag && mbar_wait(a_full(sa), (kt / kASlots) & 1, a.err, kErrTimeoutFull) &&
+             mbar_wait(b_full(sb), (kt / C::kBStages) & 1, a.err, kErrTimeoutFull);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t acol = tbase + kAColBase + 32 * sa;
+        const uint32_t bst = sbase + C::kOffB + sb * C::kBStageBytes;
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          mx = fmaxf(mx, fabsf(v[e]));
-          cp = fmaf(v[e], a.B[e & (a.d - 1)], cp);
+        for (int term = 0; term < 3; ++term) {
+          const uint64_t bd = sw128_desc(bst + term * C::kTermBytes);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)   // K = 32 bytes per MMA inside the 128-byte swizzle row
+            mma_f8_tmem_a(tbase, acol + 8 * kk, bd + 2 * kk, C::kIdesc, (kt | term | kk) != 0 ? 1u : 0u);
         }
+        mma_commit(a_empty(sa));
+        mma_commit(b_empty(sb));
       }
-#pragma unroll
-      for (int o = 16; o; o >>= 1) {
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-        cp += __shfl_xor_sync(0xffffffffu, cp, o);
-      }
-      if (lane == 0) {
-        xmax[tok] = mx;
-        cpart[tok] = cp;
-      }
+      if (ok) mma_commit(d_full);
+      else *abort_flag = 1;
+      mma_commit(drain);   // everything issued must retire before TMEM is released
+      mbar_wait(drain, 0, a.err, kErrTimeoutMma);
     }
-    named_barrier_sync(kFoldBarrier, kConsumerThreads);
-    if (tid < a.M) {
-      // 2^P scales the largest possible |x'| (<= max|x| * colnorm) below 2^15.
-      const float bound = xmax[tid] * a.colnorm;
-      int e = 0;
-      if (bound > 0.f) frexpf(bound, &e);   // bound < 2^e
-      pexp[tid] = bound > 0.f ? max(-100, min(100, 15 - e)) : 0;
-    }
-    named_barrier_sync(kFoldBarrier, kConsumerThreads);
-
-    auto fold = [&](int c) {
-      uint2* xf = reinterpret_cast<uint2*>(smem + C::kOffXfrag + (c & 1) * C::kXfragBytes);
-      const int ck0 = (kt0 + c * C::CH) * kTileCols;
-      constexpr int units = C::CH * 32;   // 4-column units per token per chunk
-      for (int u = tid; u < a.M * units; u += kConsumerThreads) {
-        const int tok = u / units;
-        const int j = u - tok * units;
-        const int k = ck0 + 4 * j;
-        uint32_t lo = 0, hi = 0;
-        if (k < kend) {
-          float v[4], o[4];
-          load4(a.x + static_cast<size_t>(tok) * a.K, k, a.K, v);
-          fold4(a, v, o);
-          const int i = (k & 63) >> 4;
-          const float sc0 = exp2i(pexp[tok] - 2 * pos_scale_class(2 * i));
-          const float sc1 = exp2i(pexp[tok] - 2 * pos_scale_class(2 * i + 1));
-          lo = pack_half2(o[0] * sc0, o[1] * sc0);
-          hi = pack_half2(o[2] * sc1, o[3] * sc1);
-        }
-        xf[((tok >> 3) * C::CH * 8 + (j >> 2)) * 32 + (tok & 7) * 4 + (j & 3)] = make_uint2(lo, hi);
-      }
-    };
-
-    const int n_ch = (n_kt + C::CH - 1) / C::CH;
-    fold(0);
-    float acc[NT][4];
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) acc[nt][e] = 0.f;
-
-    bool ok = !*abort_flag;
-    for (int kk = 0; kk < n_kt; ++kk) {
-      const int st = kk / kKB;
-      const int kb = kk - st * kKB;
-      const int slot = st % kStages;
-      if (kk % C::CH == 0) {
-        named_barrier_sync(kFoldBarrier, kConsumerThreads);
-        const int c = kk / C::CH;
-        if (c + 1 < n_ch) fold(c + 1);
-      }
-      if (ok && kb == 0) {
-        ok = !*abort_flag && mbar_wait(full_bar(slot), (st / kStages) & 1, a.err, kErrTimeoutFull);
-        if (!ok) *abort_flag = 1;
-      }
+  } else if (warp < kFoldWarp0) {
+    // ---------------- converters: shared ring -> TMEM A slots ----------------
+    const int q = warp & 3;                    // TMEM lane quarter
+    const int r = 32 * q + lane;               // row of this thread
+    bool ok = !*abort_flag && mbar_wait(tmem_ready, 0, a.err, kErrTimeoutFull);
+    tc_fence_after();
+    const uint32_t tbase = *tmem_ptr;
+    const uint32_t trow = tbase + (static_cast<uint32_t>(32 * q) << 16);
+    for (int kt = 0; kt < n_kt; ++kt) {
+      const int s = kt % C::kCodeStages, sa = kt % kASlots;
+      if (ok) ok = !*abort_flag && mbar_wait(code_full(s), (kt / C::kCodeStages) & 1, a.err, kErrTimeoutFull);
+      uint4 w0 = make_uint4(0, 0, 0, 0), w1 = w0;
       if (ok) {
-        const uint4 wv = *reinterpret_cast<const uint4*>(
-            smem + C::kOffRing + slot * C::kStageBytes + (warp * kKB + kb) * kTileBytes + lane * 16);
-        const uint2* xf = reinterpret_cast<const uint2*>(
-            smem + C::kOffXfrag + ((kk / C::CH) & 1) * C::kXfragBytes);
-        const int kl = kk % C::CH;
+        const uint8_t* tile = smem + C::kOffCode + s * kTileBytes;
+        w0 = *reinterpret_cast<const uint4*>(tile + tile_row_offset(r, 0));
+        w1 = *reinterpret_cast<const uint4*>(tile + tile_row_offset(r, 1));
+      }
+      __syncwarp();
+      if (lane == 0 && ok) mbar_arrive(code_empty(s));
+      uint32_t v[32];
+      const uint32_t ws[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
 #pragma unroll
-        for (int grp = 0; grp < 2; ++grp) {
-          const uint32_t wg = grp ? wv.z : wv.x;    // row g
-          const uint32_t wg8 = grp ? wv.w : wv.y;   // row g + 8
-          const uint32_t wgs = wg >> 10, wg8s = wg8 >> 10;
+      for (int j = 0; j < 8; ++j)
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const uint32_t a0 = extract_pos(wg, wgs, 2 * i);
-            const uint32_t a1 = extract_pos(wg8, wg8s, 2 * i);
-            const uint32_t a2 = extract_pos(wg, wgs, 2 * i + 1);
-            const uint32_t a3 = extract_pos(wg8, wg8s, 2 * i + 1);
+        for (int e = 0; e < 4; ++e) v[4 * j + e] = extract4(ws[j], e);   // TMEM column 4j + e
+      if (ok && kt >= kASlots) ok = !*abort_flag && mbar_wait(a_empty(sa), ((kt / kASlots) - 1) & 1, a.err, kErrTimeoutMma);
+      if (ok) {
+        tc_fence_after();
+        tmem_st32(trow + kAColBase + 32 * sa, v);
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+        tc_fence_before();
+      }
+      __syncwarp();
+      if (lane == 0 && ok) mbar_arrive(a_full(sa));
+      if (!ok) *abort_flag = 1;
+    }
+
+    // ---------------- epilogue: accumulator rows -> cluster reduction ----------------
+    if (ok) ok = !*abort_flag && mbar_wait(d_full, 0, a.err, kErrTimeoutMma);
+    if (ok) ok = mbar_wait(fold_done, 0, a.err, kErrTimeoutFull);
+    if (!ok) *abort_flag = 1;
+    const int rows_per = (kTileRows + KS - 1) / KS;
+    const int owner = r / rows_per;
+    const uint32_t slot_off =
+        (static_cast<uint32_t>(blockIdx.x) * rows_per + (r - owner * rows_per)) * NTOK * 4u;
+    const uint32_t red_addr = sbase + C::kOffRed;
+    tc_fence_after();
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-              const uint2 b = xf[(nt * C::CH * 8 + kl * 8 + grp * 4 + i) * 32 + lane];
-              mma_f16_16816(acc[nt], a0, a1, a2, a3, b.x, b.y);
-            }
+    for (int c0 = 0; c0 < NTOK; c0 += 16) {
+      uint32_t dv[16];
+      tmem_ld16(trow + c0, dv);
+      asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int tok = c0 + j;
+        if (ok && tok < a.M) {
+          const float val = fmaf(__uint_as_float(dv[j]), exp2i(9 - pexp[tok]), cpart[tok]);
+          const uint32_t off = slot_off + tok * 4u;
+          if (KS > 1) st_shared_cluster_f32(map_shared_rank(red_addr + off, owner), val);
+          else red[off / 4] = val;
+        }
+      }
+    }
+    tc_fence_before();
+  } else {
+    // ---------------- fold: x -> scaled three-term e4m3 B tiles ----------------
+    const int fw = warp - kFoldWarp0;
+    // Fold warp fw < kBStages owns B stage fw (k-tiles kt = fw mod kBStages),
+    // so each stage has one writer and every wait on it is one phase behind.
+    // The owner zeroes the rows of tokens >= M once (those rows stay zero).
+    if (fw < C::kBStages)
+      for (int tok = a.M; tok < NTOK; ++tok)
+        for (int term = 0; term < 3; ++term)
+          reinterpret_cast<uint32_t*>(smem + C::kOffB + fw * C::kBStageBytes + term * C::kTermBytes + tok * 128)[lane] = 0u;
+    pdl_wait();   // x may be the previous kernel's output
+    const int kbeg = kt0 * kTileCols;
+    const int kend = min(a.K, (kt0 + n_kt) * kTileCols);
+    const int kspan = n_kt * kTileCols;                       // staged row length (bf16)
+    const bool vec8 = (a.K & 7) == 0;
+    const bool staged = a.M * kspan * 2 <= C::kXBytes;
+    uint16_t* xs = reinterpret_cast<uint16_t*>(smem + C::kOffX);
+    // Pass 1: per-token max |x| (scale) and sum_k x[k] B[k mod d] over the
+    // slice; warp fw owns tokens fw, fw+4, ...; 8 columns per lane per load,
+    // 8 loads in flight. The slice is kept in shared memory when it fits.
+    for (int tok = fw; tok < a.M; tok += 4) {
+      const uint16_t* row = a.x + static_cast<size_t>(tok) * a.K;
+      float mx = 0.f, cs = 0.f;
+      for (int k0 = kbeg + 8 * lane; k0 < kbeg + kspan; k0 += 8 * 32 * 8) {
+        uint4 u[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int k = k0 + 256 * j;
+          if (vec8 && k + 7 < kend) {
+            u[j] = __ldg(reinterpret_cast<const uint4*>(row + k));
+          } else {
+            uint32_t e[8];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) e[t] = (k + t < kend) ? static_cast<uint32_t>(row[k + t]) : 0u;
+            u[j] = make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int k = k0 + 256 * j;
+          if (k >= kbeg + kspan) break;
+          if (staged) *reinterpret_cast<uint4*>(xs + tok * kspan + (k - kbeg)) = u[j];
+          const uint32_t w4[4] = {u[j].x, u[j].y, u[j].z, u[j].w};
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const float v0 = bf16_lo(w4[t]), v1 = bf16_hi(w4[t]);
+            mx = fmaxf(mx, fmaxf(fabsf(v0), fabsf(v1)));
+            cs = fmaf(v0, a.B[(2 * t) & (a.d - 1)], cs);
+            cs = fmaf(v1, a.B[(2 * t + 1) & (a.d - 1)], cs);
           }
         }
       }
-      if (kb == kKB - 1 || kk == n_kt - 1) {
-        __syncwarp();
-        if (lane == 0 && ok) mbar_arrive(empty_bar(slot));
+#pragma unroll
+      for (int off = 16; off; off >>= 1) {
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+        cs += __shfl_xor_sync(0xffffffffu, cs, off);
+      }
+      if (lane == 0) {
+        // 2^P puts the largest possible |x'| (<= max|x| * colnorm) below 2^8.
+        const float bound = mx * a.colnorm;
+        int e2 = 0;
+        if (bound > 0.f) frexpf(bound, &e2);
+        pexp[tok] = bound > 0.f ? max(-100, min(100, 8 - e2)) : 0;
+        cpart[tok] = cs;
       }
     }
+    // All fold warps need every token's scale (and staged x) from here on.
+    named_barrier_sync(1, 4 * 32);
+    if (lane == 0) mbar_arrive(fold_done);
 
-    // Partial outputs of this K slice: acc * 2^(24 - P) + partial c.
-    const int g = lane >> 2, t = lane & 3;
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int row = warp * 16 + g + ((e & 2) ? 8 : 0);
-        const int tok = nt * 8 + 2 * t + (e & 1);
-        if (tok < a.M) red[row * C::MP + tok] = fmaf(acc[nt][e], exp2i(24 - pexp[tok]), cpart[tok]);
+    // Pass 2: warp fw folds k-tiles fw, fw + kBStages, ... (its own stage) for
+    // all tokens; lane covers columns 4 lane .. 4 lane + 3 of the k-tile.
+    bool ok = !*abort_flag;
+    const uint32_t cidx = (4 * lane) & 15;
+    const uint32_t chunk = (4 * lane) >> 4;
+    for (int kt = fw; fw < C::kBStages && kt < n_kt; kt += C::kBStages) {
+      const int sb = fw;
+      const int use = kt / C::kBStages;      // how many times stage sb was filled before
+      if (ok && use > 0)
+        ok = !*abort_flag && mbar_wait(b_empty(sb), (use - 1) & 1, a.err, kErrTimeoutMma);
+      if (ok) {
+        uint8_t* bst = smem + C::kOffB + sb * C::kBStageBytes;
+        const int k = (kt0 + kt) * kTileCols + 4 * lane;
+        for (int tok = 0; tok < a.M; ++tok) {
+          uint2 xv;
+          if (staged) {
+            xv = *reinterpret_cast<const uint2*>(xs + tok * kspan + kt * kTileCols + 4 * lane);
+          } else {
+            xv = load_x4(a.x + static_cast<size_t>(tok) * a.K, k, kend, (a.K & 3) == 0);
+          }
+          const float v[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
+          float o[4];
+          fold4(a, v, o);
+          const float sc = exp2i(pexp[tok]);
+          uint16_t h0, m0, l0, h1, m1, l1;
+          split3(pack_half2(o[0] * sc, o[1] * sc), h0, m0, l0);
+          split3(pack_half2(o[2] * sc, o[3] * sc), h1, m1, l1);
+          const uint32_t off = tok * 128 + ((chunk ^ (tok & 7)) << 4) + cidx;
+          *reinterpret_cast<uint32_t*>(bst + off) = h0 | (static_cast<uint32_t>(h1) << 16);
+          *reinterpret_cast<uint32_t*>(bst + C::kTermBytes + off) = m0 | (static_cast<uint32_t>(m1) << 16);
+          *reinterpret_cast<uint32_t*>(bst + 2 * C::kTermBytes + off) = l0 | (static_cast<uint32_t>(l1) << 16);
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       }
+      __syncwarp();
+      if (lane == 0 && ok) mbar_arrive(b_full(sb));
+      if (!ok) *abort_flag = 1;
+    }
   }
 
   // ---------------- reduction over the K slices of the cluster ----------------
   __syncwarp();
   if (KS > 1) cluster_sync(); else __syncthreads();
-  const int rank = static_cast<int>(blockIdx.x);
-  const int rows_per = (kDecRows + KS - 1) / KS;
-  const int r0 = rank * rows_per;
-  const int nrows = max(0, min(kDecRows, r0 + rows_per) - r0);
-  const uint32_t red_addr = smem_u32(red);
-  for (int idx = tid; idx < nrows * a.M; idx += kDecThreads) {
-    const int tok = idx / nrows;
-    const int row = r0 + (idx - tok * nrows);
-    const int n = blockIdx.y * kDecRows + row;
-    float s = 0.f;
-    if (KS > 1) {
-      for (int q = 0; q < KS; ++q)
-        s += ld_shared_cluster_f32(map_shared_rank(red_addr + (row * C::MP + tok) * 4u, q));
-    } else {
-      s = red[row * C::MP + tok];
+  {
+    const int rows_per = (kTileRows + KS - 1) / KS;
+    const int r0 = static_cast<int>(blockIdx.x) * rows_per;
+    const int nrows = max(0, min(kTileRows, r0 + rows_per) - r0);
+    for (int idx = tid; idx < nrows * a.M; idx += kThreads) {
+      const int tok = idx / nrows;
+      const int rl = idx - tok * nrows;
+      const int n = rb * kTileRows + r0 + rl;
+      float s = 0.f;
+      for (int qq = 0; qq < KS; ++qq) s += red[(qq * rows_per + rl) * NTOK + tok];
+      if (n < a.N) a.y[static_cast<size_t>(tok) * a.N + n] = f32_to_bf16_rn(s);
     }
-    if (n < a.N) a.y[static_cast<size_t>(tok) * a.N + n] = f32_to_bf16_rn(s);
   }
-  // Copies still in flight after an abort must land before the CTA exits.
-  if (warp == kDecWarps && lane == 0 && *abort_flag) {
-    for (int st = max(0, issued - kStages); st < issued; ++st)
-      mbar_wait(full_bar(st % kStages), (st / kStages) & 1, a.err, kErrTimeoutFull);
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(*tmem_ptr), "r"(kTmemCols)
+                 : "memory");
   }
-  __syncwarp();
-  if (KS > 1) cluster_sync();
 }
 
-template <int NT>
-unisvq_status launch_nt(const unisvq_layer* L, const DecodePlan& p, const void* x, void* y, int M,
-                        cudaStream_t s) {
-  using C = DecCfg<NT>;
+template <int NTOK>
+int resident_ctas_per_sm() {
+  static int n = 0;
+  if (!n) {
+    cudaFuncSetAttribute(decode_kernel<NTOK>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<NTOK>::kSmem);
+    cudaFuncSetAttribute(decode_kernel<NTOK>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                         cudaSharedmemCarveoutMaxShared);
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<NTOK>, kThreads, Cfg<NTOK>::kSmem) !=
+            cudaSuccess ||
+        n < 1)
+      n = 1;
+    // Each resident CTA holds kTmemCols of the 512 TMEM columns.
+    n = min(n, 512 / kTmemCols);
+  }
+  return n;
+}
+
+template <int NTOK>
+unisvq_status launch_ntok(const unisvq_layer* L, const DecodePlan& p, const void* x, void* y, int M,
+                          cudaStream_t s) {
+  using C = Cfg<NTOK>;
   static bool attr_set[64] = {};
   const int dev = L->device;
   if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
   if (!attr_set[dev]) {
-    if (cudaFuncSetAttribute(decode_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             C::kSmem) != cudaSuccess)
+    if (cudaFuncSetAttribute(decode_kernel<NTOK>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(decode_kernel<NTOK>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared) != cudaSuccess)
       return UNISVQ_ERR_CUDA;
     attr_set[dev] = true;
   }
@@ -356,7 +527,7 @@ unisvq_status launch_nt(const unisvq_layer* L, const DecodePlan& p, const void* 
 
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.ks, p.nb, 1);
-  cfg.blockDim = dim3(kDecThreads, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = C::kSmem;
   cfg.stream = s;
   cudaLaunchAttribute attrs[2];
@@ -368,36 +539,42 @@ unisvq_status launch_nt(const unisvq_layer* L, const DecodePlan& p, const void* 
   attrs[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attrs;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, decode_kernel<NT>, a) == cudaSuccess ? UNISVQ_OK
-                                                                       : UNISVQ_ERR_CUDA;
+  return cudaLaunchKernelEx(&cfg, decode_kernel<NTOK>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
 }  // namespace
 
-DecodePlan plan_decode(const unisvq_layer* L, int M) {
+DecodePlan plan_skinny(const unisvq_layer* L, int M) {
   DecodePlan p{};
-  p.nt = M <= 8 ? 1 : (M <= 16 ? 2 : 4);
-  p.nb = L->Np / kDecRows;
-  const int target = 2 * L->num_sms;
+  p.nt = M <= 16 ? 16 : (M <= 32 ? 32 : 64);
+  p.nb = L->Np / kTileRows;
+  const int occ = p.nt == 16 ? resident_ctas_per_sm<16>() : (p.nt == 32 ? resident_ctas_per_sm<32>()
+                                                                         : resident_ctas_per_sm<64>());
+  // Largest K split (cluster size <= 8, >= 1 k-tile per CTA) whose grid fits
+  // in one wave of resident CTAs.
+  const int slots = occ * L->num_sms;
   int ks = 1;
-  while (ks < 8 && p.nb * ks < target && ks * 2 <= L->KT) ks *= 2;
+  for (int c = 8; c >= 1; --c)
+    if (c <= L->KT && p.nb * c <= slots) {
+      ks = c;
+      break;
+    }
   p.kt_per_cta = (L->KT + ks - 1) / ks;
   p.ks = (L->KT + p.kt_per_cta - 1) / p.kt_per_cta;
-  p.smem = p.nt == 1 ? DecCfg<1>::kSmem : (p.nt == 2 ? DecCfg<2>::kSmem : DecCfg<4>::kSmem);
+  p.smem = p.nt == 16 ? Cfg<16>::kSmem : (p.nt == 32 ? Cfg<32>::kSmem : Cfg<64>::kSmem);
   return p;
 }
 
-unisvq_status launch_decode(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
-  // Token groups of at most 32 (one launch each) keep every M on this path.
-  for (int m0 = 0; m0 < M; m0 += kMaxTok) {
-    const int mc = M - m0 < kMaxTok ? M - m0 : kMaxTok;
-    const DecodePlan p = plan_decode(L, mc);
+unisvq_status launch_skinny(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
+  for (int m0 = 0; m0 < M; m0 += kMaxTokPerLaunch) {
+    const int mc = M - m0 < kMaxTokPerLaunch ? M - m0 : kMaxTokPerLaunch;
+    const DecodePlan p = plan_skinny(L, mc);
     const void* xs = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * L->K;
     void* ys = static_cast<uint16_t*>(y) + static_cast<size_t>(m0) * L->N;
     unisvq_status st;
-    if (p.nt == 1) st = launch_nt<1>(L, p, xs, ys, mc, s);
-    else if (p.nt == 2) st = launch_nt<2>(L, p, xs, ys, mc, s);
-    else st = launch_nt<4>(L, p, xs, ys, mc, s);
+    if (p.nt == 16) st = launch_ntok<16>(L, p, xs, ys, mc, s);
+    else if (p.nt == 32) st = launch_ntok<32>(L, p, xs, ys, mc, s);
+    else st = launch_ntok<64>(L, p, xs, ys, mc, s);
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;

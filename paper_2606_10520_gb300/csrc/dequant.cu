@@ -1,8 +1,8 @@
 // Test hook: W_hat [N][K] in fp32 from the packed device layout.
 //
-// Each warp unpacks one 16 x 128 tile with the same position-extraction helper
-// the layer kernels use (layout.h), rebuilds the vector index of every
-// d-vector (coordinate c in bits [2c+1:2c]) and reads the fp32 codeword
+// Each thread unpacks one 16-byte row chunk (64 codes of one row) with the
+// same extraction helper the layer kernels use (layout.h), rebuilds the index
+// z0 | z1 << 2 | ... of every d-vector and reads the fp32 codeword
 // RN_fp32(A z + B) of Eq. (def:unisvq) from the handle's codebook.
 #include "common.cuh"
 #include "internal.h"
@@ -12,35 +12,34 @@ namespace {
 
 __global__ void __launch_bounds__(256) dequant_kernel(const uint8_t* __restrict__ codes,
                                                       const float* __restrict__ lut, float* W,
-                                                      int N, int K, int KT, int d, int ntiles) {
-  const int tile = blockIdx.x * 8 + (threadIdx.x >> 5);
-  if (tile >= ntiles) return;
-  const int lane = threadIdx.x & 31;
-  const int rt = tile / KT, kt = tile - (tile / KT) * KT;
-  const int g = lane >> 2, t = lane & 3;
-  const uint4 wv = *reinterpret_cast<const uint4*>(codes + static_cast<size_t>(tile) * kTileBytes + lane * 16);
-  const uint32_t words[4] = {wv.x, wv.y, wv.z, wv.w};
+                                                      int N, int K, int KT, int d, int nchunks) {
+  const int id = blockIdx.x * 256 + threadIdx.x;
+  if (id >= nchunks) return;
+  const int tile = id >> 8;               // 256 row chunks per tile (2 halves x 128 rows)
+  const int h = (id >> 7) & 1, r = id & 127;
+  const int rb = tile / KT, kt = tile - rb * KT;
+  const int row = rb * kTileRows + r;
+  if (row >= N) return;
+  const uint4 q = *reinterpret_cast<const uint4*>(codes + static_cast<size_t>(tile) * kTileBytes +
+                                                  tile_row_offset(r, h));
+  const uint32_t words[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int grp = q >> 1, rh = q & 1;
-    const int row = rt * kTileRows + g + 8 * rh;
-    const uint32_t w = words[q], ws = w >> 10;
-    // 4-column groups: i selects the k16 block, positions 2i (cols +0,+1) and 2i+1 (cols +2,+3).
+  for (int wi = 0; wi < 4; ++wi) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const uint32_t f0 = extract_pos(w, ws, 2 * i), f1 = extract_pos(w, ws, 2 * i + 1);
-      const uint32_t z[4] = {frag_code_lo(f0, 2 * i), frag_code_hi(f0, 2 * i),
-                             frag_code_lo(f1, 2 * i + 1), frag_code_hi(f1, 2 * i + 1)};
-      const int k0 = kt * kTileCols + 64 * grp + 16 * i + 4 * t;
-      if (row >= N) continue;
+    for (int s = 0; s < 4; ++s) {
+      const uint32_t e = extract4(words[wi], s);   // columns 4s .. 4s+3 of the word
+      const int k0 = kt * kTileCols + 64 * h + 16 * wi + 4 * s;
+      uint32_t z[4];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int k = k0 + e;
+      for (int b = 0; b < 4; ++b) z[b] = (e >> (8 * b)) & 3u;
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        const int k = k0 + b;
         if (k >= K) continue;
-        const int v0 = e & ~(d - 1);   // first coordinate of this column's vector
+        const int v0 = b & ~(d - 1);            // first coordinate of this column's vector
         uint32_t idx = 0;
         for (int c = 0; c < d; ++c) idx |= z[v0 + c] << (2 * c);
-        W[static_cast<size_t>(row) * K + k] = lut[idx * d + (e & (d - 1))];
+        W[static_cast<size_t>(row) * K + k] = lut[idx * d + (b & (d - 1))];
       }
     }
   }
@@ -49,9 +48,9 @@ __global__ void __launch_bounds__(256) dequant_kernel(const uint8_t* __restrict_
 }  // namespace
 
 unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s) {
-  const int ntiles = (L->Np / kTileRows) * L->KT;
-  dequant_kernel<<<(ntiles + 7) / 8, 256, 0, s>>>(L->codes, L->lut32, W, L->N, L->K, L->KT, L->d,
-                                                  ntiles);
+  const int nchunks = (L->Np / kTileRows) * L->KT * 256;
+  dequant_kernel<<<(nchunks + 255) / 256, 256, 0, s>>>(L->codes, L->lut32, W, L->N, L->K, L->KT, L->d,
+                                                       nchunks);
   return cudaGetLastError() == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 

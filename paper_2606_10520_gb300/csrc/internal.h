@@ -5,7 +5,7 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
-#include "../../include/unisvq.h"
+#include "unisvq.h"
 #include "layout.h"
 
 struct unisvq_layer {
@@ -28,7 +28,7 @@ struct unisvq_layer {
 namespace unisvq {
 
 struct DecodePlan {
-  int nt;          // n8 token tiles (1, 2, 4)
+  int nt;          // token tile (gemv: n8 tiles 1..2; skinny: MMA N 16/32/64)
   int ks;          // CTAs along K (cluster size)
   int kt_per_cta;  // k-tiles per CTA
   int nb;          // row blocks of 128 rows
@@ -44,8 +44,12 @@ struct PrefillPlan {
 
 int* device_error_word();   // device address of the library error word (current device)
 
-DecodePlan plan_decode(const unisvq_layer* L, int M);
-unisvq_status launch_decode(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
+// Register-operand tensor-core GEMV (gemv.cu), M <= 16 per launch.
+DecodePlan plan_gemv(const unisvq_layer* L, int M);
+unisvq_status launch_gemv(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
+// tcgen05 skinny GEMM with the codes as 8-bit TMEM operand (decode.cu), M <= 64 per launch.
+DecodePlan plan_skinny(const unisvq_layer* L, int M);
+unisvq_status launch_skinny(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
 
 bool prefill_supported(const unisvq_layer* L, int M);
 PrefillPlan plan_prefill(const unisvq_layer* L, int M);

@@ -11,30 +11,29 @@ namespace unisvq {
 
 void pack_codes_host(const uint8_t* codes, int N, int K, uint8_t* packed) {
   const int Np = round_up(N, kRowPad), Kp = round_up(K, kColPad);
-  const int RT = Np / kTileRows, KT = Kp / kTileCols;
+  const int RB = Np / kTileRows, KT = Kp / kTileCols;
 #pragma omp parallel for schedule(static)
-  for (int rt = 0; rt < RT; ++rt) {
+  for (int rb = 0; rb < RB; ++rb) {
     for (int kt = 0; kt < KT; ++kt) {
-      uint8_t* tile = packed + (static_cast<size_t>(rt) * KT + kt) * kTileBytes;
-      for (int lane = 0; lane < 32; ++lane) {
-        const int g = lane >> 2, t = lane & 3;
-        for (int q = 0; q < 4; ++q) {
-          const int grp = q >> 1, rh = q & 1;
-          const int row = rt * kTileRows + g + 8 * rh;
+      uint8_t* tile = packed + (static_cast<size_t>(rb) * KT + kt) * kTileBytes;
+      for (int h = 0; h < 2; ++h) {
+        for (int r = 0; r < kTileRows; ++r) {
+          const int row = rb * kTileRows + r;
           const uint8_t* cr = row < N ? codes + static_cast<size_t>(row) * K : nullptr;
-          uint32_t w = 0;
-          for (int p = 0; p < 8; ++p) {
-            const int k = kt * kTileCols + 64 * grp + 16 * (p >> 1) + 4 * t + 2 * (p & 1);
-            const uint32_t lo = (cr && k < K) ? (cr[k] & 3u) : 0u;
-            const uint32_t hi = (cr && k + 1 < K) ? (cr[k + 1] & 3u) : 0u;
-            w |= lo << (2 * p);
-            w |= hi << (16 + 2 * p);
+          uint8_t* dst = tile + tile_row_offset(r, h);
+          for (int wi = 0; wi < 4; ++wi) {
+            uint32_t w = 0;
+            for (int s = 0; s < 4; ++s)
+              for (int b = 0; b < 4; ++b) {
+                const int k = kt * kTileCols + 64 * h + 16 * wi + 4 * s + b;
+                const uint32_t z = (cr && k < K) ? (cr[k] & 3u) : 0u;
+                w |= z << (8 * b + 2 * s);
+              }
+            dst[4 * wi + 0] = static_cast<uint8_t>(w);
+            dst[4 * wi + 1] = static_cast<uint8_t>(w >> 8);
+            dst[4 * wi + 2] = static_cast<uint8_t>(w >> 16);
+            dst[4 * wi + 3] = static_cast<uint8_t>(w >> 24);
           }
-          uint8_t* dst = tile + lane * 16 + q * 4;
-          dst[0] = static_cast<uint8_t>(w);
-          dst[1] = static_cast<uint8_t>(w >> 8);
-          dst[2] = static_cast<uint8_t>(w >> 16);
-          dst[3] = static_cast<uint8_t>(w >> 24);
         }
       }
     }

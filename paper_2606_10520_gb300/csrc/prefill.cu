@@ -10,9 +10,9 @@
 // Roles of the 14 warps of a CTA (persistent over tiles):
 //   warp 0        TMA producer: x tile [BN x 64] per k-block, and TMEM owner
 //   warp 1        MMA issuer (one thread): 4 x tcgen05.mma (K = 16) per k-block
-//   warps 2..9    converters: one 16-row code tile each; every d-vector index
-//                 selects its exact bf16 codeword RN(A z + B) from a pack-time
-//                 table, written straight into the swizzled A tile
+//   warps 2..9    converters: one row per lane, half of each 128-byte swizzled
+//                 row per warp; every d-vector index selects its exact bf16
+//                 codeword RN(A z + B) from a pack-time table
 //   warps 10..13  epilogue: tcgen05.ld of the accumulator, bf16, global store
 // The accumulator is double-buffered in TMEM so the epilogue of one tile runs
 // under the main loop of the next.
@@ -136,8 +136,8 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-__device__ __forceinline__ void sts64(uint32_t addr, uint32_t a, uint32_t b) {
-  asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
+__device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
 __device__ __forceinline__ uint32_t lds32(uint32_t addr) {
   uint32_t v;
@@ -261,48 +261,56 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     }
   } else if (warp < kEpiWarp0) {
     // ---------------- converters: codes -> bf16 codeword tile ----------------
-    const int c = warp - kConvWarp0;            // 16-row code tile of this warp
-    const int g = lane >> 2, t = lane & 3;
+    // Warp c covers rows 32 (c % 4) .. +31 (one row per lane) and the 16-byte
+    // chunks 4 (c / 4) .. +3 of each 64-column stage.
+    const int c = warp - kConvWarp0;
+    const int r = 32 * (c & 3) + lane;          // row within the 128-row tile
+    const int ch = c >> 2;
     const uint32_t lut_s = sbase + C::kOffLut;
+    const int sw = r & 7;
     int it = 0;
     for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
       const int n_blk = tile / a.mtiles;
-      const uint8_t* tbase =
-          a.codes + (static_cast<size_t>(n_blk * 8 + c) * a.KT) * kTileBytes + lane * 16;
-      uint4 cw = make_uint4(0, 0, 0, 0);
+      const uint8_t* rbase = a.codes + static_cast<size_t>(n_blk) * a.KT * kTileBytes + r * 16 + 8 * ch;
+      // Code words of stage kb live at tile kb/2, half kb%2; prefetched 3 stages ahead.
+      auto load = [&](int kb) -> uint2 {
+        return kb < a.nkb ? __ldg(reinterpret_cast<const uint2*>(rbase + (kb >> 1) * kTileBytes +
+                                                                 (kb & 1) * kHalfBytes))
+                          : make_uint2(0, 0);
+      };
+      uint2 q0 = load(0), q1 = load(1), q2 = load(2);
       bool ok = !*abort_flag;
       for (int kb = 0; kb < a.nkb; ++kb, ++it) {
         const int s = it % STAGES;
-        if ((kb & 1) == 0) cw = __ldg(reinterpret_cast<const uint4*>(tbase + (kb >> 1) * kTileBytes));
+        const uint2 cw = q0;
+        q0 = q1;
+        q1 = q2;
+        q2 = load(kb + 3);
         if (ok && it >= STAGES) {
           ok = !*abort_flag && mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty);
           if (!ok) *abort_flag = 1;
         }
         if (ok) {
-          const uint32_t a_s = sbase + C::kOffA + s * kATileBytes;
+          const uint32_t row_addr = sbase + C::kOffA + s * kATileBytes + r * 128;
 #pragma unroll
-          for (int rh = 0; rh < 2; ++rh) {
-            const uint32_t w = (kb & 1) ? (rh ? cw.w : cw.z) : (rh ? cw.y : cw.x);
-            const int r = c * 16 + g + 8 * rh;          // row within the 128-row tile
-            const uint32_t row_addr = a_s + r * 128 + ((t & 1) << 3);
-            const int sw = r & 7;
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              uint32_t e0, e1;
-              if (a.d == 4) {
-                const uint32_t v = (w >> (4 * i)) & 0x000F000Fu;
-                const uint32_t idx = (v & 0xFu) | ((v >> 12) & 0xF0u);
-                const uint2 q = lds64(lut_s + idx * 8);
-                e0 = q.x;
-                e1 = q.y;
-              } else {
-                const uint32_t v0 = (w >> (4 * i)) & 0x00030003u;
-                const uint32_t v1 = (w >> (4 * i + 2)) & 0x00030003u;
-                e0 = lds32(lut_s + (((v0 & 3u) | ((v0 >> 14) & 0xCu)) << 2));
-                e1 = lds32(lut_s + (((v1 & 3u) | ((v1 >> 14) & 0xCu)) << 2));
-              }
-              sts64(row_addr + ((((2 * i) + (t >> 1)) ^ sw) << 4), e0, e1);
+          for (int j = 0; j < 4; ++j) {
+            const int cc = 4 * ch + j;                      // chunk: columns 8cc .. 8cc+7
+            const uint32_t w = (j < 2) ? cw.x : cw.y;
+            const uint32_t e0 = extract4(w, 2 * (j & 1));   // columns 8cc .. 8cc+3
+            const uint32_t e1 = extract4(w, 2 * (j & 1) + 1);
+            uint32_t o0, o1, o2, o3;
+            if (a.d == 4) {
+              const uint32_t i0 = (e0 & 3u) | ((e0 >> 6) & 0xCu) | ((e0 >> 12) & 0x30u) | ((e0 >> 18) & 0xC0u);
+              const uint32_t i1 = (e1 & 3u) | ((e1 >> 6) & 0xCu) | ((e1 >> 12) & 0x30u) | ((e1 >> 18) & 0xC0u);
+              const uint2 v0 = lds64(lut_s + i0 * 8), v1 = lds64(lut_s + i1 * 8);
+              o0 = v0.x; o1 = v0.y; o2 = v1.x; o3 = v1.y;
+            } else {
+              o0 = lds32(lut_s + (((e0 & 3u) | ((e0 >> 6) & 0xCu)) << 2));
+              o1 = lds32(lut_s + ((((e0 >> 16) & 3u) | ((e0 >> 22) & 0xCu)) << 2));
+              o2 = lds32(lut_s + (((e1 & 3u) | ((e1 >> 6) & 0xCu)) << 2));
+              o3 = lds32(lut_s + ((((e1 >> 16) & 3u) | ((e1 >> 22) & 0xCu)) << 2));
             }
+            sts128(row_addr + ((cc ^ sw) << 4), o0, o1, o2, o3);
           }
           fence_proxy_async_smem();
         }

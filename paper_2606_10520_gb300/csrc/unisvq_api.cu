@@ -148,11 +148,9 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
       cb[static_cast<size_t>(v) * d + r] = w;
       lut32[static_cast<size_t>(v) * d + r] = static_cast<float>(w);
     }
-  // Prefill tile table, indexed the way the converter warps read a code word:
-  //   d <= 2: 16 bf16 pairs, index lo | hi << 2 for the two columns (k, k+1)
-  //           sharing one word position;
-  //   d == 4: 256 bf16 quads, index z0 | z2 << 2 | z1 << 4 | z3 << 6 (the order
-  //           in which two adjacent positions of a word hold columns 4m..4m+3).
+  // Prefill tile table, indexed the way the converter warps read code bytes:
+  //   d <= 2: 16 bf16 pairs, index lo | hi << 2 for two adjacent columns (k, k+1);
+  //   d == 4: 256 bf16 quads, index z0 | z1 << 2 | z2 << 4 | z3 << 6.
   auto bf = [](double w) { return static_cast<uint32_t>(f64_to_bf16_rne(w)); };
   std::vector<uint32_t> tlut;
   if (d <= 2) {
@@ -165,11 +163,9 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
     }
   } else {
     tlut.resize(512);
-    for (int idx = 0; idx < 256; ++idx) {
-      const int z0 = idx & 3, z2 = (idx >> 2) & 3, z1 = (idx >> 4) & 3, z3 = (idx >> 6) & 3;
-      const size_t v = static_cast<size_t>(z0 | (z1 << 2) | (z2 << 4) | (z3 << 6));
-      tlut[2 * idx] = bf(cb[v * 4 + 0]) | (bf(cb[v * 4 + 1]) << 16);
-      tlut[2 * idx + 1] = bf(cb[v * 4 + 2]) | (bf(cb[v * 4 + 3]) << 16);
+    for (int v = 0; v < 256; ++v) {
+      tlut[2 * v] = bf(cb[static_cast<size_t>(v) * 4 + 0]) | (bf(cb[static_cast<size_t>(v) * 4 + 1]) << 16);
+      tlut[2 * v + 1] = bf(cb[static_cast<size_t>(v) * 4 + 2]) | (bf(cb[static_cast<size_t>(v) * 4 + 3]) << 16);
     }
   }
   L->tlut_words = static_cast<int>(tlut.size());
@@ -244,9 +240,11 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
   return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess) ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
+static int decode_kernel_for(int M) { return M <= 8 ? UNISVQ_KERNEL_GEMV : UNISVQ_KERNEL_SKINNY; }
+
 static int auto_kernel(const unisvq_layer* L, int M) {
-  if (M > 32 && prefill_supported(L, M)) return UNISVQ_KERNEL_PREFILL;
-  return UNISVQ_KERNEL_DECODE;
+  if (M > 64 && prefill_supported(L, M)) return UNISVQ_KERNEL_PREFILL;
+  return decode_kernel_for(M);
 }
 
 static unisvq_status check_io(unisvq_handle h, const void* x, void* y, int M) {
@@ -267,8 +265,10 @@ unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, vo
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
   if (dev != h->device) return UNISVQ_ERR_INVALID_ARG;
   if (kernel == UNISVQ_KERNEL_AUTO) kernel = auto_kernel(h, M);
+  if (kernel == UNISVQ_KERNEL_DECODE) kernel = decode_kernel_for(M);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (kernel == UNISVQ_KERNEL_DECODE) return launch_decode(h, x, y, M, s);
+  if (kernel == UNISVQ_KERNEL_GEMV) return launch_gemv(h, x, y, M, s);
+  if (kernel == UNISVQ_KERNEL_SKINNY) return launch_skinny(h, x, y, M, s);
   if (kernel == UNISVQ_KERNEL_PREFILL) {
     if (!prefill_supported(h, M)) return UNISVQ_ERR_UNSUPPORTED;
     return launch_prefill(h, x, y, M, s);
@@ -299,10 +299,14 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
                      2ll * M * h->K + 2ll * M * h->N;
   info->flops = 2.0 * M * static_cast<double>(h->N) * h->K;
   info->kernel = auto_kernel(h, M > 0 ? M : 1);
-  if (info->kernel == UNISVQ_KERNEL_DECODE) {
-    const DecodePlan p = plan_decode(h, M > 32 ? 32 : (M > 0 ? M : 1));
+  if (info->kernel == UNISVQ_KERNEL_GEMV) {
+    const DecodePlan p = plan_gemv(h, M > 16 ? 16 : (M > 0 ? M : 1));
     info->split_k = p.ks;
-    info->grid_ctas = p.ks * p.nb * ((M + 31) / 32 > 0 ? (M + 31) / 32 : 1);
+    info->grid_ctas = p.ks * p.nb * ((M + 15) / 16 > 0 ? (M + 15) / 16 : 1);
+  } else if (info->kernel == UNISVQ_KERNEL_SKINNY) {
+    const DecodePlan p = plan_skinny(h, M > 64 ? 64 : (M > 0 ? M : 1));
+    info->split_k = p.ks;
+    info->grid_ctas = p.ks * p.nb * ((M + 63) / 64 > 0 ? (M + 63) / 64 : 1);
   } else {
     const PrefillPlan p = plan_prefill(h, M);
     info->split_k = 1;

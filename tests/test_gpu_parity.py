@@ -59,30 +59,36 @@ def test_dequant_debug_bit_exact(d, N, K):
 DECODE_SHAPES = [(256, 1024), (520, 1000), (130, 4096), (1024, 8192)]
 
 
+DECODE_KERNELS = [binding.KERNEL_GEMV, binding.KERNEL_SKINNY]
+
+
+@pytest.mark.parametrize("kernel", DECODE_KERNELS)
 @pytest.mark.parametrize("d", [1, 2, 4])
 @pytest.mark.parametrize("N,K", DECODE_SHAPES)
-def test_decode_parity_small_M(d, N, K):
+def test_decode_parity_small_M(kernel, d, N, K):
     if K % d:
         pytest.skip("K % d")
     codes, A, B = synth.layer_inputs(2, 20, N, K, N, K, d)
     layer = binding.UniSVQLinear(codes, A, B)
-    for M in (1, 2, 3, 7, 8, 9, 16, 17, 31, 32):
+    for M in (1, 2, 3, 7, 8, 9, 16, 17, 31, 32, 64):
         xb = synth.activations(2, 20, 1000 * N + M, M, K)
-        check(run(layer, xb, binding.KERNEL_DECODE), xb, codes, A, B)
+        check(run(layer, xb, kernel), xb, codes, A, B)
     layer.close()
 
 
-def test_decode_many_token_groups():
+@pytest.mark.parametrize("kernel", DECODE_KERNELS)
+def test_decode_many_token_groups(kernel):
     N, K, d = 384, 768, 2
     codes, A, B = synth.layer_inputs(3, 30, 0, 0, N, K, d)
     layer = binding.UniSVQLinear(codes, A, B)
-    for M in (33, 64, 100):
+    for M in (33, 64, 100, 130):
         xb = synth.activations(3, 30, M, M, K)
-        check(run(layer, xb, binding.KERNEL_DECODE), xb, codes, A, B)
+        check(run(layer, xb, kernel), xb, codes, A, B)
     layer.close()
 
 
-def test_integer_case_bit_exact():
+@pytest.mark.parametrize("kernel", DECODE_KERNELS)
+def test_integer_case_bit_exact(kernel):
     """Integer A (the printed D4 generator), integer B and small integer x:
     every intermediate is exact, so the GPU output must equal the oracle's."""
     d = 4
@@ -97,7 +103,7 @@ def test_integer_case_bit_exact():
         xb = synth.f32_to_bf16_bits(x)
         yr, _ = oracle.linear(xb, codes, A, B)
         assert np.abs(yr).max() <= 256
-        yg = run(layer, xb, binding.KERNEL_DECODE)
+        yg = run(layer, xb, kernel)
         assert np.array_equal(yg, yr), np.abs(yg - yr).max()
     layer.close()
 
@@ -176,6 +182,8 @@ def test_full_size_decode_sampled_rows(N, K):
     for M in (1, 8, 16, 32):
         xb = synth.activations(0, 3, M, M, K)
         check(run(layer, xb), xb, codes, A, B, rows=rows)
+        if M <= 16:
+            check(run(layer, xb, binding.KERNEL_SKINNY), xb, codes, A, B, rows=rows)
     layer.close()
 
 
@@ -219,7 +227,8 @@ def test_prefill_and_decode_agree_with_auto_dispatch():
     N, K, d = 512, 1024, 2
     codes, A, B = synth.layer_inputs(9, 90, 0, 0, N, K, d)
     layer = binding.UniSVQLinear(codes, A, B)
-    assert layer.query(1)["kernel"] == binding.KERNEL_DECODE
+    assert layer.query(1)["kernel"] == binding.KERNEL_GEMV
+    assert layer.query(16)["kernel"] == binding.KERNEL_SKINNY
     assert layer.query(2048)["kernel"] == binding.KERNEL_PREFILL
     xb = synth.activations(9, 90, 0, 96, K)
     check(run(layer, xb), xb, codes, A, B)

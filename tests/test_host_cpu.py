@@ -30,21 +30,18 @@ def decode_layout(packed: np.ndarray, N: int, K: int) -> np.ndarray:
     Np = -(-N // 128) * 128
     Kp = -(-K // 128) * 128
     KT = Kp // 128
-    words = packed.view("<u4").reshape(Np // 16, KT, 32, 4)
+    words = packed.view("<u4").reshape(Np // 128, KT, 2, 128, 4)   # [rb][kt][h][r][wi]
     out = np.full((Np, Kp), 255, dtype=np.int64)
-    for rt in range(Np // 16):
+    for rb in range(Np // 128):
         for kt in range(KT):
-            for lane in range(32):
-                g, t = lane // 4, lane % 4
-                for q in range(4):
-                    grp, rh = q // 2, q % 2
-                    n = 16 * rt + g + 8 * rh
-                    w = int(words[rt, kt, lane, q])
-                    for p in range(8):
-                        i, h = p // 2, p % 2
-                        k = 128 * kt + 64 * grp + 16 * i + 4 * t + 2 * h
-                        out[n, k] = (w >> (2 * p)) & 3
-                        out[n, k + 1] = (w >> (16 + 2 * p)) & 3
+            for h in range(2):
+                for r in range(128):
+                    for wi in range(4):
+                        w = int(words[rb, kt, h, r, wi])
+                        for s in range(4):
+                            for b in range(4):
+                                k = 128 * kt + 64 * h + 16 * wi + 4 * s + b
+                                out[128 * rb + r, k] = (w >> (8 * b + 2 * s)) & 3
     return out
 
 
@@ -55,7 +52,7 @@ def test_pack_host_layout_roundtrip(lib, N, K):
     codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
     packed = binding.pack_host(codes)
     assert packed.nbytes == binding.packed_code_bytes(N, K)
-    assert packed.nbytes == (-(-N // 128) * 8) * (-(-K // 128)) * 512
+    assert packed.nbytes == (-(-N // 128)) * (-(-K // 128)) * 4096
     full = decode_layout(packed, N, K)
     assert not (full == 255).any(), "some (row, col) never written"
     assert np.array_equal(full[:N, :K], codes)
