@@ -61,10 +61,14 @@ enum {
  * (rb * (Kp/128) + kt) * 4096, so the tiles of one 128-row block are
  * consecutive along K.
  *
- * Inside a tile, half h (columns 64h .. 64h+63) fills bytes [2048h, 2048h+2048)
- * and row r of the tile owns the 16 bytes at 2048h + 16r: four little-endian
- * 32-bit words w0..w3. Word wi holds the 16 codes of columns
- *   k = 128 kt + 64 h + 16 wi + 4 s + b,   s, b in 0..3,
+ * Inside a tile, row r = 16u + 8q + g (unit u in 0..7, q in 0..1, g in 0..7)
+ * and column quarter t (0..3) of half h (columns 64h .. 64h+63) own the
+ * little-endian 32-bit word at byte
+ *   512 u + 16 (4 g + t) + 4 (2 h + q),
+ * so each unit of 16 rows fills 512 contiguous bytes and each 16-byte chunk
+ * holds rows g and g + 8 of quarter t in both halves. The word holds the 16
+ * codes of columns
+ *   k = 128 kt + 64 h + 16 t + 4 s + b,   s, b in 0..3,
  * the code of column k in bits [8b+2s+1 : 8b+2s]. Shifting a word right by 2s
  * and masking with 0x03030303 yields the codes of columns 4s..4s+3 one per
  * byte; a run of 4 columns 4m..4m+3 therefore never spans two words.

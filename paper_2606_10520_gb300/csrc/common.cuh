@@ -20,7 +20,8 @@ enum : int {
   kErrTimeoutEmpty = 2,   // waiting for consumers to free a ring slot
   kErrTimeoutMma = 3,     // waiting for the tensor core
   kErrTimeoutAcc = 4,     // waiting for the epilogue to free an accumulator
-  kErrBadLaunch = 5       // launch geometry does not match the arguments
+  kErrBadLaunch = 5,      // launch geometry does not match the arguments
+  kErrTimeoutReduce = 6   // waiting for the partial sums of the other cluster CTAs
 };
 
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
@@ -76,6 +77,32 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Same, acquiring at cluster scope: for data that other CTAs of the cluster
+// stored with st.async into this CTA (their complete_tx releases at cluster scope).
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, int* err, int code) {
+  const unsigned long long t0 = globaltimer();
+#pragma unroll 1
+  while (!mbar_try_wait_cluster(bar, parity)) {
+    if (globaltimer() - t0 > kWaitLimitNs) {
+      record_error(err, code);
+      return false;
+    }
+  }
+  return true;
+}
+
 // Bounded wait for phase `parity` of an mbarrier. Returns false (after
 // recording `code`) if the phase does not complete within kWaitLimitNs.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* err, int code) {
@@ -118,6 +145,28 @@ __device__ __forceinline__ uint64_t policy_evict_last() {
   return p;
 }
 
+// ---- ordered global loads ---------------------------------------------------
+// Inline-asm loads stay in program order relative to the other inline asm of
+// a kernel (the programmatic-launch wait, MMAs): code words can be requested
+// early on purpose, and activations are never read before the wait.
+
+__device__ __forceinline__ uint4 ldg_stream_v4(const void* p) {   // read-only data (codes)
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+  return v;
+}
+__device__ __forceinline__ uint4 ldg_v4(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+  return v;
+}
+__device__ __forceinline__ uint2 ldg_v2(const void* p) {
+  uint2 v;
+  asm volatile("ld.global.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(p));
+  return v;
+}
+
 // ---- programmatic dependent launch ----------------------------------------
 
 __device__ __forceinline__ void pdl_wait() {
@@ -140,6 +189,15 @@ __device__ __forceinline__ void cluster_sync() {
                "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
+// Split form: arrive early (every thread), wait before the first access to
+// another CTA's shared memory, so that every CTA of the cluster has started.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ uint32_t map_shared_rank(uint32_t addr, uint32_t rank) {
   uint32_t r;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
@@ -148,6 +206,19 @@ __device__ __forceinline__ uint32_t map_shared_rank(uint32_t addr, uint32_t rank
 
 __device__ __forceinline__ void st_shared_cluster_f32(uint32_t addr, float v) {
   asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
+
+// Stores into another CTA's shared memory that count their bytes as
+// transaction on that CTA's mbarrier (both addresses from map_shared_rank).
+__device__ __forceinline__ void st_async_f32(uint32_t remote_addr, float v, uint32_t remote_bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(remote_addr),
+               "r"(__float_as_uint(v)), "r"(remote_bar)
+               : "memory");
+}
+__device__ __forceinline__ void st_async_v2f32(uint32_t remote_addr, float v0, float v1, uint32_t remote_bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.b32 [%0], {%1, %2}, [%3];" ::"r"(remote_addr),
+               "r"(__float_as_uint(v0)), "r"(__float_as_uint(v1)), "r"(remote_bar)
+               : "memory");
 }
 
 __device__ __forceinline__ float ld_shared_cluster_f32(uint32_t addr) {

@@ -19,8 +19,8 @@
 // memory. Warp roles (10 warps):
 //   0      producer: 4 KB code tiles -> shared-memory ring (cp.async.bulk)
 //   1      TMEM owner; one thread issues the MMAs
-//   2..5   converters: shared ring -> TMEM A slots (one row per thread), then
-//          the epilogue (tcgen05.ld of their 32 accumulator rows)
+//   2..5   converters: shared ring -> TMEM A slots (two units of 16 rows per
+//          warp), then the epilogue (tcgen05.ld of their 32 accumulator rows)
 //   6..9   fold: x -> per-token scale, x' = x_g A, three e4m3 B terms
 // Producer and converters never touch x, so they run before the programmatic-
 // launch wait: while the previous kernel finishes, this layer's codes already
@@ -95,15 +95,15 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
 }
 
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
+// 16 lanes x 32 columns: thread 4g + t holds, for column group k (0..3),
+// v[4k + 0 .. 1] = lane g, columns 8k + 2t + (0, 1) and
+// v[4k + 2 .. 3] = lane g + 8, columns 8k + 2t + (0, 1).
+__device__ __forceinline__ void tmem_st16x256b_x4(uint32_t taddr, const uint32_t (&v)[16]) {
   asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
-      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
-      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "tcgen05.st.sync.aligned.16x256b.x4.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
       "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
-      "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]),
-      "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]),
-      "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+      "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
       : "memory");
 }
 
@@ -161,7 +161,7 @@ __device__ __forceinline__ void fold4(const DecodeArgs& a, const float (&v)[4], 
 
 // Activations x[k .. k+3] of one token as packed bf16 (zero at or past kend).
 __device__ __forceinline__ uint2 load_x4(const uint16_t* row, int k, int kend, bool vec) {
-  if (vec && k + 3 < kend) return __ldg(reinterpret_cast<const uint2*>(row + k));
+  if (vec && k + 3 < kend) return ldg_v2(row + k);
   uint32_t e[4];
 #pragma unroll
   for (int j = 0; j < 4; ++j) e[j] = (k + j < kend) ? static_cast<uint32_t>(row[k + j]) : 0u;
@@ -219,6 +219,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
     fence_mbar_init();
   }
   __syncthreads();
+  if (KS > 1) cluster_arrive_relaxed();   // waited for before the first remote store
   pdl_launch_dependents();
 
   if (warp == 0) {
@@ -282,33 +283,48 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
     }
   } else if (warp < kFoldWarp0) {
     // ---------------- converters: shared ring -> TMEM A slots ----------------
+    // Warp of TMEM lane quarter Q covers units 2Q and 2Q+1 (rows 32Q .. 32Q+31).
+    // Lane 4g + t reads the words of rows g and g + 8 of a unit for column
+    // quarter t (one 16-byte load, layout.h) and stores them as TMEM columns
+    // 8k + 2t + e of lanes g and g + 8, k = 2h + s/2, e = s % 2: the K order
+    // of the A slot is therefore a fixed permutation of the 128 columns, which
+    // the fold applies to the B operand as well (a_slot_col below).
     const int q = warp & 3;                    // TMEM lane quarter
-    const int r = 32 * q + lane;               // row of this thread
     bool ok = !*abort_flag && mbar_wait(tmem_ready, 0, a.err, kErrTimeoutFull);
     tc_fence_after();
     const uint32_t tbase = *tmem_ptr;
-    const uint32_t trow = tbase + (static_cast<uint32_t>(32 * q) << 16);
+    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * q) << 16);
     for (int kt = 0; kt < n_kt; ++kt) {
       const int s = kt % C::kCodeStages, sa = kt % kASlots;
       if (ok) ok = !*abort_flag && mbar_wait(code_full(s), (kt / C::kCodeStages) & 1, a.err, kErrTimeoutFull);
-      uint4 w0 = make_uint4(0, 0, 0, 0), w1 = w0;
+      uint4 c0 = make_uint4(0, 0, 0, 0), c1 = c0;
       if (ok) {
-        const uint8_t* tile = smem + C::kOffCode + s * kTileBytes;
-        w0 = *reinterpret_cast<const uint4*>(tile + tile_row_offset(r, 0));
-        w1 = *reinterpret_cast<const uint4*>(tile + tile_row_offset(r, 1));
+        const uint8_t* tile = smem + C::kOffCode + s * kTileBytes + (2 * q) * kUnitBytes + lane * 16;
+        c0 = *reinterpret_cast<const uint4*>(tile);
+        c1 = *reinterpret_cast<const uint4*>(tile + kUnitBytes);
       }
       __syncwarp();
       if (lane == 0 && ok) mbar_arrive(code_empty(s));
-      uint32_t v[32];
-      const uint32_t ws[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+      uint32_t v0[16], v1[16];
 #pragma unroll
-      for (int j = 0; j < 8; ++j)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) v[4 * j + e] = extract4(ws[j], e);   // TMEM column 4j + e
+      for (int k = 0; k < 4; ++k) {
+        const int h = k >> 1, s0 = 2 * (k & 1);
+        const uint32_t a0 = h ? c0.z : c0.x, a1 = h ? c0.w : c0.y;   // unit 2Q: rows g, g + 8
+        const uint32_t b0 = h ? c1.z : c1.x, b1 = h ? c1.w : c1.y;   // unit 2Q+1
+        v0[4 * k + 0] = extract4(a0, s0);
+        v0[4 * k + 1] = extract4(a0, s0 + 1);
+        v0[4 * k + 2] = extract4(a1, s0);
+        v0[4 * k + 3] = extract4(a1, s0 + 1);
+        v1[4 * k + 0] = extract4(b0, s0);
+        v1[4 * k + 1] = extract4(b0, s0 + 1);
+        v1[4 * k + 2] = extract4(b1, s0);
+        v1[4 * k + 3] = extract4(b1, s0 + 1);
+      }
       if (ok && kt >= kASlots) ok = !*abort_flag && mbar_wait(a_empty(sa), ((kt / kASlots) - 1) & 1, a.err, kErrTimeoutMma);
       if (ok) {
         tc_fence_after();
-        tmem_st32(trow + kAColBase + 32 * sa, v);
+        tmem_st16x256b_x4(tq + kAColBase + 32 * sa, v0);
+        tmem_st16x256b_x4(tq + (16u << 16) + kAColBase + 32 * sa, v1);
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         tc_fence_before();
       }
@@ -318,6 +334,8 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
     }
 
     // ---------------- epilogue: accumulator rows -> cluster reduction ----------------
+    const int r = 32 * q + lane;               // accumulator row (TMEM lane) of this thread
+    const uint32_t trow = tq;
     if (ok) ok = !*abort_flag && mbar_wait(d_full, 0, a.err, kErrTimeoutMma);
     if (ok) ok = mbar_wait(fold_done, 0, a.err, kErrTimeoutFull);
     if (!ok) *abort_flag = 1;
@@ -326,6 +344,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
     const uint32_t slot_off =
         (static_cast<uint32_t>(blockIdx.x) * rows_per + (r - owner * rows_per)) * NTOK * 4u;
     const uint32_t red_addr = sbase + C::kOffRed;
+    if (KS > 1) cluster_wait();
     tc_fence_after();
 #pragma unroll
     for (int c0 = 0; c0 < NTOK; c0 += 16) {
@@ -373,7 +392,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
         for (int j = 0; j < 8; ++j) {
           const int k = k0 + 256 * j;
           if (vec8 && k + 7 < kend) {
-            u[j] = __ldg(reinterpret_cast<const uint4*>(row + k));
+            u[j] = ldg_v4(row + k);
           } else {
             uint32_t e[8];
 #pragma unroll
@@ -417,8 +436,12 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
     // Pass 2: warp fw folds k-tiles fw, fw + kBStages, ... (its own stage) for
     // all tokens; lane covers columns 4 lane .. 4 lane + 3 of the k-tile.
     bool ok = !*abort_flag;
-    const uint32_t cidx = (4 * lane) & 15;
-    const uint32_t chunk = (4 * lane) >> 4;
+    // Columns 4 lane .. 4 lane + 3 = 64h + 16t + 4s + (0..3) sit in A-slot
+    // column 16h + 8(s/2) + 2t + s%2 (converter mapping), i.e. at bytes
+    // 4 * that column of each 128-byte B row.
+    const uint32_t a_slot_col = 16 * (lane >> 4) + 8 * ((lane & 3) >> 1) + 2 * ((lane >> 2) & 3) + (lane & 1);
+    const uint32_t cidx = (a_slot_col & 3) * 4;
+    const uint32_t chunk = a_slot_col >> 2;
     for (int kt = fw; fw < C::kBStages && kt < n_kt; kt += C::kBStages) {
       const int sb = fw;
       const int use = kt / C::kBStages;      // how many times stage sb was filled before
@@ -456,7 +479,12 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
 
   // ---------------- reduction over the K slices of the cluster ----------------
   __syncwarp();
-  if (KS > 1) cluster_sync(); else __syncthreads();
+  if (KS > 1) {
+    if (warp < 2 || warp >= kFoldWarp0) cluster_wait();   // converters waited before their stores
+    cluster_sync();
+  } else {
+    __syncthreads();
+  }
   {
     const int rows_per = (kTileRows + KS - 1) / KS;
     const int r0 = static_cast<int>(blockIdx.x) * rows_per;

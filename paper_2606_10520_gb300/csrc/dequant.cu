@@ -1,7 +1,7 @@
 // Test hook: W_hat [N][K] in fp32 from the packed device layout.
 //
-// Each thread unpacks one 16-byte row chunk (64 codes of one row) with the
-// same extraction helper the layer kernels use (layout.h), rebuilds the index
+// Each thread unpacks the four words of one (row, half) -- 64 codes -- with
+// the same extraction helper the layer kernels use (layout.h), rebuilds the index
 // z0 | z1 << 2 | ... of every d-vector and reads the fp32 codeword
 // RN_fp32(A z + B) of Eq. (def:unisvq) from the handle's codebook.
 #include "common.cuh"
@@ -15,14 +15,15 @@ __global__ void __launch_bounds__(256) dequant_kernel(const uint8_t* __restrict_
                                                       int N, int K, int KT, int d, int nchunks) {
   const int id = blockIdx.x * 256 + threadIdx.x;
   if (id >= nchunks) return;
-  const int tile = id >> 8;               // 256 row chunks per tile (2 halves x 128 rows)
+  const int tile = id >> 8;               // 256 (row, half) pairs per tile
   const int h = (id >> 7) & 1, r = id & 127;
   const int rb = tile / KT, kt = tile - rb * KT;
   const int row = rb * kTileRows + r;
   if (row >= N) return;
-  const uint4 q = *reinterpret_cast<const uint4*>(codes + static_cast<size_t>(tile) * kTileBytes +
-                                                  tile_row_offset(r, h));
-  const uint32_t words[4] = {q.x, q.y, q.z, q.w};
+  const uint8_t* tb = codes + static_cast<size_t>(tile) * kTileBytes;
+  uint32_t words[4];
+#pragma unroll
+  for (int t = 0; t < 4; ++t) words[t] = *reinterpret_cast<const uint32_t*>(tb + tile_word_offset(r, h, t));
 #pragma unroll
   for (int wi = 0; wi < 4; ++wi) {
 #pragma unroll

@@ -9,27 +9,38 @@
 //   w        & (0x00030003 << 2s)  = fp16 pair (z[4s], z[4s+2]) * 4^s * 2^-24,
 //   (w >> 8) & (0x00030003 << 2s)  = fp16 pair (z[4s+1], z[4s+3]) * 4^s * 2^-24,
 // fp16 subnormals (exact in the tensor core): one shift and eight ANDs turn 16
-// codes into 8 registers. In MMA j of a 64-column half, thread t (of row
-// group g) supplies word t of its two rows with s = j, so the MMA covers the
-// 16 columns 16 t + 4 j + b; the folded activations are stored in the same
-// order as fp16 x' * 2^P * 4^-j. Products are x' z 2^(P-24); the fp32 sums
-// are rescaled by 2^(24-P) at the end.
+// codes into 8 registers. In MMA (h, j) of a k-tile, lane 4g + t supplies the
+// quarter-t words of rows g and g + 8 of half h with s = j, so the MMA covers
+// the 16 columns 64h + 16t + 4j + b; the B operand holds the folded
+// activations of those columns as fp16 x' * 2^P * 4^-j. Products are
+// x' z 2^(P-24); the fp32 sums are rescaled by 2^(24-P) at the end.
 //
-// CTA = 128 output rows x one K slice, 8 warps of 16 rows. Each thread keeps
-// 8 k-tiles of its code words in flight with plain coalesced loads (the first
-// ones issued before the programmatic-launch wait, since codes never depend on
-// the previous kernel); the K slices of a row block form a cluster and add
-// their partial sums through distributed shared memory.
+// CTA = 128 output rows x one K slice, 8 warps: warp w owns unit w (16 rows)
+// for every k-tile of the slice. Each lane streams its codes with one 16-byte
+// load per k-tile (512 contiguous bytes per warp), kGDepth k-tiles deep, and
+// the first loads are issued before the programmatic-launch wait: codes never
+// depend on the previous kernel. Warp w also folds tokens w and w + 8 of the
+// slice into shared memory by itself (per-token scale from a warp reduction),
+// so one block barrier separates the fold from a main loop that has none. The
+// K slices of a row block form a thread-block cluster; each CTA adds up the
+// partial sums of the rows it owns, which the other CTAs deliver with st.async
+// stores counted on an mbarrier.
 #include "common.cuh"
 #include "internal.h"
 
 namespace unisvq {
 namespace {
 
-constexpr int kGWarps = 8;                     // warps; warp w owns rows 16w .. 16w+15
+constexpr int kGWarps = 8;
 constexpr int kGThreads = kGWarps * 32;
-constexpr int kGDepth = 8;                     // k-tiles of codes in flight per thread
+constexpr int kGDepth = 8;          // k-tiles of codes in flight per warp (16 bytes per lane each)
+constexpr int kMaxSplit = 8;        // K slices per row block (cluster size)
 constexpr int kGMaxTok = 16;
+constexpr int kXLoads = 4;          // 16-byte activation loads in flight per lane (fold)
+constexpr int kXPad = 4;            // fp16 elements of padding per token row (bank spread)
+constexpr int kTokBytes = 160;      // pexp[16], cpart[16], reduction mbarrier
+constexpr size_t kSmemPerSm = 228 * 1024;
+constexpr size_t kSmemPerCtaReserved = 1024;
 
 struct GemvArgs {
   const uint8_t* codes;
@@ -37,34 +48,30 @@ struct GemvArgs {
   uint16_t* y;         // bf16 [M][N]
   int M, N, K, KT, d;
   int kt_per_cta;
+  int xstride;         // fp16 elements per token row of the folded slice
+  int off_red, off_tok;
   float A[16];
   float B[4];
   float colnorm;
   int* err;
 };
 
-template <int NT>
-struct GCfg {
-  static constexpr int CHB = kGDepth;                            // k-tiles per fold chunk
-  static constexpr int kFragTile = 8 * 32 * 8 * NT;              // B fragments of one k-tile
-  static constexpr int kOffX = 0;
-  static constexpr int kXBytes = NT == 1 ? 16384 : 32768;        // staged x slice (bf16)
-  static constexpr int kOffF = kOffX + kXBytes;
-  static constexpr int kFBytes = CHB * kFragTile;                // one fold buffer
-  static constexpr int kOffRed = kOffF + 2 * kFBytes;
-  static constexpr int kRedBytes = (kTileRows + 8) * 8 * NT * 4;
-  static constexpr int kOffTok = kOffRed + kRedBytes;            // pexp[32], cpart[32]
-  static constexpr int kOffMisc = kOffTok + 256;
-  static constexpr int kSmem = kOffMisc + 64;
-};
-
 __device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
-                                          uint32_t b0, uint32_t b1) {
+                                          uint2 b) {
   asm volatile(
       "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
       "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b.x), "r"(b.y));
+}
+
+__device__ __forceinline__ uint2 lds64(uint32_t addr) {
+  uint2 v;
+  asm volatile("ld.shared.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+  return v;
+}
+__device__ __forceinline__ void sts64(uint32_t addr, uint32_t a, uint32_t b) {
+  asm volatile("st.shared.v2.u32 [%0], {%1,%2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
 }
 
 // x'[c .. c+3] for the d-vectors inside x[c .. c+3] (c % 4 == 0): row vector x_g A.
@@ -84,89 +91,96 @@ __device__ __forceinline__ void gfold4(const GemvArgs& a, const float (&v)[4], f
   }
 }
 
+// Eight activations x[k .. k+7] of one token as packed bf16 (zero at or past kend).
+__device__ __forceinline__ uint4 load_x8(const uint16_t* row, int k, int kend, bool vec8) {
+  if (vec8 && k + 7 < kend) return ldg_v4(row + k);
+  uint32_t e[8];
+#pragma unroll
+  for (int q = 0; q < 8; ++q) e[q] = (k + q < kend) ? static_cast<uint32_t>(row[k + q]) : 0u;
+  return make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
+}
+
 template <int NT>
 __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constant__ GemvArgs a) {
-  using C = GCfg<NT>;
-  extern __shared__ __align__(128) uint8_t smem[];
+  extern __shared__ __align__(16) uint8_t smem[];
   const uint32_t sbase = smem_u32(smem);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int KS = gridDim.x;
   const int kt0 = blockIdx.x * a.kt_per_cta;
   const int n_kt = min(a.kt_per_cta, a.KT - kt0);
   const int rb = blockIdx.y;
+  const int M = a.M;
+  // Rows whose K-slice partial sums this CTA adds up (it "owns" them).
+  const int rows_per = (kTileRows + KS - 1) / KS;
+  const int own0 = static_cast<int>(blockIdx.x) * rows_per;
+  const int nown = max(0, min(kTileRows, own0 + rows_per) - own0);
 
-  int* pexp = reinterpret_cast<int*>(smem + C::kOffTok);
-  float* cpart = reinterpret_cast<float*>(smem + C::kOffTok + 128);
-  float* red = reinterpret_cast<float*>(smem + C::kOffRed);
-  // A valid plan gives every CTA at least one k-tile; otherwise flag the error
-  // and fall through with empty loops so the cluster barrier is still reached.
-  if (n_kt <= 0 && tid == 0) record_error(a.err, kErrBadLaunch);
-  {  // fold buffers start at zero: fragments of tokens >= M stay zero
-    uint4* f = reinterpret_cast<uint4*>(smem + C::kOffF);
-    for (int i = tid; i < 2 * C::kFBytes / 16; i += kGThreads) f[i] = make_uint4(0, 0, 0, 0);
-  }
+  int* pexp = reinterpret_cast<int*>(smem + a.off_tok);
+  float* cpart = reinterpret_cast<float*>(smem + a.off_tok + 64);
+  float* red = reinterpret_cast<float*>(smem + a.off_red);
+  const uint32_t red_bar = sbase + a.off_tok + 128;
 
-  // Codes: warp w reads, for each k-tile, word t (lane % 4) of rows r0 = 16w + g
-  // and r0 + 8 in both 64-column halves (4 x 4 bytes; each warp load instruction
-  // covers 128 contiguous bytes). kGDepth k-tiles are kept in flight; the first
-  // ones are requested before the programmatic-launch wait (codes never depend
-  // on the previous kernel).
-  const int g = lane >> 2, t = lane & 3;
-  const int r0 = 16 * warp + g;
-  const uint8_t* cbase = a.codes + (static_cast<size_t>(rb) * a.KT + kt0) * kTileBytes + 4 * t;
-  auto load_codes = [&](int kt, uint32_t (&w)[4]) {
-    if (kt < n_kt) {
-      const uint8_t* tb = cbase + static_cast<size_t>(kt) * kTileBytes;
-      w[0] = __ldg(reinterpret_cast<const uint32_t*>(tb + tile_row_offset(r0, 0)));
-      w[1] = __ldg(reinterpret_cast<const uint32_t*>(tb + tile_row_offset(r0 + 8, 0)));
-      w[2] = __ldg(reinterpret_cast<const uint32_t*>(tb + tile_row_offset(r0, 1)));
-      w[3] = __ldg(reinterpret_cast<const uint32_t*>(tb + tile_row_offset(r0 + 8, 1)));
+  // Reduction barrier: one arrival here plus the bytes the other CTAs of the
+  // cluster store into this CTA's slots (st.async counts them).
+  if (KS > 1) {
+    if (tid == 0) {
+      mbar_init(red_bar, 1);
+      fence_mbar_init();
+      mbar_arrive_expect_tx(red_bar, static_cast<uint32_t>((KS - 1) * nown * M * 4));
     }
-  };
-  uint32_t cw[kGDepth][4];
+    cluster_arrive_relaxed();
+  }
+  // A valid plan gives every CTA at least one k-tile; otherwise flag the error
+  // and fall through with empty loops so that every partial is still sent.
+  if (n_kt <= 0 && tid == 0) record_error(a.err, kErrBadLaunch);
+
+  // ---- codes: unit `warp` (rows 16 warp .. +15) of every k-tile of the slice ----
+  const int g = lane >> 2, t = lane & 3;
+  const uint8_t* cbase =
+      a.codes + (static_cast<size_t>(rb) * a.KT + kt0) * kTileBytes + warp * kUnitBytes + lane * 16;
+  uint4 cw[kGDepth];
 #pragma unroll
-  for (int i = 0; i < kGDepth; ++i) load_codes(i, cw[i]);
-  __syncthreads();
+  for (int s = 0; s < kGDepth; ++s)
+    if (s < n_kt) cw[s] = ldg_stream_v4(cbase + static_cast<size_t>(s) * kTileBytes);
   pdl_launch_dependents();
 
   pdl_wait();   // x may be the previous kernel's output
+
+  // ---- fold: warp w prepares tokens w and w + 8 on its own (no block barrier) ----
+  // Pass A stages the slice and finds max |x| and sum_k x[k] B[k mod d]; 2^P puts
+  // the largest possible |x'| (<= max|x| * colnorm) below 2^15 (fp16). Pass B
+  // folds in place: columns c .. c+3 (c = 16t' + 4j inside a 64-column half)
+  // become the B fragment (x'[c], x'[c+2]), (x'[c+1], x'[c+3]) * 2^P * 4^-j.
   const int kbeg = kt0 * kTileCols;
   const int kend = min(a.K, (kt0 + n_kt) * kTileCols);
-  const int kspan = n_kt * kTileCols;
+  const int nch = n_kt * (kTileCols / 8);   // 8-column chunks of the slice
   const bool vec8 = (a.K & 7) == 0;
-  const bool staged = a.M * kspan * 2 <= C::kXBytes;
-  uint16_t* xs = reinterpret_cast<uint16_t*>(smem + C::kOffX);
-  // Pass 1: per-token max |x| and sum_k x[k] B[k mod d] over the slice;
-  // warp w owns tokens w, w + 8; 8 columns per lane per load, 8 in flight.
-  for (int tok = warp; tok < a.M; tok += kGWarps) {
-    const uint16_t* row = a.x + static_cast<size_t>(tok) * a.K;
+  const uint32_t xrow_bytes = static_cast<uint32_t>(a.xstride) * 2u;
+  for (int tk = warp; tk < M; tk += kGWarps) {
+    const uint16_t* row = a.x + static_cast<size_t>(tk) * a.K;
+    const uint32_t xrow = sbase + tk * xrow_bytes;
     float mx = 0.f, cs = 0.f;
-    for (int k0 = kbeg + 8 * lane; k0 < kbeg + kspan; k0 += 8 * 32 * 8) {
-      uint4 u[8];
+    uint4 u[kXLoads];
+    for (int c0 = lane; c0 < nch; c0 += 32 * kXLoads) {
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int k = k0 + 256 * j;
-        if (vec8 && k + 7 < kend) {
-          u[j] = __ldg(reinterpret_cast<const uint4*>(row + k));
-        } else {
-          uint32_t e[8];
-#pragma unroll
-          for (int q = 0; q < 8; ++q) e[q] = (k + q < kend) ? static_cast<uint32_t>(row[k + q]) : 0u;
-          u[j] = make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
-        }
+      for (int j = 0; j < kXLoads; ++j) {
+        const int ci = c0 + 32 * j;
+        u[j] = ci < nch ? load_x8(row, kbeg + 8 * ci, kend, vec8) : make_uint4(0, 0, 0, 0);
       }
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int k = k0 + 256 * j;
-        if (k >= kbeg + kspan) break;
-        if (staged) *reinterpret_cast<uint4*>(xs + tok * kspan + (k - kbeg)) = u[j];
-        const uint32_t w4[4] = {u[j].x, u[j].y, u[j].z, u[j].w};
+      for (int j = 0; j < kXLoads; ++j) {
+        const int ci = c0 + 32 * j;
+        if (ci < nch) {
+          sts64(xrow + 16u * ci, u[j].x, u[j].y);
+          sts64(xrow + 16u * ci + 8, u[j].z, u[j].w);
+          const uint32_t w4[4] = {u[j].x, u[j].y, u[j].z, u[j].w};
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const float v0 = bf16_lo(w4[q]), v1 = bf16_hi(w4[q]);
-          mx = fmaxf(mx, fmaxf(fabsf(v0), fabsf(v1)));
-          cs = fmaf(v0, a.B[(2 * q) & (a.d - 1)], cs);
-          cs = fmaf(v1, a.B[(2 * q + 1) & (a.d - 1)], cs);
+          for (int q = 0; q < 4; ++q) {
+            const float v0 = bf16_lo(w4[q]), v1 = bf16_hi(w4[q]);
+            mx = fmaxf(mx, fmaxf(fabsf(v0), fabsf(v1)));
+            cs = fmaf(v0, a.B[(2 * q) & (a.d - 1)], cs);
+            cs = fmaf(v1, a.B[(2 * q + 1) & (a.d - 1)], cs);
+          }
         }
       }
     }
@@ -175,53 +189,51 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
       cs += __shfl_xor_sync(0xffffffffu, cs, off);
     }
+    const float bound = mx * a.colnorm;
+    int e2 = 0;
+    if (bound > 0.f) frexpf(bound, &e2);
+    const int pe = bound > 0.f ? max(-100, min(100, 15 - e2)) : 0;
     if (lane == 0) {
-      // 2^P puts the largest possible |x'| (<= max|x| * colnorm) below 2^15 (fp16).
-      const float bound = mx * a.colnorm;
-      int e2 = 0;
-      if (bound > 0.f) frexpf(bound, &e2);
-      pexp[tok] = bound > 0.f ? max(-100, min(100, 15 - e2)) : 0;
-      cpart[tok] = cs;
+      pexp[tk] = pe;
+      cpart[tk] = cs;
+    }
+    auto fold8 = [&](int ci, uint4 xv) {
+      // columns 8ci .. 8ci+7 of the slice: four-column groups j0 and j0 + 1
+      const int j0 = (2 * ci) & 3;
+      const float v0[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
+      const float v1[4] = {bf16_lo(xv.z), bf16_hi(xv.z), bf16_lo(xv.w), bf16_hi(xv.w)};
+      float o0[4], o1[4];
+      gfold4(a, v0, o0);
+      gfold4(a, v1, o1);
+      const float s0 = exp2i(pe - 2 * j0), s1 = exp2i(pe - 2 * j0 - 2);
+      sts64(xrow + 16u * ci, pack_half2(o0[0] * s0, o0[2] * s0), pack_half2(o0[1] * s0, o0[3] * s0));
+      sts64(xrow + 16u * ci + 8, pack_half2(o1[0] * s1, o1[2] * s1), pack_half2(o1[1] * s1, o1[3] * s1));
+    };
+    if (nch <= 32 * kXLoads) {
+      // the whole slice is still in registers
+#pragma unroll
+      for (int j = 0; j < kXLoads; ++j)
+        if (lane + 32 * j < nch) fold8(lane + 32 * j, u[j]);
+    } else {
+      // every lane re-reads only the chunks it staged itself
+      for (int c0 = lane; c0 < nch; c0 += 32 * kXLoads) {
+#pragma unroll
+        for (int j = 0; j < kXLoads; ++j) {
+          const int ci = c0 + 32 * j;
+          if (ci < nch) {
+            const uint2 lo = lds64(xrow + 16u * ci), hi = lds64(xrow + 16u * ci + 8);
+            u[j] = make_uint4(lo.x, lo.y, hi.x, hi.y);
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < kXLoads; ++j)
+          if (c0 + 32 * j < nch) fold8(c0 + 32 * j, u[j]);
+      }
     }
   }
   __syncthreads();
 
-  // Fold chunk ch (CHB k-tiles) into B fragments: unit = (token, k-tile, half,
-  // thread t, MMA j) -> 8 bytes (x'[c], x'[c+2]), (x'[c+1], x'[c+3]) * 2^P * 4^-j,
-  // c = 64 h + 16 t + 4 j.
-  auto fold = [&](int ch) {
-    uint2* fb = reinterpret_cast<uint2*>(smem + C::kOffF + (ch & 1) * C::kFBytes);
-    const int kt_a = ch * C::CHB;
-    const int nkt = min(C::CHB, n_kt - kt_a);
-    const int units = a.M * nkt * 32;   // 32 four-column units per k-tile
-    for (int u = tid; u < units; u += kGThreads) {
-      const int tok = u / (nkt * 32);
-      const int r = u - tok * (nkt * 32);
-      const int ktl = r >> 5;
-      const int h = (r >> 4) & 1, tt = (r >> 2) & 3, j = r & 3;
-      const int koff = (kt_a + ktl) * kTileCols + 64 * h + 16 * tt + 4 * j;   // column within the slice
-      uint2 xv;
-      if (staged) {
-        xv = *reinterpret_cast<const uint2*>(xs + tok * kspan + koff);
-      } else {
-        const int k = kbeg + koff;
-        const uint16_t* row = a.x + static_cast<size_t>(tok) * a.K;
-        uint32_t e[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) e[q] = (k + q < kend) ? static_cast<uint32_t>(row[k + q]) : 0u;
-        xv = make_uint2(e[0] | (e[1] << 16), e[2] | (e[3] << 16));
-      }
-      const float v[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
-      float o[4];
-      gfold4(a, v, o);
-      const float sc = exp2i(pexp[tok] - 2 * j);
-      const uint32_t lo = pack_half2(o[0] * sc, o[2] * sc);
-      const uint32_t hi = pack_half2(o[1] * sc, o[3] * sc);
-      fb[(((tok >> 3) * C::CHB + ktl) * 8 + h * 4 + j) * 32 + (tok & 7) * 4 + tt] = make_uint2(lo, hi);
-    }
-  };
-
-  fold(0);
+  // ---- main loop: no block-wide barrier ----
   float acc[2][NT][4];
 #pragma unroll
   for (int h = 0; h < 2; ++h)
@@ -229,106 +241,127 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
     for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
       for (int e = 0; e < 4; ++e) acc[h][nt][e] = 0.f;
-
-  // One chunk of kGDepth k-tiles per step; the code registers of k-tile kt are
-  // refilled with k-tile kt + kGDepth as soon as they have been used.
-  for (int ch = 0; ch * C::CHB < n_kt; ++ch) {
-    __syncthreads();                          // fold of chunk ch complete
-    if ((ch + 1) * C::CHB < n_kt) fold(ch + 1);   // other buffer; its last readers passed the barrier
-    const uint2* fb = reinterpret_cast<const uint2*>(smem + C::kOffF + (ch & 1) * C::kFBytes);
+  bool act[NT];
+  const uint8_t* xl[NT];   // this lane's B fragments: token 8nt + g, quarter t
 #pragma unroll
-    for (int i = 0; i < kGDepth; ++i) {
-      const int kt = ch * C::CHB + i;
-      if (kt < n_kt) {
+  for (int nt = 0; nt < NT; ++nt) {
+    const int tk = 8 * nt + g;
+    act[nt] = tk < M;
+    xl[nt] = smem + (act[nt] ? tk : 0) * xrow_bytes + 32u * t;
+  }
+  for (int i0 = 0; i0 < n_kt; i0 += kGDepth) {
+#pragma unroll
+    for (int s = 0; s < kGDepth; ++s) {
+      const int i = i0 + s;
+      if (i < n_kt) {
+        const uint32_t koff = 256u * i;   // 256 bytes of B fragments per k-tile
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-          const uint32_t w = cw[i][2 * h], w8 = cw[i][2 * h + 1];
-          const uint32_t ws = w >> 8, ws8 = w8 >> 8;
+          const uint32_t wa = h ? cw[s].z : cw[s].x, wb = h ? cw[s].w : cw[s].y;   // rows g, g + 8
+          const uint32_t was = wa >> 8, wbs = wb >> 8;
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             const uint32_t m = 0x00030003u << (2 * j);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
-              const uint2 b = fb[((nt * C::CHB + i) * 8 + h * 4 + j) * 32 + lane];
-              mma_16816(acc[h][nt], w & m, w8 & m, ws & m, ws8 & m, b.x, b.y);
+              const uint2 b = act[nt] ? *reinterpret_cast<const uint2*>(xl[nt] + koff + 128u * h + 8u * j)
+                                      : make_uint2(0u, 0u);
+              mma_16816(acc[h][nt], wa & m, wb & m, was & m, wbs & m, b);
             }
           }
         }
-        load_codes(kt + kGDepth, cw[i]);
+        if (i + kGDepth < n_kt) cw[s] = ldg_stream_v4(cbase + static_cast<size_t>(i + kGDepth) * kTileBytes);
       }
     }
   }
 
-  // Partial outputs of this K slice go into the shared memory of the cluster
-  // CTA that owns the row: slot [source rank][row - owner base].
-  {
-    const int rows_per = (kTileRows + KS - 1) / KS;
-    const uint32_t red_addr = sbase + C::kOffRed;
+  // ---- partial sums -> owner CTA of the row: slot [rank][row - owner base][token] ----
+  // Remote slots are written with st.async, which counts their bytes on the
+  // owner's mbarrier; the owner waits for exactly that many bytes, so no
+  // cluster-wide barrier is needed and no CTA's shared memory is written
+  // after it has stopped waiting.
+  constexpr int MP = 8 * NT;
+  const uint32_t red_addr = sbase + a.off_red;
+  if (KS > 1) cluster_wait();   // every CTA of the cluster has initialised its barrier
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
+  for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int row = r0 + ((e & 2) ? 8 : 0);
-        const int tok = nt * 8 + 2 * t + (e & 1);
-        if (tok < a.M) {
-          const float val = fmaf(acc[0][nt][e] + acc[1][nt][e], exp2i(24 - pexp[tok]), cpart[tok]);
-          const int owner = row / rows_per;
-          const uint32_t off =
-              ((static_cast<uint32_t>(blockIdx.x) * rows_per + (row - owner * rows_per)) * 8 * NT + tok) * 4u;
-          if (KS > 1) st_shared_cluster_f32(map_shared_rank(red_addr + off, owner), val);
-          else red[off / 4] = val;
+    for (int rh = 0; rh < 2; ++rh) {
+      const int row = 16 * warp + g + 8 * rh;
+      const int tok = 8 * nt + 2 * t;   // this lane holds tokens tok and tok + 1
+      if (tok < M) {
+        const float v0 = fmaf(acc[0][nt][2 * rh] + acc[1][nt][2 * rh], exp2i(24 - pexp[tok]), cpart[tok]);
+        const float v1 = tok + 1 < M ? fmaf(acc[0][nt][2 * rh + 1] + acc[1][nt][2 * rh + 1],
+                                            exp2i(24 - pexp[tok + 1]), cpart[tok + 1])
+                                     : 0.f;
+        const int owner = row / rows_per;
+        const uint32_t off =
+            ((static_cast<uint32_t>(blockIdx.x) * rows_per + (row - owner * rows_per)) * MP + tok) * 4u;
+        if (owner == static_cast<int>(blockIdx.x)) {
+          red[off / 4] = v0;
+          if (tok + 1 < M) red[off / 4 + 1] = v1;
+        } else if (tok + 1 < M) {
+          st_async_v2f32(map_shared_rank(red_addr + off, owner), v0, v1, map_shared_rank(red_bar, owner));
+        } else {
+          st_async_f32(map_shared_rank(red_addr + off, owner), v0, map_shared_rank(red_bar, owner));
         }
       }
-  }
-
-  // ---------------- reduction over the K slices of the cluster ----------------
-  __syncwarp();
-  if (KS > 1) cluster_sync(); else __syncthreads();
-  {
-    const int rows_per = (kTileRows + KS - 1) / KS;
-    const int r0 = static_cast<int>(blockIdx.x) * rows_per;
-    const int nrows = max(0, min(kTileRows, r0 + rows_per) - r0);
-    for (int idx = tid; idx < nrows * a.M; idx += kGThreads) {
-      const int tok = idx / nrows;
-      const int rl = idx - tok * nrows;
-      const int n = rb * kTileRows + r0 + rl;
-      float s = 0.f;
-      for (int q = 0; q < KS; ++q) s += red[(q * rows_per + rl) * 8 * NT + tok];
-      if (n < a.N) a.y[static_cast<size_t>(tok) * a.N + n] = f32_to_bf16_rn(s);
     }
+
+  // ---- reduction over the K slices of the row block ----
+  __syncthreads();   // this CTA's own slots
+  if (KS > 1 && nown > 0 && !mbar_wait_cluster(red_bar, 0, a.err, kErrTimeoutReduce)) return;
+  for (int idx = tid; idx < nown * M; idx += kGThreads) {
+    const int tok = idx / nown;
+    const int rl = idx - tok * nown;
+    const int n = rb * kTileRows + own0 + rl;
+    float v[kMaxSplit];
+#pragma unroll
+    for (int q = 0; q < kMaxSplit; ++q) v[q] = q < KS ? red[(q * rows_per + rl) * MP + tok] : 0.f;
+    float sum = 0.f;
+#pragma unroll
+    for (int q = 0; q < kMaxSplit; ++q) sum += v[q];
+    if (n < a.N) a.y[static_cast<size_t>(tok) * a.N + n] = f32_to_bf16_rn(sum);
   }
 }
 
-template <int NT>
-int gemv_resident_ctas() {
-  static int n = 0;
-  if (!n) {
-    cudaFuncSetAttribute(gemv_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, GCfg<NT>::kSmem);
-    cudaFuncSetAttribute(gemv_kernel<NT>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                         cudaSharedmemCarveoutMaxShared);
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<NT>, kGThreads, GCfg<NT>::kSmem) !=
-            cudaSuccess ||
-        n < 1)
-      n = 1;
-  }
-  return n;
+struct GemvShape {
+  size_t smem;
+  int off_red, off_tok, xstride;
+};
+
+GemvShape gemv_shape(int M, int kt_per_cta, int ks, int nt) {
+  GemvShape s{};
+  s.xstride = kt_per_cta * kTileCols + kXPad;
+  const size_t xf = static_cast<size_t>(M) * s.xstride * 2;
+  const int rows_per = (kTileRows + ks - 1) / ks;
+  const size_t red = static_cast<size_t>(ks) * rows_per * 8 * nt * 4;
+  s.off_red = static_cast<int>((xf + 15) / 16 * 16);
+  s.off_tok = static_cast<int>(s.off_red + red);
+  s.smem = static_cast<size_t>(s.off_tok) + kTokBytes;
+  return s;
+}
+
+int gemv_ctas_per_sm(size_t smem) {
+  const int by_smem = static_cast<int>(kSmemPerSm / (smem + kSmemPerCtaReserved));
+  return by_smem < 2 ? by_smem : 2;   // registers allow two 256-thread CTAs
 }
 
 template <int NT>
 unisvq_status gemv_launch_nt(const unisvq_layer* L, const DecodePlan& p, const void* x, void* y, int M,
                              cudaStream_t s) {
-  using C = GCfg<NT>;
   static bool attr_set[64] = {};
   const int dev = L->device;
   if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
   if (!attr_set[dev]) {
-    if (cudaFuncSetAttribute(gemv_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem) !=
-            cudaSuccess ||
+    if (cudaFuncSetAttribute(gemv_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(kSmemPerSm - kSmemPerCtaReserved)) != cudaSuccess ||
         cudaFuncSetAttribute(gemv_kernel<NT>, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared) != cudaSuccess)
       return UNISVQ_ERR_CUDA;
     attr_set[dev] = true;
   }
+  const GemvShape sh = gemv_shape(M, p.kt_per_cta, p.ks, NT);
   GemvArgs a{};
   a.codes = L->codes;
   a.x = static_cast<const uint16_t*>(x);
@@ -339,6 +372,9 @@ unisvq_status gemv_launch_nt(const unisvq_layer* L, const DecodePlan& p, const v
   a.KT = L->KT;
   a.d = L->d;
   a.kt_per_cta = p.kt_per_cta;
+  a.xstride = sh.xstride;
+  a.off_red = sh.off_red;
+  a.off_tok = sh.off_tok;
   for (int i = 0; i < 16; ++i) a.A[i] = L->A[i];
   for (int i = 0; i < 4; ++i) a.B[i] = L->B[i];
   a.colnorm = L->colnorm;
@@ -347,7 +383,7 @@ unisvq_status gemv_launch_nt(const unisvq_layer* L, const DecodePlan& p, const v
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.ks, p.nb, 1);
   cfg.blockDim = dim3(kGThreads, 1, 1);
-  cfg.dynamicSmemBytes = C::kSmem;
+  cfg.dynamicSmemBytes = sh.smem;
   cfg.stream = s;
   cudaLaunchAttribute attrs[2];
   attrs[0].id = cudaLaunchAttributeClusterDimension;
@@ -363,21 +399,29 @@ unisvq_status gemv_launch_nt(const unisvq_layer* L, const DecodePlan& p, const v
 
 }  // namespace
 
+// Split K into ks <= 8 cluster CTAs: the largest ks whose grid fits one wave
+// of resident CTAs; if none does (many row blocks or a large folded slice),
+// the smallest ks whose slice fits in shared memory.
 DecodePlan plan_gemv(const unisvq_layer* L, int M) {
   DecodePlan p{};
   p.nt = M <= 8 ? 1 : 2;
   p.nb = L->Np / kTileRows;
-  const int occ = p.nt == 1 ? gemv_resident_ctas<1>() : gemv_resident_ctas<2>();
-  const int slots = occ * L->num_sms;
-  int ks = 1;
-  for (int c = 8; c >= 1; --c)
-    if (c <= L->KT && p.nb * c <= slots) {
-      ks = c;
-      break;
-    }
+  const size_t cap = kSmemPerSm - kSmemPerCtaReserved;
+  int best = 0, fallback = 0;
+  for (int c = kMaxSplit; c >= 1; --c) {
+    if (c > L->KT) continue;
+    const int kpc = (L->KT + c - 1) / c;
+    const int ks = (L->KT + kpc - 1) / kpc;
+    if (ks != c) continue;
+    const size_t smem = gemv_shape(M, kpc, ks, p.nt).smem;
+    if (smem > cap) continue;
+    fallback = ks;
+    if (!best && p.nb * ks <= gemv_ctas_per_sm(smem) * L->num_sms) best = ks;
+  }
+  const int ks = best ? best : (fallback ? fallback : kMaxSplit);
   p.kt_per_cta = (L->KT + ks - 1) / ks;
   p.ks = (L->KT + p.kt_per_cta - 1) / p.kt_per_cta;
-  p.smem = p.nt == 1 ? GCfg<1>::kSmem : GCfg<2>::kSmem;
+  p.smem = gemv_shape(M, p.kt_per_cta, p.ks, p.nt).smem;
   return p;
 }
 
@@ -385,9 +429,11 @@ unisvq_status launch_gemv(const unisvq_layer* L, const void* x, void* y, int M, 
   for (int m0 = 0; m0 < M; m0 += kGMaxTok) {
     const int mc = M - m0 < kGMaxTok ? M - m0 : kGMaxTok;
     const DecodePlan p = plan_gemv(L, mc);
+    if (p.smem > kSmemPerSm - kSmemPerCtaReserved) return UNISVQ_ERR_UNSUPPORTED;
     const void* xs = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * L->K;
     void* ys = static_cast<uint16_t*>(y) + static_cast<size_t>(m0) * L->N;
-    const unisvq_status st = p.nt == 1 ? gemv_launch_nt<1>(L, p, xs, ys, mc, s) : gemv_launch_nt<2>(L, p, xs, ys, mc, s);
+    const unisvq_status st =
+        p.nt == 1 ? gemv_launch_nt<1>(L, p, xs, ys, mc, s) : gemv_launch_nt<2>(L, p, xs, ys, mc, s);
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;

@@ -16,23 +16,23 @@ void pack_codes_host(const uint8_t* codes, int N, int K, uint8_t* packed) {
   for (int rb = 0; rb < RB; ++rb) {
     for (int kt = 0; kt < KT; ++kt) {
       uint8_t* tile = packed + (static_cast<size_t>(rb) * KT + kt) * kTileBytes;
-      for (int h = 0; h < 2; ++h) {
-        for (int r = 0; r < kTileRows; ++r) {
-          const int row = rb * kTileRows + r;
-          const uint8_t* cr = row < N ? codes + static_cast<size_t>(row) * K : nullptr;
-          uint8_t* dst = tile + tile_row_offset(r, h);
-          for (int wi = 0; wi < 4; ++wi) {
+      for (int r = 0; r < kTileRows; ++r) {
+        const int row = rb * kTileRows + r;
+        const uint8_t* cr = row < N ? codes + static_cast<size_t>(row) * K : nullptr;
+        for (int h = 0; h < 2; ++h) {
+          for (int t = 0; t < 4; ++t) {
             uint32_t w = 0;
             for (int s = 0; s < 4; ++s)
               for (int b = 0; b < 4; ++b) {
-                const int k = kt * kTileCols + 64 * h + 16 * wi + 4 * s + b;
+                const int k = kt * kTileCols + 64 * h + 16 * t + 4 * s + b;
                 const uint32_t z = (cr && k < K) ? (cr[k] & 3u) : 0u;
                 w |= z << (8 * b + 2 * s);
               }
-            dst[4 * wi + 0] = static_cast<uint8_t>(w);
-            dst[4 * wi + 1] = static_cast<uint8_t>(w >> 8);
-            dst[4 * wi + 2] = static_cast<uint8_t>(w >> 16);
-            dst[4 * wi + 3] = static_cast<uint8_t>(w >> 24);
+            uint8_t* dst = tile + tile_word_offset(r, h, t);
+            dst[0] = static_cast<uint8_t>(w);
+            dst[1] = static_cast<uint8_t>(w >> 8);
+            dst[2] = static_cast<uint8_t>(w >> 16);
+            dst[3] = static_cast<uint8_t>(w >> 24);
           }
         }
       }

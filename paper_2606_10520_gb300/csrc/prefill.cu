@@ -10,8 +10,8 @@
 // Roles of the 14 warps of a CTA (persistent over tiles):
 //   warp 0        TMA producer: x tile [BN x 64] per k-block, and TMEM owner
 //   warp 1        MMA issuer (one thread): 4 x tcgen05.mma (K = 16) per k-block
-//   warps 2..9    converters: one row per lane, half of each 128-byte swizzled
-//                 row per warp; every d-vector index selects its exact bf16
+//   warps 2..9    converters: one 16-row unit per warp, two rows x 16 columns
+//                 per lane; every d-vector index selects its exact bf16
 //                 codeword RN(A z + B) from a pack-time table
 //   warps 10..13  epilogue: tcgen05.ld of the accumulator, bf16, global store
 // The accumulator is double-buffered in TMEM so the epilogue of one tile runs
@@ -261,21 +261,20 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     }
   } else if (warp < kEpiWarp0) {
     // ---------------- converters: codes -> bf16 codeword tile ----------------
-    // Warp c covers rows 32 (c % 4) .. +31 (one row per lane) and the 16-byte
-    // chunks 4 (c / 4) .. +3 of each 64-column stage.
+    // Warp c covers unit c (rows 16c .. 16c+15): lane 4g + t reads the 8-byte
+    // pair of words of rows 16c + g and 16c + g + 8 for column quarter t of the
+    // stage's half (layout.h) and writes their 16 columns of each row.
     const int c = warp - kConvWarp0;
-    const int r = 32 * (c & 3) + lane;          // row within the 128-row tile
-    const int ch = c >> 2;
+    const int g = lane >> 2, t = lane & 3;
+    const int r0 = 16 * c + g, r1 = r0 + 8;
     const uint32_t lut_s = sbase + C::kOffLut;
-    const int sw = r & 7;
     int it = 0;
     for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
       const int n_blk = tile / a.mtiles;
-      const uint8_t* rbase = a.codes + static_cast<size_t>(n_blk) * a.KT * kTileBytes + r * 16 + 8 * ch;
+      const uint8_t* rbase = a.codes + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
       // Code words of stage kb live at tile kb/2, half kb%2; prefetched 3 stages ahead.
       auto load = [&](int kb) -> uint2 {
-        return kb < a.nkb ? __ldg(reinterpret_cast<const uint2*>(rbase + (kb >> 1) * kTileBytes +
-                                                                 (kb & 1) * kHalfBytes))
+        return kb < a.nkb ? __ldg(reinterpret_cast<const uint2*>(rbase + (kb >> 1) * kTileBytes + (kb & 1) * 8))
                           : make_uint2(0, 0);
       };
       uint2 q0 = load(0), q1 = load(1), q2 = load(2);
@@ -291,26 +290,30 @@ __global__ void __launch_bounds__(kPfThreads, 1)
           if (!ok) *abort_flag = 1;
         }
         if (ok) {
-          const uint32_t row_addr = sbase + C::kOffA + s * kATileBytes + r * 128;
+          const uint32_t tile_addr = sbase + C::kOffA + s * kATileBytes;
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const int cc = 4 * ch + j;                      // chunk: columns 8cc .. 8cc+7
-            const uint32_t w = (j < 2) ? cw.x : cw.y;
-            const uint32_t e0 = extract4(w, 2 * (j & 1));   // columns 8cc .. 8cc+3
-            const uint32_t e1 = extract4(w, 2 * (j & 1) + 1);
-            uint32_t o0, o1, o2, o3;
-            if (a.d == 4) {
-              const uint32_t i0 = (e0 & 3u) | ((e0 >> 6) & 0xCu) | ((e0 >> 12) & 0x30u) | ((e0 >> 18) & 0xC0u);
-              const uint32_t i1 = (e1 & 3u) | ((e1 >> 6) & 0xCu) | ((e1 >> 12) & 0x30u) | ((e1 >> 18) & 0xC0u);
-              const uint2 v0 = lds64(lut_s + i0 * 8), v1 = lds64(lut_s + i1 * 8);
-              o0 = v0.x; o1 = v0.y; o2 = v1.x; o3 = v1.y;
-            } else {
-              o0 = lds32(lut_s + (((e0 & 3u) | ((e0 >> 6) & 0xCu)) << 2));
-              o1 = lds32(lut_s + ((((e0 >> 16) & 3u) | ((e0 >> 22) & 0xCu)) << 2));
-              o2 = lds32(lut_s + (((e1 & 3u) | ((e1 >> 6) & 0xCu)) << 2));
-              o3 = lds32(lut_s + ((((e1 >> 16) & 3u) | ((e1 >> 22) & 0xCu)) << 2));
+          for (int q = 0; q < 2; ++q) {
+            const uint32_t w = q ? cw.y : cw.x;
+            const uint32_t row_addr = tile_addr + (q ? r1 : r0) * 128;
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const int cc = 2 * t + e;                       // chunk: stage columns 8cc .. 8cc+7
+              const uint32_t e0 = extract4(w, 2 * e);         // columns 8cc .. 8cc+3
+              const uint32_t e1 = extract4(w, 2 * e + 1);     // columns 8cc+4 .. 8cc+7
+              uint32_t o0, o1, o2, o3;
+              if (a.d == 4) {
+                const uint32_t i0 = (e0 & 3u) | ((e0 >> 6) & 0xCu) | ((e0 >> 12) & 0x30u) | ((e0 >> 18) & 0xC0u);
+                const uint32_t i1 = (e1 & 3u) | ((e1 >> 6) & 0xCu) | ((e1 >> 12) & 0x30u) | ((e1 >> 18) & 0xC0u);
+                const uint2 v0 = lds64(lut_s + i0 * 8), v1 = lds64(lut_s + i1 * 8);
+                o0 = v0.x; o1 = v0.y; o2 = v1.x; o3 = v1.y;
+              } else {
+                o0 = lds32(lut_s + (((e0 & 3u) | ((e0 >> 6) & 0xCu)) << 2));
+                o1 = lds32(lut_s + ((((e0 >> 16) & 3u) | ((e0 >> 22) & 0xCu)) << 2));
+                o2 = lds32(lut_s + (((e1 & 3u) | ((e1 >> 6) & 0xCu)) << 2));
+                o3 = lds32(lut_s + ((((e1 >> 16) & 3u) | ((e1 >> 22) & 0xCu)) << 2));
+              }
+              sts128(row_addr + ((cc ^ g) << 4), o0, o1, o2, o3);
             }
-            sts128(row_addr + ((cc ^ sw) << 4), o0, o1, o2, o3);
           }
           fence_proxy_async_smem();
         }

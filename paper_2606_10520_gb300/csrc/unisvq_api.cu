@@ -240,7 +240,7 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
   return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess) ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
-static int decode_kernel_for(int M) { return M <= 8 ? UNISVQ_KERNEL_GEMV : UNISVQ_KERNEL_SKINNY; }
+static int decode_kernel_for(int M) { return M <= 16 ? UNISVQ_KERNEL_GEMV : UNISVQ_KERNEL_SKINNY; }
 
 static int auto_kernel(const unisvq_layer* L, int M) {
   if (M > 64 && prefill_supported(L, M)) return UNISVQ_KERNEL_PREFILL;

@@ -30,18 +30,22 @@ def decode_layout(packed: np.ndarray, N: int, K: int) -> np.ndarray:
     Np = -(-N // 128) * 128
     Kp = -(-K // 128) * 128
     KT = Kp // 128
-    words = packed.view("<u4").reshape(Np // 128, KT, 2, 128, 4)   # [rb][kt][h][r][wi]
+    # word (rb, kt, u, g, t, slot) with slot = 2h + q holds row 128rb + 16u + 8q + g
+    words = packed.view("<u4").reshape(Np // 128, KT, 8, 8, 4, 4)
     out = np.full((Np, Kp), 255, dtype=np.int64)
     for rb in range(Np // 128):
         for kt in range(KT):
-            for h in range(2):
-                for r in range(128):
-                    for wi in range(4):
-                        w = int(words[rb, kt, h, r, wi])
-                        for s in range(4):
-                            for b in range(4):
-                                k = 128 * kt + 64 * h + 16 * wi + 4 * s + b
-                                out[128 * rb + r, k] = (w >> (8 * b + 2 * s)) & 3
+            for u in range(8):
+                for g in range(8):
+                    for t in range(4):
+                        for slot in range(4):
+                            h, q = slot >> 1, slot & 1
+                            r = 128 * rb + 16 * u + 8 * q + g
+                            w = int(words[rb, kt, u, g, t, slot])
+                            for s in range(4):
+                                for b in range(4):
+                                    k = 128 * kt + 64 * h + 16 * t + 4 * s + b
+                                    out[r, k] = (w >> (8 * b + 2 * s)) & 3
     return out
 
 
