@@ -40,6 +40,8 @@ import synth  # noqa: E402
 
 METRIC = "UniSVQ linear: GEMV HBM GB/s (% of ~8 TB/s); prefill TFLOPS (% of bf16 peak)"
 M_SWEEP = (1, 2, 4, 8, 16)
+# Projections of the Llama-2-7B set (synth.LLAMA2_7B order) that share an input.
+GROUPS_7B = [[0, 1, 2], [3], [4, 5], [6]]
 PREFILL_M = 2048
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
@@ -215,6 +217,9 @@ def workload_config(args):
             "layers": args.layers, "d": 2, "m_sweep": list(M_SWEEP),
             "l2": "inputs larger than L2 (1.62 GB of packed codes per pass at 32 layers)",
             "timing": "CUDA graphs of the full layer stack per M, CUDA events on the capture stream",
+            "calls": ("one unisvq_linear per projection (7 per layer)" if getattr(args, "ungrouped", False) else
+                      "q/k/v and gate/up as one unisvq_linear_group call each (shared input), o and down "
+                      "as unisvq_linear: 4 calls per layer"),
             "parallelism": "replicas"}
 
 
@@ -269,24 +274,36 @@ def run_ours(args, rank, world, local_rank):
     shapes = synth.LLAMA2_7B
     stack = build_stack(binding, shapes, args.layers, 1)
 
+    # Projections that read the same input are issued as one grouped call
+    # (q, k, v and gate, up), as a decode step issues them; --ungrouped makes
+    # one unisvq_linear call per projection.
+    groups = [[i] for i in range(len(shapes))] if args.ungrouped else GROUPS_7B
     xs, ys, graphs, step_bytes, launches = {}, {}, [], 0, 0
     for M in M_SWEEP:
-        for _, N, K in shapes:
+        for pi, (_, N, K) in enumerate(shapes):
             if (M, K) not in xs:
                 xb = synth.activations(0, 1, 100 + M, M, K)
                 xs[(M, K)] = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).cuda()
-            if (M, N) not in ys:
-                ys[(M, N)] = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+            ys[(M, pi)] = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+
+    def issue(layer, grp, M, sp):
+        K = shapes[grp[0]][2]
+        if len(grp) == 1:
+            st = layer[grp[0]].forward_ptr(xs[(M, K)].data_ptr(), ys[(M, grp[0])].data_ptr(), M, sp,
+                                           binding.KERNEL_AUTO)
+        else:
+            st = binding.linear_group_ptr([layer[i] for i in grp], xs[(M, K)].data_ptr(),
+                                          [ys[(M, i)].data_ptr() for i in grp], M, sp)
+        if st != 0:
+            raise RuntimeError(f"unisvq call failed: {binding.status_string(st)}")
+
     side = torch.cuda.Stream()
     for M in M_SWEEP:
         def one_pass(M=M):
             sp = torch.cuda.current_stream().cuda_stream
             for layer in stack:
-                for (_, N, K), h in zip(shapes, layer):
-                    st = h.forward_ptr(xs[(M, K)].data_ptr(), ys[(M, N)].data_ptr(), M, sp,
-                                       binding.KERNEL_DECODE)
-                    if st != 0:
-                        raise RuntimeError(f"unisvq_linear failed: {binding.status_string(st)}")
+                for grp in groups:
+                    issue(layer, grp, M, sp)
         with torch.cuda.stream(side):
             one_pass()
         torch.cuda.synchronize()
@@ -295,9 +312,9 @@ def run_ours(args, rank, world, local_rank):
             one_pass()
         graphs.append(g)
         for layer in stack:
-            for (_, N, K), h in zip(shapes, layer):
+            for _, N, K in shapes:
                 step_bytes += algo_bytes(N, K, M)
-                launches += 1
+            launches += len(groups) * ((M + 15) // 16)
     torch.cuda.synchronize()
     st = binding.sync_status()
     if st != 0:
@@ -345,13 +362,12 @@ def run_ours(args, rank, world, local_rank):
             def e2e_pass(M=M):
                 sp = torch.cuda.current_stream().cuda_stream
                 for layer in stack:
-                    for (_, N, K), h in zip(shapes, layer):
+                    for grp in groups:
+                        K = shapes[grp[0]][2]
                         xs[(M, K)].copy_(hx[(M, K)], non_blocking=True)
-                        st = h.forward_ptr(xs[(M, K)].data_ptr(), ys[(M, N)].data_ptr(), M, sp,
-                                           binding.KERNEL_DECODE)
-                        if st != 0:
-                            raise RuntimeError(binding.status_string(st))
-                        hy[(M, N)].copy_(ys[(M, N)], non_blocking=True)
+                        issue(layer, grp, M, sp)
+                        for i in grp:
+                            hy[(M, i)].copy_(ys[(M, i)], non_blocking=True)
             with torch.cuda.stream(side):
                 e2e_pass()
             torch.cuda.synchronize()
@@ -359,14 +375,15 @@ def run_ours(args, rank, world, local_rank):
             with torch.cuda.graph(g, stream=side):
                 e2e_pass()
             egraphs.append(g)
-            for _, N, K in shapes:
-                h2d += 2 * M * K * args.layers
-                d2h += 2 * M * N * args.layers
+            for grp in groups:
+                h2d += 2 * M * shapes[grp[0]][2] * args.layers
+                for i in grp:
+                    d2h += 2 * M * shapes[i][1] * args.layers
         te = time_graphs(torch, egraphs, args.steps, args.warmup, side)
         e2e = {"value": step_bytes * args.steps * world / te / 1e9, "unit": "GB/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-               "how": "per layer call: pinned-host x -> device copy, unisvq_linear, device -> pinned-host y; "
-                      "the whole sweep replayed from CUDA graphs"}
+               "how": "per call: pinned-host x -> device copy, the library call, device -> pinned-host y "
+                      "of every projection; the whole sweep replayed from CUDA graphs"}
 
     # ---- prefill (tcgen05 GEMM), Llama-3-8B-shaped set at M = 2048 -------
     prefill = None
@@ -486,6 +503,8 @@ def main():
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--ungrouped", action="store_true",
+                    help="one unisvq_linear call per projection instead of grouped calls for q/k/v and gate/up")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--only", choices=["decode", "prefill"], default=None,
                     help="profiling aid: run only the decode sweep (no e2e/cpu/prefill) or only the prefill set")

@@ -127,6 +127,27 @@ unisvq_status unisvq_linear(unisvq_handle h, const void* x, void* y, int M, void
 unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, void* y, int M,
                                   void* stream);
 
+/*
+ * y_i = x W_hat_i^T for n layers that read the same x (Eq. def:ptq_loss for
+ * each layer, with its own codes and its own A, B of Eq. col:dequant), e.g.
+ * the q, k, v projections or the gate and up projections of one transformer
+ * block. The paper defines the layer, not this grouping; it is a launch
+ * convenience: for M <= 16 all n layers run in one kernel launch (the row
+ * blocks of the layers side by side), otherwise one unisvq_linear per layer.
+ *   hs : n handles on the current device, all with the same K
+ *   n  : 1 .. UNISVQ_MAX_GROUP
+ *   x  : device, [M][K] bf16, 16-byte aligned (shared by all layers)
+ *   ys : host array of n device pointers, ys[i] is [M][N_i] bf16, 4-byte
+ *        aligned; no y may overlap x or another y
+ * Results equal those of n unisvq_linear calls up to the order of the fp32
+ * partial sums. Never allocates and never synchronises.
+ * Errors: INVALID_ARG (null, n out of range, K mismatch, device mismatch,
+ * misaligned, overlap, M < 0), UNSUPPORTED, CUDA.
+ */
+#define UNISVQ_MAX_GROUP 4
+unisvq_status unisvq_linear_group(const unisvq_handle* hs, int n, const void* x, void* const* ys, int M,
+                                  void* stream);
+
 /* Test hook: writes W_hat as fp32 [N][K] row-major to device memory W (each
  * entry RN_fp32 of the exact A z + B), unpacking the device layout with the
  * same code-extraction helpers the layer kernels use. */

@@ -21,7 +21,9 @@ EXPORTS = [
     "unisvq_pack", "unisvq_linear", "unisvq_linear_force", "unisvq_dequant_debug",
     "unisvq_query", "unisvq_sync_status", "unisvq_destroy", "unisvq_clone",
     "unisvq_status_string", "unisvq_packed_code_bytes", "unisvq_pack_host", "unisvq_version",
+    "unisvq_linear_group",
 ]
+MAX_GROUP = 4
 
 
 class UnisvqError(RuntimeError):
@@ -53,6 +55,7 @@ def load():
     lib.unisvq_pack.argtypes = [vp, vp, vp, i, i, i, vp, ctypes.POINTER(vp)]
     lib.unisvq_linear.argtypes = [vp, vp, vp, i, vp]
     lib.unisvq_linear_force.argtypes = [vp, i, vp, vp, i, vp]
+    lib.unisvq_linear_group.argtypes = [vp, i, vp, vp, i, vp]
     lib.unisvq_dequant_debug.argtypes = [vp, vp, vp]
     lib.unisvq_query.argtypes = [vp, i, ctypes.POINTER(Info)]
     lib.unisvq_sync_status.argtypes = [vp]
@@ -177,3 +180,25 @@ class UniSVQLinear:
             self.close()
         except Exception:
             pass
+
+
+def linear_group_ptr(layers, x_ptr: int, y_ptrs, M: int, stream_ptr: int) -> int:
+    """Raw-pointer unisvq_linear_group over `layers` (same K); returns the status."""
+    n = len(layers)
+    hs = (ctypes.c_void_p * n)(*[l._h.value if isinstance(l._h, ctypes.c_void_p) else l._h for l in layers])
+    ys = (ctypes.c_void_p * n)(*[int(p) for p in y_ptrs])
+    return load().unisvq_linear_group(hs, n, ctypes.c_void_p(x_ptr), ys, M, ctypes.c_void_p(stream_ptr))
+
+
+def linear_group(layers, x, outs=None, stream=None):
+    """y_i = x W_hat_i^T for layers that share x ([M][K] bf16 CUDA tensor)."""
+    import torch
+    if x.dtype != torch.bfloat16 or not x.is_cuda or x.dim() != 2:
+        raise ValueError("x must be a CUDA bf16 tensor of shape [M, K]")
+    x = x.contiguous()
+    M = x.shape[0]
+    if outs is None:
+        outs = [torch.empty((M, l.N), dtype=torch.bfloat16, device=x.device) for l in layers]
+    _check(linear_group_ptr(layers, x.data_ptr(), [o.data_ptr() for o in outs], M,
+                            _stream_ptr(stream).value or 0), "unisvq_linear_group")
+    return outs

@@ -36,24 +36,34 @@ constexpr int kGThreads = kGWarps * 32;
 constexpr int kGDepth = 8;          // k-tiles of codes in flight per warp (16 bytes per lane each)
 constexpr int kMaxSplit = 8;        // K slices per row block (cluster size)
 constexpr int kGMaxTok = 16;
+constexpr int kMaxGroup = UNISVQ_MAX_GROUP;   // layers per launch
 constexpr int kXLoads = 4;          // 16-byte activation loads in flight per lane (fold)
 constexpr int kXPad = 4;            // fp16 elements of padding per token row (bank spread)
 constexpr int kTokBytes = 160;      // pexp[16], cpart[16], reduction mbarrier
 constexpr size_t kSmemPerSm = 228 * 1024;
 constexpr size_t kSmemPerCtaReserved = 1024;
 
-struct GemvArgs {
+// One layer of a launch. A launch covers one layer, or several layers that
+// read the same x (same K): their row blocks are stacked along grid.y.
+struct GemvLayer {
   const uint8_t* codes;
-  const uint16_t* x;   // bf16 [M][K]
   uint16_t* y;         // bf16 [M][N]
-  int M, N, K, KT, d;
+  int N, d;
+  int rb0;             // first grid.y row block of this layer
+  float colnorm;
+  float A[16];
+  float B[4];
+};
+
+struct GemvArgs {
+  const uint16_t* x;   // bf16 [M][K]
+  int M, K, KT;
   int kt_per_cta;
   int xstride;         // fp16 elements per token row of the folded slice
   int off_red, off_tok;
-  float A[16];
-  float B[4];
-  float colnorm;
+  int nlayers;
   int* err;
+  GemvLayer layer[kMaxGroup];
 };
 
 __device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
@@ -65,30 +75,45 @@ __device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b.x), "r"(b.y));
 }
 
-__device__ __forceinline__ uint2 lds64(uint32_t addr) {
-  uint2 v;
-  asm volatile("ld.shared.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
-  return v;
-}
-__device__ __forceinline__ void sts64(uint32_t addr, uint32_t a, uint32_t b) {
-  asm volatile("st.shared.v2.u32 [%0], {%1,%2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
-}
-
 // x'[c .. c+3] for the d-vectors inside x[c .. c+3] (c % 4 == 0): row vector x_g A.
-__device__ __forceinline__ void gfold4(const GemvArgs& a, const float (&v)[4], float (&o)[4]) {
-  if (a.d == 1) {
+// A is a register copy of the kernel parameter (reading the parameter through a
+// reference inside a lambda turns every access into a slow generic load).
+__device__ __forceinline__ void gfold4(int d, const float (&A)[16], const float (&v)[4], float (&o)[4]) {
+  if (d == 1) {
 #pragma unroll
-    for (int e = 0; e < 4; ++e) o[e] = v[e] * a.A[0];
-  } else if (a.d == 2) {
-    o[0] = fmaf(v[1], a.A[2], v[0] * a.A[0]);
-    o[1] = fmaf(v[1], a.A[3], v[0] * a.A[1]);
-    o[2] = fmaf(v[3], a.A[2], v[2] * a.A[0]);
-    o[3] = fmaf(v[3], a.A[3], v[2] * a.A[1]);
+    for (int e = 0; e < 4; ++e) o[e] = v[e] * A[0];
+  } else if (d == 2) {
+    o[0] = fmaf(v[1], A[2], v[0] * A[0]);
+    o[1] = fmaf(v[1], A[3], v[0] * A[1]);
+    o[2] = fmaf(v[3], A[2], v[2] * A[0]);
+    o[3] = fmaf(v[3], A[3], v[2] * A[1]);
   } else {
 #pragma unroll
     for (int c = 0; c < 4; ++c)
-      o[c] = fmaf(v[3], a.A[12 + c], fmaf(v[2], a.A[8 + c], fmaf(v[1], a.A[4 + c], v[0] * a.A[c])));
+      o[c] = fmaf(v[3], A[12 + c], fmaf(v[2], A[8 + c], fmaf(v[1], A[4 + c], v[0] * A[c])));
   }
+}
+
+// Columns 8ci .. 8ci+7 of a token's slice (packed bf16 xv) -> their B fragments:
+// four-column groups j0 = 2ci mod 4 and j0 + 1, scaled by 2^(pe - 2j).
+__device__ __forceinline__ uint4 fold8(int ci, uint4 xv, int pe, int d, const float (&A)[16]) {
+  const int j0 = (2 * ci) & 3;
+  const float v0[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
+  const float v1[4] = {bf16_lo(xv.z), bf16_hi(xv.z), bf16_lo(xv.w), bf16_hi(xv.w)};
+  float o0[4], o1[4];
+  gfold4(d, A, v0, o0);
+  gfold4(d, A, v1, o1);
+  const float s0 = exp2i(pe - 2 * j0), s1 = exp2i(pe - 2 * j0 - 2);
+  return make_uint4(pack_half2(o0[0] * s0, o0[2] * s0), pack_half2(o0[1] * s0, o0[3] * s0),
+                    pack_half2(o1[0] * s1, o1[2] * s1), pack_half2(o1[1] * s1, o1[3] * s1));
+}
+
+// 2^P with P = 15 - e, e the binary exponent of bound in [2^(e-1), 2^e): puts
+// the largest possible |x'| (<= bound) below 2^15, the fp16 range.
+__device__ __forceinline__ int token_scale_exp(float bound) {
+  if (!(bound > 0.f)) return 0;
+  const int e = static_cast<int>(__float_as_uint(bound) >> 23) - 126;
+  return max(-100, min(100, 15 - e));
 }
 
 // Eight activations x[k .. k+7] of one token as packed bf16 (zero at or past kend).
@@ -108,8 +133,34 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   const int KS = gridDim.x;
   const int kt0 = blockIdx.x * a.kt_per_cta;
   const int n_kt = min(a.kt_per_cta, a.KT - kt0);
-  const int rb = blockIdx.y;
   const int M = a.M;
+  // This CTA's layer, read with constant parameter offsets only.
+  int li = 0;
+#pragma unroll
+  for (int i = 1; i < kMaxGroup; ++i)
+    if (i < a.nlayers && static_cast<int>(blockIdx.y) >= a.layer[i].rb0) li = i;
+  const uint8_t* codes = nullptr;
+  uint16_t* yout = nullptr;
+  int N = 0, d = 1, rb = 0;
+  float colnorm = 0.f, Areg[16], Bq[4];
+#pragma unroll
+  for (int i = 0; i < kMaxGroup; ++i) {
+    if (i == li) {
+      codes = a.layer[i].codes;
+      yout = a.layer[i].y;
+      N = a.layer[i].N;
+      d = a.layer[i].d;
+      rb = static_cast<int>(blockIdx.y) - a.layer[i].rb0;
+      colnorm = a.layer[i].colnorm;
+#pragma unroll
+      for (int e = 0; e < 16; ++e) Areg[e] = a.layer[i].A[e];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) Bq[e] = a.layer[i].B[e];
+    }
+  }
+  float Bcol[8];   // B[e mod d] for column e of an 8-column chunk
+#pragma unroll
+  for (int e = 0; e < 8; ++e) Bcol[e] = d == 1 ? Bq[0] : (d == 2 ? Bq[e & 1] : Bq[e & 3]);
   // Rows whose K-slice partial sums this CTA adds up (it "owns" them).
   const int rows_per = (kTileRows + KS - 1) / KS;
   const int own0 = static_cast<int>(blockIdx.x) * rows_per;
@@ -137,7 +188,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   // ---- codes: unit `warp` (rows 16 warp .. +15) of every k-tile of the slice ----
   const int g = lane >> 2, t = lane & 3;
   const uint8_t* cbase =
-      a.codes + (static_cast<size_t>(rb) * a.KT + kt0) * kTileBytes + warp * kUnitBytes + lane * 16;
+      codes + (static_cast<size_t>(rb) * a.KT + kt0) * kTileBytes + warp * kUnitBytes + lane * 16;
   uint4 cw[kGDepth];
 #pragma unroll
   for (int s = 0; s < kGDepth; ++s)
@@ -158,7 +209,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   const uint32_t xrow_bytes = static_cast<uint32_t>(a.xstride) * 2u;
   for (int tk = warp; tk < M; tk += kGWarps) {
     const uint16_t* row = a.x + static_cast<size_t>(tk) * a.K;
-    const uint32_t xrow = sbase + tk * xrow_bytes;
+    uint8_t* xrow = smem + tk * xrow_bytes;
     float mx = 0.f, cs = 0.f;
     uint4 u[kXLoads];
     for (int c0 = lane; c0 < nch; c0 += 32 * kXLoads) {
@@ -171,15 +222,17 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
       for (int j = 0; j < kXLoads; ++j) {
         const int ci = c0 + 32 * j;
         if (ci < nch) {
-          sts64(xrow + 16u * ci, u[j].x, u[j].y);
-          sts64(xrow + 16u * ci + 8, u[j].z, u[j].w);
+          if (nch > 32 * kXLoads) {   // staged for the second pass
+            *reinterpret_cast<uint2*>(xrow + 16u * ci) = make_uint2(u[j].x, u[j].y);
+            *reinterpret_cast<uint2*>(xrow + 16u * ci + 8) = make_uint2(u[j].z, u[j].w);
+          }
           const uint32_t w4[4] = {u[j].x, u[j].y, u[j].z, u[j].w};
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const float v0 = bf16_lo(w4[q]), v1 = bf16_hi(w4[q]);
             mx = fmaxf(mx, fmaxf(fabsf(v0), fabsf(v1)));
-            cs = fmaf(v0, a.B[(2 * q) & (a.d - 1)], cs);
-            cs = fmaf(v1, a.B[(2 * q + 1) & (a.d - 1)], cs);
+            cs = fmaf(v0, Bcol[2 * q], cs);
+            cs = fmaf(v1, Bcol[2 * q + 1], cs);
           }
         }
       }
@@ -189,31 +242,24 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
       cs += __shfl_xor_sync(0xffffffffu, cs, off);
     }
-    const float bound = mx * a.colnorm;
-    int e2 = 0;
-    if (bound > 0.f) frexpf(bound, &e2);
-    const int pe = bound > 0.f ? max(-100, min(100, 15 - e2)) : 0;
+    const int pe = token_scale_exp(mx * colnorm);
     if (lane == 0) {
       pexp[tk] = pe;
       cpart[tk] = cs;
     }
-    auto fold8 = [&](int ci, uint4 xv) {
-      // columns 8ci .. 8ci+7 of the slice: four-column groups j0 and j0 + 1
-      const int j0 = (2 * ci) & 3;
-      const float v0[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
-      const float v1[4] = {bf16_lo(xv.z), bf16_hi(xv.z), bf16_lo(xv.w), bf16_hi(xv.w)};
-      float o0[4], o1[4];
-      gfold4(a, v0, o0);
-      gfold4(a, v1, o1);
-      const float s0 = exp2i(pe - 2 * j0), s1 = exp2i(pe - 2 * j0 - 2);
-      sts64(xrow + 16u * ci, pack_half2(o0[0] * s0, o0[2] * s0), pack_half2(o0[1] * s0, o0[3] * s0));
-      sts64(xrow + 16u * ci + 8, pack_half2(o1[0] * s1, o1[2] * s1), pack_half2(o1[1] * s1, o1[3] * s1));
-    };
     if (nch <= 32 * kXLoads) {
-      // the whole slice is still in registers
+      // the whole slice is still in registers: fold, then store
+      uint4 f[kXLoads];
 #pragma unroll
-      for (int j = 0; j < kXLoads; ++j)
-        if (lane + 32 * j < nch) fold8(lane + 32 * j, u[j]);
+      for (int j = 0; j < kXLoads; ++j) f[j] = fold8(lane + 32 * j, u[j], pe, d, Areg);
+#pragma unroll
+      for (int j = 0; j < kXLoads; ++j) {
+        const int ci = lane + 32 * j;
+        if (ci < nch) {
+          *reinterpret_cast<uint2*>(xrow + 16u * ci) = make_uint2(f[j].x, f[j].y);
+          *reinterpret_cast<uint2*>(xrow + 16u * ci + 8) = make_uint2(f[j].z, f[j].w);
+        }
+      }
     } else {
       // every lane re-reads only the chunks it staged itself
       for (int c0 = lane; c0 < nch; c0 += 32 * kXLoads) {
@@ -221,13 +267,19 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
         for (int j = 0; j < kXLoads; ++j) {
           const int ci = c0 + 32 * j;
           if (ci < nch) {
-            const uint2 lo = lds64(xrow + 16u * ci), hi = lds64(xrow + 16u * ci + 8);
-            u[j] = make_uint4(lo.x, lo.y, hi.x, hi.y);
+            const uint2 lo = *reinterpret_cast<const uint2*>(xrow + 16u * ci);
+            const uint2 hi = *reinterpret_cast<const uint2*>(xrow + 16u * ci + 8);
+            u[j] = fold8(ci, make_uint4(lo.x, lo.y, hi.x, hi.y), pe, d, Areg);
           }
         }
 #pragma unroll
-        for (int j = 0; j < kXLoads; ++j)
-          if (c0 + 32 * j < nch) fold8(c0 + 32 * j, u[j]);
+        for (int j = 0; j < kXLoads; ++j) {
+          const int ci = c0 + 32 * j;
+          if (ci < nch) {
+            *reinterpret_cast<uint2*>(xrow + 16u * ci) = make_uint2(u[j].x, u[j].y);
+            *reinterpret_cast<uint2*>(xrow + 16u * ci + 8) = make_uint2(u[j].z, u[j].w);
+          }
+        }
       }
     }
   }
@@ -283,30 +335,41 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   constexpr int MP = 8 * NT;
   const uint32_t red_addr = sbase + a.off_red;
   if (KS > 1) cluster_wait();   // every CTA of the cluster has initialised its barrier
+  float pv[NT][2][2];
 #pragma unroll
-  for (int nt = 0; nt < NT; ++nt)
+  for (int nt = 0; nt < NT; ++nt) {
+    const int tok = 8 * nt + 2 * t;   // this lane holds tokens tok and tok + 1
+    const float sc0 = tok < M ? exp2i(24 - pexp[tok]) : 0.f, c0v = tok < M ? cpart[tok] : 0.f;
+    const float sc1 = tok + 1 < M ? exp2i(24 - pexp[tok + 1]) : 0.f, c1v = tok + 1 < M ? cpart[tok + 1] : 0.f;
 #pragma unroll
     for (int rh = 0; rh < 2; ++rh) {
-      const int row = 16 * warp + g + 8 * rh;
-      const int tok = 8 * nt + 2 * t;   // this lane holds tokens tok and tok + 1
+      pv[nt][rh][0] = fmaf(acc[0][nt][2 * rh] + acc[1][nt][2 * rh], sc0, c0v);
+      pv[nt][rh][1] = fmaf(acc[0][nt][2 * rh + 1] + acc[1][nt][2 * rh + 1], sc1, c1v);
+    }
+  }
+#pragma unroll
+  for (int rh = 0; rh < 2; ++rh) {
+    const int row = 16 * warp + g + 8 * rh;
+    const int owner = row / rows_per;
+    const uint32_t row_off = (static_cast<uint32_t>(blockIdx.x) * rows_per + (row - owner * rows_per)) * MP;
+    const bool local = owner == static_cast<int>(blockIdx.x);
+    const uint32_t rbar = local ? 0u : map_shared_rank(red_bar, owner);
+    const uint32_t rslot = local ? 0u : map_shared_rank(red_addr + row_off * 4u, owner);
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      const int tok = 8 * nt + 2 * t;
       if (tok < M) {
-        const float v0 = fmaf(acc[0][nt][2 * rh] + acc[1][nt][2 * rh], exp2i(24 - pexp[tok]), cpart[tok]);
-        const float v1 = tok + 1 < M ? fmaf(acc[0][nt][2 * rh + 1] + acc[1][nt][2 * rh + 1],
-                                            exp2i(24 - pexp[tok + 1]), cpart[tok + 1])
-                                     : 0.f;
-        const int owner = row / rows_per;
-        const uint32_t off =
-            ((static_cast<uint32_t>(blockIdx.x) * rows_per + (row - owner * rows_per)) * MP + tok) * 4u;
-        if (owner == static_cast<int>(blockIdx.x)) {
-          red[off / 4] = v0;
-          if (tok + 1 < M) red[off / 4 + 1] = v1;
+        if (local) {
+          red[row_off + tok] = pv[nt][rh][0];
+          if (tok + 1 < M) red[row_off + tok + 1] = pv[nt][rh][1];
         } else if (tok + 1 < M) {
-          st_async_v2f32(map_shared_rank(red_addr + off, owner), v0, v1, map_shared_rank(red_bar, owner));
+          st_async_v2f32(rslot + tok * 4u, pv[nt][rh][0], pv[nt][rh][1], rbar);
         } else {
-          st_async_f32(map_shared_rank(red_addr + off, owner), v0, map_shared_rank(red_bar, owner));
+          st_async_f32(rslot + tok * 4u, pv[nt][rh][0], rbar);
         }
       }
     }
+  }
 
   // ---- reduction over the K slices of the row block ----
   __syncthreads();   // this CTA's own slots
@@ -321,7 +384,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
     float sum = 0.f;
 #pragma unroll
     for (int q = 0; q < kMaxSplit; ++q) sum += v[q];
-    if (n < a.N) a.y[static_cast<size_t>(tok) * a.N + n] = f32_to_bf16_rn(sum);
+    if (n < N) yout[static_cast<size_t>(tok) * N + n] = f32_to_bf16_rn(sum);
   }
 }
 
@@ -342,16 +405,11 @@ GemvShape gemv_shape(int M, int kt_per_cta, int ks, int nt) {
   return s;
 }
 
-int gemv_ctas_per_sm(size_t smem) {
-  const int by_smem = static_cast<int>(kSmemPerSm / (smem + kSmemPerCtaReserved));
-  return by_smem < 2 ? by_smem : 2;   // registers allow two 256-thread CTAs
-}
-
 template <int NT>
-unisvq_status gemv_launch_nt(const unisvq_layer* L, const DecodePlan& p, const void* x, void* y, int M,
-                             cudaStream_t s) {
+unisvq_status gemv_launch_nt(const unisvq_layer* const* Ls, int n, const DecodePlan& p, const void* x,
+                             void* const* ys, int m0, int M, cudaStream_t s) {
   static bool attr_set[64] = {};
-  const int dev = L->device;
+  const int dev = Ls[0]->device;
   if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
   if (!attr_set[dev]) {
     if (cudaFuncSetAttribute(gemv_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -363,22 +421,30 @@ unisvq_status gemv_launch_nt(const unisvq_layer* L, const DecodePlan& p, const v
   }
   const GemvShape sh = gemv_shape(M, p.kt_per_cta, p.ks, NT);
   GemvArgs a{};
-  a.codes = L->codes;
-  a.x = static_cast<const uint16_t*>(x);
-  a.y = static_cast<uint16_t*>(y);
+  a.x = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * Ls[0]->K;
   a.M = M;
-  a.N = L->N;
-  a.K = L->K;
-  a.KT = L->KT;
-  a.d = L->d;
+  a.K = Ls[0]->K;
+  a.KT = Ls[0]->KT;
   a.kt_per_cta = p.kt_per_cta;
   a.xstride = sh.xstride;
   a.off_red = sh.off_red;
   a.off_tok = sh.off_tok;
-  for (int i = 0; i < 16; ++i) a.A[i] = L->A[i];
-  for (int i = 0; i < 4; ++i) a.B[i] = L->B[i];
-  a.colnorm = L->colnorm;
+  a.nlayers = n;
   a.err = device_error_word();
+  int rb0 = 0;
+  for (int i = 0; i < n; ++i) {
+    const unisvq_layer* L = Ls[i];
+    GemvLayer& g = a.layer[i];
+    g.codes = L->codes;
+    g.y = static_cast<uint16_t*>(ys[i]) + static_cast<size_t>(m0) * L->N;
+    g.N = L->N;
+    g.d = L->d;
+    g.rb0 = rb0;
+    g.colnorm = L->colnorm;
+    for (int e = 0; e < 16; ++e) g.A[e] = L->A[e];
+    for (int e = 0; e < 4; ++e) g.B[e] = L->B[e];
+    rb0 += L->Np / kTileRows;
+  }
 
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.ks, p.nb, 1);
@@ -397,46 +463,55 @@ unisvq_status gemv_launch_nt(const unisvq_layer* L, const DecodePlan& p, const v
   return cudaLaunchKernelEx(&cfg, gemv_kernel<NT>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
-}  // namespace
-
-// Split K into ks <= 8 cluster CTAs: the largest ks whose grid fits one wave
-// of resident CTAs; if none does (many row blocks or a large folded slice),
-// the smallest ks whose slice fits in shared memory.
-DecodePlan plan_gemv(const unisvq_layer* L, int M) {
+// Split K into ks <= 8 cluster CTAs for nb row blocks: the largest ks whose
+// grid fits one wave of resident CTAs (two per SM); if none does, the
+// smallest ks whose folded slice fits in shared memory.
+DecodePlan plan_rows(int nb, int KT, int num_sms, int M) {
   DecodePlan p{};
   p.nt = M <= 8 ? 1 : 2;
-  p.nb = L->Np / kTileRows;
+  p.nb = nb;
   const size_t cap = kSmemPerSm - kSmemPerCtaReserved;
   int best = 0, fallback = 0;
   for (int c = kMaxSplit; c >= 1; --c) {
-    if (c > L->KT) continue;
-    const int kpc = (L->KT + c - 1) / c;
-    const int ks = (L->KT + kpc - 1) / kpc;
+    if (c > KT) continue;
+    const int kpc = (KT + c - 1) / c;
+    const int ks = (KT + kpc - 1) / kpc;
     if (ks != c) continue;
     const size_t smem = gemv_shape(M, kpc, ks, p.nt).smem;
     if (smem > cap) continue;
     fallback = ks;
-    if (!best && p.nb * ks <= gemv_ctas_per_sm(smem) * L->num_sms) best = ks;
+    const int per_sm = static_cast<int>(kSmemPerSm / (smem + kSmemPerCtaReserved)) < 2 ? 1 : 2;
+    if (!best && nb * ks <= per_sm * num_sms) best = ks;
   }
   const int ks = best ? best : (fallback ? fallback : kMaxSplit);
-  p.kt_per_cta = (L->KT + ks - 1) / ks;
-  p.ks = (L->KT + p.kt_per_cta - 1) / p.kt_per_cta;
+  p.kt_per_cta = (KT + ks - 1) / ks;
+  p.ks = (KT + p.kt_per_cta - 1) / p.kt_per_cta;
   p.smem = gemv_shape(M, p.kt_per_cta, p.ks, p.nt).smem;
   return p;
 }
 
-unisvq_status launch_gemv(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
+}  // namespace
+
+DecodePlan plan_gemv(const unisvq_layer* L, int M) { return plan_rows(L->Np / kTileRows, L->KT, L->num_sms, M); }
+
+unisvq_status launch_gemv_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                                cudaStream_t s) {
+  if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
+  int nb = 0;
+  for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
   for (int m0 = 0; m0 < M; m0 += kGMaxTok) {
     const int mc = M - m0 < kGMaxTok ? M - m0 : kGMaxTok;
-    const DecodePlan p = plan_gemv(L, mc);
+    const DecodePlan p = plan_rows(nb, Ls[0]->KT, Ls[0]->num_sms, mc);
     if (p.smem > kSmemPerSm - kSmemPerCtaReserved) return UNISVQ_ERR_UNSUPPORTED;
-    const void* xs = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * L->K;
-    void* ys = static_cast<uint16_t*>(y) + static_cast<size_t>(m0) * L->N;
-    const unisvq_status st =
-        p.nt == 1 ? gemv_launch_nt<1>(L, p, xs, ys, mc, s) : gemv_launch_nt<2>(L, p, xs, ys, mc, s);
+    const unisvq_status st = p.nt == 1 ? gemv_launch_nt<1>(Ls, n, p, x, ys, m0, mc, s)
+                                       : gemv_launch_nt<2>(Ls, n, p, x, ys, m0, mc, s);
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;
+}
+
+unisvq_status launch_gemv(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
+  return launch_gemv_group(&L, 1, x, &y, M, s);
 }
 
 }  // namespace unisvq

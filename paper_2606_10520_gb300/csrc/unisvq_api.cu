@@ -280,6 +280,34 @@ unisvq_status unisvq_linear(unisvq_handle h, const void* x, void* y, int M, void
   return unisvq_linear_force(h, UNISVQ_KERNEL_AUTO, x, y, M, stream);
 }
 
+unisvq_status unisvq_linear_group(const unisvq_handle* hs, int n, const void* x, void* const* ys, int M,
+                                  void* stream) {
+  if (!hs || !ys || n < 1 || n > UNISVQ_MAX_GROUP || M < 0) return UNISVQ_ERR_INVALID_ARG;
+  for (int i = 0; i < n; ++i) {
+    if (!hs[i] || hs[i]->K != hs[0]->K || hs[i]->device != hs[0]->device) return UNISVQ_ERR_INVALID_ARG;
+    const unisvq_status st = check_io(hs[i], x, ys[i], M);
+    if (st != UNISVQ_OK) return st;
+    for (int j = 0; j < i; ++j)
+      if (ys[j] && ys[i] &&
+          overlaps(ys[i], static_cast<size_t>(M) * hs[i]->N * 2, ys[j], static_cast<size_t>(M) * hs[j]->N * 2))
+        return UNISVQ_ERR_INVALID_ARG;
+  }
+  if (M == 0) return UNISVQ_OK;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
+  if (dev != hs[0]->device) return UNISVQ_ERR_INVALID_ARG;
+  if (auto_kernel(hs[0], M) == UNISVQ_KERNEL_GEMV) {
+    const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
+    for (int i = 0; i < n; ++i) Ls[i] = hs[i];
+    return launch_gemv_group(Ls, n, x, ys, M, static_cast<cudaStream_t>(stream));
+  }
+  for (int i = 0; i < n; ++i) {
+    const unisvq_status st = unisvq_linear(hs[i], x, ys[i], M, stream);
+    if (st != UNISVQ_OK) return st;
+  }
+  return UNISVQ_OK;
+}
+
 unisvq_status unisvq_dequant_debug(unisvq_handle h, float* W, void* stream) {
   if (!h || !W || !aligned(W, 4)) return UNISVQ_ERR_INVALID_ARG;
   return launch_dequant(h, W, static_cast<cudaStream_t>(stream));

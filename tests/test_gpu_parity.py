@@ -250,3 +250,64 @@ def test_full_size_prefill_sampled_rows(N, K):
     res = oracle.compare(yg[:, rows], yr, S)
     assert res["ok"], res
     layer.close()
+
+
+# ---------------------------------------------------------------------------
+# grouped call: several layers that read the same x
+# ---------------------------------------------------------------------------
+def run_group(layers, xbits):
+    ys = binding.linear_group(layers, to_dev(xbits))
+    st = binding.sync_status()
+    assert st == binding.OK, binding.status_string(st)
+    return [y.float().cpu().numpy().astype(np.float64) for y in ys]
+
+
+@pytest.mark.parametrize("K", [1000, 4096])
+@pytest.mark.parametrize("M", [1, 3, 8, 9, 16, 17, 40])
+def test_group_matches_oracle(K, M):
+    """Layers of different N and d sharing x, in one call: each output meets
+    the tolerance against the oracle of its own layer (M > 16 takes the
+    per-layer path)."""
+    specs = [(520, 2), (130, 4), (256, 1)]
+    data = [synth.layer_inputs(7, 70, i, K, N, K, d) for i, (N, d) in enumerate(specs)]
+    layers = [binding.UniSVQLinear(c, A, B) for c, A, B in data]
+    xb = synth.activations(7, 70, M, M, K)
+    for (c, A, B), yg in zip(data, run_group(layers, xb)):
+        check(yg, xb, c, A, B)
+    for l in layers:
+        l.close()
+
+
+def test_group_integer_case_bit_exact():
+    A = np.array([[1, -1, 0, 0], [0, 1, -1, 0], [0, 0, 1, -1], [0, 0, 1, 1]], dtype=np.float16)
+    B = np.array([1, -2, 0, 1], dtype=np.float16)
+    g = np.random.default_rng(13)
+    K = 512
+    codes = [g.integers(0, 4, size=(N, K), dtype=np.uint8) for N in (256, 384, 128, 130)]
+    layers = [binding.UniSVQLinear(c, A, B) for c in codes]
+    for M in (1, 7, 16):
+        x = g.integers(-1, 2, size=(M, K)).astype(np.float32) * (g.random((M, K)) < 0.05)
+        xb = synth.f32_to_bf16_bits(x)
+        for c, yg in zip(codes, run_group(layers, xb)):
+            yr, _ = oracle.linear(xb, c, A, B)
+            assert np.array_equal(yg, yr), np.abs(yg - yr).max()
+    for l in layers:
+        l.close()
+
+
+def test_group_rejects_mismatched_k_and_overlap():
+    a = binding.UniSVQLinear(*synth.layer_inputs(3, 30, 0, 0, 256, 512, 2))
+    b = binding.UniSVQLinear(*synth.layer_inputs(3, 30, 1, 0, 256, 1024, 2))
+    x = torch.zeros((2, 512), dtype=torch.bfloat16, device="cuda")
+    y0 = torch.zeros((2, 256), dtype=torch.bfloat16, device="cuda")
+    y1 = torch.zeros((2, 256), dtype=torch.bfloat16, device="cuda")
+    s = torch.cuda.current_stream().cuda_stream
+    assert binding.linear_group_ptr([a, b], x.data_ptr(), [y0.data_ptr(), y1.data_ptr()], 2, s) == \
+        binding.ERR_INVALID_ARG
+    c = a.clone()
+    assert binding.linear_group_ptr([a, c], x.data_ptr(), [y0.data_ptr(), y0.data_ptr()], 2, s) == \
+        binding.ERR_INVALID_ARG
+    assert binding.linear_group_ptr([a, c], x.data_ptr(), [y0.data_ptr(), y1.data_ptr()], 2, s) == binding.OK
+    assert binding.sync_status() == binding.OK
+    for l in (a, b, c):
+        l.close()

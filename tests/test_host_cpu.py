@@ -104,6 +104,12 @@ def test_linear_rejects_bad_arguments(lib):
     assert lib.unisvq_destroy(None) == binding.OK
     info = binding.Info()
     assert lib.unisvq_query(None, 1, ctypes.byref(info)) == binding.ERR_INVALID_ARG
+    hs = (ctypes.c_void_p * 2)(None, None)
+    ys = (ctypes.c_void_p * 2)(None, None)
+    assert lib.unisvq_linear_group(None, 1, None, ys, 1, None) == binding.ERR_INVALID_ARG
+    assert lib.unisvq_linear_group(hs, 0, None, ys, 1, None) == binding.ERR_INVALID_ARG
+    assert lib.unisvq_linear_group(hs, binding.MAX_GROUP + 1, None, ys, 1, None) == binding.ERR_INVALID_ARG
+    assert lib.unisvq_linear_group(hs, 2, None, ys, 1, None) == binding.ERR_INVALID_ARG   # null handles
 
 
 def test_version(lib):
