@@ -60,7 +60,7 @@ def algo_bytes(N, K, M, d=2):
     return N * K // 4 + (d * d + d) * 2 + 2 * M * K + 2 * M * N
 
 
-KERNEL_NAMES = {1: "decode", 2: "prefill_kernel", 3: "gemv_kernel", 4: "decode_kernel"}
+KERNEL_NAMES = {1: "decode", 2: "prefill_kernel", 3: "gemv_kernel", 4: "decode_kernel", 5: "gemv_rows_kernel"}
 GEMV_SOURCES = ("paper_2606_10520_gb300/csrc/gemv.cu", "paper_2606_10520_gb300/csrc/common.cuh",
                 "paper_2606_10520_gb300/csrc/layout.h")
 TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "gemv_kernel_llama2_7b_decode_sweep.txt")

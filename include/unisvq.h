@@ -48,7 +48,8 @@ enum {
   UNISVQ_KERNEL_DECODE = 1,   /* the decode kernel for this M (GEMV or SKINNY)         */
   UNISVQ_KERNEL_PREFILL = 2,  /* tcgen05 GEMM, exact bf16 codeword tiles in smem       */
   UNISVQ_KERNEL_GEMV = 3,     /* fold + register-operand tensor-core GEMV, M <= 16/launch */
-  UNISVQ_KERNEL_SKINNY = 4    /* fold + tcgen05 with codes as 8-bit TMEM operand, M <= 64/launch */
+  UNISVQ_KERNEL_SKINNY = 4,   /* fold + tcgen05 with codes as 8-bit TMEM operand, M <= 64/launch */
+  UNISVQ_KERNEL_GEMV_ROWS = 5 /* GEMV with whole-K row slices per CTA (no cluster), M <= 4/launch */
 };
 
 /*

@@ -388,6 +388,229 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   }
 }
 
+// ---------------------------------------------------------------------------
+// Row-slice GEMV for M <= kRMaxTok: CTA = 32 rows (units 2c and 2c+1 of the
+// layer) x the whole K, so no K-slice partial sums leave the CTA. Warp w owns
+// the contiguous k-tiles [w kpw, (w+1) kpw) of both units and folds exactly
+// those columns into its own shared-memory region with its own per-token
+// scale: no block barrier precedes its MMAs. The eight partial sums per
+// output are added in shared memory at the end. Each CTA folds all of x
+// (M x K), which is cheap next to the codes for a few tokens.
+// ---------------------------------------------------------------------------
+constexpr int kRMaxTok = 4;
+constexpr int kRDepth = 4;    // k-tiles of codes in flight per warp (2 x 16 bytes per lane each)
+constexpr int kRItems = 4;    // activation loads in flight per lane in the fold
+
+__global__ void __launch_bounds__(kGThreads, 2) gemv_rows_kernel(const __grid_constant__ GemvArgs a) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int M = a.M;
+  int li = 0;
+#pragma unroll
+  for (int i = 1; i < kMaxGroup; ++i)
+    if (i < a.nlayers && static_cast<int>(blockIdx.x) >= a.layer[i].rb0) li = i;
+  const uint8_t* codes = nullptr;
+  uint16_t* yout = nullptr;
+  int N = 0, d = 1, pr = 0;
+  float colnorm = 0.f, Areg[16], Bq[4];
+#pragma unroll
+  for (int i = 0; i < kMaxGroup; ++i) {
+    if (i == li) {
+      codes = a.layer[i].codes;
+      yout = a.layer[i].y;
+      N = a.layer[i].N;
+      d = a.layer[i].d;
+      pr = static_cast<int>(blockIdx.x) - a.layer[i].rb0;   // pair of units within the layer
+      colnorm = a.layer[i].colnorm;
+#pragma unroll
+      for (int e = 0; e < 16; ++e) Areg[e] = a.layer[i].A[e];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) Bq[e] = a.layer[i].B[e];
+    }
+  }
+  float Bcol[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) Bcol[e] = d == 1 ? Bq[0] : (d == 2 ? Bq[e & 1] : Bq[e & 3]);
+
+  const int kpw = a.kt_per_cta;
+  const int kw0 = warp * kpw;
+  const int nkw = max(0, min(kpw, a.KT - kw0));
+  const uint32_t wstride = static_cast<uint32_t>(a.xstride) * 2u;   // bytes per token row of a warp region
+  uint8_t* wreg = smem + warp * M * wstride;
+  float* red = reinterpret_cast<float*>(smem + a.off_red);         // [warp][32 rows][8 tokens]
+
+  // ---- codes: units 2 pr and 2 pr + 1 (512 contiguous bytes each per k-tile) ----
+  const int g = lane >> 2, t = lane & 3;
+  const int u0 = 2 * pr;
+  const uint8_t* cbase = codes + (static_cast<size_t>(u0 >> 3) * a.KT + kw0) * kTileBytes + (u0 & 7) * kUnitBytes +
+                         lane * 16;
+  uint4 cw[kRDepth][2];
+#pragma unroll
+  for (int s = 0; s < kRDepth; ++s)
+    if (s < nkw) {
+      cw[s][0] = ldg_stream_v4(cbase + static_cast<size_t>(s) * kTileBytes);
+      cw[s][1] = ldg_stream_v4(cbase + static_cast<size_t>(s) * kTileBytes + kUnitBytes);
+    }
+  pdl_launch_dependents();
+
+  pdl_wait();   // x may be the previous kernel's output
+
+  // ---- fold of this warp's columns for every token (private, no block barrier) ----
+  const int kbeg = kw0 * kTileCols;
+  const int kend = min(a.K, (kw0 + nkw) * kTileCols);
+  const int ncw = nkw * (kTileCols / 8);          // chunks per token
+  const int jt = (ncw + 31) / 32;                 // loads per lane per token
+  const int items = M * jt;
+  const bool vec8 = (a.K & 7) == 0;
+  float mx[kRMaxTok], cs[kRMaxTok];
+#pragma unroll
+  for (int q = 0; q < kRMaxTok; ++q) mx[q] = cs[q] = 0.f;
+  for (int b0 = 0; b0 < items; b0 += kRItems) {
+    uint4 u[kRItems];
+#pragma unroll
+    for (int r = 0; r < kRItems; ++r) {
+      const int it = b0 + r;
+      const int tk = it / jt, ci = lane + 32 * (it - tk * jt);
+      u[r] = (it < items && ci < ncw)
+                 ? load_x8(a.x + static_cast<size_t>(tk) * a.K, kbeg + 8 * ci, kend, vec8)
+                 : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int r = 0; r < kRItems; ++r) {
+      const int it = b0 + r;
+      const int tk = it / jt, ci = lane + 32 * (it - tk * jt);
+      if (it < items && ci < ncw) {
+        uint8_t* dst = wreg + tk * wstride + 16u * ci;
+        *reinterpret_cast<uint2*>(dst) = make_uint2(u[r].x, u[r].y);
+        *reinterpret_cast<uint2*>(dst + 8) = make_uint2(u[r].z, u[r].w);
+      }
+      float m8 = 0.f, c8 = 0.f;
+      const uint32_t w4[4] = {u[r].x, u[r].y, u[r].z, u[r].w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float v0 = bf16_lo(w4[q]), v1 = bf16_hi(w4[q]);
+        m8 = fmaxf(m8, fmaxf(fabsf(v0), fabsf(v1)));
+        c8 = fmaf(v0, Bcol[2 * q], c8);
+        c8 = fmaf(v1, Bcol[2 * q + 1], c8);
+      }
+#pragma unroll
+      for (int q = 0; q < kRMaxTok; ++q)
+        if (q == tk) {
+          mx[q] = fmaxf(mx[q], m8);
+          cs[q] += c8;
+        }
+    }
+  }
+  int pe[kRMaxTok];
+#pragma unroll
+  for (int q = 0; q < kRMaxTok; ++q) {
+#pragma unroll
+    for (int off = 16; off; off >>= 1) {
+      mx[q] = fmaxf(mx[q], __shfl_xor_sync(0xffffffffu, mx[q], off));
+      cs[q] += __shfl_xor_sync(0xffffffffu, cs[q], off);
+    }
+    pe[q] = token_scale_exp(mx[q] * colnorm);
+  }
+  for (int b0 = 0; b0 < items; b0 += kRItems) {
+    uint4 f[kRItems];
+#pragma unroll
+    for (int r = 0; r < kRItems; ++r) {
+      const int it = b0 + r;
+      const int tk = it / jt, ci = lane + 32 * (it - tk * jt);
+      if (it < items && ci < ncw) {
+        int pt = 0;
+#pragma unroll
+        for (int q = 0; q < kRMaxTok; ++q)
+          if (q == tk) pt = pe[q];
+        const uint8_t* src = wreg + tk * wstride + 16u * ci;
+        const uint2 lo = *reinterpret_cast<const uint2*>(src), hi = *reinterpret_cast<const uint2*>(src + 8);
+        f[r] = fold8(ci, make_uint4(lo.x, lo.y, hi.x, hi.y), pt, d, Areg);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < kRItems; ++r) {
+      const int it = b0 + r;
+      const int tk = it / jt, ci = lane + 32 * (it - tk * jt);
+      if (it < items && ci < ncw) {
+        uint8_t* dst = wreg + tk * wstride + 16u * ci;
+        *reinterpret_cast<uint2*>(dst) = make_uint2(f[r].x, f[r].y);
+        *reinterpret_cast<uint2*>(dst + 8) = make_uint2(f[r].z, f[r].w);
+      }
+    }
+  }
+  __syncwarp();
+
+  // ---- main loop over this warp's k-tiles ----
+  float acc[2][4];
+#pragma unroll
+  for (int u = 0; u < 2; ++u)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) acc[u][e] = 0.f;
+  const bool act = g < M;
+  const uint8_t* xl = wreg + (act ? g : 0) * wstride + 32u * t;
+  for (int i0 = 0; i0 < nkw; i0 += kRDepth) {
+#pragma unroll
+    for (int s = 0; s < kRDepth; ++s) {
+      const int i = i0 + s;
+      if (i < nkw) {
+        const uint32_t koff = 256u * i;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const uint32_t a0 = h ? cw[s][0].z : cw[s][0].x, a1 = h ? cw[s][0].w : cw[s][0].y;
+          const uint32_t b0 = h ? cw[s][1].z : cw[s][1].x, b1 = h ? cw[s][1].w : cw[s][1].y;
+          const uint32_t a0s = a0 >> 8, a1s = a1 >> 8, b0s = b0 >> 8, b1s = b1 >> 8;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const uint32_t m = 0x00030003u << (2 * j);
+            const uint2 bf = act ? *reinterpret_cast<const uint2*>(xl + koff + 128u * h + 8u * j) : make_uint2(0u, 0u);
+            mma_16816(acc[0], a0 & m, a1 & m, a0s & m, a1s & m, bf);
+            mma_16816(acc[1], b0 & m, b1 & m, b0s & m, b1s & m, bf);
+          }
+        }
+        if (i + kRDepth < nkw) {
+          cw[s][0] = ldg_stream_v4(cbase + static_cast<size_t>(i + kRDepth) * kTileBytes);
+          cw[s][1] = ldg_stream_v4(cbase + static_cast<size_t>(i + kRDepth) * kTileBytes + kUnitBytes);
+        }
+      }
+    }
+  }
+
+  // ---- partial sums of this warp -> red[warp][row][token], then add the 8 warps ----
+  float sc[2], cv[2];
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    const int tok = 2 * t + e;
+    sc[e] = 0.f;
+    cv[e] = 0.f;
+#pragma unroll
+    for (int q = 0; q < kRMaxTok; ++q)
+      if (q == tok) {
+        sc[e] = exp2i(24 - pe[q]);
+        cv[e] = cs[q];
+      }
+  }
+#pragma unroll
+  for (int u = 0; u < 2; ++u)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int row = 16 * u + g + ((e & 2) ? 8 : 0);
+      const int tok = 2 * t + (e & 1);
+      if (tok < M) red[(warp * 32 + row) * 8 + tok] = fmaf(acc[u][e], sc[e & 1], cv[e & 1]);
+    }
+  __syncthreads();
+  for (int idx = tid; idx < 32 * M; idx += kGThreads) {
+    const int tok = idx >> 5, row = idx & 31;
+    float v[kGWarps];
+#pragma unroll
+    for (int w = 0; w < kGWarps; ++w) v[w] = red[(w * 32 + row) * 8 + tok];
+    float sum = 0.f;
+#pragma unroll
+    for (int w = 0; w < kGWarps; ++w) sum += v[w];
+    const int n = 16 * u0 + row;
+    if (n < N) yout[static_cast<size_t>(tok) * N + n] = f32_to_bf16_rn(sum);
+  }
+}
+
 struct GemvShape {
   size_t smem;
   int off_red, off_tok, xstride;
@@ -490,6 +713,71 @@ DecodePlan plan_rows(int nb, int KT, int num_sms, int M) {
   return p;
 }
 
+// Row-slice kernel: k-tiles per warp, shared memory and launch.
+int rows_kpw(int KT) { return (KT + kGWarps - 1) / kGWarps; }
+
+size_t rows_smem(int M, int KT, int* off_red, int* xstride) {
+  const int kpw = rows_kpw(KT);
+  const int xs = kpw * kTileCols + kXPad;
+  const size_t fold = static_cast<size_t>(kGWarps) * M * xs * 2;
+  const size_t offr = (fold + 15) / 16 * 16;
+  if (off_red) *off_red = static_cast<int>(offr);
+  if (xstride) *xstride = xs;
+  return offr + static_cast<size_t>(kGWarps) * 32 * 8 * 4;
+}
+
+unisvq_status rows_launch(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int m0, int M,
+                          cudaStream_t s) {
+  static bool attr_set[64] = {};
+  const int dev = Ls[0]->device;
+  if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
+  if (!attr_set[dev]) {
+    if (cudaFuncSetAttribute(gemv_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(kSmemPerSm - kSmemPerCtaReserved)) != cudaSuccess ||
+        cudaFuncSetAttribute(gemv_rows_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared) != cudaSuccess)
+      return UNISVQ_ERR_CUDA;
+    attr_set[dev] = true;
+  }
+  GemvArgs a{};
+  int off_red = 0, xstride = 0;
+  const size_t smem = rows_smem(M, Ls[0]->KT, &off_red, &xstride);
+  a.x = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * Ls[0]->K;
+  a.M = M;
+  a.K = Ls[0]->K;
+  a.KT = Ls[0]->KT;
+  a.kt_per_cta = rows_kpw(Ls[0]->KT);
+  a.xstride = xstride;
+  a.off_red = off_red;
+  a.nlayers = n;
+  a.err = device_error_word();
+  int pairs = 0;
+  for (int i = 0; i < n; ++i) {
+    const unisvq_layer* L = Ls[i];
+    GemvLayer& g = a.layer[i];
+    g.codes = L->codes;
+    g.y = static_cast<uint16_t*>(ys[i]) + static_cast<size_t>(m0) * L->N;
+    g.N = L->N;
+    g.d = L->d;
+    g.rb0 = pairs;
+    g.colnorm = L->colnorm;
+    for (int e = 0; e < 16; ++e) g.A[e] = L->A[e];
+    for (int e = 0; e < 4; ++e) g.B[e] = L->B[e];
+    pairs += L->Np / (2 * kUnitRows);
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(pairs, 1, 1);
+  cfg.blockDim = dim3(kGThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr.val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, gemv_rows_kernel, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+}
+
 }  // namespace
 
 DecodePlan plan_gemv(const unisvq_layer* L, int M) { return plan_rows(L->Np / kTileRows, L->KT, L->num_sms, M); }
@@ -512,6 +800,22 @@ unisvq_status launch_gemv_group(const unisvq_layer* const* Ls, int n, const void
 
 unisvq_status launch_gemv(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
   return launch_gemv_group(&L, 1, x, &y, M, s);
+}
+
+bool gemv_rows_supported(const unisvq_layer* L, int M) {
+  return M >= 1 && M <= kRMaxTok && rows_smem(M, L->KT, nullptr, nullptr) <= kSmemPerSm / 2 - kSmemPerCtaReserved;
+}
+
+unisvq_status launch_gemv_rows_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                                     cudaStream_t s) {
+  if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
+  for (int m0 = 0; m0 < M; m0 += kRMaxTok) {
+    const int mc = M - m0 < kRMaxTok ? M - m0 : kRMaxTok;
+    if (!gemv_rows_supported(Ls[0], mc)) return UNISVQ_ERR_UNSUPPORTED;
+    const unisvq_status st = rows_launch(Ls, n, x, ys, m0, mc, s);
+    if (st != UNISVQ_OK) return st;
+  }
+  return UNISVQ_OK;
 }
 
 }  // namespace unisvq

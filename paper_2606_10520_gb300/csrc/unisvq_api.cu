@@ -240,11 +240,19 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
   return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess) ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
-static int decode_kernel_for(int M) { return M <= 16 ? UNISVQ_KERNEL_GEMV : UNISVQ_KERNEL_SKINNY; }
+// Decode kernel for M tokens over `weights` = sum of N*K of the layers of one
+// launch (measured crossovers on GB300): the whole-K row-slice GEMV for one or
+// two tokens on launches of at least 2^26 weights (no cross-CTA reduction,
+// many small CTAs), the K-split cluster GEMV up to 16 tokens, the tcgen05
+// skinny GEMM beyond.
+static int decode_kernel_for(const unisvq_layer* L, long long weights, int M) {
+  if (M <= 2 && weights >= (1ll << 26) && gemv_rows_supported(L, M)) return UNISVQ_KERNEL_GEMV_ROWS;
+  return M <= 16 ? UNISVQ_KERNEL_GEMV : UNISVQ_KERNEL_SKINNY;
+}
 
 static int auto_kernel(const unisvq_layer* L, int M) {
   if (M > 64 && prefill_supported(L, M)) return UNISVQ_KERNEL_PREFILL;
-  return decode_kernel_for(M);
+  return decode_kernel_for(L, static_cast<long long>(L->N) * L->K, M);
 }
 
 static unisvq_status check_io(unisvq_handle h, const void* x, void* y, int M) {
@@ -265,9 +273,15 @@ unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, vo
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
   if (dev != h->device) return UNISVQ_ERR_INVALID_ARG;
   if (kernel == UNISVQ_KERNEL_AUTO) kernel = auto_kernel(h, M);
-  if (kernel == UNISVQ_KERNEL_DECODE) kernel = decode_kernel_for(M);
+  if (kernel == UNISVQ_KERNEL_DECODE) kernel = decode_kernel_for(h, static_cast<long long>(h->N) * h->K, M);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (kernel == UNISVQ_KERNEL_GEMV) return launch_gemv(h, x, y, M, s);
+  if (kernel == UNISVQ_KERNEL_GEMV_ROWS) {
+    if (!gemv_rows_supported(h, M < 4 ? M : 4)) return UNISVQ_ERR_UNSUPPORTED;
+    const unisvq_layer* Ls[1] = {h};
+    void* ys[1] = {y};
+    return launch_gemv_rows_group(Ls, 1, x, ys, M, s);
+  }
   if (kernel == UNISVQ_KERNEL_SKINNY) return launch_skinny(h, x, y, M, s);
   if (kernel == UNISVQ_KERNEL_PREFILL) {
     if (!prefill_supported(h, M)) return UNISVQ_ERR_UNSUPPORTED;
@@ -296,10 +310,15 @@ unisvq_status unisvq_linear_group(const unisvq_handle* hs, int n, const void* x,
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
   if (dev != hs[0]->device) return UNISVQ_ERR_INVALID_ARG;
-  if (auto_kernel(hs[0], M) == UNISVQ_KERNEL_GEMV) {
+  long long weights = 0;
+  for (int i = 0; i < n; ++i) weights += static_cast<long long>(hs[i]->N) * hs[i]->K;
+  const int kernel = M > 64 && prefill_supported(hs[0], M) ? UNISVQ_KERNEL_PREFILL : decode_kernel_for(hs[0], weights, M);
+  if (kernel == UNISVQ_KERNEL_GEMV || kernel == UNISVQ_KERNEL_GEMV_ROWS) {
     const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
     for (int i = 0; i < n; ++i) Ls[i] = hs[i];
-    return launch_gemv_group(Ls, n, x, ys, M, static_cast<cudaStream_t>(stream));
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    return kernel == UNISVQ_KERNEL_GEMV ? launch_gemv_group(Ls, n, x, ys, M, s)
+                                        : launch_gemv_rows_group(Ls, n, x, ys, M, s);
   }
   for (int i = 0; i < n; ++i) {
     const unisvq_status st = unisvq_linear(hs[i], x, ys[i], M, stream);
@@ -327,7 +346,10 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
                      2ll * M * h->K + 2ll * M * h->N;
   info->flops = 2.0 * M * static_cast<double>(h->N) * h->K;
   info->kernel = auto_kernel(h, M > 0 ? M : 1);
-  if (info->kernel == UNISVQ_KERNEL_GEMV) {
+  if (info->kernel == UNISVQ_KERNEL_GEMV_ROWS) {
+    info->split_k = 1;
+    info->grid_ctas = h->Np / 32;
+  } else if (info->kernel == UNISVQ_KERNEL_GEMV) {
     const DecodePlan p = plan_gemv(h, M > 16 ? 16 : (M > 0 ? M : 1));
     info->split_k = p.ks;
     info->grid_ctas = p.ks * p.nb * ((M + 15) / 16 > 0 ? (M + 15) / 16 : 1);

@@ -59,7 +59,7 @@ def test_dequant_debug_bit_exact(d, N, K):
 DECODE_SHAPES = [(256, 1024), (520, 1000), (130, 4096), (1024, 8192)]
 
 
-DECODE_KERNELS = [binding.KERNEL_GEMV, binding.KERNEL_SKINNY]
+DECODE_KERNELS = [binding.KERNEL_GEMV, binding.KERNEL_GEMV_ROWS, binding.KERNEL_SKINNY]
 
 
 @pytest.mark.parametrize("kernel", DECODE_KERNELS)
