@@ -45,9 +45,9 @@ typedef enum {
 /* Kernel selectors for unisvq_linear_force and unisvq_info.kernel. */
 enum {
   UNISVQ_KERNEL_AUTO = 0,     /* pick by M (unisvq_linear does this)                   */
-  UNISVQ_KERNEL_DECODE = 1,   /* the decode kernel for this M (GEMV or SKINNY)         */
+  UNISVQ_KERNEL_DECODE = 1,   /* the decode kernel auto would pick for this M (a GEMV)  */
   UNISVQ_KERNEL_PREFILL = 2,  /* tcgen05 GEMM, exact bf16 codeword tiles in smem       */
-  UNISVQ_KERNEL_GEMV = 3,     /* fold + register-operand tensor-core GEMV, M <= 16/launch */
+  UNISVQ_KERNEL_GEMV = 3,     /* fold + register-operand tensor-core GEMV, M <= 32/launch */
   UNISVQ_KERNEL_SKINNY = 4,   /* fold + tcgen05 with codes as 8-bit TMEM operand, M <= 64/launch */
   UNISVQ_KERNEL_GEMV_ROWS = 5 /* GEMV with whole-K row slices per CTA (no cluster), M <= 4/launch */
 };
@@ -133,7 +133,7 @@ unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, vo
  * each layer, with its own codes and its own A, B of Eq. col:dequant), e.g.
  * the q, k, v projections or the gate and up projections of one transformer
  * block. The paper defines the layer, not this grouping; it is a launch
- * convenience: for M <= 16 all n layers run in one kernel launch (the row
+ * convenience: for M <= 64 the n layers share each kernel launch (the row
  * blocks of the layers side by side), otherwise one unisvq_linear per layer.
  *   hs : n handles on the current device, all with the same K
  *   n  : 1 .. UNISVQ_MAX_GROUP

@@ -1,4 +1,4 @@
-// GEMV for M <= 16 tokens per launch: register-operand tensor-core MMAs.
+// GEMV for M <= 32 tokens per launch: register-operand tensor-core MMAs.
 //
 // Computes y = x W_hat^T through the fold of Eq. (col:matmul):
 //   y[m, n] = sum_k x'[m, k] z[n, k] + c[m],  x' = x_g A,  c = sum_g x_g . B.
@@ -35,11 +35,11 @@ constexpr int kGWarps = 8;
 constexpr int kGThreads = kGWarps * 32;
 constexpr int kGDepth = 8;          // k-tiles of codes in flight per warp (16 bytes per lane each)
 constexpr int kMaxSplit = 8;        // K slices per row block (cluster size)
-constexpr int kGMaxTok = 16;
+constexpr int kGMaxTok = 32;
 constexpr int kMaxGroup = UNISVQ_MAX_GROUP;   // layers per launch
 constexpr int kXLoads = 4;          // 16-byte activation loads in flight per lane (fold)
 constexpr int kXPad = 4;            // fp16 elements of padding per token row (bank spread)
-constexpr int kTokBytes = 160;      // pexp[16], cpart[16], reduction mbarrier
+constexpr int kTokBytes = 272;      // pexp[32], cpart[32], reduction mbarrier
 constexpr size_t kSmemPerSm = 228 * 1024;
 constexpr size_t kSmemPerCtaReserved = 1024;
 
@@ -167,9 +167,9 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   const int nown = max(0, min(kTileRows, own0 + rows_per) - own0);
 
   int* pexp = reinterpret_cast<int*>(smem + a.off_tok);
-  float* cpart = reinterpret_cast<float*>(smem + a.off_tok + 64);
+  float* cpart = reinterpret_cast<float*>(smem + a.off_tok + 128);
   float* red = reinterpret_cast<float*>(smem + a.off_red);
-  const uint32_t red_bar = sbase + a.off_tok + 128;
+  const uint32_t red_bar = sbase + a.off_tok + 256;
 
   // Reduction barrier: one arrival here plus the bytes the other CTAs of the
   // cluster store into this CTA's slots (st.async counts them).
@@ -207,26 +207,31 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   const int nch = n_kt * (kTileCols / 8);   // 8-column chunks of the slice
   const bool vec8 = (a.K & 7) == 0;
   const uint32_t xrow_bytes = static_cast<uint32_t>(a.xstride) * 2u;
-  for (int tk = warp; tk < M; tk += kGWarps) {
-    const uint16_t* row = a.x + static_cast<size_t>(tk) * a.K;
-    uint8_t* xrow = smem + tk * xrow_bytes;
-    float mx = 0.f, cs = 0.f;
-    uint4 u[kXLoads];
-    for (int c0 = lane; c0 < nch; c0 += 32 * kXLoads) {
+  if (nch <= 32 * kXLoads) {
+    // Whole slice in registers: the loads of both of this warp's tokens go
+    // out together, then each token is reduced, folded and stored.
+    constexpr int kPair = NT < 2 ? NT : 2;   // tokens whose loads are in flight together
+#pragma unroll 1
+    for (int p0 = 0; p0 < NT; p0 += kPair) {
+    uint4 u[kPair][kXLoads];
+#pragma unroll
+    for (int p = 0; p < kPair; ++p) {
+      const int tk = warp + kGWarps * (p0 + p);
 #pragma unroll
       for (int j = 0; j < kXLoads; ++j) {
-        const int ci = c0 + 32 * j;
-        u[j] = ci < nch ? load_x8(row, kbeg + 8 * ci, kend, vec8) : make_uint4(0, 0, 0, 0);
+        const int ci = lane + 32 * j;
+        u[p][j] = (tk < M && ci < nch) ? load_x8(a.x + static_cast<size_t>(tk) * a.K, kbeg + 8 * ci, kend, vec8)
+                                       : make_uint4(0, 0, 0, 0);
       }
+    }
 #pragma unroll
-      for (int j = 0; j < kXLoads; ++j) {
-        const int ci = c0 + 32 * j;
-        if (ci < nch) {
-          if (nch > 32 * kXLoads) {   // staged for the second pass
-            *reinterpret_cast<uint2*>(xrow + 16u * ci) = make_uint2(u[j].x, u[j].y);
-            *reinterpret_cast<uint2*>(xrow + 16u * ci + 8) = make_uint2(u[j].z, u[j].w);
-          }
-          const uint32_t w4[4] = {u[j].x, u[j].y, u[j].z, u[j].w};
+    for (int p = 0; p < kPair; ++p) {
+      const int tk = warp + kGWarps * (p0 + p);
+      if (tk < M) {
+        float mx = 0.f, cs = 0.f;
+#pragma unroll
+        for (int j = 0; j < kXLoads; ++j) {
+          const uint32_t w4[4] = {u[p][j].x, u[p][j].y, u[p][j].z, u[p][j].w};
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const float v0 = bf16_lo(w4[q]), v1 = bf16_hi(w4[q]);
@@ -235,33 +240,72 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
             cs = fmaf(v1, Bcol[2 * q + 1], cs);
           }
         }
-      }
-    }
 #pragma unroll
-    for (int off = 16; off; off >>= 1) {
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-      cs += __shfl_xor_sync(0xffffffffu, cs, off);
-    }
-    const int pe = token_scale_exp(mx * colnorm);
-    if (lane == 0) {
-      pexp[tk] = pe;
-      cpart[tk] = cs;
-    }
-    if (nch <= 32 * kXLoads) {
-      // the whole slice is still in registers: fold, then store
-      uint4 f[kXLoads];
+        for (int off = 16; off; off >>= 1) {
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+          cs += __shfl_xor_sync(0xffffffffu, cs, off);
+        }
+        const int pe = token_scale_exp(mx * colnorm);
+        if (lane == 0) {
+          pexp[tk] = pe;
+          cpart[tk] = cs;
+        }
+        uint8_t* xrow = smem + tk * xrow_bytes;
+        uint4 f[kXLoads];
 #pragma unroll
-      for (int j = 0; j < kXLoads; ++j) f[j] = fold8(lane + 32 * j, u[j], pe, d, Areg);
+        for (int j = 0; j < kXLoads; ++j) f[j] = fold8(lane + 32 * j, u[p][j], pe, d, Areg);
 #pragma unroll
-      for (int j = 0; j < kXLoads; ++j) {
-        const int ci = lane + 32 * j;
-        if (ci < nch) {
-          *reinterpret_cast<uint2*>(xrow + 16u * ci) = make_uint2(f[j].x, f[j].y);
-          *reinterpret_cast<uint2*>(xrow + 16u * ci + 8) = make_uint2(f[j].z, f[j].w);
+        for (int j = 0; j < kXLoads; ++j) {
+          const int ci = lane + 32 * j;
+          if (ci < nch) {
+            *reinterpret_cast<uint2*>(xrow + 16u * ci) = make_uint2(f[j].x, f[j].y);
+            *reinterpret_cast<uint2*>(xrow + 16u * ci + 8) = make_uint2(f[j].z, f[j].w);
+          }
         }
       }
-    } else {
-      // every lane re-reads only the chunks it staged itself
+    }
+    }
+  } else {
+    for (int tk = warp; tk < M; tk += kGWarps) {
+      const uint16_t* row = a.x + static_cast<size_t>(tk) * a.K;
+      uint8_t* xrow = smem + tk * xrow_bytes;
+      float mx = 0.f, cs = 0.f;
+      uint4 u[kXLoads];
+      // pass A: stage the chunks, max and c-sum
+      for (int c0 = lane; c0 < nch; c0 += 32 * kXLoads) {
+#pragma unroll
+        for (int j = 0; j < kXLoads; ++j) {
+          const int ci = c0 + 32 * j;
+          u[j] = ci < nch ? load_x8(row, kbeg + 8 * ci, kend, vec8) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int j = 0; j < kXLoads; ++j) {
+          const int ci = c0 + 32 * j;
+          if (ci < nch) {
+            *reinterpret_cast<uint2*>(xrow + 16u * ci) = make_uint2(u[j].x, u[j].y);
+            *reinterpret_cast<uint2*>(xrow + 16u * ci + 8) = make_uint2(u[j].z, u[j].w);
+            const uint32_t w4[4] = {u[j].x, u[j].y, u[j].z, u[j].w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const float v0 = bf16_lo(w4[q]), v1 = bf16_hi(w4[q]);
+              mx = fmaxf(mx, fmaxf(fabsf(v0), fabsf(v1)));
+              cs = fmaf(v0, Bcol[2 * q], cs);
+              cs = fmaf(v1, Bcol[2 * q + 1], cs);
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int off = 16; off; off >>= 1) {
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+        cs += __shfl_xor_sync(0xffffffffu, cs, off);
+      }
+      const int pe = token_scale_exp(mx * colnorm);
+      if (lane == 0) {
+        pexp[tk] = pe;
+        cpart[tk] = cs;
+      }
+      // pass B: every lane re-reads only the chunks it staged itself
       for (int c0 = lane; c0 < nch; c0 += 32 * kXLoads) {
 #pragma unroll
         for (int j = 0; j < kXLoads; ++j) {
@@ -286,13 +330,11 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   __syncthreads();
 
   // ---- main loop: no block-wide barrier ----
-  float acc[2][NT][4];
+  float acc[NT][4];   // both halves of a k-tile accumulate into one chain per token octet
 #pragma unroll
-  for (int h = 0; h < 2; ++h)
+  for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) acc[h][nt][e] = 0.f;
+    for (int e = 0; e < 4; ++e) acc[nt][e] = 0.f;
   bool act[NT];
   const uint8_t* xl[NT];   // this lane's B fragments: token 8nt + g, quarter t
 #pragma unroll
@@ -318,7 +360,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
             for (int nt = 0; nt < NT; ++nt) {
               const uint2 b = act[nt] ? *reinterpret_cast<const uint2*>(xl[nt] + koff + 128u * h + 8u * j)
                                       : make_uint2(0u, 0u);
-              mma_16816(acc[h][nt], wa & m, wb & m, was & m, wbs & m, b);
+              mma_16816(acc[nt], wa & m, wb & m, was & m, wbs & m, b);
             }
           }
         }
@@ -343,8 +385,8 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
     const float sc1 = tok + 1 < M ? exp2i(24 - pexp[tok + 1]) : 0.f, c1v = tok + 1 < M ? cpart[tok + 1] : 0.f;
 #pragma unroll
     for (int rh = 0; rh < 2; ++rh) {
-      pv[nt][rh][0] = fmaf(acc[0][nt][2 * rh] + acc[1][nt][2 * rh], sc0, c0v);
-      pv[nt][rh][1] = fmaf(acc[0][nt][2 * rh + 1] + acc[1][nt][2 * rh + 1], sc1, c1v);
+      pv[nt][rh][0] = fmaf(acc[nt][2 * rh], sc0, c0v);
+      pv[nt][rh][1] = fmaf(acc[nt][2 * rh + 1], sc1, c1v);
     }
   }
 #pragma unroll
@@ -691,7 +733,7 @@ unisvq_status gemv_launch_nt(const unisvq_layer* const* Ls, int n, const DecodeP
 // smallest ks whose folded slice fits in shared memory.
 DecodePlan plan_rows(int nb, int KT, int num_sms, int M) {
   DecodePlan p{};
-  p.nt = M <= 8 ? 1 : 2;
+  p.nt = M <= 8 ? 1 : (M <= 16 ? 2 : 4);
   p.nb = nb;
   const size_t cap = kSmemPerSm - kSmemPerCtaReserved;
   int best = 0, fallback = 0;
@@ -787,13 +829,21 @@ unisvq_status launch_gemv_group(const unisvq_layer* const* Ls, int n, const void
   if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
   int nb = 0;
   for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
-  for (int m0 = 0; m0 < M; m0 += kGMaxTok) {
-    const int mc = M - m0 < kGMaxTok ? M - m0 : kGMaxTok;
-    const DecodePlan p = plan_rows(nb, Ls[0]->KT, Ls[0]->num_sms, mc);
+  for (int m0 = 0; m0 < M;) {
+    // up to 32 tokens per launch; fewer when the folded slice of a long K
+    // would not fit in shared memory
+    int mc = M - m0 < kGMaxTok ? M - m0 : kGMaxTok;
+    DecodePlan p = plan_rows(nb, Ls[0]->KT, Ls[0]->num_sms, mc);
+    while (p.smem > kSmemPerSm - kSmemPerCtaReserved && mc > 1) {
+      mc = (mc + 1) / 2;
+      p = plan_rows(nb, Ls[0]->KT, Ls[0]->num_sms, mc);
+    }
     if (p.smem > kSmemPerSm - kSmemPerCtaReserved) return UNISVQ_ERR_UNSUPPORTED;
-    const unisvq_status st = p.nt == 1 ? gemv_launch_nt<1>(Ls, n, p, x, ys, m0, mc, s)
-                                       : gemv_launch_nt<2>(Ls, n, p, x, ys, m0, mc, s);
+    const unisvq_status st = p.nt == 1   ? gemv_launch_nt<1>(Ls, n, p, x, ys, m0, mc, s)
+                             : p.nt == 2 ? gemv_launch_nt<2>(Ls, n, p, x, ys, m0, mc, s)
+                                         : gemv_launch_nt<4>(Ls, n, p, x, ys, m0, mc, s);
     if (st != UNISVQ_OK) return st;
+    m0 += mc;
   }
   return UNISVQ_OK;
 }

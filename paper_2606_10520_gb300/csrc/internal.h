@@ -44,14 +44,14 @@ struct PrefillPlan {
 
 int* device_error_word();   // device address of the library error word (current device)
 
-// Register-operand tensor-core GEMV (gemv.cu), M <= 16 per launch.
+// Register-operand tensor-core GEMV (gemv.cu), M <= 32 per launch.
 DecodePlan plan_gemv(const unisvq_layer* L, int M);
 unisvq_status launch_gemv(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
 // Row-slice GEMV (whole K per CTA, no cluster), M <= 4 per launch.
 bool gemv_rows_supported(const unisvq_layer* L, int M);
 unisvq_status launch_gemv_rows_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
                                      cudaStream_t s);
-// Several layers with the same K that read the same x, in one launch per 16 tokens.
+// Several layers with the same K that read the same x, in one launch per 32 tokens.
 unisvq_status launch_gemv_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
                                 cudaStream_t s);
 // tcgen05 skinny GEMM with the codes as 8-bit TMEM operand (decode.cu), M <= 64 per launch.

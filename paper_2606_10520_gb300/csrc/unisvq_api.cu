@@ -240,14 +240,15 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
   return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess) ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
-// Decode kernel for M tokens over `weights` = sum of N*K of the layers of one
-// launch (measured crossovers on GB300): the whole-K row-slice GEMV for one or
-// two tokens on launches of at least 2^26 weights (no cross-CTA reduction,
-// many small CTAs), the K-split cluster GEMV up to 16 tokens, the tcgen05
-// skinny GEMM beyond.
+// Decode kernel for M <= 64 tokens over `weights` = sum of N*K of the layers
+// of one launch (measured crossovers on GB300): the whole-K row-slice GEMV for
+// one or two tokens on launches of at least 2^26 weights (no cross-CTA
+// reduction, many small CTAs), otherwise the K-split cluster GEMV (32 tokens
+// per launch). The tcgen05 skinny kernel is reachable through
+// unisvq_linear_force only: as built it is slower than the GEMV at every M.
 static int decode_kernel_for(const unisvq_layer* L, long long weights, int M) {
   if (M <= 2 && weights >= (1ll << 26) && gemv_rows_supported(L, M)) return UNISVQ_KERNEL_GEMV_ROWS;
-  return M <= 16 ? UNISVQ_KERNEL_GEMV : UNISVQ_KERNEL_SKINNY;
+  return UNISVQ_KERNEL_GEMV;
 }
 
 static int auto_kernel(const unisvq_layer* L, int M) {
@@ -350,9 +351,9 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
     info->split_k = 1;
     info->grid_ctas = h->Np / 32;
   } else if (info->kernel == UNISVQ_KERNEL_GEMV) {
-    const DecodePlan p = plan_gemv(h, M > 16 ? 16 : (M > 0 ? M : 1));
+    const DecodePlan p = plan_gemv(h, M > 32 ? 32 : (M > 0 ? M : 1));
     info->split_k = p.ks;
-    info->grid_ctas = p.ks * p.nb * ((M + 15) / 16 > 0 ? (M + 15) / 16 : 1);
+    info->grid_ctas = p.ks * p.nb * ((M + 31) / 32 > 0 ? (M + 31) / 32 : 1);
   } else if (info->kernel == UNISVQ_KERNEL_SKINNY) {
     const DecodePlan p = plan_skinny(h, M > 64 ? 64 : (M > 0 ? M : 1));
     info->split_k = p.ks;

@@ -229,7 +229,7 @@ def test_prefill_and_decode_agree_with_auto_dispatch():
     layer = binding.UniSVQLinear(codes, A, B)
     assert layer.query(1)["kernel"] == binding.KERNEL_GEMV
     assert layer.query(16)["kernel"] == binding.KERNEL_GEMV
-    assert layer.query(17)["kernel"] == binding.KERNEL_SKINNY
+    assert layer.query(64)["kernel"] == binding.KERNEL_GEMV
     assert layer.query(2048)["kernel"] == binding.KERNEL_PREFILL
     xb = synth.activations(9, 90, 0, 96, K)
     check(run(layer, xb), xb, codes, A, B)
