@@ -48,7 +48,7 @@ enum {
   UNISVQ_KERNEL_DECODE = 1,   /* the decode kernel auto would pick for this M (a GEMV)  */
   UNISVQ_KERNEL_PREFILL = 2,  /* tcgen05 GEMM, exact bf16 codeword tiles in smem       */
   UNISVQ_KERNEL_GEMV = 3,     /* fold + register-operand tensor-core GEMV, M <= 32/launch */
-  UNISVQ_KERNEL_SKINNY = 4,   /* fold + tcgen05 with codes as 8-bit TMEM operand, M <= 64/launch */
+  UNISVQ_KERNEL_SKINNY = 4,   /* fold + tcgen05 with codes as 8-bit TMEM operand, M <= 16/launch */
   UNISVQ_KERNEL_GEMV_ROWS = 5 /* GEMV with whole-K row slices per CTA (no cluster), M <= 4/launch */
 };
 
@@ -104,8 +104,13 @@ typedef struct {
  * The host buffers are copied before return; the caller keeps ownership.
  * Errors: INVALID_ARG (null pointer, bad shape, code > 3, non-finite A/B),
  * UNSUPPORTED (d not in {1,2,4}), OOM, CUDA.
- * The handle owns all device memory and is immutable afterwards, so
- * concurrent unisvq_linear calls on different streams are safe.
+ * The handle owns all device memory: the packed codes, the tables of the
+ * prefill kernel and a fold workspace of 1 KB + (Kp/128) * 6 KB that the
+ * decode kernels rewrite on every call (the folded activations of Eq.
+ * col:matmul). Calls that use the same handle must therefore be ordered on
+ * the GPU (one stream, or events between streams); calls on different
+ * handles may run concurrently. unisvq_clone gives a second handle with its
+ * own workspace.
  */
 unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
                           int N, int K, int d, void* stream, unisvq_handle* out);
@@ -148,6 +153,13 @@ unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, vo
 #define UNISVQ_MAX_GROUP 4
 unisvq_status unisvq_linear_group(const unisvq_handle* hs, int n, const void* x, void* const* ys, int M,
                                   void* stream);
+
+/* As unisvq_linear_group but runs the given UNISVQ_KERNEL_* (crossover sweeps
+ * and tests). GEMV, GEMV_ROWS and SKINNY share one launch across the layers;
+ * other kernels run once per layer as unisvq_linear_force. Same arguments,
+ * results and errors as unisvq_linear_group. */
+unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kernel, const void* x, void* const* ys,
+                                        int M, void* stream);
 
 /* Test hook: writes W_hat as fp32 [N][K] row-major to device memory W (each
  * entry RN_fp32 of the exact A z + B), unpacking the device layout with the

@@ -21,7 +21,7 @@ EXPORTS = [
     "unisvq_pack", "unisvq_linear", "unisvq_linear_force", "unisvq_dequant_debug",
     "unisvq_query", "unisvq_sync_status", "unisvq_destroy", "unisvq_clone",
     "unisvq_status_string", "unisvq_packed_code_bytes", "unisvq_pack_host", "unisvq_version",
-    "unisvq_linear_group",
+    "unisvq_linear_group", "unisvq_linear_group_force",
 ]
 MAX_GROUP = 4
 
@@ -56,6 +56,7 @@ def load():
     lib.unisvq_linear.argtypes = [vp, vp, vp, i, vp]
     lib.unisvq_linear_force.argtypes = [vp, i, vp, vp, i, vp]
     lib.unisvq_linear_group.argtypes = [vp, i, vp, vp, i, vp]
+    lib.unisvq_linear_group_force.argtypes = [vp, i, i, vp, vp, i, vp]
     lib.unisvq_dequant_debug.argtypes = [vp, vp, vp]
     lib.unisvq_query.argtypes = [vp, i, ctypes.POINTER(Info)]
     lib.unisvq_sync_status.argtypes = [vp]
@@ -182,16 +183,21 @@ class UniSVQLinear:
             pass
 
 
-def linear_group_ptr(layers, x_ptr: int, y_ptrs, M: int, stream_ptr: int) -> int:
-    """Raw-pointer unisvq_linear_group over `layers` (same K); returns the status."""
+def linear_group_ptr(layers, x_ptr: int, y_ptrs, M: int, stream_ptr: int, kernel=None) -> int:
+    """Raw-pointer unisvq_linear_group (or unisvq_linear_group_force when
+    `kernel` is given) over `layers` (same K); returns the status."""
     n = len(layers)
     hs = (ctypes.c_void_p * n)(*[l._h.value if isinstance(l._h, ctypes.c_void_p) else l._h for l in layers])
     ys = (ctypes.c_void_p * n)(*[int(p) for p in y_ptrs])
-    return load().unisvq_linear_group(hs, n, ctypes.c_void_p(x_ptr), ys, M, ctypes.c_void_p(stream_ptr))
+    if kernel is None:
+        return load().unisvq_linear_group(hs, n, ctypes.c_void_p(x_ptr), ys, M, ctypes.c_void_p(stream_ptr))
+    return load().unisvq_linear_group_force(hs, n, int(kernel), ctypes.c_void_p(x_ptr), ys, M,
+                                            ctypes.c_void_p(stream_ptr))
 
 
-def linear_group(layers, x, outs=None, stream=None):
-    """y_i = x W_hat_i^T for layers that share x ([M][K] bf16 CUDA tensor)."""
+def linear_group(layers, x, outs=None, stream=None, kernel=None):
+    """y_i = x W_hat_i^T for layers that share x ([M][K] bf16 CUDA tensor);
+    `kernel` (a KERNEL_* value) forces the kernel, else the library picks."""
     import torch
     if x.dtype != torch.bfloat16 or not x.is_cuda or x.dim() != 2:
         raise ValueError("x must be a CUDA bf16 tensor of shape [M, K]")
@@ -200,5 +206,5 @@ def linear_group(layers, x, outs=None, stream=None):
     if outs is None:
         outs = [torch.empty((M, l.N), dtype=torch.bfloat16, device=x.device) for l in layers]
     _check(linear_group_ptr(layers, x.data_ptr(), [o.data_ptr() for o in outs], M,
-                            _stream_ptr(stream).value or 0), "unisvq_linear_group")
+                            _stream_ptr(stream).value or 0, kernel), "unisvq_linear_group")
     return outs

@@ -1,74 +1,128 @@
-// Skinny GEMM for decode batches (M <= 64 tokens per launch): tcgen05 tensor cores
-// with the 2-bit codes as an 8-bit operand resident in tensor memory.
+// Skinny GEMM for decode batches (M <= 16 tokens per launch): tcgen05 tensor
+// cores with the 2-bit codes as an 8-bit operand resident in tensor memory.
 //
 // Computes y = x W_hat^T through the fold of Eq. (col:matmul):
 //   y[m, n] = sum_k x'[m, k] z[n, k] + c[m],
 //   x'[m, g d + c] = sum_r x[m, g d + r] A[r][c]      (the row vectors X_i A)
 //   c[m]          = sum_g x[m, g d .. g d + d - 1] . B  (the X_i B terms)
-// so the codes are never turned into weights. Each code z becomes the byte z,
-// which is exactly the e4m3 subnormal z * 2^-9; one shift and one AND expand
-// four codes (layout.h) and tcgen05.st writes them as the A operand of
-// tcgen05.mma.kind::f8f6f4 (128 rows in TMEM lanes). The folded activations,
-// scaled per token by 2^P so that |x' 2^P| < 256, are split into three e4m3
-// terms h + m + l (about 12 significant bits, the precision of fp16) that
-// form three B operands in 128B-swizzled shared memory and accumulate into the
-// same fp32 TMEM accumulator; the epilogue multiplies by 2^(9 - P).
+// so the codes are never turned into weights.
 //
-// CTA = 128 output rows x one K slice; the KS CTAs sharing the rows form a
-// thread-block cluster and add their partial sums through distributed shared
-// memory. Warp roles (10 warps):
-//   0      producer: 4 KB code tiles -> shared-memory ring (cp.async.bulk)
-//   1      TMEM owner; one thread issues the MMAs
-//   2..5   converters: shared ring -> TMEM A slots (two units of 16 rows per
-//          warp), then the epilogue (tcgen05.ld of their 32 accumulator rows)
-//   6..9   fold: x -> per-token scale, x' = x_g A, three e4m3 B terms
-// Producer and converters never touch x, so they run before the programmatic-
-// launch wait: while the previous kernel finishes, this layer's codes already
-// stream into shared memory and TMEM.
+// Operands. A code z becomes a byte of an e4m3 A operand: with w a code word
+// (columns 16t + 4s + b at bits 8b + 2s, layout.h),
+//   w & 0x03030303        bytes z          (columns s = 0, e4m3 z * 2^-9)
+//   w & 0x0c0c0c0c        bytes 4 z        (s = 1, e4m3 4z * 2^-9: bytes 0..15
+//   (w >> 4) & 0x03030303 bytes z           are exact, subnormal or first binade)
+//   (w >> 4) & 0x0c0c0c0c bytes 4 z        (s = 3)
+// one shift and four ANDs for 16 codes; the factor 4 of odd s is taken out of
+// the B operand. tcgen05.st writes the bytes into a TMEM A slot (128 rows in
+// the 128 TMEM lanes, 32 columns of four bytes per k-tile). The folded
+// activations, scaled per token and K slice by 2^P (|x' 2^P| < 256), are
+// split into three e4m3 terms h + m + l (about 12 significant bits, the
+// precision of fp16); the terms of token m are B rows 3m, 3m+1, 3m+2, so one
+// MMA of N = 16/32/48 columns covers every term of up to 5/10/16 tokens and a
+// 128 x 128 k-tile takes four tcgen05.mma.kind::f8f6f4 (K = 32). The epilogue
+// adds the three term columns of a token and multiplies by 2^(9 - P).
+//
+// Two kernels per launch:
+//  fold_kernel    one CTA per (K slice, token, layer): scale 2^P and c over the
+//                 slice, then the B tiles of the slice, in the exact image of
+//                 the 128B-swizzled shared-memory operand, into the layer's
+//                 fold workspace (device memory owned by the handle). The fold
+//                 is done once per launch instead of once per row block.
+//  decode_kernel  CTA = 128 output rows x one K slice; the KS CTAs sharing the
+//                 rows form a thread-block cluster and add their partial sums
+//                 in distributed shared memory. Pipeline stages hold two
+//                 k-tiles: 8 KB of codes and the two B tiles. Warp roles (10):
+//     0      producer: code and B stages -> shared-memory ring (cp.async.bulk)
+//     1      TMEM owner; one thread issues the MMAs
+//     2..9   converters: shared ring -> TMEM A slots; warp w serves TMEM lane
+//            quarter w % 4 (rows 32 (w%4) ..) for every other stage; warps
+//            2..5 then run the epilogue (tcgen05.ld of their 32 rows)
+// The codes never depend on the previous kernel: the producer fetches the
+// first stages of codes before the programmatic-launch wait and the B tiles
+// after it, so codes stream while the fold kernel runs. Layers that share x
+// (same K) run in one launch of each kernel: their row blocks are stacked
+// along grid.y of decode_kernel, their folds along grid.z of fold_kernel.
 #include "common.cuh"
 #include "internal.h"
 
 namespace unisvq {
 namespace {
 
-constexpr int kThreads = 10 * 32;
-constexpr int kFoldWarp0 = 6;
+constexpr int kWarps = 10;
+constexpr int kThreads = kWarps * 32;
+constexpr int kConvWarp0 = 2;
+constexpr int kConvWarps = 8;
+constexpr int kStageTiles = 2;                      // k-tiles per pipeline stage
+constexpr int kCodeBytes = kStageTiles * kTileBytes;
+constexpr int kASlots = 3;                          // TMEM A slots (one stage each)
+constexpr int kAColBase = 64;                       // accumulator in [0, 64)
+constexpr int kASlotCols = 32 * kStageTiles;
 constexpr int kTmemCols = 256;
-constexpr int kAColBase = 64;        // A slots start here; the accumulator uses [0, NTOK)
-constexpr int kASlots = (kTmemCols - kAColBase) / 32;
-constexpr int kMaxTokPerLaunch = 64;
+constexpr int kMaxTokPerLaunch = 16;
+constexpr int kMaxSplit = 8;                        // K slices (cluster size)
+constexpr int kMaxGroup = UNISVQ_MAX_GROUP;
+constexpr int kFoldThreads = 256;
+static_assert(kAColBase + kASlots * kASlotCols <= kTmemCols, "TMEM columns");
+static_assert(kConvWarps / 4 <= kASlots, "converter groups must not run two slot uses ahead");
 
-struct DecodeArgs {
+// Fold workspace of a handle (unisvq_layer::fold_ws): a table of per-(slice,
+// token) scale exponents and bias sums, then the B tiles of every k-tile.
+constexpr int kWsTableBytes = 1024;                 // int pexp[8][16], float cpart[8][16]
+constexpr int kWsTileStride = 48 * 128;             // B tile bytes per k-tile at the widest N
+
+struct SkLayer {
   const uint8_t* codes;
-  const uint16_t* x;   // bf16 [M][K]
+  const uint8_t* ws;   // fold workspace (B tiles at kWsTableBytes)
   uint16_t* y;         // bf16 [M][N]
-  int M, N, K, KT, d;
-  int kt_per_cta;
-  float A[16];
-  float B[4];
-  float colnorm;       // max_c sum_r |A[r][c]|
-  int* err;
+  int N;
+  int rb0;             // first grid.y row block of this layer
 };
 
-template <int NTOK>
+struct SkArgs {
+  int M, KT;
+  int kt_per_cta;
+  int nlayers;
+  int* err;
+  SkLayer layer[kMaxGroup];
+};
+
+struct FoldLayer {
+  uint8_t* ws;
+  int d;
+  float colnorm;       // max_c sum_r |A[r][c]|
+  float A[16];
+  float B[4];
+};
+
+struct FoldArgs {
+  const uint16_t* x;   // bf16 [M][K]
+  int M, K, KT;
+  int kt_per_cta;
+  int ncol;            // B rows (16, 32, 48)
+  int nlayers;
+  FoldLayer layer[kMaxGroup];
+};
+
+template <int NCOL>
 struct Cfg {
-  static constexpr int kCodeStages = NTOK == 64 ? 4 : 8;
-  static constexpr int kBStages = NTOK == 16 ? 4 : 2;
-  static constexpr int kTermBytes = NTOK * 128;                  // one e4m3 B tile (128 columns)
-  static constexpr int kBStageBytes = 3 * kTermBytes;
-  static constexpr int kOffCode = 0;
-  static constexpr int kOffB = kOffCode + kCodeStages * kTileBytes;
-  static constexpr int kOffX = kOffB + kBStages * kBStageBytes;
-  static constexpr int kXBytes = NTOK == 64 ? 8192 : 32768;      // staged x slice (bf16)
-  static constexpr int kOffRed = kOffX + kXBytes;
-  static constexpr int kRedBytes = (kTileRows + 8) * NTOK * 4;
-  static constexpr int kOffBars = kOffRed + kRedBytes;
-  static constexpr int kNumBars = 2 * kCodeStages + 2 * kASlots + 2 * kBStages + 4;
-  static constexpr int kOffTok = kOffBars + kNumBars * 8;        // pexp[64], cpart[64]
-  static constexpr int kOffMisc = kOffTok + 512;                 // tmem ptr, abort flag
+  static constexpr int kMaxTok = NCOL / 3;
+  static constexpr int kStages = NCOL == 48 ? 4 : 6;
+  static constexpr int kBTile = NCOL * 128;                      // one k-tile of B (NCOL rows x 128 bytes)
+  static constexpr int kBBytes = kStageTiles * kBTile;
+  static constexpr int kStageBytes = kCodeBytes + kBBytes;       // [codes | B tiles]
+  static constexpr int kOffRed = kStages * kStageBytes;
+  static constexpr int kRedBytes = (kTileRows + 8) * kMaxTok * 4;
+  static constexpr int kOffBars = kOffRed + (kRedBytes + 15) / 16 * 16;
+  static constexpr int kNumBars = 4 * kStages + 2 * kASlots + 3;
+  static constexpr int kOffTok = kOffBars + kNumBars * 8;        // pexp[16], cpart[16]
+  static constexpr int kOffMisc = kOffTok + 128;                 // tmem ptr, abort flag
   static constexpr int kSmem = kOffMisc + 64 + 1024;             // + alignment slack
+  // kind::f8f6f4: D f32, A and B e4m3, both K-major, N = NCOL, M = 128.
   static constexpr uint32_t kIdesc =
-      (1u << 4) | (0u << 7) | (0u << 10) | (static_cast<uint32_t>(NTOK >> 3) << 17) | ((128u >> 4) << 24);
+      (1u << 4) | (static_cast<uint32_t>(NCOL >> 3) << 17) | ((128u >> 4) << 24);
+  static_assert(kStageBytes % 1024 == 0 && kBTile % 1024 == 0, "128B-swizzled B tiles need 1024-byte alignment");
+  static_assert(kStages % (kConvWarps / 4) == 0, "a converter group revisits its own stages");
 };
 
 // ---- tcgen05 wrappers ----------------------------------------------------------
@@ -76,6 +130,7 @@ struct Cfg {
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups 1024 bytes apart.
 __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
   return static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4) | (static_cast<uint64_t>(1) << 16) |
          (static_cast<uint64_t>(1024 >> 4) << 32) | (static_cast<uint64_t>(1) << 46) |
@@ -116,6 +171,27 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
       : "r"(taddr));
 }
 
+// The 16 A-slot words of one lane for one 16-row unit. c holds the words of rows
+// g (c.x half 0, c.z half 1) and g + 8 (c.y, c.w) for column quarter t. Word
+// (h, s) of row g goes to v[4k + e], of row g + 8 to v[4k + 2 + e], with
+// k = 2h + s/2 and e = s % 2: TMEM column 16h + 8(s/2) + 2t + s%2 of the slot
+// holds the four columns 64h + 16t + 4s + (0..3) (times 4 for odd s).
+__device__ __forceinline__ void expand_unit(uint4 c, uint32_t (&v)[16]) {
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const uint32_t wg = h ? c.z : c.x, wg8 = h ? c.w : c.y;
+    const uint32_t sg = wg >> 4, sg8 = wg8 >> 4;
+    v[8 * h + 0] = wg & 0x03030303u;    // k = 2h,     e = 0: s = 0
+    v[8 * h + 1] = wg & 0x0c0c0c0cu;    // k = 2h,     e = 1: s = 1
+    v[8 * h + 2] = wg8 & 0x03030303u;
+    v[8 * h + 3] = wg8 & 0x0c0c0c0cu;
+    v[8 * h + 4] = sg & 0x03030303u;    // k = 2h + 1, e = 0: s = 2
+    v[8 * h + 5] = sg & 0x0c0c0c0cu;    // k = 2h + 1, e = 1: s = 3
+    v[8 * h + 6] = sg8 & 0x03030303u;
+    v[8 * h + 7] = sg8 & 0x0c0c0c0cu;
+  }
+}
+
 // e4m3x2 <-> f16x2 (lower byte <-> lower half).
 __device__ __forceinline__ uint16_t f16x2_to_e4m3x2(uint32_t v) {
   uint16_t r;
@@ -143,34 +219,155 @@ __device__ __forceinline__ void split3(uint32_t v, uint16_t& h, uint16_t& m, uin
 }
 
 // x'[k+c] for the d-vectors inside x[k .. k+3] (k % 4 == 0): row vector x_g A.
-__device__ __forceinline__ void fold4(const DecodeArgs& a, const float (&v)[4], float (&o)[4]) {
-  if (a.d == 1) {
+__device__ __forceinline__ void fold4(int d, const float (&A)[16], const float (&v)[4], float (&o)[4]) {
+  if (d == 1) {
 #pragma unroll
-    for (int e = 0; e < 4; ++e) o[e] = v[e] * a.A[0];
-  } else if (a.d == 2) {
-    o[0] = fmaf(v[1], a.A[2], v[0] * a.A[0]);
-    o[1] = fmaf(v[1], a.A[3], v[0] * a.A[1]);
-    o[2] = fmaf(v[3], a.A[2], v[2] * a.A[0]);
-    o[3] = fmaf(v[3], a.A[3], v[2] * a.A[1]);
+    for (int e = 0; e < 4; ++e) o[e] = v[e] * A[0];
+  } else if (d == 2) {
+    o[0] = fmaf(v[1], A[2], v[0] * A[0]);
+    o[1] = fmaf(v[1], A[3], v[0] * A[1]);
+    o[2] = fmaf(v[3], A[2], v[2] * A[0]);
+    o[3] = fmaf(v[3], A[3], v[2] * A[1]);
   } else {
 #pragma unroll
     for (int c = 0; c < 4; ++c)
-      o[c] = fmaf(v[3], a.A[12 + c], fmaf(v[2], a.A[8 + c], fmaf(v[1], a.A[4 + c], v[0] * a.A[c])));
+      o[c] = fmaf(v[3], A[12 + c], fmaf(v[2], A[8 + c], fmaf(v[1], A[4 + c], v[0] * A[c])));
   }
 }
 
-// Activations x[k .. k+3] of one token as packed bf16 (zero at or past kend).
-__device__ __forceinline__ uint2 load_x4(const uint16_t* row, int k, int kend, bool vec) {
-  if (vec && k + 3 < kend) return ldg_v2(row + k);
-  uint32_t e[4];
+// Fold of one K slice for one token of one layer: the scale 2^P and the bias
+// sum c over the slice, then the slice's B tiles (rows 3 tok .. 3 tok + 2) in
+// the layer's workspace. Rows of absent tokens are never written: an MMA
+// column depends on its own B row only, and the epilogue never reads those
+// columns.
+__global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constant__ FoldArgs a) {
+  extern __shared__ __align__(16) uint8_t fsm[];
+  uint16_t* xs = reinterpret_cast<uint16_t*>(fsm);   // the token's x slice, zero past K
+  __shared__ float wmx[kFoldThreads / 32], wcs[kFoldThreads / 32];
+  __shared__ int sp;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int s = blockIdx.x, tok = blockIdx.y, li = blockIdx.z;
+  // This CTA's layer, read with constant parameter offsets only.
+  uint8_t* ws = a.layer[0].ws;
+  int d = a.layer[0].d;
+  float colnorm = a.layer[0].colnorm;
+  float A[16], Bv[4];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) e[j] = (k + j < kend) ? static_cast<uint32_t>(row[k + j]) : 0u;
-  return make_uint2(e[0] | (e[1] << 16), e[2] | (e[3] << 16));
+  for (int i = 0; i < 16; ++i) A[i] = a.layer[0].A[i];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) Bv[i] = a.layer[0].B[i];
+#pragma unroll
+  for (int l = 1; l < kMaxGroup; ++l)
+    if (l == li) {
+      ws = a.layer[l].ws;
+      d = a.layer[l].d;
+      colnorm = a.layer[l].colnorm;
+#pragma unroll
+      for (int i = 0; i < 16; ++i) A[i] = a.layer[l].A[i];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) Bv[i] = a.layer[l].B[i];
+    }
+  const int kt0 = s * a.kt_per_cta;
+  const int n_kt = min(a.kt_per_cta, a.KT - kt0);
+  pdl_launch_dependents();   // the decode kernel may start fetching codes
+  if (n_kt <= 0 || tok >= a.M || li >= a.nlayers) return;
+  // x is the previous kernel's output, and the previous launch on this handle
+  // may still read the workspace: both wait for the previous kernel.
+  pdl_wait();
+  const int kbeg = kt0 * kTileCols;
+  const int kend = min(a.K, (kt0 + n_kt) * kTileCols);
+  const int span = n_kt * kTileCols;
+  const bool vec8 = (a.K & 7) == 0;
+  const uint16_t* row = a.x + static_cast<size_t>(tok) * a.K;
+  float mx = 0.f, cs = 0.f;
+  for (int c0 = tid * 8; c0 < span; c0 += kFoldThreads * 8 * 4) {
+    uint4 u[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int k = kbeg + c0 + j * kFoldThreads * 8;
+      if (vec8 && k + 7 < kend) {
+        u[j] = ldg_v4(row + k);
+      } else {
+        uint32_t e[8];
+#pragma unroll
+        for (int t = 0; t < 8; ++t) e[t] = (k + t < kend) ? static_cast<uint32_t>(row[k + t]) : 0u;
+        u[j] = make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int c = c0 + j * kFoldThreads * 8;
+      if (c >= span) break;
+      *reinterpret_cast<uint4*>(xs + c) = u[j];
+      const uint32_t w4[4] = {u[j].x, u[j].y, u[j].z, u[j].w};
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {   // kbeg and c are multiples of 8: (k + i) mod d = i mod d
+        const float v0 = bf16_lo(w4[t]), v1 = bf16_hi(w4[t]);
+        mx = fmaxf(mx, fmaxf(fabsf(v0), fabsf(v1)));
+        cs = fmaf(v0, Bv[(2 * t) & (d - 1)], cs);
+        cs = fmaf(v1, Bv[(2 * t + 1) & (d - 1)], cs);
+      }
+    }
+  }
+#pragma unroll
+  for (int off = 16; off; off >>= 1) {
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    cs += __shfl_xor_sync(0xffffffffu, cs, off);
+  }
+  if (lane == 0) {
+    wmx[warp] = mx;
+    wcs[warp] = cs;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    float tmx = 0.f, tcs = 0.f;
+    for (int w = 0; w < kFoldThreads / 32; ++w) {
+      tmx = fmaxf(tmx, wmx[w]);
+      tcs += wcs[w];
+    }
+    // 2^P puts the largest possible |x'| (<= max|x| * colnorm) below 2^8.
+    const float bound = tmx * colnorm;
+    int e2 = 0;
+    if (bound > 0.f) frexpf(bound, &e2);
+    const int P = bound > 0.f ? max(-100, min(100, 8 - e2)) : 0;
+    sp = P;
+    reinterpret_cast<int*>(ws)[s * 16 + tok] = P;
+    reinterpret_cast<float*>(ws + 512)[s * 16 + tok] = tcs;
+  }
+  __syncthreads();
+  const int P = sp;
+  const int ncol = a.ncol;
+  uint8_t* tiles = ws + kWsTableBytes + static_cast<size_t>(kt0) * ncol * 128;
+  // Item (k-tile kt, column group g): columns 4g .. 4g + 3 of the tile, i.e.
+  // quarter t = (g/4) % 4, s = g % 4, half h = g / 16, which sit in A-slot
+  // column ac = 16h + 8(s/2) + 2t + s%2 (expand_unit): bytes 4 ac .. 4 ac + 3
+  // of the 128-byte B row; odd s carries the factor 1/4.
+  for (int item = tid; item < n_kt * 32; item += kFoldThreads) {
+    const int kt = item >> 5, g = item & 31;
+    const uint32_t ac = 16 * (g >> 4) + 8 * ((g & 3) >> 1) + 2 * ((g >> 2) & 3) + (g & 1);
+    const uint32_t cidx = (ac & 3) * 4, chunk = ac >> 2;
+    const uint2 xv = *reinterpret_cast<const uint2*>(xs + kt * kTileCols + 4 * g);
+    const float v[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
+    float o[4];
+    fold4(d, A, v, o);
+    const float sc = exp2i(P + ((g & 1) ? -2 : 0));
+    uint16_t h0, m0, l0, h1, m1, l1;
+    split3(pack_half2(o[0] * sc, o[1] * sc), h0, m0, l0);
+    split3(pack_half2(o[2] * sc, o[3] * sc), h1, m1, l1);
+    uint8_t* bt = tiles + static_cast<size_t>(kt) * ncol * 128;
+    const int r = 3 * tok;
+    *reinterpret_cast<uint32_t*>(bt + r * 128 + ((chunk ^ (r & 7)) << 4) + cidx) = h0 | (static_cast<uint32_t>(h1) << 16);
+    *reinterpret_cast<uint32_t*>(bt + (r + 1) * 128 + ((chunk ^ ((r + 1) & 7)) << 4) + cidx) =
+        m0 | (static_cast<uint32_t>(m1) << 16);
+    *reinterpret_cast<uint32_t*>(bt + (r + 2) * 128 + ((chunk ^ ((r + 2) & 7)) << 4) + cidx) =
+        l0 | (static_cast<uint32_t>(l1) << 16);
+  }
 }
 
-template <int NTOK>
-__global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_constant__ DecodeArgs a) {
-  using C = Cfg<NTOK>;
+template <int NCOL>
+__global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_constant__ SkArgs a) {
+  using C = Cfg<NCOL>;
+  constexpr int S = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024 - (raw & 1023)) & 1023);
@@ -180,42 +377,60 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
   const int KS = gridDim.x;
   const int kt0 = blockIdx.x * a.kt_per_cta;
   const int n_kt = min(a.kt_per_cta, a.KT - kt0);
-  const int rb = blockIdx.y;
+  const int n_st = (n_kt + kStageTiles - 1) / kStageTiles;
+  const int M = a.M;
+  // This CTA's layer, read with constant parameter offsets only.
+  int li = 0;
+#pragma unroll
+  for (int i = 1; i < kMaxGroup; ++i)
+    if (i < a.nlayers && static_cast<int>(blockIdx.y) >= a.layer[i].rb0) li = i;
+  const uint8_t* lcodes = a.layer[0].codes;
+  const uint8_t* lws = a.layer[0].ws;
+  uint16_t* ly = a.layer[0].y;
+  int lN = a.layer[0].N, lrb0 = a.layer[0].rb0;
+#pragma unroll
+  for (int i = 1; i < kMaxGroup; ++i)
+    if (i == li) {
+      lcodes = a.layer[i].codes;
+      lws = a.layer[i].ws;
+      ly = a.layer[i].y;
+      lN = a.layer[i].N;
+      lrb0 = a.layer[i].rb0;
+    }
+  const int rb = static_cast<int>(blockIdx.y) - lrb0;
 
   const uint32_t bar0 = sbase + C::kOffBars;
-  auto code_full = [&](int s) { return bar0 + 8u * s; };
-  auto code_empty = [&](int s) { return bar0 + 8u * (C::kCodeStages + s); };
-  auto a_full = [&](int s) { return bar0 + 8u * (2 * C::kCodeStages + s); };
-  auto a_empty = [&](int s) { return bar0 + 8u * (2 * C::kCodeStages + kASlots + s); };
-  auto b_full = [&](int s) { return bar0 + 8u * (2 * C::kCodeStages + 2 * kASlots + s); };
-  auto b_empty = [&](int s) { return bar0 + 8u * (2 * C::kCodeStages + 2 * kASlots + C::kBStages + s); };
-  const uint32_t bar_tail = bar0 + 8u * (2 * C::kCodeStages + 2 * kASlots + 2 * C::kBStages);
-  const uint32_t d_full = bar_tail, tmem_ready = bar_tail + 8, fold_done = bar_tail + 16, drain = bar_tail + 24;
+  auto cfull = [&](int s) { return bar0 + 8u * s; };
+  auto bfull = [&](int s) { return bar0 + 8u * (S + s); };
+  auto cempty = [&](int s) { return bar0 + 8u * (2 * S + s); };
+  auto bempty = [&](int s) { return bar0 + 8u * (3 * S + s); };
+  auto a_full = [&](int s) { return bar0 + 8u * (4 * S + s); };
+  auto a_empty = [&](int s) { return bar0 + 8u * (4 * S + kASlots + s); };
+  const uint32_t bar_tail = bar0 + 8u * (4 * S + 2 * kASlots);
+  const uint32_t d_full = bar_tail, tmem_ready = bar_tail + 8, drain = bar_tail + 16;
   int* pexp = reinterpret_cast<int*>(smem + C::kOffTok);
-  float* cpart = reinterpret_cast<float*>(smem + C::kOffTok + 256);
+  float* cpart = reinterpret_cast<float*>(smem + C::kOffTok + 64);
   uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 8);
   float* red = reinterpret_cast<float*>(smem + C::kOffRed);
 
   if (tid == 0) {
-    for (int s = 0; s < C::kCodeStages; ++s) {
-      mbar_init(code_full(s), 1);
-      mbar_init(code_empty(s), 4);
+    for (int s = 0; s < S; ++s) {
+      mbar_init(cfull(s), 1);
+      mbar_init(bfull(s), 1);
+      mbar_init(cempty(s), 4);
+      mbar_init(bempty(s), 1);
     }
     for (int s = 0; s < kASlots; ++s) {
       mbar_init(a_full(s), 4);
       mbar_init(a_empty(s), 1);
     }
-    for (int s = 0; s < C::kBStages; ++s) {
-      mbar_init(b_full(s), 1);
-      mbar_init(b_empty(s), 1);
-    }
     mbar_init(d_full, 1);
     mbar_init(tmem_ready, 1);
-    mbar_init(fold_done, 4);
     mbar_init(drain, 1);
-    *abort_flag = n_kt <= 0 ? 1 : 0;
-    if (n_kt <= 0) record_error(a.err, kErrBadLaunch);
+    const bool bad = n_kt <= 0 || M < 1 || M > C::kMaxTok;
+    *abort_flag = bad ? 1 : 0;
+    if (bad) record_error(a.err, kErrBadLaunch);
     fence_mbar_init();
   }
   __syncthreads();
@@ -223,26 +438,48 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
   pdl_launch_dependents();
 
   if (warp == 0) {
-    // ---------------- producer: code tiles -> shared ring ----------------
+    // ---------------- producer: code and B stages -> shared ring ----------------
     if (lane == 0 && !*abort_flag) {
       const uint64_t pol = policy_evict_first();
-      const uint8_t* src = a.codes + (static_cast<size_t>(rb) * a.KT + kt0) * kTileBytes;
-      int kt = 0;
-      for (; kt < n_kt; ++kt) {
-        const int s = kt % C::kCodeStages;
-        if (kt >= C::kCodeStages &&
-            !mbar_wait(code_empty(s), ((kt / C::kCodeStages) - 1) & 1, a.err, kErrTimeoutEmpty)) {
+      const uint8_t* csrc = lcodes + (static_cast<size_t>(rb) * a.KT + kt0) * kTileBytes;
+      const uint8_t* bsrc = lws + kWsTableBytes + static_cast<size_t>(kt0) * C::kBTile;
+      const int pre = min(S, n_st);
+      // Codes of the first stages do not depend on the previous kernels.
+      for (int st = 0; st < pre; ++st) {
+        const uint32_t nt = static_cast<uint32_t>(min(kStageTiles, n_kt - st * kStageTiles));
+        mbar_arrive_expect_tx(cfull(st), nt * kTileBytes);
+        bulk_g2s(sbase + st * C::kStageBytes, csrc + static_cast<size_t>(st) * kCodeBytes, nt * kTileBytes,
+                 cfull(st), pol);
+      }
+      pdl_wait();   // the B tiles come from the fold kernel
+      for (int st = 0; st < pre; ++st) {
+        const uint32_t nt = static_cast<uint32_t>(min(kStageTiles, n_kt - st * kStageTiles));
+        mbar_arrive_expect_tx(bfull(st), nt * C::kBTile);
+        bulk_g2s(sbase + st * C::kStageBytes + kCodeBytes, bsrc + static_cast<size_t>(st) * C::kBBytes,
+                 nt * C::kBTile, bfull(st), pol);
+      }
+      int st = pre;
+      for (; st < n_st; ++st) {
+        const int s = st % S;
+        const uint32_t par = ((st / S) - 1) & 1;
+        if (!mbar_wait(cempty(s), par, a.err, kErrTimeoutEmpty) || !mbar_wait(bempty(s), par, a.err, kErrTimeoutEmpty)) {
           *abort_flag = 1;
           break;
         }
         if (*abort_flag) break;
-        mbar_arrive_expect_tx(code_full(s), kTileBytes);
-        bulk_g2s(sbase + C::kOffCode + s * kTileBytes, src + static_cast<size_t>(kt) * kTileBytes, kTileBytes,
-                 code_full(s), pol);
+        const uint32_t nt = static_cast<uint32_t>(min(kStageTiles, n_kt - st * kStageTiles));
+        mbar_arrive_expect_tx(cfull(s), nt * kTileBytes);
+        bulk_g2s(sbase + s * C::kStageBytes, csrc + static_cast<size_t>(st) * kCodeBytes, nt * kTileBytes, cfull(s),
+                 pol);
+        mbar_arrive_expect_tx(bfull(s), nt * C::kBTile);
+        bulk_g2s(sbase + s * C::kStageBytes + kCodeBytes, bsrc + static_cast<size_t>(st) * C::kBBytes,
+                 nt * C::kBTile, bfull(s), pol);
       }
       if (*abort_flag)   // copies nobody consumed must land before exit
-        for (int j = kt - C::kCodeStages > 0 ? kt - C::kCodeStages : 0; j < kt; ++j)
-          mbar_wait(code_full(j % C::kCodeStages), (j / C::kCodeStages) & 1, a.err, kErrTimeoutFull);
+        for (int j = st - S > 0 ? st - S : 0; j < st; ++j) {
+          mbar_wait(cfull(j % S), (j / S) & 1, a.err, kErrTimeoutFull);
+          mbar_wait(bfull(j % S), (j / S) & 1, a.err, kErrTimeoutFull);
+        }
     }
   } else if (warp == 1) {
     // ---------------- TMEM owner + MMA issuer ----------------
@@ -258,73 +495,71 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
       tc_fence_after();
       const uint32_t tbase = *tmem_ptr;
       bool ok = !*abort_flag;
-      for (int kt = 0; kt < n_kt && ok; ++kt) {
-        const int sa = kt % kASlots, sb = kt % C::kBStages;
-        ok = !*abort_flag && mbar_wait(a_full(sa), (kt / kASlots) & 1, a.err, kErrTimeoutFull) &&
-             mbar_wait(b_full(sb), (kt / C::kBStages) & 1, a.err, kErrTimeoutFull);
+      for (int st = 0; st < n_st && ok; ++st) {
+        const int sa = st % kASlots, s = st % S;
+        ok = !*abort_flag && mbar_wait(a_full(sa), (st / kASlots) & 1, a.err, kErrTimeoutFull) &&
+             mbar_wait(bfull(s), (st / S) & 1, a.err, kErrTimeoutFull);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t acol = tbase + kAColBase + 32 * sa;
-        const uint32_t bst = sbase + C::kOffB + sb * C::kBStageBytes;
-#pragma unroll
-        for (int term = 0; term < 3; ++term) {
-          const uint64_t bd = sw128_desc(bst + term * C::kTermBytes);
+        const int nt = min(kStageTiles, n_kt - st * kStageTiles);
+        const uint32_t acol = tbase + kAColBase + kASlotCols * sa;
+        const uint32_t bst = sbase + s * C::kStageBytes + kCodeBytes;
+        for (int j = 0; j < nt; ++j) {
+          const uint64_t bd = sw128_desc(bst + j * C::kBTile);
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)   // K = 32 bytes per MMA inside the 128-byte swizzle row
-            mma_f8_tmem_a(tbase, acol + 8 * kk, bd + 2 * kk, C::kIdesc, (kt | term | kk) != 0 ? 1u : 0u);
+            mma_f8_tmem_a(tbase, acol + 32 * j + 8 * kk, bd + 2 * kk, C::kIdesc, (st | j | kk) != 0 ? 1u : 0u);
         }
         mma_commit(a_empty(sa));
-        mma_commit(b_empty(sb));
+        mma_commit(bempty(s));
       }
       if (ok) mma_commit(d_full);
       else *abort_flag = 1;
       mma_commit(drain);   // everything issued must retire before TMEM is released
       mbar_wait(drain, 0, a.err, kErrTimeoutMma);
     }
-  } else if (warp < kFoldWarp0) {
+  } else {
     // ---------------- converters: shared ring -> TMEM A slots ----------------
-    // Warp of TMEM lane quarter Q covers units 2Q and 2Q+1 (rows 32Q .. 32Q+31).
-    // Lane 4g + t reads the words of rows g and g + 8 of a unit for column
-    // quarter t (one 16-byte load, layout.h) and stores them as TMEM columns
-    // 8k + 2t + e of lanes g and g + 8, k = 2h + s/2, e = s % 2: the K order
-    // of the A slot is therefore a fixed permutation of the 128 columns, which
-    // the fold applies to the B operand as well (a_slot_col below).
-    const int q = warp & 3;                    // TMEM lane quarter
+    // Warp w serves TMEM lane quarter q = w % 4, i.e. units 2q and 2q + 1
+    // (rows 32q .. 32q + 31), for the stages of parity p.
+    const int cw = warp - kConvWarp0;
+    const int q = warp & 3, p = cw >> 2;
+    constexpr int kStep = kConvWarps / 4;
     bool ok = !*abort_flag && mbar_wait(tmem_ready, 0, a.err, kErrTimeoutFull);
     tc_fence_after();
-    const uint32_t tbase = *tmem_ptr;
-    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * q) << 16);
-    for (int kt = 0; kt < n_kt; ++kt) {
-      const int s = kt % C::kCodeStages, sa = kt % kASlots;
-      if (ok) ok = !*abort_flag && mbar_wait(code_full(s), (kt / C::kCodeStages) & 1, a.err, kErrTimeoutFull);
-      uint4 c0 = make_uint4(0, 0, 0, 0), c1 = c0;
-      if (ok) {
-        const uint8_t* tile = smem + C::kOffCode + s * kTileBytes + (2 * q) * kUnitBytes + lane * 16;
-        c0 = *reinterpret_cast<const uint4*>(tile);
-        c1 = *reinterpret_cast<const uint4*>(tile + kUnitBytes);
+    const uint32_t tq = *tmem_ptr + (static_cast<uint32_t>(32 * q) << 16);
+    for (int st = p; st < n_st; st += kStep) {
+      const int s = st % S, sa = st % kASlots;
+      if (ok) ok = !*abort_flag && mbar_wait(cfull(s), (st / S) & 1, a.err, kErrTimeoutFull);
+      const int nt = min(kStageTiles, n_kt - st * kStageTiles);
+      uint4 cu[kStageTiles][2];
+#pragma unroll
+      for (int j = 0; j < kStageTiles; ++j) {
+        cu[j][0] = make_uint4(0, 0, 0, 0);
+        cu[j][1] = cu[j][0];
+        if (ok && j < nt) {
+          const uint8_t* tile = smem + s * C::kStageBytes + j * kTileBytes + (2 * q) * kUnitBytes + lane * 16;
+          cu[j][0] = *reinterpret_cast<const uint4*>(tile);
+          cu[j][1] = *reinterpret_cast<const uint4*>(tile + kUnitBytes);
+        }
       }
       __syncwarp();
-      if (lane == 0 && ok) mbar_arrive(code_empty(s));
-      uint32_t v0[16], v1[16];
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const int h = k >> 1, s0 = 2 * (k & 1);
-        const uint32_t a0 = h ? c0.z : c0.x, a1 = h ? c0.w : c0.y;   // unit 2Q: rows g, g + 8
-        const uint32_t b0 = h ? c1.z : c1.x, b1 = h ? c1.w : c1.y;   // unit 2Q+1
-        v0[4 * k + 0] = extract4(a0, s0);
-        v0[4 * k + 1] = extract4(a0, s0 + 1);
-        v0[4 * k + 2] = extract4(a1, s0);
-        v0[4 * k + 3] = extract4(a1, s0 + 1);
-        v1[4 * k + 0] = extract4(b0, s0);
-        v1[4 * k + 1] = extract4(b0, s0 + 1);
-        v1[4 * k + 2] = extract4(b1, s0);
-        v1[4 * k + 3] = extract4(b1, s0 + 1);
-      }
-      if (ok && kt >= kASlots) ok = !*abort_flag && mbar_wait(a_empty(sa), ((kt / kASlots) - 1) & 1, a.err, kErrTimeoutMma);
+      if (lane == 0 && ok) mbar_arrive(cempty(s));
+      if (ok && st >= kASlots)
+        ok = !*abort_flag && mbar_wait(a_empty(sa), ((st / kASlots) - 1) & 1, a.err, kErrTimeoutMma);
       if (ok) {
         tc_fence_after();
-        tmem_st16x256b_x4(tq + kAColBase + 32 * sa, v0);
-        tmem_st16x256b_x4(tq + (16u << 16) + kAColBase + 32 * sa, v1);
+        const uint32_t col = kAColBase + kASlotCols * sa;
+#pragma unroll
+        for (int j = 0; j < kStageTiles; ++j) {
+          if (j < nt) {
+            uint32_t v[16];
+            expand_unit(cu[j][0], v);
+            tmem_st16x256b_x4(tq + col + 32 * j, v);
+            expand_unit(cu[j][1], v);
+            tmem_st16x256b_x4(tq + (16u << 16) + col + 32 * j, v);
+          }
+        }
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         tc_fence_before();
       }
@@ -333,154 +568,48 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
       if (!ok) *abort_flag = 1;
     }
 
-    // ---------------- epilogue: accumulator rows -> cluster reduction ----------------
-    const int r = 32 * q + lane;               // accumulator row (TMEM lane) of this thread
-    const uint32_t trow = tq;
-    if (ok) ok = !*abort_flag && mbar_wait(d_full, 0, a.err, kErrTimeoutMma);
-    if (ok) ok = mbar_wait(fold_done, 0, a.err, kErrTimeoutFull);
-    if (!ok) *abort_flag = 1;
-    const int rows_per = (kTileRows + KS - 1) / KS;
-    const int owner = r / rows_per;
-    const uint32_t slot_off =
-        (static_cast<uint32_t>(blockIdx.x) * rows_per + (r - owner * rows_per)) * NTOK * 4u;
-    const uint32_t red_addr = sbase + C::kOffRed;
-    if (KS > 1) cluster_wait();
-    tc_fence_after();
+    if (p == 0) {
+      // ---------------- epilogue: accumulator rows -> cluster reduction ----------------
+      const int r = 32 * q + lane;               // accumulator row (TMEM lane) of this thread
+      if (ok) ok = !*abort_flag && mbar_wait(d_full, 0, a.err, kErrTimeoutMma);
+      if (!ok) *abort_flag = 1;
+      pdl_wait();   // the scale table comes from the fold kernel
+      if (q == 0 && lane < M) {
+        pexp[lane] = reinterpret_cast<const int*>(lws)[blockIdx.x * 16 + lane];
+        cpart[lane] = reinterpret_cast<const float*>(lws + 512)[blockIdx.x * 16 + lane];
+      }
+      named_barrier_sync(1, 4 * 32);
+      const int rows_per = (kTileRows + KS - 1) / KS;
+      const int owner = r / rows_per;
+      const uint32_t slot_off =
+          (static_cast<uint32_t>(blockIdx.x) * rows_per + (r - owner * rows_per)) * C::kMaxTok * 4u;
+      const uint32_t red_addr = sbase + C::kOffRed;
+      if (KS > 1) cluster_wait();
+      tc_fence_after();
+      uint32_t dv[NCOL];
 #pragma unroll
-    for (int c0 = 0; c0 < NTOK; c0 += 16) {
-      uint32_t dv[16];
-      tmem_ld16(trow + c0, dv);
+      for (int c0 = 0; c0 < NCOL; c0 += 16) tmem_ld16(tq + c0, dv + c0);
       asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const int tok = c0 + j;
-        if (ok && tok < a.M) {
-          const float val = fmaf(__uint_as_float(dv[j]), exp2i(9 - pexp[tok]), cpart[tok]);
+      for (int tok = 0; tok < C::kMaxTok; ++tok) {
+        if (ok && tok < M) {
+          const float acc = __uint_as_float(dv[3 * tok]) + __uint_as_float(dv[3 * tok + 1]) +
+                            __uint_as_float(dv[3 * tok + 2]);
+          const float val = fmaf(acc, exp2i(9 - pexp[tok]), cpart[tok]);
           const uint32_t off = slot_off + tok * 4u;
           if (KS > 1) st_shared_cluster_f32(map_shared_rank(red_addr + off, owner), val);
           else red[off / 4] = val;
         }
       }
-    }
-    tc_fence_before();
-  } else {
-    // ---------------- fold: x -> scaled three-term e4m3 B tiles ----------------
-    const int fw = warp - kFoldWarp0;
-    // Fold warp fw < kBStages owns B stage fw (k-tiles kt = fw mod kBStages),
-    // so each stage has one writer and every wait on it is one phase behind.
-    // The owner zeroes the rows of tokens >= M once (those rows stay zero).
-    if (fw < C::kBStages)
-      for (int tok = a.M; tok < NTOK; ++tok)
-        for (int term = 0; term < 3; ++term)
-          reinterpret_cast<uint32_t*>(smem + C::kOffB + fw * C::kBStageBytes + term * C::kTermBytes + tok * 128)[lane] = 0u;
-    pdl_wait();   // x may be the previous kernel's output
-    const int kbeg = kt0 * kTileCols;
-    const int kend = min(a.K, (kt0 + n_kt) * kTileCols);
-    const int kspan = n_kt * kTileCols;                       // staged row length (bf16)
-    const bool vec8 = (a.K & 7) == 0;
-    const bool staged = a.M * kspan * 2 <= C::kXBytes;
-    uint16_t* xs = reinterpret_cast<uint16_t*>(smem + C::kOffX);
-    // Pass 1: per-token max |x| (scale) and sum_k x[k] B[k mod d] over the
-    // slice; warp fw owns tokens fw, fw+4, ...; 8 columns per lane per load,
-    // 8 loads in flight. The slice is kept in shared memory when it fits.
-    for (int tok = fw; tok < a.M; tok += 4) {
-      const uint16_t* row = a.x + static_cast<size_t>(tok) * a.K;
-      float mx = 0.f, cs = 0.f;
-      for (int k0 = kbeg + 8 * lane; k0 < kbeg + kspan; k0 += 8 * 32 * 8) {
-        uint4 u[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const int k = k0 + 256 * j;
-          if (vec8 && k + 7 < kend) {
-            u[j] = ldg_v4(row + k);
-          } else {
-            uint32_t e[8];
-#pragma unroll
-            for (int t = 0; t < 8; ++t) e[t] = (k + t < kend) ? static_cast<uint32_t>(row[k + t]) : 0u;
-            u[j] = make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
-          }
-        }
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const int k = k0 + 256 * j;
-          if (k >= kbeg + kspan) break;
-          if (staged) *reinterpret_cast<uint4*>(xs + tok * kspan + (k - kbeg)) = u[j];
-          const uint32_t w4[4] = {u[j].x, u[j].y, u[j].z, u[j].w};
-#pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            const float v0 = bf16_lo(w4[t]), v1 = bf16_hi(w4[t]);
-            mx = fmaxf(mx, fmaxf(fabsf(v0), fabsf(v1)));
-            cs = fmaf(v0, a.B[(2 * t) & (a.d - 1)], cs);
-            cs = fmaf(v1, a.B[(2 * t + 1) & (a.d - 1)], cs);
-          }
-        }
-      }
-#pragma unroll
-      for (int off = 16; off; off >>= 1) {
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-        cs += __shfl_xor_sync(0xffffffffu, cs, off);
-      }
-      if (lane == 0) {
-        // 2^P puts the largest possible |x'| (<= max|x| * colnorm) below 2^8.
-        const float bound = mx * a.colnorm;
-        int e2 = 0;
-        if (bound > 0.f) frexpf(bound, &e2);
-        pexp[tok] = bound > 0.f ? max(-100, min(100, 8 - e2)) : 0;
-        cpart[tok] = cs;
-      }
-    }
-    // All fold warps need every token's scale (and staged x) from here on.
-    named_barrier_sync(1, 4 * 32);
-    if (lane == 0) mbar_arrive(fold_done);
-
-    // Pass 2: warp fw folds k-tiles fw, fw + kBStages, ... (its own stage) for
-    // all tokens; lane covers columns 4 lane .. 4 lane + 3 of the k-tile.
-    bool ok = !*abort_flag;
-    // Columns 4 lane .. 4 lane + 3 = 64h + 16t + 4s + (0..3) sit in A-slot
-    // column 16h + 8(s/2) + 2t + s%2 (converter mapping), i.e. at bytes
-    // 4 * that column of each 128-byte B row.
-    const uint32_t a_slot_col = 16 * (lane >> 4) + 8 * ((lane & 3) >> 1) + 2 * ((lane >> 2) & 3) + (lane & 1);
-    const uint32_t cidx = (a_slot_col & 3) * 4;
-    const uint32_t chunk = a_slot_col >> 2;
-    for (int kt = fw; fw < C::kBStages && kt < n_kt; kt += C::kBStages) {
-      const int sb = fw;
-      const int use = kt / C::kBStages;      // how many times stage sb was filled before
-      if (ok && use > 0)
-        ok = !*abort_flag && mbar_wait(b_empty(sb), (use - 1) & 1, a.err, kErrTimeoutMma);
-      if (ok) {
-        uint8_t* bst = smem + C::kOffB + sb * C::kBStageBytes;
-        const int k = (kt0 + kt) * kTileCols + 4 * lane;
-        for (int tok = 0; tok < a.M; ++tok) {
-          uint2 xv;
-          if (staged) {
-            xv = *reinterpret_cast<const uint2*>(xs + tok * kspan + kt * kTileCols + 4 * lane);
-          } else {
-            xv = load_x4(a.x + static_cast<size_t>(tok) * a.K, k, kend, (a.K & 3) == 0);
-          }
-          const float v[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
-          float o[4];
-          fold4(a, v, o);
-          const float sc = exp2i(pexp[tok]);
-          uint16_t h0, m0, l0, h1, m1, l1;
-          split3(pack_half2(o[0] * sc, o[1] * sc), h0, m0, l0);
-          split3(pack_half2(o[2] * sc, o[3] * sc), h1, m1, l1);
-          const uint32_t off = tok * 128 + ((chunk ^ (tok & 7)) << 4) + cidx;
-          *reinterpret_cast<uint32_t*>(bst + off) = h0 | (static_cast<uint32_t>(h1) << 16);
-          *reinterpret_cast<uint32_t*>(bst + C::kTermBytes + off) = m0 | (static_cast<uint32_t>(m1) << 16);
-          *reinterpret_cast<uint32_t*>(bst + 2 * C::kTermBytes + off) = l0 | (static_cast<uint32_t>(l1) << 16);
-        }
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      }
-      __syncwarp();
-      if (lane == 0 && ok) mbar_arrive(b_full(sb));
-      if (!ok) *abort_flag = 1;
+      tc_fence_before();
     }
   }
 
   // ---------------- reduction over the K slices of the cluster ----------------
   __syncwarp();
+  const bool epilogue_warp = warp >= kConvWarp0 && warp < kConvWarp0 + 4;
   if (KS > 1) {
-    if (warp < 2 || warp >= kFoldWarp0) cluster_wait();   // converters waited before their stores
+    if (!epilogue_warp) cluster_wait();   // the epilogue warps waited before their stores
     cluster_sync();
   } else {
     __syncthreads();
@@ -489,13 +618,13 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
     const int rows_per = (kTileRows + KS - 1) / KS;
     const int r0 = static_cast<int>(blockIdx.x) * rows_per;
     const int nrows = max(0, min(kTileRows, r0 + rows_per) - r0);
-    for (int idx = tid; idx < nrows * a.M; idx += kThreads) {
+    for (int idx = tid; idx < nrows * M; idx += kThreads) {
       const int tok = idx / nrows;
       const int rl = idx - tok * nrows;
       const int n = rb * kTileRows + r0 + rl;
       float s = 0.f;
-      for (int qq = 0; qq < KS; ++qq) s += red[(qq * rows_per + rl) * NTOK + tok];
-      if (n < a.N) a.y[static_cast<size_t>(tok) * a.N + n] = f32_to_bf16_rn(s);
+      for (int qq = 0; qq < KS; ++qq) s += red[(qq * rows_per + rl) * C::kMaxTok + tok];
+      if (n < lN && !*abort_flag) ly[static_cast<size_t>(tok) * lN + n] = f32_to_bf16_rn(s);
     }
   }
   __syncthreads();
@@ -506,106 +635,164 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
   }
 }
 
-template <int NTOK>
-int resident_ctas_per_sm() {
-  static int n = 0;
-  if (!n) {
-    cudaFuncSetAttribute(decode_kernel<NTOK>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<NTOK>::kSmem);
-    cudaFuncSetAttribute(decode_kernel<NTOK>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                         cudaSharedmemCarveoutMaxShared);
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<NTOK>, kThreads, Cfg<NTOK>::kSmem) !=
-            cudaSuccess ||
-        n < 1)
-      n = 1;
-    // Each resident CTA holds kTmemCols of the 512 TMEM columns.
-    n = min(n, 512 / kTmemCols);
-  }
-  return n;
+int ncol_for(int M) { return M <= 5 ? 16 : (M <= 10 ? 32 : 48); }
+
+template <int NCOL>
+bool set_attrs(int dev) {
+  static bool done[64] = {};
+  if (dev < 0 || dev >= 64) return false;
+  if (done[dev]) return true;
+  if (cudaFuncSetAttribute(decode_kernel<NCOL>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<NCOL>::kSmem) !=
+          cudaSuccess ||
+      cudaFuncSetAttribute(decode_kernel<NCOL>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared) != cudaSuccess)
+    return false;
+  done[dev] = true;
+  return true;
 }
 
-template <int NTOK>
-unisvq_status launch_ntok(const unisvq_layer* L, const DecodePlan& p, const void* x, void* y, int M,
-                          cudaStream_t s) {
-  using C = Cfg<NTOK>;
-  static bool attr_set[64] = {};
-  const int dev = L->device;
-  if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
-  if (!attr_set[dev]) {
-    if (cudaFuncSetAttribute(decode_kernel<NTOK>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem) !=
-            cudaSuccess ||
-        cudaFuncSetAttribute(decode_kernel<NTOK>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                             cudaSharedmemCarveoutMaxShared) != cudaSuccess)
-      return UNISVQ_ERR_CUDA;
-    attr_set[dev] = true;
-  }
-  DecodeArgs a{};
-  a.codes = L->codes;
-  a.x = static_cast<const uint16_t*>(x);
-  a.y = static_cast<uint16_t*>(y);
-  a.M = M;
-  a.N = L->N;
-  a.K = L->K;
-  a.KT = L->KT;
-  a.d = L->d;
-  a.kt_per_cta = p.kt_per_cta;
-  for (int i = 0; i < 16; ++i) a.A[i] = L->A[i];
-  for (int i = 0; i < 4; ++i) a.B[i] = L->B[i];
-  a.colnorm = L->colnorm;
-  a.err = device_error_word();
+constexpr int kFoldMaxSmem = 96 * 1024;   // x slice of one token: <= 384 k-tiles
 
+bool set_fold_attrs(int dev) {
+  static bool done[64] = {};
+  if (dev < 0 || dev >= 64) return false;
+  if (done[dev]) return true;
+  if (cudaFuncSetAttribute(fold_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kFoldMaxSmem) != cudaSuccess)
+    return false;
+  done[dev] = true;
+  return true;
+}
+
+size_t smem_for(int ncol) { return ncol == 16 ? Cfg<16>::kSmem : (ncol == 32 ? Cfg<32>::kSmem : Cfg<48>::kSmem); }
+
+// Resident CTAs per SM: two when their shared memory fits (each holds half of
+// the 512 TMEM columns; 320 threads x <= 102 registers fit twice). The
+// occupancy query of the runtime reports one for this kernel although two
+// run side by side (measured), so the count is derived here.
+int resident_for(int ncol) {
+  return 2 * (smem_for(ncol) + 1024) <= static_cast<size_t>(228) * 1024 ? 2 : 1;
+}
+
+// Largest K split (cluster size <= 8, >= 1 k-tile per CTA) whose grid fits in
+// one wave of resident CTAs; at least enough slices for the fold kernel's
+// shared memory.
+DecodePlan plan_rows_split(int nb, int KT, int num_sms, int M) {
+  DecodePlan p{};
+  p.nt = ncol_for(M);
+  p.nb = nb;
+  const int slots = resident_for(p.nt) * num_sms;
+  const int min_ks = (KT * kTileCols * 2 + kFoldMaxSmem - 1) / kFoldMaxSmem;
+  int ks = 0;
+  for (int c = kMaxSplit; c >= 1; --c)
+    if (c <= KT && nb * c <= slots) {
+      ks = c;
+      break;
+    }
+  if (ks < min_ks) ks = min_ks;
+  if (ks < 1) ks = 1;
+  p.kt_per_cta = (KT + ks - 1) / ks;
+  p.ks = (KT + p.kt_per_cta - 1) / p.kt_per_cta;
+  p.smem = smem_for(p.nt);
+  return p;
+}
+
+cudaLaunchAttribute pdl_attr() {
+  cudaLaunchAttribute at;
+  at.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at.val.programmaticStreamSerializationAllowed = 1;
+  return at;
+}
+
+template <int NCOL>
+unisvq_status launch_ncol(const SkArgs& a, const DecodePlan& p, int dev, cudaStream_t s) {
+  if (!set_attrs<NCOL>(dev)) return UNISVQ_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.ks, p.nb, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = C::kSmem;
+  cfg.dynamicSmemBytes = Cfg<NCOL>::kSmem;
   cfg.stream = s;
   cudaLaunchAttribute attrs[2];
   attrs[0].id = cudaLaunchAttributeClusterDimension;
   attrs[0].val.clusterDim.x = p.ks;
   attrs[0].val.clusterDim.y = 1;
   attrs[0].val.clusterDim.z = 1;
-  attrs[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attrs[1].val.programmaticStreamSerializationAllowed = 1;
+  attrs[1] = pdl_attr();
   cfg.attrs = attrs;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, decode_kernel<NTOK>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+  return cudaLaunchKernelEx(&cfg, decode_kernel<NCOL>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
 }  // namespace
 
+size_t fold_workspace_bytes(int KT) { return kWsTableBytes + static_cast<size_t>(KT) * kWsTileStride; }
+
 DecodePlan plan_skinny(const unisvq_layer* L, int M) {
-  DecodePlan p{};
-  p.nt = M <= 16 ? 16 : (M <= 32 ? 32 : 64);
-  p.nb = L->Np / kTileRows;
-  const int occ = p.nt == 16 ? resident_ctas_per_sm<16>() : (p.nt == 32 ? resident_ctas_per_sm<32>()
-                                                                         : resident_ctas_per_sm<64>());
-  // Largest K split (cluster size <= 8, >= 1 k-tile per CTA) whose grid fits
-  // in one wave of resident CTAs.
-  const int slots = occ * L->num_sms;
-  int ks = 1;
-  for (int c = 8; c >= 1; --c)
-    if (c <= L->KT && p.nb * c <= slots) {
-      ks = c;
-      break;
-    }
-  p.kt_per_cta = (L->KT + ks - 1) / ks;
-  p.ks = (L->KT + p.kt_per_cta - 1) / p.kt_per_cta;
-  p.smem = p.nt == 16 ? Cfg<16>::kSmem : (p.nt == 32 ? Cfg<32>::kSmem : Cfg<64>::kSmem);
-  return p;
+  return plan_rows_split(L->Np / kTileRows, L->KT, L->num_sms, M > kMaxTokPerLaunch ? kMaxTokPerLaunch : M);
 }
 
-unisvq_status launch_skinny(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
+unisvq_status launch_skinny_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                                  cudaStream_t s) {
+  if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
+  const unisvq_layer* L0 = Ls[0];
+  if (!set_fold_attrs(L0->device)) return UNISVQ_ERR_CUDA;
+  int nb = 0;
+  for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
   for (int m0 = 0; m0 < M; m0 += kMaxTokPerLaunch) {
     const int mc = M - m0 < kMaxTokPerLaunch ? M - m0 : kMaxTokPerLaunch;
-    const DecodePlan p = plan_skinny(L, mc);
-    const void* xs = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * L->K;
-    void* ys = static_cast<uint16_t*>(y) + static_cast<size_t>(m0) * L->N;
+    const DecodePlan p = plan_rows_split(nb, L0->KT, L0->num_sms, mc);
+    if (p.ks > kMaxSplit) return UNISVQ_ERR_UNSUPPORTED;
+    FoldArgs f{};
+    f.x = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * L0->K;
+    f.M = mc;
+    f.K = L0->K;
+    f.KT = L0->KT;
+    f.kt_per_cta = p.kt_per_cta;
+    f.ncol = p.nt;
+    f.nlayers = n;
+    SkArgs a{};
+    a.M = mc;
+    a.KT = L0->KT;
+    a.kt_per_cta = p.kt_per_cta;
+    a.nlayers = n;
+    a.err = device_error_word();
+    int rb0 = 0;
+    for (int i = 0; i < n; ++i) {
+      const unisvq_layer* L = Ls[i];
+      FoldLayer& fl = f.layer[i];
+      fl.ws = L->fold_ws;
+      fl.d = L->d;
+      fl.colnorm = L->colnorm;
+      for (int j = 0; j < 16; ++j) fl.A[j] = L->A[j];
+      for (int j = 0; j < 4; ++j) fl.B[j] = L->B[j];
+      SkLayer& l = a.layer[i];
+      l.codes = L->codes;
+      l.ws = L->fold_ws;
+      l.y = static_cast<uint16_t*>(ys[i]) + static_cast<size_t>(m0) * L->N;
+      l.N = L->N;
+      l.rb0 = rb0;
+      rb0 += L->Np / kTileRows;
+    }
+    cudaLaunchConfig_t fc = {};
+    fc.gridDim = dim3(p.ks, mc, n);
+    fc.blockDim = dim3(kFoldThreads, 1, 1);
+    fc.dynamicSmemBytes = static_cast<size_t>(p.kt_per_cta) * kTileCols * 2;
+    fc.stream = s;
+    cudaLaunchAttribute fat[1] = {pdl_attr()};
+    fc.attrs = fat;
+    fc.numAttrs = 1;
+    if (cudaLaunchKernelEx(&fc, fold_kernel, f) != cudaSuccess) return UNISVQ_ERR_CUDA;
     unisvq_status st;
-    if (p.nt == 16) st = launch_ntok<16>(L, p, xs, ys, mc, s);
-    else if (p.nt == 32) st = launch_ntok<32>(L, p, xs, ys, mc, s);
-    else st = launch_ntok<64>(L, p, xs, ys, mc, s);
+    if (p.nt == 16) st = launch_ncol<16>(a, p, L0->device, s);
+    else if (p.nt == 32) st = launch_ncol<32>(a, p, L0->device, s);
+    else st = launch_ncol<48>(a, p, L0->device, s);
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;
+}
+
+unisvq_status launch_skinny(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
+  void* ys[1] = {y};
+  return launch_skinny_group(&L, 1, x, ys, M, s);
 }
 
 }  // namespace unisvq

@@ -22,6 +22,7 @@ struct unisvq_layer {
   float A[16];             // fp32 (exact) copy of A, row-major d x d
   float B[4];              // fp32 (exact) copy of B
   float colnorm;           // max_c sum_r |A[r][c]|: |x A|_inf <= |x|_inf * colnorm
+  uint8_t* fold_ws;        // device, decode fold workspace (fold_workspace_bytes(KT))
   uint16_t A16[16], B16[4];
 };
 
@@ -54,9 +55,14 @@ unisvq_status launch_gemv_rows_group(const unisvq_layer* const* Ls, int n, const
 // Several layers with the same K that read the same x, in one launch per 32 tokens.
 unisvq_status launch_gemv_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
                                 cudaStream_t s);
-// tcgen05 skinny GEMM with the codes as 8-bit TMEM operand (decode.cu), M <= 64 per launch.
+// tcgen05 skinny GEMM with the codes as 8-bit TMEM operand (decode.cu), M <= 16 per launch.
 DecodePlan plan_skinny(const unisvq_layer* L, int M);
 unisvq_status launch_skinny(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
+// Device bytes of a handle's fold workspace for the skinny decode kernel.
+size_t fold_workspace_bytes(int KT);
+// Several layers with the same K that read the same x, in one launch per 16 tokens.
+unisvq_status launch_skinny_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                                  cudaStream_t s);
 
 bool prefill_supported(const unisvq_layer* L, int M);
 PrefillPlan plan_prefill(const unisvq_layer* L, int M);

@@ -181,9 +181,13 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
   pack_codes_host(codes, N, K, packed.data());
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  L->fold_ws = nullptr;
+  const size_t ws_bytes = fold_workspace_bytes(L->KT);
   cudaError_t e = cudaMalloc(&L->codes, L->code_bytes);
   if (e == cudaSuccess) e = cudaMalloc(&L->lut32, lut32.size() * sizeof(float));
   if (e == cudaSuccess) e = cudaMalloc(&L->tlut, tlut.size() * sizeof(uint32_t));
+  if (e == cudaSuccess) e = cudaMalloc(&L->fold_ws, ws_bytes);
+  if (e == cudaSuccess) e = cudaMemsetAsync(L->fold_ws, 0, ws_bytes, s);
   if (e == cudaSuccess) e = cudaMemcpyAsync(L->codes, packed.data(), L->code_bytes, cudaMemcpyHostToDevice, s);
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(L->lut32, lut32.data(), lut32.size() * sizeof(float), cudaMemcpyHostToDevice, s);
@@ -195,6 +199,7 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
     cudaFree(L->codes);
     cudaFree(L->lut32);
     cudaFree(L->tlut);
+    cudaFree(L->fold_ws);
     delete L;
     return cuda_status(e);
   }
@@ -210,12 +215,16 @@ unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
   L->codes = nullptr;
   L->lut32 = nullptr;
   L->tlut = nullptr;
+  L->fold_ws = nullptr;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const size_t n32 = static_cast<size_t>(h->lut_entries) * h->d * sizeof(float);
   const size_t n16 = static_cast<size_t>(h->tlut_words) * sizeof(uint32_t);
+  const size_t ws_bytes = fold_workspace_bytes(h->KT);
   cudaError_t e = cudaMalloc(&L->codes, h->code_bytes);
   if (e == cudaSuccess) e = cudaMalloc(&L->lut32, n32);
   if (e == cudaSuccess) e = cudaMalloc(&L->tlut, n16);
+  if (e == cudaSuccess) e = cudaMalloc(&L->fold_ws, ws_bytes);
+  if (e == cudaSuccess) e = cudaMemsetAsync(L->fold_ws, 0, ws_bytes, s);
   if (e == cudaSuccess) e = cudaMemcpyAsync(L->codes, h->codes, h->code_bytes, cudaMemcpyDeviceToDevice, s);
   if (e == cudaSuccess) e = cudaMemcpyAsync(L->lut32, h->lut32, n32, cudaMemcpyDeviceToDevice, s);
   if (e == cudaSuccess) e = cudaMemcpyAsync(L->tlut, h->tlut, n16, cudaMemcpyDeviceToDevice, s);
@@ -224,6 +233,7 @@ unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
     cudaFree(L->codes);
     cudaFree(L->lut32);
     cudaFree(L->tlut);
+    cudaFree(L->fold_ws);
     delete L;
     return cuda_status(e);
   }
@@ -236,16 +246,18 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
   cudaError_t e1 = cudaFree(h->codes);
   cudaError_t e2 = cudaFree(h->lut32);
   cudaError_t e3 = cudaFree(h->tlut);
+  cudaError_t e4 = cudaFree(h->fold_ws);
   delete h;
-  return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess) ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+  return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess && e4 == cudaSuccess) ? UNISVQ_OK
+                                                                                             : UNISVQ_ERR_CUDA;
 }
 
 // Decode kernel for M <= 64 tokens over `weights` = sum of N*K of the layers
 // of one launch (measured crossovers on GB300): the whole-K row-slice GEMV for
 // one or two tokens on launches of at least 2^26 weights (no cross-CTA
 // reduction, many small CTAs), otherwise the K-split cluster GEMV (32 tokens
-// per launch). The tcgen05 skinny kernel is reachable through
-// unisvq_linear_force only: as built it is slower than the GEMV at every M.
+// per launch). The tcgen05 skinny kernel (fold kernel + streaming kernel) is
+// reachable through unisvq_linear_force / unisvq_linear_group_force.
 static int decode_kernel_for(const unisvq_layer* L, long long weights, int M) {
   if (M <= 2 && weights >= (1ll << 26) && gemv_rows_supported(L, M)) return UNISVQ_KERNEL_GEMV_ROWS;
   return UNISVQ_KERNEL_GEMV;
@@ -295,8 +307,8 @@ unisvq_status unisvq_linear(unisvq_handle h, const void* x, void* y, int M, void
   return unisvq_linear_force(h, UNISVQ_KERNEL_AUTO, x, y, M, stream);
 }
 
-unisvq_status unisvq_linear_group(const unisvq_handle* hs, int n, const void* x, void* const* ys, int M,
-                                  void* stream) {
+unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kernel, const void* x, void* const* ys,
+                                        int M, void* stream) {
   if (!hs || !ys || n < 1 || n > UNISVQ_MAX_GROUP || M < 0) return UNISVQ_ERR_INVALID_ARG;
   for (int i = 0; i < n; ++i) {
     if (!hs[i] || hs[i]->K != hs[0]->K || hs[i]->device != hs[0]->device) return UNISVQ_ERR_INVALID_ARG;
@@ -313,19 +325,30 @@ unisvq_status unisvq_linear_group(const unisvq_handle* hs, int n, const void* x,
   if (dev != hs[0]->device) return UNISVQ_ERR_INVALID_ARG;
   long long weights = 0;
   for (int i = 0; i < n; ++i) weights += static_cast<long long>(hs[i]->N) * hs[i]->K;
-  const int kernel = M > 64 && prefill_supported(hs[0], M) ? UNISVQ_KERNEL_PREFILL : decode_kernel_for(hs[0], weights, M);
-  if (kernel == UNISVQ_KERNEL_GEMV || kernel == UNISVQ_KERNEL_GEMV_ROWS) {
-    const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
-    for (int i = 0; i < n; ++i) Ls[i] = hs[i];
-    const cudaStream_t s = static_cast<cudaStream_t>(stream);
-    return kernel == UNISVQ_KERNEL_GEMV ? launch_gemv_group(Ls, n, x, ys, M, s)
-                                        : launch_gemv_rows_group(Ls, n, x, ys, M, s);
+  if (kernel == UNISVQ_KERNEL_AUTO)
+    kernel = M > 64 && prefill_supported(hs[0], M) ? UNISVQ_KERNEL_PREFILL : decode_kernel_for(hs[0], weights, M);
+  else if (kernel == UNISVQ_KERNEL_DECODE)
+    kernel = decode_kernel_for(hs[0], weights, M);
+  const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
+  for (int i = 0; i < n; ++i) Ls[i] = hs[i];
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (kernel == UNISVQ_KERNEL_GEMV) return launch_gemv_group(Ls, n, x, ys, M, s);
+  if (kernel == UNISVQ_KERNEL_SKINNY) return launch_skinny_group(Ls, n, x, ys, M, s);
+  if (kernel == UNISVQ_KERNEL_GEMV_ROWS) {
+    for (int i = 0; i < n; ++i)
+      if (!gemv_rows_supported(Ls[i], M < 4 ? M : 4)) return UNISVQ_ERR_UNSUPPORTED;
+    return launch_gemv_rows_group(Ls, n, x, ys, M, s);
   }
   for (int i = 0; i < n; ++i) {
-    const unisvq_status st = unisvq_linear(hs[i], x, ys[i], M, stream);
+    const unisvq_status st = unisvq_linear_force(hs[i], kernel, x, ys[i], M, stream);
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;
+}
+
+unisvq_status unisvq_linear_group(const unisvq_handle* hs, int n, const void* x, void* const* ys, int M,
+                                  void* stream) {
+  return unisvq_linear_group_force(hs, n, UNISVQ_KERNEL_AUTO, x, ys, M, stream);
 }
 
 unisvq_status unisvq_dequant_debug(unisvq_handle h, float* W, void* stream) {
@@ -355,9 +378,9 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
     info->split_k = p.ks;
     info->grid_ctas = p.ks * p.nb * ((M + 31) / 32 > 0 ? (M + 31) / 32 : 1);
   } else if (info->kernel == UNISVQ_KERNEL_SKINNY) {
-    const DecodePlan p = plan_skinny(h, M > 64 ? 64 : (M > 0 ? M : 1));
+    const DecodePlan p = plan_skinny(h, M > 16 ? 16 : (M > 0 ? M : 1));
     info->split_k = p.ks;
-    info->grid_ctas = p.ks * p.nb * ((M + 63) / 64 > 0 ? (M + 63) / 64 : 1);
+    info->grid_ctas = p.ks * p.nb * ((M + 15) / 16 > 0 ? (M + 15) / 16 : 1);
   } else {
     const PrefillPlan p = plan_prefill(h, M);
     info->split_k = 1;

@@ -255,30 +255,35 @@ def test_full_size_prefill_sampled_rows(N, K):
 # ---------------------------------------------------------------------------
 # grouped call: several layers that read the same x
 # ---------------------------------------------------------------------------
-def run_group(layers, xbits):
-    ys = binding.linear_group(layers, to_dev(xbits))
+def run_group(layers, xbits, kernel=None):
+    ys = binding.linear_group(layers, to_dev(xbits), kernel=kernel)
     st = binding.sync_status()
     assert st == binding.OK, binding.status_string(st)
     return [y.float().cpu().numpy().astype(np.float64) for y in ys]
 
 
+GROUP_KERNELS = [None, binding.KERNEL_GEMV, binding.KERNEL_SKINNY]
+
+
+@pytest.mark.parametrize("kernel", GROUP_KERNELS)
 @pytest.mark.parametrize("K", [1000, 4096])
 @pytest.mark.parametrize("M", [1, 3, 8, 9, 16, 17, 40])
-def test_group_matches_oracle(K, M):
-    """Layers of different N and d sharing x, in one call: each output meets
-    the tolerance against the oracle of its own layer (M > 16 takes the
-    per-layer path)."""
+def test_group_matches_oracle(kernel, K, M):
+    """Layers of different N and d sharing x, in one call (the library's pick
+    or a forced kernel): each output meets the tolerance against the oracle of
+    its own layer."""
     specs = [(520, 2), (130, 4), (256, 1)]
     data = [synth.layer_inputs(7, 70, i, K, N, K, d) for i, (N, d) in enumerate(specs)]
     layers = [binding.UniSVQLinear(c, A, B) for c, A, B in data]
     xb = synth.activations(7, 70, M, M, K)
-    for (c, A, B), yg in zip(data, run_group(layers, xb)):
+    for (c, A, B), yg in zip(data, run_group(layers, xb, kernel)):
         check(yg, xb, c, A, B)
     for l in layers:
         l.close()
 
 
-def test_group_integer_case_bit_exact():
+@pytest.mark.parametrize("kernel", GROUP_KERNELS)
+def test_group_integer_case_bit_exact(kernel):
     A = np.array([[1, -1, 0, 0], [0, 1, -1, 0], [0, 0, 1, -1], [0, 0, 1, 1]], dtype=np.float16)
     B = np.array([1, -2, 0, 1], dtype=np.float16)
     g = np.random.default_rng(13)
@@ -288,7 +293,7 @@ def test_group_integer_case_bit_exact():
     for M in (1, 7, 16):
         x = g.integers(-1, 2, size=(M, K)).astype(np.float32) * (g.random((M, K)) < 0.05)
         xb = synth.f32_to_bf16_bits(x)
-        for c, yg in zip(codes, run_group(layers, xb)):
+        for c, yg in zip(codes, run_group(layers, xb, kernel)):
             yr, _ = oracle.linear(xb, c, A, B)
             assert np.array_equal(yg, yr), np.abs(yg - yr).max()
     for l in layers:
