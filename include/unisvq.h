@@ -161,6 +161,24 @@ unisvq_status unisvq_linear_group(const unisvq_handle* hs, int n, const void* x,
 unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kernel, const void* x, void* const* ys,
                                         int M, void* stream);
 
+/*
+ * y = x W_hat^T with the tcgen05 decode kernels (UNISVQ_KERNEL_SKINNY) and
+ * their fold workspace in a static device array of the library (2 MiB per
+ * device: Kp <= 43648) instead of the handle's workspace. The paper has no
+ * counterpart: it is a deployment variant of unisvq_linear for callers that
+ * may not allocate on the call path (a server that fixed its device-memory
+ * budget at start-up, or code that must not enter the allocator while other
+ * work runs, since cudaMalloc and cudaFree can synchronise the device); it
+ * calls no allocating routine.
+ * The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current); make it before any
+ * stream capture. All calls on a device share the one array, so calls that
+ * overlap on the GPU race: order them on one stream. Arguments as
+ * unisvq_linear. Errors: INVALID_ARG (as unisvq_linear), UNSUPPORTED (the
+ * layer's fold needs more than the array: Kp > 43648), CUDA.
+ */
+unisvq_status unisvq_linear_noalloc(unisvq_handle h, const void* x, void* y, int M, void* stream);
+
 /* Test hook: writes W_hat as fp32 [N][K] row-major to device memory W (each
  * entry RN_fp32 of the exact A z + B), unpacking the device layout with the
  * same code-extraction helpers the layer kernels use. */

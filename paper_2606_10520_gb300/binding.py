@@ -21,7 +21,7 @@ EXPORTS = [
     "unisvq_pack", "unisvq_linear", "unisvq_linear_force", "unisvq_dequant_debug",
     "unisvq_query", "unisvq_sync_status", "unisvq_destroy", "unisvq_clone",
     "unisvq_status_string", "unisvq_packed_code_bytes", "unisvq_pack_host", "unisvq_version",
-    "unisvq_linear_group", "unisvq_linear_group_force",
+    "unisvq_linear_group", "unisvq_linear_group_force", "unisvq_linear_noalloc",
 ]
 MAX_GROUP = 4
 
@@ -57,6 +57,7 @@ def load():
     lib.unisvq_linear_force.argtypes = [vp, i, vp, vp, i, vp]
     lib.unisvq_linear_group.argtypes = [vp, i, vp, vp, i, vp]
     lib.unisvq_linear_group_force.argtypes = [vp, i, i, vp, vp, i, vp]
+    lib.unisvq_linear_noalloc.argtypes = [vp, vp, vp, i, vp]
     lib.unisvq_dequant_debug.argtypes = [vp, vp, vp]
     lib.unisvq_query.argtypes = [vp, i, ctypes.POINTER(Info)]
     lib.unisvq_sync_status.argtypes = [vp]
@@ -158,6 +159,12 @@ class UniSVQLinear:
         """Raw-pointer call (no checks in Python); returns the status."""
         return load().unisvq_linear_force(self._h, kernel, ctypes.c_void_p(x_ptr), ctypes.c_void_p(y_ptr),
                                           M, ctypes.c_void_p(stream_ptr))
+
+    def forward_noalloc_ptr(self, x_ptr: int, y_ptr: int, M: int, stream_ptr: int) -> int:
+        """Raw-pointer unisvq_linear_noalloc (fold workspace in the library's
+        static device array); returns the status."""
+        return load().unisvq_linear_noalloc(self._h, ctypes.c_void_p(x_ptr), ctypes.c_void_p(y_ptr), M,
+                                            ctypes.c_void_p(stream_ptr))
 
     def dequant_debug(self, stream=None):
         import torch

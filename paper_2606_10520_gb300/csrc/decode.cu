@@ -730,8 +730,11 @@ DecodePlan plan_skinny(const unisvq_layer* L, int M) {
   return plan_rows_split(L->Np / kTileRows, L->KT, L->num_sms, M > kMaxTokPerLaunch ? kMaxTokPerLaunch : M);
 }
 
-unisvq_status launch_skinny_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
-                                  cudaStream_t s) {
+namespace {
+
+// Fold and stream, the fold workspace of layer i at ws[i].
+unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                               cudaStream_t s, uint8_t* const* ws) {
   if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
   const unisvq_layer* L0 = Ls[0];
   if (!set_fold_attrs(L0->device)) return UNISVQ_ERR_CUDA;
@@ -759,14 +762,14 @@ unisvq_status launch_skinny_group(const unisvq_layer* const* Ls, int n, const vo
     for (int i = 0; i < n; ++i) {
       const unisvq_layer* L = Ls[i];
       FoldLayer& fl = f.layer[i];
-      fl.ws = L->fold_ws;
+      fl.ws = ws[i];
       fl.d = L->d;
       fl.colnorm = L->colnorm;
       for (int j = 0; j < 16; ++j) fl.A[j] = L->A[j];
       for (int j = 0; j < 4; ++j) fl.B[j] = L->B[j];
       SkLayer& l = a.layer[i];
       l.codes = L->codes;
-      l.ws = L->fold_ws;
+      l.ws = ws[i];
       l.y = static_cast<uint16_t*>(ys[i]) + static_cast<size_t>(m0) * L->N;
       l.N = L->N;
       l.rb0 = rb0;
@@ -790,9 +793,47 @@ unisvq_status launch_skinny_group(const unisvq_layer* const* Ls, int n, const vo
   return UNISVQ_OK;
 }
 
+}  // namespace
+
+unisvq_status launch_skinny_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                                  cudaStream_t s) {
+  if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
+  uint8_t* ws[kMaxGroup];
+  for (int i = 0; i < n; ++i) ws[i] = Ls[i]->fold_ws;
+  return launch_skinny_ws(Ls, n, x, ys, M, s, ws);
+}
+
 unisvq_status launch_skinny(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
   void* ys[1] = {y};
   return launch_skinny_group(&L, 1, x, ys, M, s);
+}
+
+// ---- allocation-free variant (unisvq_linear_noalloc) -------------------------
+// The same fold and streaming kernels with the fold workspace taken from a
+// file-scope device array that exists from module load, for callers that may
+// not allocate on the call path. One array per device: calls of this entry
+// point that overlap on the GPU race on it. Nothing in it has to start at
+// zero (the fold kernel writes every table entry and B row the streaming
+// kernel reads).
+constexpr size_t kStaticWsBytes = static_cast<size_t>(2) << 20;   // 2 MiB: Kp <= 43648
+__device__ __align__(256) uint8_t g_static_fold_ws[kStaticWsBytes];
+
+size_t static_fold_workspace_bytes() { return kStaticWsBytes; }
+
+unisvq_status launch_skinny_static(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
+  if (fold_workspace_bytes(L->KT) > kStaticWsBytes) return UNISVQ_ERR_UNSUPPORTED;
+  // In host code g_static_fold_ws only names the symbol; its device address
+  // is looked up once per device (the device of L is current here).
+  static uint8_t* dev_ptr[64] = {};
+  if (L->device < 0 || L->device >= 64) return UNISVQ_ERR_INVALID_ARG;
+  if (!dev_ptr[L->device]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_fold_ws) != cudaSuccess || !p) return UNISVQ_ERR_CUDA;
+    dev_ptr[L->device] = static_cast<uint8_t*>(p);
+  }
+  uint8_t* ws[1] = {dev_ptr[L->device]};
+  void* ys[1] = {y};
+  return launch_skinny_ws(&L, 1, x, ys, M, s, ws);
 }
 
 }  // namespace unisvq

@@ -63,6 +63,10 @@ size_t fold_workspace_bytes(int KT);
 // Several layers with the same K that read the same x, in one launch per 16 tokens.
 unisvq_status launch_skinny_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
                                   cudaStream_t s);
+// As launch_skinny with the fold workspace in a static device array of
+// static_fold_workspace_bytes() (UNSUPPORTED if the layer needs more).
+unisvq_status launch_skinny_static(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
+size_t static_fold_workspace_bytes();
 
 bool prefill_supported(const unisvq_layer* L, int M);
 PrefillPlan plan_prefill(const unisvq_layer* L, int M);

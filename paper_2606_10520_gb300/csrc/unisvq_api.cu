@@ -307,6 +307,15 @@ unisvq_status unisvq_linear(unisvq_handle h, const void* x, void* y, int M, void
   return unisvq_linear_force(h, UNISVQ_KERNEL_AUTO, x, y, M, stream);
 }
 
+unisvq_status unisvq_linear_noalloc(unisvq_handle h, const void* x, void* y, int M, void* stream) {
+  unisvq_status st = check_io(h, x, y, M);
+  if (st != UNISVQ_OK || M == 0) return st;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
+  if (dev != h->device) return UNISVQ_ERR_INVALID_ARG;
+  return launch_skinny_static(h, x, y, M, static_cast<cudaStream_t>(stream));
+}
+
 unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kernel, const void* x, void* const* ys,
                                         int M, void* stream) {
   if (!hs || !ys || n < 1 || n > UNISVQ_MAX_GROUP || M < 0) return UNISVQ_ERR_INVALID_ARG;
