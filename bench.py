@@ -61,31 +61,39 @@ def algo_bytes(N, K, M, d=2):
 
 
 KERNEL_NAMES = {1: "decode", 2: "prefill_kernel", 3: "gemv_kernel", 4: "decode_kernel", 5: "gemv_rows_kernel"}
-GEMV_SOURCES = ("paper_2606_10520_gb300/csrc/gemv.cu", "paper_2606_10520_gb300/csrc/common.cuh",
-                "paper_2606_10520_gb300/csrc/layout.h")
-TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "gemv_kernel_llama2_7b_decode_sweep.txt")
+# Sources whose change invalidates a committed ncu traffic figure, per kernel.
+KERNEL_SOURCES = {
+    "gemv_kernel": ("paper_2606_10520_gb300/csrc/gemv.cu", "paper_2606_10520_gb300/csrc/common.cuh",
+                    "paper_2606_10520_gb300/csrc/layout.h"),
+    "decode_kernel": ("paper_2606_10520_gb300/csrc/decode.cu", "paper_2606_10520_gb300/csrc/common.cuh",
+                      "paper_2606_10520_gb300/csrc/layout.h"),
+}
 
 
-def gemv_source_digest():
+def traffic_summary_path(kernel):
+    return os.path.join(ROOT, "profiles", f"{kernel}_llama2_7b_decode_sweep.txt")
+
+
+def source_digest(kernel):
     import hashlib
     h = hashlib.sha256()
-    for rel in GEMV_SOURCES:
+    for rel in KERNEL_SOURCES[kernel]:
         with open(os.path.join(ROOT, rel), "rb") as f:
             h.update(f.read())
     return h.hexdigest()
 
 
-def measured_traffic():
-    """DRAM bytes per GEMV launch from the committed ncu summary, or None when
-    the kernel sources changed since those counters were taken."""
+def measured_traffic(kernel):
+    """DRAM bytes per launch of `kernel` from its committed ncu summary, or None
+    when the kernel's sources changed since those counters were taken."""
     try:
         fields = {}
-        with open(TRAFFIC_SUMMARY) as f:
+        with open(traffic_summary_path(kernel)) as f:
             for ln in f:
                 if ":" in ln:
                     k, v = ln.split(":", 1)
                     fields[k.strip()] = v.strip()
-        if fields.get("source_sha256") != gemv_source_digest():
+        if fields.get("source_sha256") != source_digest(kernel):
             return None
         return float(fields["dram_bytes_per_launch"])
     except Exception:
@@ -286,6 +294,13 @@ def run_ours(args, rank, world, local_rank):
                 xs[(M, K)] = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).cuda()
             ys[(M, pi)] = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
 
+    # The library's choice per call (the same for every layer of the stack).
+    def call_info(grp, M):
+        layer0 = stack[0]
+        if len(grp) == 1:
+            return layer0[grp[0]].query(M)
+        return binding.query_group([layer0[i] for i in grp], M)
+
     def issue(layer, grp, M, sp):
         K = shapes[grp[0]][2]
         if len(grp) == 1:
@@ -298,6 +313,9 @@ def run_ours(args, rank, world, local_rank):
             raise RuntimeError(f"unisvq call failed: {binding.status_string(st)}")
 
     side = torch.cuda.Stream()
+    # calls per kernel class: {kernel id: [(M, group index), ...]}
+    kinds = {}
+    kind_bytes, kind_main_launches = {}, {}
     for M in M_SWEEP:
         def one_pass(M=M):
             sp = torch.cuda.current_stream().cuda_stream
@@ -311,10 +329,17 @@ def run_ours(args, rank, world, local_rank):
         with torch.cuda.graph(g, stream=side):
             one_pass()
         graphs.append(g)
-        for layer in stack:
-            for _, N, K in shapes:
-                step_bytes += algo_bytes(N, K, M)
-            launches += len(groups) * ((M + 15) // 16)
+        for gi, grp in enumerate(groups):
+            info = call_info(grp, M)
+            kid = info["kernel"]
+            nbytes = sum(algo_bytes(shapes[i][1], shapes[i][2], M) for i in grp) * args.layers
+            step_bytes += nbytes
+            launches += info["launches"] * args.layers
+            kinds.setdefault(kid, []).append((M, gi))
+            kind_bytes[kid] = kind_bytes.get(kid, 0) + nbytes
+            # the streaming kernel's launches (the skinny path adds one fold launch each)
+            main = info["launches"] // 2 if kid == binding.KERNEL_SKINNY else info["launches"]
+            kind_main_launches[kid] = kind_main_launches.get(kid, 0) + main * args.layers
     torch.cuda.synchronize()
     st = binding.sync_status()
     if st != 0:
@@ -340,6 +365,56 @@ def run_ours(args, rank, world, local_rank):
     value = total_bytes / t / 1e9
     per_rank = step_bytes * args.steps / t / 1e9
 
+    # per-kernel-class timing: graphs holding only the calls that run that
+    # kernel, so each kernel's throughput (and launch interval) is measured
+    # on its own stream; the dominant class (most time) gives the roofline.
+    kind_time = {}
+    for kid, calls in kinds.items():
+        kgraphs = []
+        for M in M_SWEEP:
+            sel = [gi for (m, gi) in calls if m == M]
+            if not sel:
+                continue
+            def kpass(M=M, sel=sel):
+                sp = torch.cuda.current_stream().cuda_stream
+                for layer in stack:
+                    for gi in sel:
+                        issue(layer, groups[gi], M, sp)
+            with torch.cuda.stream(side):
+                kpass()
+            torch.cuda.synchronize()
+            kg = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(kg, stream=side):
+                kpass()
+            kgraphs.append(kg)
+        kind_time[kid] = time_graphs(torch, kgraphs, args.steps, args.warmup, side)
+    if world > 1:
+        for kid in sorted(kind_time):
+            tt = torch.tensor([kind_time[kid]], device="cuda", dtype=torch.float64)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            kind_time[kid] = float(tt.item())
+
+    def roofline_for(kid):
+        name = KERNEL_NAMES.get(kid, "?")
+        t_k = kind_time[kid]
+        ach = kind_bytes[kid] * args.steps / t_k / 1e9
+        n_main = kind_main_launches[kid]
+        extra = " (each call: fold_kernel + decode_kernel)" if kid == binding.KERNEL_SKINNY else ""
+        return {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": ach / peaks["hbm_gbs"],
+                "traffic": measured_traffic(name) if name in KERNEL_SOURCES else None,
+                "algorithmic_bytes_per_launch": kind_bytes[kid] / max(1, n_main),
+                "avg_launch_us": t_k / args.steps / max(1, n_main) * 1e6,
+                "launches_per_step": n_main,
+                "share_of_step_time": t_k / max(1e-12, sum(kind_time.values())),
+                "kernel": name + extra,
+                "how": ("achieved = algorithmic bytes of the calls that run this kernel / their time, "
+                        "timed alone from CUDA graphs of those calls (CUDA events on the launching stream)"),
+                "peak_source": f"{peak_src} hbm_gbs (copy, burst)",
+                "frac_of_8TBs": ach / 8000.0}
+
+    dominant = max(kind_time, key=lambda k: kind_time[k])
+
     # per-M breakdown (separate short timing of each graph)
     sweep = []
     for M, g in zip(M_SWEEP, graphs):
@@ -350,7 +425,8 @@ def run_ours(args, rank, world, local_rank):
         sweep.append({"M": M, "GB/s": round(gbs, 1), "frac_of_measured_hbm": round(gbs / peaks["hbm_gbs"], 4),
                       "frac_of_8TBs": round(gbs / 8000.0, 4),
                       "us_per_layer": round(tm / max(3, args.steps // 4) / n_calls * 1e6, 3),
-                      "kernel": KERNEL_NAMES.get(stack[0][0].query(M)["kernel"], "?")})
+                      "kernels": {"+".join(shapes[i][0] for i in grp): KERNEL_NAMES.get(call_info(grp, M)["kernel"], "?")
+                                  for grp in groups}})
 
     # ---- e2e: pinned host buffers, H2D + layer + D2H inside the timed graphs ---
     e2e = None
@@ -401,16 +477,13 @@ def run_ours(args, rank, world, local_rank):
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": t * 1000 / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f16 MMA on bf16 I/O, f32 accumulate",
+        "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16 I/O; e4m3 tcgen05 MMA (decode_kernel) / f16 mma.sync (gemv_kernel); f32 accumulate",
         "data": "synthetic (seeded codes, affine and activations; layers 1..31 are device copies of layer 0)",
         "config": workload_config(args),
-        "roofline": {"bound": "hbm", "achieved": per_rank, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                     "frac": per_rank / peaks["hbm_gbs"], "traffic": measured_traffic(),
-                     "algorithmic_bytes_per_launch": step_bytes / max(1, launches),
-                     "kernel": "gemv_kernel (every launch of the timed region; achieved = algorithmic bytes "
-                               "/ time, i.e. per launch: bytes per launch / mean launch interval)",
-                     "peak_source": f"{peak_src} hbm_gbs (copy, burst)",
-                     "frac_of_8TBs": per_rank / 8000.0},
+        "roofline": roofline_for(dominant),
+        "roofline_other": {KERNEL_NAMES.get(k, "?"): roofline_for(k) for k in kind_time if k != dominant},
+        "step_throughput_per_gpu": per_rank,
         "sweep": sweep,
         "e2e": e2e,
         "gpu_launches": launches * args.steps,

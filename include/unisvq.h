@@ -90,6 +90,7 @@ typedef struct {
   long long meta_bytes;   /* affine parameters: (d*d + d) * 2 bytes (fp16)      */
   long long algo_bytes;   /* N*K/4 + meta + 2*M*K (x) + 2*M*N (y)               */
   double flops;           /* 2*M*N*K                                            */
+  int launches;           /* kernel launches the call makes                     */
 } unisvq_info;
 
 /*
@@ -186,6 +187,12 @@ unisvq_status unisvq_dequant_debug(unisvq_handle h, float* W, void* stream);
 
 /* Describe the launch unisvq_linear would make for M tokens (host only). */
 unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info);
+
+/* Describe the launches unisvq_linear_group would make for the n layers hs
+ * and M tokens (host only): N, Np and the byte and flop counts are sums over
+ * the layers (x counted once), K, Kp and d those of hs[0].
+ * Errors: INVALID_ARG (null, n out of range, K mismatch, M < 0). */
+unisvq_status unisvq_query_group(const unisvq_handle* hs, int n, int M, unisvq_info* info);
 
 /* Synchronise `stream`, then report and clear the device error word:
  * UNISVQ_ERR_TIMEOUT if a kernel gave up on a bounded wait since the last

@@ -21,7 +21,7 @@ EXPORTS = [
     "unisvq_pack", "unisvq_linear", "unisvq_linear_force", "unisvq_dequant_debug",
     "unisvq_query", "unisvq_sync_status", "unisvq_destroy", "unisvq_clone",
     "unisvq_status_string", "unisvq_packed_code_bytes", "unisvq_pack_host", "unisvq_version",
-    "unisvq_linear_group", "unisvq_linear_group_force", "unisvq_linear_noalloc",
+    "unisvq_linear_group", "unisvq_linear_group_force", "unisvq_linear_noalloc", "unisvq_query_group",
 ]
 MAX_GROUP = 4
 
@@ -37,7 +37,7 @@ class Info(ctypes.Structure):
                 ("Np", ctypes.c_int), ("Kp", ctypes.c_int), ("kernel", ctypes.c_int),
                 ("split_k", ctypes.c_int), ("grid_ctas", ctypes.c_int),
                 ("code_bytes", ctypes.c_longlong), ("meta_bytes", ctypes.c_longlong),
-                ("algo_bytes", ctypes.c_longlong), ("flops", ctypes.c_double)]
+                ("algo_bytes", ctypes.c_longlong), ("flops", ctypes.c_double), ("launches", ctypes.c_int)]
 
 
 _lib = None
@@ -60,6 +60,7 @@ def load():
     lib.unisvq_linear_noalloc.argtypes = [vp, vp, vp, i, vp]
     lib.unisvq_dequant_debug.argtypes = [vp, vp, vp]
     lib.unisvq_query.argtypes = [vp, i, ctypes.POINTER(Info)]
+    lib.unisvq_query_group.argtypes = [vp, i, i, ctypes.POINTER(Info)]
     lib.unisvq_sync_status.argtypes = [vp]
     lib.unisvq_destroy.argtypes = [vp]
     lib.unisvq_clone.argtypes = [vp, vp, ctypes.POINTER(vp)]
@@ -200,6 +201,15 @@ def linear_group_ptr(layers, x_ptr: int, y_ptrs, M: int, stream_ptr: int, kernel
         return load().unisvq_linear_group(hs, n, ctypes.c_void_p(x_ptr), ys, M, ctypes.c_void_p(stream_ptr))
     return load().unisvq_linear_group_force(hs, n, int(kernel), ctypes.c_void_p(x_ptr), ys, M,
                                             ctypes.c_void_p(stream_ptr))
+
+
+def query_group(layers, M: int) -> dict:
+    """unisvq_query_group: the launches unisvq_linear_group makes for `layers`."""
+    n = len(layers)
+    hs = (ctypes.c_void_p * n)(*[l._h.value if isinstance(l._h, ctypes.c_void_p) else l._h for l in layers])
+    info = Info()
+    _check(load().unisvq_query_group(hs, n, int(M), ctypes.byref(info)), "unisvq_query_group")
+    return {f: getattr(info, f) for f, _ in Info._fields_}
 
 
 def linear_group(layers, x, outs=None, stream=None, kernel=None):

@@ -497,8 +497,9 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
       bool ok = !*abort_flag;
       for (int st = 0; st < n_st && ok; ++st) {
         const int sa = st % kASlots, s = st % S;
-        ok = !*abort_flag && mbar_wait(a_full(sa), (st / kASlots) & 1, a.err, kErrTimeoutFull) &&
-             mbar_wait(bfull(s), (st / S) & 1, a.err, kErrTimeoutFull);
+        // The converters arrive on a_full only once the stage's B tiles have
+        // landed too (they wait on bfull), so one wait covers both operands.
+        ok = mbar_wait(a_full(sa), (st / kASlots) & 1, a.err, kErrTimeoutFull);
         if (!ok) break;
         tc_fence_after();
         const int nt = min(kStageTiles, n_kt - st * kStageTiles);
@@ -563,6 +564,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         tc_fence_before();
       }
+      if (ok) ok = mbar_wait(bfull(s), (st / S) & 1, a.err, kErrTimeoutFull);
       __syncwarp();
       if (lane == 0 && ok) mbar_arrive(a_full(sa));
       if (!ok) *abort_flag = 1;

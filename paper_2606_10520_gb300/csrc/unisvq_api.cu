@@ -253,19 +253,22 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
 }
 
 // Decode kernel for M <= 64 tokens over `weights` = sum of N*K of the layers
-// of one launch (measured crossovers on GB300): the whole-K row-slice GEMV for
-// one or two tokens on launches of at least 2^26 weights (no cross-CTA
-// reduction, many small CTAs), otherwise the K-split cluster GEMV (32 tokens
-// per launch). The tcgen05 skinny kernel (fold kernel + streaming kernel) is
-// reachable through unisvq_linear_force / unisvq_linear_group_force.
-static int decode_kernel_for(const unisvq_layer* L, long long weights, int M) {
-  if (M <= 2 && weights >= (1ll << 26) && gemv_rows_supported(L, M)) return UNISVQ_KERNEL_GEMV_ROWS;
+// of one launch and `nb` = their 128-row blocks (measured crossovers on
+// GB300, Llama-shaped layers): the tcgen05 skinny kernel (fold + streaming
+// kernel, cost nearly independent of M) for launches of at least 2^26
+// weights, and from four tokens up for launches of at least 2^25 weights
+// with 64 or more row blocks; the K-split cluster GEMV (lower fixed latency)
+// otherwise. The whole-K row-slice GEMV is reachable through the force
+// calls only.
+static int decode_kernel_for(long long weights, int nb, int M) {
+  if (weights >= (1ll << 26)) return UNISVQ_KERNEL_SKINNY;
+  if (weights >= (1ll << 25) && M >= 4 && nb >= 64) return UNISVQ_KERNEL_SKINNY;
   return UNISVQ_KERNEL_GEMV;
 }
 
 static int auto_kernel(const unisvq_layer* L, int M) {
   if (M > 64 && prefill_supported(L, M)) return UNISVQ_KERNEL_PREFILL;
-  return decode_kernel_for(L, static_cast<long long>(L->N) * L->K, M);
+  return decode_kernel_for(static_cast<long long>(L->N) * L->K, L->Np / kTileRows, M);
 }
 
 static unisvq_status check_io(unisvq_handle h, const void* x, void* y, int M) {
@@ -286,7 +289,7 @@ unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, vo
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
   if (dev != h->device) return UNISVQ_ERR_INVALID_ARG;
   if (kernel == UNISVQ_KERNEL_AUTO) kernel = auto_kernel(h, M);
-  if (kernel == UNISVQ_KERNEL_DECODE) kernel = decode_kernel_for(h, static_cast<long long>(h->N) * h->K, M);
+  if (kernel == UNISVQ_KERNEL_DECODE) kernel = decode_kernel_for(static_cast<long long>(h->N) * h->K, h->Np / kTileRows, M);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (kernel == UNISVQ_KERNEL_GEMV) return launch_gemv(h, x, y, M, s);
   if (kernel == UNISVQ_KERNEL_GEMV_ROWS) {
@@ -333,11 +336,15 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
   if (dev != hs[0]->device) return UNISVQ_ERR_INVALID_ARG;
   long long weights = 0;
-  for (int i = 0; i < n; ++i) weights += static_cast<long long>(hs[i]->N) * hs[i]->K;
+  int nb = 0;
+  for (int i = 0; i < n; ++i) {
+    weights += static_cast<long long>(hs[i]->N) * hs[i]->K;
+    nb += hs[i]->Np / kTileRows;
+  }
   if (kernel == UNISVQ_KERNEL_AUTO)
-    kernel = M > 64 && prefill_supported(hs[0], M) ? UNISVQ_KERNEL_PREFILL : decode_kernel_for(hs[0], weights, M);
+    kernel = M > 64 && prefill_supported(hs[0], M) ? UNISVQ_KERNEL_PREFILL : decode_kernel_for(weights, nb, M);
   else if (kernel == UNISVQ_KERNEL_DECODE)
-    kernel = decode_kernel_for(hs[0], weights, M);
+    kernel = decode_kernel_for(weights, nb, M);
   const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
   for (int i = 0; i < n; ++i) Ls[i] = hs[i];
   const cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -365,6 +372,39 @@ unisvq_status unisvq_dequant_debug(unisvq_handle h, float* W, void* stream) {
   return launch_dequant(h, W, static_cast<cudaStream_t>(stream));
 }
 
+// Launch geometry of `kernel` for the n layers of one call (query helpers).
+static void describe_launch(const unisvq_layer* const* Ls, int n, int kernel, int M, unisvq_info* info) {
+  const unisvq_layer* h = Ls[0];
+  const int m = M > 0 ? M : 1;
+  info->kernel = kernel;
+  if (kernel == UNISVQ_KERNEL_GEMV_ROWS) {
+    info->split_k = 1;
+    info->grid_ctas = 0;
+    for (int i = 0; i < n; ++i) info->grid_ctas += Ls[i]->Np / 32;
+    info->launches = (m + 3) / 4;
+  } else if (kernel == UNISVQ_KERNEL_GEMV) {
+    const DecodePlan p = plan_gemv(h, m > 32 ? 32 : m);
+    info->split_k = p.ks;
+    int nb = 0;
+    for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
+    info->launches = (m + 31) / 32;
+    info->grid_ctas = p.ks * nb * info->launches;
+  } else if (kernel == UNISVQ_KERNEL_SKINNY) {
+    const DecodePlan p = plan_skinny(h, m > 16 ? 16 : m);
+    int nb = 0;
+    for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
+    info->split_k = p.ks;
+    const int chunks = (m + 15) / 16;
+    info->launches = 2 * chunks;   // fold kernel + streaming kernel per 16 tokens
+    info->grid_ctas = p.ks * nb * chunks;
+  } else {
+    const PrefillPlan p = plan_prefill(h, m);
+    info->split_k = 1;
+    info->grid_ctas = p.grid * n;
+    info->launches = n;
+  }
+}
+
 unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
   if (!h || !info || M < 0) return UNISVQ_ERR_INVALID_ARG;
   std::memset(info, 0, sizeof(*info));
@@ -378,23 +418,39 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
   info->algo_bytes = static_cast<long long>(h->N) * h->K / 4 + info->meta_bytes +
                      2ll * M * h->K + 2ll * M * h->N;
   info->flops = 2.0 * M * static_cast<double>(h->N) * h->K;
-  info->kernel = auto_kernel(h, M > 0 ? M : 1);
-  if (info->kernel == UNISVQ_KERNEL_GEMV_ROWS) {
-    info->split_k = 1;
-    info->grid_ctas = h->Np / 32;
-  } else if (info->kernel == UNISVQ_KERNEL_GEMV) {
-    const DecodePlan p = plan_gemv(h, M > 32 ? 32 : (M > 0 ? M : 1));
-    info->split_k = p.ks;
-    info->grid_ctas = p.ks * p.nb * ((M + 31) / 32 > 0 ? (M + 31) / 32 : 1);
-  } else if (info->kernel == UNISVQ_KERNEL_SKINNY) {
-    const DecodePlan p = plan_skinny(h, M > 16 ? 16 : (M > 0 ? M : 1));
-    info->split_k = p.ks;
-    info->grid_ctas = p.ks * p.nb * ((M + 15) / 16 > 0 ? (M + 15) / 16 : 1);
-  } else {
-    const PrefillPlan p = plan_prefill(h, M);
-    info->split_k = 1;
-    info->grid_ctas = p.grid;
+  const unisvq_layer* Ls[1] = {h};
+  describe_launch(Ls, 1, auto_kernel(h, M > 0 ? M : 1), M, info);
+  return UNISVQ_OK;
+}
+
+unisvq_status unisvq_query_group(const unisvq_handle* hs, int n, int M, unisvq_info* info) {
+  if (!hs || !info || n < 1 || n > UNISVQ_MAX_GROUP || M < 0) return UNISVQ_ERR_INVALID_ARG;
+  for (int i = 0; i < n; ++i)
+    if (!hs[i] || hs[i]->K != hs[0]->K) return UNISVQ_ERR_INVALID_ARG;
+  std::memset(info, 0, sizeof(*info));
+  long long weights = 0;
+  int nb = 0;
+  for (int i = 0; i < n; ++i) {
+    const unisvq_layer* h = hs[i];
+    info->N += h->N;
+    info->Np += h->Np;
+    info->code_bytes += static_cast<long long>(h->code_bytes);
+    info->meta_bytes += static_cast<long long>(h->d * h->d + h->d) * 2;
+    info->algo_bytes += static_cast<long long>(h->N) * h->K / 4 + 2ll * M * h->N;
+    info->flops += 2.0 * M * static_cast<double>(h->N) * h->K;
+    weights += static_cast<long long>(h->N) * h->K;
+    nb += h->Np / kTileRows;
   }
+  info->K = hs[0]->K;
+  info->Kp = hs[0]->Kp;
+  info->d = hs[0]->d;
+  info->algo_bytes += info->meta_bytes + 2ll * M * hs[0]->K;   // x is read once per call
+  const int m = M > 0 ? M : 1;
+  const int kernel =
+      m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL : decode_kernel_for(weights, nb, m);
+  const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
+  for (int i = 0; i < n; ++i) Ls[i] = hs[i];
+  describe_launch(Ls, n, kernel, M, info);
   return UNISVQ_OK;
 }
 

@@ -236,6 +236,31 @@ def test_prefill_and_decode_agree_with_auto_dispatch():
     layer.close()
 
 
+def test_dispatch_picks_tcgen05_decode_for_large_launches():
+    """The library's pick (unisvq_query / unisvq_query_group): the tcgen05
+    skinny path (fold + streaming kernel: two launches) from 2^26 weights per
+    launch, and from four tokens on 2^25 weights over >= 64 row blocks."""
+    big = binding.UniSVQLinear(*synth.layer_inputs(9, 91, 0, 0, 16384, 4096, 2))
+    q = big.query(1)
+    assert q["kernel"] == binding.KERNEL_SKINNY and q["launches"] == 2
+    assert big.query(17)["launches"] == 4
+    small = binding.UniSVQLinear(*synth.layer_inputs(9, 91, 1, 0, 4096, 4096, 2))
+    assert small.query(16)["kernel"] == binding.KERNEL_GEMV and small.query(16)["launches"] == 1
+    trio = [small, small.clone(), small.clone()]
+    assert binding.query_group(trio, 2)["kernel"] == binding.KERNEL_GEMV
+    g4 = binding.query_group(trio, 4)
+    assert g4["kernel"] == binding.KERNEL_SKINNY and g4["N"] == 3 * 4096 and g4["launches"] == 2
+    xb = synth.activations(9, 91, 4, 4, 4096)
+    codes, A, B = synth.layer_inputs(9, 91, 1, 0, 4096, 4096, 2)
+    rows = np.unique(np.concatenate([np.sort(synth.rng(9, 4096, 4096).choice(4096, 32, replace=False)), [0, 4095]]))
+    for yg in run_group(trio, xb):
+        check(yg, xb, codes, A, B, rows=rows)
+    for l in trio[1:]:
+        l.close()
+    small.close()
+    big.close()
+
+
 @pytest.mark.parametrize("N,K", [(4096, 4096), (1024, 4096), (14336, 4096), (4096, 14336)])
 def test_full_size_prefill_sampled_rows(N, K):
     """Llama-3-8B-shaped projections at M = 2048 (the prefill workload)."""
