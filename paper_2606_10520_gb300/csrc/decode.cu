@@ -53,17 +53,11 @@ constexpr int kWarps = 10;
 constexpr int kThreads = kWarps * 32;
 constexpr int kConvWarp0 = 2;
 constexpr int kConvWarps = 8;
-constexpr int kStageTiles = 2;                      // k-tiles per pipeline stage
-constexpr int kCodeBytes = kStageTiles * kTileBytes;
 constexpr int kASlots = 3;                          // TMEM A slots (one stage each)
-constexpr int kAColBase = 64;                       // accumulator in [0, 64)
-constexpr int kASlotCols = 32 * kStageTiles;
-constexpr int kTmemCols = 256;
 constexpr int kMaxTokPerLaunch = 16;
 constexpr int kMaxSplit = 8;                        // K slices (cluster size)
 constexpr int kMaxGroup = UNISVQ_MAX_GROUP;
 constexpr int kFoldThreads = 256;
-static_assert(kAColBase + kASlots * kASlotCols <= kTmemCols, "TMEM columns");
 static_assert(kConvWarps / 4 <= kASlots, "converter groups must not run two slot uses ahead");
 
 // Fold workspace of a handle (unisvq_layer::fold_ws): a table of per-(slice,
@@ -104,12 +98,21 @@ struct FoldArgs {
   FoldLayer layer[kMaxGroup];
 };
 
-template <int NCOL>
+// Geometry: T k-tiles per pipeline stage. T = 2: 256 TMEM columns (accumulator
+// in [0, 64), three A slots of 64), two CTAs per SM. T = 1: 128 TMEM columns
+// (accumulator in [0, 32), three A slots of 32), N <= 32, three CTAs per SM.
+template <int NCOL, int T>
 struct Cfg {
+  static constexpr int kT = T;
+  static constexpr int kMinBlocks = T == 1 ? 3 : 2;
+  static constexpr int kCodeBytes = T * kTileBytes;
+  static constexpr int kAColBase = T == 1 ? 32 : 64;
+  static constexpr int kASlotCols = 32 * T;
+  static constexpr int kTmemCols = T == 1 ? 128 : 256;
   static constexpr int kMaxTok = NCOL / 3;
   static constexpr int kStages = NCOL == 48 ? 4 : 6;
   static constexpr int kBTile = NCOL * 128;                      // one k-tile of B (NCOL rows x 128 bytes)
-  static constexpr int kBBytes = kStageTiles * kBTile;
+  static constexpr int kBBytes = T * kBTile;
   static constexpr int kStageBytes = kCodeBytes + kBBytes;       // [codes | B tiles]
   static constexpr int kOffRed = kStages * kStageBytes;
   static constexpr int kRedBytes = (kTileRows + 8) * kMaxTok * 4;
@@ -123,6 +126,8 @@ struct Cfg {
       (1u << 4) | (static_cast<uint32_t>(NCOL >> 3) << 17) | ((128u >> 4) << 24);
   static_assert(kStageBytes % 1024 == 0 && kBTile % 1024 == 0, "128B-swizzled B tiles need 1024-byte alignment");
   static_assert(kStages % (kConvWarps / 4) == 0, "a converter group revisits its own stages");
+  static_assert(NCOL <= kAColBase, "accumulator columns");
+  static_assert(kAColBase + kASlots * kASlotCols <= kTmemCols, "TMEM columns");
 };
 
 // ---- tcgen05 wrappers ----------------------------------------------------------
@@ -364,9 +369,14 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
   }
 }
 
-template <int NCOL>
-__global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_constant__ SkArgs a) {
-  using C = Cfg<NCOL>;
+template <int NCOL, int T>
+__global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_kernel(const __grid_constant__ SkArgs a) {
+  using C = Cfg<NCOL, T>;
+  constexpr int kStageTiles = C::kT;
+  constexpr int kCodeBytes = C::kCodeBytes;
+  constexpr int kAColBase = C::kAColBase;
+  constexpr int kASlotCols = C::kASlotCols;
+  constexpr int kTmemCols = C::kTmemCols;
   constexpr int S = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -639,14 +649,14 @@ __global__ void __launch_bounds__(kThreads, 2) decode_kernel(const __grid_consta
 
 int ncol_for(int M) { return M <= 5 ? 16 : (M <= 10 ? 32 : 48); }
 
-template <int NCOL>
+template <int NCOL, int T>
 bool set_attrs(int dev) {
   static bool done[64] = {};
   if (dev < 0 || dev >= 64) return false;
   if (done[dev]) return true;
-  if (cudaFuncSetAttribute(decode_kernel<NCOL>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<NCOL>::kSmem) !=
-          cudaSuccess ||
-      cudaFuncSetAttribute(decode_kernel<NCOL>, cudaFuncAttributePreferredSharedMemoryCarveout,
+  if (cudaFuncSetAttribute(decode_kernel<NCOL, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           Cfg<NCOL, T>::kSmem) != cudaSuccess ||
+      cudaFuncSetAttribute(decode_kernel<NCOL, T>, cudaFuncAttributePreferredSharedMemoryCarveout,
                            cudaSharedmemCarveoutMaxShared) != cudaSuccess)
     return false;
   done[dev] = true;
@@ -665,24 +675,33 @@ bool set_fold_attrs(int dev) {
   return true;
 }
 
-size_t smem_for(int ncol) { return ncol == 16 ? Cfg<16>::kSmem : (ncol == 32 ? Cfg<32>::kSmem : Cfg<48>::kSmem); }
+template <int T>
+size_t smem_of(int ncol) {
+  return ncol == 16 ? Cfg<16, T>::kSmem : (ncol == 32 ? Cfg<32, T>::kSmem : Cfg<48, 2>::kSmem);
+}
 
-// Resident CTAs per SM: two when their shared memory fits (each holds half of
-// the 512 TMEM columns; 320 threads x <= 102 registers fit twice). The
-// occupancy query of the runtime reports one for this kernel although two
-// run side by side (measured), so the count is derived here.
-int resident_for(int ncol) {
-  return 2 * (smem_for(ncol) + 1024) <= static_cast<size_t>(228) * 1024 ? 2 : 1;
+// Resident CTAs per SM: as many as the shared memory, the TMEM columns
+// (512 / kTmemCols) and the registers of 320 threads allow (two for T = 2,
+// three for T = 1). The occupancy query of the runtime reports one for this
+// kernel although two or three run side by side (measured), so the count is
+// derived here.
+int resident_for(int ncol, int T) {
+  const size_t smem = T == 1 ? smem_of<1>(ncol) : smem_of<2>(ncol);
+  const int by_smem = static_cast<int>((static_cast<size_t>(228) * 1024) / (smem + 1024));
+  const int by_tmem = T == 1 ? 4 : 2;
+  const int by_regs = T == 1 ? 3 : 2;
+  return max(1, min(by_smem, min(by_tmem, by_regs)));
 }
 
 // Largest K split (cluster size <= 8, >= 1 k-tile per CTA) whose grid fits in
-// one wave of resident CTAs; at least enough slices for the fold kernel's
-// shared memory.
-DecodePlan plan_rows_split(int nb, int KT, int num_sms, int M) {
+// one wave of resident CTAs of geometry T; at least enough slices for the
+// fold kernel's shared memory.
+DecodePlan plan_with(int nb, int KT, int num_sms, int ncol, int T) {
   DecodePlan p{};
-  p.nt = ncol_for(M);
+  p.nt = ncol;
   p.nb = nb;
-  const int slots = resident_for(p.nt) * num_sms;
+  p.geom = T;
+  const int slots = resident_for(ncol, T) * num_sms;
   const int min_ks = (KT * kTileCols * 2 + kFoldMaxSmem - 1) / kFoldMaxSmem;
   int ks = 0;
   for (int c = kMaxSplit; c >= 1; --c)
@@ -694,8 +713,23 @@ DecodePlan plan_rows_split(int nb, int KT, int num_sms, int M) {
   if (ks < 1) ks = 1;
   p.kt_per_cta = (KT + ks - 1) / ks;
   p.ks = (KT + p.kt_per_cta - 1) / p.kt_per_cta;
-  p.smem = smem_for(p.nt);
+  p.smem = T == 1 ? smem_of<1>(ncol) : smem_of<2>(ncol);
   return p;
+}
+
+// Two-tile stages (two CTAs per SM) unless one-tile stages (three CTAs per
+// SM, accumulator <= 32 columns) allow a larger K split: per byte the longer
+// stages are cheaper, but more slices spread a launch over more CTAs
+// (measured on GB300: 4096 x 11008 prefers two-tile stages at K split 8;
+// 3 x 4096 x 4096 and 28672 x 8192 prefer one-tile stages).
+DecodePlan plan_rows_split(int nb, int KT, int num_sms, int M) {
+  const int ncol = ncol_for(M);
+  const DecodePlan p2 = plan_with(nb, KT, num_sms, ncol, 2);
+  if (ncol <= 32) {
+    const DecodePlan p1 = plan_with(nb, KT, num_sms, ncol, 1);
+    if (p1.ks > p2.ks) return p1;
+  }
+  return p2;
 }
 
 cudaLaunchAttribute pdl_attr() {
@@ -705,13 +739,13 @@ cudaLaunchAttribute pdl_attr() {
   return at;
 }
 
-template <int NCOL>
+template <int NCOL, int T>
 unisvq_status launch_ncol(const SkArgs& a, const DecodePlan& p, int dev, cudaStream_t s) {
-  if (!set_attrs<NCOL>(dev)) return UNISVQ_ERR_CUDA;
+  if (!set_attrs<NCOL, T>(dev)) return UNISVQ_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.ks, p.nb, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = Cfg<NCOL>::kSmem;
+  cfg.dynamicSmemBytes = Cfg<NCOL, T>::kSmem;
   cfg.stream = s;
   cudaLaunchAttribute attrs[2];
   attrs[0].id = cudaLaunchAttributeClusterDimension;
@@ -721,7 +755,7 @@ unisvq_status launch_ncol(const SkArgs& a, const DecodePlan& p, int dev, cudaStr
   attrs[1] = pdl_attr();
   cfg.attrs = attrs;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, decode_kernel<NCOL>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+  return cudaLaunchKernelEx(&cfg, decode_kernel<NCOL, T>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
 }  // namespace
@@ -787,9 +821,9 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
     fc.numAttrs = 1;
     if (cudaLaunchKernelEx(&fc, fold_kernel, f) != cudaSuccess) return UNISVQ_ERR_CUDA;
     unisvq_status st;
-    if (p.nt == 16) st = launch_ncol<16>(a, p, L0->device, s);
-    else if (p.nt == 32) st = launch_ncol<32>(a, p, L0->device, s);
-    else st = launch_ncol<48>(a, p, L0->device, s);
+    if (p.nt == 16) st = p.geom == 1 ? launch_ncol<16, 1>(a, p, L0->device, s) : launch_ncol<16, 2>(a, p, L0->device, s);
+    else if (p.nt == 32) st = p.geom == 1 ? launch_ncol<32, 1>(a, p, L0->device, s) : launch_ncol<32, 2>(a, p, L0->device, s);
+    else st = launch_ncol<48, 2>(a, p, L0->device, s);
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;

@@ -34,6 +34,7 @@ struct DecodePlan {
   int kt_per_cta;  // k-tiles per CTA
   int nb;          // row blocks of 128 rows
   size_t smem;     // dynamic shared memory bytes
+  int geom;        // skinny: k-tiles per pipeline stage (1 or 2)
 };
 
 struct PrefillPlan {

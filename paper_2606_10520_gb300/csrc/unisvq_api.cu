@@ -256,13 +256,13 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
 // of one launch and `nb` = their 128-row blocks (measured crossovers on
 // GB300, Llama-shaped layers): the tcgen05 skinny kernel (fold + streaming
 // kernel, cost nearly independent of M) for launches of at least 2^26
-// weights, and from four tokens up for launches of at least 2^25 weights
-// with 64 or more row blocks; the K-split cluster GEMV (lower fixed latency)
-// otherwise. The whole-K row-slice GEMV is reachable through the force
-// calls only.
+// weights, or of at least 2^25 weights over 64 or more row blocks; the K-split
+// cluster GEMV (lower fixed latency, better for few row blocks) otherwise.
+// The whole-K row-slice GEMV is reachable through the force calls only.
 static int decode_kernel_for(long long weights, int nb, int M) {
+  (void)M;
   if (weights >= (1ll << 26)) return UNISVQ_KERNEL_SKINNY;
-  if (weights >= (1ll << 25) && M >= 4 && nb >= 64) return UNISVQ_KERNEL_SKINNY;
+  if (weights >= (1ll << 25) && nb >= 64) return UNISVQ_KERNEL_SKINNY;
   return UNISVQ_KERNEL_GEMV;
 }
 

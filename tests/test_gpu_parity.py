@@ -239,15 +239,19 @@ def test_prefill_and_decode_agree_with_auto_dispatch():
 def test_dispatch_picks_tcgen05_decode_for_large_launches():
     """The library's pick (unisvq_query / unisvq_query_group): the tcgen05
     skinny path (fold + streaming kernel: two launches) from 2^26 weights per
-    launch, and from four tokens on 2^25 weights over >= 64 row blocks."""
+    launch, or from 2^25 weights over >= 64 row blocks; the GEMV otherwise."""
     big = binding.UniSVQLinear(*synth.layer_inputs(9, 91, 0, 0, 16384, 4096, 2))
     q = big.query(1)
     assert q["kernel"] == binding.KERNEL_SKINNY and q["launches"] == 2
     assert big.query(17)["launches"] == 4
     small = binding.UniSVQLinear(*synth.layer_inputs(9, 91, 1, 0, 4096, 4096, 2))
     assert small.query(16)["kernel"] == binding.KERNEL_GEMV and small.query(16)["launches"] == 1
+    tall = binding.UniSVQLinear(*synth.layer_inputs(9, 91, 2, 0, 4096, 11008, 2))   # 2^25.4 weights, 32 row blocks
+    assert tall.query(1)["kernel"] == binding.KERNEL_GEMV and tall.query(16)["kernel"] == binding.KERNEL_GEMV
+    tall.close()
     trio = [small, small.clone(), small.clone()]
-    assert binding.query_group(trio, 2)["kernel"] == binding.KERNEL_GEMV
+    assert binding.query_group(trio, 1)["kernel"] == binding.KERNEL_SKINNY
+    assert binding.query_group(trio[:1], 4)["kernel"] == binding.KERNEL_GEMV
     g4 = binding.query_group(trio, 4)
     assert g4["kernel"] == binding.KERNEL_SKINNY and g4["N"] == 3 * 4096 and g4["launches"] == 2
     xb = synth.activations(9, 91, 4, 4, 4096)
