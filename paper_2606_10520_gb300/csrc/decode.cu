@@ -53,12 +53,10 @@ constexpr int kWarps = 10;
 constexpr int kThreads = kWarps * 32;
 constexpr int kConvWarp0 = 2;
 constexpr int kConvWarps = 8;
-constexpr int kASlots = 3;                          // TMEM A slots (one stage each)
 constexpr int kMaxTokPerLaunch = 16;
 constexpr int kMaxSplit = 8;                        // K slices (cluster size)
 constexpr int kMaxGroup = UNISVQ_MAX_GROUP;
 constexpr int kFoldThreads = 256;
-static_assert(kConvWarps / 4 <= kASlots, "converter groups must not run two slot uses ahead");
 
 // Fold workspace of a handle (unisvq_layer::fold_ws): a table of per-(slice,
 // token) scale exponents and bias sums, then the B tiles of every k-tile.
@@ -101,12 +99,15 @@ struct FoldArgs {
 // Geometry: T k-tiles per pipeline stage. T = 2: 256 TMEM columns (accumulator
 // in [0, 64), three A slots of 64), two CTAs per SM. T = 1: 128 TMEM columns
 // (accumulator in [0, 32), three A slots of 32), N <= 32, three CTAs per SM.
+// (One-tile stages for N = 48 would leave room for two A slots only; measured
+// slower than two-tile stages on every Llama shape.)
 template <int NCOL, int T>
 struct Cfg {
   static constexpr int kT = T;
   static constexpr int kMinBlocks = T == 1 ? 3 : 2;
   static constexpr int kCodeBytes = T * kTileBytes;
   static constexpr int kAColBase = T == 1 ? 32 : 64;
+  static constexpr int kASlots = 3;                              // TMEM A slots (one stage each)
   static constexpr int kASlotCols = 32 * T;
   static constexpr int kTmemCols = T == 1 ? 128 : 256;
   static constexpr int kMaxTok = NCOL / 3;
@@ -128,6 +129,7 @@ struct Cfg {
   static_assert(kStages % (kConvWarps / 4) == 0, "a converter group revisits its own stages");
   static_assert(NCOL <= kAColBase, "accumulator columns");
   static_assert(kAColBase + kASlots * kASlotCols <= kTmemCols, "TMEM columns");
+  static_assert(kConvWarps / 4 <= kASlots, "converter groups must not run two slot uses ahead");
 };
 
 // ---- tcgen05 wrappers ----------------------------------------------------------
@@ -377,6 +379,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
   constexpr int kAColBase = C::kAColBase;
   constexpr int kASlotCols = C::kASlotCols;
   constexpr int kTmemCols = C::kTmemCols;
+  constexpr int kASlots = C::kASlots;
   constexpr int S = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);

@@ -76,6 +76,19 @@ def test_decode_parity_small_M(kernel, d, N, K):
     layer.close()
 
 
+def test_skinny_one_tile_stages_parity():
+    """12800 x 1024: 100 row blocks, so one-tile stages (three CTAs per SM)
+    allow a K split of 4 against 3 and the planner takes them for the 16- and
+    32-column accumulators (M = 3, 10); M = 16 and 17 mix in two-tile stages."""
+    N, K, d = 12800, 1024, 2
+    codes, A, B = synth.layer_inputs(6, 60, 0, 0, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    for M in (3, 10, 16, 17):
+        xb = synth.activations(6, 60, M, M, K)
+        check(run(layer, xb, binding.KERNEL_SKINNY), xb, codes, A, B)
+    layer.close()
+
+
 @pytest.mark.parametrize("kernel", DECODE_KERNELS)
 def test_decode_many_token_groups(kernel):
     N, K, d = 384, 768, 2
