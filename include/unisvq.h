@@ -12,7 +12,7 @@
  *     sum_i (X_i A) W_int,i^T + sum_i (X_i B) 1^T without a dequantised W.
  *
  * Shapes: x [M][K] bf16 (tokens x inputs), codes [N][K] (outputs x inputs),
- * y [M][N] bf16. d in {1, 2, 4}. No entry point ever writes a dequantised
+ * y [M][N] bf16. d in {1, 2, 4, 8}. No entry point ever writes a dequantised
  * weight matrix to device memory, except the test hook unisvq_dequant_debug.
  *
  * Streams are passed as `void*` holding a cudaStream_t (NULL = legacy default
@@ -99,12 +99,15 @@ typedef struct {
  *   A_f16 : host, [d][d] row-major IEEE fp16 bit patterns, w = A z + B
  *   B_f16 : host, [d] fp16 bit patterns
  *   N, K  : output / input features, N >= 1, K >= d, K % d == 0
- *   d     : vector length, 1, 2 or 4 (Eq. def:unisvq; the paper uses d = 4)
+ *   d     : vector length, 1, 2, 4 or 8 (Eq. def:unisvq; the paper uses d = 4
+ *           and d = 8 in its vector-length ablation, Table tab:ablation_dim).
+ *           The prefill GEMM takes d <= 4; d = 8 layers use the decode
+ *           kernels at every M.
  *   stream: stream for the upload; pack synchronises it before returning
  *   out   : receives the handle
  * The host buffers are copied before return; the caller keeps ownership.
  * Errors: INVALID_ARG (null pointer, bad shape, code > 3, non-finite A/B),
- * UNSUPPORTED (d not in {1,2,4}), OOM, CUDA.
+ * UNSUPPORTED (d not in {1,2,4,8}), OOM, CUDA.
  * The handle owns all device memory: the packed codes, the tables of the
  * prefill kernel and a fold workspace of 1 KB + (Kp/128) * 6 KB that the
  * decode kernels rewrite on every call (the folded activations of Eq.

@@ -83,8 +83,8 @@ struct FoldLayer {
   uint8_t* ws;
   int d;
   float colnorm;       // max_c sum_r |A[r][c]|
-  float A[16];
-  float B[4];
+  float A[64];         // row-major d x d (d <= 8)
+  float B[8];
 };
 
 struct FoldArgs {
@@ -254,26 +254,36 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
   __shared__ int sp;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int s = blockIdx.x, tok = blockIdx.y, li = blockIdx.z;
-  // This CTA's layer, read with constant parameter offsets only.
+  // This CTA's layer, read with constant parameter offsets only; A (up to
+  // 8 x 8) goes to shared memory, B[e mod d] for the 8 columns of a chunk to
+  // registers.
+  __shared__ float sA[64];
   uint8_t* ws = a.layer[0].ws;
   int d = a.layer[0].d;
   float colnorm = a.layer[0].colnorm;
-  float A[16], Bv[4];
-#pragma unroll
-  for (int i = 0; i < 16; ++i) A[i] = a.layer[0].A[i];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) Bv[i] = a.layer[0].B[i];
+  float Bv[8];
 #pragma unroll
   for (int l = 1; l < kMaxGroup; ++l)
     if (l == li) {
       ws = a.layer[l].ws;
       d = a.layer[l].d;
       colnorm = a.layer[l].colnorm;
-#pragma unroll
-      for (int i = 0; i < 16; ++i) A[i] = a.layer[l].A[i];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) Bv[i] = a.layer[l].B[i];
     }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    float v = a.layer[0].B[i & (a.layer[0].d - 1)];
+#pragma unroll
+    for (int l = 1; l < kMaxGroup; ++l)
+      if (l == li) v = a.layer[l].B[i & (a.layer[l].d - 1)];
+    Bv[i] = v;
+  }
+  if (tid < 64) {
+    float v = a.layer[0].A[tid];
+#pragma unroll
+    for (int l = 1; l < kMaxGroup; ++l)
+      if (l == li) v = a.layer[l].A[tid];
+    sA[tid] = v;
+  }
   const int kt0 = s * a.kt_per_cta;
   const int n_kt = min(a.kt_per_cta, a.KT - kt0);
   pdl_launch_dependents();   // the decode kernel may start fetching codes
@@ -311,8 +321,8 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
       for (int t = 0; t < 4; ++t) {   // kbeg and c are multiples of 8: (k + i) mod d = i mod d
         const float v0 = bf16_lo(w4[t]), v1 = bf16_hi(w4[t]);
         mx = fmaxf(mx, fmaxf(fabsf(v0), fabsf(v1)));
-        cs = fmaf(v0, Bv[(2 * t) & (d - 1)], cs);
-        cs = fmaf(v1, Bv[(2 * t + 1) & (d - 1)], cs);
+        cs = fmaf(v0, Bv[2 * t], cs);
+        cs = fmaf(v1, Bv[2 * t + 1], cs);
       }
     }
   }
@@ -353,10 +363,28 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
     const int kt = item >> 5, g = item & 31;
     const uint32_t ac = 16 * (g >> 4) + 8 * ((g & 3) >> 1) + 2 * ((g >> 2) & 3) + (g & 1);
     const uint32_t cidx = (ac & 3) * 4, chunk = ac >> 2;
-    const uint2 xv = *reinterpret_cast<const uint2*>(xs + kt * kTileCols + 4 * g);
-    const float v[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
     float o[4];
-    fold4(d, A, v, o);
+    if (d == 8) {
+      // Columns 4g .. 4g+3 are coordinates 4(g%2) .. of the vector 8(g/2) ..
+      const uint4 xv = *reinterpret_cast<const uint4*>(xs + kt * kTileCols + 8 * (g >> 1));
+      const float v[8] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y),
+                          bf16_lo(xv.z), bf16_hi(xv.z), bf16_lo(xv.w), bf16_hi(xv.w)};
+      const int c0 = 4 * (g & 1);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        float acc = 0.f;
+#pragma unroll
+        for (int r = 0; r < 8; ++r) acc = fmaf(v[r], sA[8 * r + c0 + j], acc);
+        o[j] = acc;
+      }
+    } else {
+      const uint2 xv = *reinterpret_cast<const uint2*>(xs + kt * kTileCols + 4 * g);
+      const float v[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
+      float A[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) A[i] = sA[i];
+      fold4(d, A, v, o);
+    }
     const float sc = exp2i(P + ((g & 1) ? -2 : 0));
     uint16_t h0, m0, l0, h1, m1, l1;
     split3(pack_half2(o[0] * sc, o[1] * sc), h0, m0, l0);
@@ -804,8 +832,8 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
       fl.ws = ws[i];
       fl.d = L->d;
       fl.colnorm = L->colnorm;
-      for (int j = 0; j < 16; ++j) fl.A[j] = L->A[j];
-      for (int j = 0; j < 4; ++j) fl.B[j] = L->B[j];
+      for (int j = 0; j < 64; ++j) fl.A[j] = L->A[j];
+      for (int j = 0; j < 8; ++j) fl.B[j] = L->B[j];
       SkLayer& l = a.layer[i];
       l.codes = L->codes;
       l.ws = ws[i];

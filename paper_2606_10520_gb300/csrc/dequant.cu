@@ -26,22 +26,24 @@ __global__ void __launch_bounds__(256) dequant_kernel(const uint8_t* __restrict_
   for (int t = 0; t < 4; ++t) words[t] = *reinterpret_cast<const uint32_t*>(tb + tile_word_offset(r, h, t));
 #pragma unroll
   for (int wi = 0; wi < 4; ++wi) {
+    // The 16 codes of the word: z[4s + b] = column 4s + b (16 consecutive
+    // columns, so a d-vector, d <= 8, never leaves the word).
+    uint32_t z[16];
 #pragma unroll
     for (int s = 0; s < 4; ++s) {
       const uint32_t e = extract4(words[wi], s);   // columns 4s .. 4s+3 of the word
-      const int k0 = kt * kTileCols + 64 * h + 16 * wi + 4 * s;
-      uint32_t z[4];
 #pragma unroll
-      for (int b = 0; b < 4; ++b) z[b] = (e >> (8 * b)) & 3u;
+      for (int b = 0; b < 4; ++b) z[4 * s + b] = (e >> (8 * b)) & 3u;
+    }
+    const int k0 = kt * kTileCols + 64 * h + 16 * wi;
 #pragma unroll
-      for (int b = 0; b < 4; ++b) {
-        const int k = k0 + b;
-        if (k >= K) continue;
-        const int v0 = b & ~(d - 1);            // first coordinate of this column's vector
-        uint32_t idx = 0;
-        for (int c = 0; c < d; ++c) idx |= z[v0 + c] << (2 * c);
-        W[static_cast<size_t>(row) * K + k] = lut[idx * d + (b & (d - 1))];
-      }
+    for (int j = 0; j < 16; ++j) {
+      const int k = k0 + j;
+      if (k >= K) continue;
+      const int v0 = j & ~(d - 1);              // first coordinate of this column's vector
+      uint32_t idx = 0;
+      for (int c = 0; c < d; ++c) idx |= z[v0 + c] << (2 * c);
+      W[static_cast<size_t>(row) * K + k] = lut[idx * d + (j & (d - 1))];
     }
   }
 }

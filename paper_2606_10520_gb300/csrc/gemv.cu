@@ -42,6 +42,8 @@ constexpr int kXPad = 4;            // fp16 elements of padding per token row (b
 constexpr int kTokBytes = 272;      // pexp[32], cpart[32], reduction mbarrier
 constexpr size_t kSmemPerSm = 228 * 1024;
 constexpr size_t kSmemPerCtaReserved = 1024;
+constexpr size_t kStaticSmem = 64 * sizeof(float);   // sA8 of both kernels
+constexpr size_t kDynSmemMax = kSmemPerSm - kSmemPerCtaReserved - kStaticSmem;
 
 // One layer of a launch. A launch covers one layer, or several layers that
 // read the same x (same K): their row blocks are stacked along grid.y.
@@ -51,8 +53,8 @@ struct GemvLayer {
   int N, d;
   int rb0;             // first grid.y row block of this layer
   float colnorm;
-  float A[16];
-  float B[4];
+  float A[64];         // row-major d x d (d <= 8)
+  float B[8];
 };
 
 struct GemvArgs {
@@ -94,15 +96,45 @@ __device__ __forceinline__ void gfold4(int d, const float (&A)[16], const float 
   }
 }
 
+struct Vec8 {
+  float v[8];
+};
+
+// x' = x_g A for one vector of d = 8 (A row-major in shared memory). Kept out
+// of line: it runs in the fold only and would otherwise crowd the registers
+// of the main loop.
+__device__ __noinline__ Vec8 fold_vec8(const float* sA8, Vec8 x) {
+  Vec8 o;
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    float acc = 0.f;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) acc = fmaf(x.v[r], sA8[8 * r + c], acc);
+    o.v[c] = acc;
+  }
+  return o;
+}
+
 // Columns 8ci .. 8ci+7 of a token's slice (packed bf16 xv) -> their B fragments:
-// four-column groups j0 = 2ci mod 4 and j0 + 1, scaled by 2^(pe - 2j).
-__device__ __forceinline__ uint4 fold8(int ci, uint4 xv, int pe, int d, const float (&A)[16]) {
+// four-column groups j0 = 2ci mod 4 and j0 + 1, scaled by 2^(pe - 2j). For
+// d = 8 the eight columns are one vector and A comes from shared memory (sA8,
+// row-major 8 x 8); otherwise from the register copy A.
+__device__ __forceinline__ uint4 fold8(int ci, uint4 xv, int pe, int d, const float (&A)[16], const float* sA8) {
   const int j0 = (2 * ci) & 3;
   const float v0[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
   const float v1[4] = {bf16_lo(xv.z), bf16_hi(xv.z), bf16_lo(xv.w), bf16_hi(xv.w)};
   float o0[4], o1[4];
-  gfold4(d, A, v0, o0);
-  gfold4(d, A, v1, o1);
+  if (d == 8) {
+    const Vec8 o = fold_vec8(sA8, Vec8{{v0[0], v0[1], v0[2], v0[3], v1[0], v1[1], v1[2], v1[3]}});
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      o0[c] = o.v[c];
+      o1[c] = o.v[4 + c];
+    }
+  } else {
+    gfold4(d, A, v0, o0);
+    gfold4(d, A, v1, o1);
+  }
   const float s0 = exp2i(pe - 2 * j0), s1 = exp2i(pe - 2 * j0 - 2);
   return make_uint4(pack_half2(o0[0] * s0, o0[2] * s0), pack_half2(o0[1] * s0, o0[3] * s0),
                     pack_half2(o1[0] * s1, o1[2] * s1), pack_half2(o1[1] * s1, o1[3] * s1));
@@ -142,7 +174,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   const uint8_t* codes = nullptr;
   uint16_t* yout = nullptr;
   int N = 0, d = 1, rb = 0;
-  float colnorm = 0.f, Areg[16], Bq[4];
+  float colnorm = 0.f, Areg[16], Bcol[8];   // Bcol[e] = B[e mod d] for column e of an 8-column chunk
 #pragma unroll
   for (int i = 0; i < kMaxGroup; ++i) {
     if (i == li) {
@@ -155,12 +187,20 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
 #pragma unroll
       for (int e = 0; e < 16; ++e) Areg[e] = a.layer[i].A[e];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) Bq[e] = a.layer[i].B[e];
+      for (int e = 0; e < 8; ++e) Bcol[e] = a.layer[i].B[e & (a.layer[i].d - 1)];
     }
   }
-  float Bcol[8];   // B[e mod d] for column e of an 8-column chunk
+  __shared__ float sA8[64];   // A for d = 8 (the fold reads it from here)
+  if (d == 8) {
+    if (tid < 64) {
+      float v = a.layer[0].A[tid];
 #pragma unroll
-  for (int e = 0; e < 8; ++e) Bcol[e] = d == 1 ? Bq[0] : (d == 2 ? Bq[e & 1] : Bq[e & 3]);
+      for (int i = 1; i < kMaxGroup; ++i)
+        if (i == li) v = a.layer[i].A[tid];
+      sA8[tid] = v;
+    }
+    __syncthreads();
+  }
   // Rows whose K-slice partial sums this CTA adds up (it "owns" them).
   const int rows_per = (kTileRows + KS - 1) / KS;
   const int own0 = static_cast<int>(blockIdx.x) * rows_per;
@@ -253,7 +293,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
         uint8_t* xrow = smem + tk * xrow_bytes;
         uint4 f[kXLoads];
 #pragma unroll
-        for (int j = 0; j < kXLoads; ++j) f[j] = fold8(lane + 32 * j, u[p][j], pe, d, Areg);
+        for (int j = 0; j < kXLoads; ++j) f[j] = fold8(lane + 32 * j, u[p][j], pe, d, Areg, sA8);
 #pragma unroll
         for (int j = 0; j < kXLoads; ++j) {
           const int ci = lane + 32 * j;
@@ -313,7 +353,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
           if (ci < nch) {
             const uint2 lo = *reinterpret_cast<const uint2*>(xrow + 16u * ci);
             const uint2 hi = *reinterpret_cast<const uint2*>(xrow + 16u * ci + 8);
-            u[j] = fold8(ci, make_uint4(lo.x, lo.y, hi.x, hi.y), pe, d, Areg);
+            u[j] = fold8(ci, make_uint4(lo.x, lo.y, hi.x, hi.y), pe, d, Areg, sA8);
           }
         }
 #pragma unroll
@@ -454,7 +494,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_rows_kernel(const __grid_co
   const uint8_t* codes = nullptr;
   uint16_t* yout = nullptr;
   int N = 0, d = 1, pr = 0;
-  float colnorm = 0.f, Areg[16], Bq[4];
+  float colnorm = 0.f, Areg[16], Bcol[8];   // Bcol[e] = B[e mod d] for column e of an 8-column chunk
 #pragma unroll
   for (int i = 0; i < kMaxGroup; ++i) {
     if (i == li) {
@@ -467,12 +507,20 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_rows_kernel(const __grid_co
 #pragma unroll
       for (int e = 0; e < 16; ++e) Areg[e] = a.layer[i].A[e];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) Bq[e] = a.layer[i].B[e];
+      for (int e = 0; e < 8; ++e) Bcol[e] = a.layer[i].B[e & (a.layer[i].d - 1)];
     }
   }
-  float Bcol[8];
+  __shared__ float sA8[64];   // A for d = 8 (the fold reads it from here)
+  if (d == 8) {
+    if (threadIdx.x < 64) {
+      float v = a.layer[0].A[threadIdx.x];
 #pragma unroll
-  for (int e = 0; e < 8; ++e) Bcol[e] = d == 1 ? Bq[0] : (d == 2 ? Bq[e & 1] : Bq[e & 3]);
+      for (int i = 1; i < kMaxGroup; ++i)
+        if (i == li) v = a.layer[i].A[threadIdx.x];
+      sA8[threadIdx.x] = v;
+    }
+    __syncthreads();
+  }
 
   const int kpw = a.kt_per_cta;
   const int kw0 = warp * kpw;
@@ -566,7 +614,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_rows_kernel(const __grid_co
           if (q == tk) pt = pe[q];
         const uint8_t* src = wreg + tk * wstride + 16u * ci;
         const uint2 lo = *reinterpret_cast<const uint2*>(src), hi = *reinterpret_cast<const uint2*>(src + 8);
-        f[r] = fold8(ci, make_uint4(lo.x, lo.y, hi.x, hi.y), pt, d, Areg);
+        f[r] = fold8(ci, make_uint4(lo.x, lo.y, hi.x, hi.y), pt, d, Areg, sA8);
       }
     }
 #pragma unroll
@@ -678,7 +726,7 @@ unisvq_status gemv_launch_nt(const unisvq_layer* const* Ls, int n, const DecodeP
   if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
   if (!attr_set[dev]) {
     if (cudaFuncSetAttribute(gemv_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(kSmemPerSm - kSmemPerCtaReserved)) != cudaSuccess ||
+                             static_cast<int>(kDynSmemMax)) != cudaSuccess ||
         cudaFuncSetAttribute(gemv_kernel<NT>, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared) != cudaSuccess)
       return UNISVQ_ERR_CUDA;
@@ -706,8 +754,8 @@ unisvq_status gemv_launch_nt(const unisvq_layer* const* Ls, int n, const DecodeP
     g.d = L->d;
     g.rb0 = rb0;
     g.colnorm = L->colnorm;
-    for (int e = 0; e < 16; ++e) g.A[e] = L->A[e];
-    for (int e = 0; e < 4; ++e) g.B[e] = L->B[e];
+    for (int e = 0; e < 64; ++e) g.A[e] = L->A[e];
+    for (int e = 0; e < 8; ++e) g.B[e] = L->B[e];
     rb0 += L->Np / kTileRows;
   }
 
@@ -735,7 +783,7 @@ DecodePlan plan_rows(int nb, int KT, int num_sms, int M) {
   DecodePlan p{};
   p.nt = M <= 8 ? 1 : (M <= 16 ? 2 : 4);
   p.nb = nb;
-  const size_t cap = kSmemPerSm - kSmemPerCtaReserved;
+  const size_t cap = kDynSmemMax;
   int best = 0, fallback = 0;
   for (int c = kMaxSplit; c >= 1; --c) {
     if (c > KT) continue;
@@ -745,7 +793,7 @@ DecodePlan plan_rows(int nb, int KT, int num_sms, int M) {
     const size_t smem = gemv_shape(M, kpc, ks, p.nt).smem;
     if (smem > cap) continue;
     fallback = ks;
-    const int per_sm = static_cast<int>(kSmemPerSm / (smem + kSmemPerCtaReserved)) < 2 ? 1 : 2;
+    const int per_sm = static_cast<int>(kSmemPerSm / (smem + kStaticSmem + kSmemPerCtaReserved)) < 2 ? 1 : 2;
     if (!best && nb * ks <= per_sm * num_sms) best = ks;
   }
   const int ks = best ? best : (fallback ? fallback : kMaxSplit);
@@ -775,7 +823,7 @@ unisvq_status rows_launch(const unisvq_layer* const* Ls, int n, const void* x, v
   if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
   if (!attr_set[dev]) {
     if (cudaFuncSetAttribute(gemv_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(kSmemPerSm - kSmemPerCtaReserved)) != cudaSuccess ||
+                             static_cast<int>(kDynSmemMax)) != cudaSuccess ||
         cudaFuncSetAttribute(gemv_rows_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared) != cudaSuccess)
       return UNISVQ_ERR_CUDA;
@@ -803,8 +851,8 @@ unisvq_status rows_launch(const unisvq_layer* const* Ls, int n, const void* x, v
     g.d = L->d;
     g.rb0 = pairs;
     g.colnorm = L->colnorm;
-    for (int e = 0; e < 16; ++e) g.A[e] = L->A[e];
-    for (int e = 0; e < 4; ++e) g.B[e] = L->B[e];
+    for (int e = 0; e < 64; ++e) g.A[e] = L->A[e];
+    for (int e = 0; e < 8; ++e) g.B[e] = L->B[e];
     pairs += L->Np / (2 * kUnitRows);
   }
   cudaLaunchConfig_t cfg = {};
@@ -834,11 +882,11 @@ unisvq_status launch_gemv_group(const unisvq_layer* const* Ls, int n, const void
     // would not fit in shared memory
     int mc = M - m0 < kGMaxTok ? M - m0 : kGMaxTok;
     DecodePlan p = plan_rows(nb, Ls[0]->KT, Ls[0]->num_sms, mc);
-    while (p.smem > kSmemPerSm - kSmemPerCtaReserved && mc > 1) {
+    while (p.smem > kDynSmemMax && mc > 1) {
       mc = (mc + 1) / 2;
       p = plan_rows(nb, Ls[0]->KT, Ls[0]->num_sms, mc);
     }
-    if (p.smem > kSmemPerSm - kSmemPerCtaReserved) return UNISVQ_ERR_UNSUPPORTED;
+    if (p.smem > kDynSmemMax) return UNISVQ_ERR_UNSUPPORTED;
     const unisvq_status st = p.nt == 1   ? gemv_launch_nt<1>(Ls, n, p, x, ys, m0, mc, s)
                              : p.nt == 2 ? gemv_launch_nt<2>(Ls, n, p, x, ys, m0, mc, s)
                                          : gemv_launch_nt<4>(Ls, n, p, x, ys, m0, mc, s);
@@ -853,7 +901,7 @@ unisvq_status launch_gemv(const unisvq_layer* L, const void* x, void* y, int M, 
 }
 
 bool gemv_rows_supported(const unisvq_layer* L, int M) {
-  return M >= 1 && M <= kRMaxTok && rows_smem(M, L->KT, nullptr, nullptr) <= kSmemPerSm / 2 - kSmemPerCtaReserved;
+  return M >= 1 && M <= kRMaxTok && rows_smem(M, L->KT, nullptr, nullptr) <= kSmemPerSm / 2 - kSmemPerCtaReserved - kStaticSmem;
 }
 
 unisvq_status launch_gemv_rows_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,

@@ -19,11 +19,11 @@ struct unisvq_layer {
   uint32_t* tlut;          // device, prefill codeword table (bf16 pairs / quads), see pack
   int tlut_words;
   int lut_entries;         // 4^d
-  float A[16];             // fp32 (exact) copy of A, row-major d x d
-  float B[4];              // fp32 (exact) copy of B
+  float A[64];             // fp32 (exact) copy of A, row-major d x d (d <= 8)
+  float B[8];              // fp32 (exact) copy of B
   float colnorm;           // max_c sum_r |A[r][c]|: |x A|_inf <= |x|_inf * colnorm
   uint8_t* fold_ws;        // device, decode fold workspace (fold_workspace_bytes(KT))
-  uint16_t A16[16], B16[4];
+  uint16_t A16[64], B16[8];
 };
 
 namespace unisvq {

@@ -82,7 +82,7 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
   if (!out) return UNISVQ_ERR_INVALID_ARG;
   *out = nullptr;
   if (!codes || !A_f16 || !B_f16) return UNISVQ_ERR_INVALID_ARG;
-  if (d != 1 && d != 2 && d != 4) return UNISVQ_ERR_UNSUPPORTED;
+  if (d != 1 && d != 2 && d != 4 && d != 8) return UNISVQ_ERR_UNSUPPORTED;
   if (N <= 0 || K <= 0 || K % d != 0) return UNISVQ_ERR_INVALID_ARG;
   if (static_cast<long long>(round_up(N, kRowPad)) * round_up(K, kColPad) >= (1ll << 40))
     return UNISVQ_ERR_UNSUPPORTED;
@@ -93,7 +93,7 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
   for (long long i = 0; i < static_cast<long long>(total); ++i) bad |= codes[i] > 3;
   if (bad) return UNISVQ_ERR_INVALID_ARG;
 
-  double A[16], B[4];
+  double A[64], B[8];
   for (int i = 0; i < d * d; ++i) {
     A[i] = f16_bits_to_f64(A_f16[i]);
     if (!std::isfinite(A[i])) return UNISVQ_ERR_INVALID_ARG;
@@ -150,10 +150,14 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
     }
   // Prefill tile table, indexed the way the converter warps read code bytes:
   //   d <= 2: 16 bf16 pairs, index lo | hi << 2 for two adjacent columns (k, k+1);
-  //   d == 4: 256 bf16 quads, index z0 | z1 << 2 | z2 << 4 | z3 << 6.
+  //   d == 4: 256 bf16 quads, index z0 | z1 << 2 | z2 << 4 | z3 << 6;
+  //   d == 8: none (4^8 codewords do not fit the converters' shared memory;
+  //   such layers run the decode kernels at every M).
   auto bf = [](double w) { return static_cast<uint32_t>(f64_to_bf16_rne(w)); };
   std::vector<uint32_t> tlut;
-  if (d <= 2) {
+  if (d == 8) {
+    tlut.assign(1, 0u);
+  } else if (d <= 2) {
     tlut.resize(16);
     for (int v = 0; v < 16; ++v) {
       const int lo = v & 3, hi = v >> 2;

@@ -44,7 +44,7 @@ def check(yg, xbits, codes, A, B, rows=None):
     return res
 
 
-@pytest.mark.parametrize("d", [1, 2, 4])
+@pytest.mark.parametrize("d", [1, 2, 4, 8])
 @pytest.mark.parametrize("N,K", [(200, 520), (128, 128), (300, 1024)])
 def test_dequant_debug_bit_exact(d, N, K):
     codes, A, B = synth.layer_inputs(1, 10, N, K, N, K, d)
@@ -63,7 +63,7 @@ DECODE_KERNELS = [binding.KERNEL_GEMV, binding.KERNEL_GEMV_ROWS, binding.KERNEL_
 
 
 @pytest.mark.parametrize("kernel", DECODE_KERNELS)
-@pytest.mark.parametrize("d", [1, 2, 4])
+@pytest.mark.parametrize("d", [1, 2, 4, 8])
 @pytest.mark.parametrize("N,K", DECODE_SHAPES)
 def test_decode_parity_small_M(kernel, d, N, K):
     if K % d:
@@ -215,6 +215,47 @@ def test_prefill_parity(d, N, K):
     for M in (33, 64, 65, 128, 200, 256, 300, 777):
         xb = synth.activations(8, 80, 1000 * N + M, M, K)
         check(run(layer, xb, binding.KERNEL_PREFILL), xb, codes, A, B)
+    layer.close()
+
+
+def test_d8_layers_run_the_decode_kernels_at_every_M():
+    """d = 8 (the paper's ablation length): the prefill kernel declines it (its
+    exact codeword table would have 4^8 entries), so M > 64 runs the decode
+    kernels, chunk by chunk, and still meets the oracle."""
+    d, N, K = 8, 300, 1024
+    codes, A, B = synth.layer_inputs(8, 81, N, K, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    x = torch.zeros((80, K), dtype=torch.bfloat16, device="cuda")
+    y = torch.zeros((80, N), dtype=torch.bfloat16, device="cuda")
+    st = layer.forward_ptr(x.data_ptr(), y.data_ptr(), 80, torch.cuda.current_stream().cuda_stream,
+                           binding.KERNEL_PREFILL)
+    assert st == binding.ERR_UNSUPPORTED
+    assert layer.query(200)["kernel"] != binding.KERNEL_PREFILL
+    for M in (65, 200):
+        xb = synth.activations(8, 81, M, M, K)
+        check(run(layer, xb), xb, codes, A, B)
+    layer.close()
+
+
+@pytest.mark.parametrize("kernel", DECODE_KERNELS)
+def test_d8_integer_case_bit_exact(kernel):
+    """Integer 8 x 8 A (unit lower bidiagonal with -1 below the diagonal),
+    integer B and sparse integer x: exact at every step, so the output must
+    equal the oracle's bit for bit."""
+    d = 8
+    A = (np.eye(d) - np.eye(d, k=-1)).astype(np.float16)
+    B = np.array([1, -2, 0, 1, 3, -1, 0, 2], dtype=np.float16)
+    N, K = 256, 512
+    g = np.random.default_rng(17)
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    layer = binding.UniSVQLinear(codes, A, B)
+    for M in (1, 5, 16):
+        x = g.integers(-1, 2, size=(M, K)).astype(np.float32) * (g.random((M, K)) < 0.05)
+        xb = synth.f32_to_bf16_bits(x)
+        yr, _ = oracle.linear(xb, codes, A, B)
+        assert np.abs(yr).max() <= 256
+        yg = run(layer, xb, kernel)
+        assert np.array_equal(yg, yr), np.abs(yg - yr).max()
     layer.close()
 
 

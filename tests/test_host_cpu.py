@@ -98,6 +98,21 @@ def test_pack_rejects_bad_arguments_before_touching_the_gpu(lib):
     assert _pack_status(lib, codes, Anan, B, 4, 8, 2) == binding.ERR_INVALID_ARG
 
 
+def test_pack_takes_the_paper_vector_lengths_only(lib):
+    """d in {1, 2, 4, 8}: the lengths the paper evaluates (d = 8 in its vector
+    length ablation); anything else is UNSUPPORTED, and K must be a multiple of d."""
+    from paper_2606_10520_gb300 import binding
+    codes = np.zeros((4, 24), dtype=np.uint8)
+    A8 = np.eye(8, dtype=np.float16).view(np.uint16)
+    B8 = np.zeros(8, dtype=np.float16).view(np.uint16)
+    A8nan = A8.copy()
+    A8nan[7, 7] = np.array([np.inf], dtype=np.float16).view(np.uint16)[0]
+    for d in (3, 5, 6, 16):
+        assert _pack_status(lib, codes, A8, B8, 4, 24, d) == binding.ERR_UNSUPPORTED
+    assert _pack_status(lib, codes, A8, B8, 4, 20, 8) == binding.ERR_INVALID_ARG      # K % 8
+    assert _pack_status(lib, codes, A8nan, B8, 4, 24, 8) == binding.ERR_INVALID_ARG   # A[7][7] = inf
+
+
 def test_linear_rejects_bad_arguments(lib):
     from paper_2606_10520_gb300 import binding
     assert lib.unisvq_linear(None, None, None, 1, None) == binding.ERR_INVALID_ARG

@@ -150,7 +150,7 @@ def test_sq_special_case():
     pin_sq_special_case(oracle.dequant)
 
 
-@pytest.mark.parametrize("d", [1, 2, 4])
+@pytest.mark.parametrize("d", [1, 2, 4, 8])
 def test_block_form_matches_vector_form(d):
     pin_block_form(oracle.dequant, d)
 
@@ -172,7 +172,7 @@ def test_linearity():
     pin_linearity(oracle_linear_y)
 
 
-@pytest.mark.parametrize("d", [1, 2, 4])
+@pytest.mark.parametrize("d", [1, 2, 4, 8])
 def test_fold_identity(d):
     """Eq. (col:matmul) (fold onto activations) equals the direct form."""
     g = synth.rng(0, 99, d)
@@ -187,7 +187,7 @@ def test_fold_identity(d):
 def test_codebook_is_dequant_of_every_index():
     """`codebook` row v is the dequantisation of the lattice point whose
     coordinate c is bit-field [2c+1:2c] of v."""
-    for d in (1, 2, 4):
+    for d in (1, 2, 4, 8):
         g = np.random.default_rng(d)
         A = g.standard_normal((d, d))
         B = g.standard_normal(d)
