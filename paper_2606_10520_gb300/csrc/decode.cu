@@ -79,21 +79,26 @@ struct SkArgs {
   SkLayer layer[kMaxGroup];
 };
 
+// The fold kernel is instantiated for DV, the largest vector length of the
+// launch's layers: DV = 4 (d in {1, 2, 4}) keeps A in registers and the
+// parameter block small; DV = 8 stages the 8 x 8 A in shared memory.
+template <int DV>
 struct FoldLayer {
   uint8_t* ws;
   int d;
   float colnorm;       // max_c sum_r |A[r][c]|
-  float A[64];         // row-major d x d (d <= 8)
-  float B[8];
+  float A[DV * DV];    // row-major d x d (d <= DV)
+  float B[DV];
 };
 
+template <int DV>
 struct FoldArgs {
   const uint16_t* x;   // bf16 [M][K]
   int M, K, KT;
   int kt_per_cta;
   int ncol;            // B rows (16, 32, 48)
   int nlayers;
-  FoldLayer layer[kMaxGroup];
+  FoldLayer<DV> layer[kMaxGroup];
 };
 
 // Geometry: T k-tiles per pipeline stage. T = 2: 256 TMEM columns (accumulator
@@ -247,42 +252,57 @@ __device__ __forceinline__ void fold4(int d, const float (&A)[16], const float (
 // the layer's workspace. Rows of absent tokens are never written: an MMA
 // column depends on its own B row only, and the epilogue never reads those
 // columns.
-__global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constant__ FoldArgs a) {
+template <int DV>
+__global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constant__ FoldArgs<DV> a) {
   extern __shared__ __align__(16) uint8_t fsm[];
   uint16_t* xs = reinterpret_cast<uint16_t*>(fsm);   // the token's x slice, zero past K
   __shared__ float wmx[kFoldThreads / 32], wcs[kFoldThreads / 32];
   __shared__ int sp;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int s = blockIdx.x, tok = blockIdx.y, li = blockIdx.z;
-  // This CTA's layer, read with constant parameter offsets only; A (up to
-  // 8 x 8) goes to shared memory, B[e mod d] for the 8 columns of a chunk to
-  // registers.
-  __shared__ float sA[64];
+  // This CTA's layer, read with constant parameter offsets only. For DV = 4,
+  // A and B go to registers; for DV = 8, A goes to shared memory and
+  // Bv[i] = B[i mod d] (the 8 columns of a chunk) to registers.
+  __shared__ float sA[DV == 8 ? 64 : 1];
   uint8_t* ws = a.layer[0].ws;
   int d = a.layer[0].d;
   float colnorm = a.layer[0].colnorm;
-  float Bv[8];
+  float A4[16], Bv[DV == 8 ? 8 : 4];
+  if constexpr (DV == 4) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) A4[i] = a.layer[0].A[i];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) Bv[i] = a.layer[0].B[i];
+  }
 #pragma unroll
   for (int l = 1; l < kMaxGroup; ++l)
     if (l == li) {
       ws = a.layer[l].ws;
       d = a.layer[l].d;
       colnorm = a.layer[l].colnorm;
+      if constexpr (DV == 4) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) A4[i] = a.layer[l].A[i];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) Bv[i] = a.layer[l].B[i];
+      }
     }
+  if constexpr (DV == 8) {
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    float v = a.layer[0].B[i & (a.layer[0].d - 1)];
+    for (int i = 0; i < 8; ++i) {
+      float v = a.layer[0].B[i & (a.layer[0].d - 1)];
 #pragma unroll
-    for (int l = 1; l < kMaxGroup; ++l)
-      if (l == li) v = a.layer[l].B[i & (a.layer[l].d - 1)];
-    Bv[i] = v;
-  }
-  if (tid < 64) {
-    float v = a.layer[0].A[tid];
+      for (int l = 1; l < kMaxGroup; ++l)
+        if (l == li) v = a.layer[l].B[i & (a.layer[l].d - 1)];
+      Bv[i] = v;
+    }
+    if (tid < 64) {
+      float v = a.layer[0].A[tid];
 #pragma unroll
-    for (int l = 1; l < kMaxGroup; ++l)
-      if (l == li) v = a.layer[l].A[tid];
-    sA[tid] = v;
+      for (int l = 1; l < kMaxGroup; ++l)
+        if (l == li) v = a.layer[l].A[tid];
+      sA[tid] = v;
+    }
   }
   const int kt0 = s * a.kt_per_cta;
   const int n_kt = min(a.kt_per_cta, a.KT - kt0);
@@ -321,8 +341,13 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
       for (int t = 0; t < 4; ++t) {   // kbeg and c are multiples of 8: (k + i) mod d = i mod d
         const float v0 = bf16_lo(w4[t]), v1 = bf16_hi(w4[t]);
         mx = fmaxf(mx, fmaxf(fabsf(v0), fabsf(v1)));
-        cs = fmaf(v0, Bv[2 * t], cs);
-        cs = fmaf(v1, Bv[2 * t + 1], cs);
+        if constexpr (DV == 8) {
+          cs = fmaf(v0, Bv[2 * t], cs);
+          cs = fmaf(v1, Bv[2 * t + 1], cs);
+        } else {
+          cs = fmaf(v0, Bv[(2 * t) & (d - 1)], cs);
+          cs = fmaf(v1, Bv[(2 * t + 1) & (d - 1)], cs);
+        }
       }
     }
   }
@@ -355,6 +380,10 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
   const int P = sp;
   const int ncol = a.ncol;
   uint8_t* tiles = ws + kWsTableBytes + static_cast<size_t>(kt0) * ncol * 128;
+  if constexpr (DV == 8) {   // A for d <= 4 layers of the launch, in registers for the item loop
+#pragma unroll
+    for (int i = 0; i < 16; ++i) A4[i] = sA[i];
+  }
   // Item (k-tile kt, column group g): columns 4g .. 4g + 3 of the tile, i.e.
   // quarter t = (g/4) % 4, s = g % 4, half h = g / 16, which sit in A-slot
   // column ac = 16h + 8(s/2) + 2t + s%2 (expand_unit): bytes 4 ac .. 4 ac + 3
@@ -364,7 +393,7 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
     const uint32_t ac = 16 * (g >> 4) + 8 * ((g & 3) >> 1) + 2 * ((g >> 2) & 3) + (g & 1);
     const uint32_t cidx = (ac & 3) * 4, chunk = ac >> 2;
     float o[4];
-    if (d == 8) {
+    if (DV == 8 && d == 8) {
       // Columns 4g .. 4g+3 are coordinates 4(g%2) .. of the vector 8(g/2) ..
       const uint4 xv = *reinterpret_cast<const uint4*>(xs + kt * kTileCols + 8 * (g >> 1));
       const float v[8] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y),
@@ -380,10 +409,7 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
     } else {
       const uint2 xv = *reinterpret_cast<const uint2*>(xs + kt * kTileCols + 4 * g);
       const float v[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
-      float A[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) A[i] = sA[i];
-      fold4(d, A, v, o);
+      fold4(d, A4, v, o);
     }
     const float sc = exp2i(P + ((g & 1) ? -2 : 0));
     uint16_t h0, m0, l0, h1, m1, l1;
@@ -700,7 +726,8 @@ bool set_fold_attrs(int dev) {
   static bool done[64] = {};
   if (dev < 0 || dev >= 64) return false;
   if (done[dev]) return true;
-  if (cudaFuncSetAttribute(fold_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kFoldMaxSmem) != cudaSuccess)
+  if (cudaFuncSetAttribute(fold_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFoldMaxSmem) != cudaSuccess ||
+      cudaFuncSetAttribute(fold_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFoldMaxSmem) != cudaSuccess)
     return false;
   done[dev] = true;
   return true;
@@ -799,6 +826,39 @@ DecodePlan plan_skinny(const unisvq_layer* L, int M) {
 
 namespace {
 
+// The fold of tokens m0 .. m0 + mc - 1 for plan p (fold_kernel<DV>).
+template <int DV>
+unisvq_status launch_fold(const unisvq_layer* const* Ls, int n, const void* x, int m0, int mc, const DecodePlan& p,
+                          cudaStream_t s, uint8_t* const* ws) {
+  const unisvq_layer* L0 = Ls[0];
+  FoldArgs<DV> f{};
+  f.x = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * L0->K;
+  f.M = mc;
+  f.K = L0->K;
+  f.KT = L0->KT;
+  f.kt_per_cta = p.kt_per_cta;
+  f.ncol = p.nt;
+  f.nlayers = n;
+  for (int i = 0; i < n; ++i) {
+    const unisvq_layer* L = Ls[i];
+    FoldLayer<DV>& fl = f.layer[i];
+    fl.ws = ws[i];
+    fl.d = L->d;
+    fl.colnorm = L->colnorm;
+    for (int j = 0; j < DV * DV; ++j) fl.A[j] = L->A[j];
+    for (int j = 0; j < DV; ++j) fl.B[j] = L->B[j];
+  }
+  cudaLaunchConfig_t fc = {};
+  fc.gridDim = dim3(p.ks, mc, n);
+  fc.blockDim = dim3(kFoldThreads, 1, 1);
+  fc.dynamicSmemBytes = static_cast<size_t>(p.kt_per_cta) * kTileCols * 2;
+  fc.stream = s;
+  cudaLaunchAttribute fat[1] = {pdl_attr()};
+  fc.attrs = fat;
+  fc.numAttrs = 1;
+  return cudaLaunchKernelEx(&fc, fold_kernel<DV>, f) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+}
+
 // Fold and stream, the fold workspace of layer i at ws[i].
 unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
                                cudaStream_t s, uint8_t* const* ws) {
@@ -806,19 +866,15 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
   const unisvq_layer* L0 = Ls[0];
   if (!set_fold_attrs(L0->device)) return UNISVQ_ERR_CUDA;
   int nb = 0;
-  for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
+  bool d8 = false;
+  for (int i = 0; i < n; ++i) {
+    nb += Ls[i]->Np / kTileRows;
+    d8 = d8 || Ls[i]->d == 8;
+  }
   for (int m0 = 0; m0 < M; m0 += kMaxTokPerLaunch) {
     const int mc = M - m0 < kMaxTokPerLaunch ? M - m0 : kMaxTokPerLaunch;
     const DecodePlan p = plan_rows_split(nb, L0->KT, L0->num_sms, mc);
     if (p.ks > kMaxSplit) return UNISVQ_ERR_UNSUPPORTED;
-    FoldArgs f{};
-    f.x = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * L0->K;
-    f.M = mc;
-    f.K = L0->K;
-    f.KT = L0->KT;
-    f.kt_per_cta = p.kt_per_cta;
-    f.ncol = p.nt;
-    f.nlayers = n;
     SkArgs a{};
     a.M = mc;
     a.KT = L0->KT;
@@ -828,12 +884,6 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
     int rb0 = 0;
     for (int i = 0; i < n; ++i) {
       const unisvq_layer* L = Ls[i];
-      FoldLayer& fl = f.layer[i];
-      fl.ws = ws[i];
-      fl.d = L->d;
-      fl.colnorm = L->colnorm;
-      for (int j = 0; j < 64; ++j) fl.A[j] = L->A[j];
-      for (int j = 0; j < 8; ++j) fl.B[j] = L->B[j];
       SkLayer& l = a.layer[i];
       l.codes = L->codes;
       l.ws = ws[i];
@@ -842,16 +892,8 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
       l.rb0 = rb0;
       rb0 += L->Np / kTileRows;
     }
-    cudaLaunchConfig_t fc = {};
-    fc.gridDim = dim3(p.ks, mc, n);
-    fc.blockDim = dim3(kFoldThreads, 1, 1);
-    fc.dynamicSmemBytes = static_cast<size_t>(p.kt_per_cta) * kTileCols * 2;
-    fc.stream = s;
-    cudaLaunchAttribute fat[1] = {pdl_attr()};
-    fc.attrs = fat;
-    fc.numAttrs = 1;
-    if (cudaLaunchKernelEx(&fc, fold_kernel, f) != cudaSuccess) return UNISVQ_ERR_CUDA;
-    unisvq_status st;
+    unisvq_status st = d8 ? launch_fold<8>(Ls, n, x, m0, mc, p, s, ws) : launch_fold<4>(Ls, n, x, m0, mc, p, s, ws);
+    if (st != UNISVQ_OK) return st;
     if (p.nt == 16) st = p.geom == 1 ? launch_ncol<16, 1>(a, p, L0->device, s) : launch_ncol<16, 2>(a, p, L0->device, s);
     else if (p.nt == 32) st = p.geom == 1 ? launch_ncol<32, 1>(a, p, L0->device, s) : launch_ncol<32, 2>(a, p, L0->device, s);
     else st = launch_ncol<48, 2>(a, p, L0->device, s);

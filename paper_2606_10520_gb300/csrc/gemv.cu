@@ -42,21 +42,29 @@ constexpr int kXPad = 4;            // fp16 elements of padding per token row (b
 constexpr int kTokBytes = 272;      // pexp[32], cpart[32], reduction mbarrier
 constexpr size_t kSmemPerSm = 228 * 1024;
 constexpr size_t kSmemPerCtaReserved = 1024;
-constexpr size_t kStaticSmem = 64 * sizeof(float);   // sA8 of both kernels
-constexpr size_t kDynSmemMax = kSmemPerSm - kSmemPerCtaReserved - kStaticSmem;
+
+// Kernels are instantiated for DV, the largest vector length of the launch's
+// layers: DV = 4 (d in {1, 2, 4}) keeps A in registers and the parameter block
+// small; DV = 8 adds the 8 x 8 fold, with A staged in shared memory.
+template <int DV>
+constexpr size_t static_smem() { return DV == 8 ? 64 * sizeof(float) : 0; }
+template <int DV>
+constexpr size_t dyn_smem_max() { return kSmemPerSm - kSmemPerCtaReserved - static_smem<DV>(); }
 
 // One layer of a launch. A launch covers one layer, or several layers that
 // read the same x (same K): their row blocks are stacked along grid.y.
+template <int DV>
 struct GemvLayer {
   const uint8_t* codes;
   uint16_t* y;         // bf16 [M][N]
   int N, d;
   int rb0;             // first grid.y row block of this layer
   float colnorm;
-  float A[64];         // row-major d x d (d <= 8)
-  float B[8];
+  float A[DV * DV];    // row-major d x d (d <= DV)
+  float B[DV];
 };
 
+template <int DV>
 struct GemvArgs {
   const uint16_t* x;   // bf16 [M][K]
   int M, K, KT;
@@ -65,7 +73,7 @@ struct GemvArgs {
   int off_red, off_tok;
   int nlayers;
   int* err;
-  GemvLayer layer[kMaxGroup];
+  GemvLayer<DV> layer[kMaxGroup];
 };
 
 __device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
@@ -119,12 +127,13 @@ __device__ __noinline__ Vec8 fold_vec8(const float* sA8, Vec8 x) {
 // four-column groups j0 = 2ci mod 4 and j0 + 1, scaled by 2^(pe - 2j). For
 // d = 8 the eight columns are one vector and A comes from shared memory (sA8,
 // row-major 8 x 8); otherwise from the register copy A.
+template <int DV>
 __device__ __forceinline__ uint4 fold8(int ci, uint4 xv, int pe, int d, const float (&A)[16], const float* sA8) {
   const int j0 = (2 * ci) & 3;
   const float v0[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
   const float v1[4] = {bf16_lo(xv.z), bf16_hi(xv.z), bf16_lo(xv.w), bf16_hi(xv.w)};
   float o0[4], o1[4];
-  if (d == 8) {
+  if (DV == 8 && d == 8) {
     const Vec8 o = fold_vec8(sA8, Vec8{{v0[0], v0[1], v0[2], v0[3], v1[0], v1[1], v1[2], v1[3]}});
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
@@ -157,8 +166,8 @@ __device__ __forceinline__ uint4 load_x8(const uint16_t* row, int k, int kend, b
   return make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
 }
 
-template <int NT>
-__global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constant__ GemvArgs a) {
+template <int NT, int DV>
+__global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constant__ GemvArgs<DV> a) {
   extern __shared__ __align__(16) uint8_t smem[];
   const uint32_t sbase = smem_u32(smem);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -174,7 +183,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   const uint8_t* codes = nullptr;
   uint16_t* yout = nullptr;
   int N = 0, d = 1, rb = 0;
-  float colnorm = 0.f, Areg[16], Bcol[8];   // Bcol[e] = B[e mod d] for column e of an 8-column chunk
+  float colnorm = 0.f, Areg[16], Bq[DV];
 #pragma unroll
   for (int i = 0; i < kMaxGroup; ++i) {
     if (i == li) {
@@ -187,19 +196,24 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
 #pragma unroll
       for (int e = 0; e < 16; ++e) Areg[e] = a.layer[i].A[e];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) Bcol[e] = a.layer[i].B[e & (a.layer[i].d - 1)];
+      for (int e = 0; e < DV; ++e) Bq[e] = a.layer[i].B[e];
     }
   }
-  __shared__ float sA8[64];   // A for d = 8 (the fold reads it from here)
-  if (d == 8) {
-    if (tid < 64) {
-      float v = a.layer[0].A[tid];
+  float Bcol[8];   // B[e mod d] for column e of an 8-column chunk
 #pragma unroll
-      for (int i = 1; i < kMaxGroup; ++i)
-        if (i == li) v = a.layer[i].A[tid];
-      sA8[tid] = v;
+  for (int e = 0; e < 8; ++e) Bcol[e] = d == 1 ? Bq[0] : (d == 2 ? Bq[e & 1] : (DV == 4 || d == 4 ? Bq[e & 3] : Bq[e & (DV - 1)]));
+  __shared__ float sA8[DV == 8 ? 64 : 1];   // A for d = 8 (the fold reads it from here)
+  if constexpr (DV == 8) {
+    if (d == 8) {
+      if (tid < 64) {
+        float v = a.layer[0].A[tid];
+#pragma unroll
+        for (int i = 1; i < kMaxGroup; ++i)
+          if (i == li) v = a.layer[i].A[tid];
+        sA8[tid] = v;
+      }
+      __syncthreads();
     }
-    __syncthreads();
   }
   // Rows whose K-slice partial sums this CTA adds up (it "owns" them).
   const int rows_per = (kTileRows + KS - 1) / KS;
@@ -293,7 +307,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
         uint8_t* xrow = smem + tk * xrow_bytes;
         uint4 f[kXLoads];
 #pragma unroll
-        for (int j = 0; j < kXLoads; ++j) f[j] = fold8(lane + 32 * j, u[p][j], pe, d, Areg, sA8);
+        for (int j = 0; j < kXLoads; ++j) f[j] = fold8<DV>(lane + 32 * j, u[p][j], pe, d, Areg, sA8);
 #pragma unroll
         for (int j = 0; j < kXLoads; ++j) {
           const int ci = lane + 32 * j;
@@ -353,7 +367,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
           if (ci < nch) {
             const uint2 lo = *reinterpret_cast<const uint2*>(xrow + 16u * ci);
             const uint2 hi = *reinterpret_cast<const uint2*>(xrow + 16u * ci + 8);
-            u[j] = fold8(ci, make_uint4(lo.x, lo.y, hi.x, hi.y), pe, d, Areg, sA8);
+            u[j] = fold8<DV>(ci, make_uint4(lo.x, lo.y, hi.x, hi.y), pe, d, Areg, sA8);
           }
         }
 #pragma unroll
@@ -483,7 +497,8 @@ constexpr int kRMaxTok = 4;
 constexpr int kRDepth = 4;    // k-tiles of codes in flight per warp (2 x 16 bytes per lane each)
 constexpr int kRItems = 4;    // activation loads in flight per lane in the fold
 
-__global__ void __launch_bounds__(kGThreads, 2) gemv_rows_kernel(const __grid_constant__ GemvArgs a) {
+template <int DV>
+__global__ void __launch_bounds__(kGThreads, 2) gemv_rows_kernel(const __grid_constant__ GemvArgs<DV> a) {
   extern __shared__ __align__(16) uint8_t smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int M = a.M;
@@ -494,7 +509,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_rows_kernel(const __grid_co
   const uint8_t* codes = nullptr;
   uint16_t* yout = nullptr;
   int N = 0, d = 1, pr = 0;
-  float colnorm = 0.f, Areg[16], Bcol[8];   // Bcol[e] = B[e mod d] for column e of an 8-column chunk
+  float colnorm = 0.f, Areg[16], Bq[DV];
 #pragma unroll
   for (int i = 0; i < kMaxGroup; ++i) {
     if (i == li) {
@@ -507,19 +522,24 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_rows_kernel(const __grid_co
 #pragma unroll
       for (int e = 0; e < 16; ++e) Areg[e] = a.layer[i].A[e];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) Bcol[e] = a.layer[i].B[e & (a.layer[i].d - 1)];
+      for (int e = 0; e < DV; ++e) Bq[e] = a.layer[i].B[e];
     }
   }
-  __shared__ float sA8[64];   // A for d = 8 (the fold reads it from here)
-  if (d == 8) {
-    if (threadIdx.x < 64) {
-      float v = a.layer[0].A[threadIdx.x];
+  float Bcol[8];   // B[e mod d] for column e of an 8-column chunk
 #pragma unroll
-      for (int i = 1; i < kMaxGroup; ++i)
-        if (i == li) v = a.layer[i].A[threadIdx.x];
-      sA8[threadIdx.x] = v;
+  for (int e = 0; e < 8; ++e) Bcol[e] = d == 1 ? Bq[0] : (d == 2 ? Bq[e & 1] : (DV == 4 || d == 4 ? Bq[e & 3] : Bq[e & (DV - 1)]));
+  __shared__ float sA8[DV == 8 ? 64 : 1];   // A for d = 8 (the fold reads it from here)
+  if constexpr (DV == 8) {
+    if (d == 8) {
+      if (threadIdx.x < 64) {
+        float v = a.layer[0].A[threadIdx.x];
+#pragma unroll
+        for (int i = 1; i < kMaxGroup; ++i)
+          if (i == li) v = a.layer[i].A[threadIdx.x];
+        sA8[threadIdx.x] = v;
+      }
+      __syncthreads();
     }
-    __syncthreads();
   }
 
   const int kpw = a.kt_per_cta;
@@ -614,7 +634,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_rows_kernel(const __grid_co
           if (q == tk) pt = pe[q];
         const uint8_t* src = wreg + tk * wstride + 16u * ci;
         const uint2 lo = *reinterpret_cast<const uint2*>(src), hi = *reinterpret_cast<const uint2*>(src + 8);
-        f[r] = fold8(ci, make_uint4(lo.x, lo.y, hi.x, hi.y), pt, d, Areg, sA8);
+        f[r] = fold8<DV>(ci, make_uint4(lo.x, lo.y, hi.x, hi.y), pt, d, Areg, sA8);
       }
     }
 #pragma unroll
@@ -718,22 +738,36 @@ GemvShape gemv_shape(int M, int kt_per_cta, int ks, int nt) {
   return s;
 }
 
-template <int NT>
+// Copies a layer's affine map into a launch's parameter block.
+template <int DV>
+void set_affine(GemvLayer<DV>& g, const unisvq_layer* L) {
+  for (int e = 0; e < DV * DV; ++e) g.A[e] = L->A[e];
+  for (int e = 0; e < DV; ++e) g.B[e] = L->B[e];
+}
+
+// 8 if any layer of the launch has d = 8, else 4.
+int group_dv(const unisvq_layer* const* Ls, int n) {
+  for (int i = 0; i < n; ++i)
+    if (Ls[i]->d == 8) return 8;
+  return 4;
+}
+
+template <int NT, int DV>
 unisvq_status gemv_launch_nt(const unisvq_layer* const* Ls, int n, const DecodePlan& p, const void* x,
                              void* const* ys, int m0, int M, cudaStream_t s) {
   static bool attr_set[64] = {};
   const int dev = Ls[0]->device;
   if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
   if (!attr_set[dev]) {
-    if (cudaFuncSetAttribute(gemv_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(kDynSmemMax)) != cudaSuccess ||
-        cudaFuncSetAttribute(gemv_kernel<NT>, cudaFuncAttributePreferredSharedMemoryCarveout,
+    if (cudaFuncSetAttribute(gemv_kernel<NT, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(dyn_smem_max<DV>())) != cudaSuccess ||
+        cudaFuncSetAttribute(gemv_kernel<NT, DV>, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared) != cudaSuccess)
       return UNISVQ_ERR_CUDA;
     attr_set[dev] = true;
   }
   const GemvShape sh = gemv_shape(M, p.kt_per_cta, p.ks, NT);
-  GemvArgs a{};
+  GemvArgs<DV> a{};
   a.x = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * Ls[0]->K;
   a.M = M;
   a.K = Ls[0]->K;
@@ -747,15 +781,14 @@ unisvq_status gemv_launch_nt(const unisvq_layer* const* Ls, int n, const DecodeP
   int rb0 = 0;
   for (int i = 0; i < n; ++i) {
     const unisvq_layer* L = Ls[i];
-    GemvLayer& g = a.layer[i];
+    GemvLayer<DV>& g = a.layer[i];
     g.codes = L->codes;
     g.y = static_cast<uint16_t*>(ys[i]) + static_cast<size_t>(m0) * L->N;
     g.N = L->N;
     g.d = L->d;
     g.rb0 = rb0;
     g.colnorm = L->colnorm;
-    for (int e = 0; e < 64; ++e) g.A[e] = L->A[e];
-    for (int e = 0; e < 8; ++e) g.B[e] = L->B[e];
+    set_affine(g, L);
     rb0 += L->Np / kTileRows;
   }
 
@@ -773,17 +806,18 @@ unisvq_status gemv_launch_nt(const unisvq_layer* const* Ls, int n, const DecodeP
   attrs[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attrs;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, gemv_kernel<NT>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+  return cudaLaunchKernelEx(&cfg, gemv_kernel<NT, DV>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
 // Split K into ks <= 8 cluster CTAs for nb row blocks: the largest ks whose
 // grid fits one wave of resident CTAs (two per SM); if none does, the
-// smallest ks whose folded slice fits in shared memory.
-DecodePlan plan_rows(int nb, int KT, int num_sms, int M) {
+// smallest ks whose folded slice fits in shared memory. `sstat` is the
+// kernel's static shared memory (static_smem<DV>()).
+DecodePlan plan_rows(int nb, int KT, int num_sms, int M, size_t sstat) {
   DecodePlan p{};
   p.nt = M <= 8 ? 1 : (M <= 16 ? 2 : 4);
   p.nb = nb;
-  const size_t cap = kDynSmemMax;
+  const size_t cap = kSmemPerSm - kSmemPerCtaReserved - sstat;
   int best = 0, fallback = 0;
   for (int c = kMaxSplit; c >= 1; --c) {
     if (c > KT) continue;
@@ -793,7 +827,7 @@ DecodePlan plan_rows(int nb, int KT, int num_sms, int M) {
     const size_t smem = gemv_shape(M, kpc, ks, p.nt).smem;
     if (smem > cap) continue;
     fallback = ks;
-    const int per_sm = static_cast<int>(kSmemPerSm / (smem + kStaticSmem + kSmemPerCtaReserved)) < 2 ? 1 : 2;
+    const int per_sm = static_cast<int>(kSmemPerSm / (smem + sstat + kSmemPerCtaReserved)) < 2 ? 1 : 2;
     if (!best && nb * ks <= per_sm * num_sms) best = ks;
   }
   const int ks = best ? best : (fallback ? fallback : kMaxSplit);
@@ -816,20 +850,21 @@ size_t rows_smem(int M, int KT, int* off_red, int* xstride) {
   return offr + static_cast<size_t>(kGWarps) * 32 * 8 * 4;
 }
 
+template <int DV>
 unisvq_status rows_launch(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int m0, int M,
                           cudaStream_t s) {
   static bool attr_set[64] = {};
   const int dev = Ls[0]->device;
   if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
   if (!attr_set[dev]) {
-    if (cudaFuncSetAttribute(gemv_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(kDynSmemMax)) != cudaSuccess ||
-        cudaFuncSetAttribute(gemv_rows_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+    if (cudaFuncSetAttribute(gemv_rows_kernel<DV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(dyn_smem_max<DV>())) != cudaSuccess ||
+        cudaFuncSetAttribute(gemv_rows_kernel<DV>, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared) != cudaSuccess)
       return UNISVQ_ERR_CUDA;
     attr_set[dev] = true;
   }
-  GemvArgs a{};
+  GemvArgs<DV> a{};
   int off_red = 0, xstride = 0;
   const size_t smem = rows_smem(M, Ls[0]->KT, &off_red, &xstride);
   a.x = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * Ls[0]->K;
@@ -844,15 +879,14 @@ unisvq_status rows_launch(const unisvq_layer* const* Ls, int n, const void* x, v
   int pairs = 0;
   for (int i = 0; i < n; ++i) {
     const unisvq_layer* L = Ls[i];
-    GemvLayer& g = a.layer[i];
+    GemvLayer<DV>& g = a.layer[i];
     g.codes = L->codes;
     g.y = static_cast<uint16_t*>(ys[i]) + static_cast<size_t>(m0) * L->N;
     g.N = L->N;
     g.d = L->d;
     g.rb0 = pairs;
     g.colnorm = L->colnorm;
-    for (int e = 0; e < 64; ++e) g.A[e] = L->A[e];
-    for (int e = 0; e < 8; ++e) g.B[e] = L->B[e];
+    set_affine(g, L);
     pairs += L->Np / (2 * kUnitRows);
   }
   cudaLaunchConfig_t cfg = {};
@@ -865,31 +899,42 @@ unisvq_status rows_launch(const unisvq_layer* const* Ls, int n, const void* x, v
   attr.val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, gemv_rows_kernel, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+  return cudaLaunchKernelEx(&cfg, gemv_rows_kernel<DV>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
 }  // namespace
 
-DecodePlan plan_gemv(const unisvq_layer* L, int M) { return plan_rows(L->Np / kTileRows, L->KT, L->num_sms, M); }
+DecodePlan plan_gemv(const unisvq_layer* L, int M) {
+  return plan_rows(L->Np / kTileRows, L->KT, L->num_sms, M, L->d == 8 ? static_smem<8>() : static_smem<4>());
+}
 
 unisvq_status launch_gemv_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
                                 cudaStream_t s) {
   if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
   int nb = 0;
   for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
+  const bool d8 = group_dv(Ls, n) == 8;
+  const size_t sstat = d8 ? static_smem<8>() : static_smem<4>();
+  const size_t cap = kSmemPerSm - kSmemPerCtaReserved - sstat;
   for (int m0 = 0; m0 < M;) {
     // up to 32 tokens per launch; fewer when the folded slice of a long K
     // would not fit in shared memory
     int mc = M - m0 < kGMaxTok ? M - m0 : kGMaxTok;
-    DecodePlan p = plan_rows(nb, Ls[0]->KT, Ls[0]->num_sms, mc);
-    while (p.smem > kDynSmemMax && mc > 1) {
+    DecodePlan p = plan_rows(nb, Ls[0]->KT, Ls[0]->num_sms, mc, sstat);
+    while (p.smem > cap && mc > 1) {
       mc = (mc + 1) / 2;
-      p = plan_rows(nb, Ls[0]->KT, Ls[0]->num_sms, mc);
+      p = plan_rows(nb, Ls[0]->KT, Ls[0]->num_sms, mc, sstat);
     }
-    if (p.smem > kDynSmemMax) return UNISVQ_ERR_UNSUPPORTED;
-    const unisvq_status st = p.nt == 1   ? gemv_launch_nt<1>(Ls, n, p, x, ys, m0, mc, s)
-                             : p.nt == 2 ? gemv_launch_nt<2>(Ls, n, p, x, ys, m0, mc, s)
-                                         : gemv_launch_nt<4>(Ls, n, p, x, ys, m0, mc, s);
+    if (p.smem > cap) return UNISVQ_ERR_UNSUPPORTED;
+    unisvq_status st;
+    if (d8)
+      st = p.nt == 1   ? gemv_launch_nt<1, 8>(Ls, n, p, x, ys, m0, mc, s)
+           : p.nt == 2 ? gemv_launch_nt<2, 8>(Ls, n, p, x, ys, m0, mc, s)
+                       : gemv_launch_nt<4, 8>(Ls, n, p, x, ys, m0, mc, s);
+    else
+      st = p.nt == 1   ? gemv_launch_nt<1, 4>(Ls, n, p, x, ys, m0, mc, s)
+           : p.nt == 2 ? gemv_launch_nt<2, 4>(Ls, n, p, x, ys, m0, mc, s)
+                       : gemv_launch_nt<4, 4>(Ls, n, p, x, ys, m0, mc, s);
     if (st != UNISVQ_OK) return st;
     m0 += mc;
   }
@@ -900,17 +945,24 @@ unisvq_status launch_gemv(const unisvq_layer* L, const void* x, void* y, int M, 
   return launch_gemv_group(&L, 1, x, &y, M, s);
 }
 
-bool gemv_rows_supported(const unisvq_layer* L, int M) {
-  return M >= 1 && M <= kRMaxTok && rows_smem(M, L->KT, nullptr, nullptr) <= kSmemPerSm / 2 - kSmemPerCtaReserved - kStaticSmem;
+namespace {
+bool rows_fit(int M, int KT, bool d8) {
+  return M >= 1 && M <= kRMaxTok &&
+         rows_smem(M, KT, nullptr, nullptr) <= kSmemPerSm / 2 - kSmemPerCtaReserved -
+                                                   (d8 ? static_smem<8>() : static_smem<4>());
 }
+}  // namespace
+
+bool gemv_rows_supported(const unisvq_layer* L, int M) { return rows_fit(M, L->KT, L->d == 8); }
 
 unisvq_status launch_gemv_rows_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
                                      cudaStream_t s) {
   if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
+  const bool d8 = group_dv(Ls, n) == 8;
   for (int m0 = 0; m0 < M; m0 += kRMaxTok) {
     const int mc = M - m0 < kRMaxTok ? M - m0 : kRMaxTok;
-    if (!gemv_rows_supported(Ls[0], mc)) return UNISVQ_ERR_UNSUPPORTED;
-    const unisvq_status st = rows_launch(Ls, n, x, ys, m0, mc, s);
+    if (!rows_fit(mc, Ls[0]->KT, d8)) return UNISVQ_ERR_UNSUPPORTED;
+    const unisvq_status st = d8 ? rows_launch<8>(Ls, n, x, ys, m0, mc, s) : rows_launch<4>(Ls, n, x, ys, m0, mc, s);
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;
