@@ -21,12 +21,20 @@ Inputs are exactly widened to fp64 (bf16 activations, fp16 affine). Where the
 paper fixes no rounding, the oracle keeps everything exact in fp64 and rounds
 once at the very end (`dequant_f32`).
 
+The per-(row, group) functions (`dequant_grouped`, `linear_grouped`,
+`linear_grouped_moments`) restate Eq. (def:unisvq) with one (A, B) per output
+row and group of input columns; the paper itself uses one per matrix.
+
 Pins (tests/test_oracle_pins.py): exhaustive codebook enumeration with the
 orthogonal initial grid (mean 0, covariance I, App. A.1), the scalar
 quantisation special case (Eq. def:sq), an integer-matrix case checked against
 exact Python integers, the hand-worked example in tests/golden/, linearity in
 x, agreement of Eq. (col:dequant) with Eq. (def:unisvq), and the fold
-identity of Eq. (col:matmul). No function here is "parity unpinned".
+identity of Eq. (col:matmul); for the per-group functions, the hand-worked
+example in tests/golden/grouped_hand_worked.json, group-wise uniform scalar
+quantisation (A = s I), reduction to the per-matrix oracle when all groups
+share one map, and the exchange-of-sums identity. No function here is
+"parity unpinned".
 """
 from __future__ import annotations
 
@@ -131,6 +139,84 @@ def linear_folded(x: np.ndarray, codes: np.ndarray, A, B) -> np.ndarray:
     XA = (Xi @ as_f64(A)).reshape(M, K)          # the row vectors X_i A
     XB = (Xi @ as_f64(B)).sum(axis=1)            # sum_i X_i B, one scalar per token
     return XA @ codes.astype(np.float64).T + XB[:, None]
+
+
+def _check_grouped(codes: np.ndarray, A: np.ndarray, B: np.ndarray, group_cols: int):
+    N, K = codes.shape
+    d = A.shape[-1]
+    G = -(-K // group_cols)
+    if A.shape != (N, G, d, d) or B.shape != (N, G, d):
+        raise ValueError("A must be [N][G][d][d] and B [N][G][d], G = ceil(K / group_cols)")
+    if K % d or group_cols % d:
+        raise ValueError("K and group_cols must be multiples of d")
+    return N, K, d, G
+
+
+def dequant_grouped(codes: np.ndarray, A, B, group_cols: int = 128) -> np.ndarray:
+    """Dequantised weights [N][K] in fp64 with one affine map per (output row,
+    group of `group_cols` input columns).
+
+    Eq. (def:unisvq) applied to every vector, each with the (A, B) of its own
+    row n and column group g = k // group_cols (per-row, per-group granularity,
+    finer than the paper's one map per matrix). A is [N][G][d][d], B [N][G][d],
+    G = ceil(K / group_cols); group_cols is a multiple of d, so a vector never
+    straddles two groups: W_hat[n, k] = sum_c A[n, g, r, c] z[n, k - r + c]
+    + B[n, g, r] with r = k mod d.
+    """
+    A = as_f64(A)
+    B = as_f64(B)
+    N, K, d, G = _check_grouped(codes, A, B, group_cols)
+    Z = codes.reshape(N, K // d, d).astype(np.float64)
+    g_of_vec = (np.arange(K // d) * d) // group_cols          # group of each vector
+    W = np.einsum("nvrc,nvc->nvr", A[:, g_of_vec], Z) + B[:, g_of_vec]
+    return W.reshape(N, K)
+
+
+def linear_grouped(x: np.ndarray, codes: np.ndarray, A, B, group_cols: int = 128, row_chunk: int = 256):
+    """Layer output y = x W_hat^T and tolerance scale S = |x| |W_hat|^T for
+    per-(row, group) affine maps (`dequant_grouped`); Eq. (def:ptq_loss).
+    Returns (y, S), both float64 [M][N].
+    """
+    xf = bf16_bits_to_f64(x) if x.dtype == np.uint16 else as_f64(x)
+    A = np.asarray(A)
+    B = np.asarray(B)
+    M = xf.shape[0]
+    N = codes.shape[0]
+    y = np.empty((M, N))
+    S = np.empty((M, N))
+    ax = np.abs(xf)
+    for r0 in range(0, N, row_chunk):
+        r1 = min(N, r0 + row_chunk)
+        W = dequant_grouped(codes[r0:r1], A[r0:r1], B[r0:r1], group_cols)
+        y[:, r0:r1] = xf @ W.T
+        S[:, r0:r1] = ax @ np.abs(W).T
+    return y, S
+
+
+def linear_grouped_moments(x: np.ndarray, codes: np.ndarray, A, B, group_cols: int = 128) -> np.ndarray:
+    """The same output contracted before the affine map is applied: for row n
+    and group g, S_rc = sum_v x[v d + r] z[n, v d + c] over the group's
+    vectors v and X_r = sum_v x[v d + r]; then
+    y[n] = sum_g sum_{r,c} A[n, g, r, c] S_rc + sum_g sum_r B[n, g, r] X_r.
+
+    This is Eq. (def:unisvq) summed over a group with the order of the sums
+    exchanged (x_v . (A z_v + B) = sum_{r,c} A_rc x_vr z_vc + sum_r B_r x_vr),
+    the form in which the codes meet the activations before A does. fp64.
+    """
+    A = as_f64(A)
+    B = as_f64(B)
+    xf = bf16_bits_to_f64(x) if x.dtype == np.uint16 else as_f64(x)
+    N, K, d, G = _check_grouped(codes, A, B, group_cols)
+    M = xf.shape[0]
+    y = np.zeros((M, N))
+    for g in range(G):
+        k0, k1 = g * group_cols, min(K, (g + 1) * group_cols)
+        xg = xf[:, k0:k1].reshape(M, -1, d)                   # [M][V][r]
+        zg = codes[:, k0:k1].reshape(N, -1, d).astype(np.float64)   # [N][V][c]
+        Smom = np.einsum("mvr,nvc->mnrc", xg, zg)
+        X = xg.sum(axis=1)                                    # [M][r]
+        y += np.einsum("mnrc,nrc->mn", Smom, A[:, g]) + X @ B[:, g].T
+    return y
 
 
 def compare(y: np.ndarray, y_ref: np.ndarray, S: np.ndarray) -> dict:

@@ -62,6 +62,17 @@ def gen_affine(g: np.random.Generator, d: int, s_mean: float = 0.02, s_std: floa
     return A, B
 
 
+def gen_affine_grouped(g: np.random.Generator, N: int, G: int, d: int, s_mean: float = 0.02,
+                       s_std: float = 0.005, mix: float = 0.1):
+    """(A [N][G][d][d], B [N][G][d]) fp16: one independent draw of the
+    `gen_affine` distribution per (output row, column group)."""
+    s = np.abs(g.normal(s_mean, s_std, size=(N, G)))
+    Gm = g.standard_normal((N, G, d, d))
+    A = (s[:, :, None, None] * (np.eye(d) + mix * Gm)).astype(np.float16)
+    B = np.repeat((-1.5 * s)[:, :, None], d, axis=2).astype(np.float16)
+    return A, B
+
+
 def f32_to_bf16_bits(v: np.ndarray) -> np.ndarray:
     """Round fp32 values to bf16 (round to nearest even); returns uint16 bits."""
     v = np.ascontiguousarray(v, dtype=np.float32)
@@ -95,6 +106,17 @@ def layer_inputs(seed: int, config: int, layer: int, proj: int, N: int, K: int, 
     ga = rng(seed, config, layer, proj, 2)
     codes = gen_codes(gc, N, K)
     A, B = gen_affine(ga, d)
+    return codes, A, B
+
+
+def layer_inputs_grouped(seed: int, config: int, layer: int, proj: int, N: int, K: int, d: int,
+                         group_cols: int = 128):
+    """(codes, A, B) with one affine map per (output row, `group_cols` input
+    columns), for one projection of one layer of a synthetic config."""
+    gc = rng(seed, config, layer, proj, 1)
+    ga = rng(seed, config, layer, proj, 4)
+    codes = gen_codes(gc, N, K)
+    A, B = gen_affine_grouped(ga, N, -(-K // group_cols), d)
     return codes, A, B
 
 

@@ -289,3 +289,87 @@ def test_synth_bf16_rounding_matches_torch():
     ours = synth.f32_to_bf16_bits(v)
     ref = torch.from_numpy(v).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
     assert np.array_equal(ours, ref)
+
+
+# --------------------------------------------------------------------------
+# per-(row, group) affine maps
+# --------------------------------------------------------------------------
+
+GROUPED_GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "grouped_hand_worked.json")
+
+
+def test_grouped_golden_hand_worked():
+    """The hand-worked per-group example: W, y and S exactly."""
+    with open(GROUPED_GOLDEN) as f:
+        cases = json.load(f)["cases"]
+    for c in cases:
+        A = np.array(c["A"])
+        B = np.array(c["B"])
+        codes = np.array(c["codes"], dtype=np.uint8)
+        x = np.array(c["x"])
+        gc = c["group_cols"]
+        assert np.array_equal(oracle.dequant_grouped(codes, A, B, gc), np.array(c["W"])), c["name"]
+        y, S = oracle.linear_grouped(x, codes, A, B, gc)
+        assert np.array_equal(y, np.array(c["y"])), c["name"]
+        assert np.array_equal(S, np.array(c["S"])), c["name"]
+        assert np.array_equal(oracle.linear_grouped_moments(x, codes, A, B, gc), np.array(c["y"])), c["name"]
+
+
+@pytest.mark.parametrize("d", [1, 2, 4, 8])
+def test_grouped_scalar_case_is_groupwise_uniform_quantisation(d):
+    """A[n][g] = s[n][g] I, B[n][g] = b[n][g] 1: every weight is s z + b with
+    the scale and offset of its row and 128-column group -- group-wise uniform
+    2-bit dequantisation (per-row scale/offset broadcast along columns)."""
+    g = np.random.default_rng(40 + d)
+    N, K, gc = 5, 3 * 128 + 64, 128
+    G = -(-K // gc)
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    s = g.standard_normal((N, G))
+    b = g.standard_normal((N, G))
+    A = s[:, :, None, None] * np.eye(d)
+    B = np.repeat(b[:, :, None], d, axis=2)
+    s_col = np.repeat(s, gc, axis=1)[:, :K]
+    b_col = np.repeat(b, gc, axis=1)[:, :K]
+    expect = s_col * codes + b_col
+    assert np.array_equal(oracle.dequant_grouped(codes, A, B, gc), expect)
+
+
+@pytest.mark.parametrize("d", [1, 2, 4, 8])
+def test_grouped_with_one_map_everywhere_is_the_per_matrix_layer(d):
+    g = synth.rng(0, 98, d)
+    N, K = 7, 2 * 128 + 8 * d
+    codes = synth.gen_codes(g, N, K)
+    A1, B1 = synth.gen_affine(g, d)
+    G = -(-K // 128)
+    A = np.broadcast_to(A1, (N, G, d, d))
+    B = np.broadcast_to(B1, (N, G, d))
+    assert np.array_equal(oracle.dequant_grouped(codes, A, B), oracle.dequant(codes, A1, B1))
+
+
+@pytest.mark.parametrize("d", [1, 2, 4, 8])
+def test_grouped_moment_form_matches_direct_form(d):
+    """Exchanging the sums (codes meet the activations before A does) gives
+    the same output, with a different non-symmetric A per row and group."""
+    g = np.random.default_rng(70 + d)
+    N, M, K = 6, 3, 2 * 128 + 16 * d
+    G = -(-K // 128)
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    A = g.standard_normal((N, G, d, d))
+    B = g.standard_normal((N, G, d))
+    x = g.standard_normal((M, K))
+    y, S = oracle.linear_grouped(x, codes, A, B)
+    ym = oracle.linear_grouped_moments(x, codes, A, B)
+    assert np.allclose(ym, y, rtol=0, atol=1e-12 * S.max())
+
+
+def test_grouped_linearity_and_row_chunks():
+    g = np.random.default_rng(5)
+    N, K, d = 11, 256, 2
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    A = g.standard_normal((N, 2, d, d))
+    B = g.standard_normal((N, 2, d))
+    x1 = g.standard_normal((2, K))
+    x2 = g.standard_normal((2, K))
+    f = lambda x, rc=256: oracle.linear_grouped(x, codes, A, B, 128, rc)[0]
+    assert np.allclose(f(0.5 * x1 + 2 * x2), 0.5 * f(x1) + 2 * f(x2), rtol=1e-12, atol=1e-12)
+    assert np.allclose(f(x1, 3), f(x1), rtol=1e-13, atol=1e-13)
