@@ -60,7 +60,9 @@ def algo_bytes(N, K, M, d=2):
     return N * K // 4 + (d * d + d) * 2 + 2 * M * K + 2 * M * N
 
 
-KERNEL_NAMES = {1: "decode", 2: "prefill_kernel", 3: "gemv_kernel", 4: "decode_kernel", 5: "gemv_rows_kernel"}
+KERNEL_NAMES = {1: "decode", 2: "prefill_kernel", 3: "gemv_kernel", 4: "decode_kernel", 5: "gemv_rows_kernel",
+                6: "gemv_grouped_kernel"}
+GROUPED_LAYERS = 16   # 16 x 69.6 MB of codes + per-group maps: larger than L2
 # Sources whose change invalidates a committed ncu traffic figure, per kernel.
 KERNEL_SOURCES = {
     "gemv_kernel": ("paper_2606_10520_gb300/csrc/gemv.cu", "paper_2606_10520_gb300/csrc/common.cuh",
@@ -278,7 +280,7 @@ def run_ours(args, rank, world, local_rank):
         print(json.dumps({"prefill": run_prefill(torch, binding, peaks, args, side)}), flush=True)
         return
     if args.only == "decode":
-        args.no_e2e = args.no_cpu = args.no_prefill = True
+        args.no_e2e = args.no_cpu = args.no_prefill = args.no_grouped = True
     shapes = synth.LLAMA2_7B
     stack = build_stack(binding, shapes, args.layers, 1)
 
@@ -461,6 +463,11 @@ def run_ours(args, rank, world, local_rank):
                "how": "per call: pinned-host x -> device copy, the library call, device -> pinned-host y "
                       "of every projection; the whole sweep replayed from CUDA graphs"}
 
+    # ---- per-(row, 128-column group) affine layers ------------------------
+    grouped = None
+    if not args.no_grouped:
+        grouped = run_grouped(torch, binding, peaks, args, side)
+
     # ---- prefill (tcgen05 GEMM), Llama-3-8B-shaped set at M = 2048 -------
     prefill = None
     if not args.no_prefill:
@@ -490,9 +497,75 @@ def run_ours(args, rank, world, local_rank):
         "clocks": clocks,
         "cpu_baseline": cpu,
         "prefill": prefill,
+        "per_group_affine": grouped,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
+
+
+def run_grouped(torch, binding, peaks, args, stream):
+    """The decode sweep on Llama-2-7B-shaped layers with one fp16 affine map
+    per (output row, 128-column group): the per-group GEMV (gemv_grouped_kernel),
+    algorithmic bytes counting the maps (N * K/128 * 12 bytes at d = 2)."""
+    shapes = synth.LLAMA2_7B
+    base = []
+    for pi, (_, N, K) in enumerate(shapes):
+        codes, A, B = synth.layer_inputs_grouped(0, 1, 0, pi, N, K, 2)
+        base.append(binding.UniSVQLinear(codes, A, B, group_cols=128))
+    stack = [base] + [[b.clone() for b in base] for _ in range(GROUPED_LAYERS - 1)]
+    xs = {}
+    ys = {}
+    for M in M_SWEEP:
+        for pi, (_, N, K) in enumerate(shapes):
+            if (M, K) not in xs:
+                xb = synth.activations(0, 1, 100 + M, M, K)
+                xs[(M, K)] = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).cuda()
+            ys[(M, pi)] = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    graphs, sweep_bytes, launches = [], [], 0
+    for M in M_SWEEP:
+        def one_pass(M=M):
+            sp = torch.cuda.current_stream().cuda_stream
+            for layer in stack:
+                for grp in GROUPS_7B:
+                    K = shapes[grp[0]][2]
+                    st = binding.linear_group_ptr([layer[i] for i in grp], xs[(M, K)].data_ptr(),
+                                                  [ys[(M, i)].data_ptr() for i in grp], M, sp)
+                    if st != 0:
+                        raise RuntimeError(f"unisvq call failed: {binding.status_string(st)}")
+        with torch.cuda.stream(stream):
+            one_pass()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            one_pass()
+        graphs.append(g)
+        nbytes = 0
+        for grp in GROUPS_7B:
+            info = binding.query_group([base[i] for i in grp], M)
+            assert info["kernel"] == binding.KERNEL_GROUPED
+            nbytes += info["algo_bytes"] * GROUPED_LAYERS
+            launches += info["launches"] * GROUPED_LAYERS
+        sweep_bytes.append(nbytes)
+    st = binding.sync_status(stream)
+    if st != 0:
+        raise RuntimeError(f"device status {binding.status_string(st)}")
+    steps = max(5, args.steps // 4)
+    t = time_graphs(torch, graphs, steps, args.warmup, stream)
+    per_m = []
+    for M, g, nb in zip(M_SWEEP, graphs, sweep_bytes):
+        tm = time_graphs(torch, [g], steps, 2, stream)
+        per_m.append({"M": M, "GB/s": round(nb * steps / tm / 1e9, 1),
+                      "us_per_layer": round(tm / steps / GROUPED_LAYERS * 1e6, 3)})
+    for layer in stack:
+        for b in layer:
+            b.close()
+    gbs = sum(sweep_bytes) * steps / t / 1e9
+    return {"workload": f"Llama-2-7B-shaped projection set x {GROUPED_LAYERS} layers, decode sweep M in "
+                        f"{list(M_SWEEP)}, 2-bit codes d=2, one fp16 affine per output row per 128-column group",
+            "GB/s": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"], "sweep": per_m,
+            "kernel": "gemv_grouped_kernel", "launches_per_step": launches,
+            "bytes": "codes N*K/4 + maps N*ceil(K/128)*12 + x + y per call",
+            "timing": "CUDA graphs of the layer stack per M, CUDA events on the capture stream"}
 
 
 def run_prefill(torch, binding, peaks, args, stream):
@@ -576,6 +649,8 @@ def main():
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-grouped", action="store_true",
+                    help="skip the per-(row, 128-column group) affine sweep")
     ap.add_argument("--ungrouped", action="store_true",
                     help="one unisvq_linear call per projection instead of grouped calls for q/k/v and gate/up")
     ap.add_argument("--cpu-budget", type=float, default=12.0)

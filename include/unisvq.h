@@ -49,7 +49,8 @@ enum {
   UNISVQ_KERNEL_PREFILL = 2,  /* tcgen05 GEMM, exact bf16 codeword tiles in smem       */
   UNISVQ_KERNEL_GEMV = 3,     /* fold + register-operand tensor-core GEMV, M <= 32/launch */
   UNISVQ_KERNEL_SKINNY = 4,   /* fold + tcgen05 with codes as 8-bit TMEM operand, M <= 16/launch */
-  UNISVQ_KERNEL_GEMV_ROWS = 5 /* GEMV with whole-K row slices per CTA (no cluster), M <= 4/launch */
+  UNISVQ_KERNEL_GEMV_ROWS = 5, /* GEMV with whole-K row slices per CTA (no cluster), M <= 4/launch */
+  UNISVQ_KERNEL_GROUPED = 6    /* per-(row, group) affine GEMV (layers of unisvq_pack_grouped), M <= 32/d per launch */
 };
 
 /*
@@ -87,7 +88,8 @@ typedef struct {
   int split_k;            /* CTAs cooperating along K (decode kernel)           */
   int grid_ctas;          /* CTAs launched                                      */
   long long code_bytes;   /* packed code bytes resident on the device           */
-  long long meta_bytes;   /* affine parameters: (d*d + d) * 2 bytes (fp16)      */
+  long long meta_bytes;   /* affine parameters: (d*d + d) * 2 bytes (fp16), times
+                             N * ceil(K/128) for a unisvq_pack_grouped layer    */
   long long algo_bytes;   /* N*K/4 + meta + 2*M*K (x) + 2*M*N (y)               */
   double flops;           /* 2*M*N*K                                            */
   int launches;           /* kernel launches the call makes                     */
@@ -118,6 +120,34 @@ typedef struct {
  */
 unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
                           int N, int K, int d, void* stream, unisvq_handle* out);
+
+/*
+ * Pack a layer whose affine map varies per output row and per group of
+ * `group_cols` input columns: W_hat[n, k] = sum_c A[n][g][r][c] z[n, k - r + c]
+ * + B[n][g][r], g = k / group_cols, r = k mod d (Eq. def:unisvq applied with
+ * the map of the vector's row and column group). This granularity is finer
+ * than the paper's (one map per matrix, Sec. 4.2: use unisvq_pack for that);
+ * it cannot be folded onto the activations, so these layers run their own
+ * GEMV (UNISVQ_KERNEL_GROUPED), which forms the moments
+ * S_rc = sum_v x[v d + r] z[v d + c] of each group on the tensor cores and
+ * applies the row's A and B to them.
+ *   codes      : host, [N][K] uint8, each 0..3
+ *   A_f16      : host, [N][G][d][d] fp16 bits, G = ceil(K / group_cols)
+ *   B_f16      : host, [N][G][d] fp16 bits
+ *   d          : 1, 2, 4 or 8; K % d == 0
+ *   group_cols : 128 (one packed k-tile); other values UNSUPPORTED
+ * The code array uses the packed layout above with the columns of every
+ * 128-column group permuted (coordinate c of the group's vectors gathered
+ * into 16-column runs); the maps are stored as fp16 [Np/128][Kp/128][128]
+ * [d*d + d] (A row-major, then B), zero for padding rows.
+ * unisvq_linear, _group (all layers grouped, same d), _force (AUTO, DECODE or
+ * GROUPED; other kernels UNSUPPORTED), _noalloc, _query and
+ * unisvq_dequant_debug accept the handle. The host buffers are copied before
+ * return. Errors: INVALID_ARG (null pointer, bad shape, code > 3, non-finite
+ * A/B), UNSUPPORTED (d or group_cols), OOM, CUDA.
+ */
+unisvq_status unisvq_pack_grouped(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
+                                  int N, int K, int d, int group_cols, void* stream, unisvq_handle* out);
 
 /*
  * y = x W_hat^T (Eq. def:ptq_loss with W_hat of Eq. col:dequant).

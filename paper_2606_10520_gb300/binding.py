@@ -14,7 +14,7 @@ import numpy as np
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libunisvq.so")
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM, ERR_TIMEOUT = range(6)
-KERNEL_AUTO, KERNEL_DECODE, KERNEL_PREFILL, KERNEL_GEMV, KERNEL_SKINNY, KERNEL_GEMV_ROWS = 0, 1, 2, 3, 4, 5
+KERNEL_AUTO, KERNEL_DECODE, KERNEL_PREFILL, KERNEL_GEMV, KERNEL_SKINNY, KERNEL_GEMV_ROWS, KERNEL_GROUPED = range(7)
 
 # Every function include/unisvq.h declares.
 EXPORTS = [
@@ -22,6 +22,7 @@ EXPORTS = [
     "unisvq_query", "unisvq_sync_status", "unisvq_destroy", "unisvq_clone",
     "unisvq_status_string", "unisvq_packed_code_bytes", "unisvq_pack_host", "unisvq_version",
     "unisvq_linear_group", "unisvq_linear_group_force", "unisvq_linear_noalloc", "unisvq_query_group",
+    "unisvq_pack_grouped",
 ]
 MAX_GROUP = 4
 
@@ -53,6 +54,7 @@ def load():
     lib = ctypes.CDLL(LIB_PATH)
     vp, i, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
     lib.unisvq_pack.argtypes = [vp, vp, vp, i, i, i, vp, ctypes.POINTER(vp)]
+    lib.unisvq_pack_grouped.argtypes = [vp, vp, vp, i, i, i, i, vp, ctypes.POINTER(vp)]
     lib.unisvq_linear.argtypes = [vp, vp, vp, i, vp]
     lib.unisvq_linear_force.argtypes = [vp, i, vp, vp, i, vp]
     lib.unisvq_linear_group.argtypes = [vp, i, vp, vp, i, vp]
@@ -116,7 +118,10 @@ def sync_status(stream=None) -> int:
 class UniSVQLinear:
     """One packed UniSVQ linear layer resident on the current CUDA device."""
 
-    def __init__(self, codes: np.ndarray, A, B, stream=None, _handle=None):
+    def __init__(self, codes: np.ndarray, A, B, stream=None, _handle=None, group_cols: int | None = None):
+        """One (A [d][d], B [d]) for the matrix (unisvq_pack), or, with
+        `group_cols`, one per (row, group of columns): A [N][G][d][d],
+        B [N][G][d] (unisvq_pack_grouped)."""
         lib = load()
         if _handle is not None:
             self._h = _handle
@@ -124,11 +129,19 @@ class UniSVQLinear:
             codes = np.ascontiguousarray(codes, dtype=np.uint8)
             A16 = _f16_bits(A)
             B16 = _f16_bits(B)
-            d = A16.shape[0]
+            d = A16.shape[-1]
             N, K = codes.shape
             h = ctypes.c_void_p()
-            _check(lib.unisvq_pack(codes.ctypes.data, A16.ctypes.data, B16.ctypes.data, N, K, d,
-                                   _stream_ptr(stream), ctypes.byref(h)), "unisvq_pack")
+            if group_cols is None:
+                _check(lib.unisvq_pack(codes.ctypes.data, A16.ctypes.data, B16.ctypes.data, N, K, d,
+                                       _stream_ptr(stream), ctypes.byref(h)), "unisvq_pack")
+            else:
+                G = -(-K // group_cols)
+                if A16.shape != (N, G, d, d) or B16.shape != (N, G, d):
+                    raise ValueError("per-group A must be [N][G][d][d] and B [N][G][d]")
+                _check(lib.unisvq_pack_grouped(codes.ctypes.data, A16.ctypes.data, B16.ctypes.data, N, K, d,
+                                               group_cols, _stream_ptr(stream), ctypes.byref(h)),
+                       "unisvq_pack_grouped")
             self._h = h
         info = self.query(1)
         self.N, self.K, self.d = info["N"], info["K"], info["d"]

@@ -4,6 +4,8 @@
 // the same extraction helper the layer kernels use (layout.h), rebuilds the index
 // z0 | z1 << 2 | ... of every d-vector and reads the fp32 codeword
 // RN_fp32(A z + B) of Eq. (def:unisvq) from the handle's codebook.
+#include <cuda_fp16.h>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -48,9 +50,44 @@ __global__ void __launch_bounds__(256) dequant_kernel(const uint8_t* __restrict_
   }
 }
 
+// Per-(row, group) layers: one thread per weight. Column k of row n is
+// coordinate r = k mod d of vector v of group g = k / 128; coordinate c of
+// that vector sits at chunk q = c (8/d) + v / 16, quarter t = (v mod 16) / 4,
+// byte b = e(v mod 4) of the permuted tile (pack_codes_grouped_host), and
+// RN_fp32(sum_c A[n][g][r][c] z_c + B[n][g][r]) is formed exactly in fp64.
+__global__ void __launch_bounds__(256) dequant_grouped_kernel(const uint8_t* __restrict__ codes,
+                                                              const uint16_t* __restrict__ meta, float* W, int N,
+                                                              int K, int KT, int d) {
+  const size_t id = static_cast<size_t>(blockIdx.x) * 256 + threadIdx.x;
+  if (id >= static_cast<size_t>(N) * K) return;
+  const int n = static_cast<int>(id / K), k = static_cast<int>(id % K);
+  const int g = k / kTileCols, col = k % kTileCols;
+  const int v = col / d, r = col % d, nq = 8 / d;
+  const int rb = n / kTileRows, rr = n % kTileRows;
+  const uint8_t* tile = codes + (static_cast<size_t>(rb) * KT + g) * kTileBytes;
+  const int md = d * d + d;
+  const uint16_t* rec = meta + ((static_cast<size_t>(rb) * KT + g) * kTileRows + rr) * md;
+  const int q = v / 16, t = (v % 16) / 4, e = v % 4;
+  const int b = (e >> 1) | ((e & 1) << 1);
+  double w = static_cast<double>(__half2float(__ushort_as_half(rec[d * d + r])));
+  for (int c = 0; c < d; ++c) {
+    const int qc = c * nq + q;
+    const uint32_t word = *reinterpret_cast<const uint32_t*>(tile + tile_word_offset(rr, qc >> 2, t));
+    const uint32_t z = (word >> (8 * b + 2 * (qc & 3))) & 3u;
+    w += static_cast<double>(__half2float(__ushort_as_half(rec[r * d + c]))) * static_cast<double>(z);
+  }
+  W[id] = static_cast<float>(w);
+}
+
 }  // namespace
 
 unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s) {
+  if (L->grouped) {
+    const size_t total = static_cast<size_t>(L->N) * L->K;
+    dequant_grouped_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, s>>>(L->codes, L->meta, W, L->N,
+                                                                                      L->K, L->KT, L->d);
+    return cudaGetLastError() == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+  }
   const int nchunks = (L->Np / kTileRows) * L->KT * 256;
   dequant_kernel<<<(nchunks + 255) / 256, 256, 0, s>>>(L->codes, L->lut32, W, L->N, L->K, L->KT, L->d,
                                                        nchunks);

@@ -24,6 +24,12 @@ struct unisvq_layer {
   float colnorm;           // max_c sum_r |A[r][c]|: |x A|_inf <= |x|_inf * colnorm
   uint8_t* fold_ws;        // device, decode fold workspace (fold_workspace_bytes(KT))
   uint16_t A16[64], B16[8];
+  // Per-(row, 128-column group) affine maps (unisvq_pack_grouped): the codes
+  // are packed with pack_codes_grouped_host and the maps live in `meta`;
+  // A, B, lut32, tlut and fold_ws are unused (zero / null).
+  int grouped;
+  uint16_t* meta;          // device, fp16 [Np/128][KT][128][d*d + d]
+  size_t meta_bytes;
 };
 
 namespace unisvq {
@@ -75,8 +81,21 @@ unisvq_status launch_prefill(const unisvq_layer* L, const void* x, void* y, int 
 
 unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s);
 
+// Per-(row, group) affine layers (gemv_grouped.cu): every M, at most 32 / d
+// tokens per launch; all layers of one call must be grouped with the same d.
+unisvq_status launch_grouped_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                                   cudaStream_t s);
+// Plan of the first launch for nb row blocks (the layers of one call) and M
+// tokens; *tokens_per_launch receives the tokens each launch takes (0: none fits).
+DecodePlan plan_grouped(const unisvq_layer* L, int nb, int M, int* tokens_per_launch);
+
 // Host packer (pack.cpp).
 void pack_codes_host(const uint8_t* codes, int N, int K, uint8_t* packed);
+// Same layout with the columns of every 128-column group permuted by
+// grouped_column (per-group layers), and their fp16 metadata.
+int grouped_column(int d, int h, int t, int s, int b);
+void pack_codes_grouped_host(const uint8_t* codes, int N, int K, int d, uint8_t* packed);
+void pack_meta_grouped_host(const uint16_t* A_f16, const uint16_t* B_f16, int N, int K, int d, uint16_t* meta);
 // fp64 -> bf16 round-to-nearest-even (single rounding).
 uint16_t f64_to_bf16_rne(double v);
 double f16_bits_to_f64(uint16_t h);

@@ -211,6 +211,73 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
   return UNISVQ_OK;
 }
 
+unisvq_status unisvq_pack_grouped(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
+                                  int N, int K, int d, int group_cols, void* stream, unisvq_handle* out) {
+  if (!out) return UNISVQ_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!codes || !A_f16 || !B_f16) return UNISVQ_ERR_INVALID_ARG;
+  if (d != 1 && d != 2 && d != 4 && d != 8) return UNISVQ_ERR_UNSUPPORTED;
+  if (group_cols != kTileCols) return UNISVQ_ERR_UNSUPPORTED;
+  if (N <= 0 || K <= 0 || K % d != 0) return UNISVQ_ERR_INVALID_ARG;
+  if (static_cast<long long>(round_up(N, kRowPad)) * round_up(K, kColPad) >= (1ll << 40))
+    return UNISVQ_ERR_UNSUPPORTED;
+  const size_t total = static_cast<size_t>(N) * K;
+  const int G = (K + group_cols - 1) / group_cols;
+  const size_t nA = static_cast<size_t>(N) * G * d * d, nB = static_cast<size_t>(N) * G * d;
+  int bad = 0;
+#pragma omp parallel for reduction(| : bad) schedule(static)
+  for (long long i = 0; i < static_cast<long long>(total); ++i) bad |= codes[i] > 3;
+  // fp16 exponent field all ones: inf or NaN
+#pragma omp parallel for reduction(| : bad) schedule(static)
+  for (long long i = 0; i < static_cast<long long>(nA); ++i) bad |= (A_f16[i] & 0x7C00u) == 0x7C00u;
+#pragma omp parallel for reduction(| : bad) schedule(static)
+  for (long long i = 0; i < static_cast<long long>(nB); ++i) bad |= (B_f16[i] & 0x7C00u) == 0x7C00u;
+  if (bad) return UNISVQ_ERR_INVALID_ARG;
+
+  unisvq_layer* L = new (std::nothrow) unisvq_layer();
+  if (!L) return UNISVQ_ERR_OOM;
+  L->N = N;
+  L->K = K;
+  L->d = d;
+  L->Np = round_up(N, kRowPad);
+  L->Kp = round_up(K, kColPad);
+  L->KT = L->Kp / kTileCols;
+  L->grouped = 1;
+  if (cudaGetDevice(&L->device) != cudaSuccess ||
+      cudaDeviceGetAttribute(&L->num_sms, cudaDevAttrMultiProcessorCount, L->device) != cudaSuccess) {
+    delete L;
+    return UNISVQ_ERR_CUDA;
+  }
+  L->code_bytes = unisvq_packed_code_bytes(N, K);
+  L->meta_bytes = static_cast<size_t>(L->Np / kTileRows) * L->KT * kTileRows * (d * d + d) * sizeof(uint16_t);
+  std::vector<uint8_t> packed;
+  std::vector<uint16_t> meta;
+  try {
+    packed.resize(L->code_bytes);
+    meta.resize(L->meta_bytes / sizeof(uint16_t));
+  } catch (...) {
+    delete L;
+    return UNISVQ_ERR_OOM;
+  }
+  pack_codes_grouped_host(codes, N, K, d, packed.data());
+  pack_meta_grouped_host(A_f16, B_f16, N, K, d, meta.data());
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMalloc(&L->codes, L->code_bytes);
+  if (e == cudaSuccess) e = cudaMalloc(&L->meta, L->meta_bytes);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(L->codes, packed.data(), L->code_bytes, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(L->meta, meta.data(), L->meta_bytes, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess && !device_error_word()) e = cudaErrorUnknown;
+  if (e != cudaSuccess) {
+    cudaFree(L->codes);
+    cudaFree(L->meta);
+    delete L;
+    return cuda_status(e);
+  }
+  *out = L;
+  return UNISVQ_OK;
+}
+
 unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
   if (!h || !out) return UNISVQ_ERR_INVALID_ARG;
   *out = nullptr;
@@ -220,24 +287,33 @@ unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
   L->lut32 = nullptr;
   L->tlut = nullptr;
   L->fold_ws = nullptr;
+  L->meta = nullptr;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const size_t n32 = static_cast<size_t>(h->lut_entries) * h->d * sizeof(float);
-  const size_t n16 = static_cast<size_t>(h->tlut_words) * sizeof(uint32_t);
-  const size_t ws_bytes = fold_workspace_bytes(h->KT);
-  cudaError_t e = cudaMalloc(&L->codes, h->code_bytes);
-  if (e == cudaSuccess) e = cudaMalloc(&L->lut32, n32);
-  if (e == cudaSuccess) e = cudaMalloc(&L->tlut, n16);
-  if (e == cudaSuccess) e = cudaMalloc(&L->fold_ws, ws_bytes);
-  if (e == cudaSuccess) e = cudaMemsetAsync(L->fold_ws, 0, ws_bytes, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(L->codes, h->codes, h->code_bytes, cudaMemcpyDeviceToDevice, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(L->lut32, h->lut32, n32, cudaMemcpyDeviceToDevice, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(L->tlut, h->tlut, n16, cudaMemcpyDeviceToDevice, s);
+  // A device buffer of the source handle copied into a new allocation (none if the source has none).
+  auto copy = [&](void** dst, const void* src, size_t bytes) -> cudaError_t {
+    if (!src || !bytes) return cudaSuccess;
+    cudaError_t e = cudaMalloc(dst, bytes);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(*dst, src, bytes, cudaMemcpyDeviceToDevice, s);
+    return e;
+  };
+  cudaError_t e = copy(reinterpret_cast<void**>(&L->codes), h->codes, h->code_bytes);
+  if (e == cudaSuccess && !h->grouped) {
+    e = copy(reinterpret_cast<void**>(&L->lut32), h->lut32,
+             static_cast<size_t>(h->lut_entries) * h->d * sizeof(float));
+    if (e == cudaSuccess)
+      e = copy(reinterpret_cast<void**>(&L->tlut), h->tlut, static_cast<size_t>(h->tlut_words) * sizeof(uint32_t));
+    const size_t ws_bytes = fold_workspace_bytes(h->KT);
+    if (e == cudaSuccess) e = cudaMalloc(&L->fold_ws, ws_bytes);
+    if (e == cudaSuccess) e = cudaMemsetAsync(L->fold_ws, 0, ws_bytes, s);
+  }
+  if (e == cudaSuccess && h->grouped) e = copy(reinterpret_cast<void**>(&L->meta), h->meta, h->meta_bytes);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) {
     cudaFree(L->codes);
     cudaFree(L->lut32);
     cudaFree(L->tlut);
     cudaFree(L->fold_ws);
+    cudaFree(L->meta);
     delete L;
     return cuda_status(e);
   }
@@ -251,9 +327,11 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
   cudaError_t e2 = cudaFree(h->lut32);
   cudaError_t e3 = cudaFree(h->tlut);
   cudaError_t e4 = cudaFree(h->fold_ws);
+  cudaError_t e5 = cudaFree(h->meta);
   delete h;
-  return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess && e4 == cudaSuccess) ? UNISVQ_OK
-                                                                                             : UNISVQ_ERR_CUDA;
+  return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess && e4 == cudaSuccess && e5 == cudaSuccess)
+             ? UNISVQ_OK
+             : UNISVQ_ERR_CUDA;
 }
 
 // Decode kernel for M <= 64 tokens over `weights` = sum of N*K of the layers
@@ -292,6 +370,14 @@ unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, vo
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
   if (dev != h->device) return UNISVQ_ERR_INVALID_ARG;
+  if (h->grouped) {
+    if (kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GROUPED)
+      return kernel >= 0 && kernel <= UNISVQ_KERNEL_GROUPED ? UNISVQ_ERR_UNSUPPORTED : UNISVQ_ERR_INVALID_ARG;
+    const unisvq_layer* Ls[1] = {h};
+    void* ys[1] = {y};
+    return launch_grouped_group(Ls, 1, x, ys, M, static_cast<cudaStream_t>(stream));
+  }
+  if (kernel == UNISVQ_KERNEL_GROUPED) return UNISVQ_ERR_UNSUPPORTED;
   if (kernel == UNISVQ_KERNEL_AUTO) kernel = auto_kernel(h, M);
   if (kernel == UNISVQ_KERNEL_DECODE) kernel = decode_kernel_for(static_cast<long long>(h->N) * h->K, h->Np / kTileRows, M);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -320,6 +406,11 @@ unisvq_status unisvq_linear_noalloc(unisvq_handle h, const void* x, void* y, int
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
   if (dev != h->device) return UNISVQ_ERR_INVALID_ARG;
+  if (h->grouped) {   // the per-group GEMV has no workspace
+    const unisvq_layer* Ls[1] = {h};
+    void* ys[1] = {y};
+    return launch_grouped_group(Ls, 1, x, ys, M, static_cast<cudaStream_t>(stream));
+  }
   return launch_skinny_static(h, x, y, M, static_cast<cudaStream_t>(stream));
 }
 
@@ -339,6 +430,20 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
   if (dev != hs[0]->device) return UNISVQ_ERR_INVALID_ARG;
+  int ngrouped = 0;
+  for (int i = 0; i < n; ++i) ngrouped += hs[i]->grouped ? 1 : 0;
+  if (ngrouped) {   // all layers per-group with one d, run by the per-group GEMV
+    if (ngrouped != n) return UNISVQ_ERR_UNSUPPORTED;
+    if (kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GROUPED)
+      return UNISVQ_ERR_UNSUPPORTED;
+    const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
+    for (int i = 0; i < n; ++i) {
+      if (hs[i]->d != hs[0]->d) return UNISVQ_ERR_UNSUPPORTED;
+      Ls[i] = hs[i];
+    }
+    return launch_grouped_group(Ls, n, x, ys, M, static_cast<cudaStream_t>(stream));
+  }
+  if (kernel == UNISVQ_KERNEL_GROUPED) return UNISVQ_ERR_UNSUPPORTED;
   long long weights = 0;
   int nb = 0;
   for (int i = 0; i < n; ++i) {
@@ -376,12 +481,27 @@ unisvq_status unisvq_dequant_debug(unisvq_handle h, float* W, void* stream) {
   return launch_dequant(h, W, static_cast<cudaStream_t>(stream));
 }
 
+// Algorithmic metadata bytes: one fp16 (A, B) per matrix, or per (row, group)
+// of 128 columns for a per-group layer (padding excluded).
+static long long meta_bytes_of(const unisvq_layer* h) {
+  const long long per = static_cast<long long>(h->d * h->d + h->d) * 2;
+  return h->grouped ? per * h->N * ((h->K + kTileCols - 1) / kTileCols) : per;
+}
+
 // Launch geometry of `kernel` for the n layers of one call (query helpers).
 static void describe_launch(const unisvq_layer* const* Ls, int n, int kernel, int M, unisvq_info* info) {
   const unisvq_layer* h = Ls[0];
   const int m = M > 0 ? M : 1;
   info->kernel = kernel;
-  if (kernel == UNISVQ_KERNEL_GEMV_ROWS) {
+  if (kernel == UNISVQ_KERNEL_GROUPED) {
+    int nb = 0;
+    for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
+    int per = 0;
+    const DecodePlan p = plan_grouped(h, nb, m, &per);
+    info->split_k = p.ks;
+    info->launches = per > 0 ? (m + per - 1) / per : 0;
+    info->grid_ctas = p.ks * nb * info->launches;
+  } else if (kernel == UNISVQ_KERNEL_GEMV_ROWS) {
     info->split_k = 1;
     info->grid_ctas = 0;
     for (int i = 0; i < n; ++i) info->grid_ctas += Ls[i]->Np / 32;
@@ -418,12 +538,12 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
   info->Np = h->Np;
   info->Kp = h->Kp;
   info->code_bytes = static_cast<long long>(h->code_bytes);
-  info->meta_bytes = static_cast<long long>(h->d * h->d + h->d) * 2;
+  info->meta_bytes = meta_bytes_of(h);
   info->algo_bytes = static_cast<long long>(h->N) * h->K / 4 + info->meta_bytes +
                      2ll * M * h->K + 2ll * M * h->N;
   info->flops = 2.0 * M * static_cast<double>(h->N) * h->K;
   const unisvq_layer* Ls[1] = {h};
-  describe_launch(Ls, 1, auto_kernel(h, M > 0 ? M : 1), M, info);
+  describe_launch(Ls, 1, h->grouped ? UNISVQ_KERNEL_GROUPED : auto_kernel(h, M > 0 ? M : 1), M, info);
   return UNISVQ_OK;
 }
 
@@ -439,7 +559,7 @@ unisvq_status unisvq_query_group(const unisvq_handle* hs, int n, int M, unisvq_i
     info->N += h->N;
     info->Np += h->Np;
     info->code_bytes += static_cast<long long>(h->code_bytes);
-    info->meta_bytes += static_cast<long long>(h->d * h->d + h->d) * 2;
+    info->meta_bytes += meta_bytes_of(h);
     info->algo_bytes += static_cast<long long>(h->N) * h->K / 4 + 2ll * M * h->N;
     info->flops += 2.0 * M * static_cast<double>(h->N) * h->K;
     weights += static_cast<long long>(h->N) * h->K;
@@ -450,8 +570,9 @@ unisvq_status unisvq_query_group(const unisvq_handle* hs, int n, int M, unisvq_i
   info->d = hs[0]->d;
   info->algo_bytes += info->meta_bytes + 2ll * M * hs[0]->K;   // x is read once per call
   const int m = M > 0 ? M : 1;
-  const int kernel =
-      m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL : decode_kernel_for(weights, nb, m);
+  const int kernel = hs[0]->grouped ? UNISVQ_KERNEL_GROUPED
+                     : m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL
+                                                             : decode_kernel_for(weights, nb, m);
   const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
   for (int i = 0; i < n; ++i) Ls[i] = hs[i];
   describe_launch(Ls, n, kernel, M, info);

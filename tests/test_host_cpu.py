@@ -129,3 +129,32 @@ def test_linear_rejects_bad_arguments(lib):
 
 def test_version(lib):
     assert lib.unisvq_version() >= 100
+
+
+def _pack_grouped_status(lib, codes, A, B, N, K, d, gc):
+    h = ctypes.c_void_p()
+    return lib.unisvq_pack_grouped(codes.ctypes.data if codes is not None else None,
+                                   A.ctypes.data if A is not None else None,
+                                   B.ctypes.data if B is not None else None, N, K, d, gc, None, ctypes.byref(h))
+
+
+def test_pack_grouped_rejects_bad_arguments_before_touching_the_gpu(lib):
+    from paper_2606_10520_gb300 import binding
+    N, K, d = 4, 256, 2
+    G = K // 128
+    codes = np.zeros((N, K), dtype=np.uint8)
+    A = np.zeros((N, G, d, d), dtype=np.float16).view(np.uint16)
+    B = np.zeros((N, G, d), dtype=np.float16).view(np.uint16)
+    assert _pack_grouped_status(lib, None, A, B, N, K, d, 128) == binding.ERR_INVALID_ARG
+    assert _pack_grouped_status(lib, codes, A, B, N, K, 3, 128) == binding.ERR_UNSUPPORTED
+    assert _pack_grouped_status(lib, codes, A, B, N, K, d, 64) == binding.ERR_UNSUPPORTED
+    assert _pack_grouped_status(lib, codes, A, B, N, 255, d, 128) == binding.ERR_INVALID_ARG   # K % d
+    bad = codes.copy()
+    bad[2, 100] = 7
+    assert _pack_grouped_status(lib, bad, A, B, N, K, d, 128) == binding.ERR_INVALID_ARG
+    Ainf = A.copy()
+    Ainf[3, 1, 1, 0] = np.array([np.inf], dtype=np.float16).view(np.uint16)[0]
+    assert _pack_grouped_status(lib, codes, Ainf, B, N, K, d, 128) == binding.ERR_INVALID_ARG
+    Bnan = B.copy()
+    Bnan[0, 0, 1] = np.array([np.nan], dtype=np.float16).view(np.uint16)[0]
+    assert _pack_grouped_status(lib, codes, A, Bnan, N, K, d, 128) == binding.ERR_INVALID_ARG
