@@ -21,6 +21,11 @@ Inputs are exactly widened to fp64 (bf16 activations, fp16 affine). Where the
 paper fixes no rounding, the oracle keeps everything exact in fp64 and rounds
 once at the very end (`dequant_f32`).
 
+The RHT functions (`hadamard`, `rht_weight`, `rht_input`, `rht_output`,
+`linear_rht`) restate Eq. (def:hadamard): the weights are rotated before
+quantisation, so at inference the activations are rotated on the way in and
+the outputs on the way out.
+
 The per-(row, group) functions (`dequant_grouped`, `linear_grouped`,
 `linear_grouped_moments`) restate Eq. (def:unisvq) with one (A, B) per output
 row and group of input columns; the paper itself uses one per matrix.
@@ -33,8 +38,10 @@ x, agreement of Eq. (col:dequant) with Eq. (def:unisvq), and the fold
 identity of Eq. (col:matmul); for the per-group functions, the hand-worked
 example in tests/golden/grouped_hand_worked.json, group-wise uniform scalar
 quantisation (A = s I), reduction to the per-matrix oracle when all groups
-share one map, and the exchange-of-sums identity. No function here is
-"parity unpinned".
+share one map, and the exchange-of-sums identity; for the RHT functions,
+H H^T = n I for every order built, Sylvester's matrix against SciPy's, and the
+undo identity: the RHT layer applied to W_hat = R(W) returns x W^T. No
+function here is "parity unpinned".
 """
 from __future__ import annotations
 
@@ -217,6 +224,110 @@ def linear_grouped_moments(x: np.ndarray, codes: np.ndarray, A, B, group_cols: i
         X = xg.sum(axis=1)                                    # [M][r]
         y += np.einsum("mnrc,nrc->mn", Smom, A[:, g]) + X @ B[:, g].T
     return y
+
+
+# ---------------------------------------------------------------------------
+# Randomized Hadamard transform around the layer, Eq. (def:hadamard), Sec. 3.2.1
+# ---------------------------------------------------------------------------
+
+def _quadratic_character(q: int) -> np.ndarray:
+    """chi(a) for a in 0..q-1, q prime: 0 at 0, +1 on quadratic residues, -1 otherwise."""
+    chi = -np.ones(q, dtype=np.int64)
+    chi[0] = 0
+    chi[(np.arange(1, q) ** 2) % q] = 1
+    return chi
+
+
+def paley_hadamard(m: int) -> np.ndarray:
+    """A +-1 Hadamard matrix of order m in {12, 20, 28} (Paley's constructions).
+
+    Order q + 1 with q = 11, 19 (q = 3 mod 4, prime): with the Jacobsthal matrix
+    Q[i][j] = chi(j - i), H = I + [[0, 1^T], [-1, Q]].
+    Order 2(q + 1) with q = 13 (q = 1 mod 4, prime): with the symmetric
+    conference matrix C = [[0, 1^T], [1, Q]], H = [[C + I, C - I], [C - I, -C - I]].
+    """
+    if m in (12, 20):
+        q = m - 1
+        chi = _quadratic_character(q)
+        Q = chi[(np.arange(q)[None, :] - np.arange(q)[:, None]) % q]
+        S = np.zeros((m, m), dtype=np.int64)
+        S[0, 1:] = 1
+        S[1:, 0] = -1
+        S[1:, 1:] = Q
+        return np.eye(m, dtype=np.int64) + S
+    if m == 28:
+        q = 13
+        chi = _quadratic_character(q)
+        Q = chi[(np.arange(q)[None, :] - np.arange(q)[:, None]) % q]
+        C = np.zeros((q + 1, q + 1), dtype=np.int64)
+        C[0, 1:] = 1
+        C[1:, 0] = 1
+        C[1:, 1:] = Q
+        I = np.eye(q + 1, dtype=np.int64)
+        return np.block([[C + I, C - I], [C - I, -C - I]])
+    raise ValueError("Paley order must be 12, 20 or 28")
+
+
+def hadamard_factor(n: int):
+    """(2^a, m) with n = 2^a m and m in {1, 12, 20, 28} (the largest such m), or None."""
+    for m in (28, 20, 12, 1):
+        if n % m == 0:
+            p = n // m
+            if p & (p - 1) == 0:
+                return p, m
+    return None
+
+
+def hadamard(n: int) -> np.ndarray:
+    """+-1 Hadamard matrix of order n = 2^a m: Sylvester's H_{2^a} (H_1 = [1],
+    H_{2k} = [[H_k, H_k], [H_k, -H_k]]) Kronecker H_m (Paley, m > 1), so entry
+    [(p, q), (p', q')] at index p m + q is H_{2^a}[p][p'] H_m[q][q']."""
+    f = hadamard_factor(n)
+    if f is None:
+        raise ValueError(f"no Hadamard matrix of order {n} is built (n = 2^a m, m in 1, 12, 20, 28)")
+    p, m = f
+    H = np.ones((1, 1), dtype=np.int64)
+    while H.shape[0] < p:
+        H = np.block([[H, H], [H, -H]])
+    return H if m == 1 else np.kron(H, paley_hadamard(m))
+
+
+def rht_weight(W: np.ndarray, s_U, s_V) -> np.ndarray:
+    """Eq. (def:hadamard): R(W) = U S_U W S_V V with U = H_N / sqrt(N), V = H_K / sqrt(K)
+    (orthogonal) and S_U, S_V the diagonal +-1 matrices of the sign vectors. fp64."""
+    W = as_f64(W)
+    N, K = W.shape
+    U = hadamard(N) / np.sqrt(N)
+    V = hadamard(K) / np.sqrt(K)
+    return U @ (as_f64(s_U)[:, None] * W * as_f64(s_V)[None, :]) @ V
+
+
+def rht_input(x: np.ndarray, s_V) -> np.ndarray:
+    """The activations the quantised R(W) multiplies: x S_V V (row vectors). fp64."""
+    xf = bf16_bits_to_f64(x) if x.dtype == np.uint16 else as_f64(x)
+    K = xf.shape[1]
+    return (xf * as_f64(s_V)[None, :]) @ (hadamard(K) / np.sqrt(K))
+
+
+def rht_output(yt: np.ndarray, s_U) -> np.ndarray:
+    """The layer output from that of R(W): yt U S_U (row vectors). fp64."""
+    yt = as_f64(yt)
+    N = yt.shape[1]
+    return (yt @ (hadamard(N) / np.sqrt(N))) * as_f64(s_U)[None, :]
+
+
+def linear_rht(x: np.ndarray, codes: np.ndarray, A, B, s_U, s_V, row_chunk: int = 4096):
+    """y = x W^T for W = S_U U^T W_hat V^T S_V, the weight whose RHT (Eq.
+    def:hadamard) was quantised to W_hat: y = ((x S_V V) W_hat^T) U S_U.
+
+    Returns (y, S) with S = S_t |U|: S_t = |x S_V V| |W_hat|^T bounds the error
+    of the inner layer element by element, and the output transform mixes those
+    bounds with weights |U| = 1 / sqrt(N).
+    """
+    xt = rht_input(x, s_V)
+    yt, St = linear(xt, codes, A, B, row_chunk)
+    N = codes.shape[0]
+    return rht_output(yt, s_U), St @ (np.abs(hadamard(N)) / np.sqrt(N))
 
 
 def compare(y: np.ndarray, y_ref: np.ndarray, S: np.ndarray) -> dict:

@@ -373,3 +373,65 @@ def test_grouped_linearity_and_row_chunks():
     f = lambda x, rc=256: oracle.linear_grouped(x, codes, A, B, 128, rc)[0]
     assert np.allclose(f(0.5 * x1 + 2 * x2), 0.5 * f(x1) + 2 * f(x2), rtol=1e-12, atol=1e-12)
     assert np.allclose(f(x1, 3), f(x1), rtol=1e-13, atol=1e-13)
+
+
+# --------------------------------------------------------------------------
+# randomized Hadamard transform, Eq. (def:hadamard)
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n", [1, 2, 8, 12, 20, 28, 64, 96, 112, 160, 448, 1024])
+def test_hadamard_is_orthogonal_pm1(n):
+    H = oracle.hadamard(n)
+    assert H.shape == (n, n) and set(np.unique(H)) <= {-1, 1}
+    assert np.array_equal(H @ H.T, n * np.eye(n, dtype=np.int64))
+
+
+def test_sylvester_matches_scipy():
+    scipy_linalg = pytest.importorskip("scipy.linalg")
+    for n in (1, 2, 4, 64, 512):
+        assert np.array_equal(oracle.hadamard(n), scipy_linalg.hadamard(n))
+
+
+def test_hadamard_factor_of_model_widths():
+    assert oracle.hadamard_factor(4096) == (4096, 1)
+    assert oracle.hadamard_factor(14336) == (512, 28)
+    assert oracle.hadamard_factor(28672) == (1024, 28)
+    assert oracle.hadamard_factor(11008) is None        # 64 * 172: no order-172 matrix is built
+    with pytest.raises(ValueError):
+        oracle.hadamard(11008)
+
+
+@pytest.mark.parametrize("N,K", [(24, 64), (56, 40), (16, 112)])
+def test_rht_layer_undoes_the_weight_rotation(N, K):
+    """Eq. (def:hadamard): if W_hat is exactly R(W) = U S_U W S_V V, the layer
+    with the inverse transform around it returns x W^T. Checked with a dense W
+    expressed through d = 1 codes and A = 1 (so W_hat is an integer matrix and
+    R^-1(W_hat) is the W whose product we know)."""
+    g = np.random.default_rng(N * K)
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    A = np.ones((1, 1))
+    B = np.zeros(1)
+    s_U = g.choice([-1.0, 1.0], size=N)
+    s_V = g.choice([-1.0, 1.0], size=K)
+    W_hat = codes.astype(np.float64)
+    # W with R(W) = W_hat: W = S_U U^T W_hat V^T S_V
+    U = oracle.hadamard(N) / np.sqrt(N)
+    V = oracle.hadamard(K) / np.sqrt(K)
+    W = s_U[:, None] * (U.T @ W_hat @ V.T) * s_V[None, :]
+    assert np.allclose(oracle.rht_weight(W, s_U, s_V), W_hat, atol=1e-12)
+    x = g.standard_normal((3, K))
+    y, S = oracle.linear_rht(x, codes, A, B, s_U, s_V)
+    assert np.allclose(y, x @ W.T, rtol=0, atol=1e-11 * np.abs(x).sum())
+    assert np.all(S >= 0)
+
+
+def test_rht_input_output_are_inverse_rotations():
+    g = np.random.default_rng(9)
+    K = 448
+    s = g.choice([-1.0, 1.0], size=K)
+    x = g.standard_normal((2, K))
+    xt = oracle.rht_input(x, s)
+    assert np.allclose(np.linalg.norm(xt, axis=1), np.linalg.norm(x, axis=1), rtol=1e-13)
+    # rht_output applies U then S; with U = V its transpose undoes rht_input
+    V = oracle.hadamard(K) / np.sqrt(K)
+    assert np.allclose((xt @ V.T) * s, x, atol=1e-12)
