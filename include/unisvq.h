@@ -213,6 +213,41 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
  */
 unisvq_status unisvq_linear_noalloc(unisvq_handle h, const void* x, void* y, int M, void* stream);
 
+/*
+ * Inverse randomized Hadamard transform around the layer (Eq. def:hadamard,
+ * Sec. 3.2.1). The weights were rotated before quantisation, R(W) =
+ * U S_U W S_V V, with U = H_N / sqrt(N), V = H_K / sqrt(K) and S_U, S_V
+ * diagonal +-1; W_hat quantises R(W). After this call every unisvq_linear*
+ * on the handle returns y = x W^T for W = S_U U^T W_hat V^T S_V, computed as
+ *   x_t = (x S_V) V,   y_t = x_t W_hat^T,   y = (y_t U) S_U
+ * (row vectors): a rotation kernel on the way in, the layer's kernel, a
+ * rotation kernel on the way out, per chunk of max_tokens tokens.
+ * H_n is Sylvester's H_{2^a} Kronecker a Paley matrix H_m for n = 2^a m,
+ * m in {1, 12, 20, 28} (entry [(p,q),(p',q')] = H_{2^a}[p][p'] H_m[q][q'],
+ * index p m + q; H_12 and H_20 from Paley's first construction with q = 11
+ * and 19, H_28 from the second with q = 13); n <= 58112 (n floats in shared memory).
+ *   sign_in  : host, K bytes, 1 = -1 (the diagonal of S_V), 0 = +1
+ *   sign_out : host, N bytes (S_U)
+ *   max_tokens : rows of the rotated-activation buffer the handle allocates
+ *                here (bf16, max_tokens x K); longer calls run in chunks
+ * Both sign pointers NULL removes the transform (and its buffers). Calls on
+ * the handle must be stream-ordered (they share the buffer). Grouped calls
+ * with such handles run one layer at a time (each layer rotates x with its
+ * own S_V). Errors: INVALID_ARG (null handle, one sign pointer null, a sign
+ * byte > 1, max_tokens < 1), UNSUPPORTED (K or N not of the form above),
+ * OOM, CUDA.
+ */
+unisvq_status unisvq_set_rht(unisvq_handle h, const uint8_t* sign_in, const uint8_t* sign_out, int max_tokens,
+                             void* stream);
+
+/* The rotation by itself, on M rows of n bf16 values (device x, y; x == y
+ * allowed, otherwise no overlap): signs_first = 1 gives y = (x S) H_n /
+ * sqrt(n), signs_first = 0 gives y = ((x H_n) / sqrt(n)) S, S the diagonal
+ * of `signs` (device, n bytes, 1 = -1; NULL = identity). fp32 inside, bf16
+ * rounding once at the end. Errors: INVALID_ARG, UNSUPPORTED (n), CUDA. */
+unisvq_status unisvq_hadamard(const void* x, void* y, int M, int n, const uint8_t* signs, int signs_first,
+                              void* stream);
+
 /* Test hook: writes W_hat as fp32 [N][K] row-major to device memory W (each
  * entry RN_fp32 of the exact A z + B), unpacking the device layout with the
  * same code-extraction helpers the layer kernels use. */

@@ -22,7 +22,7 @@ EXPORTS = [
     "unisvq_query", "unisvq_sync_status", "unisvq_destroy", "unisvq_clone",
     "unisvq_status_string", "unisvq_packed_code_bytes", "unisvq_pack_host", "unisvq_version",
     "unisvq_linear_group", "unisvq_linear_group_force", "unisvq_linear_noalloc", "unisvq_query_group",
-    "unisvq_pack_grouped",
+    "unisvq_pack_grouped", "unisvq_set_rht", "unisvq_hadamard",
 ]
 MAX_GROUP = 4
 
@@ -55,6 +55,8 @@ def load():
     vp, i, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
     lib.unisvq_pack.argtypes = [vp, vp, vp, i, i, i, vp, ctypes.POINTER(vp)]
     lib.unisvq_pack_grouped.argtypes = [vp, vp, vp, i, i, i, i, vp, ctypes.POINTER(vp)]
+    lib.unisvq_set_rht.argtypes = [vp, vp, vp, i, vp]
+    lib.unisvq_hadamard.argtypes = [vp, vp, i, i, vp, i, vp]
     lib.unisvq_linear.argtypes = [vp, vp, vp, i, vp]
     lib.unisvq_linear_force.argtypes = [vp, i, vp, vp, i, vp]
     lib.unisvq_linear_group.argtypes = [vp, i, vp, vp, i, vp]
@@ -109,6 +111,20 @@ def _f16_bits(a) -> np.ndarray:
     if a.dtype == np.uint16:
         return np.ascontiguousarray(a)
     return np.ascontiguousarray(a.astype(np.float16)).view(np.uint16)
+
+
+def _sign_bytes(s) -> np.ndarray:
+    """+-1 values (or 0/1 bytes) -> uint8 with 1 = -1."""
+    a = np.asarray(s)
+    if a.dtype == np.uint8:
+        return np.ascontiguousarray(a)
+    return np.ascontiguousarray((a < 0).astype(np.uint8))
+
+
+def hadamard_ptr(x_ptr: int, y_ptr: int, M: int, n: int, signs_ptr: int, signs_first: int, stream_ptr: int) -> int:
+    """Raw-pointer unisvq_hadamard; returns the status."""
+    return load().unisvq_hadamard(ctypes.c_void_p(x_ptr), ctypes.c_void_p(y_ptr), int(M), int(n),
+                                  ctypes.c_void_p(signs_ptr or None), int(signs_first), ctypes.c_void_p(stream_ptr))
 
 
 def sync_status(stream=None) -> int:
@@ -186,6 +202,18 @@ class UniSVQLinear:
         _check(load().unisvq_dequant_debug(self._h, ctypes.c_void_p(W.data_ptr()), _stream_ptr(stream)),
                "unisvq_dequant_debug")
         return W
+
+    def set_rht(self, s_in, s_out, max_tokens: int = 64, stream=None):
+        """Rotate inputs by (S_V, V) and outputs by (U, S_U) around the layer
+        (unisvq_set_rht). s_in [K], s_out [N]: +-1 values or 0/1 bytes (1 = -1);
+        both None removes the transform."""
+        if s_in is None and s_out is None:
+            _check(load().unisvq_set_rht(self._h, None, None, 0, _stream_ptr(stream)), "unisvq_set_rht")
+            return
+        si = _sign_bytes(s_in)
+        so = _sign_bytes(s_out)
+        _check(load().unisvq_set_rht(self._h, si.ctypes.data, so.ctypes.data, int(max_tokens), _stream_ptr(stream)),
+               "unisvq_set_rht")
 
     def query(self, M: int) -> dict:
         info = Info()

@@ -30,6 +30,13 @@ struct unisvq_layer {
   int grouped;
   uint16_t* meta;          // device, fp16 [Np/128][KT][128][d*d + d]
   size_t meta_bytes;
+  // Inverse randomized Hadamard transform around the layer (unisvq_set_rht):
+  // device signs [K] (S_V) then [N] (S_U), 1 = -1, and a bf16 [rht_tokens][K]
+  // buffer for the rotated activations.
+  int rht;
+  uint8_t* rht_signs;
+  uint16_t* rht_x;
+  int rht_tokens;
 };
 
 namespace unisvq {
@@ -80,6 +87,14 @@ PrefillPlan plan_prefill(const unisvq_layer* L, int M);
 unisvq_status launch_prefill(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
 
 unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s);
+
+// Randomized Hadamard transform of M rows of n bf16 values (rht.cu):
+// signs_first = 1: out = (s x) H / sqrt(n); 0: out = s ((x H) / sqrt(n)).
+// n = 2^a m, m in {1, 12, 20, 28}; in and out may be the same rows.
+bool rht_factor(int n, int* p2, int* m);
+size_t rht_smem_bytes(int n);
+unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_stride, int M, int n,
+                         const uint8_t* signs, int signs_first, cudaStream_t s);
 
 // Per-(row, group) affine layers (gemv_grouped.cu): every M, at most 32 / d
 // tokens per launch; all layers of one call must be grouped with the same d.

@@ -1,0 +1,247 @@
+// Randomized Hadamard transform of activation rows (Eq. def:hadamard, Sec. 3.2.1).
+//
+// The weights were rotated before quantisation, R(W) = U S_U W S_V V, so the
+// layer computes y = ((x S_V V) W_hat^T) U S_U: the rows of x are rotated on
+// the way in (signs, then V) and the rows of the output on the way out (U,
+// then signs). U and V are normalised Hadamard matrices H_n / sqrt(n) of order
+// n = 2^a m: Sylvester's H_{2^a} Kronecker a Paley matrix H_m, m in
+// {1, 12, 20, 28}; entry [(p, q), (p', q')] (index p m + q) is
+// H_{2^a}[p][p'] H_m[q][q'].
+//
+// One CTA transforms one row in shared memory (fp32): the row-vector product
+// with H_m inside every block of m consecutive entries (registers, signs of
+// H_m as per-column bit masks), then the Sylvester butterflies across blocks in
+// radix-8 passes (three stages per pass in registers, one barrier per pass),
+// then the scale 1/sqrt(n) and, on the way out, the signs.
+#include <cmath>
+#include <vector>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace unisvq {
+namespace {
+
+constexpr int kRThreads = 512;
+constexpr int kMaxPaley = 28;
+
+struct RhtArgs {
+  const uint16_t* in;       // bf16 [M][in_stride]
+  uint16_t* out;            // bf16 [M][out_stride] (may equal in)
+  const uint8_t* signs;     // [n], 1 = negate; null = all +1
+  int n, p2, m;             // n = p2 * m
+  int log2p;
+  int in_stride, out_stride;
+  int signs_first;          // 1: x -> (s x) H; 0: x -> (x H) s
+  float scale;              // 1 / sqrt(n)
+  uint32_t hm_neg[kMaxPaley];   // bit q of column q': H_m[q][q'] = -1
+};
+
+__device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float(static_cast<uint32_t>(b) << 16); }
+
+// Row vector times H_m for one block of M_ consecutive entries, in place.
+template <int M_>
+__device__ __forceinline__ void paley_block(float* blk, const uint32_t (&neg)[kMaxPaley]) {
+  float v[M_];
+#pragma unroll
+  for (int q = 0; q < M_; ++q) v[q] = blk[q];
+#pragma unroll
+  for (int c = 0; c < M_; ++c) {
+    const uint32_t mask = neg[c];
+    float acc = 0.f;
+#pragma unroll
+    for (int q = 0; q < M_; ++q) acc += ((mask >> q) & 1u) ? -v[q] : v[q];
+    blk[c] = acc;
+  }
+}
+
+// Sylvester stages s0 .. s0 + R - 1 (butterfly distances 2^s0 .. 2^(s0+R-1)
+// blocks) for every column of the p2 x m view, R stages per pass in registers.
+template <int R>
+__device__ __forceinline__ void sylvester_pass(float* buf, int p2, int m, int s0) {
+  constexpr int G = 1 << R;
+  const int h = 1 << s0;
+  const int groups = (p2 >> R) * m;
+  for (int gi = threadIdx.x; gi < groups; gi += kRThreads) {
+    const int col = gi % m, rest = gi / m;
+    const int lo = (rest & (h - 1)) | ((rest >> s0) << (s0 + R));   // R zero bits inserted at s0
+    float v[G];
+#pragma unroll
+    for (int j = 0; j < G; ++j) v[j] = buf[(lo + j * h) * m + col];
+#pragma unroll
+    for (int st = 0; st < R; ++st) {
+      const int d = 1 << st;
+#pragma unroll
+      for (int j = 0; j < G; ++j)
+        if (!(j & d)) {
+          const float a = v[j], b = v[j + d];
+          v[j] = a + b;
+          v[j + d] = a - b;
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < G; ++j) buf[(lo + j * h) * m + col] = v[j];
+  }
+}
+
+__global__ void __launch_bounds__(kRThreads) rht_kernel(const __grid_constant__ RhtArgs a) {
+  extern __shared__ __align__(16) float buf[];
+  const int row = blockIdx.x;
+  const int n = a.n;
+  pdl_launch_dependents();
+  pdl_wait();   // the row may be the previous kernel's output
+  const uint16_t* src = a.in + static_cast<size_t>(row) * a.in_stride;
+  for (int i = threadIdx.x; i < n; i += kRThreads) {
+    float v = bf16_to_f32(src[i]);
+    if (a.signs_first && a.signs && a.signs[i]) v = -v;
+    buf[i] = v;
+  }
+  __syncthreads();
+  if (a.m > 1) {
+    uint32_t neg[kMaxPaley];
+#pragma unroll
+    for (int c = 0; c < kMaxPaley; ++c) neg[c] = a.hm_neg[c];
+    for (int p = threadIdx.x; p < a.p2; p += kRThreads) {
+      float* blk = buf + p * a.m;
+      if (a.m == 12) paley_block<12>(blk, neg);
+      else if (a.m == 20) paley_block<20>(blk, neg);
+      else paley_block<28>(blk, neg);
+    }
+    __syncthreads();
+  }
+  for (int s0 = 0; s0 < a.log2p;) {
+    const int r = min(3, a.log2p - s0);
+    if (r == 3) sylvester_pass<3>(buf, a.p2, a.m, s0);
+    else if (r == 2) sylvester_pass<2>(buf, a.p2, a.m, s0);
+    else sylvester_pass<1>(buf, a.p2, a.m, s0);
+    s0 += r;
+    __syncthreads();
+  }
+  uint16_t* dst = a.out + static_cast<size_t>(row) * a.out_stride;
+  for (int i = threadIdx.x; i < n; i += kRThreads) {
+    float v = buf[i] * a.scale;
+    if (!a.signs_first && a.signs && a.signs[i]) v = -v;
+    dst[i] = f32_to_bf16_rn(v);
+  }
+}
+
+// chi(v) mod q for prime q: +1 on nonzero squares, -1 on non-squares, 0 at 0.
+int quad_char(int v, int q) {
+  v = ((v % q) + q) % q;
+  if (v == 0) return 0;
+  for (int t = 1; t < q; ++t)
+    if ((t * t) % q == v) return 1;
+  return -1;
+}
+
+// Signs of a Paley Hadamard matrix of order m in {12, 20, 28}, H[i][j] in {+1, -1}.
+std::vector<int> paley_signs(int m) {
+  std::vector<int> H(static_cast<size_t>(m) * m, 0);
+  if (m == 12 || m == 20) {
+    // Paley I, q = m - 1 = 3 mod 4: H = I + S, S = [[0, 1..1], [-1.., Q]], Q[i][j] = chi(j - i)
+    const int q = m - 1;
+    for (int i = 0; i < m; ++i)
+      for (int j = 0; j < m; ++j) {
+        int s;
+        if (i == 0 && j == 0) s = 0;
+        else if (i == 0) s = 1;
+        else if (j == 0) s = -1;
+        else s = quad_char((j - 1) - (i - 1), q);
+        H[static_cast<size_t>(i) * m + j] = s + (i == j ? 1 : 0);
+      }
+  } else {
+    // Paley II, q = 13 = 1 mod 4: C = [[0, 1..1], [1.., Q]] (order 14, symmetric),
+    // H = [[C + I, C - I], [C - I, -C - I]]
+    const int q = 13, c = q + 1;
+    std::vector<int> C(static_cast<size_t>(c) * c, 0);
+    for (int i = 0; i < c; ++i)
+      for (int j = 0; j < c; ++j) {
+        if (i == 0 && j == 0) C[i * c + j] = 0;
+        else if (i == 0 || j == 0) C[i * c + j] = 1;
+        else C[i * c + j] = quad_char((j - 1) - (i - 1), q);
+      }
+    for (int bi = 0; bi < 2; ++bi)
+      for (int bj = 0; bj < 2; ++bj)
+        for (int i = 0; i < c; ++i)
+          for (int j = 0; j < c; ++j) {
+            const int cij = C[i * c + j], id = i == j ? 1 : 0;
+            int v;
+            if (bi == 0 && bj == 0) v = cij + id;
+            else if (bi == 1 && bj == 1) v = -cij - id;
+            else v = cij - id;
+            H[static_cast<size_t>(bi * c + i) * m + bj * c + j] = v;
+          }
+  }
+  return H;
+}
+
+}  // namespace
+
+bool rht_factor(int n, int* p2, int* m) {
+  if (n <= 0) return false;
+  const int ms[4] = {28, 20, 12, 1};
+  for (int k = 0; k < 4; ++k) {
+    if (n % ms[k]) continue;
+    const int p = n / ms[k];
+    if ((p & (p - 1)) == 0) {
+      *p2 = p;
+      *m = ms[k];
+      return true;
+    }
+  }
+  return false;
+}
+
+size_t rht_smem_bytes(int n) { return static_cast<size_t>(n) * sizeof(float); }
+
+unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_stride, int M, int n,
+                         const uint8_t* signs, int signs_first, cudaStream_t s) {
+  int p2 = 0, m = 0;
+  if (!rht_factor(n, &p2, &m)) return UNISVQ_ERR_UNSUPPORTED;
+  if (rht_smem_bytes(n) > 227 * 1024) return UNISVQ_ERR_UNSUPPORTED;
+  if (M <= 0) return UNISVQ_OK;
+  static bool attr_set[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
+  if (!attr_set[dev]) {
+    if (cudaFuncSetAttribute(rht_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024) != cudaSuccess)
+      return UNISVQ_ERR_CUDA;
+    attr_set[dev] = true;
+  }
+  RhtArgs a{};
+  a.in = static_cast<const uint16_t*>(in);
+  a.out = static_cast<uint16_t*>(out);
+  a.signs = signs;
+  a.n = n;
+  a.p2 = p2;
+  a.m = m;
+  int lg = 0;
+  while ((1 << lg) < p2) ++lg;
+  a.log2p = lg;
+  a.in_stride = in_stride;
+  a.out_stride = out_stride;
+  a.signs_first = signs_first;
+  a.scale = static_cast<float>(1.0 / std::sqrt(static_cast<double>(n)));
+  if (m > 1) {
+    const std::vector<int> H = paley_signs(m);
+    for (int c = 0; c < m; ++c) {
+      uint32_t mask = 0;
+      for (int q = 0; q < m; ++q)
+        if (H[static_cast<size_t>(q) * m + c] < 0) mask |= 1u << q;
+      a.hm_neg[c] = mask;
+    }
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(M, 1, 1);
+  cfg.blockDim = dim3(kRThreads, 1, 1);
+  cfg.dynamicSmemBytes = rht_smem_bytes(n);
+  cfg.stream = s;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr.val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, rht_kernel, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+}
+
+}  // namespace unisvq

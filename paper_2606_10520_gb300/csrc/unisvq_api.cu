@@ -271,6 +271,8 @@ unisvq_status unisvq_pack_grouped(const uint8_t* codes, const uint16_t* A_f16, c
   if (e != cudaSuccess) {
     cudaFree(L->codes);
     cudaFree(L->meta);
+    cudaFree(L->rht_signs);
+    cudaFree(L->rht_x);
     delete L;
     return cuda_status(e);
   }
@@ -288,6 +290,8 @@ unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
   L->tlut = nullptr;
   L->fold_ws = nullptr;
   L->meta = nullptr;
+  L->rht_signs = nullptr;
+  L->rht_x = nullptr;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // A device buffer of the source handle copied into a new allocation (none if the source has none).
   auto copy = [&](void** dst, const void* src, size_t bytes) -> cudaError_t {
@@ -307,6 +311,10 @@ unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
     if (e == cudaSuccess) e = cudaMemsetAsync(L->fold_ws, 0, ws_bytes, s);
   }
   if (e == cudaSuccess && h->grouped) e = copy(reinterpret_cast<void**>(&L->meta), h->meta, h->meta_bytes);
+  if (e == cudaSuccess && h->rht) {
+    e = copy(reinterpret_cast<void**>(&L->rht_signs), h->rht_signs, static_cast<size_t>(h->K) + h->N);
+    if (e == cudaSuccess) e = cudaMalloc(&L->rht_x, static_cast<size_t>(h->rht_tokens) * h->K * sizeof(uint16_t));
+  }
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) {
     cudaFree(L->codes);
@@ -314,6 +322,8 @@ unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
     cudaFree(L->tlut);
     cudaFree(L->fold_ws);
     cudaFree(L->meta);
+    cudaFree(L->rht_signs);
+    cudaFree(L->rht_x);
     delete L;
     return cuda_status(e);
   }
@@ -328,8 +338,11 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
   cudaError_t e3 = cudaFree(h->tlut);
   cudaError_t e4 = cudaFree(h->fold_ws);
   cudaError_t e5 = cudaFree(h->meta);
+  cudaError_t e6 = cudaFree(h->rht_signs);
+  cudaError_t e7 = cudaFree(h->rht_x);
   delete h;
-  return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess && e4 == cudaSuccess && e5 == cudaSuccess)
+  return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess && e4 == cudaSuccess && e5 == cudaSuccess &&
+          e6 == cudaSuccess && e7 == cudaSuccess)
              ? UNISVQ_OK
              : UNISVQ_ERR_CUDA;
 }
@@ -363,24 +376,28 @@ static unisvq_status check_io(unisvq_handle h, const void* x, void* y, int M) {
   return UNISVQ_OK;
 }
 
-unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, void* y, int M,
-                                  void* stream) {
-  unisvq_status st = check_io(h, x, y, M);
-  if (st != UNISVQ_OK || M == 0) return st;
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
-  if (dev != h->device) return UNISVQ_ERR_INVALID_ARG;
+// The layer itself (no RHT): `kernel` on x -> y; `noalloc` takes the tcgen05
+// decode path with the library's static fold workspace.
+static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, void* y, int M, cudaStream_t s,
+                                  bool noalloc) {
+  if (noalloc) {
+    if (h->grouped) {   // the per-group GEMV has no workspace
+      const unisvq_layer* Ls[1] = {h};
+      void* ys[1] = {y};
+      return launch_grouped_group(Ls, 1, x, ys, M, s);
+    }
+    return launch_skinny_static(h, x, y, M, s);
+  }
   if (h->grouped) {
     if (kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GROUPED)
       return kernel >= 0 && kernel <= UNISVQ_KERNEL_GROUPED ? UNISVQ_ERR_UNSUPPORTED : UNISVQ_ERR_INVALID_ARG;
     const unisvq_layer* Ls[1] = {h};
     void* ys[1] = {y};
-    return launch_grouped_group(Ls, 1, x, ys, M, static_cast<cudaStream_t>(stream));
+    return launch_grouped_group(Ls, 1, x, ys, M, s);
   }
   if (kernel == UNISVQ_KERNEL_GROUPED) return UNISVQ_ERR_UNSUPPORTED;
   if (kernel == UNISVQ_KERNEL_AUTO) kernel = auto_kernel(h, M);
   if (kernel == UNISVQ_KERNEL_DECODE) kernel = decode_kernel_for(static_cast<long long>(h->N) * h->K, h->Np / kTileRows, M);
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (kernel == UNISVQ_KERNEL_GEMV) return launch_gemv(h, x, y, M, s);
   if (kernel == UNISVQ_KERNEL_GEMV_ROWS) {
     if (!gemv_rows_supported(h, M < 4 ? M : 4)) return UNISVQ_ERR_UNSUPPORTED;
@@ -396,6 +413,37 @@ unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, vo
   return UNISVQ_ERR_INVALID_ARG;
 }
 
+// The layer with the inverse RHT around it when the handle has one (Eq.
+// def:hadamard: y = ((x S_V V) W_hat^T) U S_U), in chunks of the handle's
+// rotated-activation buffer; else the layer alone.
+static unisvq_status linear_rht(unisvq_handle h, int kernel, const void* x, void* y, int M, cudaStream_t s,
+                                bool noalloc) {
+  if (!h->rht) return linear_inner(h, kernel, x, y, M, s, noalloc);
+  if (kernel < UNISVQ_KERNEL_AUTO || kernel > UNISVQ_KERNEL_GROUPED) return UNISVQ_ERR_INVALID_ARG;
+  const uint8_t* s_in = h->rht_signs;
+  const uint8_t* s_out = h->rht_signs + h->K;
+  for (int m0 = 0; m0 < M; m0 += h->rht_tokens) {
+    const int mc = M - m0 < h->rht_tokens ? M - m0 : h->rht_tokens;
+    const uint16_t* xc = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * h->K;
+    uint16_t* yc = static_cast<uint16_t*>(y) + static_cast<size_t>(m0) * h->N;
+    unisvq_status st = launch_rht(xc, h->K, h->rht_x, h->K, mc, h->K, s_in, 1, s);
+    if (st == UNISVQ_OK) st = linear_inner(h, kernel, h->rht_x, yc, mc, s, noalloc);
+    if (st == UNISVQ_OK) st = launch_rht(yc, h->N, yc, h->N, mc, h->N, s_out, 0, s);
+    if (st != UNISVQ_OK) return st;
+  }
+  return UNISVQ_OK;
+}
+
+unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, void* y, int M,
+                                  void* stream) {
+  unisvq_status st = check_io(h, x, y, M);
+  if (st != UNISVQ_OK || M == 0) return st;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
+  if (dev != h->device) return UNISVQ_ERR_INVALID_ARG;
+  return linear_rht(h, kernel, x, y, M, static_cast<cudaStream_t>(stream), false);
+}
+
 unisvq_status unisvq_linear(unisvq_handle h, const void* x, void* y, int M, void* stream) {
   return unisvq_linear_force(h, UNISVQ_KERNEL_AUTO, x, y, M, stream);
 }
@@ -406,12 +454,64 @@ unisvq_status unisvq_linear_noalloc(unisvq_handle h, const void* x, void* y, int
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
   if (dev != h->device) return UNISVQ_ERR_INVALID_ARG;
-  if (h->grouped) {   // the per-group GEMV has no workspace
-    const unisvq_layer* Ls[1] = {h};
-    void* ys[1] = {y};
-    return launch_grouped_group(Ls, 1, x, ys, M, static_cast<cudaStream_t>(stream));
+  return linear_rht(h, UNISVQ_KERNEL_AUTO, x, y, M, static_cast<cudaStream_t>(stream), true);
+}
+
+unisvq_status unisvq_set_rht(unisvq_handle h, const uint8_t* sign_in, const uint8_t* sign_out, int max_tokens,
+                             void* stream) {
+  if (!h) return UNISVQ_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (!sign_in && !sign_out) {   // remove the transform
+    if (cudaStreamSynchronize(s) != cudaSuccess) return UNISVQ_ERR_CUDA;
+    cudaFree(h->rht_signs);
+    cudaFree(h->rht_x);
+    h->rht_signs = nullptr;
+    h->rht_x = nullptr;
+    h->rht = 0;
+    h->rht_tokens = 0;
+    return UNISVQ_OK;
   }
-  return launch_skinny_static(h, x, y, M, static_cast<cudaStream_t>(stream));
+  if (!sign_in || !sign_out || max_tokens < 1) return UNISVQ_ERR_INVALID_ARG;
+  for (int i = 0; i < h->K; ++i)
+    if (sign_in[i] > 1) return UNISVQ_ERR_INVALID_ARG;
+  for (int i = 0; i < h->N; ++i)
+    if (sign_out[i] > 1) return UNISVQ_ERR_INVALID_ARG;
+  int p2 = 0, m = 0;
+  if (!rht_factor(h->K, &p2, &m) || !rht_factor(h->N, &p2, &m)) return UNISVQ_ERR_UNSUPPORTED;
+  if (rht_smem_bytes(h->K) > 227 * 1024 || rht_smem_bytes(h->N) > 227 * 1024) return UNISVQ_ERR_UNSUPPORTED;
+  std::vector<uint8_t> signs(static_cast<size_t>(h->K) + h->N);
+  std::memcpy(signs.data(), sign_in, h->K);
+  std::memcpy(signs.data() + h->K, sign_out, h->N);
+  uint8_t* d_signs = nullptr;
+  uint16_t* d_x = nullptr;
+  cudaError_t e = cudaMalloc(&d_signs, signs.size());
+  if (e == cudaSuccess) e = cudaMalloc(&d_x, static_cast<size_t>(max_tokens) * h->K * sizeof(uint16_t));
+  if (e == cudaSuccess) e = cudaMemcpyAsync(d_signs, signs.data(), signs.size(), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) {
+    cudaFree(d_signs);
+    cudaFree(d_x);
+    return cuda_status(e);
+  }
+  cudaFree(h->rht_signs);
+  cudaFree(h->rht_x);
+  h->rht_signs = d_signs;
+  h->rht_x = d_x;
+  h->rht_tokens = max_tokens;
+  h->rht = 1;
+  return UNISVQ_OK;
+}
+
+unisvq_status unisvq_hadamard(const void* x, void* y, int M, int n, const uint8_t* signs, int signs_first,
+                              void* stream) {
+  if (M < 0 || n <= 0 || (signs_first != 0 && signs_first != 1)) return UNISVQ_ERR_INVALID_ARG;
+  if (M == 0) return UNISVQ_OK;
+  if (!x || !y || !aligned(x, 2) || !aligned(y, 2)) return UNISVQ_ERR_INVALID_ARG;
+  const size_t bytes = static_cast<size_t>(M) * n * 2;
+  if (x != y && overlaps(x, bytes, y, bytes)) return UNISVQ_ERR_INVALID_ARG;
+  int p2 = 0, m = 0;
+  if (!rht_factor(n, &p2, &m)) return UNISVQ_ERR_UNSUPPORTED;
+  return launch_rht(x, n, y, n, M, n, signs, signs_first, static_cast<cudaStream_t>(stream));
 }
 
 unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kernel, const void* x, void* const* ys,
@@ -430,6 +530,15 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
   if (dev != hs[0]->device) return UNISVQ_ERR_INVALID_ARG;
+  bool any_rht = false;
+  for (int i = 0; i < n; ++i) any_rht = any_rht || hs[i]->rht;
+  if (any_rht) {   // every layer rotates x with its own S_V: one call per layer
+    for (int i = 0; i < n; ++i) {
+      const unisvq_status st = linear_rht(hs[i], kernel, x, ys[i], M, static_cast<cudaStream_t>(stream), false);
+      if (st != UNISVQ_OK) return st;
+    }
+    return UNISVQ_OK;
+  }
   int ngrouped = 0;
   for (int i = 0; i < n; ++i) ngrouped += hs[i]->grouped ? 1 : 0;
   if (ngrouped) {   // all layers per-group with one d, run by the per-group GEMV
@@ -544,6 +653,10 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
   info->flops = 2.0 * M * static_cast<double>(h->N) * h->K;
   const unisvq_layer* Ls[1] = {h};
   describe_launch(Ls, 1, h->grouped ? UNISVQ_KERNEL_GROUPED : auto_kernel(h, M > 0 ? M : 1), M, info);
+  if (h->rht) {   // an input and an output rotation per chunk of the rotated-activation buffer
+    const int m = M > 0 ? M : 1;
+    info->launches += 2 * ((m + h->rht_tokens - 1) / h->rht_tokens);
+  }
   return UNISVQ_OK;
 }
 

@@ -1,0 +1,145 @@
+"""The randomized Hadamard transform (Eq. def:hadamard) on the GPU against the
+fp64 oracle: the rotation alone (every supported order family, both sign
+placements, in place and out of place), and the layer with the inverse
+rotation around it (per-matrix and per-group layers, chunked token counts,
+forced kernels, grouped calls)."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():
+    pytest.skip("no CUDA device", allow_module_level=True)
+
+from paper_2606_10520_gb300 import binding  # noqa: E402
+
+
+def to_dev(xbits: np.ndarray):
+    return torch.from_numpy(np.ascontiguousarray(xbits).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def host(t):
+    return t.float().cpu().numpy().astype(np.float64)
+
+
+def signs(n, seed):
+    return np.random.default_rng(seed).choice([-1.0, 1.0], size=n)
+
+
+@pytest.mark.parametrize("n", [12, 20, 28, 64, 96, 448, 4096, 5120, 14336, 28672])
+@pytest.mark.parametrize("signs_first", [1, 0])
+def test_rotation_matches_oracle(n, signs_first):
+    M = 3
+    xb = synth.activations(7, 50, n, M, n)
+    x = to_dev(xb)
+    s = signs(n, n)
+    sd = torch.from_numpy((s < 0).astype(np.uint8)).cuda()
+    y = torch.empty_like(x)
+    stream = torch.cuda.current_stream().cuda_stream
+    assert binding.hadamard_ptr(x.data_ptr(), y.data_ptr(), M, n, sd.data_ptr(), signs_first, stream) == binding.OK
+    assert binding.sync_status() == binding.OK
+    xf = oracle.bf16_bits_to_f64(xb)
+    H = oracle.hadamard(n) / np.sqrt(n)
+    ref = (xf * s) @ H if signs_first else (xf @ H) * s
+    got = host(y)
+    rms = np.sqrt(np.mean(ref ** 2))
+    assert np.all(np.abs(got - ref) <= 2.0 ** -8 * np.abs(ref) + 1e-5 * rms), np.abs(got - ref).max()
+    # in place gives the same bits
+    z = x.clone()
+    assert binding.hadamard_ptr(z.data_ptr(), z.data_ptr(), M, n, sd.data_ptr(), signs_first, stream) == binding.OK
+    assert binding.sync_status() == binding.OK
+    assert torch.equal(z, y)
+
+
+def test_rotation_without_signs_and_bad_orders():
+    n, M = 256, 2
+    xb = synth.activations(7, 51, 0, M, n)
+    x = to_dev(xb)
+    y = torch.empty_like(x)
+    stream = torch.cuda.current_stream().cuda_stream
+    assert binding.hadamard_ptr(x.data_ptr(), y.data_ptr(), M, n, 0, 1, stream) == binding.OK
+    assert binding.sync_status() == binding.OK
+    ref = oracle.bf16_bits_to_f64(xb) @ (oracle.hadamard(n) / 16.0)
+    assert np.allclose(host(y), ref, rtol=2.0 ** -8, atol=1e-5)
+    for bad in (11008, 36, 100):
+        xb2 = torch.zeros((1, bad), dtype=torch.bfloat16, device="cuda")
+        yb2 = torch.zeros((1, bad), dtype=torch.bfloat16, device="cuda")
+        assert binding.hadamard_ptr(xb2.data_ptr(), yb2.data_ptr(), 1, bad, 0, 1, stream) == binding.ERR_UNSUPPORTED
+    assert binding.hadamard_ptr(x.data_ptr(), y.data_ptr(), 1, n, 0, 2, stream) == binding.ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("N,K,d", [(4096, 4096, 2), (1792, 3584, 2), (640, 1280, 4), (768, 2560, 1)])
+def test_layer_with_inverse_rht(N, K, d):
+    codes, A, B = synth.layer_inputs(7, 52, N, K, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    s_U, s_V = signs(N, 1 + N), signs(K, 2 + K)
+    layer.set_rht(s_V, s_U, max_tokens=64)
+    Ms = (1, 5, 16, 70)
+    xall = synth.activations(7, 52, N + K, sum(Ms), K)
+    yr, S = oracle.linear_rht(xall, codes, A, B, s_U, s_V)
+    o = 0
+    for M in Ms:
+        y = layer.forward(to_dev(xall[o:o + M]))
+        assert binding.sync_status() == binding.OK
+        res = oracle.compare(host(y), yr[o:o + M], S[o:o + M])
+        assert res["ok"], (M, res)
+        o += M
+    info = layer.query(70)
+    assert info["launches"] >= 2 * 2   # two chunks, an input and an output rotation each
+    # a forced kernel keeps the rotations; removing them restores the plain layer
+    x5 = to_dev(xall[:5])
+    for kern in (binding.KERNEL_GEMV, binding.KERNEL_SKINNY):
+        y = layer.forward(x5, kernel=kern)
+        assert binding.sync_status() == binding.OK
+        assert oracle.compare(host(y), yr[:5], S[:5])["ok"]
+    layer.set_rht(None, None)
+    y = layer.forward(x5)
+    assert binding.sync_status() == binding.OK
+    yp, Sp = oracle.linear(xall[:5], codes, A, B)
+    assert oracle.compare(host(y), yp, Sp)["ok"]
+    layer.close()
+
+
+def test_grouped_layer_and_group_call_with_rht():
+    K, d = 1024, 2
+    shapes = [(512, K), (256, K)]
+    made = [synth.layer_inputs_grouped(7, 53, i, 0, N, K_, d) for i, (N, K_) in enumerate(shapes)]
+    layers = [binding.UniSVQLinear(c, A, B, group_cols=128) for c, A, B in made]
+    sg = [(signs(N, 10 + i), signs(K, 20 + i)) for i, (N, _) in enumerate(shapes)]
+    for layer, (s_U, s_V) in zip(layers, sg):
+        layer.set_rht(s_V, s_U, max_tokens=8)
+    M = 12
+    xb = synth.activations(7, 53, 0, M, K)
+    ys = binding.linear_group(layers, to_dev(xb))
+    assert binding.sync_status() == binding.OK
+    for (c, A, B), (s_U, s_V), y in zip(made, sg, ys):
+        xt = oracle.rht_input(xb, s_V)
+        yt, St = oracle.linear_grouped(xt, c, A, B, 128)
+        N = c.shape[0]
+        ref = oracle.rht_output(yt, s_U)
+        Sref = St @ (np.abs(oracle.hadamard(N)) / np.sqrt(N))
+        assert oracle.compare(host(y), ref, Sref)["ok"]
+    for layer in layers:
+        layer.close()
+
+
+def test_set_rht_rejects_unsupported_widths_and_bad_signs():
+    N, K = 11008, 4096
+    codes = np.zeros((N, K), dtype=np.uint8)
+    layer = binding.UniSVQLinear(codes, np.eye(2, dtype=np.float16), np.zeros(2, dtype=np.float16))
+    with pytest.raises(binding.UnisvqError) as e:
+        layer.set_rht(np.ones(K), np.ones(N))
+    assert e.value.status == binding.ERR_UNSUPPORTED
+    layer.close()
+    layer = binding.UniSVQLinear(np.zeros((256, 512), dtype=np.uint8), np.eye(2, dtype=np.float16),
+                                 np.zeros(2, dtype=np.float16))
+    bad = np.zeros(512, dtype=np.uint8)
+    bad[3] = 2
+    with pytest.raises(binding.UnisvqError) as e:
+        layer.set_rht(bad, np.zeros(256, dtype=np.uint8))
+    assert e.value.status == binding.ERR_INVALID_ARG
+    layer.close()
