@@ -280,7 +280,7 @@ def run_ours(args, rank, world, local_rank):
         print(json.dumps({"prefill": run_prefill(torch, binding, peaks, args, side)}), flush=True)
         return
     if args.only == "decode":
-        args.no_e2e = args.no_cpu = args.no_prefill = args.no_grouped = True
+        args.no_e2e = args.no_cpu = args.no_prefill = args.no_grouped = args.no_rht = True
     shapes = synth.LLAMA2_7B
     stack = build_stack(binding, shapes, args.layers, 1)
 
@@ -468,6 +468,11 @@ def run_ours(args, rank, world, local_rank):
     if not args.no_grouped:
         grouped = run_grouped(torch, binding, peaks, args, side)
 
+    # ---- inverse RHT around the layers -------------------------------------
+    rht = None
+    if not args.no_rht:
+        rht = run_rht(torch, binding, peaks, args, side)
+
     # ---- prefill (tcgen05 GEMM), Llama-3-8B-shaped set at M = 2048 -------
     prefill = None
     if not args.no_prefill:
@@ -498,6 +503,7 @@ def run_ours(args, rank, world, local_rank):
         "cpu_baseline": cpu,
         "prefill": prefill,
         "per_group_affine": grouped,
+        "rht": rht,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -565,6 +571,73 @@ def run_grouped(torch, binding, peaks, args, stream):
             "GB/s": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"], "sweep": per_m,
             "kernel": "gemv_grouped_kernel", "launches_per_step": launches,
             "bytes": "codes N*K/4 + maps N*ceil(K/128)*12 + x + y per call",
+            "timing": "CUDA graphs of the layer stack per M, CUDA events on the capture stream"}
+
+
+def run_rht(torch, binding, peaks, args, stream):
+    """The decode sweep on Llama-3-8B-shaped layers (every width 2^a m with a
+    Hadamard order here) with and without the inverse randomized Hadamard
+    transform around each layer (Eq. def:hadamard): q/k/v and gate/up share
+    their input rotation S_V V, every layer has its own output rotation U S_U.
+    GB/s counts the layers' algorithmic bytes only."""
+    shapes = synth.LLAMA3_8B
+    g = np.random.default_rng(5)
+    base = []
+    for pi, (_, N, K) in enumerate(shapes):
+        codes, A, B = synth.layer_inputs(0, 2, 0, pi, N, K, 2)
+        base.append(binding.UniSVQLinear(codes, A, B))
+    s_in = {K: g.choice([-1.0, 1.0], K) for K in sorted({K for _, _, K in shapes})}
+    s_out = [g.choice([-1.0, 1.0], N) for _, N, _ in shapes]
+    stack = [base] + [[b.clone() for b in base] for _ in range(GROUPED_LAYERS - 1)]
+    xs, ys = {}, {}
+    for M in M_SWEEP:
+        for pi, (_, N, K) in enumerate(shapes):
+            if (M, K) not in xs:
+                xb = synth.activations(0, 2, 100 + M, M, K)
+                xs[(M, K)] = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).cuda()
+            ys[(M, pi)] = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    step_bytes = sum(algo_bytes(N, K, M) for M in M_SWEEP for _, N, K in shapes) * GROUPED_LAYERS
+    steps = max(5, args.steps // 4)
+    out = {}
+    for rht in (False, True):
+        for layer in stack:
+            for pi, b in enumerate(layer):
+                if rht:
+                    b.set_rht(s_in[shapes[pi][2]], s_out[pi], max_tokens=max(M_SWEEP))
+                else:
+                    b.set_rht(None, None)
+        graphs = []
+        for M in M_SWEEP:
+            def one_pass(M=M):
+                sp = torch.cuda.current_stream().cuda_stream
+                for layer in stack:
+                    for grp in GROUPS_7B:
+                        K = shapes[grp[0]][2]
+                        st = binding.linear_group_ptr([layer[i] for i in grp], xs[(M, K)].data_ptr(),
+                                                      [ys[(M, i)].data_ptr() for i in grp], M, sp)
+                        if st != 0:
+                            raise RuntimeError(f"unisvq call failed: {binding.status_string(st)}")
+            with torch.cuda.stream(stream):
+                one_pass()
+            torch.cuda.synchronize()
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=stream):
+                one_pass()
+            graphs.append(gr)
+        st = binding.sync_status(stream)
+        if st != 0:
+            raise RuntimeError(f"device status {binding.status_string(st)}")
+        t = time_graphs(torch, graphs, steps, args.warmup, stream)
+        out["with_rht" if rht else "without_rht"] = step_bytes * steps / t / 1e9
+    for layer in stack:
+        for b in layer:
+            b.close()
+    return {"workload": f"Llama-3-8B-shaped projection set x {GROUPED_LAYERS} layers, decode sweep M in "
+                        f"{list(M_SWEEP)}, d=2, per-matrix fp16 affine, inverse RHT around every layer",
+            "GB/s": out["with_rht"], "GB/s_without_rht": out["without_rht"],
+            "frac_of_measured_hbm": out["with_rht"] / peaks["hbm_gbs"],
+            "kernels": "rht_kernel (input and output rotations, cluster of 8 CTAs per row) + the layers' kernels",
+            "bytes": "the layers' algorithmic bytes (codes + affine + x + y); the rotations are overhead",
             "timing": "CUDA graphs of the layer stack per M, CUDA events on the capture stream"}
 
 
@@ -649,6 +722,8 @@ def main():
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-rht", action="store_true",
+                    help="skip the inverse-RHT sweep (Llama-3-8B shapes)")
     ap.add_argument("--no-grouped", action="store_true",
                     help="skip the per-(row, 128-column group) affine sweep")
     ap.add_argument("--ungrouped", action="store_true",

@@ -3,6 +3,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <vector>
 #include <cuda_runtime.h>
 
 #include "unisvq.h"
@@ -37,6 +38,7 @@ struct unisvq_layer {
   uint8_t* rht_signs;
   uint16_t* rht_x;
   int rht_tokens;
+  std::vector<uint8_t> rht_in_host;   // host copy of S_V: layers of a grouped call that share it rotate x once
 };
 
 namespace unisvq {

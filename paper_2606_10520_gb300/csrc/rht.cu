@@ -8,11 +8,17 @@
 // {1, 12, 20, 28}; entry [(p, q), (p', q')] (index p m + q) is
 // H_{2^a}[p][p'] H_m[q][q'].
 //
-// One CTA transforms one row in shared memory (fp32): the row-vector product
-// with H_m inside every block of m consecutive entries (registers, signs of
-// H_m as per-column bit masks), then the Sylvester butterflies across blocks in
-// radix-8 passes (three stages per pass in registers, one barrier per pass),
-// then the scale 1/sqrt(n) and, on the way out, the signs.
+// A row is split over a cluster of G <= 8 CTAs (G = min(8, 2^a)), CTA j
+// holding the 2^a / G consecutive m-blocks j 2^a / G .. in shared memory
+// (fp32). Phase 1, local: signs (on the way in), the row-vector product with
+// H_m inside every block (registers; signs of H_m as per-column bit masks),
+// and the Sylvester butterflies between blocks of the chunk (radix-8 passes,
+// three stages per pass in registers, one barrier per pass). Phase 2, after a
+// cluster barrier: the remaining log2 G Sylvester stages run across the
+// chunks; CTA j takes the j-th G-th of the positions, reads the G values of a
+// position from the G CTAs' shared memory, transforms them in registers and
+// writes the scaled (and, on the way out, signed) bf16 results. A second
+// cluster barrier keeps every CTA's shared memory alive until all reads end.
 #include <cmath>
 #include <vector>
 
@@ -22,7 +28,7 @@
 namespace unisvq {
 namespace {
 
-constexpr int kRThreads = 512;
+constexpr int kRThreads = 256;
 constexpr int kMaxPaley = 28;
 
 struct RhtArgs {
@@ -30,7 +36,7 @@ struct RhtArgs {
   uint16_t* out;            // bf16 [M][out_stride] (may equal in)
   const uint8_t* signs;     // [n], 1 = negate; null = all +1
   int n, p2, m;             // n = p2 * m
-  int log2p;
+  int G;                    // CTAs per row (cluster size), a power of 2 <= min(8, p2)
   int in_stride, out_stride;
   int signs_first;          // 1: x -> (s x) H; 0: x -> (x H) s
   float scale;              // 1 / sqrt(n)
@@ -39,19 +45,25 @@ struct RhtArgs {
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float(static_cast<uint32_t>(b) << 16); }
 
-// Row vector times H_m for one block of M_ consecutive entries, in place.
+// Row vector times H_m for every block of M_ consecutive entries of src,
+// into dst: four threads per block, each forming M_/4 of its outputs.
 template <int M_>
-__device__ __forceinline__ void paley_block(float* blk, const uint32_t (&neg)[kMaxPaley]) {
-  float v[M_];
+__device__ __forceinline__ void paley_blocks(const float* src, float* dst, int nblk, const uint32_t* neg) {
+  constexpr int C = M_ / 4;
+  for (int it = threadIdx.x; it < nblk * 4; it += kRThreads) {
+    const int p = it >> 2, c0 = (it & 3) * C;
+    const float* blk = src + p * M_;
+    float v[M_];
 #pragma unroll
-  for (int q = 0; q < M_; ++q) v[q] = blk[q];
+    for (int q = 0; q < M_; ++q) v[q] = blk[q];
 #pragma unroll
-  for (int c = 0; c < M_; ++c) {
-    const uint32_t mask = neg[c];
-    float acc = 0.f;
+    for (int c = 0; c < C; ++c) {
+      const uint32_t mask = neg[c0 + c];
+      float acc = 0.f;
 #pragma unroll
-    for (int q = 0; q < M_; ++q) acc += ((mask >> q) & 1u) ? -v[q] : v[q];
-    blk[c] = acc;
+      for (int q = 0; q < M_; ++q) acc += ((mask >> q) & 1u) ? -v[q] : v[q];
+      dst[p * M_ + c0 + c] = acc;
+    }
   }
 }
 
@@ -84,45 +96,100 @@ __device__ __forceinline__ void sylvester_pass(float* buf, int p2, int m, int s0
   }
 }
 
+// G-point Sylvester transform of position e of the chunk across the cluster.
+template <int G>
+__device__ __forceinline__ void cross_chunk(const RhtArgs& a, const float* buf, uint16_t* dst, int chunk, int e) {
+  float v[G];
+  const uint32_t local = smem_u32(buf + e);
+#pragma unroll
+  for (int r = 0; r < G; ++r) v[r] = ld_shared_cluster_f32(map_shared_rank(local, r));
+#pragma unroll
+  for (int d = 1; d < G; d <<= 1)
+#pragma unroll
+    for (int j = 0; j < G; ++j)
+      if (!(j & d)) {
+        const float x0 = v[j], x1 = v[j + d];
+        v[j] = x0 + x1;
+        v[j + d] = x0 - x1;
+      }
+#pragma unroll
+  for (int r = 0; r < G; ++r) {
+    const int i = r * chunk + e;
+    float o = v[r] * a.scale;
+    if (!a.signs_first && a.signs && a.signs[i]) o = -o;
+    dst[i] = f32_to_bf16_rn(o);
+  }
+}
+
 __global__ void __launch_bounds__(kRThreads) rht_kernel(const __grid_constant__ RhtArgs a) {
-  extern __shared__ __align__(16) float buf[];
-  const int row = blockIdx.x;
-  const int n = a.n;
+  extern __shared__ __align__(16) float smem_f[];
+  float* buf = smem_f;   // the chunk; a second chunk-sized buffer follows when m > 1
+  const int G = a.G;
+  const int rank = G > 1 ? static_cast<int>(cluster_ctarank()) : 0;
+  const int row = blockIdx.x / G;
+  const int pl = a.p2 / G;             // m-blocks per CTA
+  const int chunk = pl * a.m;          // values per CTA
+  const int base = rank * chunk;
   pdl_launch_dependents();
   pdl_wait();   // the row may be the previous kernel's output
-  const uint16_t* src = a.in + static_cast<size_t>(row) * a.in_stride;
-  for (int i = threadIdx.x; i < n; i += kRThreads) {
-    float v = bf16_to_f32(src[i]);
-    if (a.signs_first && a.signs && a.signs[i]) v = -v;
-    buf[i] = v;
+  const uint16_t* src = a.in + static_cast<size_t>(row) * a.in_stride + base;
+  const bool sgn_in = a.signs_first && a.signs;
+  if ((chunk & 7) == 0 && (a.in_stride & 7) == 0) {   // 16-byte loads of 8 values
+    for (int i8 = threadIdx.x; i8 < chunk / 8; i8 += kRThreads) {
+      const uint4 w = ldg_v4(src + 8 * i8);
+      const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        float v = (k & 1) ? bf16_hi(ws[k >> 1]) : bf16_lo(ws[k >> 1]);
+        if (sgn_in && a.signs[base + 8 * i8 + k]) v = -v;
+        buf[8 * i8 + k] = v;
+      }
+    }
+  } else {
+    for (int i = threadIdx.x; i < chunk; i += kRThreads) {
+      float v = bf16_to_f32(src[i]);
+      if (sgn_in && a.signs[base + i]) v = -v;
+      buf[i] = v;
+    }
   }
   __syncthreads();
   if (a.m > 1) {
-    uint32_t neg[kMaxPaley];
-#pragma unroll
-    for (int c = 0; c < kMaxPaley; ++c) neg[c] = a.hm_neg[c];
-    for (int p = threadIdx.x; p < a.p2; p += kRThreads) {
-      float* blk = buf + p * a.m;
-      if (a.m == 12) paley_block<12>(blk, neg);
-      else if (a.m == 20) paley_block<20>(blk, neg);
-      else paley_block<28>(blk, neg);
-    }
+    float* out2 = smem_f + chunk;
+    if (a.m == 12) paley_blocks<12>(buf, out2, pl, a.hm_neg);
+    else if (a.m == 20) paley_blocks<20>(buf, out2, pl, a.hm_neg);
+    else paley_blocks<28>(buf, out2, pl, a.hm_neg);
+    buf = out2;
     __syncthreads();
   }
-  for (int s0 = 0; s0 < a.log2p;) {
-    const int r = min(3, a.log2p - s0);
-    if (r == 3) sylvester_pass<3>(buf, a.p2, a.m, s0);
-    else if (r == 2) sylvester_pass<2>(buf, a.p2, a.m, s0);
-    else sylvester_pass<1>(buf, a.p2, a.m, s0);
+  int lg = 0;
+  while ((1 << lg) < pl) ++lg;
+  for (int s0 = 0; s0 < lg;) {
+    const int r = min(3, lg - s0);
+    if (r == 3) sylvester_pass<3>(buf, pl, a.m, s0);
+    else if (r == 2) sylvester_pass<2>(buf, pl, a.m, s0);
+    else sylvester_pass<1>(buf, pl, a.m, s0);
     s0 += r;
     __syncthreads();
   }
   uint16_t* dst = a.out + static_cast<size_t>(row) * a.out_stride;
-  for (int i = threadIdx.x; i < n; i += kRThreads) {
-    float v = buf[i] * a.scale;
-    if (!a.signs_first && a.signs && a.signs[i]) v = -v;
-    dst[i] = f32_to_bf16_rn(v);
+  if (G == 1) {
+    for (int i = threadIdx.x; i < chunk; i += kRThreads) {
+      float v = buf[i] * a.scale;
+      if (!a.signs_first && a.signs && a.signs[i]) v = -v;
+      dst[i] = f32_to_bf16_rn(v);
+    }
+    return;
   }
+  cluster_sync();   // every chunk is transformed locally
+  // CTA `rank` finishes positions [rank span, (rank + 1) span) of all G chunks
+  const int span = (chunk + G - 1) / G;
+  const int e1 = min(chunk, (rank + 1) * span);
+  for (int e = rank * span + static_cast<int>(threadIdx.x); e < e1; e += kRThreads) {
+    if (G == 8) cross_chunk<8>(a, buf, dst, chunk, e);
+    else if (G == 4) cross_chunk<4>(a, buf, dst, chunk, e);
+    else cross_chunk<2>(a, buf, dst, chunk, e);
+  }
+  cluster_sync();   // no CTA leaves while another still reads its shared memory
 }
 
 // chi(v) mod q for prime q: +1 on nonzero squares, -1 on non-squares, 0 at 0.
@@ -192,7 +259,13 @@ bool rht_factor(int n, int* p2, int* m) {
   return false;
 }
 
-size_t rht_smem_bytes(int n) { return static_cast<size_t>(n) * sizeof(float); }
+// Shared memory of one CTA: its chunk of n / min(8, 2^a) values (twice that
+// when m > 1: the product with H_m writes a second buffer).
+size_t rht_smem_bytes(int n) {
+  int p2 = 0, m = 0;
+  if (!rht_factor(n, &p2, &m)) return static_cast<size_t>(n) * sizeof(float);
+  return static_cast<size_t>(n / (p2 >= 8 ? 8 : p2)) * sizeof(float) * (m > 1 ? 2 : 1);
+}
 
 unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_stride, int M, int n,
                          const uint8_t* signs, int signs_first, cudaStream_t s) {
@@ -215,9 +288,7 @@ unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_strid
   a.n = n;
   a.p2 = p2;
   a.m = m;
-  int lg = 0;
-  while ((1 << lg) < p2) ++lg;
-  a.log2p = lg;
+  a.G = p2 >= 8 ? 8 : p2;
   a.in_stride = in_stride;
   a.out_stride = out_stride;
   a.signs_first = signs_first;
@@ -232,15 +303,19 @@ unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_strid
     }
   }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(M, 1, 1);
+  cfg.gridDim = dim3(M * a.G, 1, 1);
   cfg.blockDim = dim3(kRThreads, 1, 1);
   cfg.dynamicSmemBytes = rht_smem_bytes(n);
   cfg.stream = s;
-  cudaLaunchAttribute attr;
-  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr.val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = &attr;
-  cfg.numAttrs = 1;
+  cudaLaunchAttribute attrs[2];
+  attrs[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attrs[0].val.programmaticStreamSerializationAllowed = 1;
+  attrs[1].id = cudaLaunchAttributeClusterDimension;
+  attrs[1].val.clusterDim.x = a.G;
+  attrs[1].val.clusterDim.y = 1;
+  attrs[1].val.clusterDim.z = 1;
+  cfg.attrs = attrs;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, rht_kernel, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 

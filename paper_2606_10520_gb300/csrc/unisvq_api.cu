@@ -469,6 +469,7 @@ unisvq_status unisvq_set_rht(unisvq_handle h, const uint8_t* sign_in, const uint
     h->rht_x = nullptr;
     h->rht = 0;
     h->rht_tokens = 0;
+    h->rht_in_host.clear();
     return UNISVQ_OK;
   }
   if (!sign_in || !sign_out || max_tokens < 1) return UNISVQ_ERR_INVALID_ARG;
@@ -499,6 +500,7 @@ unisvq_status unisvq_set_rht(unisvq_handle h, const uint8_t* sign_in, const uint
   h->rht_x = d_x;
   h->rht_tokens = max_tokens;
   h->rht = 1;
+  h->rht_in_host.assign(sign_in, sign_in + h->K);
   return UNISVQ_OK;
 }
 
@@ -513,6 +515,9 @@ unisvq_status unisvq_hadamard(const void* x, void* y, int M, int n, const uint8_
   if (!rht_factor(n, &p2, &m)) return UNISVQ_ERR_UNSUPPORTED;
   return launch_rht(x, n, y, n, M, n, signs, signs_first, static_cast<cudaStream_t>(stream));
 }
+
+static unisvq_status group_inner(const unisvq_handle* hs, int n, int kernel, const void* x, void* const* ys, int M,
+                                 cudaStream_t s);
 
 unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kernel, const void* x, void* const* ys,
                                         int M, void* stream) {
@@ -530,15 +535,43 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISVQ_ERR_CUDA;
   if (dev != hs[0]->device) return UNISVQ_ERR_INVALID_ARG;
-  bool any_rht = false;
-  for (int i = 0; i < n; ++i) any_rht = any_rht || hs[i]->rht;
-  if (any_rht) {   // every layer rotates x with its own S_V: one call per layer
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int nrht = 0;
+  for (int i = 0; i < n; ++i) nrht += hs[i]->rht ? 1 : 0;
+  if (!nrht) return group_inner(hs, n, kernel, x, ys, M, s);
+  bool shared = nrht == n;
+  for (int i = 1; i < n && shared; ++i) shared = hs[i]->rht_in_host == hs[0]->rht_in_host;
+  if (!shared) {   // each layer rotates x with its own S_V: one call per layer
     for (int i = 0; i < n; ++i) {
-      const unisvq_status st = linear_rht(hs[i], kernel, x, ys[i], M, static_cast<cudaStream_t>(stream), false);
+      const unisvq_status st = linear_rht(hs[i], kernel, x, ys[i], M, s, false);
       if (st != UNISVQ_OK) return st;
     }
     return UNISVQ_OK;
   }
+  // One S_V for every layer: rotate x once (into the first handle's buffer),
+  // run the layers as one group, rotate each output with its own U S_U.
+  if (kernel < UNISVQ_KERNEL_AUTO || kernel > UNISVQ_KERNEL_GROUPED) return UNISVQ_ERR_INVALID_ARG;
+  int cap = hs[0]->rht_tokens;
+  for (int i = 1; i < n; ++i) cap = hs[i]->rht_tokens < cap ? hs[i]->rht_tokens : cap;
+  const int K = hs[0]->K;
+  for (int m0 = 0; m0 < M; m0 += cap) {
+    const int mc = M - m0 < cap ? M - m0 : cap;
+    void* yc[UNISVQ_MAX_GROUP];
+    for (int i = 0; i < n; ++i) yc[i] = static_cast<uint16_t*>(ys[i]) + static_cast<size_t>(m0) * hs[i]->N;
+    unisvq_status st = launch_rht(static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * K, K, hs[0]->rht_x, K,
+                                  mc, K, hs[0]->rht_signs, 1, s);
+    if (st == UNISVQ_OK) st = group_inner(hs, n, kernel, hs[0]->rht_x, yc, mc, s);
+    for (int i = 0; i < n && st == UNISVQ_OK; ++i)
+      st = launch_rht(yc[i], hs[i]->N, yc[i], hs[i]->N, mc, hs[i]->N, hs[i]->rht_signs + K, 0, s);
+    if (st != UNISVQ_OK) return st;
+  }
+  return UNISVQ_OK;
+}
+
+// A grouped call without the RHT: one launch across the layers where the
+// kernel allows it, else one per layer.
+static unisvq_status group_inner(const unisvq_handle* hs, int n, int kernel, const void* x, void* const* ys, int M,
+                                 cudaStream_t s) {
   int ngrouped = 0;
   for (int i = 0; i < n; ++i) ngrouped += hs[i]->grouped ? 1 : 0;
   if (ngrouped) {   // all layers per-group with one d, run by the per-group GEMV
@@ -550,7 +583,7 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
       if (hs[i]->d != hs[0]->d) return UNISVQ_ERR_UNSUPPORTED;
       Ls[i] = hs[i];
     }
-    return launch_grouped_group(Ls, n, x, ys, M, static_cast<cudaStream_t>(stream));
+    return launch_grouped_group(Ls, n, x, ys, M, s);
   }
   if (kernel == UNISVQ_KERNEL_GROUPED) return UNISVQ_ERR_UNSUPPORTED;
   long long weights = 0;
@@ -565,7 +598,6 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
     kernel = decode_kernel_for(weights, nb, M);
   const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
   for (int i = 0; i < n; ++i) Ls[i] = hs[i];
-  const cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (kernel == UNISVQ_KERNEL_GEMV) return launch_gemv_group(Ls, n, x, ys, M, s);
   if (kernel == UNISVQ_KERNEL_SKINNY) return launch_skinny_group(Ls, n, x, ys, M, s);
   if (kernel == UNISVQ_KERNEL_GEMV_ROWS) {
@@ -574,7 +606,7 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
     return launch_gemv_rows_group(Ls, n, x, ys, M, s);
   }
   for (int i = 0; i < n; ++i) {
-    const unisvq_status st = unisvq_linear_force(hs[i], kernel, x, ys[i], M, stream);
+    const unisvq_status st = linear_inner(hs[i], kernel, x, ys[i], M, s, false);
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;

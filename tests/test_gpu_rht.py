@@ -143,3 +143,26 @@ def test_set_rht_rejects_unsupported_widths_and_bad_signs():
         layer.set_rht(bad, np.zeros(256, dtype=np.uint8))
     assert e.value.status == binding.ERR_INVALID_ARG
     layer.close()
+
+
+@pytest.mark.parametrize("M", [1, 16, 40])
+def test_group_call_sharing_the_input_rotation(M):
+    """Layers that share S_V (same input space) rotate x once and run as one
+    group; each output still gets its own U S_U."""
+    K, d = 4096, 2
+    shapes = [(4096, K), (1024, K), (1024, K)]
+    made = [synth.layer_inputs(7, 54, i, 0, N, K_, d) for i, (N, K_) in enumerate(shapes)]
+    layers = [binding.UniSVQLinear(c, A, B) for c, A, B in made]
+    s_V = signs(K, 99)
+    s_Us = [signs(N, 100 + i) for i, (N, _) in enumerate(shapes)]
+    for layer, s_U in zip(layers, s_Us):
+        layer.set_rht(s_V, s_U, max_tokens=16)
+    xb = synth.activations(7, 54, M, M, K)
+    ys = binding.linear_group(layers, to_dev(xb))
+    assert binding.sync_status() == binding.OK
+    for (c, A, B), s_U, y in zip(made, s_Us, ys):
+        ref, S = oracle.linear_rht(xb, c, A, B, s_U, s_V)
+        res = oracle.compare(host(y), ref, S)
+        assert res["ok"], res
+    for layer in layers:
+        layer.close()
