@@ -17,6 +17,10 @@ Every function cites the passage of the paper it follows:
 * Eq. (def:ptq_loss), Sec. 2.1 -- the layer output is Y = X W^T with X tokens x
   inputs and W outputs x inputs.
 
+`dequant`, `linear` and `linear_folded` take integer codes of any width:
+2-bit codes z in {0..3} and the 3-bit variant z in {0..7} (Sec. 5.2, Table
+tab:bitwidth: only the integer vectors widen).
+
 Inputs are exactly widened to fp64 (bf16 activations, fp16 affine). Where the
 paper fixes no rounding, the oracle keeps everything exact in fp64 and rounds
 once at the very end (`dequant_f32`).
@@ -81,15 +85,17 @@ def codeword(z, A, B) -> np.ndarray:
     return A @ np.asarray(z, dtype=np.float64) + B
 
 
-def codebook(A, B) -> np.ndarray:
-    """All 4^d codewords, row v = A z(v) + B with z_c(v) = (v >> 2c) & 3.
+def codebook(A, B, bits: int = 2) -> np.ndarray:
+    """All 2^(bits d) codewords, row v = A z(v) + B with z_c(v) the bit-field
+    [bits (c+1) - 1 : bits c] of v.
 
-    Eq. (def:unisvq) evaluated on every point of {0,1,2,3}^d; coordinate c of
-    the lattice point is bit-field [2c+1:2c] of the vector index v.
+    Eq. (def:unisvq) evaluated on every point of {0..2^bits - 1}^d (2-bit codes
+    by default; 3-bit codes only widen the lattice, Sec. 5.2).
     """
     d = np.asarray(A).shape[0]
-    v = np.arange(4 ** d)
-    Z = np.stack([(v >> (2 * c)) & 3 for c in range(d)], axis=1).astype(np.float64)
+    v = np.arange(2 ** (bits * d))
+    mask = (1 << bits) - 1
+    Z = np.stack([(v >> (bits * c)) & mask for c in range(d)], axis=1).astype(np.float64)
     return Z @ as_f64(A).T + as_f64(B)
 
 

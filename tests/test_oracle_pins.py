@@ -29,17 +29,17 @@ def haar_orthogonal(d, seed):
     return Q * np.sign(np.diag(R))
 
 
-def pin_enumeration_moments(dequant_fn, d, seed=0):
-    """App. A.1: with A = sG (G orthogonal), B = -sG b 1, b = (2^2-1)/2 and
-    s = sqrt(12/(2^4-1)), the 4^d codewords, each taken once (the uniform law
-    on {0..3}^d), have mean exactly 0 and covariance exactly I."""
+def pin_enumeration_moments(dequant_fn, d, seed=0, bits=2):
+    """Eq. (def:affine), App. A.1: with A = sG (G orthogonal), B = -sG b 1,
+    b = (2^bits-1)/2 and s = sqrt(12/(2^(2 bits)-1)), the 2^(bits d)
+    codewords, each taken once (the uniform law on {0..2^bits-1}^d), have mean
+    exactly 0 and covariance exactly I."""
     G = haar_orthogonal(d, seed)
-    bits = 2
     b = (2 ** bits - 1) / 2
     s = np.sqrt(12.0 / (2 ** (2 * bits) - 1))
     A = s * G
     B = -s * G @ (b * np.ones(d))
-    pts = np.array(list(itertools.product(range(4), repeat=d)), dtype=np.uint8)
+    pts = np.array(list(itertools.product(range(2 ** bits), repeat=d)), dtype=np.uint8)
     W = dequant_fn(pts, A, B)            # one codeword per row (K = d)
     mean = W.mean(axis=0)
     cov = (W - mean).T @ (W - mean) / W.shape[0]
@@ -435,3 +435,36 @@ def test_rht_input_output_are_inverse_rotations():
     # rht_output applies U then S; with U = V its transpose undoes rht_input
     V = oracle.hadamard(K) / np.sqrt(K)
     assert np.allclose((xt @ V.T) * s, x, atol=1e-12)
+
+
+
+# --------------------------------------------------------------------------
+# 3-bit codes (Sec. 5.2, Table tab:bitwidth): the lattice {0..7}^d
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("d", [1, 2, 4])
+def test_enumeration_moments_3bit(d):
+    pin_enumeration_moments(oracle.dequant, d, bits=3)
+
+
+def test_codebook_3bit_is_dequant_of_every_index():
+    """`codebook(A, B, bits=3)` row v is the dequantisation of the lattice
+    point whose coordinate c is bit-field [3c+2:3c] of v."""
+    for d in (1, 2, 4):
+        g = np.random.default_rng(30 + d)
+        A = g.standard_normal((d, d))
+        B = g.standard_normal(d)
+        v = np.arange(8 ** d)
+        pts = np.stack([(v >> (3 * c)) & 7 for c in range(d)], axis=1).astype(np.uint8)
+        cb = oracle.codebook(A, B, bits=3)
+        assert cb.shape == (8 ** d, d)
+        assert np.allclose(cb, oracle.dequant(pts, A, B), rtol=0, atol=1e-14 * np.abs(cb).max())
+
+
+def test_3bit_scalar_case_is_uniform_3bit_dequantisation():
+    """A = s I, B = -s zp 1 with codes 0..7: every weight is s (q - zp)."""
+    g = np.random.default_rng(7)
+    s_, zp = 0.03125, 3.5
+    codes = g.integers(0, 8, size=(5, 64), dtype=np.uint8)
+    W = oracle.dequant(codes, s_ * np.eye(2), -s_ * zp * np.ones(2))
+    assert np.array_equal(W, s_ * (codes.astype(np.float64) - zp))
