@@ -280,7 +280,7 @@ def run_ours(args, rank, world, local_rank):
         print(json.dumps({"prefill": run_prefill(torch, binding, peaks, args, side)}), flush=True)
         return
     if args.only == "decode":
-        args.no_e2e = args.no_cpu = args.no_prefill = args.no_grouped = args.no_rht = True
+        args.no_e2e = args.no_cpu = args.no_prefill = args.no_grouped = args.no_rht = args.no_bits3 = True
     shapes = synth.LLAMA2_7B
     stack = build_stack(binding, shapes, args.layers, 1)
 
@@ -468,6 +468,11 @@ def run_ours(args, rank, world, local_rank):
     if not args.no_grouped:
         grouped = run_grouped(torch, binding, peaks, args, side)
 
+    # ---- 3-bit codes --------------------------------------------------------
+    bits3 = None
+    if not args.no_bits3:
+        bits3 = run_bits3(torch, binding, peaks, args, side)
+
     # ---- inverse RHT around the layers -------------------------------------
     rht = None
     if not args.no_rht:
@@ -504,23 +509,19 @@ def run_ours(args, rank, world, local_rank):
         "prefill": prefill,
         "per_group_affine": grouped,
         "rht": rht,
+        "bits3": bits3,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
 
 
-def run_grouped(torch, binding, peaks, args, stream):
-    """The decode sweep on Llama-2-7B-shaped layers with one fp16 affine map
-    per (output row, 128-column group): the per-group GEMV (gemv_grouped_kernel),
-    algorithmic bytes counting the maps (N * K/128 * 12 bytes at d = 2)."""
+def sweep_variant(torch, binding, args, stream, base, kernel_id):
+    """The Llama-2-7B decode sweep (GROUPED_LAYERS layers: `base` and device
+    copies) for one layer variant; returns (GB/s over the sweep, per-M list,
+    launches per step). Bytes are the library's algorithmic bytes per call."""
     shapes = synth.LLAMA2_7B
-    base = []
-    for pi, (_, N, K) in enumerate(shapes):
-        codes, A, B = synth.layer_inputs_grouped(0, 1, 0, pi, N, K, 2)
-        base.append(binding.UniSVQLinear(codes, A, B, group_cols=128))
     stack = [base] + [[b.clone() for b in base] for _ in range(GROUPED_LAYERS - 1)]
-    xs = {}
-    ys = {}
+    xs, ys = {}, {}
     for M in M_SWEEP:
         for pi, (_, N, K) in enumerate(shapes):
             if (M, K) not in xs:
@@ -548,7 +549,7 @@ def run_grouped(torch, binding, peaks, args, stream):
         nbytes = 0
         for grp in GROUPS_7B:
             info = binding.query_group([base[i] for i in grp], M)
-            assert info["kernel"] == binding.KERNEL_GROUPED
+            assert info["kernel"] == kernel_id
             nbytes += info["algo_bytes"] * GROUPED_LAYERS
             launches += info["launches"] * GROUPED_LAYERS
         sweep_bytes.append(nbytes)
@@ -565,12 +566,39 @@ def run_grouped(torch, binding, peaks, args, stream):
     for layer in stack:
         for b in layer:
             b.close()
-    gbs = sum(sweep_bytes) * steps / t / 1e9
+    return sum(sweep_bytes) * steps / t / 1e9, per_m, launches
+
+
+def run_grouped(torch, binding, peaks, args, stream):
+    """The decode sweep on Llama-2-7B-shaped layers with one fp16 affine map
+    per (output row, 128-column group): the per-group GEMV (gemv_grouped_kernel),
+    algorithmic bytes counting the maps (N * K/128 * 12 bytes at d = 2)."""
+    base = []
+    for pi, (_, N, K) in enumerate(synth.LLAMA2_7B):
+        codes, A, B = synth.layer_inputs_grouped(0, 1, 0, pi, N, K, 2)
+        base.append(binding.UniSVQLinear(codes, A, B, group_cols=128))
+    gbs, per_m, launches = sweep_variant(torch, binding, args, stream, base, binding.KERNEL_GROUPED)
     return {"workload": f"Llama-2-7B-shaped projection set x {GROUPED_LAYERS} layers, decode sweep M in "
                         f"{list(M_SWEEP)}, 2-bit codes d=2, one fp16 affine per output row per 128-column group",
             "GB/s": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"], "sweep": per_m,
             "kernel": "gemv_grouped_kernel", "launches_per_step": launches,
             "bytes": "codes N*K/4 + maps N*ceil(K/128)*12 + x + y per call",
+            "timing": "CUDA graphs of the layer stack per M, CUDA events on the capture stream"}
+
+
+def run_bits3(torch, binding, peaks, args, stream):
+    """The decode sweep on Llama-2-7B-shaped layers with 3-bit codes (z in
+    0..7, Sec. 5.2): the GEMV with the high-bit plane (gemv_kernel, BITS = 3)."""
+    base = []
+    for pi, (_, N, K) in enumerate(synth.LLAMA2_7B):
+        codes, A, B = synth.layer_inputs_bits(0, 1, 0, pi, N, K, 2, 3)
+        base.append(binding.UniSVQLinear(codes, A, B, bits=3))
+    gbs, per_m, launches = sweep_variant(torch, binding, args, stream, base, binding.KERNEL_GEMV)
+    return {"workload": f"Llama-2-7B-shaped projection set x {GROUPED_LAYERS} layers, decode sweep M in "
+                        f"{list(M_SWEEP)}, 3-bit codes d=2, per-matrix fp16 affine",
+            "GB/s": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"], "sweep": per_m,
+            "kernel": "gemv_kernel (3-bit instance)", "launches_per_step": launches,
+            "bytes": "codes 3*N*K/8 + affine + x + y per call",
             "timing": "CUDA graphs of the layer stack per M, CUDA events on the capture stream"}
 
 
@@ -722,6 +750,7 @@ def main():
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-bits3", action="store_true", help="skip the 3-bit-code sweep")
     ap.add_argument("--no-rht", action="store_true",
                     help="skip the inverse-RHT sweep (Llama-3-8B shapes)")
     ap.add_argument("--no-grouped", action="store_true",

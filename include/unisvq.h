@@ -122,6 +122,22 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
                           int N, int K, int d, void* stream, unisvq_handle* out);
 
 /*
+ * As unisvq_pack for codes of `bits` bits: 2, or 3 (z in {0..7}, the 3-bit
+ * variant of Sec. 5.2: only the integer vectors widen, Eq. def:affine with
+ * b = 3). A 3-bit code z = z_lo + 4 z_hi keeps z_lo in the packed layout
+ * above and z_hi in a bit plane of Np*Kp/8 bytes: for the 16-byte chunk of
+ * unit u, lane 4g + t of tile (rb, kt), four little-endian halfwords at byte
+ * 2048 (rb Kp/128 + kt) + 256 u + 8 (4g + t); halfword i belongs to word i of
+ * the chunk and its bit 4b + s is bit 2 of the code at bits [8b+2s+1 : 8b+2s]
+ * of that word. 3-bit layers take d in {1, 2, 4} and run the GEMV
+ * (UNISVQ_KERNEL_GEMV, 32 tokens per launch) at every M; other forced kernels
+ * return UNSUPPORTED. Errors as unisvq_pack, plus UNSUPPORTED (bits, or
+ * bits = 3 with d = 8) and INVALID_ARG (a code >= 2^bits).
+ */
+unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
+                               int N, int K, int d, int bits, void* stream, unisvq_handle* out);
+
+/*
  * Pack a layer whose affine map varies per output row and per group of
  * `group_cols` input columns: W_hat[n, k] = sum_c A[n][g][r][c] z[n, k - r + c]
  * + B[n][g][r], g = k / group_cols, r = k mod d (Eq. def:unisvq applied with

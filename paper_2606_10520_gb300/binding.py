@@ -22,7 +22,7 @@ EXPORTS = [
     "unisvq_query", "unisvq_sync_status", "unisvq_destroy", "unisvq_clone",
     "unisvq_status_string", "unisvq_packed_code_bytes", "unisvq_pack_host", "unisvq_version",
     "unisvq_linear_group", "unisvq_linear_group_force", "unisvq_linear_noalloc", "unisvq_query_group",
-    "unisvq_pack_grouped", "unisvq_set_rht", "unisvq_hadamard",
+    "unisvq_pack_grouped", "unisvq_set_rht", "unisvq_hadamard", "unisvq_pack_bits",
 ]
 MAX_GROUP = 4
 
@@ -55,6 +55,7 @@ def load():
     vp, i, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
     lib.unisvq_pack.argtypes = [vp, vp, vp, i, i, i, vp, ctypes.POINTER(vp)]
     lib.unisvq_pack_grouped.argtypes = [vp, vp, vp, i, i, i, i, vp, ctypes.POINTER(vp)]
+    lib.unisvq_pack_bits.argtypes = [vp, vp, vp, i, i, i, i, vp, ctypes.POINTER(vp)]
     lib.unisvq_set_rht.argtypes = [vp, vp, vp, i, vp]
     lib.unisvq_hadamard.argtypes = [vp, vp, i, i, vp, i, vp]
     lib.unisvq_linear.argtypes = [vp, vp, vp, i, vp]
@@ -134,10 +135,11 @@ def sync_status(stream=None) -> int:
 class UniSVQLinear:
     """One packed UniSVQ linear layer resident on the current CUDA device."""
 
-    def __init__(self, codes: np.ndarray, A, B, stream=None, _handle=None, group_cols: int | None = None):
-        """One (A [d][d], B [d]) for the matrix (unisvq_pack), or, with
-        `group_cols`, one per (row, group of columns): A [N][G][d][d],
-        B [N][G][d] (unisvq_pack_grouped)."""
+    def __init__(self, codes: np.ndarray, A, B, stream=None, _handle=None, group_cols: int | None = None,
+                 bits: int = 2):
+        """One (A [d][d], B [d]) for the matrix (unisvq_pack; `bits` = 3 for
+        codes 0..7, unisvq_pack_bits), or, with `group_cols`, one per (row,
+        group of columns): A [N][G][d][d], B [N][G][d] (unisvq_pack_grouped)."""
         lib = load()
         if _handle is not None:
             self._h = _handle
@@ -149,8 +151,8 @@ class UniSVQLinear:
             N, K = codes.shape
             h = ctypes.c_void_p()
             if group_cols is None:
-                _check(lib.unisvq_pack(codes.ctypes.data, A16.ctypes.data, B16.ctypes.data, N, K, d,
-                                       _stream_ptr(stream), ctypes.byref(h)), "unisvq_pack")
+                _check(lib.unisvq_pack_bits(codes.ctypes.data, A16.ctypes.data, B16.ctypes.data, N, K, d, int(bits),
+                                            _stream_ptr(stream), ctypes.byref(h)), "unisvq_pack_bits")
             else:
                 G = -(-K // group_cols)
                 if A16.shape != (N, G, d, d) or B16.shape != (N, G, d):

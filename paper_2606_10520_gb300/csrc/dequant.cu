@@ -1,9 +1,10 @@
 // Test hook: W_hat [N][K] in fp32 from the packed device layout.
 //
 // Each thread unpacks the four words of one (row, half) -- 64 codes -- with
-// the same extraction helper the layer kernels use (layout.h), rebuilds the index
-// z0 | z1 << 2 | ... of every d-vector and reads the fp32 codeword
-// RN_fp32(A z + B) of Eq. (def:unisvq) from the handle's codebook.
+// the same extraction helper the layer kernels use (layout.h), adds the high
+// bits of 3-bit codes, rebuilds the index z0 | z1 << bits | ... of every
+// d-vector and reads the fp32 codeword RN_fp32(A z + B) of Eq. (def:unisvq)
+// from the handle's codebook.
 #include <cuda_fp16.h>
 
 #include "common.cuh"
@@ -13,8 +14,9 @@ namespace unisvq {
 namespace {
 
 __global__ void __launch_bounds__(256) dequant_kernel(const uint8_t* __restrict__ codes,
+                                                      const uint8_t* __restrict__ hi,
                                                       const float* __restrict__ lut, float* W,
-                                                      int N, int K, int KT, int d, int nchunks) {
+                                                      int N, int K, int KT, int d, int bits, int nchunks) {
   const int id = blockIdx.x * 256 + threadIdx.x;
   if (id >= nchunks) return;
   const int tile = id >> 8;               // 256 (row, half) pairs per tile
@@ -29,13 +31,19 @@ __global__ void __launch_bounds__(256) dequant_kernel(const uint8_t* __restrict_
 #pragma unroll
   for (int wi = 0; wi < 4; ++wi) {
     // The 16 codes of the word: z[4s + b] = column 4s + b (16 consecutive
-    // columns, so a d-vector, d <= 8, never leaves the word).
+    // columns, so a d-vector, d <= 8, never leaves the word). 3-bit codes add
+    // bit 4b + s of the word's halfword in the high-bit plane as bit 2.
+    uint32_t hw = 0;
+    if (bits == 3)
+      hw = *reinterpret_cast<const uint16_t*>(hi + static_cast<size_t>(tile) * (kTileBytes / 2) +
+                                              (r >> 4) * (kUnitBytes / 2) + ((r & 7) * 4 + wi) * 8 +
+                                              2 * (2 * h + ((r >> 3) & 1)));
     uint32_t z[16];
 #pragma unroll
     for (int s = 0; s < 4; ++s) {
       const uint32_t e = extract4(words[wi], s);   // columns 4s .. 4s+3 of the word
 #pragma unroll
-      for (int b = 0; b < 4; ++b) z[4 * s + b] = (e >> (8 * b)) & 3u;
+      for (int b = 0; b < 4; ++b) z[4 * s + b] = ((e >> (8 * b)) & 3u) | (((hw >> (4 * b + s)) & 1u) << 2);
     }
     const int k0 = kt * kTileCols + 64 * h + 16 * wi;
 #pragma unroll
@@ -44,7 +52,7 @@ __global__ void __launch_bounds__(256) dequant_kernel(const uint8_t* __restrict_
       if (k >= K) continue;
       const int v0 = j & ~(d - 1);              // first coordinate of this column's vector
       uint32_t idx = 0;
-      for (int c = 0; c < d; ++c) idx |= z[v0 + c] << (2 * c);
+      for (int c = 0; c < d; ++c) idx |= z[v0 + c] << (bits * c);
       W[static_cast<size_t>(row) * K + k] = lut[idx * d + (j & (d - 1))];
     }
   }
@@ -89,8 +97,8 @@ unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s) {
     return cudaGetLastError() == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
   }
   const int nchunks = (L->Np / kTileRows) * L->KT * 256;
-  dequant_kernel<<<(nchunks + 255) / 256, 256, 0, s>>>(L->codes, L->lut32, W, L->N, L->K, L->KT, L->d,
-                                                       nchunks);
+  dequant_kernel<<<(nchunks + 255) / 256, 256, 0, s>>>(L->codes, L->hi, L->lut32, W, L->N, L->K, L->KT, L->d,
+                                                       L->bits, nchunks);
   return cudaGetLastError() == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 

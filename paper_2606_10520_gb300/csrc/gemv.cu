@@ -56,6 +56,7 @@ constexpr size_t dyn_smem_max() { return kSmemPerSm - kSmemPerCtaReserved - stat
 template <int DV>
 struct GemvLayer {
   const uint8_t* codes;
+  const uint8_t* hi;   // high-bit plane of 3-bit codes (layout in internal.h), else null
   uint16_t* y;         // bf16 [M][N]
   int N, d;
   int rb0;             // first grid.y row block of this layer
@@ -166,7 +167,20 @@ __device__ __forceinline__ uint4 load_x8(const uint16_t* row, int k, int kend, b
   return make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
 }
 
-template <int NT, int DV>
+// Bit j of x -> bit 2j (x < 2^16).
+__device__ __forceinline__ uint32_t spread16(uint32_t x) {
+  x = (x | (x << 8)) & 0x00FF00FFu;
+  x = (x | (x << 4)) & 0x0F0F0F0Fu;
+  x = (x | (x << 2)) & 0x33333333u;
+  return (x | (x << 1)) & 0x55555555u;
+}
+
+// BITS = 3: codes z = z_lo + 4 z_hi; z_lo from the packed words as for 2-bit
+// codes, z_hi from the layer's bit plane, spread so that the high bit of the
+// code at bits [8b + 2s + 1 : 8b + 2s] lands on bit 8b + 2s + 2: the A
+// registers become (w & m) | (h & m') = z 4^s 2^-24, z <= 7, the same
+// subnormal scale as 2-bit codes, so the B fragments do not change.
+template <int NT, int DV, int BITS>
 __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constant__ GemvArgs<DV> a) {
   extern __shared__ __align__(16) uint8_t smem[];
   const uint32_t sbase = smem_u32(smem);
@@ -181,6 +195,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   for (int i = 1; i < kMaxGroup; ++i)
     if (i < a.nlayers && static_cast<int>(blockIdx.y) >= a.layer[i].rb0) li = i;
   const uint8_t* codes = nullptr;
+  const uint8_t* hiplane = nullptr;
   uint16_t* yout = nullptr;
   int N = 0, d = 1, rb = 0;
   float colnorm = 0.f, Areg[16], Bq[DV];
@@ -188,6 +203,7 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
   for (int i = 0; i < kMaxGroup; ++i) {
     if (i == li) {
       codes = a.layer[i].codes;
+      if constexpr (BITS == 3) hiplane = a.layer[i].hi;
       yout = a.layer[i].y;
       N = a.layer[i].N;
       d = a.layer[i].d;
@@ -247,6 +263,15 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
 #pragma unroll
   for (int s = 0; s < kGDepth; ++s)
     if (s < n_kt) cw[s] = ldg_stream_v4(cbase + static_cast<size_t>(s) * kTileBytes);
+  constexpr int kHiDepth = BITS == 3 ? kGDepth : 1;
+  uint2 hw[kHiDepth];   // high bits of the four words of cw (halfword per word)
+  const uint8_t* hbase = nullptr;
+  if constexpr (BITS == 3) {
+    hbase = hiplane + (static_cast<size_t>(rb) * a.KT + kt0) * (kTileBytes / 2) + warp * (kUnitBytes / 2) + lane * 8;
+#pragma unroll
+    for (int s = 0; s < kGDepth; ++s)
+      if (s < n_kt) hw[s] = ldg_v2(hbase + static_cast<size_t>(s) * (kTileBytes / 2));
+  }
   pdl_launch_dependents();
 
   pdl_wait();   // x may be the previous kernel's output
@@ -407,18 +432,38 @@ __global__ void __launch_bounds__(kGThreads, 2) gemv_kernel(const __grid_constan
         for (int h = 0; h < 2; ++h) {
           const uint32_t wa = h ? cw[s].z : cw[s].x, wb = h ? cw[s].w : cw[s].y;   // rows g, g + 8
           const uint32_t was = wa >> 8, wbs = wb >> 8;
+          uint32_t ha = 0, hb = 0, has = 0, hbs = 0;
+          if constexpr (BITS == 3) {
+            const uint32_t hwd = h ? hw[s].y : hw[s].x;   // words 2h (row g) and 2h + 1 (row g + 8)
+            const uint32_t sa = spread16(hwd & 0xFFFFu), sb = spread16(hwd >> 16);
+            ha = sa << 2;   // bytes 0 and 2 (bit 32 of byte 3 falls off; a0, a1 do not use it)
+            hb = sb << 2;
+            has = sa >> 6;  // bytes 1 and 3, moved down one byte as w >> 8
+            hbs = sb >> 6;
+          }
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             const uint32_t m = 0x00030003u << (2 * j);
+            uint32_t a0 = wa & m, a1 = wb & m, a2 = was & m, a3 = wbs & m;
+            if constexpr (BITS == 3) {
+              const uint32_t mh = 0x00040004u << (2 * j);
+              a0 |= ha & mh;
+              a1 |= hb & mh;
+              a2 |= has & mh;
+              a3 |= hbs & mh;
+            }
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
               const uint2 b = act[nt] ? *reinterpret_cast<const uint2*>(xl[nt] + koff + 128u * h + 8u * j)
                                       : make_uint2(0u, 0u);
-              mma_16816(acc[nt], wa & m, wb & m, was & m, wbs & m, b);
+              mma_16816(acc[nt], a0, a1, a2, a3, b);
             }
           }
         }
-        if (i + kGDepth < n_kt) cw[s] = ldg_stream_v4(cbase + static_cast<size_t>(i + kGDepth) * kTileBytes);
+        if (i + kGDepth < n_kt) {
+          cw[s] = ldg_stream_v4(cbase + static_cast<size_t>(i + kGDepth) * kTileBytes);
+          if constexpr (BITS == 3) hw[s] = ldg_v2(hbase + static_cast<size_t>(i + kGDepth) * (kTileBytes / 2));
+        }
       }
     }
   }
@@ -752,16 +797,16 @@ int group_dv(const unisvq_layer* const* Ls, int n) {
   return 4;
 }
 
-template <int NT, int DV>
+template <int NT, int DV, int BITS>
 unisvq_status gemv_launch_nt(const unisvq_layer* const* Ls, int n, const DecodePlan& p, const void* x,
                              void* const* ys, int m0, int M, cudaStream_t s) {
   static bool attr_set[64] = {};
   const int dev = Ls[0]->device;
   if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
   if (!attr_set[dev]) {
-    if (cudaFuncSetAttribute(gemv_kernel<NT, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(gemv_kernel<NT, DV, BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(dyn_smem_max<DV>())) != cudaSuccess ||
-        cudaFuncSetAttribute(gemv_kernel<NT, DV>, cudaFuncAttributePreferredSharedMemoryCarveout,
+        cudaFuncSetAttribute(gemv_kernel<NT, DV, BITS>, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared) != cudaSuccess)
       return UNISVQ_ERR_CUDA;
     attr_set[dev] = true;
@@ -783,6 +828,7 @@ unisvq_status gemv_launch_nt(const unisvq_layer* const* Ls, int n, const DecodeP
     const unisvq_layer* L = Ls[i];
     GemvLayer<DV>& g = a.layer[i];
     g.codes = L->codes;
+    g.hi = L->hi;
     g.y = static_cast<uint16_t*>(ys[i]) + static_cast<size_t>(m0) * L->N;
     g.N = L->N;
     g.d = L->d;
@@ -806,7 +852,7 @@ unisvq_status gemv_launch_nt(const unisvq_layer* const* Ls, int n, const DecodeP
   attrs[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attrs;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, gemv_kernel<NT, DV>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+  return cudaLaunchKernelEx(&cfg, gemv_kernel<NT, DV, BITS>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
 // Split K into ks <= 8 cluster CTAs for nb row blocks: the largest ks whose
@@ -913,6 +959,9 @@ unisvq_status launch_gemv_group(const unisvq_layer* const* Ls, int n, const void
   if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
   int nb = 0;
   for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
+  for (int i = 1; i < n; ++i)
+    if (Ls[i]->bits != Ls[0]->bits) return UNISVQ_ERR_UNSUPPORTED;
+  const bool bits3 = Ls[0]->bits == 3;   // d <= 4 (unisvq_pack_bits)
   const bool d8 = group_dv(Ls, n) == 8;
   const size_t sstat = d8 ? static_smem<8>() : static_smem<4>();
   const size_t cap = kSmemPerSm - kSmemPerCtaReserved - sstat;
@@ -927,14 +976,18 @@ unisvq_status launch_gemv_group(const unisvq_layer* const* Ls, int n, const void
     }
     if (p.smem > cap) return UNISVQ_ERR_UNSUPPORTED;
     unisvq_status st;
-    if (d8)
-      st = p.nt == 1   ? gemv_launch_nt<1, 8>(Ls, n, p, x, ys, m0, mc, s)
-           : p.nt == 2 ? gemv_launch_nt<2, 8>(Ls, n, p, x, ys, m0, mc, s)
-                       : gemv_launch_nt<4, 8>(Ls, n, p, x, ys, m0, mc, s);
+    if (bits3)
+      st = p.nt == 1   ? gemv_launch_nt<1, 4, 3>(Ls, n, p, x, ys, m0, mc, s)
+           : p.nt == 2 ? gemv_launch_nt<2, 4, 3>(Ls, n, p, x, ys, m0, mc, s)
+                       : gemv_launch_nt<4, 4, 3>(Ls, n, p, x, ys, m0, mc, s);
+    else if (d8)
+      st = p.nt == 1   ? gemv_launch_nt<1, 8, 2>(Ls, n, p, x, ys, m0, mc, s)
+           : p.nt == 2 ? gemv_launch_nt<2, 8, 2>(Ls, n, p, x, ys, m0, mc, s)
+                       : gemv_launch_nt<4, 8, 2>(Ls, n, p, x, ys, m0, mc, s);
     else
-      st = p.nt == 1   ? gemv_launch_nt<1, 4>(Ls, n, p, x, ys, m0, mc, s)
-           : p.nt == 2 ? gemv_launch_nt<2, 4>(Ls, n, p, x, ys, m0, mc, s)
-                       : gemv_launch_nt<4, 4>(Ls, n, p, x, ys, m0, mc, s);
+      st = p.nt == 1   ? gemv_launch_nt<1, 4, 2>(Ls, n, p, x, ys, m0, mc, s)
+           : p.nt == 2 ? gemv_launch_nt<2, 4, 2>(Ls, n, p, x, ys, m0, mc, s)
+                       : gemv_launch_nt<4, 4, 2>(Ls, n, p, x, ys, m0, mc, s);
     if (st != UNISVQ_OK) return st;
     m0 += mc;
   }
@@ -953,7 +1006,7 @@ bool rows_fit(int M, int KT, bool d8) {
 }
 }  // namespace
 
-bool gemv_rows_supported(const unisvq_layer* L, int M) { return rows_fit(M, L->KT, L->d == 8); }
+bool gemv_rows_supported(const unisvq_layer* L, int M) { return L->bits == 2 && rows_fit(M, L->KT, L->d == 8); }
 
 unisvq_status launch_gemv_rows_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
                                      cudaStream_t s) {

@@ -28,6 +28,11 @@ struct unisvq_layer {
   // Per-(row, 128-column group) affine maps (unisvq_pack_grouped): the codes
   // are packed with pack_codes_grouped_host and the maps live in `meta`;
   // A, B, lut32, tlut and fold_ws are unused (zero / null).
+  // Code width: 2, or 3 (unisvq_pack_bits). A 3-bit code z = z_lo + 4 z_hi
+  // keeps z_lo in `codes` and z_hi in the bit plane `hi` (hi_plane_offset).
+  int bits;
+  uint8_t* hi;             // device, Np*Kp/8 bytes (bits == 3), else null
+  size_t hi_bytes;
   int grouped;
   uint16_t* meta;          // device, fp16 [Np/128][KT][128][d*d + d]
   size_t meta_bytes;
@@ -108,6 +113,11 @@ DecodePlan plan_grouped(const unisvq_layer* L, int nb, int M, int* tokens_per_la
 
 // Host packer (pack.cpp).
 void pack_codes_host(const uint8_t* codes, int N, int K, uint8_t* packed);
+// High-bit plane of 3-bit codes: for the 16-byte chunk (unit u, lane 4g + t)
+// of tile (rb, kt), four halfwords at 2048 (rb KT + kt) + 256 u + 8 (4g + t);
+// halfword i belongs to word i of the chunk, and its bit 4b + s is bit 2 of
+// the code whose low bits sit at bits [8b + 2s + 1 : 8b + 2s] of that word.
+void pack_hi_plane_host(const uint8_t* codes, int N, int K, uint8_t* hi);
 // Same layout with the columns of every 128-column group permuted by
 // grouped_column (per-group layers), and their fp16 metadata.
 int grouped_column(int d, int h, int t, int s, int b);

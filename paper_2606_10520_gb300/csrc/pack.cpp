@@ -40,6 +40,35 @@ void pack_codes_host(const uint8_t* codes, int N, int K, uint8_t* packed) {
   }
 }
 
+void pack_hi_plane_host(const uint8_t* codes, int N, int K, uint8_t* hi) {
+  const int Np = round_up(N, kRowPad), Kp = round_up(K, kColPad);
+  const int RB = Np / kTileRows, KT = Kp / kTileCols;
+#pragma omp parallel for schedule(static)
+  for (int rb = 0; rb < RB; ++rb) {
+    for (int kt = 0; kt < KT; ++kt) {
+      uint8_t* tile = hi + (static_cast<size_t>(rb) * KT + kt) * (kTileBytes / 2);
+      for (int r = 0; r < kTileRows; ++r) {
+        const int row = rb * kTileRows + r;
+        const uint8_t* cr = row < N ? codes + static_cast<size_t>(row) * K : nullptr;
+        const int u = r >> 4, q = (r >> 3) & 1, g = r & 7;
+        for (int h = 0; h < 2; ++h)
+          for (int t = 0; t < 4; ++t) {
+            uint32_t hw = 0;
+            for (int s = 0; s < 4; ++s)
+              for (int b = 0; b < 4; ++b) {
+                const int k = kt * kTileCols + 64 * h + 16 * t + 4 * s + b;
+                const uint32_t z = (cr && k < K) ? cr[k] : 0u;
+                hw |= ((z >> 2) & 1u) << (4 * b + s);
+              }
+            uint8_t* dst = tile + u * (kUnitBytes / 2) + (4 * g + t) * 8 + 2 * (2 * h + q);
+            dst[0] = static_cast<uint8_t>(hw);
+            dst[1] = static_cast<uint8_t>(hw >> 8);
+          }
+      }
+    }
+  }
+}
+
 // Column, inside its 128-column group, whose code sits at packed position
 // (half h, quarter t, shift s, byte b) of a per-group layer: chunk q = 4h + s
 // holds coordinate c = q / (8/d) of vectors 16 (q mod 8/d) + 4t + e with

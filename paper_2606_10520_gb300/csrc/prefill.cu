@@ -423,7 +423,7 @@ int pick_bn(int M) { return M <= 64 ? 64 : (M <= 128 ? 128 : 256); }
 }  // namespace
 
 bool prefill_supported(const unisvq_layer* L, int M) {
-  return M > 0 && L->d <= 4 && (L->K % 8) == 0 && get_encode() != nullptr;
+  return M > 0 && L->d <= 4 && L->bits == 2 && (L->K % 8) == 0 && get_encode() != nullptr;
 }
 
 PrefillPlan plan_prefill(const unisvq_layer* L, int M) {

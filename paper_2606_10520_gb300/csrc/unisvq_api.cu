@@ -79,18 +79,26 @@ unisvq_status unisvq_pack_host(const uint8_t* codes, int N, int K, uint8_t* pack
 
 unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
                           int N, int K, int d, void* stream, unisvq_handle* out) {
+  return unisvq_pack_bits(codes, A_f16, B_f16, N, K, d, 2, stream, out);
+}
+
+unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
+                               int N, int K, int d, int bits, void* stream, unisvq_handle* out) {
   if (!out) return UNISVQ_ERR_INVALID_ARG;
   *out = nullptr;
   if (!codes || !A_f16 || !B_f16) return UNISVQ_ERR_INVALID_ARG;
   if (d != 1 && d != 2 && d != 4 && d != 8) return UNISVQ_ERR_UNSUPPORTED;
+  if (bits != 2 && bits != 3) return UNISVQ_ERR_UNSUPPORTED;
+  if (bits == 3 && d == 8) return UNISVQ_ERR_UNSUPPORTED;   // 8^8 codewords: no debug codebook
   if (N <= 0 || K <= 0 || K % d != 0) return UNISVQ_ERR_INVALID_ARG;
   if (static_cast<long long>(round_up(N, kRowPad)) * round_up(K, kColPad) >= (1ll << 40))
     return UNISVQ_ERR_UNSUPPORTED;
 
   const size_t total = static_cast<size_t>(N) * K;
   int bad = 0;
+  const int zmax = (1 << bits) - 1;
 #pragma omp parallel for reduction(| : bad) schedule(static)
-  for (long long i = 0; i < static_cast<long long>(total); ++i) bad |= codes[i] > 3;
+  for (long long i = 0; i < static_cast<long long>(total); ++i) bad |= codes[i] > zmax;
   if (bad) return UNISVQ_ERR_INVALID_ARG;
 
   double A[64], B[8];
@@ -108,6 +116,7 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
   L->N = N;
   L->K = K;
   L->d = d;
+  L->bits = bits;
   L->Np = round_up(N, kRowPad);
   L->Kp = round_up(K, kColPad);
   L->KT = L->Kp / kTileCols;
@@ -135,16 +144,17 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
   // Rounded up so the activation scale never underestimates |x A|.
   L->colnorm = static_cast<float>(colnorm) * (1.0f + 1e-6f);
 
-  // Codebook of Eq. (def:unisvq): entry v holds A z(v) + B, z_c(v) = (v >> 2c) & 3,
-  // exact in fp64 and rounded once (to fp32 here, to bf16 below).
-  const int E = 1 << (2 * d);
+  // Codebook of Eq. (def:unisvq): entry v holds A z(v) + B with z_c(v) the
+  // bit-field [bits (c+1) - 1 : bits c] of v, exact in fp64 and rounded once
+  // (to fp32 here, to bf16 below).
+  const int E = 1 << (bits * d);
   L->lut_entries = E;
   std::vector<double> cb(static_cast<size_t>(E) * d);
   std::vector<float> lut32(static_cast<size_t>(E) * d);
   for (int v = 0; v < E; ++v)
     for (int r = 0; r < d; ++r) {
       double w = B[r];
-      for (int c = 0; c < d; ++c) w += A[r * d + c] * static_cast<double>((v >> (2 * c)) & 3);
+      for (int c = 0; c < d; ++c) w += A[r * d + c] * static_cast<double>((v >> (bits * c)) & zmax);
       cb[static_cast<size_t>(v) * d + r] = w;
       lut32[static_cast<size_t>(v) * d + r] = static_cast<float>(w);
     }
@@ -155,7 +165,7 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
   //   such layers run the decode kernels at every M).
   auto bf = [](double w) { return static_cast<uint32_t>(f64_to_bf16_rne(w)); };
   std::vector<uint32_t> tlut;
-  if (d == 8) {
+  if (d == 8 || bits != 2) {   // the prefill GEMM takes 2-bit layers with d <= 4 only
     tlut.assign(1, 0u);
   } else if (d <= 2) {
     tlut.resize(16);
@@ -183,6 +193,17 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
     return UNISVQ_ERR_OOM;
   }
   pack_codes_host(codes, N, K, packed.data());
+  std::vector<uint8_t> hi;
+  if (bits == 3) {
+    L->hi_bytes = L->code_bytes / 2;
+    try {
+      hi.resize(L->hi_bytes);
+    } catch (...) {
+      delete L;
+      return UNISVQ_ERR_OOM;
+    }
+    pack_hi_plane_host(codes, N, K, hi.data());
+  }
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   L->fold_ws = nullptr;
@@ -193,6 +214,8 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
   if (e == cudaSuccess) e = cudaMalloc(&L->fold_ws, ws_bytes);
   if (e == cudaSuccess) e = cudaMemsetAsync(L->fold_ws, 0, ws_bytes, s);
   if (e == cudaSuccess) e = cudaMemcpyAsync(L->codes, packed.data(), L->code_bytes, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess && bits == 3) e = cudaMalloc(&L->hi, L->hi_bytes);
+  if (e == cudaSuccess && bits == 3) e = cudaMemcpyAsync(L->hi, hi.data(), L->hi_bytes, cudaMemcpyHostToDevice, s);
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(L->lut32, lut32.data(), lut32.size() * sizeof(float), cudaMemcpyHostToDevice, s);
   if (e == cudaSuccess)
@@ -201,6 +224,7 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
   if (e == cudaSuccess && !device_error_word()) e = cudaErrorUnknown;
   if (e != cudaSuccess) {
     cudaFree(L->codes);
+    cudaFree(L->hi);
     cudaFree(L->lut32);
     cudaFree(L->tlut);
     cudaFree(L->fold_ws);
@@ -242,6 +266,7 @@ unisvq_status unisvq_pack_grouped(const uint8_t* codes, const uint16_t* A_f16, c
   L->Np = round_up(N, kRowPad);
   L->Kp = round_up(K, kColPad);
   L->KT = L->Kp / kTileCols;
+  L->bits = 2;
   L->grouped = 1;
   if (cudaGetDevice(&L->device) != cudaSuccess ||
       cudaDeviceGetAttribute(&L->num_sms, cudaDevAttrMultiProcessorCount, L->device) != cudaSuccess) {
@@ -271,6 +296,7 @@ unisvq_status unisvq_pack_grouped(const uint8_t* codes, const uint16_t* A_f16, c
   if (e != cudaSuccess) {
     cudaFree(L->codes);
     cudaFree(L->meta);
+    cudaFree(L->hi);
     cudaFree(L->rht_signs);
     cudaFree(L->rht_x);
     delete L;
@@ -290,6 +316,7 @@ unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
   L->tlut = nullptr;
   L->fold_ws = nullptr;
   L->meta = nullptr;
+  L->hi = nullptr;
   L->rht_signs = nullptr;
   L->rht_x = nullptr;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -301,6 +328,7 @@ unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
     return e;
   };
   cudaError_t e = copy(reinterpret_cast<void**>(&L->codes), h->codes, h->code_bytes);
+  if (e == cudaSuccess) e = copy(reinterpret_cast<void**>(&L->hi), h->hi, h->hi_bytes);
   if (e == cudaSuccess && !h->grouped) {
     e = copy(reinterpret_cast<void**>(&L->lut32), h->lut32,
              static_cast<size_t>(h->lut_entries) * h->d * sizeof(float));
@@ -322,6 +350,7 @@ unisvq_status unisvq_clone(unisvq_handle h, void* stream, unisvq_handle* out) {
     cudaFree(L->tlut);
     cudaFree(L->fold_ws);
     cudaFree(L->meta);
+    cudaFree(L->hi);
     cudaFree(L->rht_signs);
     cudaFree(L->rht_x);
     delete L;
@@ -340,6 +369,7 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
   cudaError_t e5 = cudaFree(h->meta);
   cudaError_t e6 = cudaFree(h->rht_signs);
   cudaError_t e7 = cudaFree(h->rht_x);
+  cudaFree(h->hi);
   delete h;
   return (e1 == cudaSuccess && e2 == cudaSuccess && e3 == cudaSuccess && e4 == cudaSuccess && e5 == cudaSuccess &&
           e6 == cudaSuccess && e7 == cudaSuccess)
@@ -380,6 +410,11 @@ static unisvq_status check_io(unisvq_handle h, const void* x, void* y, int M) {
 // decode path with the library's static fold workspace.
 static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, void* y, int M, cudaStream_t s,
                                   bool noalloc) {
+  if (h->bits == 3) {   // 3-bit codes: the GEMV at every M (no workspace, so also for noalloc)
+    if (!noalloc && kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GEMV)
+      return kernel >= 0 && kernel <= UNISVQ_KERNEL_GROUPED ? UNISVQ_ERR_UNSUPPORTED : UNISVQ_ERR_INVALID_ARG;
+    return launch_gemv(h, x, y, M, s);
+  }
   if (noalloc) {
     if (h->grouped) {   // the per-group GEMV has no workspace
       const unisvq_layer* Ls[1] = {h};
@@ -572,6 +607,20 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
 // kernel allows it, else one per layer.
 static unisvq_status group_inner(const unisvq_handle* hs, int n, int kernel, const void* x, void* const* ys, int M,
                                  cudaStream_t s) {
+  int n3 = 0;
+  for (int i = 0; i < n; ++i) n3 += hs[i]->bits == 3 ? 1 : 0;
+  if (n3) {   // 3-bit layers: one GEMV launch when every layer is 3-bit, else layer by layer
+    if (n3 == n && (kernel == UNISVQ_KERNEL_AUTO || kernel == UNISVQ_KERNEL_DECODE || kernel == UNISVQ_KERNEL_GEMV)) {
+      const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
+      for (int i = 0; i < n; ++i) Ls[i] = hs[i];
+      return launch_gemv_group(Ls, n, x, ys, M, s);
+    }
+    for (int i = 0; i < n; ++i) {
+      const unisvq_status st = linear_inner(hs[i], kernel, x, ys[i], M, s, false);
+      if (st != UNISVQ_OK) return st;
+    }
+    return UNISVQ_OK;
+  }
   int ngrouped = 0;
   for (int i = 0; i < n; ++i) ngrouped += hs[i]->grouped ? 1 : 0;
   if (ngrouped) {   // all layers per-group with one d, run by the per-group GEMV
@@ -678,13 +727,14 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
   info->d = h->d;
   info->Np = h->Np;
   info->Kp = h->Kp;
-  info->code_bytes = static_cast<long long>(h->code_bytes);
+  info->code_bytes = static_cast<long long>(h->code_bytes + h->hi_bytes);
   info->meta_bytes = meta_bytes_of(h);
-  info->algo_bytes = static_cast<long long>(h->N) * h->K / 4 + info->meta_bytes +
+  info->algo_bytes = static_cast<long long>(h->N) * h->K * h->bits / 8 + info->meta_bytes +
                      2ll * M * h->K + 2ll * M * h->N;
   info->flops = 2.0 * M * static_cast<double>(h->N) * h->K;
   const unisvq_layer* Ls[1] = {h};
-  describe_launch(Ls, 1, h->grouped ? UNISVQ_KERNEL_GROUPED : auto_kernel(h, M > 0 ? M : 1), M, info);
+  describe_launch(Ls, 1, h->grouped ? UNISVQ_KERNEL_GROUPED : h->bits == 3 ? UNISVQ_KERNEL_GEMV : auto_kernel(h, M > 0 ? M : 1),
+                  M, info);
   if (h->rht) {   // an input and an output rotation per chunk of the rotated-activation buffer
     const int m = M > 0 ? M : 1;
     info->launches += 2 * ((m + h->rht_tokens - 1) / h->rht_tokens);
@@ -703,9 +753,9 @@ unisvq_status unisvq_query_group(const unisvq_handle* hs, int n, int M, unisvq_i
     const unisvq_layer* h = hs[i];
     info->N += h->N;
     info->Np += h->Np;
-    info->code_bytes += static_cast<long long>(h->code_bytes);
+    info->code_bytes += static_cast<long long>(h->code_bytes + h->hi_bytes);
     info->meta_bytes += meta_bytes_of(h);
-    info->algo_bytes += static_cast<long long>(h->N) * h->K / 4 + 2ll * M * h->N;
+    info->algo_bytes += static_cast<long long>(h->N) * h->K * h->bits / 8 + 2ll * M * h->N;
     info->flops += 2.0 * M * static_cast<double>(h->N) * h->K;
     weights += static_cast<long long>(h->N) * h->K;
     nb += h->Np / kTileRows;
@@ -716,6 +766,7 @@ unisvq_status unisvq_query_group(const unisvq_handle* hs, int n, int M, unisvq_i
   info->algo_bytes += info->meta_bytes + 2ll * M * hs[0]->K;   // x is read once per call
   const int m = M > 0 ? M : 1;
   const int kernel = hs[0]->grouped ? UNISVQ_KERNEL_GROUPED
+                     : hs[0]->bits == 3 ? UNISVQ_KERNEL_GEMV
                      : m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL
                                                              : decode_kernel_for(weights, nb, m);
   const unisvq_layer* Ls[UNISVQ_MAX_GROUP];

@@ -120,6 +120,28 @@ def layer_inputs_grouped(seed: int, config: int, layer: int, proj: int, N: int, 
     return codes, A, B
 
 
+# 3-bit codes: a unit Gaussian weight on the grid of Eq. (def:affine) with
+# b = 3 (step s = sqrt(12/63), centre 3.5), probability of each of 0..7.
+_Z3 = np.arange(8) - 3.5
+_P3 = np.exp(-0.5 * (_Z3 * np.sqrt(12.0 / 63.0)) ** 2)
+CODE_PROBS_3BIT = tuple(_P3 / _P3.sum())
+
+
+def layer_inputs_bits(seed: int, config: int, layer: int, proj: int, N: int, K: int, d: int, bits: int):
+    """(codes, A, B) with codes of `bits` bits: 2 as `layer_inputs`; 3 draws
+    codes i.i.d. from CODE_PROBS_3BIT and centres B at (2^3 - 1)/2 = 3.5 steps."""
+    if bits == 2:
+        return layer_inputs(seed, config, layer, proj, N, K, d)
+    gc = rng(seed, config, layer, proj, 5)
+    ga = rng(seed, config, layer, proj, 6)
+    codes = gc.choice(8, size=(N, K), p=CODE_PROBS_3BIT).astype(np.uint8)
+    s = abs(ga.normal(0.02, 0.005)) / 2.0
+    G = ga.standard_normal((d, d))
+    A = (s * (np.eye(d) + 0.1 * G)).astype(np.float16)
+    B = np.full((d,), -3.5 * s).astype(np.float16)
+    return codes, A, B
+
+
 def activations(seed: int, config: int, stream: int, M: int, K: int) -> np.ndarray:
     """bf16 bits [M][K] for one activation stream of a synthetic config."""
     return gen_activations(rng(seed, config, stream, 3), M, K, seed=seed)

@@ -158,3 +158,23 @@ def test_pack_grouped_rejects_bad_arguments_before_touching_the_gpu(lib):
     Bnan = B.copy()
     Bnan[0, 0, 1] = np.array([np.nan], dtype=np.float16).view(np.uint16)[0]
     assert _pack_grouped_status(lib, codes, A, Bnan, N, K, d, 128) == binding.ERR_INVALID_ARG
+
+
+def test_pack_bits_rejects_bad_widths_and_codes(lib):
+    from paper_2606_10520_gb300 import binding
+    codes = np.zeros((4, 16), dtype=np.uint8)
+    A = np.eye(2, dtype=np.float16).view(np.uint16)
+    B = np.zeros(2, dtype=np.float16).view(np.uint16)
+    A8 = np.eye(8, dtype=np.float16).view(np.uint16)
+    B8 = np.zeros(8, dtype=np.float16).view(np.uint16)
+    h = ctypes.c_void_p()
+    st = lambda c, a, b, d, bits: lib.unisvq_pack_bits(c.ctypes.data, a.ctypes.data, b.ctypes.data, 4, 16, d, bits,
+                                                        None, ctypes.byref(h))
+    assert st(codes, A, B, 2, 4) == binding.ERR_UNSUPPORTED
+    assert st(codes, A, B, 2, 1) == binding.ERR_UNSUPPORTED
+    assert st(codes, A8, B8, 8, 3) == binding.ERR_UNSUPPORTED      # 8^8 codewords
+    bad = codes.copy()
+    bad[1, 5] = 8
+    assert st(bad, A, B, 2, 3) == binding.ERR_INVALID_ARG          # code >= 2^3
+    bad[1, 5] = 4
+    assert st(bad, A, B, 2, 2) == binding.ERR_INVALID_ARG          # code >= 2^2
