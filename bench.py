@@ -194,6 +194,23 @@ def oracle_sample(budget_s: float):
 # ---------------------------------------------------------------------------
 # reference arm: the oracle on the host cores
 # ---------------------------------------------------------------------------
+def max_over_ranks(values, world, device):
+    """Element-wise maximum of per-rank floats over the process group (every
+    rank receives it); the identity for one rank."""
+    if world <= 1:
+        return [float(v) for v in values]
+    import torch
+    import torch.distributed as dist
+    tt = torch.tensor([float(v) for v in values], device=device, dtype=torch.float64)
+    dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+    return [float(v) for v in tt.tolist()]
+
+
+def whole_job_gbs(bytes_per_step_per_rank, steps, world, t_max):
+    """Whole-job throughput: every rank's bytes over the slowest rank's time."""
+    return bytes_per_step_per_rank * steps * world / t_max / 1e9
+
+
 def run_reference(args, rank, world):
     if rank != 0:
         return
@@ -356,15 +373,11 @@ def run_ours(args, rank, world, local_rank):
     time.sleep(0.3)
     t = time_graphs(torch, graphs, args.steps, args.warmup, side)
     clocks = clk.stop()
-    if world > 1:
-        tt = torch.tensor([t], device="cuda", dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t = float(tt.item())
+    t = max_over_ranks([t], world, "cuda")[0]
     st = binding.sync_status(side)
     if st != 0:
         raise RuntimeError(f"device status {binding.status_string(st)}")
-    total_bytes = step_bytes * args.steps * world
-    value = total_bytes / t / 1e9
+    value = whole_job_gbs(step_bytes, args.steps, world, t)
     per_rank = step_bytes * args.steps / t / 1e9
 
     # per-kernel-class timing: graphs holding only the calls that run that
@@ -390,11 +403,9 @@ def run_ours(args, rank, world, local_rank):
                 kpass()
             kgraphs.append(kg)
         kind_time[kid] = time_graphs(torch, kgraphs, args.steps, args.warmup, side)
-    if world > 1:
-        for kid in sorted(kind_time):
-            tt = torch.tensor([kind_time[kid]], device="cuda", dtype=torch.float64)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            kind_time[kid] = float(tt.item())
+    kids = sorted(kind_time)
+    for kid, tk in zip(kids, max_over_ranks([kind_time[k] for k in kids], world, "cuda")):
+        kind_time[kid] = tk
 
     def roofline_for(kid):
         name = KERNEL_NAMES.get(kid, "?")
@@ -458,7 +469,8 @@ def run_ours(args, rank, world, local_rank):
                 for i in grp:
                     d2h += 2 * M * shapes[i][1] * args.layers
         te = time_graphs(torch, egraphs, args.steps, args.warmup, side)
-        e2e = {"value": step_bytes * args.steps * world / te / 1e9, "unit": "GB/s",
+        te = max_over_ranks([te], world, "cuda")[0]
+        e2e = {"value": whole_job_gbs(step_bytes, args.steps, world, te), "unit": "GB/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "how": "per call: pinned-host x -> device copy, the library call, device -> pinned-host y "
                       "of every projection; the whole sweep replayed from CUDA graphs"}

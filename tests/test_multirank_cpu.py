@@ -1,0 +1,69 @@
+"""The multi-rank paths of bench.py on CPU: two gloo ranks reduce their step
+times to the maximum and report whole-job throughput; the reference arm runs
+on rank 0 only. (On the GPU machine every rank is an independent replica: the
+data path has no collective.)"""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+torch = pytest.importorskip("torch")
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, out_dir):
+    import torch.distributed as dist
+    sys.path.insert(0, ROOT)
+    import bench
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        times = [0.5 + rank, 2.0 - rank]          # rank 0: (0.5, 2.0); rank 1: (1.5, 1.0)
+        got = bench.max_over_ranks(times, world, "cpu")
+        value = bench.whole_job_gbs(3e9, 10, world, got[0])
+        with open(os.path.join(out_dir, f"r{rank}.json"), "w") as f:
+            json.dump({"max": got, "value": value}, f)
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_take_the_slowest_time(tmp_path):
+    import torch.multiprocessing as mp
+    port = _free_port()
+    mp.spawn(_rank_main, args=(2, port, str(tmp_path)), nprocs=2, join=True)
+    for r in range(2):
+        res = json.load(open(tmp_path / f"r{r}.json"))
+        assert res["max"] == [1.5, 2.0]
+        assert res["value"] == pytest.approx(3e9 * 10 * 2 / 1.5 / 1e9)
+
+
+def test_single_rank_is_the_identity():
+    sys.path.insert(0, ROOT)
+    import bench
+    assert bench.max_over_ranks([0.25, 4.0], 1, "cpu") == [0.25, 4.0]
+    assert bench.whole_job_gbs(1e9, 2, 1, 0.5) == pytest.approx(4.0)
+
+
+@pytest.mark.parametrize("rank", [0, 1])
+def test_reference_arm_prints_on_rank_zero_only(rank):
+    env = dict(os.environ, RANK=str(rank), WORLD_SIZE="2", LOCAL_RANK=str(rank))
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--gpus", "2",
+                        "--steps", "1", "--warmup", "3"], capture_output=True, text=True, env=env, timeout=300)
+    assert r.returncode == 0, r.stderr
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    if rank == 0:
+        line = json.loads(lines[-1])
+        assert line["impl"] == "reference" and line["n_gpus"] == 2 and line["value"] > 0
+        assert line["cpu_baseline"]["kind"] == "oracle" and line["e2e"]["h2d_bytes_per_step"] == 0
+    else:
+        assert not lines
