@@ -63,6 +63,12 @@ def algo_bytes(N, K, M, d=2):
 KERNEL_NAMES = {1: "decode", 2: "prefill_kernel", 3: "gemv_kernel", 4: "decode_kernel", 5: "gemv_rows_kernel",
                 6: "gemv_grouped_kernel"}
 GROUPED_LAYERS = 16   # 16 x 69.6 MB of codes + per-group maps: larger than L2
+
+
+def variant_layers(args):
+    """Layers of the secondary sweeps: 16, or --layers when one of them runs
+    alone (--only grouped / rht / bits3, a profiling aid)."""
+    return args.layers if args.only in ("grouped", "rht", "bits3") else GROUPED_LAYERS
 # Sources whose change invalidates a committed ncu traffic figure, per kernel.
 KERNEL_SOURCES = {
     "gemv_kernel": ("paper_2606_10520_gb300/csrc/gemv.cu", "paper_2606_10520_gb300/csrc/common.cuh",
@@ -295,6 +301,11 @@ def run_ours(args, rank, world, local_rank):
     if args.only == "prefill":
         side = torch.cuda.Stream()
         print(json.dumps({"prefill": run_prefill(torch, binding, peaks, args, side)}), flush=True)
+        return
+    variants = {"grouped": ("per_group_affine", run_grouped), "rht": ("rht", run_rht), "bits3": ("bits3", run_bits3)}
+    if args.only in variants:
+        key, fn = variants[args.only]
+        print(json.dumps({key: fn(torch, binding, peaks, args, torch.cuda.Stream())}), flush=True)
         return
     if args.only == "decode":
         args.no_e2e = args.no_cpu = args.no_prefill = args.no_grouped = args.no_rht = args.no_bits3 = True
@@ -532,7 +543,8 @@ def sweep_variant(torch, binding, args, stream, base, kernel_id):
     copies) for one layer variant; returns (GB/s over the sweep, per-M list,
     launches per step). Bytes are the library's algorithmic bytes per call."""
     shapes = synth.LLAMA2_7B
-    stack = [base] + [[b.clone() for b in base] for _ in range(GROUPED_LAYERS - 1)]
+    nl = variant_layers(args)
+    stack = [base] + [[b.clone() for b in base] for _ in range(nl - 1)]
     xs, ys = {}, {}
     for M in M_SWEEP:
         for pi, (_, N, K) in enumerate(shapes):
@@ -562,8 +574,8 @@ def sweep_variant(torch, binding, args, stream, base, kernel_id):
         for grp in GROUPS_7B:
             info = binding.query_group([base[i] for i in grp], M)
             assert info["kernel"] == kernel_id
-            nbytes += info["algo_bytes"] * GROUPED_LAYERS
-            launches += info["launches"] * GROUPED_LAYERS
+            nbytes += info["algo_bytes"] * nl
+            launches += info["launches"] * nl
         sweep_bytes.append(nbytes)
     st = binding.sync_status(stream)
     if st != 0:
@@ -574,7 +586,7 @@ def sweep_variant(torch, binding, args, stream, base, kernel_id):
     for M, g, nb in zip(M_SWEEP, graphs, sweep_bytes):
         tm = time_graphs(torch, [g], steps, 2, stream)
         per_m.append({"M": M, "GB/s": round(nb * steps / tm / 1e9, 1),
-                      "us_per_layer": round(tm / steps / GROUPED_LAYERS * 1e6, 3)})
+                      "us_per_layer": round(tm / steps / nl * 1e6, 3)})
     for layer in stack:
         for b in layer:
             b.close()
@@ -590,7 +602,7 @@ def run_grouped(torch, binding, peaks, args, stream):
         codes, A, B = synth.layer_inputs_grouped(0, 1, 0, pi, N, K, 2)
         base.append(binding.UniSVQLinear(codes, A, B, group_cols=128))
     gbs, per_m, launches = sweep_variant(torch, binding, args, stream, base, binding.KERNEL_GROUPED)
-    return {"workload": f"Llama-2-7B-shaped projection set x {GROUPED_LAYERS} layers, decode sweep M in "
+    return {"workload": f"Llama-2-7B-shaped projection set x {variant_layers(args)} layers, decode sweep M in "
                         f"{list(M_SWEEP)}, 2-bit codes d=2, one fp16 affine per output row per 128-column group",
             "GB/s": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"], "sweep": per_m,
             "kernel": "gemv_grouped_kernel", "launches_per_step": launches,
@@ -606,7 +618,7 @@ def run_bits3(torch, binding, peaks, args, stream):
         codes, A, B = synth.layer_inputs_bits(0, 1, 0, pi, N, K, 2, 3)
         base.append(binding.UniSVQLinear(codes, A, B, bits=3))
     gbs, per_m, launches = sweep_variant(torch, binding, args, stream, base, binding.KERNEL_GEMV)
-    return {"workload": f"Llama-2-7B-shaped projection set x {GROUPED_LAYERS} layers, decode sweep M in "
+    return {"workload": f"Llama-2-7B-shaped projection set x {variant_layers(args)} layers, decode sweep M in "
                         f"{list(M_SWEEP)}, 3-bit codes d=2, per-matrix fp16 affine",
             "GB/s": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"], "sweep": per_m,
             "kernel": "gemv_kernel (3-bit instance)", "launches_per_step": launches,
@@ -628,7 +640,8 @@ def run_rht(torch, binding, peaks, args, stream):
         base.append(binding.UniSVQLinear(codes, A, B))
     s_in = {K: g.choice([-1.0, 1.0], K) for K in sorted({K for _, _, K in shapes})}
     s_out = [g.choice([-1.0, 1.0], N) for _, N, _ in shapes]
-    stack = [base] + [[b.clone() for b in base] for _ in range(GROUPED_LAYERS - 1)]
+    nl = variant_layers(args)
+    stack = [base] + [[b.clone() for b in base] for _ in range(nl - 1)]
     xs, ys = {}, {}
     for M in M_SWEEP:
         for pi, (_, N, K) in enumerate(shapes):
@@ -636,7 +649,7 @@ def run_rht(torch, binding, peaks, args, stream):
                 xb = synth.activations(0, 2, 100 + M, M, K)
                 xs[(M, K)] = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).cuda()
             ys[(M, pi)] = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
-    step_bytes = sum(algo_bytes(N, K, M) for M in M_SWEEP for _, N, K in shapes) * GROUPED_LAYERS
+    step_bytes = sum(algo_bytes(N, K, M) for M in M_SWEEP for _, N, K in shapes) * nl
     steps = max(5, args.steps // 4)
     out = {}
     for rht in (False, True):
@@ -672,7 +685,7 @@ def run_rht(torch, binding, peaks, args, stream):
     for layer in stack:
         for b in layer:
             b.close()
-    return {"workload": f"Llama-3-8B-shaped projection set x {GROUPED_LAYERS} layers, decode sweep M in "
+    return {"workload": f"Llama-3-8B-shaped projection set x {nl} layers, decode sweep M in "
                         f"{list(M_SWEEP)}, d=2, per-matrix fp16 affine, inverse RHT around every layer",
             "GB/s": out["with_rht"], "GB/s_without_rht": out["without_rht"],
             "frac_of_measured_hbm": out["with_rht"] / peaks["hbm_gbs"],
@@ -770,8 +783,9 @@ def main():
     ap.add_argument("--ungrouped", action="store_true",
                     help="one unisvq_linear call per projection instead of grouped calls for q/k/v and gate/up")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
-    ap.add_argument("--only", choices=["decode", "prefill"], default=None,
-                    help="profiling aid: run only the decode sweep (no e2e/cpu/prefill) or only the prefill set")
+    ap.add_argument("--only", choices=["decode", "prefill", "grouped", "rht", "bits3"], default=None,
+                    help="profiling aid: run only the decode sweep (no e2e/cpu/secondary sweeps), only the "
+                         "prefill set, or only one secondary sweep (with --layers layers)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
