@@ -12,10 +12,13 @@
 //   warp 1        MMA issuer (one thread): 4 x tcgen05.mma (K = 16) per k-block
 //   warps 2..9    converters: one 16-row unit per warp, two rows x 16 columns
 //                 per lane; every d-vector index selects its exact bf16
-//                 codeword RN(A z + B) from a pack-time table
+//                 codeword RN(A z + B) from a pack-time table (per-matrix
+//                 maps), or from a table of the row's map that the warp
+//                 builds for every 128-column group (per-group maps, d = 2)
 //   warps 10..13  epilogue: tcgen05.ld of the accumulator, bf16, global store
 // The accumulator is double-buffered in TMEM so the epilogue of one tile runs
 // under the main loop of the next.
+#include <cuda_fp16.h>
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
@@ -34,6 +37,7 @@ constexpr int kEpiWarp0 = 10;
 struct PrefillArgs {
   const uint8_t* codes;
   const uint32_t* lut;   // d <= 2: 16 x bf16x2 pair codewords; d == 4: 256 x 4 bf16
+  const uint16_t* meta;  // per-group layers (d = 2): fp16 [Np/128][KT][128][6] (A row-major, B), else null
   uint16_t* y;
   int M, N, K, KT, d;
   int nkb;               // k-blocks of 64 columns: ceil(K / 64)
@@ -48,7 +52,8 @@ struct PfCfg {
   static constexpr int kOffA = 0;
   static constexpr int kOffB = STAGES * kATileBytes;
   static constexpr int kOffLut = STAGES * kStageBytes;            // 2 KB
-  static constexpr int kOffBars = kOffLut + 2048;
+  static constexpr int kOffGrp = kOffLut + 2048;                   // 8 x 1 KB: per-group tables
+  static constexpr int kOffBars = kOffGrp + 8 * 1024;
   // bars: bfull[S], afull[S], empty[S], accfull[2], accempty[2]
   static constexpr int kOffTmemPtr = kOffBars + (3 * STAGES + 5) * 8;   // + drain barrier
   static constexpr int kOffFlag = kOffTmemPtr + 8;
@@ -144,6 +149,15 @@ __device__ __forceinline__ uint32_t lds32(uint32_t addr) {
   asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(addr));
   return v;
 }
+__device__ __forceinline__ void sts32(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared.b32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+__device__ __forceinline__ float half_lo_f(uint32_t v) {
+  return __half2float(__ushort_as_half(static_cast<unsigned short>(v & 0xFFFFu)));
+}
+__device__ __forceinline__ float half_hi_f(uint32_t v) {
+  return __half2float(__ushort_as_half(static_cast<unsigned short>(v >> 16)));
+}
 __device__ __forceinline__ uint2 lds64(uint32_t addr) {
   uint2 v;
   asm volatile("ld.shared.v2.b32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
@@ -187,8 +201,9 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     fence_mbar_init();
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmap_x)) : "memory");
   }
-  // Codeword table -> shared memory.
-  {
+  // Codeword table -> shared memory (per-matrix maps only; per-group layers
+  // build theirs in the converters).
+  if (!a.meta) {
     const int words = a.d == 4 ? 512 : 16;
     uint32_t* lut_s = reinterpret_cast<uint32_t*>(smem + C::kOffLut);
     for (int i = threadIdx.x; i < words; i += kPfThreads) lut_s[i] = a.lut[i];
@@ -269,6 +284,93 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     const int r0 = 16 * c + g, r1 = r0 + 8;
     const uint32_t lut_s = sbase + C::kOffLut;
     int it = 0;
+    if (a.meta) {
+      // Per-(row, 128-column group) maps, d = 2, codes permuted within each group
+      // (pack_codes_grouped_host): coordinate c of vector v = 16 s + 4 t + e(b)
+      // sits in the word of half c at shift s and byte b. The A tile keeps the
+      // natural column order, so lane t writes the chunks t and t + 4 of a stage:
+      // natural columns 64 h + 8 cc + j are vector 32 h + 4 cc + j/2 (quarter t,
+      // shift 2h + cc/4, byte e(j/2)), coordinate j mod 2 -- all in the lane's own
+      // 16-byte load. Per k-tile the warp builds, for each of its 16 rows, the 16
+      // bf16 pairs RN(A z + B) of the row's map (four entries per lane and row).
+      const uint32_t tab_s = sbase + C::kOffGrp + c * 1024;   // [16 rows][16 entries] bf16x2
+      for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
+        const int n_blk = tile / a.mtiles;
+        const uint8_t* rbase = a.codes + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
+        const uint16_t* mbase = a.meta + static_cast<size_t>(n_blk) * a.KT * kBM * 6;
+        const int nkt = (a.nkb + 1) >> 1;
+        auto load_codes = [&](int kt) -> uint4 {
+          return kt < nkt ? __ldg(reinterpret_cast<const uint4*>(rbase + static_cast<size_t>(kt) * kTileBytes))
+                          : make_uint4(0, 0, 0, 0);
+        };
+        // the six fp16 of a row's map, as three words
+        auto load_map = [&](int kt, int row) -> uint3 {
+          if (kt >= nkt) return make_uint3(0, 0, 0);
+          const uint32_t* m = reinterpret_cast<const uint32_t*>(mbase + (static_cast<size_t>(kt) * kBM + row) * 6);
+          return make_uint3(__ldg(m), __ldg(m + 1), __ldg(m + 2));
+        };
+        uint4 cn = load_codes(0), cur = cn;
+        uint3 mn0 = load_map(0, r0), mn1 = load_map(0, r1);
+        bool ok = !*abort_flag;
+        for (int kb = 0; kb < a.nkb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const int hs = kb & 1;
+          if (hs == 0) {
+            cur = cn;
+            const uint3 m0 = mn0, m1 = mn1;
+            cn = load_codes((kb >> 1) + 1);
+            mn0 = load_map((kb >> 1) + 1, r0);
+            mn1 = load_map((kb >> 1) + 1, r1);
+            __syncwarp();   // every lane is done with the previous group's table
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const uint3 m = q ? m1 : m0;
+              const float a00 = half_lo_f(m.x), a01 = half_hi_f(m.x), a10 = half_lo_f(m.y), a11 = half_hi_f(m.y);
+              const float b0 = half_lo_f(m.z), b1 = half_hi_f(m.z);
+              const int rr = g + 8 * q;
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const int idx = 4 * t + k;
+                const float z0 = static_cast<float>(idx & 3), z1 = static_cast<float>(idx >> 2);
+                const float w0 = fmaf(a00, z0, fmaf(a01, z1, b0));
+                const float w1 = fmaf(a10, z0, fmaf(a11, z1, b1));
+                sts32(tab_s + (rr * 16 + idx) * 4, pack_bf16x2(w0, w1));
+              }
+            }
+            __syncwarp();
+          }
+          if (ok && it >= STAGES) {
+            ok = !*abort_flag && mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty);
+            if (!ok) *abort_flag = 1;
+          }
+          if (ok) {
+            const uint32_t tile_addr = sbase + C::kOffA + s * kATileBytes;
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const uint32_t wh0 = q ? cur.y : cur.x, wh1 = q ? cur.w : cur.z;   // halves 0 and 1 of the row
+              const uint32_t row_addr = tile_addr + (q ? r1 : r0) * 128;
+              const uint32_t trow = tab_s + (g + 8 * q) * 64;
+#pragma unroll
+              for (int u = 0; u < 2; ++u) {
+                const int cc = t + 4 * u;
+                const int sh = 2 * (2 * hs + u);   // 2 s
+                uint32_t o[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  const int bsh = 8 * ((e >> 1) | ((e & 1) << 1)) + sh;
+                  const uint32_t idx = ((wh0 >> bsh) & 3u) | (((wh1 >> bsh) & 3u) << 2);
+                  o[e] = lds32(trow + idx * 4);
+                }
+                sts128(row_addr + ((cc ^ g) << 4), o[0], o[1], o[2], o[3]);
+              }
+            }
+            fence_proxy_async_smem();
+          }
+          __syncwarp();
+          if (lane == 0 && ok) mbar_arrive(afull(s));
+        }
+      }
+    } else
     for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
       const int n_blk = tile / a.mtiles;
       const uint8_t* rbase = a.codes + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
@@ -404,6 +506,7 @@ unisvq_status launch_bn(const unisvq_layer* L, const PrefillPlan& p, const void*
   PrefillArgs a{};
   a.codes = L->codes;
   a.lut = L->tlut;
+  a.meta = L->grouped ? L->meta : nullptr;
   a.y = static_cast<uint16_t*>(y);
   a.M = M;
   a.N = L->N;
@@ -423,7 +526,9 @@ int pick_bn(int M) { return M <= 64 ? 64 : (M <= 128 ? 128 : 256); }
 }  // namespace
 
 bool prefill_supported(const unisvq_layer* L, int M) {
-  return M > 0 && L->d <= 4 && L->bits == 2 && (L->K % 8) == 0 && get_encode() != nullptr;
+  // per-group layers: d = 2 (the converters build a 16-pair table per row and group)
+  const bool maps_ok = L->grouped ? L->d == 2 : L->d <= 4;
+  return M > 0 && maps_ok && L->bits == 2 && (L->K % 8) == 0 && get_encode() != nullptr;
 }
 
 PrefillPlan plan_prefill(const unisvq_layer* L, int M) {

@@ -423,7 +423,9 @@ static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, vo
     }
     return launch_skinny_static(h, x, y, M, s);
   }
-  if (h->grouped) {
+  if (h->grouped) {   // per-group maps: the prefill GEMM (d = 2) for M > 64, else the per-group GEMV
+    if ((kernel == UNISVQ_KERNEL_AUTO && M > 64 && prefill_supported(h, M)) || kernel == UNISVQ_KERNEL_PREFILL)
+      return prefill_supported(h, M) ? launch_prefill(h, x, y, M, s) : UNISVQ_ERR_UNSUPPORTED;
     if (kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GROUPED)
       return kernel >= 0 && kernel <= UNISVQ_KERNEL_GROUPED ? UNISVQ_ERR_UNSUPPORTED : UNISVQ_ERR_INVALID_ARG;
     const unisvq_layer* Ls[1] = {h};
@@ -625,6 +627,15 @@ static unisvq_status group_inner(const unisvq_handle* hs, int n, int kernel, con
   for (int i = 0; i < n; ++i) ngrouped += hs[i]->grouped ? 1 : 0;
   if (ngrouped) {   // all layers per-group with one d, run by the per-group GEMV
     if (ngrouped != n) return UNISVQ_ERR_UNSUPPORTED;
+    bool pf = kernel == UNISVQ_KERNEL_PREFILL || (kernel == UNISVQ_KERNEL_AUTO && M > 64);
+    for (int i = 0; i < n && pf; ++i) pf = prefill_supported(hs[i], M);
+    if (pf || kernel == UNISVQ_KERNEL_PREFILL) {   // the prefill GEMM, layer by layer
+      for (int i = 0; i < n; ++i) {
+        const unisvq_status st = linear_inner(hs[i], kernel, x, ys[i], M, s, false);
+        if (st != UNISVQ_OK) return st;
+      }
+      return UNISVQ_OK;
+    }
     if (kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GROUPED)
       return UNISVQ_ERR_UNSUPPORTED;
     const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
@@ -733,8 +744,11 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
                      2ll * M * h->K + 2ll * M * h->N;
   info->flops = 2.0 * M * static_cast<double>(h->N) * h->K;
   const unisvq_layer* Ls[1] = {h};
-  describe_launch(Ls, 1, h->grouped ? UNISVQ_KERNEL_GROUPED : h->bits == 3 ? UNISVQ_KERNEL_GEMV : auto_kernel(h, M > 0 ? M : 1),
-                  M, info);
+  const int mq = M > 0 ? M : 1;
+  const int kq = h->grouped ? (mq > 64 && prefill_supported(h, mq) ? UNISVQ_KERNEL_PREFILL : UNISVQ_KERNEL_GROUPED)
+                 : h->bits == 3 ? UNISVQ_KERNEL_GEMV
+                                : auto_kernel(h, mq);
+  describe_launch(Ls, 1, kq, M, info);
   if (h->rht) {   // an input and an output rotation per chunk of the rotated-activation buffer
     const int m = M > 0 ? M : 1;
     info->launches += 2 * ((m + h->rht_tokens - 1) / h->rht_tokens);
@@ -765,7 +779,8 @@ unisvq_status unisvq_query_group(const unisvq_handle* hs, int n, int M, unisvq_i
   info->d = hs[0]->d;
   info->algo_bytes += info->meta_bytes + 2ll * M * hs[0]->K;   // x is read once per call
   const int m = M > 0 ? M : 1;
-  const int kernel = hs[0]->grouped ? UNISVQ_KERNEL_GROUPED
+  const int kernel = hs[0]->grouped ? (m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL
+                                                                            : UNISVQ_KERNEL_GROUPED)
                      : hs[0]->bits == 3 ? UNISVQ_KERNEL_GEMV
                      : m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL
                                                              : decode_kernel_for(weights, nb, m);

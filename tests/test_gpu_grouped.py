@@ -156,9 +156,9 @@ def test_grouped_entry_points():
     x = to_dev(xb)
     stream = torch.cuda.current_stream().cuda_stream
     y = torch.zeros((5, N), dtype=torch.bfloat16, device="cuda")
-    for kern in (binding.KERNEL_PREFILL, binding.KERNEL_GEMV, binding.KERNEL_SKINNY, binding.KERNEL_GEMV_ROWS):
+    for kern in (binding.KERNEL_GEMV, binding.KERNEL_SKINNY, binding.KERNEL_GEMV_ROWS):
         assert layer.forward_ptr(x.data_ptr(), y.data_ptr(), 5, stream, kern) == binding.ERR_UNSUPPORTED
-    for kern in (binding.KERNEL_AUTO, binding.KERNEL_DECODE, binding.KERNEL_GROUPED):
+    for kern in (binding.KERNEL_AUTO, binding.KERNEL_DECODE, binding.KERNEL_GROUPED, binding.KERNEL_PREFILL):
         assert layer.forward_ptr(x.data_ptr(), y.data_ptr(), 5, stream, kern) == binding.OK
     assert layer.forward_noalloc_ptr(x.data_ptr(), y.data_ptr(), 5, stream) == binding.OK
     assert binding.sync_status() == binding.OK
@@ -175,3 +175,67 @@ def test_grouped_entry_points():
     assert binding.sync_status() == binding.OK
     for h in (layer, c2, plain):
         h.close()
+
+
+@pytest.mark.parametrize("N,K", [(256, 1024), (520, 1000), (1000, 2048), (384, 640)])
+def test_grouped_prefill_parity(N, K):
+    """d = 2 per-group layers run the tcgen05 prefill GEMM above 64 tokens,
+    with per-(row, group) codeword tables built by its converter warps."""
+    codes, A, B, layer = make(N, K, 2, seed=7)
+    assert layer.query(65)["kernel"] == binding.KERNEL_PREFILL
+    assert layer.query(64)["kernel"] == binding.KERNEL_GROUPED
+    Ms = (65, 200, 300)
+    xall = synth.activations(7, 40, N + K, sum(Ms), K)
+    yr, S = oracle.linear_grouped(xall, codes, A, B, GC)
+    o = 0
+    for M in Ms:
+        res = oracle.compare(run(layer, xall[o:o + M]), yr[o:o + M], S[o:o + M])
+        assert res["ok"], (M, res)
+        o += M
+    # forced at few tokens too
+    res = oracle.compare(run(layer, xall[:9], binding.KERNEL_PREFILL), yr[:9], S[:9])
+    assert res["ok"], res
+    layer.close()
+
+
+def test_grouped_prefill_integer_case_bit_exact():
+    g = np.random.default_rng(77)
+    N, K, d = 256, 640, 2
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    A = g.integers(-2, 3, size=(N, K // GC, d, d)).astype(np.float16)
+    B = g.integers(-2, 3, size=(N, K // GC, d)).astype(np.float16)
+    layer = binding.UniSVQLinear(codes, A, B, group_cols=GC)
+    x = g.integers(-1, 2, size=(150, K)).astype(np.float32) * (g.random((150, K)) < 0.03)
+    xb = synth.f32_to_bf16_bits(x)
+    yr, _ = oracle.linear_grouped(xb, codes, A, B, GC)
+    assert np.abs(yr).max() <= 256
+    yg = run(layer, xb, binding.KERNEL_PREFILL)
+    assert np.array_equal(yg, yr), np.abs(yg - yr).max()
+    layer.close()
+
+
+def test_grouped_prefill_only_for_d2():
+    codes, A, B, layer = make(256, 512, 4, seed=8)
+    assert layer.query(200)["kernel"] == binding.KERNEL_GROUPED
+    x = torch.zeros((100, 512), dtype=torch.bfloat16, device="cuda")
+    y = torch.zeros((100, 256), dtype=torch.bfloat16, device="cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+    assert layer.forward_ptr(x.data_ptr(), y.data_ptr(), 100, stream, binding.KERNEL_PREFILL) == binding.ERR_UNSUPPORTED
+    xb = synth.activations(8, 40, 0, 100, 512)
+    check(run(layer, xb), xb, codes, A, B)
+    layer.close()
+
+
+def test_grouped_group_call_at_prefill_sizes():
+    K, d, M = 1024, 2, 96
+    shapes = [(512, K), (256, K)]
+    made = [synth.layer_inputs_grouped(9, 42, i, 0, N, K_, d) for i, (N, K_) in enumerate(shapes)]
+    layers = [binding.UniSVQLinear(c, A, B, group_cols=GC) for c, A, B in made]
+    assert binding.query_group(layers, M)["kernel"] == binding.KERNEL_PREFILL
+    xb = synth.activations(9, 42, M, M, K)
+    ys = binding.linear_group(layers, to_dev(xb))
+    assert binding.sync_status() == binding.OK
+    for (c, A, B), y in zip(made, ys):
+        check(y.float().cpu().numpy().astype(np.float64), xb, c, A, B)
+    for layer in layers:
+        layer.close()
