@@ -14,7 +14,8 @@
 //                 per lane; every d-vector index selects its exact bf16
 //                 codeword RN(A z + B) from a pack-time table (per-matrix
 //                 maps), or from a table of the row's map that the warp
-//                 builds for every 128-column group (per-group maps, d = 2)
+//                 builds for every 128-column group (per-group maps, d = 2),
+//                 or as A z + B from the row's map (per-group maps, d = 4)
 //   warps 10..13  epilogue: tcgen05.ld of the accumulator, bf16, global store
 // The accumulator is double-buffered in TMEM so the epilogue of one tile runs
 // under the main loop of the next.
@@ -284,7 +285,105 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     const int r0 = 16 * c + g, r1 = r0 + 8;
     const uint32_t lut_s = sbase + C::kOffLut;
     int it = 0;
-    if (a.meta) {
+    if (a.meta && a.d == 4) {
+      // Per-(row, 128-column group) maps, d = 4: 256 codewords per row and group
+      // are too many to tabulate per k-tile, so each output is formed directly,
+      // sum_c' A[c][c'] z_c' + B[c] in fp32. Natural columns 64 h + 8 cc + j
+      // (cc = 2t, 2t + 1: the lane's own chunks) are vector 16 h + 2 cc + j/4,
+      // coordinate c = j mod 4; its coordinate c' sits in the word of half c'/2
+      // at shift 2 (c' mod 2) + h and byte e(2 (cc mod 2) + j/4), quarter t. The
+      // warp stages its 16 rows' maps (20 fp16 each, 640 contiguous bytes) in
+      // shared memory once per k-tile.
+      const uint32_t map_s = sbase + C::kOffGrp + c * 1024;   // [16 rows][20] fp16
+      for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
+        const int n_blk = tile / a.mtiles;
+        const uint8_t* rbase = a.codes + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
+        const uint32_t* mbase = reinterpret_cast<const uint32_t*>(a.meta + static_cast<size_t>(n_blk) * a.KT * kBM * 20 +
+                                                                  static_cast<size_t>(16 * c) * 20);
+        const int nkt = (a.nkb + 1) >> 1;
+        auto load_codes = [&](int kt) -> uint4 {
+          return kt < nkt ? __ldg(reinterpret_cast<const uint4*>(rbase + static_cast<size_t>(kt) * kTileBytes))
+                          : make_uint4(0, 0, 0, 0);
+        };
+        // this lane's 5 of the 160 words of the warp's 16 row maps of group kt
+        auto load_maps = [&](int kt, uint32_t (&w)[5]) {
+#pragma unroll
+          for (int i = 0; i < 5; ++i)
+            w[i] = kt < nkt ? __ldg(mbase + static_cast<size_t>(kt) * kBM * 10 + lane + 32 * i) : 0u;
+        };
+        uint4 cn = load_codes(0), cur = cn;
+        uint32_t mw[5];
+        load_maps(0, mw);
+        float am[2][16], bm[2][4];   // the maps of rows r0, r1 for the current group
+        bool ok = !*abort_flag;
+        for (int kb = 0; kb < a.nkb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const int hs = kb & 1;
+          if (hs == 0) {
+            cur = cn;
+            __syncwarp();   // the previous group's maps are in registers already
+#pragma unroll
+            for (int i = 0; i < 5; ++i) sts32(map_s + (lane + 32 * i) * 4, mw[i]);
+            __syncwarp();
+            cn = load_codes((kb >> 1) + 1);
+            load_maps((kb >> 1) + 1, mw);
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const uint32_t rec = map_s + (g + 8 * q) * 40;
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                const uint32_t w = lds32(rec + 4 * i);
+                am[q][2 * i] = half_lo_f(w);
+                am[q][2 * i + 1] = half_hi_f(w);
+              }
+#pragma unroll
+              for (int i = 0; i < 2; ++i) {
+                const uint32_t w = lds32(rec + 32 + 4 * i);
+                bm[q][2 * i] = half_lo_f(w);
+                bm[q][2 * i + 1] = half_hi_f(w);
+              }
+            }
+          }
+          if (ok && it >= STAGES) {
+            ok = !*abort_flag && mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty);
+            if (!ok) *abort_flag = 1;
+          }
+          if (ok) {
+            const uint32_t tile_addr = sbase + C::kOffA + s * kATileBytes;
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const uint32_t wh[2] = {q ? cur.y : cur.x, q ? cur.w : cur.z};   // halves 0 and 1 of the row
+              const uint32_t row_addr = tile_addr + (q ? r1 : r0) * 128;
+#pragma unroll
+              for (int u = 0; u < 2; ++u) {
+                const int cc = 2 * t + u;
+                uint32_t o[4];
+#pragma unroll
+                for (int vv = 0; vv < 2; ++vv) {
+                  const int e = 2 * u + vv;
+                  const int bsh = 8 * ((e >> 1) | ((e & 1) << 1));
+                  float z[4];
+#pragma unroll
+                  for (int c2 = 0; c2 < 4; ++c2)
+                    z[c2] = static_cast<float>((wh[c2 >> 1] >> (bsh + 2 * (2 * (c2 & 1) + hs))) & 3u);
+                  float w[4];
+#pragma unroll
+                  for (int cr = 0; cr < 4; ++cr)
+                    w[cr] = fmaf(am[q][4 * cr + 3], z[3],
+                                 fmaf(am[q][4 * cr + 2], z[2], fmaf(am[q][4 * cr + 1], z[1], fmaf(am[q][4 * cr], z[0], bm[q][cr]))));
+                  o[2 * vv] = pack_bf16x2(w[0], w[1]);
+                  o[2 * vv + 1] = pack_bf16x2(w[2], w[3]);
+                }
+                sts128(row_addr + ((cc ^ g) << 4), o[0], o[1], o[2], o[3]);
+              }
+            }
+            fence_proxy_async_smem();
+          }
+          __syncwarp();
+          if (lane == 0 && ok) mbar_arrive(afull(s));
+        }
+      }
+    } else if (a.meta) {
       // Per-(row, 128-column group) maps, d = 2, codes permuted within each group
       // (pack_codes_grouped_host): coordinate c of vector v = 16 s + 4 t + e(b)
       // sits in the word of half c at shift s and byte b. The A tile keeps the
@@ -526,8 +625,8 @@ int pick_bn(int M) { return M <= 64 ? 64 : (M <= 128 ? 128 : 256); }
 }  // namespace
 
 bool prefill_supported(const unisvq_layer* L, int M) {
-  // per-group layers: d = 2 (the converters build a 16-pair table per row and group)
-  const bool maps_ok = L->grouped ? L->d == 2 : L->d <= 4;
+  // per-group layers: d = 2 (a 16-pair table per row and group) or d = 4 (direct sums)
+  const bool maps_ok = L->grouped ? (L->d == 2 || L->d == 4) : L->d <= 4;
   return M > 0 && maps_ok && L->bits == 2 && (L->K % 8) == 0 && get_encode() != nullptr;
 }
 

@@ -177,11 +177,12 @@ def test_grouped_entry_points():
         h.close()
 
 
+@pytest.mark.parametrize("d", [2, 4])
 @pytest.mark.parametrize("N,K", [(256, 1024), (520, 1000), (1000, 2048), (384, 640)])
-def test_grouped_prefill_parity(N, K):
-    """d = 2 per-group layers run the tcgen05 prefill GEMM above 64 tokens,
-    with per-(row, group) codeword tables built by its converter warps."""
-    codes, A, B, layer = make(N, K, 2, seed=7)
+def test_grouped_prefill_parity(N, K, d):
+    """d = 2 and d = 4 per-group layers run the tcgen05 prefill GEMM above 64
+    tokens (d = 2: per-(row, group) codeword tables; d = 4: direct sums)."""
+    codes, A, B, layer = make(N, K, d, seed=7)
     assert layer.query(65)["kernel"] == binding.KERNEL_PREFILL
     assert layer.query(64)["kernel"] == binding.KERNEL_GROUPED
     Ms = (65, 200, 300)
@@ -198,9 +199,10 @@ def test_grouped_prefill_parity(N, K):
     layer.close()
 
 
-def test_grouped_prefill_integer_case_bit_exact():
-    g = np.random.default_rng(77)
-    N, K, d = 256, 640, 2
+@pytest.mark.parametrize("d", [2, 4])
+def test_grouped_prefill_integer_case_bit_exact(d):
+    g = np.random.default_rng(77 + d)
+    N, K = 256, 640
     codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
     A = g.integers(-2, 3, size=(N, K // GC, d, d)).astype(np.float16)
     B = g.integers(-2, 3, size=(N, K // GC, d)).astype(np.float16)
@@ -214,14 +216,15 @@ def test_grouped_prefill_integer_case_bit_exact():
     layer.close()
 
 
-def test_grouped_prefill_only_for_d2():
-    codes, A, B, layer = make(256, 512, 4, seed=8)
+@pytest.mark.parametrize("d", [1, 8])
+def test_grouped_prefill_only_for_d2_and_d4(d):
+    codes, A, B, layer = make(256, 512, d, seed=8)
     assert layer.query(200)["kernel"] == binding.KERNEL_GROUPED
     x = torch.zeros((100, 512), dtype=torch.bfloat16, device="cuda")
     y = torch.zeros((100, 256), dtype=torch.bfloat16, device="cuda")
     stream = torch.cuda.current_stream().cuda_stream
     assert layer.forward_ptr(x.data_ptr(), y.data_ptr(), 100, stream, binding.KERNEL_PREFILL) == binding.ERR_UNSUPPORTED
-    xb = synth.activations(8, 40, 0, 100, 512)
+    xb = synth.activations(8, 40, d, 100, 512)
     check(run(layer, xb), xb, codes, A, B)
     layer.close()
 
