@@ -146,7 +146,8 @@ unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, cons
  * it cannot be folded onto the activations, so these layers run their own
  * GEMV (UNISVQ_KERNEL_GROUPED), which forms the moments
  * S_rc = sum_v x[v d + r] z[v d + c] of each group on the tensor cores and
- * applies the row's A and B to them.
+ * applies the row's A and B to them; for M > 64 and d in {2, 4} they run the
+ * prefill GEMM, whose converters dequantise with the row's map of each group.
  *   codes      : host, [N][K] uint8, each 0..3
  *   A_f16      : host, [N][G][d][d] fp16 bits, G = ceil(K / group_cols)
  *   B_f16      : host, [N][G][d] fp16 bits
@@ -156,8 +157,9 @@ unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, cons
  * 128-column group permuted (coordinate c of the group's vectors gathered
  * into 16-column runs); the maps are stored as fp16 [Np/128][Kp/128][128]
  * [d*d + d] (A row-major, then B), zero for padding rows.
- * unisvq_linear, _group (all layers grouped, same d), _force (AUTO, DECODE or
- * GROUPED; other kernels UNSUPPORTED), _noalloc, _query and
+ * unisvq_linear, _group (all layers grouped, same d), _force (AUTO, DECODE,
+ * GROUPED, or PREFILL for d in {2, 4}; other kernels UNSUPPORTED), _noalloc,
+ * _query and
  * unisvq_dequant_debug accept the handle. The host buffers are copied before
  * return. Errors: INVALID_ARG (null pointer, bad shape, code > 3, non-finite
  * A/B), UNSUPPORTED (d or group_cols), OOM, CUDA.
