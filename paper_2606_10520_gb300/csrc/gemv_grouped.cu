@@ -484,17 +484,49 @@ DecodePlan plan_grp(int nb, int KT, int num_sms, int M, int D) {
   return p;
 }
 
-// Tokens per launch: at most 32 / D (the columns of four n8 tiles), halved
-// until the CTA's shared memory fits.
+// Estimated time of one launch of plan p: waves x (k-tiles per CTA x NT + 2),
+// NT n8 column tiles per k-tile and 2 for a CTA's fixed cost (activation
+// staging, fold, reduction).
+long long grp_cost(const DecodePlan& p, int M, int D, int num_sms) {
+  const size_t smem = grp_shape(M, p.kt_per_cta, p.ks, D, p.nt).smem;
+  const int per_sm = (D < 8 && kWSmemPerSm / (smem + kWSmemReserved) >= 2) ? 2 : 1;
+  const long long slots = static_cast<long long>(per_sm) * num_sms;
+  const long long waves = (static_cast<long long>(p.nb) * p.ks + slots - 1) / slots;
+  return waves * (static_cast<long long>(p.kt_per_cta) * p.nt + 2);
+}
+
+// Tokens per launch: 32/D, 16/D or 8/D (four, two or one n8 column tiles),
+// whichever gives the least estimated time for the M tokens (launches x
+// grp_cost): a launch that fits two CTAs per SM often beats one with twice the
+// tokens that fits only one. A cap whose shared memory does not fit is skipped.
 int grp_tokens(int nb, int KT, int num_sms, int M, int D, DecodePlan* out) {
-  int mc = M < 32 / D ? M : 32 / D;
-  DecodePlan p = plan_grp(nb, KT, num_sms, mc, D);
-  while (!p.ks && mc > 1) {
-    mc = (mc + 1) / 2;
-    p = plan_grp(nb, KT, num_sms, mc, D);
+  int best_mc = 0;
+  long long best = -1;
+  DecodePlan best_p{};
+  for (int cap = 32 / D; cap >= 1 && cap >= 8 / D; cap /= 2) {
+    const int mc = M < cap ? M : cap;
+    const DecodePlan p = plan_grp(nb, KT, num_sms, mc, D);
+    if (!p.ks) continue;
+    const long long cost = static_cast<long long>((M + mc - 1) / mc) * grp_cost(p, mc, D, num_sms);
+    if (best < 0 || cost < best) {
+      best = cost;
+      best_mc = mc;
+      best_p = p;
+    }
+    if (M <= cap / 2) break;   // the next cap would give the same launch
   }
-  *out = p;
-  return p.ks ? mc : 0;
+  if (!best_mc) {   // nothing fits at 8/D tokens: halve further
+    int mc = M < 8 / D ? M : (8 / D > 0 ? 8 / D : 1);
+    DecodePlan p = plan_grp(nb, KT, num_sms, mc, D);
+    while (!p.ks && mc > 1) {
+      mc = (mc + 1) / 2;
+      p = plan_grp(nb, KT, num_sms, mc, D);
+    }
+    *out = p;
+    return p.ks ? mc : 0;
+  }
+  *out = best_p;
+  return best_mc;
 }
 
 template <int D, int NT>
