@@ -71,8 +71,8 @@ def variant_layers(args):
     return args.layers if args.only in ("grouped", "rht", "bits3") else GROUPED_LAYERS
 # Sources whose change invalidates a committed ncu traffic figure, per kernel.
 KERNEL_SOURCES = {
-    "gemv_kernel": ("paper_2606_10520_gb300/csrc/gemv.cu", "paper_2606_10520_gb300/csrc/common.cuh",
-                    "paper_2606_10520_gb300/csrc/layout.h"),
+    "gemv_kernel": ("paper_2606_10520_gb300/csrc/gemv.cu", "paper_2606_10520_gb300/csrc/mma_sync.cuh",
+                    "paper_2606_10520_gb300/csrc/common.cuh", "paper_2606_10520_gb300/csrc/layout.h"),
     "decode_kernel": ("paper_2606_10520_gb300/csrc/decode.cu", "paper_2606_10520_gb300/csrc/common.cuh",
                       "paper_2606_10520_gb300/csrc/layout.h"),
 }

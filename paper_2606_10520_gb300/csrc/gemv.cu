@@ -26,6 +26,7 @@
 // partial sums of the rows it owns, which the other CTAs deliver with st.async
 // stores counted on an mbarrier.
 #include "common.cuh"
+#include "mma_sync.cuh"
 #include "internal.h"
 
 namespace unisvq {
@@ -76,15 +77,6 @@ struct GemvArgs {
   int* err;
   GemvLayer<DV> layer[kMaxGroup];
 };
-
-__device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
-                                          uint2 b) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
-      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b.x), "r"(b.y));
-}
 
 // x'[c .. c+3] for the d-vectors inside x[c .. c+3] (c % 4 == 0): row vector x_g A.
 // A is a register copy of the kernel parameter (reading the parameter through a
@@ -148,23 +140,6 @@ __device__ __forceinline__ uint4 fold8(int ci, uint4 xv, int pe, int d, const fl
   const float s0 = exp2i(pe - 2 * j0), s1 = exp2i(pe - 2 * j0 - 2);
   return make_uint4(pack_half2(o0[0] * s0, o0[2] * s0), pack_half2(o0[1] * s0, o0[3] * s0),
                     pack_half2(o1[0] * s1, o1[2] * s1), pack_half2(o1[1] * s1, o1[3] * s1));
-}
-
-// 2^P with P = 15 - e, e the binary exponent of bound in [2^(e-1), 2^e): puts
-// the largest possible |x'| (<= bound) below 2^15, the fp16 range.
-__device__ __forceinline__ int token_scale_exp(float bound) {
-  if (!(bound > 0.f)) return 0;
-  const int e = static_cast<int>(__float_as_uint(bound) >> 23) - 126;
-  return max(-100, min(100, 15 - e));
-}
-
-// Eight activations x[k .. k+7] of one token as packed bf16 (zero at or past kend).
-__device__ __forceinline__ uint4 load_x8(const uint16_t* row, int k, int kend, bool vec8) {
-  if (vec8 && k + 7 < kend) return ldg_v4(row + k);
-  uint32_t e[8];
-#pragma unroll
-  for (int q = 0; q < 8; ++q) e[q] = (k + q < kend) ? static_cast<uint32_t>(row[k + q]) : 0u;
-  return make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
 }
 
 // Bit j of x -> bit 2j (x < 2^16).

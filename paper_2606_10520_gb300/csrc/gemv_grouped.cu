@@ -27,9 +27,8 @@
 // gemv_kernel. A lane's MMA columns are (m, r) pairs with fixed r in
 // {2t mod d, (2t + 1) mod d}; after the chunks of class c it adds
 // A[row][r][c] * S to its running sums, and once per k-tile B[row][r] * X_r.
-#include <cuda_fp16.h>
-
 #include "common.cuh"
+#include "mma_sync.cuh"
 #include "internal.h"
 
 namespace unisvq {
@@ -70,39 +69,6 @@ struct GrpShape {
   int off_b, off_xs, off_meta, off_xsum, off_red, off_tok, xs_stride;
 };
 
-__device__ __forceinline__ void mma_f16_16816(float (&acc)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
-                                              uint2 b) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
-      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
-      : "+f"(acc[0]), "+f"(acc[1]), "+f"(acc[2]), "+f"(acc[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b.x), "r"(b.y));
-}
-
-// 2^P with P = 15 - e for max|x| in [2^(e-1), 2^e): the scaled activations
-// (and so every B value, <= max|x| 2^P) stay below 2^15, in fp16 range.
-__device__ __forceinline__ int act_scale_exp(float mx) {
-  if (!(mx > 0.f)) return 0;
-  const int e = static_cast<int>(__float_as_uint(mx) >> 23) - 126;
-  return max(-100, min(100, 15 - e));
-}
-
-__device__ __forceinline__ float half_lo(uint32_t v) {
-  return __half2float(__ushort_as_half(static_cast<unsigned short>(v & 0xFFFFu)));
-}
-__device__ __forceinline__ float half_hi(uint32_t v) {
-  return __half2float(__ushort_as_half(static_cast<unsigned short>(v >> 16)));
-}
-
-// Eight activations x[k .. k+7] of one token as packed bf16 (zero at or past kend).
-__device__ __forceinline__ uint4 load_x8_grp(const uint16_t* row, int k, int kend, bool vec8) {
-  if (vec8 && k + 7 < kend) return ldg_v4(row + k);
-  uint32_t e[8];
-#pragma unroll
-  for (int q = 0; q < 8; ++q) e[q] = (k + q < kend) ? static_cast<uint32_t>(row[k + q]) : 0u;
-  return make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
-}
-
 // A[r][0..D-1] of one row's record as floats (fp16 in shared memory).
 template <int D>
 __device__ __forceinline__ void load_arow(const uint16_t* rec, int r, float (&a)[D]) {
@@ -111,21 +77,21 @@ __device__ __forceinline__ void load_arow(const uint16_t* rec, int r, float (&a)
     a[0] = __half2float(__ushort_as_half(p[0]));
   } else if constexpr (D == 2) {
     const uint32_t w = *reinterpret_cast<const uint32_t*>(p);
-    a[0] = half_lo(w);
-    a[1] = half_hi(w);
+    a[0] = f16_lo(w);
+    a[1] = f16_hi(w);
   } else if constexpr (D == 4) {
     const uint2 w = *reinterpret_cast<const uint2*>(p);
-    a[0] = half_lo(w.x);
-    a[1] = half_hi(w.x);
-    a[2] = half_lo(w.y);
-    a[3] = half_hi(w.y);
+    a[0] = f16_lo(w.x);
+    a[1] = f16_hi(w.x);
+    a[2] = f16_lo(w.y);
+    a[3] = f16_hi(w.y);
   } else {
     const uint4 w = *reinterpret_cast<const uint4*>(p);
     const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      a[2 * i] = half_lo(ws[i]);
-      a[2 * i + 1] = half_hi(ws[i]);
+      a[2 * i] = f16_lo(ws[i]);
+      a[2 * i + 1] = f16_hi(ws[i]);
     }
   }
 }
@@ -226,7 +192,7 @@ __global__ void __launch_bounds__(kWThreads, D == 8 ? 1 : 2) gemv_grouped_kernel
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const int ci = c0 + lane + 32 * j;
-        u[j] = ci < nch ? load_x8_grp(row, kbeg + 8 * ci, kend, vec8) : make_uint4(0, 0, 0, 0);
+        u[j] = ci < nch ? load_x8(row, kbeg + 8 * ci, kend, vec8) : make_uint4(0, 0, 0, 0);
       }
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
@@ -257,7 +223,7 @@ __global__ void __launch_bounds__(kWThreads, D == 8 ? 1 : 2) gemv_grouped_kernel
     }
 #pragma unroll
     for (int off = 16; off; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-    const int P = act_scale_exp(mx);
+    const int P = token_scale_exp(mx);
     __syncwarp();
     const float xscale = exp2i(P - 24);
     for (int idx = lane; idx < n_kt * D; idx += 32) xsum[((idx / D) * MP + tk) * D + idx % D] *= xscale;
@@ -318,10 +284,10 @@ __global__ void __launch_bounds__(kWThreads, D == 8 ? 1 : 2) gemv_grouped_kernel
         } else {
           const uint32_t w0 = *reinterpret_cast<const uint32_t*>(m0 + D * D + rA);
           const uint32_t w1 = *reinterpret_cast<const uint32_t*>(m1 + D * D + rA);
-          b0A = half_lo(w0);
-          b0B = half_hi(w0);
-          b1A = half_lo(w1);
-          b1B = half_hi(w1);
+          b0A = f16_lo(w0);
+          b0B = f16_hi(w0);
+          b1A = f16_lo(w1);
+          b1B = f16_hi(w1);
         }
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
@@ -334,7 +300,7 @@ __global__ void __launch_bounds__(kWThreads, D == 8 ? 1 : 2) gemv_grouped_kernel
           const uint32_t msk = 0x00030003u << (2 * s);
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt)
-            mma_f16_16816(acc[nt], wa & msk, wb & msk, (wa >> 8) & msk, (wb >> 8) & msk,
+            mma_16816(acc[nt], wa & msk, wb & msk, (wa >> 8) & msk, (wb >> 8) & msk,
                           bl[((i * 8 + q) * NT + nt) * 32]);
           if (q % NQ == NQ - 1) {   // last chunk of class c: apply A[row][r][c]
             const int c = q / NQ;

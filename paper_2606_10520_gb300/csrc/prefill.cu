@@ -19,10 +19,10 @@
 //   warps 10..13  epilogue: tcgen05.ld of the accumulator, bf16, global store
 // The accumulator is double-buffered in TMEM so the epilogue of one tile runs
 // under the main loop of the next.
-#include <cuda_fp16.h>
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
+#include "mma_sync.cuh"
 #include "internal.h"
 
 namespace unisvq {
@@ -152,12 +152,6 @@ __device__ __forceinline__ uint32_t lds32(uint32_t addr) {
 }
 __device__ __forceinline__ void sts32(uint32_t addr, uint32_t v) {
   asm volatile("st.shared.b32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
-}
-__device__ __forceinline__ float half_lo_f(uint32_t v) {
-  return __half2float(__ushort_as_half(static_cast<unsigned short>(v & 0xFFFFu)));
-}
-__device__ __forceinline__ float half_hi_f(uint32_t v) {
-  return __half2float(__ushort_as_half(static_cast<unsigned short>(v >> 16)));
 }
 __device__ __forceinline__ uint2 lds64(uint32_t addr) {
   uint2 v;
@@ -333,14 +327,14 @@ __global__ void __launch_bounds__(kPfThreads, 1)
 #pragma unroll
               for (int i = 0; i < 8; ++i) {
                 const uint32_t w = lds32(rec + 4 * i);
-                am[q][2 * i] = half_lo_f(w);
-                am[q][2 * i + 1] = half_hi_f(w);
+                am[q][2 * i] = f16_lo(w);
+                am[q][2 * i + 1] = f16_hi(w);
               }
 #pragma unroll
               for (int i = 0; i < 2; ++i) {
                 const uint32_t w = lds32(rec + 32 + 4 * i);
-                bm[q][2 * i] = half_lo_f(w);
-                bm[q][2 * i + 1] = half_hi_f(w);
+                bm[q][2 * i] = f16_lo(w);
+                bm[q][2 * i + 1] = f16_hi(w);
               }
             }
           }
@@ -424,8 +418,8 @@ __global__ void __launch_bounds__(kPfThreads, 1)
 #pragma unroll
             for (int q = 0; q < 2; ++q) {
               const uint3 m = q ? m1 : m0;
-              const float a00 = half_lo_f(m.x), a01 = half_hi_f(m.x), a10 = half_lo_f(m.y), a11 = half_hi_f(m.y);
-              const float b0 = half_lo_f(m.z), b1 = half_hi_f(m.z);
+              const float a00 = f16_lo(m.x), a01 = f16_hi(m.x), a10 = f16_lo(m.y), a11 = f16_hi(m.y);
+              const float b0 = f16_lo(m.z), b1 = f16_hi(m.z);
               const int rr = g + 8 * q;
 #pragma unroll
               for (int k = 0; k < 4; ++k) {
