@@ -452,22 +452,26 @@ def run_ours(args, rank, world, local_rank):
                       "kernels": {"+".join(shapes[i][0] for i in grp): KERNEL_NAMES.get(call_info(grp, M)["kernel"], "?")
                                   for grp in groups}})
 
-    # ---- e2e: pinned host buffers, H2D + layer + D2H inside the timed graphs ---
+    # ---- e2e: pinned host buffers; every step copies its inputs in and its
+    # results out inside the timed graphs (activations stay on the device
+    # between the layers of a step, as in a model) ---------------------------
     e2e = None
     if not args.no_e2e:
         hx = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True).copy_(v.cpu()) for k, v in xs.items()}
         hy = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in ys.items()}
         egraphs, h2d, d2h = [], 0, 0
         for M in M_SWEEP:
-            def e2e_pass(M=M):
+            in_keys = sorted(k for k in xs if k[0] == M)
+            out_keys = sorted(k for k in ys if k[0] == M)
+            def e2e_pass(M=M, in_keys=in_keys, out_keys=out_keys):
                 sp = torch.cuda.current_stream().cuda_stream
+                for k in in_keys:
+                    xs[k].copy_(hx[k], non_blocking=True)
                 for layer in stack:
                     for grp in groups:
-                        K = shapes[grp[0]][2]
-                        xs[(M, K)].copy_(hx[(M, K)], non_blocking=True)
                         issue(layer, grp, M, sp)
-                        for i in grp:
-                            hy[(M, i)].copy_(ys[(M, i)], non_blocking=True)
+                for k in out_keys:
+                    hy[k].copy_(ys[k], non_blocking=True)
             with torch.cuda.stream(side):
                 e2e_pass()
             torch.cuda.synchronize()
@@ -475,21 +479,15 @@ def run_ours(args, rank, world, local_rank):
             with torch.cuda.graph(g, stream=side):
                 e2e_pass()
             egraphs.append(g)
-            for grp in groups:
-                h2d += 2 * M * shapes[grp[0]][2] * args.layers
-                for i in grp:
-                    d2h += 2 * M * shapes[i][1] * args.layers
+            h2d += sum(xs[k].numel() * xs[k].element_size() for k in in_keys)
+            d2h += sum(ys[k].numel() * ys[k].element_size() for k in out_keys)
         te = time_graphs(torch, egraphs, args.steps, args.warmup, side)
         te = max_over_ranks([te], world, "cuda")[0]
         e2e = {"value": whole_job_gbs(step_bytes, args.steps, world, te), "unit": "GB/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-               "how": "per call: pinned-host x -> device copy, the library call, device -> pinned-host y "
-                      "of every projection; the whole sweep replayed from CUDA graphs"}
-
-    # ---- per-(row, 128-column group) affine layers ------------------------
-    grouped = None
-    if not args.no_grouped:
-        grouped = run_grouped(torch, binding, peaks, args, side)
+               "how": "per step (the sweep's M passes): pinned-host -> device copies of the step's activations "
+                      "before the layers, the library calls, device -> pinned-host copies of every projection's "
+                      "output after them; replayed from CUDA graphs"}
 
     # ---- 3-bit codes --------------------------------------------------------
     bits3 = None
