@@ -762,21 +762,30 @@ def run_prefill(torch, binding, peaks, args, stream):
         for pi, (_, N, K) in enumerate(shapes):
             codes, A, B = synth.layer_inputs_grouped(0, 2, 0, pi, N, K, dg)
             glayers.append(b.UniSVQLinear(codes, A, B, group_cols=128))
-        per_group[dg] = time_grouped_prefill(torch, b, shapes, glayers, xs, ys, M, reps, stream)
+        per_group[dg] = time_prefill_layers(torch, b, shapes, glayers, xs, ys, M, reps, stream)
         for l in glayers:
             l.close()
+    # the same set with 3-bit codes (per-matrix maps)
+    l3 = []
+    for pi, (_, N, K) in enumerate(shapes):
+        codes, A, B = synth.layer_inputs_bits(0, 2, 0, pi, N, K, 2, 3)
+        l3.append(b.UniSVQLinear(codes, A, B, bits=3))
+    t3 = time_prefill_layers(torch, b, shapes, l3, xs, ys, M, reps, stream)
+    for l in l3:
+        l.close()
     return {"workload": f"Llama-3-8B-shaped projection set (7 GEMMs) at M={M}, d=2",
             "TFLOP/s": tflops, "frac_of_measured_bf16": tflops / peaks["bf16_tflops"],
             "per_group_maps_TFLOP/s": flops * reps / per_group[2] / 1e12,
             "per_group_maps_d4_TFLOP/s": flops * reps / per_group[4] / 1e12,
+            "bits3_TFLOP/s": flops * reps / t3 / 1e12,
             "frac_of_measured_bf16_sustained": tflops / peaks["bf16_tflops_sustained"],
             "us_per_layer_set": t / reps * 1e6, "per_projection": per,
             "cublas_bf16_dense_TFLOP/s": flops * reps / td / 1e12,
             "kernel": "prefill_kernel (tcgen05)"}
 
 
-def time_grouped_prefill(torch, b, shapes, glayers, xs, ys, M, reps, stream):
-    """Seconds for `reps` passes of the prefill GEMM over per-group layers."""
+def time_prefill_layers(torch, b, shapes, glayers, xs, ys, M, reps, stream):
+    """Seconds for `reps` passes of the prefill GEMM over the layer set `glayers`."""
     def grouped_pass():
         sp = torch.cuda.current_stream().cuda_stream
         for (_, N, K), h in zip(shapes, glayers):

@@ -130,8 +130,9 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
  * 2048 (rb Kp/128 + kt) + 256 u + 8 (4g + t); halfword i belongs to word i of
  * the chunk and its bit 4b + s is bit 2 of the code at bits [8b+2s+1 : 8b+2s]
  * of that word. 3-bit layers take d in {1, 2, 4} and run the GEMV
- * (UNISVQ_KERNEL_GEMV, 32 tokens per launch) at every M; other forced kernels
- * return UNSUPPORTED. Errors as unisvq_pack, plus UNSUPPORTED (bits, or
+ * (UNISVQ_KERNEL_GEMV, 32 tokens per launch) up to 64 tokens; above that,
+ * layers with d <= 2 run the prefill GEMM (also forceable), d = 4 stays on
+ * the GEMV. Other forced kernels return UNSUPPORTED. Errors as unisvq_pack, plus UNSUPPORTED (bits, or
  * bits = 3 with d = 8) and INVALID_ARG (a code >= 2^bits).
  */
 unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
@@ -162,7 +163,8 @@ unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, cons
  * _query and
  * unisvq_dequant_debug accept the handle. The host buffers are copied before
  * return. Errors: INVALID_ARG (null pointer, bad shape, code > 3, non-finite
- * A/B), UNSUPPORTED (d or group_cols), OOM, CUDA.
+ * A/B), UNSUPPORTED (d or group_cols, or a K whose per-CTA slice of maps does
+ * not fit in shared memory: d = 8 with K above about 10240), OOM, CUDA.
  */
 unisvq_status unisvq_pack_grouped(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
                                   int N, int K, int d, int group_cols, void* stream, unisvq_handle* out);

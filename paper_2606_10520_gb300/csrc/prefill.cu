@@ -21,6 +21,8 @@
 // under the main loop of the next.
 #include <cudaTypedefs.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 #include "mma_sync.cuh"
 #include "internal.h"
@@ -39,6 +41,7 @@ struct PrefillArgs {
   const uint8_t* codes;
   const uint32_t* lut;   // d <= 2: 16 x bf16x2 pair codewords; d == 4: 256 x 4 bf16
   const uint16_t* meta;  // per-group layers (d = 2): fp16 [Np/128][KT][128][6] (A row-major, B), else null
+  const uint8_t* hi;     // 3-bit codes (d <= 2): the high-bit plane; the table has 64 pairs, index z0 | z1 << 3
   uint16_t* y;
   int M, N, K, KT, d;
   int nkb;               // k-blocks of 64 columns: ceil(K / 64)
@@ -199,7 +202,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   // Codeword table -> shared memory (per-matrix maps only; per-group layers
   // build theirs in the converters).
   if (!a.meta) {
-    const int words = a.d == 4 ? 512 : 16;
+    const int words = a.hi ? 64 : (a.d == 4 ? 512 : 16);
     uint32_t* lut_s = reinterpret_cast<uint32_t*>(smem + C::kOffLut);
     for (int i = threadIdx.x; i < words; i += kPfThreads) lut_s[i] = a.lut[i];
   }
@@ -463,58 +466,96 @@ __global__ void __launch_bounds__(kPfThreads, 1)
           if (lane == 0 && ok) mbar_arrive(afull(s));
         }
       }
-    } else
-    for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
-      const int n_blk = tile / a.mtiles;
-      const uint8_t* rbase = a.codes + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
-      // Code words of stage kb live at tile kb/2, half kb%2; prefetched 3 stages ahead.
-      auto load = [&](int kb) -> uint2 {
-        return kb < a.nkb ? __ldg(reinterpret_cast<const uint2*>(rbase + (kb >> 1) * kTileBytes + (kb & 1) * 8))
-                          : make_uint2(0, 0);
-      };
-      uint2 q0 = load(0), q1 = load(1), q2 = load(2);
-      bool ok = !*abort_flag;
-      for (int kb = 0; kb < a.nkb; ++kb, ++it) {
-        const int s = it % STAGES;
-        const uint2 cw = q0;
-        q0 = q1;
-        q1 = q2;
-        q2 = load(kb + 3);
-        if (ok && it >= STAGES) {
-          ok = !*abort_flag && mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty);
-          if (!ok) *abort_flag = 1;
-        }
-        if (ok) {
-          const uint32_t tile_addr = sbase + C::kOffA + s * kATileBytes;
-#pragma unroll
-          for (int q = 0; q < 2; ++q) {
-            const uint32_t w = q ? cw.y : cw.x;
-            const uint32_t row_addr = tile_addr + (q ? r1 : r0) * 128;
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-              const int cc = 2 * t + e;                       // chunk: stage columns 8cc .. 8cc+7
-              const uint32_t e0 = extract4(w, 2 * e);         // columns 8cc .. 8cc+3
-              const uint32_t e1 = extract4(w, 2 * e + 1);     // columns 8cc+4 .. 8cc+7
-              uint32_t o0, o1, o2, o3;
-              if (a.d == 4) {
-                const uint32_t i0 = (e0 & 3u) | ((e0 >> 6) & 0xCu) | ((e0 >> 12) & 0x30u) | ((e0 >> 18) & 0xC0u);
-                const uint32_t i1 = (e1 & 3u) | ((e1 >> 6) & 0xCu) | ((e1 >> 12) & 0x30u) | ((e1 >> 18) & 0xC0u);
-                const uint2 v0 = lds64(lut_s + i0 * 8), v1 = lds64(lut_s + i1 * 8);
-                o0 = v0.x; o1 = v0.y; o2 = v1.x; o3 = v1.y;
-              } else {
-                o0 = lds32(lut_s + (((e0 & 3u) | ((e0 >> 6) & 0xCu)) << 2));
-                o1 = lds32(lut_s + ((((e0 >> 16) & 3u) | ((e0 >> 22) & 0xCu)) << 2));
-                o2 = lds32(lut_s + (((e1 & 3u) | ((e1 >> 6) & 0xCu)) << 2));
-                o3 = lds32(lut_s + ((((e1 >> 16) & 3u) | ((e1 >> 22) & 0xCu)) << 2));
-              }
-              sts128(row_addr + ((cc ^ g) << 4), o0, o1, o2, o3);
+    } else {
+      // Per-matrix maps. The loop is compiled twice (HI = 3-bit codes or not) so
+      // that the 2-bit loop carries no high-bit loads or branches.
+      auto convert = [&](auto hi_tag) {
+        constexpr bool HI = decltype(hi_tag)::value;
+        for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
+          const int n_blk = tile / a.mtiles;
+          const uint8_t* rbase =
+              a.codes + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
+          // Code words of stage kb live at tile kb/2, half kb%2; prefetched 3 stages ahead.
+          auto load = [&](int kb) -> uint2 {
+            return kb < a.nkb ? __ldg(reinterpret_cast<const uint2*>(rbase + (kb >> 1) * kTileBytes + (kb & 1) * 8))
+                              : make_uint2(0, 0);
+          };
+          // 3-bit codes: the halfwords of those two words in the high-bit plane
+          const uint8_t* hbase =
+              HI ? a.hi + static_cast<size_t>(n_blk) * a.KT * (kTileBytes / 2) + c * (kUnitBytes / 2) + lane * 8
+                 : nullptr;
+          auto load_hi = [&](int kb) -> uint32_t {
+            if constexpr (HI)
+              return kb < a.nkb
+                         ? __ldg(reinterpret_cast<const uint32_t*>(hbase + (kb >> 1) * (kTileBytes / 2) + (kb & 1) * 4))
+                         : 0u;
+            return 0u;
+          };
+          uint2 q0 = load(0), q1 = load(1), q2 = load(2);
+          uint32_t h0 = load_hi(0), h1 = load_hi(1), h2 = load_hi(2);
+          bool ok = !*abort_flag;
+          for (int kb = 0; kb < a.nkb; ++kb, ++it) {
+            const int s = it % STAGES;
+            const uint2 cw = q0;
+            q0 = q1;
+            q1 = q2;
+            q2 = load(kb + 3);
+            const uint32_t hw = h0;
+            if constexpr (HI) {
+              h0 = h1;
+              h1 = h2;
+              h2 = load_hi(kb + 3);
             }
+            if (ok && it >= STAGES) {
+              ok = !*abort_flag && mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty);
+              if (!ok) *abort_flag = 1;
+            }
+            if (ok) {
+              const uint32_t tile_addr = sbase + C::kOffA + s * kATileBytes;
+#pragma unroll
+              for (int q = 0; q < 2; ++q) {
+                const uint32_t w = q ? cw.y : cw.x;
+                const uint32_t hq = q ? (hw >> 16) : (hw & 0xFFFFu);   // bit 4b + s: high bit of byte b, shift s
+                const uint32_t row_addr = tile_addr + (q ? r1 : r0) * 128;
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                  const int cc = 2 * t + e;                       // chunk: stage columns 8cc .. 8cc+7
+                  const uint32_t e0 = extract4(w, 2 * e);         // columns 8cc .. 8cc+3
+                  const uint32_t e1 = extract4(w, 2 * e + 1);     // columns 8cc+4 .. 8cc+7
+                  uint32_t o0, o1, o2, o3;
+                  if constexpr (HI) {
+                    // 3-bit codes of columns 8cc + 4u + b: low bits (e_u >> 8b) & 3, high bit
+                    // bit 4b + 2e + u of hq; pairs (b = 0, 1) and (2, 3) index the 64-pair table
+                    auto code3 = [&](uint32_t eu, int u, int b) -> uint32_t {
+                      return ((eu >> (8 * b)) & 3u) | (((hq >> (4 * b + 2 * e + u)) & 1u) << 2);
+                    };
+                    o0 = lds32(lut_s + ((code3(e0, 0, 0) | (code3(e0, 0, 1) << 3)) << 2));
+                    o1 = lds32(lut_s + ((code3(e0, 0, 2) | (code3(e0, 0, 3) << 3)) << 2));
+                    o2 = lds32(lut_s + ((code3(e1, 1, 0) | (code3(e1, 1, 1) << 3)) << 2));
+                    o3 = lds32(lut_s + ((code3(e1, 1, 2) | (code3(e1, 1, 3) << 3)) << 2));
+                  } else if (a.d == 4) {
+                    const uint32_t i0 = (e0 & 3u) | ((e0 >> 6) & 0xCu) | ((e0 >> 12) & 0x30u) | ((e0 >> 18) & 0xC0u);
+                    const uint32_t i1 = (e1 & 3u) | ((e1 >> 6) & 0xCu) | ((e1 >> 12) & 0x30u) | ((e1 >> 18) & 0xC0u);
+                    const uint2 v0 = lds64(lut_s + i0 * 8), v1 = lds64(lut_s + i1 * 8);
+                    o0 = v0.x; o1 = v0.y; o2 = v1.x; o3 = v1.y;
+                  } else {
+                    o0 = lds32(lut_s + (((e0 & 3u) | ((e0 >> 6) & 0xCu)) << 2));
+                    o1 = lds32(lut_s + ((((e0 >> 16) & 3u) | ((e0 >> 22) & 0xCu)) << 2));
+                    o2 = lds32(lut_s + (((e1 & 3u) | ((e1 >> 6) & 0xCu)) << 2));
+                    o3 = lds32(lut_s + ((((e1 >> 16) & 3u) | ((e1 >> 22) & 0xCu)) << 2));
+                  }
+                  sts128(row_addr + ((cc ^ g) << 4), o0, o1, o2, o3);
+                }
+              }
+              fence_proxy_async_smem();
+            }
+            __syncwarp();
+            if (lane == 0 && ok) mbar_arrive(afull(s));
           }
-          fence_proxy_async_smem();
         }
-        __syncwarp();
-        if (lane == 0 && ok) mbar_arrive(afull(s));
-      }
+      };
+      if (a.hi) convert(std::true_type{});
+      else convert(std::false_type{});
     }
   } else {
     // ---------------- epilogue ----------------
@@ -600,6 +641,7 @@ unisvq_status launch_bn(const unisvq_layer* L, const PrefillPlan& p, const void*
   a.codes = L->codes;
   a.lut = L->tlut;
   a.meta = L->grouped ? L->meta : nullptr;
+  a.hi = L->bits == 3 ? L->hi : nullptr;
   a.y = static_cast<uint16_t*>(y);
   a.M = M;
   a.N = L->N;
@@ -619,9 +661,10 @@ int pick_bn(int M) { return M <= 64 ? 64 : (M <= 128 ? 128 : 256); }
 }  // namespace
 
 bool prefill_supported(const unisvq_layer* L, int M) {
-  // per-group layers: d = 2 (a 16-pair table per row and group) or d = 4 (direct sums)
-  const bool maps_ok = L->grouped ? (L->d == 2 || L->d == 4) : L->d <= 4;
-  return M > 0 && maps_ok && L->bits == 2 && (L->K % 8) == 0 && get_encode() != nullptr;
+  // per-group layers: d = 2 (a 16-pair table per row and group) or d = 4 (direct
+  // sums); 3-bit layers: d <= 2 (a 64-pair table; 8^4 quads would not fit)
+  const bool maps_ok = L->grouped ? (L->d == 2 || L->d == 4) : (L->bits == 3 ? L->d <= 2 : L->d <= 4);
+  return M > 0 && maps_ok && (L->K % 8) == 0 && get_encode() != nullptr;
 }
 
 PrefillPlan plan_prefill(const unisvq_layer* L, int M) {

@@ -164,8 +164,18 @@ unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, cons
   //   d == 8: none (4^8 codewords do not fit the converters' shared memory;
   //   such layers run the decode kernels at every M).
   auto bf = [](double w) { return static_cast<uint32_t>(f64_to_bf16_rne(w)); };
+  //   3-bit codes, d <= 2: 64 bf16 pairs, index lo | hi << 3 for columns (k, k+1);
+  //   3-bit codes, d = 4: none (8^4 quads do not fit beside the stage ring).
   std::vector<uint32_t> tlut;
-  if (d == 8 || bits != 2) {   // the prefill GEMM takes 2-bit layers with d <= 4 only
+  if (bits == 3 && d <= 2) {
+    tlut.resize(64);
+    for (int v = 0; v < 64; ++v) {
+      const int lo = v & 7, hi = v >> 3;
+      const double w0 = d == 2 ? cb[static_cast<size_t>(lo | (hi << 3)) * 2 + 0] : cb[lo];
+      const double w1 = d == 2 ? cb[static_cast<size_t>(lo | (hi << 3)) * 2 + 1] : cb[hi];
+      tlut[v] = bf(w0) | (bf(w1) << 16);
+    }
+  } else if (d == 8 || bits != 2) {   // the prefill GEMM takes no table for these
     tlut.assign(1, 0u);
   } else if (d <= 2) {
     tlut.resize(16);
@@ -272,6 +282,14 @@ unisvq_status unisvq_pack_grouped(const uint8_t* codes, const uint16_t* A_f16, c
       cudaDeviceGetAttribute(&L->num_sms, cudaDevAttrMultiProcessorCount, L->device) != cudaSuccess) {
     delete L;
     return UNISVQ_ERR_CUDA;
+  }
+  {   // the per-group GEMV stages a CTA's K slice of maps in shared memory
+    int per = 0;
+    plan_grouped(L, L->Np / kTileRows, 1, &per);
+    if (!per) {   // e.g. d = 8 with K above about 10240 (18 KB of maps per k-tile)
+      delete L;
+      return UNISVQ_ERR_UNSUPPORTED;
+    }
   }
   L->code_bytes = unisvq_packed_code_bytes(N, K);
   L->meta_bytes = static_cast<size_t>(L->Np / kTileRows) * L->KT * kTileRows * (d * d + d) * sizeof(uint16_t);
@@ -410,7 +428,10 @@ static unisvq_status check_io(unisvq_handle h, const void* x, void* y, int M) {
 // decode path with the library's static fold workspace.
 static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, void* y, int M, cudaStream_t s,
                                   bool noalloc) {
-  if (h->bits == 3) {   // 3-bit codes: the GEMV at every M (no workspace, so also for noalloc)
+  if (h->bits == 3) {   // 3-bit codes: the prefill GEMM (d <= 2) above 64 tokens, else the GEMV
+    if (!noalloc && ((kernel == UNISVQ_KERNEL_AUTO && M > 64 && prefill_supported(h, M)) ||
+                     kernel == UNISVQ_KERNEL_PREFILL))
+      return prefill_supported(h, M) ? launch_prefill(h, x, y, M, s) : UNISVQ_ERR_UNSUPPORTED;
     if (!noalloc && kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GEMV)
       return kernel >= 0 && kernel <= UNISVQ_KERNEL_GROUPED ? UNISVQ_ERR_UNSUPPORTED : UNISVQ_ERR_INVALID_ARG;
     return launch_gemv(h, x, y, M, s);
@@ -612,7 +633,10 @@ static unisvq_status group_inner(const unisvq_handle* hs, int n, int kernel, con
   int n3 = 0;
   for (int i = 0; i < n; ++i) n3 += hs[i]->bits == 3 ? 1 : 0;
   if (n3) {   // 3-bit layers: one GEMV launch when every layer is 3-bit, else layer by layer
-    if (n3 == n && (kernel == UNISVQ_KERNEL_AUTO || kernel == UNISVQ_KERNEL_DECODE || kernel == UNISVQ_KERNEL_GEMV)) {
+    bool pf = kernel == UNISVQ_KERNEL_AUTO && M > 64;
+    for (int i = 0; i < n && pf; ++i) pf = prefill_supported(hs[i], M);
+    if (!pf && n3 == n &&
+        (kernel == UNISVQ_KERNEL_AUTO || kernel == UNISVQ_KERNEL_DECODE || kernel == UNISVQ_KERNEL_GEMV)) {
       const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
       for (int i = 0; i < n; ++i) Ls[i] = hs[i];
       return launch_gemv_group(Ls, n, x, ys, M, s);
@@ -746,7 +770,7 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
   const unisvq_layer* Ls[1] = {h};
   const int mq = M > 0 ? M : 1;
   const int kq = h->grouped ? (mq > 64 && prefill_supported(h, mq) ? UNISVQ_KERNEL_PREFILL : UNISVQ_KERNEL_GROUPED)
-                 : h->bits == 3 ? UNISVQ_KERNEL_GEMV
+                 : h->bits == 3 ? (mq > 64 && prefill_supported(h, mq) ? UNISVQ_KERNEL_PREFILL : UNISVQ_KERNEL_GEMV)
                                 : auto_kernel(h, mq);
   describe_launch(Ls, 1, kq, M, info);
   if (h->rht) {   // an input and an output rotation per chunk of the rotated-activation buffer
@@ -781,7 +805,8 @@ unisvq_status unisvq_query_group(const unisvq_handle* hs, int n, int M, unisvq_i
   const int m = M > 0 ? M : 1;
   const int kernel = hs[0]->grouped ? (m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL
                                                                             : UNISVQ_KERNEL_GROUPED)
-                     : hs[0]->bits == 3 ? UNISVQ_KERNEL_GEMV
+                     : hs[0]->bits == 3 ? (m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL
+                                                                                 : UNISVQ_KERNEL_GEMV)
                      : m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL
                                                              : decode_kernel_for(weights, nb, m);
   const unisvq_layer* Ls[UNISVQ_MAX_GROUP];

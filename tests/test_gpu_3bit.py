@@ -80,15 +80,15 @@ def test_3bit_integer_case_bit_exact(d):
 def test_3bit_dispatch_groups_and_entry_points():
     N, K, d = 512, 1024, 2
     codes, A, B, layer = make(N, K, d, 3)
-    for M in (1, 16, 2048):
-        info = layer.query(M)
-        assert info["kernel"] == binding.KERNEL_GEMV
+    for M in (1, 16, 64):
+        assert layer.query(M)["kernel"] == binding.KERNEL_GEMV
+    assert layer.query(65)["kernel"] == binding.KERNEL_PREFILL
     assert layer.query(1)["algo_bytes"] == N * K * 3 // 8 + (d * d + d) * 2 + 2 * K + 2 * N
     xb = synth.activations(3, 60, 0, 5, K)
     x = to_dev(xb)
     stream = torch.cuda.current_stream().cuda_stream
     y = torch.zeros((5, N), dtype=torch.bfloat16, device="cuda")
-    for kern in (binding.KERNEL_PREFILL, binding.KERNEL_SKINNY, binding.KERNEL_GEMV_ROWS, binding.KERNEL_GROUPED):
+    for kern in (binding.KERNEL_SKINNY, binding.KERNEL_GEMV_ROWS, binding.KERNEL_GROUPED):
         assert layer.forward_ptr(x.data_ptr(), y.data_ptr(), 5, stream, kern) == binding.ERR_UNSUPPORTED
     assert layer.forward_noalloc_ptr(x.data_ptr(), y.data_ptr(), 5, stream) == binding.OK
     assert binding.sync_status() == binding.OK
@@ -119,4 +119,53 @@ def test_3bit_full_size_sampled_rows(N, K):
         y = run(layer, xb)
         yr, S = oracle.linear(xb, codes[rows], A, B)
         assert oracle.compare(y[:, rows], yr, S)["ok"]
+    layer.close()
+
+
+@pytest.mark.parametrize("d", [1, 2])
+@pytest.mark.parametrize("N,K", [(256, 1024), (520, 1000), (384, 4096)])
+def test_3bit_prefill_parity(d, N, K):
+    """3-bit layers with d <= 2 run the tcgen05 prefill GEMM above 64 tokens
+    (64-pair codeword table, high bits from the bit plane)."""
+    codes, A, B, layer = make(N, K, d, 6)
+    Ms = (65, 300)
+    xall = synth.activations(6, 60, N + d, sum(Ms), K)
+    yr, S = oracle.linear(xall, codes, A, B)
+    o = 0
+    for M in Ms:
+        assert layer.query(M)["kernel"] == binding.KERNEL_PREFILL
+        res = oracle.compare(run(layer, xall[o:o + M]), yr[o:o + M], S[o:o + M])
+        assert res["ok"], (M, res)
+        o += M
+    res = oracle.compare(run(layer, xall[:7], binding.KERNEL_PREFILL), yr[:7], S[:7])
+    assert res["ok"], res
+    layer.close()
+
+
+@pytest.mark.parametrize("d", [1, 2])
+def test_3bit_prefill_integer_case_bit_exact(d):
+    g = np.random.default_rng(50 + d)
+    N, K = 256, 512
+    codes = g.integers(0, 8, size=(N, K), dtype=np.uint8)
+    A = (np.eye(d) - np.eye(d, k=1)).astype(np.float16)
+    B = g.integers(-3, 4, size=d).astype(np.float16)
+    layer = binding.UniSVQLinear(codes, A, B, bits=3)
+    x = g.integers(-1, 2, size=(130, K)).astype(np.float32) * (g.random((130, K)) < 0.03)
+    xb = synth.f32_to_bf16_bits(x)
+    yr, _ = oracle.linear(xb, codes, A, B)
+    assert np.abs(yr).max() <= 256
+    assert np.array_equal(run(layer, xb), yr)
+    layer.close()
+
+
+def test_3bit_d4_stays_on_the_gemv():
+    codes, A, B, layer = make(256, 512, 4, 7)
+    assert layer.query(200)["kernel"] == binding.KERNEL_GEMV
+    x = torch.zeros((100, 512), dtype=torch.bfloat16, device="cuda")
+    y = torch.zeros((100, 256), dtype=torch.bfloat16, device="cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+    assert layer.forward_ptr(x.data_ptr(), y.data_ptr(), 100, stream, binding.KERNEL_PREFILL) == binding.ERR_UNSUPPORTED
+    xb = synth.activations(7, 60, 4, 100, 512)
+    yr, S = oracle.linear(xb, codes, A, B)
+    assert oracle.compare(run(layer, xb), yr, S)["ok"]
     layer.close()

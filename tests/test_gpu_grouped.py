@@ -242,3 +242,23 @@ def test_grouped_group_call_at_prefill_sizes():
         check(y.float().cpu().numpy().astype(np.float64), xb, c, A, B)
     for layer in layers:
         layer.close()
+
+
+def test_grouped_pack_rejects_maps_that_do_not_fit():
+    """d = 8 per-group maps take 18 KB per k-tile: a 28672-wide layer has no
+    GEMV plan, so packing it is refused instead of every call failing."""
+    N, K, d = 128, 28672, 8
+    G = K // GC
+    codes = np.zeros((N, K), dtype=np.uint8)
+    A = np.zeros((N, G, d, d), dtype=np.float16)
+    B = np.zeros((N, G, d), dtype=np.float16)
+    with pytest.raises(binding.UnisvqError) as e:
+        binding.UniSVQLinear(codes, A, B, group_cols=GC)
+    assert e.value.status == binding.ERR_UNSUPPORTED
+    # d = 4 at the same width packs and runs
+    A4 = np.zeros((N, G, 4, 4), dtype=np.float16)
+    B4 = np.ones((N, G, 4), dtype=np.float16)
+    layer = binding.UniSVQLinear(codes, A4, B4, group_cols=GC)
+    xb = synth.activations(10, 40, 0, 2, K)
+    check(run(layer, xb), xb, codes, A4, B4)
+    layer.close()
