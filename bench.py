@@ -489,6 +489,11 @@ def run_ours(args, rank, world, local_rank):
                       "before the layers, the library calls, device -> pinned-host copies of every projection's "
                       "output after them; replayed from CUDA graphs"}
 
+    # ---- per-(row, 128-column group) affine layers ------------------------
+    grouped = None
+    if not args.no_grouped:
+        grouped = run_grouped(torch, binding, peaks, args, side)
+
     # ---- 3-bit codes --------------------------------------------------------
     bits3 = None
     if not args.no_bits3:
