@@ -448,7 +448,7 @@ def run_ours(args, rank, world, local_rank):
         gbs = nb * max(3, args.steps // 4) / tm / 1e9
         sweep.append({"M": M, "GB/s": round(gbs, 1), "frac_of_measured_hbm": round(gbs / peaks["hbm_gbs"], 4),
                       "frac_of_8TBs": round(gbs / 8000.0, 4),
-                      "us_per_layer": round(tm / max(3, args.steps // 4) / n_calls * 1e6, 3),
+                      "us_per_projection": round(tm / max(3, args.steps // 4) / n_calls * 1e6, 3),
                       "kernels": {"+".join(shapes[i][0] for i in grp): KERNEL_NAMES.get(call_info(grp, M)["kernel"], "?")
                                   for grp in groups}})
 

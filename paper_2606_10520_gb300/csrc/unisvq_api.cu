@@ -444,7 +444,7 @@ static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, vo
     }
     return launch_skinny_static(h, x, y, M, s);
   }
-  if (h->grouped) {   // per-group maps: the prefill GEMM (d = 2) for M > 64, else the per-group GEMV
+  if (h->grouped) {   // per-group maps: the prefill GEMM (d = 2, 4) for M > 64, else the per-group GEMV
     if ((kernel == UNISVQ_KERNEL_AUTO && M > 64 && prefill_supported(h, M)) || kernel == UNISVQ_KERNEL_PREFILL)
       return prefill_supported(h, M) ? launch_prefill(h, x, y, M, s) : UNISVQ_ERR_UNSUPPORTED;
     if (kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GROUPED)
