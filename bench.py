@@ -514,7 +514,8 @@ def run_ours(args, rank, world, local_rank):
     if rank == 0 and world == 1 and not args.no_cpu:
         gbs_cpu, t_cpu, names = oracle_sample(args.cpu_budget)
         cpu = {"value": gbs_cpu, "unit": "GB/s", "cores": cpu_threads(), "kind": "oracle",
-               "sample": f"oracle.linear (fp64 NumPy) on layer-0 projections {names} at M=1, "
+               "sample": f"oracle.linear (fp64 NumPy) at M=1 on {len(names)} projection calls cycling over "
+                         f"the layer-0 set ({', '.join(n for n, _, _ in synth.LLAMA2_7B)}), "
                          f"{t_cpu:.1f} s of CPU work"}
 
     line = {
