@@ -46,7 +46,7 @@ typedef enum {
 enum {
   UNISVQ_KERNEL_AUTO = 0,     /* pick by M (unisvq_linear does this)                   */
   UNISVQ_KERNEL_DECODE = 1,   /* the decode kernel auto would pick for this M (a GEMV)  */
-  UNISVQ_KERNEL_PREFILL = 2,  /* tcgen05 GEMM, exact bf16 codeword tiles in smem       */
+  UNISVQ_KERNEL_PREFILL = 2,  /* tcgen05 GEMM, bf16 weight tiles in smem (exact codewords for d <= 4) */
   UNISVQ_KERNEL_GEMV = 3,     /* fold + register-operand tensor-core GEMV, M <= 32/launch */
   UNISVQ_KERNEL_SKINNY = 4,   /* fold + tcgen05 with codes as 8-bit TMEM operand, M <= 16/launch */
   UNISVQ_KERNEL_GEMV_ROWS = 5, /* GEMV with whole-K row slices per CTA (no cluster), M <= 4/launch */
@@ -103,8 +103,9 @@ typedef struct {
  *   N, K  : output / input features, N >= 1, K >= d, K % d == 0
  *   d     : vector length, 1, 2, 4 or 8 (Eq. def:unisvq; the paper uses d = 4
  *           and d = 8 in its vector-length ablation, Table tab:ablation_dim).
- *           The prefill GEMM takes d <= 4; d = 8 layers use the decode
- *           kernels at every M.
+ *           The prefill GEMM takes every d: exact bf16 codewords from a
+ *           pack-time table for d <= 4, and for d = 8 the fp32 sum of two
+ *           quad-table rows rounded once to bf16.
  *   stream: stream for the upload; pack synchronises it before returning
  *   out   : receives the handle
  * The host buffers are copied before return; the caller keeps ownership.

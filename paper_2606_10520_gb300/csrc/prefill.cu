@@ -13,7 +13,8 @@
 //   warps 2..9    converters: one 16-row unit per warp, two rows x 16 columns
 //                 per lane; every d-vector index selects its exact bf16
 //                 codeword RN(A z + B) from a pack-time table (per-matrix
-//                 maps), or from a table of the row's map that the warp
+//                 maps, d <= 4; for d = 8 the sum of two quad-table rows,
+//                 fp32), or from a table of the row's map that the warp
 //                 builds for every 128-column group (per-group maps, d = 2),
 //                 or as A z + B from the row's map (per-group maps, d = 4)
 //   warps 10..13  epilogue: tcgen05.ld of the accumulator, bf16, global store
@@ -39,7 +40,7 @@ constexpr int kEpiWarp0 = 10;
 
 struct PrefillArgs {
   const uint8_t* codes;
-  const uint32_t* lut;   // d <= 2: 16 x bf16x2 pair codewords; d == 4: 256 x 4 bf16
+  const uint32_t* lut;   // d <= 2: 16 x bf16x2 pair codewords; d == 4: 256 x 4 bf16; d == 8: [2][256][8] fp32 quad tables
   const uint16_t* meta;  // per-group layers (d = 2): fp16 [Np/128][KT][128][6] (A row-major, B), else null
   const uint8_t* hi;     // 3-bit codes (d <= 2): the high-bit plane; the table has 64 pairs, index z0 | z1 << 3
   uint16_t* y;
@@ -55,9 +56,9 @@ struct PfCfg {
   static constexpr int kStageBytes = kATileBytes + kBTileBytes;
   static constexpr int kOffA = 0;
   static constexpr int kOffB = STAGES * kATileBytes;
-  static constexpr int kOffLut = STAGES * kStageBytes;            // 2 KB
+  static constexpr int kOffLut = STAGES * kStageBytes;            // 2 KB (d = 8: the 16 KB region)
   static constexpr int kOffGrp = kOffLut + 2048;                   // 8 x 1 KB: per-group tables
-  static constexpr int kOffBars = kOffGrp + 8 * 1024;
+  static constexpr int kOffBars = kOffLut + 16 * 1024;
   // bars: bfull[S], afull[S], empty[S], accfull[2], accempty[2]
   static constexpr int kOffTmemPtr = kOffBars + (3 * STAGES + 5) * 8;   // + drain barrier
   static constexpr int kOffFlag = kOffTmemPtr + 8;
@@ -161,6 +162,11 @@ __device__ __forceinline__ uint2 lds64(uint32_t addr) {
   asm volatile("ld.shared.v2.b32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
   return v;
 }
+__device__ __forceinline__ float4 lds128f(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
+  return v;
+}
 
 template <int BN, int STAGES>
 __global__ void __launch_bounds__(kPfThreads, 1)
@@ -202,7 +208,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   // Codeword table -> shared memory (per-matrix maps only; per-group layers
   // build theirs in the converters).
   if (!a.meta) {
-    const int words = a.hi ? 64 : (a.d == 4 ? 512 : 16);
+    const int words = a.hi ? 64 : (a.d == 8 ? 4096 : (a.d == 4 ? 512 : 16));
     uint32_t* lut_s = reinterpret_cast<uint32_t*>(smem + C::kOffLut);
     for (int i = threadIdx.x; i < words; i += kPfThreads) lut_s[i] = a.lut[i];
   }
@@ -467,10 +473,12 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         }
       }
     } else {
-      // Per-matrix maps. The loop is compiled twice (HI = 3-bit codes or not) so
-      // that the 2-bit loop carries no high-bit loads or branches.
-      auto convert = [&](auto hi_tag) {
+      // Per-matrix maps. The loop is compiled three times (HI = 3-bit codes,
+      // D8 = vectors of 8 through the pair tables, or neither) so that the
+      // common loop carries no high-bit loads and no extra branches.
+      auto convert = [&](auto hi_tag, auto d8_tag) {
         constexpr bool HI = decltype(hi_tag)::value;
+        constexpr bool D8 = decltype(d8_tag)::value;
         for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
           const int n_blk = tile / a.mtiles;
           const uint8_t* rbase =
@@ -533,6 +541,18 @@ __global__ void __launch_bounds__(kPfThreads, 1)
                     o1 = lds32(lut_s + ((code3(e0, 0, 2) | (code3(e0, 0, 3) << 3)) << 2));
                     o2 = lds32(lut_s + ((code3(e1, 1, 0) | (code3(e1, 1, 1) << 3)) << 2));
                     o3 = lds32(lut_s + ((code3(e1, 1, 2) | (code3(e1, 1, 3) << 3)) << 2));
+                  } else if constexpr (D8) {
+                    // the chunk is one vector: coordinates 0..3 in bytes 0..3 of e0, 4..7 of e1;
+                    // w = T_0[z0 z1 z2 z3] + T_1[z4 z5 z6 z7] (quad tables, fp32)
+                    const uint32_t i0 = (e0 & 3u) | ((e0 >> 6) & 0xCu) | ((e0 >> 12) & 0x30u) | ((e0 >> 18) & 0xC0u);
+                    const uint32_t i1 = (e1 & 3u) | ((e1 >> 6) & 0xCu) | ((e1 >> 12) & 0x30u) | ((e1 >> 18) & 0xC0u);
+                    const uint32_t t0 = lut_s + i0 * 32, t1 = lut_s + 8192 + i1 * 32;
+                    const float4 a0 = lds128f(t0), a1 = lds128f(t0 + 16);
+                    const float4 b0 = lds128f(t1), b1 = lds128f(t1 + 16);
+                    o0 = pack_bf16x2(a0.x + b0.x, a0.y + b0.y);
+                    o1 = pack_bf16x2(a0.z + b0.z, a0.w + b0.w);
+                    o2 = pack_bf16x2(a1.x + b1.x, a1.y + b1.y);
+                    o3 = pack_bf16x2(a1.z + b1.z, a1.w + b1.w);
                   } else if (a.d == 4) {
                     const uint32_t i0 = (e0 & 3u) | ((e0 >> 6) & 0xCu) | ((e0 >> 12) & 0x30u) | ((e0 >> 18) & 0xC0u);
                     const uint32_t i1 = (e1 & 3u) | ((e1 >> 6) & 0xCu) | ((e1 >> 12) & 0x30u) | ((e1 >> 18) & 0xC0u);
@@ -554,8 +574,9 @@ __global__ void __launch_bounds__(kPfThreads, 1)
           }
         }
       };
-      if (a.hi) convert(std::true_type{});
-      else convert(std::false_type{});
+      if (a.hi) convert(std::true_type{}, std::false_type{});
+      else if (a.d == 8) convert(std::false_type{}, std::true_type{});
+      else convert(std::false_type{}, std::false_type{});
     }
   } else {
     // ---------------- epilogue ----------------
@@ -662,8 +683,9 @@ int pick_bn(int M) { return M <= 64 ? 64 : (M <= 128 ? 128 : 256); }
 
 bool prefill_supported(const unisvq_layer* L, int M) {
   // per-group layers: d = 2 (a 16-pair table per row and group) or d = 4 (direct
-  // sums); 3-bit layers: d <= 2 (a 64-pair table; 8^4 quads would not fit)
-  const bool maps_ok = L->grouped ? (L->d == 2 || L->d == 4) : (L->bits == 3 ? L->d <= 2 : L->d <= 4);
+  // sums); 3-bit layers: d <= 2 (a 64-pair table; 8^4 quads would not fit);
+  // per-matrix 2-bit layers: every d (d = 8 through two quad tables)
+  const bool maps_ok = L->grouped ? (L->d == 2 || L->d == 4) : (L->bits == 3 ? L->d <= 2 : true);
   return M > 0 && maps_ok && (L->K % 8) == 0 && get_encode() != nullptr;
 }
 

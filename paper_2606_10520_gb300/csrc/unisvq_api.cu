@@ -175,6 +175,20 @@ unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, cons
       const double w1 = d == 2 ? cb[static_cast<size_t>(lo | (hi << 3)) * 2 + 1] : cb[hi];
       tlut[v] = bf(w0) | (bf(w1) << 16);
     }
+  } else if (d == 8 && bits == 2) {
+    // 4^8 codewords are too many for shared memory: two partial tables, one
+    // per coordinate quad q, T_q[z_4q | z_4q+1 << 2 | z_4q+2 << 4 | z_4q+3 << 6][r]
+    // = sum_c A[r][4q + c] z_4q+c (+ B[r] for q = 0), each exact in fp64 and
+    // rounded once to fp32; the prefill GEMM adds the two rows of a vector in fp32.
+    tlut.resize(4096);
+    for (int qd = 0; qd < 2; ++qd)
+      for (int v = 0; v < 256; ++v)
+        for (int r = 0; r < 8; ++r) {
+          double t = qd == 0 ? B[r] : 0.0;
+          for (int c = 0; c < 4; ++c) t += A[r * 8 + 4 * qd + c] * ((v >> (2 * c)) & 3);
+          const float f = static_cast<float>(t);
+          std::memcpy(&tlut[static_cast<size_t>(qd * 256 + v) * 8 + r], &f, sizeof(float));
+        }
   } else if (d == 8 || bits != 2) {   // the prefill GEMM takes no table for these
     tlut.assign(1, 0u);
   } else if (d <= 2) {

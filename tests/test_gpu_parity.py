@@ -207,7 +207,7 @@ def test_full_size_decode_sampled_rows(N, K):
 PREFILL_SHAPES = [(128, 128), (200, 520), (384, 1024), (1000, 2048)]
 
 
-@pytest.mark.parametrize("d", [1, 2, 4])
+@pytest.mark.parametrize("d", [1, 2, 4, 8])
 @pytest.mark.parametrize("N,K", PREFILL_SHAPES)
 def test_prefill_parity(d, N, K):
     codes, A, B = synth.layer_inputs(8, 80, N, K, N, K, d)
@@ -218,22 +218,39 @@ def test_prefill_parity(d, N, K):
     layer.close()
 
 
-def test_d8_layers_run_the_decode_kernels_at_every_M():
-    """d = 8 (the paper's ablation length): the prefill kernel declines it (its
-    exact codeword table would have 4^8 entries), so M > 64 runs the decode
-    kernels, chunk by chunk, and still meets the oracle."""
+def test_d8_layers_dispatch_to_the_prefill_kernel():
+    """d = 8 (the paper's ablation length): above 64 tokens the library picks
+    the prefill GEMM, whose converters add two quad-table rows per vector
+    (4^8 exact codewords would not fit in shared memory)."""
     d, N, K = 8, 300, 1024
     codes, A, B = synth.layer_inputs(8, 81, N, K, N, K, d)
     layer = binding.UniSVQLinear(codes, A, B)
-    x = torch.zeros((80, K), dtype=torch.bfloat16, device="cuda")
-    y = torch.zeros((80, N), dtype=torch.bfloat16, device="cuda")
-    st = layer.forward_ptr(x.data_ptr(), y.data_ptr(), 80, torch.cuda.current_stream().cuda_stream,
-                           binding.KERNEL_PREFILL)
-    assert st == binding.ERR_UNSUPPORTED
-    assert layer.query(200)["kernel"] != binding.KERNEL_PREFILL
+    assert layer.query(200)["kernel"] == binding.KERNEL_PREFILL
+    assert layer.query(64)["kernel"] != binding.KERNEL_PREFILL
     for M in (65, 200):
         xb = synth.activations(8, 81, M, M, K)
         check(run(layer, xb), xb, codes, A, B)
+    layer.close()
+
+
+def test_d8_prefill_integer_case_bit_exact():
+    """Integer 8 x 8 A and B: every quad-table entry and every fp32 sum of two
+    is an exact small integer, so the bf16 weight tile is exact and the output
+    must equal the oracle's bit for bit."""
+    d = 8
+    A = (np.eye(d) - np.eye(d, k=-1) + np.eye(d, k=3)).astype(np.float16)
+    B = np.array([1, -2, 0, 1, 3, -1, 0, 2], dtype=np.float16)
+    N, K = 384, 1024
+    g = np.random.default_rng(18)
+    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
+    layer = binding.UniSVQLinear(codes, A, B)
+    for M in (40, 65, 300):
+        x = g.integers(-1, 2, size=(M, K)).astype(np.float32) * (g.random((M, K)) < 0.03)
+        xb = synth.f32_to_bf16_bits(x)
+        yr, _ = oracle.linear(xb, codes, A, B)
+        assert np.abs(yr).max() <= 256
+        yg = run(layer, xb, binding.KERNEL_PREFILL)
+        assert np.array_equal(yg, yr), np.abs(yg - yr).max()
     layer.close()
 
 
