@@ -92,6 +92,12 @@ size_t static_fold_workspace_bytes();
 bool prefill_supported(const unisvq_layer* L, int M);
 PrefillPlan plan_prefill(const unisvq_layer* L, int M);
 unisvq_status launch_prefill(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
+// Several layers that read the same x in one persistent launch (their tiles
+// one after the other): per-matrix 2-bit layers with one d <= 4 and one K.
+bool prefill_group_supported(const unisvq_layer* const* Ls, int n, int M);
+PrefillPlan plan_prefill_group(const unisvq_layer* const* Ls, int n, int M);
+unisvq_status launch_prefill_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                                   cudaStream_t s);
 
 unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s);
 

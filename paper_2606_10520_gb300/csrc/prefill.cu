@@ -38,17 +38,43 @@ constexpr int kATileBytes = kBM * 128;   // 16 KB
 constexpr int kConvWarp0 = 2;
 constexpr int kEpiWarp0 = 10;
 
+// Layers of one launch (several only for per-matrix 2-bit layers with one
+// d <= 4 that read the same x): their tiles are numbered one layer after the
+// other, layer i from tile0[i] on, and each keeps its own codeword table in a
+// 2 KB slot of shared memory.
+constexpr int kPfMaxLayers = UNISVQ_MAX_GROUP;
+
 struct PrefillArgs {
-  const uint8_t* codes;
-  const uint32_t* lut;   // d <= 2: 16 x bf16x2 pair codewords; d == 4: 256 x 4 bf16; d == 8: [2][256][8] fp32 quad tables
+  const uint8_t* codes[kPfMaxLayers];
+  const uint32_t* lut[kPfMaxLayers];   // d <= 2: 16 x bf16x2 pair codewords; d == 4: 256 x 4 bf16; d == 8: [2][256][8] fp32 quad tables
+  uint16_t* y[kPfMaxLayers];
+  int N[kPfMaxLayers];
+  int tile0[kPfMaxLayers];
+  int nlayers;
   const uint16_t* meta;  // per-group layers (d = 2): fp16 [Np/128][KT][128][6] (A row-major, B), else null
   const uint8_t* hi;     // 3-bit codes (d <= 2): the high-bit plane; the table has 64 pairs, index z0 | z1 << 3
-  uint16_t* y;
-  int M, N, K, KT, d;
+  int M, K, KT, d;
   int nkb;               // k-blocks of 64 columns: ceil(K / 64)
   int mtiles, tiles;
   int* err;
 };
+
+// The launch's layer of a tile (constant parameter offsets only).
+__device__ __forceinline__ int tile_layer(const PrefillArgs& a, int tile) {
+  int li = 0;
+#pragma unroll
+  for (int i = 1; i < kPfMaxLayers; ++i)
+    if (i < a.nlayers && tile >= a.tile0[i]) li = i;
+  return li;
+}
+template <class T>
+__device__ __forceinline__ T pick_layer(const T (&v)[kPfMaxLayers], int li) {
+  T r = v[0];
+#pragma unroll
+  for (int i = 1; i < kPfMaxLayers; ++i)
+    if (i == li) r = v[i];
+  return r;
+}
 
 template <int BN, int STAGES>
 struct PfCfg {
@@ -207,10 +233,16 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   }
   // Codeword table -> shared memory (per-matrix maps only; per-group layers
   // build theirs in the converters).
-  if (!a.meta) {
+  if (!a.meta) {   // layer i's table at kOffLut + 2 KB i (one layer for d = 8: 16 KB)
     const int words = a.hi ? 64 : (a.d == 8 ? 4096 : (a.d == 4 ? 512 : 16));
-    uint32_t* lut_s = reinterpret_cast<uint32_t*>(smem + C::kOffLut);
-    for (int i = threadIdx.x; i < words; i += kPfThreads) lut_s[i] = a.lut[i];
+#pragma unroll
+    for (int l = 0; l < kPfMaxLayers; ++l) {
+      if (l < a.nlayers) {
+        uint32_t* lut_s = reinterpret_cast<uint32_t*>(smem + C::kOffLut + 2048 * l);
+        const uint32_t* src = a.lut[l];
+        for (int i = threadIdx.x; i < words; i += kPfThreads) lut_s[i] = src[i];
+      }
+    }
   }
   if (warp == 0) {
     tmem_alloc(sbase + C::kOffTmemPtr, C::kTmemCols);
@@ -226,7 +258,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     if (lane == 0) {
       int it = 0;
       for (int tile = blockIdx.x; tile < a.tiles && !*abort_flag; tile += gridDim.x) {
-        const int m0 = (tile % a.mtiles) * BN;
+        const int m0 = ((tile - pick_layer(a.tile0, tile_layer(a, tile))) % a.mtiles) * BN;
         for (int kb = 0; kb < a.nkb; ++kb, ++it) {
           const int s = it % STAGES;
           if (it >= STAGES && !mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty)) {
@@ -286,7 +318,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     const int c = warp - kConvWarp0;
     const int g = lane >> 2, t = lane & 3;
     const int r0 = 16 * c + g, r1 = r0 + 8;
-    const uint32_t lut_s = sbase + C::kOffLut;
+    const uint32_t lut_base = sbase + C::kOffLut;   // layer i's table at + 2 KB i
     int it = 0;
     if (a.meta && a.d == 4) {
       // Per-(row, 128-column group) maps, d = 4: 256 codewords per row and group
@@ -299,8 +331,10 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       // shared memory once per k-tile.
       const uint32_t map_s = sbase + C::kOffGrp + c * 1024;   // [16 rows][20] fp16
       for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
-        const int n_blk = tile / a.mtiles;
-        const uint8_t* rbase = a.codes + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
+        const int li = tile_layer(a, tile);
+        const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
+        const uint8_t* rbase =
+            pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
         const uint32_t* mbase = reinterpret_cast<const uint32_t*>(a.meta + static_cast<size_t>(n_blk) * a.KT * kBM * 20 +
                                                                   static_cast<size_t>(16 * c) * 20);
         const int nkt = (a.nkb + 1) >> 1;
@@ -397,8 +431,10 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       // bf16 pairs RN(A z + B) of the row's map (four entries per lane and row).
       const uint32_t tab_s = sbase + C::kOffGrp + c * 1024;   // [16 rows][16 entries] bf16x2
       for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
-        const int n_blk = tile / a.mtiles;
-        const uint8_t* rbase = a.codes + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
+        const int li = tile_layer(a, tile);
+        const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
+        const uint8_t* rbase =
+            pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
         const uint16_t* mbase = a.meta + static_cast<size_t>(n_blk) * a.KT * kBM * 6;
         const int nkt = (a.nkb + 1) >> 1;
         auto load_codes = [&](int kt) -> uint4 {
@@ -480,9 +516,11 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         constexpr bool HI = decltype(hi_tag)::value;
         constexpr bool D8 = decltype(d8_tag)::value;
         for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
-          const int n_blk = tile / a.mtiles;
+          const int li = tile_layer(a, tile);
+          const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
           const uint8_t* rbase =
-              a.codes + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
+              pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
+          const uint32_t lut_s = lut_base + 2048u * static_cast<uint32_t>(li);
           // Code words of stage kb live at tile kb/2, half kb%2; prefetched 3 stages ahead.
           auto load = [&](int kb) -> uint2 {
             return kb < a.nkb ? __ldg(reinterpret_cast<const uint2*>(rbase + (kb >> 1) * kTileBytes + (kb & 1) * 8))
@@ -585,8 +623,12 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     bool ok = true;
     for (int tile = blockIdx.x; tile < a.tiles && ok; tile += gridDim.x, ++lt) {
       const int b = lt & 1;
-      const int n0 = (tile / a.mtiles) * kBM;
-      const int m0 = (tile % a.mtiles) * BN;
+      const int li = tile_layer(a, tile);
+      const int local = tile - pick_layer(a.tile0, li);
+      const int n0 = (local / a.mtiles) * kBM;
+      const int m0 = (local % a.mtiles) * BN;
+      uint16_t* const yl = pick_layer(a.y, li);
+      const int Nl = pick_layer(a.N, li);
       ok = !*abort_flag && mbar_wait(accfull(b), (lt >> 1) & 1, a.err, kErrTimeoutMma);
       if (!ok) {
         *abort_flag = 1;
@@ -598,11 +640,11 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       for (int c0 = 0; c0 < BN; c0 += 32) {
         uint32_t r[32];
         tmem_ld32(tmem_base + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(b * BN + c0), r);
-        if (n < a.N) {
+        if (n < Nl) {
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
             const int m = m0 + c0 + j;
-            if (m < a.M) a.y[static_cast<size_t>(m) * a.N + n] = f32_to_bf16_rn(__uint_as_float(r[j]));
+            if (m < a.M) yl[static_cast<size_t>(m) * Nl + n] = f32_to_bf16_rn(__uint_as_float(r[j]));
           }
         }
       }
@@ -634,9 +676,10 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 }
 
 template <int BN, int STAGES>
-unisvq_status launch_bn(const unisvq_layer* L, const PrefillPlan& p, const void* x, void* y, int M,
-                        cudaStream_t s) {
+unisvq_status launch_bn(const unisvq_layer* const* Ls, int n, const PrefillPlan& p, const void* x,
+                        void* const* ys, int M, cudaStream_t s) {
   using C = PfCfg<BN, STAGES>;
+  const unisvq_layer* L = Ls[0];
   static bool attr_set[64] = {};
   const int dev = L->device;
   if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
@@ -659,20 +702,27 @@ unisvq_status launch_bn(const unisvq_layer* L, const PrefillPlan& p, const void*
     return UNISVQ_ERR_CUDA;
 
   PrefillArgs a{};
-  a.codes = L->codes;
-  a.lut = L->tlut;
+  a.mtiles = (M + BN - 1) / BN;
+  int tile = 0;
+  for (int i = 0; i < n; ++i) {
+    a.codes[i] = Ls[i]->codes;
+    a.lut[i] = Ls[i]->tlut;
+    a.y[i] = static_cast<uint16_t*>(ys[i]);
+    a.N[i] = Ls[i]->N;
+    a.tile0[i] = tile;
+    tile += (Ls[i]->Np / kBM) * a.mtiles;
+  }
+  a.nlayers = n;
   a.meta = L->grouped ? L->meta : nullptr;
   a.hi = L->bits == 3 ? L->hi : nullptr;
-  a.y = static_cast<uint16_t*>(y);
   a.M = M;
-  a.N = L->N;
   a.K = L->K;
   a.KT = L->KT;
   a.d = L->d;
   a.nkb = (L->K + kBK - 1) / kBK;
-  a.mtiles = (M + BN - 1) / BN;
   a.tiles = p.tiles;
   a.err = device_error_word();
+  if (tile != p.tiles) return UNISVQ_ERR_INVALID_ARG;
   prefill_kernel<BN, STAGES><<<p.grid, kPfThreads, C::kSmem, s>>>(map, a);
   return cudaGetLastError() == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
@@ -689,22 +739,44 @@ bool prefill_supported(const unisvq_layer* L, int M) {
   return M > 0 && maps_ok && (L->K % 8) == 0 && get_encode() != nullptr;
 }
 
-PrefillPlan plan_prefill(const unisvq_layer* L, int M) {
+bool prefill_group_supported(const unisvq_layer* const* Ls, int n, int M) {
+  if (n < 1 || n > kPfMaxLayers) return false;
+  if (n == 1) return prefill_supported(Ls[0], M);
+  // several layers in one launch: per-matrix 2-bit layers with one d <= 4 and
+  // one K, whose tables (<= 2 KB each) share the table region
+  for (int i = 0; i < n; ++i)
+    if (Ls[i]->grouped || Ls[i]->bits != 2 || Ls[i]->d > 4 || Ls[i]->d != Ls[0]->d || Ls[i]->K != Ls[0]->K ||
+        !prefill_supported(Ls[i], M))
+      return false;
+  return true;
+}
+
+PrefillPlan plan_prefill_group(const unisvq_layer* const* Ls, int n, int M) {
   PrefillPlan p{};
   p.bn = pick_bn(M);
   const int mtiles = (M + p.bn - 1) / p.bn;
-  p.tiles = (L->Np / kBM) * mtiles;
-  p.grid = p.tiles < L->num_sms ? p.tiles : L->num_sms;
+  p.tiles = 0;
+  for (int i = 0; i < n; ++i) p.tiles += (Ls[i]->Np / kBM) * mtiles;
+  p.grid = p.tiles < Ls[0]->num_sms ? p.tiles : Ls[0]->num_sms;
   if (p.grid < 1) p.grid = 1;
   p.smem = p.bn == 64 ? PfCfg<64, 8>::kSmem : (p.bn == 128 ? PfCfg<128, 6>::kSmem : PfCfg<256, 4>::kSmem);
   return p;
 }
 
+PrefillPlan plan_prefill(const unisvq_layer* L, int M) { return plan_prefill_group(&L, 1, M); }
+
+unisvq_status launch_prefill_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                                   cudaStream_t s) {
+  if (!prefill_group_supported(Ls, n, M)) return UNISVQ_ERR_UNSUPPORTED;
+  const PrefillPlan p = plan_prefill_group(Ls, n, M);
+  if (p.bn == 64) return launch_bn<64, 8>(Ls, n, p, x, ys, M, s);
+  if (p.bn == 128) return launch_bn<128, 6>(Ls, n, p, x, ys, M, s);
+  return launch_bn<256, 4>(Ls, n, p, x, ys, M, s);
+}
+
 unisvq_status launch_prefill(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
-  const PrefillPlan p = plan_prefill(L, M);
-  if (p.bn == 64) return launch_bn<64, 8>(L, p, x, y, M, s);
-  if (p.bn == 128) return launch_bn<128, 6>(L, p, x, y, M, s);
-  return launch_bn<256, 4>(L, p, x, y, M, s);
+  void* ys[1] = {y};
+  return launch_prefill_group(&L, 1, x, ys, M, s);
 }
 
 }  // namespace unisvq

@@ -703,6 +703,10 @@ static unisvq_status group_inner(const unisvq_handle* hs, int n, int kernel, con
       if (!gemv_rows_supported(Ls[i], M < 4 ? M : 4)) return UNISVQ_ERR_UNSUPPORTED;
     return launch_gemv_rows_group(Ls, n, x, ys, M, s);
   }
+  // the prefill GEMM: one persistent launch over every layer's tiles where the
+  // layers allow it, else layer by layer below
+  if (kernel == UNISVQ_KERNEL_PREFILL && prefill_group_supported(Ls, n, M))
+    return launch_prefill_group(Ls, n, x, ys, M, s);
   for (int i = 0; i < n; ++i) {
     const unisvq_status st = linear_inner(hs[i], kernel, x, ys[i], M, s, false);
     if (st != UNISVQ_OK) return st;
@@ -760,10 +764,15 @@ static void describe_launch(const unisvq_layer* const* Ls, int n, int kernel, in
     const int chunks = (m + 15) / 16;
     info->launches = 2 * chunks;   // fold kernel + streaming kernel per 16 tokens
     info->grid_ctas = p.ks * nb * chunks;
-  } else {
-    const PrefillPlan p = plan_prefill(h, m);
+  } else if (prefill_group_supported(Ls, n, m)) {   // one launch over every layer's tiles
+    const PrefillPlan p = plan_prefill_group(Ls, n, m);
     info->split_k = 1;
-    info->grid_ctas = p.grid * n;
+    info->grid_ctas = p.grid;
+    info->launches = 1;
+  } else {
+    info->split_k = 1;
+    info->grid_ctas = 0;
+    for (int i = 0; i < n; ++i) info->grid_ctas += plan_prefill(Ls[i], m).grid;
     info->launches = n;
   }
 }

@@ -218,6 +218,55 @@ def test_prefill_parity(d, N, K):
     layer.close()
 
 
+@pytest.mark.parametrize("d", [1, 2, 4])
+def test_prefill_group_one_launch(d):
+    """Layers that share x (q/k/v-like, ragged N) in one persistent prefill
+    launch: every tile computes exactly what the layer's own launch computes,
+    so the outputs are bit-identical to per-layer calls and meet the oracle."""
+    K = 1024
+    shapes = [(520, K), (200, K), (1000, K), (128, K)]
+    layers, data = [], []
+    for i, (N, _) in enumerate(shapes):
+        c, A, B = synth.layer_inputs(8, 85 + i, 0, 0, N, K, d)
+        layers.append(binding.UniSVQLinear(c, A, B))
+        data.append((c, A, B))
+    for n in (2, 3, 4):
+        q = binding.query_group(layers[:n], 300)
+        assert q["kernel"] == binding.KERNEL_PREFILL and q["launches"] == 1
+    for M in (65, 300, 777):
+        xb = synth.activations(8, 85, M, M, K)
+        x = to_dev(xb)
+        got = binding.linear_group(layers, x, kernel=binding.KERNEL_PREFILL)
+        assert binding.sync_status() == binding.OK
+        for l, y, (c, A, B) in zip(layers, got, data):
+            yl = l.forward(x, kernel=binding.KERNEL_PREFILL)
+            assert binding.sync_status() == binding.OK
+            assert np.array_equal(y.view(torch.int16).cpu().numpy(), yl.view(torch.int16).cpu().numpy())
+            check(y.float().cpu().numpy().astype(np.float64), xb, c, A, B)
+    for l in layers:
+        l.close()
+
+
+def test_prefill_group_falls_back_per_layer():
+    """Mixed d (2 and 4) or a d = 8 layer: one prefill launch per layer."""
+    K = 512
+    mk = lambda i, N, d: binding.UniSVQLinear(*synth.layer_inputs(8, 90 + i, 0, 0, N, K, d))
+    l2, l4, l8 = mk(0, 256, 2), mk(1, 384, 4), mk(2, 128, 8)
+    for grp in ([l2, l4], [l2, l8]):
+        q = binding.query_group(grp, 200)
+        assert q["kernel"] == binding.KERNEL_PREFILL and q["launches"] == 2
+    xb = synth.activations(8, 90, 200, 200, K)
+    x = to_dev(xb)
+    for grp in ([l2, l4], [l8, l2]):
+        ys = binding.linear_group(grp, x)
+        assert binding.sync_status() == binding.OK
+        for l, y in zip(grp, ys):
+            yl = l.forward(x, kernel=binding.KERNEL_PREFILL)
+            assert np.array_equal(y.view(torch.int16).cpu().numpy(), yl.view(torch.int16).cpu().numpy())
+    for l in (l2, l4, l8):
+        l.close()
+
+
 def test_d8_layers_dispatch_to_the_prefill_kernel():
     """d = 8 (the paper's ablation length): above 64 tokens the library picks
     the prefill GEMM, whose converters add two quad-table rows per vector
