@@ -584,9 +584,11 @@ __global__ void __launch_bounds__(kPfThreads, 1)
                     // w = T_0[z0 z1 z2 z3] + T_1[z4 z5 z6 z7] (quad tables, fp32)
                     const uint32_t i0 = (e0 & 3u) | ((e0 >> 6) & 0xCu) | ((e0 >> 12) & 0x30u) | ((e0 >> 18) & 0xC0u);
                     const uint32_t i1 = (e1 & 3u) | ((e1 >> 6) & 0xCu) | ((e1 >> 12) & 0x30u) | ((e1 >> 18) & 0xC0u);
+                    // (a row's two halves are swapped when bit 2 of its index is set)
                     const uint32_t t0 = lut_s + i0 * 32, t1 = lut_s + 8192 + i1 * 32;
-                    const float4 a0 = lds128f(t0), a1 = lds128f(t0 + 16);
-                    const float4 b0 = lds128f(t1), b1 = lds128f(t1 + 16);
+                    const uint32_t s0 = (i0 << 2) & 16u, s1 = (i1 << 2) & 16u;
+                    const float4 a0 = lds128f(t0 + s0), a1 = lds128f(t0 + (s0 ^ 16u));
+                    const float4 b0 = lds128f(t1 + s1), b1 = lds128f(t1 + (s1 ^ 16u));
                     o0 = pack_bf16x2(a0.x + b0.x, a0.y + b0.y);
                     o1 = pack_bf16x2(a0.z + b0.z, a0.w + b0.w);
                     o2 = pack_bf16x2(a1.x + b1.x, a1.y + b1.y);

@@ -180,6 +180,9 @@ unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, cons
     // per coordinate quad q, T_q[z_4q | z_4q+1 << 2 | z_4q+2 << 4 | z_4q+3 << 6][r]
     // = sum_c A[r][4q + c] z_4q+c (+ B[r] for q = 0), each exact in fp64 and
     // rounded once to fp32; the prefill GEMM adds the two rows of a vector in fp32.
+    // Row v is 32 bytes, entries r = 0..3 and 4..7 in its two 16-byte halves,
+    // swapped when bit 2 of v is set: a warp's loads of one half then spread
+    // over all eight 16-byte bank groups instead of four.
     tlut.resize(4096);
     for (int qd = 0; qd < 2; ++qd)
       for (int v = 0; v < 256; ++v)
@@ -187,7 +190,8 @@ unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, cons
           double t = qd == 0 ? B[r] : 0.0;
           for (int c = 0; c < 4; ++c) t += A[r * 8 + 4 * qd + c] * ((v >> (2 * c)) & 3);
           const float f = static_cast<float>(t);
-          std::memcpy(&tlut[static_cast<size_t>(qd * 256 + v) * 8 + r], &f, sizeof(float));
+          const int half = (r >> 2) ^ ((v >> 2) & 1);
+          std::memcpy(&tlut[static_cast<size_t>(qd * 256 + v) * 8 + 4 * half + (r & 3)], &f, sizeof(float));
         }
   } else if (d == 8 || bits != 2) {   // the prefill GEMM takes no table for these
     tlut.assign(1, 0u);
