@@ -791,6 +791,8 @@ def run_prefill(torch, binding, peaks, args, stream):
             codes, A, B = synth.layer_inputs_grouped(0, 2, 0, pi, N, K, dg)
             glayers.append(b.UniSVQLinear(codes, A, B, group_cols=128))
         per_group[dg] = time_prefill_layers(torch, b, shapes, glayers, xs, ys, M, reps, stream)
+        if dg == 2:
+            per_group["calls"] = time_prefill_groups(torch, b, shapes, glayers, xs, M, reps, stream)
         for l in glayers:
             l.close()
     # the same set with 3-bit codes (per-matrix maps)
@@ -815,6 +817,7 @@ def run_prefill(torch, binding, peaks, args, stream):
                       f"{group_launches} prefill launches"),
             "TFLOP/s_one_call_per_projection": tflops_single,
             "per_group_maps_TFLOP/s": flops * reps / per_group[2] / 1e12,
+            "per_group_maps_group_calls_TFLOP/s": flops * reps / per_group["calls"] / 1e12,
             "per_group_maps_d4_TFLOP/s": flops * reps / per_group[4] / 1e12,
             "bits3_TFLOP/s": flops * reps / t3 / 1e12,
             "d8_TFLOP/s": flops * reps / t8 / 1e12,
@@ -822,6 +825,28 @@ def run_prefill(torch, binding, peaks, args, stream):
             "us_per_layer_set": tg / reps * 1e6, "per_projection": per,
             "cublas_bf16_dense_TFLOP/s": flops * reps / td / 1e12,
             "kernel": "prefill_kernel (tcgen05)"}
+
+
+def time_prefill_groups(torch, b, shapes, layers, xs, M, reps, stream):
+    """Seconds for `reps` passes of the set as a model issues it (q/k/v and
+    gate/up as one group call each, forced to the prefill GEMM)."""
+    yp = [torch.empty((M, N), dtype=torch.bfloat16, device="cuda") for _, N, _ in shapes]
+
+    def group_pass():
+        sp = torch.cuda.current_stream().cuda_stream
+        for grp in GROUPS_7B:
+            K = shapes[grp[0]][2]
+            st = b.linear_group_ptr([layers[i] for i in grp], xs[K].data_ptr(), [yp[i].data_ptr() for i in grp],
+                                    M, sp, b.KERNEL_PREFILL)
+            if st != 0:
+                raise RuntimeError(b.status_string(st))
+    with torch.cuda.stream(stream):
+        group_pass()
+    torch.cuda.synchronize()
+    gg = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gg, stream=stream):
+        group_pass()
+    return time_graphs(torch, [gg], reps, 3, stream)
 
 
 def time_prefill_layers(torch, b, shapes, glayers, xs, ys, M, reps, stream):

@@ -194,10 +194,10 @@ unisvq_status unisvq_linear_force(unisvq_handle h, int kernel, const void* x, vo
  * the q, k, v projections or the gate and up projections of one transformer
  * block. The paper defines the layer, not this grouping; it is a launch
  * convenience: for M <= 64 the n layers share each kernel launch (the row
- * blocks of the layers side by side); above, per-matrix 2-bit layers with one
- * d <= 4 share one persistent prefill launch (the tiles of every layer, each
- * layer with its own codeword table), and other layers run one unisvq_linear
- * each.
+ * blocks of the layers side by side); above, 2-bit layers with one d <= 4,
+ * all per-matrix or all per-group, share one persistent prefill launch (the
+ * tiles of every layer, each with its own table or maps), and other layers
+ * run one unisvq_linear each.
  *   hs : n handles on the current device, all with the same K
  *   n  : 1 .. UNISVQ_MAX_GROUP
  *   x  : device, [M][K] bf16, 16-byte aligned (shared by all layers)

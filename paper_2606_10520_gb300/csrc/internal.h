@@ -93,7 +93,8 @@ bool prefill_supported(const unisvq_layer* L, int M);
 PrefillPlan plan_prefill(const unisvq_layer* L, int M);
 unisvq_status launch_prefill(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
 // Several layers that read the same x in one persistent launch (their tiles
-// one after the other): per-matrix 2-bit layers with one d <= 4 and one K.
+// one after the other): 2-bit layers with one d <= 4 and one K, all
+// per-matrix or all per-group.
 bool prefill_group_supported(const unisvq_layer* const* Ls, int n, int M);
 PrefillPlan plan_prefill_group(const unisvq_layer* const* Ls, int n, int M);
 unisvq_status launch_prefill_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,

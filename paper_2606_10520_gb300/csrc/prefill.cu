@@ -51,7 +51,8 @@ struct PrefillArgs {
   int N[kPfMaxLayers];
   int tile0[kPfMaxLayers];
   int nlayers;
-  const uint16_t* meta;  // per-group layers (d = 2): fp16 [Np/128][KT][128][6] (A row-major, B), else null
+  // per-group layers: fp16 [Np/128][KT][128][d*d + d] (A row-major, B) per layer, else null
+  const uint16_t* meta[kPfMaxLayers];
   const uint8_t* hi;     // 3-bit codes (d <= 2): the high-bit plane; the table has 64 pairs, index z0 | z1 << 3
   int M, K, KT, d;
   int nkb;               // k-blocks of 64 columns: ceil(K / 64)
@@ -233,7 +234,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   }
   // Codeword table -> shared memory (per-matrix maps only; per-group layers
   // build theirs in the converters).
-  if (!a.meta) {   // layer i's table at kOffLut + 2 KB i (one layer for d = 8: 16 KB)
+  if (!a.meta[0]) {   // layer i's table at kOffLut + 2 KB i (one layer for d = 8: 16 KB)
     const int words = a.hi ? 64 : (a.d == 8 ? 4096 : (a.d == 4 ? 512 : 16));
 #pragma unroll
     for (int l = 0; l < kPfMaxLayers; ++l) {
@@ -320,7 +321,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     const int r0 = 16 * c + g, r1 = r0 + 8;
     const uint32_t lut_base = sbase + C::kOffLut;   // layer i's table at + 2 KB i
     int it = 0;
-    if (a.meta && a.d == 4) {
+    if (a.meta[0] && a.d == 4) {
       // Per-(row, 128-column group) maps, d = 4: 256 codewords per row and group
       // are too many to tabulate per k-tile, so each output is formed directly,
       // sum_c' A[c][c'] z_c' + B[c] in fp32. Natural columns 64 h + 8 cc + j
@@ -335,7 +336,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
         const uint8_t* rbase =
             pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
-        const uint32_t* mbase = reinterpret_cast<const uint32_t*>(a.meta + static_cast<size_t>(n_blk) * a.KT * kBM * 20 +
+        const uint32_t* mbase = reinterpret_cast<const uint32_t*>(pick_layer(a.meta, li) + static_cast<size_t>(n_blk) * a.KT * kBM * 20 +
                                                                   static_cast<size_t>(16 * c) * 20);
         const int nkt = (a.nkb + 1) >> 1;
         auto load_codes = [&](int kt) -> uint4 {
@@ -420,7 +421,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
           if (lane == 0 && ok) mbar_arrive(afull(s));
         }
       }
-    } else if (a.meta) {
+    } else if (a.meta[0]) {
       // Per-(row, 128-column group) maps, d = 2, codes permuted within each group
       // (pack_codes_grouped_host): coordinate c of vector v = 16 s + 4 t + e(b)
       // sits in the word of half c at shift s and byte b. The A tile keeps the
@@ -435,7 +436,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
         const uint8_t* rbase =
             pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
-        const uint16_t* mbase = a.meta + static_cast<size_t>(n_blk) * a.KT * kBM * 6;
+        const uint16_t* mbase = pick_layer(a.meta, li) + static_cast<size_t>(n_blk) * a.KT * kBM * 6;
         const int nkt = (a.nkb + 1) >> 1;
         auto load_codes = [&](int kt) -> uint4 {
           return kt < nkt ? __ldg(reinterpret_cast<const uint4*>(rbase + static_cast<size_t>(kt) * kTileBytes))
@@ -711,11 +712,11 @@ unisvq_status launch_bn(const unisvq_layer* const* Ls, int n, const PrefillPlan&
     a.lut[i] = Ls[i]->tlut;
     a.y[i] = static_cast<uint16_t*>(ys[i]);
     a.N[i] = Ls[i]->N;
+    a.meta[i] = Ls[i]->grouped ? Ls[i]->meta : nullptr;
     a.tile0[i] = tile;
     tile += (Ls[i]->Np / kBM) * a.mtiles;
   }
   a.nlayers = n;
-  a.meta = L->grouped ? L->meta : nullptr;
   a.hi = L->bits == 3 ? L->hi : nullptr;
   a.M = M;
   a.K = L->K;
@@ -744,11 +745,12 @@ bool prefill_supported(const unisvq_layer* L, int M) {
 bool prefill_group_supported(const unisvq_layer* const* Ls, int n, int M) {
   if (n < 1 || n > kPfMaxLayers) return false;
   if (n == 1) return prefill_supported(Ls[0], M);
-  // several layers in one launch: per-matrix 2-bit layers with one d <= 4 and
-  // one K, whose tables (<= 2 KB each) share the table region
+  // several layers in one launch: 2-bit layers with one d <= 4 and one K, all
+  // per-matrix (their tables, <= 2 KB each, share the table region) or all
+  // per-group (each converter reads its tile's layer's maps)
   for (int i = 0; i < n; ++i)
-    if (Ls[i]->grouped || Ls[i]->bits != 2 || Ls[i]->d > 4 || Ls[i]->d != Ls[0]->d || Ls[i]->K != Ls[0]->K ||
-        !prefill_supported(Ls[i], M))
+    if (Ls[i]->grouped != Ls[0]->grouped || Ls[i]->bits != 2 || Ls[i]->d > 4 || Ls[i]->d != Ls[0]->d ||
+        Ls[i]->K != Ls[0]->K || !prefill_supported(Ls[i], M))
       return false;
   return true;
 }

@@ -671,7 +671,10 @@ static unisvq_status group_inner(const unisvq_handle* hs, int n, int kernel, con
     if (ngrouped != n) return UNISVQ_ERR_UNSUPPORTED;
     bool pf = kernel == UNISVQ_KERNEL_PREFILL || (kernel == UNISVQ_KERNEL_AUTO && M > 64);
     for (int i = 0; i < n && pf; ++i) pf = prefill_supported(hs[i], M);
-    if (pf || kernel == UNISVQ_KERNEL_PREFILL) {   // the prefill GEMM, layer by layer
+    if (pf || kernel == UNISVQ_KERNEL_PREFILL) {   // the prefill GEMM: one launch where it can, else layer by layer
+      const unisvq_layer* Lp[UNISVQ_MAX_GROUP];
+      for (int i = 0; i < n; ++i) Lp[i] = hs[i];
+      if (prefill_group_supported(Lp, n, M)) return launch_prefill_group(Lp, n, x, ys, M, s);
       for (int i = 0; i < n; ++i) {
         const unisvq_status st = linear_inner(hs[i], kernel, x, ys[i], M, s, false);
         if (st != UNISVQ_OK) return st;

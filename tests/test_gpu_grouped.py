@@ -229,17 +229,27 @@ def test_grouped_prefill_only_for_d2_and_d4(d):
     layer.close()
 
 
-def test_grouped_group_call_at_prefill_sizes():
-    K, d, M = 1024, 2, 96
-    shapes = [(512, K), (256, K)]
+@pytest.mark.parametrize("d", [2, 4])
+def test_grouped_group_call_at_prefill_sizes(d):
+    """Per-group layers that share x run one persistent prefill launch (each
+    converter reading its tile's layer's maps): bit-identical to per-layer
+    launches, and within the oracle bars."""
+    K = 1024
+    shapes = [(512, K), (256, K), (200, K)]
     made = [synth.layer_inputs_grouped(9, 42, i, 0, N, K_, d) for i, (N, K_) in enumerate(shapes)]
     layers = [binding.UniSVQLinear(c, A, B, group_cols=GC) for c, A, B in made]
-    assert binding.query_group(layers, M)["kernel"] == binding.KERNEL_PREFILL
-    xb = synth.activations(9, 42, M, M, K)
-    ys = binding.linear_group(layers, to_dev(xb))
-    assert binding.sync_status() == binding.OK
-    for (c, A, B), y in zip(made, ys):
-        check(y.float().cpu().numpy().astype(np.float64), xb, c, A, B)
+    for M in (96, 300):
+        q = binding.query_group(layers, M)
+        assert q["kernel"] == binding.KERNEL_PREFILL and q["launches"] == 1
+        xb = synth.activations(9, 42, M, M, K)
+        x = to_dev(xb)
+        ys = binding.linear_group(layers, x)
+        assert binding.sync_status() == binding.OK
+        for layer, (c, A, B), y in zip(layers, made, ys):
+            yl = layer.forward(x, kernel=binding.KERNEL_PREFILL)
+            assert binding.sync_status() == binding.OK
+            assert np.array_equal(y.view(torch.int16).cpu().numpy(), yl.view(torch.int16).cpu().numpy())
+            check(y.float().cpu().numpy().astype(np.float64), xb, c, A, B)
     for layer in layers:
         layer.close()
 
