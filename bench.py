@@ -803,6 +803,13 @@ def run_prefill(torch, binding, peaks, args, stream):
     t3 = time_prefill_layers(torch, b, shapes, l3, xs, ys, M, reps, stream)
     for l in l3:
         l.close()
+    l34 = []   # 3-bit codes, d = 4 (pair tables)
+    for pi, (_, N, K) in enumerate(shapes):
+        codes, A, B = synth.layer_inputs_bits(0, 2, 0, pi, N, K, 4, 3)
+        l34.append(b.UniSVQLinear(codes, A, B, bits=3))
+    t34 = time_prefill_layers(torch, b, shapes, l34, xs, ys, M, reps, stream)
+    for l in l34:
+        l.close()
     # the same set with vectors of length 8 (per-matrix maps, pair tables)
     l8 = []
     for pi, (_, N, K) in enumerate(shapes):
@@ -820,6 +827,7 @@ def run_prefill(torch, binding, peaks, args, stream):
             "per_group_maps_group_calls_TFLOP/s": flops * reps / per_group["calls"] / 1e12,
             "per_group_maps_d4_TFLOP/s": flops * reps / per_group[4] / 1e12,
             "bits3_TFLOP/s": flops * reps / t3 / 1e12,
+            "bits3_d4_TFLOP/s": flops * reps / t34 / 1e12,
             "d8_TFLOP/s": flops * reps / t8 / 1e12,
             "frac_of_measured_bf16_sustained": tflops / peaks["bf16_tflops_sustained"],
             "us_per_layer_set": tg / reps * 1e6, "per_projection": per,

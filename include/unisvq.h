@@ -132,9 +132,11 @@ unisvq_status unisvq_pack(const uint8_t* codes, const uint16_t* A_f16, const uin
  * the chunk and its bit 4b + s is bit 2 of the code at bits [8b+2s+1 : 8b+2s]
  * of that word. 3-bit layers take d in {1, 2, 4} and run the GEMV
  * (UNISVQ_KERNEL_GEMV, 32 tokens per launch) up to 64 tokens; above that,
- * layers with d <= 2 run the prefill GEMM (also forceable), d = 4 stays on
- * the GEMV. Other forced kernels return UNSUPPORTED. Errors as unisvq_pack, plus UNSUPPORTED (bits, or
- * bits = 3 with d = 8) and INVALID_ARG (a code >= 2^bits).
+ * the prefill GEMM (also forceable): exact codewords from a 64-pair table
+ * for d <= 2, and for d = 4 the fp32 sum of two 64-row pair-table rows
+ * rounded once to bf16. Other forced kernels return UNSUPPORTED. Errors as
+ * unisvq_pack, plus UNSUPPORTED (bits, or bits = 3 with d = 8) and
+ * INVALID_ARG (a code >= 2^bits).
  */
 unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, const uint16_t* B_f16,
                                int N, int K, int d, int bits, void* stream, unisvq_handle* out);

@@ -235,7 +235,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   // Codeword table -> shared memory (per-matrix maps only; per-group layers
   // build theirs in the converters).
   if (!a.meta[0]) {   // layer i's table at kOffLut + 2 KB i (one layer for d = 8: 16 KB)
-    const int words = a.hi ? 64 : (a.d == 8 ? 4096 : (a.d == 4 ? 512 : 16));
+    const int words = a.hi ? (a.d == 4 ? 512 : 64) : (a.d == 8 ? 4096 : (a.d == 4 ? 512 : 16));
 #pragma unroll
     for (int l = 0; l < kPfMaxLayers; ++l) {
       if (l < a.nlayers) {
@@ -510,12 +510,14 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         }
       }
     } else {
-      // Per-matrix maps. The loop is compiled three times (HI = 3-bit codes,
-      // D8 = vectors of 8 through the pair tables, or neither) so that the
-      // common loop carries no high-bit loads and no extra branches.
-      auto convert = [&](auto hi_tag, auto d8_tag) {
+      // Per-matrix maps. The loop is compiled four times (HI = 3-bit codes,
+      // with P4 = d = 4 through two pair tables; D8 = 2-bit vectors of 8
+      // through the quad tables; or none of these) so that each loop carries
+      // only its own loads and no extra branches.
+      auto convert = [&](auto hi_tag, auto d8_tag, auto p4_tag) {
         constexpr bool HI = decltype(hi_tag)::value;
         constexpr bool D8 = decltype(d8_tag)::value;
+        constexpr bool P4 = decltype(p4_tag)::value;
         for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
           const int li = tile_layer(a, tile);
           const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
@@ -576,10 +578,25 @@ __global__ void __launch_bounds__(kPfThreads, 1)
                     auto code3 = [&](uint32_t eu, int u, int b) -> uint32_t {
                       return ((eu >> (8 * b)) & 3u) | (((hq >> (4 * b + 2 * e + u)) & 1u) << 2);
                     };
-                    o0 = lds32(lut_s + ((code3(e0, 0, 0) | (code3(e0, 0, 1) << 3)) << 2));
-                    o1 = lds32(lut_s + ((code3(e0, 0, 2) | (code3(e0, 0, 3) << 3)) << 2));
-                    o2 = lds32(lut_s + ((code3(e1, 1, 0) | (code3(e1, 1, 1) << 3)) << 2));
-                    o3 = lds32(lut_s + ((code3(e1, 1, 2) | (code3(e1, 1, 3) << 3)) << 2));
+                    const uint32_t p00 = code3(e0, 0, 0) | (code3(e0, 0, 1) << 3);
+                    const uint32_t p01 = code3(e0, 0, 2) | (code3(e0, 0, 3) << 3);
+                    const uint32_t p10 = code3(e1, 1, 0) | (code3(e1, 1, 1) << 3);
+                    const uint32_t p11 = code3(e1, 1, 2) | (code3(e1, 1, 3) << 3);
+                    if constexpr (P4) {
+                      // columns 8cc .. +3 and 8cc + 4 .. +7 are two vectors; their coordinate
+                      // pairs index two 64-row fp32 tables: w = T_0[z0 z1] + T_1[z2 z3]
+                      const float4 va = lds128f(lut_s + p00 * 16), vb = lds128f(lut_s + 1024 + p01 * 16);
+                      const float4 vc = lds128f(lut_s + p10 * 16), vd = lds128f(lut_s + 1024 + p11 * 16);
+                      o0 = pack_bf16x2(va.x + vb.x, va.y + vb.y);
+                      o1 = pack_bf16x2(va.z + vb.z, va.w + vb.w);
+                      o2 = pack_bf16x2(vc.x + vd.x, vc.y + vd.y);
+                      o3 = pack_bf16x2(vc.z + vd.z, vc.w + vd.w);
+                    } else {
+                      o0 = lds32(lut_s + (p00 << 2));
+                      o1 = lds32(lut_s + (p01 << 2));
+                      o2 = lds32(lut_s + (p10 << 2));
+                      o3 = lds32(lut_s + (p11 << 2));
+                    }
                   } else if constexpr (D8) {
                     // the chunk is one vector: coordinates 0..3 in bytes 0..3 of e0, 4..7 of e1;
                     // w = T_0[z0 z1 z2 z3] + T_1[z4 z5 z6 z7] (quad tables, fp32)
@@ -615,9 +632,10 @@ __global__ void __launch_bounds__(kPfThreads, 1)
           }
         }
       };
-      if (a.hi) convert(std::true_type{}, std::false_type{});
-      else if (a.d == 8) convert(std::false_type{}, std::true_type{});
-      else convert(std::false_type{}, std::false_type{});
+      if (a.hi && a.d == 4) convert(std::true_type{}, std::false_type{}, std::true_type{});
+      else if (a.hi) convert(std::true_type{}, std::false_type{}, std::false_type{});
+      else if (a.d == 8) convert(std::false_type{}, std::true_type{}, std::false_type{});
+      else convert(std::false_type{}, std::false_type{}, std::false_type{});
     }
   } else {
     // ---------------- epilogue ----------------
@@ -736,9 +754,10 @@ int pick_bn(int M) { return M <= 64 ? 64 : (M <= 128 ? 128 : 256); }
 
 bool prefill_supported(const unisvq_layer* L, int M) {
   // per-group layers: d = 2 (a 16-pair table per row and group) or d = 4 (direct
-  // sums); 3-bit layers: d <= 2 (a 64-pair table; 8^4 quads would not fit);
-  // per-matrix 2-bit layers: every d (d = 8 through two quad tables)
-  const bool maps_ok = L->grouped ? (L->d == 2 || L->d == 4) : (L->bits == 3 ? L->d <= 2 : true);
+  // sums); 3-bit layers: d <= 4 (a 64-pair codeword table for d <= 2, two
+  // 64-row pair tables for d = 4); per-matrix 2-bit layers: every d (d = 8
+  // through two quad tables)
+  const bool maps_ok = L->grouped ? (L->d == 2 || L->d == 4) : (L->bits == 3 ? L->d <= 4 : true);
   return M > 0 && maps_ok && (L->K % 8) == 0 && get_encode() != nullptr;
 }
 

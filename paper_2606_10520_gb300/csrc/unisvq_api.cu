@@ -175,6 +175,19 @@ unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, cons
       const double w1 = d == 2 ? cb[static_cast<size_t>(lo | (hi << 3)) * 2 + 1] : cb[hi];
       tlut[v] = bf(w0) | (bf(w1) << 16);
     }
+  } else if (bits == 3 && d == 4) {
+    // 8^4 codewords would take 32 KB: two partial tables, one per coordinate
+    // pair p, T_p[z_2p | z_2p+1 << 3][r] = A[r][2p] z_2p + A[r][2p+1] z_2p+1
+    // (+ B[r] for p = 0), 64 rows of 4 fp32 each, exact in fp64 and rounded
+    // once; the prefill GEMM adds the two rows of a vector in fp32.
+    tlut.resize(512);
+    for (int pr = 0; pr < 2; ++pr)
+      for (int v = 0; v < 64; ++v)
+        for (int r = 0; r < 4; ++r) {
+          const double t = A[r * 4 + 2 * pr] * (v & 7) + A[r * 4 + 2 * pr + 1] * (v >> 3) + (pr == 0 ? B[r] : 0.0);
+          const float f = static_cast<float>(t);
+          std::memcpy(&tlut[static_cast<size_t>(pr * 64 + v) * 4 + r], &f, sizeof(float));
+        }
   } else if (d == 8 && bits == 2) {
     // 4^8 codewords are too many for shared memory: two partial tables, one
     // per coordinate quad q, T_q[z_4q | z_4q+1 << 2 | z_4q+2 << 4 | z_4q+3 << 6][r]

@@ -122,11 +122,12 @@ def test_3bit_full_size_sampled_rows(N, K):
     layer.close()
 
 
-@pytest.mark.parametrize("d", [1, 2])
+@pytest.mark.parametrize("d", [1, 2, 4])
 @pytest.mark.parametrize("N,K", [(256, 1024), (520, 1000), (384, 4096)])
 def test_3bit_prefill_parity(d, N, K):
-    """3-bit layers with d <= 2 run the tcgen05 prefill GEMM above 64 tokens
-    (64-pair codeword table, high bits from the bit plane)."""
+    """3-bit layers run the tcgen05 prefill GEMM above 64 tokens (64-pair
+    codeword table for d <= 2, two 64-row pair tables for d = 4, high bits
+    from the bit plane)."""
     codes, A, B, layer = make(N, K, d, 6)
     Ms = (65, 300)
     xall = synth.activations(6, 60, N + d, sum(Ms), K)
@@ -142,7 +143,7 @@ def test_3bit_prefill_parity(d, N, K):
     layer.close()
 
 
-@pytest.mark.parametrize("d", [1, 2])
+@pytest.mark.parametrize("d", [1, 2, 4])
 def test_3bit_prefill_integer_case_bit_exact(d):
     g = np.random.default_rng(50 + d)
     N, K = 256, 512
@@ -158,14 +159,13 @@ def test_3bit_prefill_integer_case_bit_exact(d):
     layer.close()
 
 
-def test_3bit_d4_stays_on_the_gemv():
+def test_3bit_d4_dispatch():
+    """d = 4: the GEMV up to 64 tokens, the prefill GEMM above (pair tables)."""
     codes, A, B, layer = make(256, 512, 4, 7)
-    assert layer.query(200)["kernel"] == binding.KERNEL_GEMV
-    x = torch.zeros((100, 512), dtype=torch.bfloat16, device="cuda")
-    y = torch.zeros((100, 256), dtype=torch.bfloat16, device="cuda")
-    stream = torch.cuda.current_stream().cuda_stream
-    assert layer.forward_ptr(x.data_ptr(), y.data_ptr(), 100, stream, binding.KERNEL_PREFILL) == binding.ERR_UNSUPPORTED
+    assert layer.query(64)["kernel"] == binding.KERNEL_GEMV
+    assert layer.query(200)["kernel"] == binding.KERNEL_PREFILL
     xb = synth.activations(7, 60, 4, 100, 512)
     yr, S = oracle.linear(xb, codes, A, B)
     assert oracle.compare(run(layer, xb), yr, S)["ok"]
+    assert oracle.compare(run(layer, xb, binding.KERNEL_GEMV), yr, S)["ok"]
     layer.close()
