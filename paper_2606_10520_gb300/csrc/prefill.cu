@@ -38,15 +38,18 @@ constexpr int kATileBytes = kBM * 128;   // 16 KB
 constexpr int kConvWarp0 = 2;
 constexpr int kEpiWarp0 = 10;
 
-// Layers of one launch (several only for per-matrix 2-bit layers with one
-// d <= 4 that read the same x): their tiles are numbered one layer after the
-// other, layer i from tile0[i] on, and each keeps its own codeword table in a
-// 2 KB slot of shared memory.
+// Layers of one launch (several only for 2-bit layers with one d <= 4 that
+// read the same x, all per-matrix or all per-group): their tiles are numbered
+// one layer after the other, layer i from tile0[i] on; a per-matrix layer
+// keeps its codeword table in a 2 KB slot of shared memory, a per-group layer
+// has its own maps.
 constexpr int kPfMaxLayers = UNISVQ_MAX_GROUP;
 
 struct PrefillArgs {
   const uint8_t* codes[kPfMaxLayers];
-  const uint32_t* lut[kPfMaxLayers];   // d <= 2: 16 x bf16x2 pair codewords; d == 4: 256 x 4 bf16; d == 8: [2][256][8] fp32 quad tables
+  // d <= 2: 16 x bf16x2 pair codewords (3-bit: 64); d == 4: 256 x 4 bf16 (3-bit: [2][64][4] fp32
+  // pair tables); d == 8: [2][256][8] fp32 quad tables
+  const uint32_t* lut[kPfMaxLayers];
   uint16_t* y[kPfMaxLayers];
   int N[kPfMaxLayers];
   int tile0[kPfMaxLayers];
