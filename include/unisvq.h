@@ -307,6 +307,27 @@ const char* unisvq_status_string(unisvq_status s);
 /* Bytes of the packed code array for an N x K layer (see layout above). */
 size_t unisvq_packed_code_bytes(int N, int K);
 
+/* The prefill GEMM's shared-memory table of a per-matrix layer with this A,
+ * B, d and bits, exactly as unisvq_pack builds it (host only). Every entry is
+ * the exact fp64 value rounded once:
+ *   bits 2, d <= 2: 16 words; word v = bf16 pair (low half first) for the
+ *     index v = z_k | z_k+1 << 2 of two adjacent columns: the codeword of the
+ *     vector (d = 2) or the codewords of z_k and z_k+1 (d = 1);
+ *   bits 2, d = 4: 512 words; quad v = z0 | z1 << 2 | z2 << 4 | z3 << 6 is the
+ *     bf16 codeword in words 2v (w0, w1) and 2v + 1 (w2, w3);
+ *   bits 2, d = 8: 4096 words of fp32, quad tables q = 0, 1 of 256 rows:
+ *     row v of table q holds sum_c A[r][4q + c] z_c(v) (+ B[r] for q = 0),
+ *     r = 0..7, at word 2048 q + 8 v + 4 h + (r % 4), h = r/4 XOR bit 2 of v;
+ *   bits 3, d <= 2: 64 words as for bits 2, d <= 2, index z_k | z_k+1 << 3;
+ *   bits 3, d = 4: 512 words of fp32, pair tables p = 0, 1 of 64 rows: word
+ *     256 p + 4 v + r holds A[r][2p] z_2p + A[r][2p+1] z_2p+1 (+ B[r] for
+ *     p = 0), v = z_2p | z_2p+1 << 3.
+ *   A_f16, B_f16: as for unisvq_pack; out: NULL to query *words only.
+ * Errors: INVALID_ARG (null A, B or words, d not in {1, 2, 4, 8}, bits not
+ * in {2, 3}, bits = 3 with d = 8, non-finite A/B, out_words too small), OOM. */
+unisvq_status unisvq_prefill_table_host(const uint16_t* A_f16, const uint16_t* B_f16, int d, int bits,
+                                        uint32_t* out, size_t out_words, size_t* words);
+
 /* Write the packed layout of `codes` ([N][K], each 0..3) into the host
  * buffer `packed` of unisvq_packed_code_bytes(N, K) bytes. */
 unisvq_status unisvq_pack_host(const uint8_t* codes, int N, int K, uint8_t* packed,

@@ -23,6 +23,7 @@ EXPORTS = [
     "unisvq_status_string", "unisvq_packed_code_bytes", "unisvq_pack_host", "unisvq_version",
     "unisvq_linear_group", "unisvq_linear_group_force", "unisvq_linear_noalloc", "unisvq_query_group",
     "unisvq_pack_grouped", "unisvq_set_rht", "unisvq_hadamard", "unisvq_pack_bits",
+    "unisvq_prefill_table_host",
 ]
 MAX_GROUP = 4
 
@@ -74,6 +75,7 @@ def load():
     lib.unisvq_packed_code_bytes.argtypes = [i, i]
     lib.unisvq_packed_code_bytes.restype = sz
     lib.unisvq_pack_host.argtypes = [vp, i, i, vp, sz]
+    lib.unisvq_prefill_table_host.argtypes = [vp, vp, i, i, vp, sz, ctypes.POINTER(sz)]
     lib.unisvq_version.argtypes = []
     _lib = lib
     return lib
@@ -96,6 +98,20 @@ def _stream_ptr(stream=None):
 
 def packed_code_bytes(N: int, K: int) -> int:
     return int(load().unisvq_packed_code_bytes(N, K))
+
+
+def prefill_table_host(A, B, d: int, bits: int = 2) -> np.ndarray:
+    """The prefill GEMM's table for this A (d x d), B (d), as unisvq_pack
+    builds it (unisvq_prefill_table_host; uint32 words)."""
+    a16 = np.ascontiguousarray(np.asarray(A, dtype=np.float16).reshape(-1)).view(np.uint16)
+    b16 = np.ascontiguousarray(np.asarray(B, dtype=np.float16).reshape(-1)).view(np.uint16)
+    words = ctypes.c_size_t(0)
+    _check(load().unisvq_prefill_table_host(a16.ctypes.data, b16.ctypes.data, int(d), int(bits), None, 0,
+                                            ctypes.byref(words)), "prefill_table_host")
+    out = np.zeros(words.value, dtype=np.uint32)
+    _check(load().unisvq_prefill_table_host(a16.ctypes.data, b16.ctypes.data, int(d), int(bits), out.ctypes.data,
+                                            out.size, ctypes.byref(words)), "prefill_table_host")
+    return out
 
 
 def pack_host(codes: np.ndarray) -> np.ndarray:

@@ -132,6 +132,8 @@ void pack_codes_grouped_host(const uint8_t* codes, int N, int K, int d, uint8_t*
 void pack_meta_grouped_host(const uint16_t* A_f16, const uint16_t* B_f16, int N, int K, int d, uint16_t* meta);
 // fp64 -> bf16 round-to-nearest-even (single rounding).
 uint16_t f64_to_bf16_rne(double v);
+// The prefill GEMM's table of a per-matrix layer (A row-major d x d, B; fp64).
+std::vector<uint32_t> prefill_table_host(const double* A, const double* B, int d, int bits);
 double f16_bits_to_f64(uint16_t h);
 
 }  // namespace unisvq

@@ -4,6 +4,7 @@
 #include <cmath>
 #include <cstdint>
 #include <cstring>
+#include <vector>
 
 #include "internal.h"
 
@@ -164,6 +165,78 @@ uint16_t f64_to_bf16_rne(double v) {
   }
   const uint32_t rounding = 0x7FFFu + ((u >> 16) & 1u);
   return static_cast<uint16_t>((u + rounding) >> 16);
+}
+
+// The prefill GEMM's shared-memory table of a per-matrix layer, indexed the
+// way its converter warps read code bytes (unisvq_prefill_table_host in
+// unisvq.h states the formats). Every entry is the exact fp64 value rounded
+// once, to bf16 (whole codewords) or to fp32 (partial sums that the
+// converters add).
+std::vector<uint32_t> prefill_table_host(const double* A, const double* B, int d, int bits) {
+  const int zmax = (1 << bits) - 1;
+  // the codeword of index v (coordinate c in bits [bits (c+1) - 1 : bits c]), row r
+  auto codeword = [&](int v, int r) {
+    double w = B[r];
+    for (int c = 0; c < d; ++c) w += A[r * d + c] * static_cast<double>((v >> (bits * c)) & zmax);
+    return w;
+  };
+  auto bf = [](double w) { return static_cast<uint32_t>(f64_to_bf16_rne(w)); };
+  auto f32 = [](double w) {
+    const float f = static_cast<float>(w);
+    uint32_t u;
+    std::memcpy(&u, &f, sizeof(u));
+    return u;
+  };
+  std::vector<uint32_t> t;
+  if (bits == 3 && d <= 2) {   // 64 bf16 pairs, index lo | hi << 3 for columns (k, k+1)
+    t.resize(64);
+    for (int v = 0; v < 64; ++v) {
+      const int lo = v & 7, hi = v >> 3;
+      const double w0 = d == 2 ? codeword(lo | (hi << 3), 0) : codeword(lo, 0);
+      const double w1 = d == 2 ? codeword(lo | (hi << 3), 1) : codeword(hi, 0);
+      t[v] = bf(w0) | (bf(w1) << 16);
+    }
+  } else if (bits == 3 && d == 4) {
+    // 8^4 codewords would take 32 KB: two pair tables, T_p[z_2p | z_2p+1 << 3][r]
+    // = A[r][2p] z_2p + A[r][2p+1] z_2p+1 (+ B[r] for p = 0), 64 rows of 4 fp32
+    t.resize(512);
+    for (int pr = 0; pr < 2; ++pr)
+      for (int v = 0; v < 64; ++v)
+        for (int r = 0; r < 4; ++r)
+          t[static_cast<size_t>(pr * 64 + v) * 4 + r] =
+              f32(A[r * 4 + 2 * pr] * (v & 7) + A[r * 4 + 2 * pr + 1] * (v >> 3) + (pr == 0 ? B[r] : 0.0));
+  } else if (bits == 2 && d == 8) {
+    // 4^8 codewords do not fit: two quad tables, T_q[z_4q | .. | z_4q+3 << 6][r]
+    // = sum_c A[r][4q + c] z_4q+c (+ B[r] for q = 0), 256 rows of 8 fp32; row v's
+    // 16-byte halves (r = 0..3, 4..7) are swapped when bit 2 of v is set, so a
+    // warp's loads of one half spread over all eight 16-byte bank groups
+    t.resize(4096);
+    for (int qd = 0; qd < 2; ++qd)
+      for (int v = 0; v < 256; ++v)
+        for (int r = 0; r < 8; ++r) {
+          double w = qd == 0 ? B[r] : 0.0;
+          for (int c = 0; c < 4; ++c) w += A[r * 8 + 4 * qd + c] * ((v >> (2 * c)) & 3);
+          const int half = (r >> 2) ^ ((v >> 2) & 1);
+          t[static_cast<size_t>(qd * 256 + v) * 8 + 4 * half + (r & 3)] = f32(w);
+        }
+  } else if (bits == 2 && d <= 2) {   // 16 bf16 pairs, index lo | hi << 2 for columns (k, k+1)
+    t.resize(16);
+    for (int v = 0; v < 16; ++v) {
+      const int lo = v & 3, hi = v >> 2;
+      const double w0 = d == 2 ? codeword(lo | (hi << 2), 0) : codeword(lo, 0);
+      const double w1 = d == 2 ? codeword(lo | (hi << 2), 1) : codeword(hi, 0);
+      t[v] = bf(w0) | (bf(w1) << 16);
+    }
+  } else if (bits == 2 && d == 4) {   // 256 bf16 quads, index z0 | z1 << 2 | z2 << 4 | z3 << 6
+    t.resize(512);
+    for (int v = 0; v < 256; ++v) {
+      t[2 * v] = bf(codeword(v, 0)) | (bf(codeword(v, 1)) << 16);
+      t[2 * v + 1] = bf(codeword(v, 2)) | (bf(codeword(v, 3)) << 16);
+    }
+  } else {   // no table (3-bit codes with d = 8 are not packed)
+    t.assign(1, 0u);
+  }
+  return t;
 }
 
 }  // namespace unisvq

@@ -69,6 +69,33 @@ size_t unisvq_packed_code_bytes(int N, int K) {
          static_cast<size_t>(round_up(K, kColPad) / kTileCols) * kTileBytes;
 }
 
+unisvq_status unisvq_prefill_table_host(const uint16_t* A_f16, const uint16_t* B_f16, int d, int bits,
+                                        uint32_t* out, size_t out_words, size_t* words) {
+  if (!A_f16 || !B_f16 || !words || (d != 1 && d != 2 && d != 4 && d != 8) || (bits != 2 && bits != 3) ||
+      (bits == 3 && d == 8))
+    return UNISVQ_ERR_INVALID_ARG;
+  double A[64], B[8];
+  for (int i = 0; i < d * d; ++i) {
+    A[i] = f16_bits_to_f64(A_f16[i]);
+    if (!std::isfinite(A[i])) return UNISVQ_ERR_INVALID_ARG;
+  }
+  for (int i = 0; i < d; ++i) {
+    B[i] = f16_bits_to_f64(B_f16[i]);
+    if (!std::isfinite(B[i])) return UNISVQ_ERR_INVALID_ARG;
+  }
+  std::vector<uint32_t> t;
+  try {
+    t = prefill_table_host(A, B, d, bits);
+  } catch (...) {
+    return UNISVQ_ERR_OOM;
+  }
+  *words = t.size();
+  if (!out) return UNISVQ_OK;
+  if (out_words < t.size()) return UNISVQ_ERR_INVALID_ARG;
+  std::memcpy(out, t.data(), t.size() * sizeof(uint32_t));
+  return UNISVQ_OK;
+}
+
 unisvq_status unisvq_pack_host(const uint8_t* codes, int N, int K, uint8_t* packed,
                                size_t packed_bytes) {
   if (!codes || !packed || N <= 0 || K <= 0) return UNISVQ_ERR_INVALID_ARG;
@@ -144,84 +171,26 @@ unisvq_status unisvq_pack_bits(const uint8_t* codes, const uint16_t* A_f16, cons
   // Rounded up so the activation scale never underestimates |x A|.
   L->colnorm = static_cast<float>(colnorm) * (1.0f + 1e-6f);
 
-  // Codebook of Eq. (def:unisvq): entry v holds A z(v) + B with z_c(v) the
-  // bit-field [bits (c+1) - 1 : bits c] of v, exact in fp64 and rounded once
-  // (to fp32 here, to bf16 below).
+  // Codebook of Eq. (def:unisvq) for the dequant hook: entry v holds A z(v) + B
+  // with z_c(v) the bit-field [bits (c+1) - 1 : bits c] of v, exact in fp64 and
+  // rounded once to fp32.
   const int E = 1 << (bits * d);
   L->lut_entries = E;
-  std::vector<double> cb(static_cast<size_t>(E) * d);
   std::vector<float> lut32(static_cast<size_t>(E) * d);
   for (int v = 0; v < E; ++v)
     for (int r = 0; r < d; ++r) {
       double w = B[r];
       for (int c = 0; c < d; ++c) w += A[r * d + c] * static_cast<double>((v >> (bits * c)) & zmax);
-      cb[static_cast<size_t>(v) * d + r] = w;
       lut32[static_cast<size_t>(v) * d + r] = static_cast<float>(w);
     }
-  // Prefill tile table, indexed the way the converter warps read code bytes:
-  //   d <= 2: 16 bf16 pairs, index lo | hi << 2 for two adjacent columns (k, k+1);
-  //   d == 4: 256 bf16 quads, index z0 | z1 << 2 | z2 << 4 | z3 << 6;
-  //   d == 8: none (4^8 codewords do not fit the converters' shared memory;
-  //   such layers run the decode kernels at every M).
-  auto bf = [](double w) { return static_cast<uint32_t>(f64_to_bf16_rne(w)); };
-  //   3-bit codes, d <= 2: 64 bf16 pairs, index lo | hi << 3 for columns (k, k+1);
-  //   3-bit codes, d = 4: none (8^4 quads do not fit beside the stage ring).
+  // Prefill tile table (prefill_table_host; formats in unisvq.h at
+  // unisvq_prefill_table_host).
   std::vector<uint32_t> tlut;
-  if (bits == 3 && d <= 2) {
-    tlut.resize(64);
-    for (int v = 0; v < 64; ++v) {
-      const int lo = v & 7, hi = v >> 3;
-      const double w0 = d == 2 ? cb[static_cast<size_t>(lo | (hi << 3)) * 2 + 0] : cb[lo];
-      const double w1 = d == 2 ? cb[static_cast<size_t>(lo | (hi << 3)) * 2 + 1] : cb[hi];
-      tlut[v] = bf(w0) | (bf(w1) << 16);
-    }
-  } else if (bits == 3 && d == 4) {
-    // 8^4 codewords would take 32 KB: two partial tables, one per coordinate
-    // pair p, T_p[z_2p | z_2p+1 << 3][r] = A[r][2p] z_2p + A[r][2p+1] z_2p+1
-    // (+ B[r] for p = 0), 64 rows of 4 fp32 each, exact in fp64 and rounded
-    // once; the prefill GEMM adds the two rows of a vector in fp32.
-    tlut.resize(512);
-    for (int pr = 0; pr < 2; ++pr)
-      for (int v = 0; v < 64; ++v)
-        for (int r = 0; r < 4; ++r) {
-          const double t = A[r * 4 + 2 * pr] * (v & 7) + A[r * 4 + 2 * pr + 1] * (v >> 3) + (pr == 0 ? B[r] : 0.0);
-          const float f = static_cast<float>(t);
-          std::memcpy(&tlut[static_cast<size_t>(pr * 64 + v) * 4 + r], &f, sizeof(float));
-        }
-  } else if (d == 8 && bits == 2) {
-    // 4^8 codewords are too many for shared memory: two partial tables, one
-    // per coordinate quad q, T_q[z_4q | z_4q+1 << 2 | z_4q+2 << 4 | z_4q+3 << 6][r]
-    // = sum_c A[r][4q + c] z_4q+c (+ B[r] for q = 0), each exact in fp64 and
-    // rounded once to fp32; the prefill GEMM adds the two rows of a vector in fp32.
-    // Row v is 32 bytes, entries r = 0..3 and 4..7 in its two 16-byte halves,
-    // swapped when bit 2 of v is set: a warp's loads of one half then spread
-    // over all eight 16-byte bank groups instead of four.
-    tlut.resize(4096);
-    for (int qd = 0; qd < 2; ++qd)
-      for (int v = 0; v < 256; ++v)
-        for (int r = 0; r < 8; ++r) {
-          double t = qd == 0 ? B[r] : 0.0;
-          for (int c = 0; c < 4; ++c) t += A[r * 8 + 4 * qd + c] * ((v >> (2 * c)) & 3);
-          const float f = static_cast<float>(t);
-          const int half = (r >> 2) ^ ((v >> 2) & 1);
-          std::memcpy(&tlut[static_cast<size_t>(qd * 256 + v) * 8 + 4 * half + (r & 3)], &f, sizeof(float));
-        }
-  } else if (d == 8 || bits != 2) {   // the prefill GEMM takes no table for these
-    tlut.assign(1, 0u);
-  } else if (d <= 2) {
-    tlut.resize(16);
-    for (int v = 0; v < 16; ++v) {
-      const int lo = v & 3, hi = v >> 2;
-      const double w0 = d == 2 ? cb[static_cast<size_t>(lo | (hi << 2)) * 2 + 0] : cb[lo];
-      const double w1 = d == 2 ? cb[static_cast<size_t>(lo | (hi << 2)) * 2 + 1] : cb[hi];
-      tlut[v] = bf(w0) | (bf(w1) << 16);
-    }
-  } else {
-    tlut.resize(512);
-    for (int v = 0; v < 256; ++v) {
-      tlut[2 * v] = bf(cb[static_cast<size_t>(v) * 4 + 0]) | (bf(cb[static_cast<size_t>(v) * 4 + 1]) << 16);
-      tlut[2 * v + 1] = bf(cb[static_cast<size_t>(v) * 4 + 2]) | (bf(cb[static_cast<size_t>(v) * 4 + 3]) << 16);
-    }
+  try {
+    tlut = prefill_table_host(A, B, d, bits);
+  } catch (...) {
+    delete L;
+    return UNISVQ_ERR_OOM;
   }
   L->tlut_words = static_cast<int>(tlut.size());
 

@@ -178,3 +178,95 @@ def test_pack_bits_rejects_bad_widths_and_codes(lib):
     assert st(bad, A, B, 2, 3) == binding.ERR_INVALID_ARG          # code >= 2^3
     bad[1, 5] = 4
     assert st(bad, A, B, 2, 2) == binding.ERR_INVALID_ARG          # code >= 2^2
+
+
+# ---------------------------------------------------------------------------
+# Prefill tables (unisvq_prefill_table_host), rebuilt independently: exact
+# fp64 codewords, rounded once to bf16 (round to nearest even, written here)
+# or fp32 (numpy's conversion), in the word layout include/unisvq.h states.
+# ---------------------------------------------------------------------------
+
+def _bf16_rne_bits(x):
+    x = np.asarray(x, dtype=np.float64)
+    m, e = np.frexp(x)                         # x = m 2^e, 0.5 <= |m| < 1
+    y = np.ldexp(np.rint(m * 256.0), e - 8)    # 8 significant bits, ties to even
+    return (y.astype(np.float32).view(np.uint32) >> 16).astype(np.uint32)
+
+
+def _f32_bits(x):
+    return np.asarray(x, dtype=np.float64).astype(np.float32).view(np.uint32)
+
+
+def _expected_table(A, B, d, bits):
+    A = A.astype(np.float64)
+    B = B.astype(np.float64)
+    zmax = (1 << bits) - 1
+
+    def cw(z):   # z [..., d] -> A z + B, exact in fp64
+        return np.asarray(z, dtype=np.float64) @ A.T + B
+
+    if d <= 2:
+        n = 1 << (2 * bits)
+        v = np.arange(n)
+        lo, hi = v & zmax, v >> bits
+        if d == 2:
+            w = cw(np.stack([lo, hi], axis=-1))
+            w0, w1 = w[:, 0], w[:, 1]
+        else:
+            w0, w1 = cw(lo[:, None])[:, 0], cw(hi[:, None])[:, 0]
+        return _bf16_rne_bits(w0) | (_bf16_rne_bits(w1) << 16)
+    if d == 4 and bits == 2:
+        v = np.arange(256)
+        w = cw(np.stack([(v >> (2 * c)) & 3 for c in range(4)], axis=-1))
+        t = np.zeros(512, dtype=np.uint32)
+        t[0::2] = _bf16_rne_bits(w[:, 0]) | (_bf16_rne_bits(w[:, 1]) << 16)
+        t[1::2] = _bf16_rne_bits(w[:, 2]) | (_bf16_rne_bits(w[:, 3]) << 16)
+        return t
+    if d == 4 and bits == 3:
+        t = np.zeros(512, dtype=np.uint32)
+        for p in range(2):
+            for v in range(64):
+                for r in range(4):
+                    val = A[r, 2 * p] * (v & 7) + A[r, 2 * p + 1] * (v >> 3) + (B[r] if p == 0 else 0.0)
+                    t[256 * p + 4 * v + r] = _f32_bits(val)
+        return t
+    t = np.zeros(4096, dtype=np.uint32)   # d = 8, bits = 2
+    for q in range(2):
+        for v in range(256):
+            z = np.array([(v >> (2 * c)) & 3 for c in range(4)], dtype=np.float64)
+            for r in range(8):
+                val = A[r, 4 * q:4 * q + 4] @ z + (B[r] if q == 0 else 0.0)
+                h = (r // 4) ^ ((v >> 2) & 1)
+                t[2048 * q + 8 * v + 4 * h + r % 4] = _f32_bits(val)
+    return t
+
+
+@pytest.mark.parametrize("d,bits", [(1, 2), (2, 2), (4, 2), (8, 2), (1, 3), (2, 3), (4, 3)])
+def test_prefill_tables_match_an_independent_build(lib, d, bits):
+    from paper_2606_10520_gb300 import binding
+    g = np.random.default_rng(100 * d + bits)
+    for trial in range(3):
+        A = (g.standard_normal((d, d)) * (0.5 if trial else 3.0)).astype(np.float16)
+        B = g.standard_normal(d).astype(np.float16)
+        got = binding.prefill_table_host(A, B, d, bits)
+        want = _expected_table(A, B, d, bits)
+        assert got.shape == want.shape
+        assert np.array_equal(got, want), (d, bits, np.flatnonzero(got != want)[:8])
+
+
+def test_prefill_table_rejects_bad_arguments(lib):
+    from paper_2606_10520_gb300 import binding
+    A = np.ascontiguousarray(np.eye(4, dtype=np.float16).reshape(-1)).view(np.uint16)
+    B = np.zeros(4, dtype=np.float16).view(np.uint16)
+    w = ctypes.c_size_t(0)
+    call = lambda d, bits, a=A: lib.unisvq_prefill_table_host(a.ctypes.data, B.ctypes.data, d, bits, None, 0,
+                                                              ctypes.byref(w))
+    assert call(4, 2) == binding.OK and w.value == 512
+    for d, bits in ((3, 2), (4, 4), (8, 3), (0, 2)):
+        assert call(d, bits) == binding.ERR_INVALID_ARG
+    bad = A.copy()
+    bad[5] = 0x7E00   # fp16 NaN
+    assert call(4, 2, bad) == binding.ERR_INVALID_ARG
+    out = np.zeros(8, dtype=np.uint32)
+    assert lib.unisvq_prefill_table_host(A.ctypes.data, B.ctypes.data, 4, 2, out.ctypes.data, out.size,
+                                         ctypes.byref(w)) == binding.ERR_INVALID_ARG   # too small
