@@ -1,6 +1,6 @@
 """The multi-rank paths of bench.py on CPU: two gloo ranks reduce their step
 times to the maximum and report whole-job throughput; the reference arm runs
-on rank 0 only. (On the GPU machine every rank is an independent replica: the
+on rank 0 only. (On GPUs every rank is an independent replica: the
 data path has no collective.)"""
 import json
 import os
