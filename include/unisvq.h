@@ -50,7 +50,9 @@ enum {
   UNISVQ_KERNEL_GEMV = 3,     /* fold + register-operand tensor-core GEMV, M <= 32/launch */
   UNISVQ_KERNEL_SKINNY = 4,   /* fold + tcgen05 with codes as 8-bit TMEM operand, M <= 16/launch */
   UNISVQ_KERNEL_GEMV_ROWS = 5, /* GEMV with whole-K row slices per CTA (no cluster), M <= 4/launch */
-  UNISVQ_KERNEL_GROUPED = 6    /* per-(row, group) affine GEMV (layers of unisvq_pack_grouped), M <= 32/d per launch */
+  UNISVQ_KERNEL_GROUPED = 6,   /* per-(row, group) affine GEMV (layers of unisvq_pack_grouped), M <= 32/d per launch */
+  UNISVQ_KERNEL_STREAM = 7     /* streaming GEMV: one launch per call, codes prefetched before the previous
+                                  kernel ends, whole K per CTA, no cluster; 2-bit per-matrix d <= 4, M <= 8/launch */
 };
 
 /*

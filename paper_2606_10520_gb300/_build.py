@@ -13,7 +13,7 @@ OBJ = os.path.join(PKG, "_build")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libunisvq.so")
 
-CU_SOURCES = ["unisvq_api.cu", "gemv.cu", "gemv_grouped.cu", "decode.cu", "prefill.cu", "dequant.cu", "rht.cu"]
+CU_SOURCES = ["unisvq_api.cu", "gemv.cu", "gemv_grouped.cu", "decode.cu", "prefill.cu", "dequant.cu", "rht.cu", "stream.cu"]
 CPP_SOURCES = ["pack.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

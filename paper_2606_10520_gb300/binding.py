@@ -14,7 +14,8 @@ import numpy as np
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libunisvq.so")
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM, ERR_TIMEOUT = range(6)
-KERNEL_AUTO, KERNEL_DECODE, KERNEL_PREFILL, KERNEL_GEMV, KERNEL_SKINNY, KERNEL_GEMV_ROWS, KERNEL_GROUPED = range(7)
+(KERNEL_AUTO, KERNEL_DECODE, KERNEL_PREFILL, KERNEL_GEMV, KERNEL_SKINNY, KERNEL_GEMV_ROWS, KERNEL_GROUPED,
+ KERNEL_STREAM) = range(8)
 
 # Every function include/unisvq.h declares.
 EXPORTS = [

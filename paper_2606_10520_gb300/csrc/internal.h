@@ -57,6 +57,24 @@ struct DecodePlan {
   int geom;        // skinny: k-tiles per pipeline stage (1 or 2)
 };
 
+// Streaming decode GEMV (stream.cu): one launch per call, no cluster, at most
+// one CTA per SM, kStreamMaxTok tokens per launch.
+constexpr int kStreamMaxTok = 8;
+struct StreamPlan {
+  bool ok;
+  int ucta;         // most 16-row units of a CTA
+  int ctas;         // grid (one CTA per SM at most)
+  int WU, WK;       // warp grid: unit groups x k-groups
+  int uw;           // accumulator slots per warp (2, 4 or 8)
+  int mt;           // token slots of the fold buffers (1, 2, 4 or 8)
+  int ck;           // k-tiles per fold chunk
+  int sk;           // k-tiles per code stage
+  int nslots;       // code stages resident in shared memory
+  int stage_bytes;  // ucta * sk * 512
+  int off_b, off_ptab, off_bars, off_tok;
+  size_t smem;
+};
+
 struct PrefillPlan {
   int bn;          // tokens per tile
   int tiles;
@@ -88,6 +106,13 @@ unisvq_status launch_skinny_group(const unisvq_layer* const* Ls, int n, const vo
 // static_fold_workspace_bytes() (UNSUPPORTED if the layer needs more).
 unisvq_status launch_skinny_static(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
 size_t static_fold_workspace_bytes();
+
+// Layers of one call (same K, 2-bit, per-matrix maps, d <= 4) in one
+// streaming launch per kStreamMaxTok tokens.
+StreamPlan plan_stream(const unisvq_layer* const* Ls, int n, int M);
+bool stream_supported(const unisvq_layer* const* Ls, int n, int M);
+unisvq_status launch_stream_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                                  cudaStream_t s);
 
 bool prefill_supported(const unisvq_layer* L, int M);
 PrefillPlan plan_prefill(const unisvq_layer* L, int M);

@@ -433,7 +433,7 @@ static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, vo
                      kernel == UNISVQ_KERNEL_PREFILL))
       return prefill_supported(h, M) ? launch_prefill(h, x, y, M, s) : UNISVQ_ERR_UNSUPPORTED;
     if (!noalloc && kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GEMV)
-      return kernel >= 0 && kernel <= UNISVQ_KERNEL_GROUPED ? UNISVQ_ERR_UNSUPPORTED : UNISVQ_ERR_INVALID_ARG;
+      return kernel >= 0 && kernel <= UNISVQ_KERNEL_STREAM ? UNISVQ_ERR_UNSUPPORTED : UNISVQ_ERR_INVALID_ARG;
     return launch_gemv(h, x, y, M, s);
   }
   if (noalloc) {
@@ -448,7 +448,7 @@ static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, vo
     if ((kernel == UNISVQ_KERNEL_AUTO && M > 64 && prefill_supported(h, M)) || kernel == UNISVQ_KERNEL_PREFILL)
       return prefill_supported(h, M) ? launch_prefill(h, x, y, M, s) : UNISVQ_ERR_UNSUPPORTED;
     if (kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GROUPED)
-      return kernel >= 0 && kernel <= UNISVQ_KERNEL_GROUPED ? UNISVQ_ERR_UNSUPPORTED : UNISVQ_ERR_INVALID_ARG;
+      return kernel >= 0 && kernel <= UNISVQ_KERNEL_STREAM ? UNISVQ_ERR_UNSUPPORTED : UNISVQ_ERR_INVALID_ARG;
     const unisvq_layer* Ls[1] = {h};
     void* ys[1] = {y};
     return launch_grouped_group(Ls, 1, x, ys, M, s);
@@ -464,6 +464,12 @@ static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, vo
     return launch_gemv_rows_group(Ls, 1, x, ys, M, s);
   }
   if (kernel == UNISVQ_KERNEL_SKINNY) return launch_skinny(h, x, y, M, s);
+  if (kernel == UNISVQ_KERNEL_STREAM) {
+    const unisvq_layer* Ls[1] = {h};
+    if (!stream_supported(Ls, 1, M)) return UNISVQ_ERR_UNSUPPORTED;
+    void* ys[1] = {y};
+    return launch_stream_group(Ls, 1, x, ys, M, s);
+  }
   if (kernel == UNISVQ_KERNEL_PREFILL) {
     if (!prefill_supported(h, M)) return UNISVQ_ERR_UNSUPPORTED;
     return launch_prefill(h, x, y, M, s);
@@ -477,7 +483,7 @@ static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, vo
 static unisvq_status linear_rht(unisvq_handle h, int kernel, const void* x, void* y, int M, cudaStream_t s,
                                 bool noalloc) {
   if (!h->rht) return linear_inner(h, kernel, x, y, M, s, noalloc);
-  if (kernel < UNISVQ_KERNEL_AUTO || kernel > UNISVQ_KERNEL_GROUPED) return UNISVQ_ERR_INVALID_ARG;
+  if (kernel < UNISVQ_KERNEL_AUTO || kernel > UNISVQ_KERNEL_STREAM) return UNISVQ_ERR_INVALID_ARG;
   const uint8_t* s_in = h->rht_signs;
   const uint8_t* s_out = h->rht_signs + h->K;
   for (int m0 = 0; m0 < M; m0 += h->rht_tokens) {
@@ -608,7 +614,7 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
   }
   // One S_V for every layer: rotate x once (into the first handle's buffer),
   // run the layers as one group, rotate each output with its own U S_U.
-  if (kernel < UNISVQ_KERNEL_AUTO || kernel > UNISVQ_KERNEL_GROUPED) return UNISVQ_ERR_INVALID_ARG;
+  if (kernel < UNISVQ_KERNEL_AUTO || kernel > UNISVQ_KERNEL_STREAM) return UNISVQ_ERR_INVALID_ARG;
   int cap = hs[0]->rht_tokens;
   for (int i = 1; i < n; ++i) cap = hs[i]->rht_tokens < cap ? hs[i]->rht_tokens : cap;
   const int K = hs[0]->K;
@@ -687,6 +693,10 @@ static unisvq_status group_inner(const unisvq_handle* hs, int n, int kernel, con
   for (int i = 0; i < n; ++i) Ls[i] = hs[i];
   if (kernel == UNISVQ_KERNEL_GEMV) return launch_gemv_group(Ls, n, x, ys, M, s);
   if (kernel == UNISVQ_KERNEL_SKINNY) return launch_skinny_group(Ls, n, x, ys, M, s);
+  if (kernel == UNISVQ_KERNEL_STREAM) {
+    if (!stream_supported(Ls, n, M)) return UNISVQ_ERR_UNSUPPORTED;
+    return launch_stream_group(Ls, n, x, ys, M, s);
+  }
   if (kernel == UNISVQ_KERNEL_GEMV_ROWS) {
     for (int i = 0; i < n; ++i)
       if (!gemv_rows_supported(Ls[i], M < 4 ? M : 4)) return UNISVQ_ERR_UNSUPPORTED;
@@ -733,6 +743,11 @@ static void describe_launch(const unisvq_layer* const* Ls, int n, int kernel, in
     info->split_k = p.ks;
     info->launches = per > 0 ? (m + per - 1) / per : 0;
     info->grid_ctas = p.ks * nb * info->launches;
+  } else if (kernel == UNISVQ_KERNEL_STREAM) {
+    const StreamPlan p = plan_stream(Ls, n, m < kStreamMaxTok ? m : kStreamMaxTok);
+    info->split_k = 1;
+    info->launches = (m + kStreamMaxTok - 1) / kStreamMaxTok;
+    info->grid_ctas = p.ctas * info->launches;
   } else if (kernel == UNISVQ_KERNEL_GEMV_ROWS) {
     info->split_k = 1;
     info->grid_ctas = 0;
