@@ -44,8 +44,10 @@ example in tests/golden/grouped_hand_worked.json, group-wise uniform scalar
 quantisation (A = s I), reduction to the per-matrix oracle when all groups
 share one map, and the exchange-of-sums identity; for the RHT functions,
 H H^T = n I for every order built, Sylvester's matrix against SciPy's, and the
-undo identity: the RHT layer applied to W_hat = R(W) returns x W^T. No
-function here is "parity unpinned".
+undo identity: the RHT layer applied to W_hat = R(W) returns x W^T; for the
+bf16 widening that every activation passes through, hand-chosen bit patterns
+(signed zero, subnormals, the largest finite value, infinities) against the
+IEEE bfloat16 definition. No function here is "parity unpinned".
 """
 from __future__ import annotations
 
@@ -61,7 +63,8 @@ REL_L2_BOUND = 4e-3
 def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
     """Exact widening of bf16 bit patterns (uint16) to float64."""
     b = np.ascontiguousarray(bits, dtype=np.uint16).astype(np.uint32) << 16
-    return b.view(np.float32).astype(np.float64)
+    with np.errstate(invalid="ignore"):   # signalling-NaN patterns stay NaN
+        return b.view(np.float32).astype(np.float64)
 
 
 def as_f64(a) -> np.ndarray:
@@ -76,13 +79,6 @@ def _check(codes: np.ndarray, A: np.ndarray, B: np.ndarray):
     if codes.ndim != 2 or codes.shape[1] % d:
         raise ValueError("codes must be [N][K] with K a multiple of d")
     return d
-
-
-def codeword(z, A, B) -> np.ndarray:
-    """Eq. (def:unisvq): the weight vector A z + B of one lattice point z."""
-    A = as_f64(A)
-    B = as_f64(B)
-    return A @ np.asarray(z, dtype=np.float64) + B
 
 
 def codebook(A, B, bits: int = 2) -> np.ndarray:

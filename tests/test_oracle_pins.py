@@ -468,3 +468,78 @@ def test_3bit_scalar_case_is_uniform_3bit_dequantisation():
     codes = g.integers(0, 8, size=(5, 64), dtype=np.uint8)
     W = oracle.dequant(codes, s_ * np.eye(2), -s_ * zp * np.ones(2))
     assert np.array_equal(W, s_ * (codes.astype(np.float64) - zp))
+
+
+# --------------------------------------------------------------------------
+# bf16 widening: every activation of the layer (the X of Eq. def:ptq_loss,
+# Sec. 2.1, stored as bfloat16) reaches the oracle through bf16_bits_to_f64
+# --------------------------------------------------------------------------
+
+# (bit pattern, value written out by hand from the bfloat16 format: sign bit,
+# 8 exponent bits with bias 127, 7 fraction bits)
+BF16_CASES = [
+    (0x3F80, 1.0),
+    (0xBF80, -1.0),
+    (0xC0A0, -5.0),                      # 1 10000001 0100000: -(1 + 1/4) * 2^2
+    (0x4049, 3.140625),                  # 0 10000000 1001001: (1 + 73/128) * 2
+    (0x3F81, 1.0 + 2.0 ** -7),           # the next bf16 above 1
+    (0x0080, 2.0 ** -126),               # smallest normal
+    (0x0001, 2.0 ** -133),               # smallest subnormal: 2^-126 * 2^-7
+    (0x807F, -(127 / 128) * 2.0 ** -126),  # largest negative subnormal
+    (0x7F7F, (2.0 - 2.0 ** -7) * 2.0 ** 127),  # largest finite
+    (0x7F80, float("inf")),
+    (0xFF80, float("-inf")),
+    (0x0000, 0.0),
+]
+
+
+def bf16_by_definition(b: int) -> float:
+    """IEEE-style bfloat16 value of a 16-bit pattern, from its fields."""
+    sign = -1.0 if b >> 15 else 1.0
+    e = (b >> 7) & 0xFF
+    f = b & 0x7F
+    if e == 0xFF:
+        return sign * float("inf") if f == 0 else float("nan")
+    if e == 0:
+        return sign * (f / 128.0) * 2.0 ** -126
+    return sign * (1.0 + f / 128.0) * 2.0 ** (e - 127)
+
+
+def pin_bf16_widening(widen_fn):
+    bits = np.array([b for b, _ in BF16_CASES], dtype=np.uint16)
+    got = widen_fn(bits)
+    for (b, v), g in zip(BF16_CASES, got):
+        assert g == v, (hex(b), g, v)
+        assert bf16_by_definition(b) == v, hex(b)
+    # -0.0 keeps its sign
+    z = widen_fn(np.array([0x8000], dtype=np.uint16))[0]
+    assert z == 0.0 and np.signbit(z)
+    # every finite pattern against the field definition (all 65536 patterns)
+    allb = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    w = widen_fn(allb)
+    e = (allb.astype(np.int64) >> 7) & 0xFF
+    fin = e != 0xFF
+    ref = np.array([bf16_by_definition(int(b)) for b in allb[fin][::97]])
+    assert np.array_equal(w[fin][::97], ref)
+    nan_pat = (e == 0xFF) & ((allb & 0x7F) != 0)
+    assert np.all(np.isnan(w[nan_pat]))
+
+
+def test_bf16_widening_pinned():
+    pin_bf16_widening(oracle.bf16_bits_to_f64)
+
+
+@pytest.mark.parametrize("kind", ["as_fp16", "byteswap", "shift15", "drop_sign"])
+def test_bf16_pin_catches_planted_mistakes(kind):
+    def widen(bits):
+        b = np.ascontiguousarray(bits, dtype=np.uint16)
+        if kind == "as_fp16":
+            return b.view(np.float16).astype(np.float64)
+        if kind == "byteswap":
+            b = b.byteswap()
+        if kind == "drop_sign":
+            b = b & 0x7FFF
+        sh = 15 if kind == "shift15" else 16
+        return (b.astype(np.uint32) << sh).view(np.float32).astype(np.float64)
+    with pytest.raises(AssertionError):
+        pin_bf16_widening(widen)
