@@ -60,6 +60,13 @@ def algo_bytes(N, K, M, d=2):
     return N * K // 4 + (d * d + d) * 2 + 2 * M * K + 2 * M * N
 
 
+def group_bytes(shapes, grp, M, d=2):
+    """Algorithmic bytes of one call over the projections `grp`, which share
+    one input: codes, affine and output per projection, the input x once."""
+    K = shapes[grp[0]][2]
+    return sum(shapes[i][1] * K // 4 + (d * d + d) * 2 + 2 * M * shapes[i][1] for i in grp) + 2 * M * K
+
+
 KERNEL_NAMES = {1: "decode", 2: "prefill_kernel", 3: "gemv_kernel", 4: "decode_kernel", 5: "gemv_rows_kernel",
                 6: "gemv_grouped_kernel"}
 GROUPED_LAYERS = 16   # 16 x 69.6 MB of codes + per-group maps: larger than L2
@@ -168,10 +175,32 @@ class ClockSampler:
 # CPU oracle baseline (bounded sample)
 # ---------------------------------------------------------------------------
 def cpu_threads():
+    """Threads the oracle's BLAS runs with: from threadpoolctl where it is
+    installed, else the thread-count environment variables, else every core
+    (the BLAS default)."""
+    try:
+        from threadpoolctl import threadpool_info
+        n = [p.get("num_threads") for p in threadpool_info() if p.get("user_api") == "blas"]
+        if n and all(isinstance(v, int) for v in n):
+            return max(n)
+    except Exception:
+        pass
     for v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
         if os.environ.get(v, "").isdigit():
             return int(os.environ[v])
     return os.cpu_count() or 1
+
+
+def oracle_sample_one_thread(budget_s: float):
+    """oracle_sample in a child process whose BLAS runs one thread."""
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    code = ("import json, sys; sys.path.insert(0, %r); import bench; "
+            "g, t, n = bench.oracle_sample(%f); print(json.dumps([g, t, len(n), bench.cpu_threads()]))") % (ROOT, budget_s)
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=600)
+    if r.returncode != 0:
+        return None
+    g, t, n, th = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"value": g, "unit": "GB/s", "cores": th, "seconds": t, "calls": n}
 
 
 def oracle_sample(budget_s: float):
@@ -218,20 +247,38 @@ def whole_job_gbs(bytes_per_step_per_rank, steps, world, t_max):
 
 
 def run_reference(args, rank, world):
+    """The oracle on a bounded sample of the workload: step i is one call on
+    512 output rows of projection i mod 7 of the layer-0 set at M =
+    M_SWEEP[(i // 7) mod 5], so K steps cover the projections and batch sizes
+    in the workload's proportions (the 32 layers are copies of layer 0)."""
     if rank != 0:
         return
     import oracle
-    name, N, K = synth.LLAMA2_7B[0]
-    codes, A, B = synth.layer_inputs(0, 1, 0, 0, N, K, 2)
-    xb = synth.activations(0, 1, 1, 1, K)
-    for _ in range(args.warmup):
-        oracle.linear(xb, codes, A, B)
+    shapes = synth.LLAMA2_7B
+    mats = [synth.layer_inputs(0, 1, 0, pi, N, K, 2) for pi, (_, N, K) in enumerate(shapes)]
+    xs = {(M, K): synth.activations(0, 1, 100 + M, M, K) for M in M_SWEEP for K in {K for _, _, K in shapes}}
+
+    rows = 512   # output rows per step, cycling over each matrix
+
+    def step(i):
+        pi = i % len(shapes)
+        M = M_SWEEP[(i // len(shapes)) % len(M_SWEEP)]
+        _, N, K = shapes[pi]
+        codes, A, B = mats[pi]
+        r0 = (i // (len(shapes) * len(M_SWEEP)) * rows) % N
+        part = codes[r0:r0 + rows]
+        oracle.linear(xs[(M, K)], part, A, B)
+        return algo_bytes(part.shape[0], K, M)
+    for i in range(args.warmup):
+        step(i)
+    nbytes = 0
     t0 = time.perf_counter()
-    for _ in range(args.steps):
-        oracle.linear(xb, codes, A, B)
+    for i in range(args.steps):
+        nbytes += step(i)
     dt = time.perf_counter() - t0
-    gbs = args.steps * algo_bytes(N, K, 1) / dt / 1e9
-    sample = f"per step: one {N}x{K} projection (q, layer 0) at M=1 through oracle.linear (fp64 NumPy)"
+    gbs = nbytes / dt / 1e9
+    sample = (f"{args.steps} oracle.linear calls (fp64 NumPy), each on {rows} output rows of one projection, "
+              f"cycling over the 7 layer-0 projections, M in {list(M_SWEEP)} and the rows of each matrix")
     line = {
         "impl": "reference", "metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1000 / args.steps,
@@ -309,6 +356,7 @@ def run_ours(args, rank, world, local_rank):
         return
     if args.only == "decode":
         args.no_e2e = args.no_cpu = args.no_prefill = args.no_grouped = args.no_rht = args.no_bits3 = True
+        args.no_70b = args.no_dense = True
     shapes = synth.LLAMA2_7B
     stack = build_stack(binding, shapes, args.layers, 1)
 
@@ -362,7 +410,7 @@ def run_ours(args, rank, world, local_rank):
         for gi, grp in enumerate(groups):
             info = call_info(grp, M)
             kid = info["kernel"]
-            nbytes = sum(algo_bytes(shapes[i][1], shapes[i][2], M) for i in grp) * args.layers
+            nbytes = group_bytes(shapes, grp, M) * args.layers
             step_bytes += nbytes
             launches += info["launches"] * args.layers
             kinds.setdefault(kid, []).append((M, gi))
@@ -443,7 +491,7 @@ def run_ours(args, rank, world, local_rank):
     sweep = []
     for M, g in zip(M_SWEEP, graphs):
         tm = time_graphs(torch, [g], max(3, args.steps // 4), 2, side)
-        nb = sum(algo_bytes(N, K, M) for _, N, K in shapes) * args.layers
+        nb = sum(group_bytes(shapes, grp, M) for grp in groups) * args.layers
         n_calls = len(shapes) * args.layers
         gbs = nb * max(3, args.steps // 4) / tm / 1e9
         sweep.append({"M": M, "GB/s": round(gbs, 1), "frac_of_measured_hbm": round(gbs / peaks["hbm_gbs"], 4),
@@ -509,6 +557,18 @@ def run_ours(args, rank, world, local_rank):
     if not args.no_prefill:
         prefill = run_prefill(torch, binding, peaks, args, side)
 
+    # ---- configs 0, 3 (70B stack), 4 (crossover) and the dense reference ----
+    config0 = run_config0(torch, binding, peaks, args, side)
+    cfg3 = crossover = None
+    if not args.no_70b:
+        cfg3, stack70 = run_70b(torch, binding, peaks, args, side)
+        crossover = run_crossover(torch, binding, peaks, args, side, stack70)
+        for layer in stack70:
+            for h in layer:
+                h.close()
+        del stack70
+    dense = None if args.no_dense else run_cublas_decode(torch, peaks, args, side, sweep)
+
     # ---- CPU oracle baseline (rank 0, N=1 only) --------------------------
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
@@ -516,7 +576,8 @@ def run_ours(args, rank, world, local_rank):
         cpu = {"value": gbs_cpu, "unit": "GB/s", "cores": cpu_threads(), "kind": "oracle",
                "sample": f"oracle.linear (fp64 NumPy) at M=1 on {len(names)} projection calls cycling over "
                          f"the layer-0 set ({', '.join(n for n, _, _ in synth.LLAMA2_7B)}), "
-                         f"{t_cpu:.1f} s of CPU work"}
+                         f"{t_cpu:.1f} s of CPU work",
+               "single_thread": oracle_sample_one_thread(min(8.0, args.cpu_budget))}
 
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
@@ -534,6 +595,10 @@ def run_ours(args, rank, world, local_rank):
         "clocks": clocks,
         "cpu_baseline": cpu,
         "prefill": prefill,
+        "config0_4096x4096_m1": config0,
+        "llama2_70b": cfg3,
+        "crossover_70b": crossover,
+        "cublas_dense_decode": dense,
         "per_group_affine": grouped,
         "rht": rht,
         "bits3": bits3,
@@ -874,6 +939,175 @@ def time_prefill_layers(torch, b, shapes, glayers, xs, ys, M, reps, stream):
     return time_graphs(torch, [gg], reps, 3, stream)
 
 
+# ---------------------------------------------------------------------------
+# configs 0, 3, 4 and the dense decode reference
+# ---------------------------------------------------------------------------
+def capture(torch, fn, stream):
+    """Run `fn` once on `stream`, then capture it in a CUDA graph."""
+    with torch.cuda.stream(stream):
+        fn()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        fn()
+    return g
+
+
+def make_io(torch, shapes, M):
+    xs, ys = {}, {}
+    for pi, (_, N, K) in enumerate(shapes):
+        if K not in xs:
+            xb = synth.activations(0, 4, 100 + M, M, K)
+            xs[K] = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).cuda()
+        ys[pi] = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    return xs, ys
+
+
+def stack_pass(binding, stack, shapes, groups, xs, ys, M):
+    def fn():
+        sp = __import__("torch").cuda.current_stream().cuda_stream
+        for layer in stack:
+            for grp in groups:
+                K = shapes[grp[0]][2]
+                st = binding.linear_group_ptr([layer[i] for i in grp], xs[K].data_ptr(),
+                                              [ys[i].data_ptr() for i in grp], M, sp)
+                if st != 0:
+                    raise RuntimeError(f"unisvq call failed: {binding.status_string(st)}")
+    return fn
+
+
+def run_config0(torch, binding, peaks, args, stream):
+    """One 4096 x 4096 projection at M = 1 (d = 2): 64 distinct device copies
+    (268 MB, larger than L2) called one after the other from a CUDA graph."""
+    N = K = 4096
+    copies = 64
+    codes, A, B = synth.layer_inputs(0, 0, 0, 0, N, K, 2)
+    base = binding.UniSVQLinear(codes, A, B)
+    hs = [base] + [base.clone() for _ in range(copies - 1)]
+    x = torch.from_numpy(synth.activations(0, 0, 1, 1, K).view(np.int16)).view(torch.bfloat16).cuda()
+    y = torch.empty((1, N), dtype=torch.bfloat16, device="cuda")
+
+    def fn():
+        sp = torch.cuda.current_stream().cuda_stream
+        for h in hs:
+            st = h.forward_ptr(x.data_ptr(), y.data_ptr(), 1, sp, binding.KERNEL_AUTO)
+            if st != 0:
+                raise RuntimeError(binding.status_string(st))
+    g = capture(torch, fn, stream)
+    reps = max(5, args.steps // 8)
+    t = time_graphs(torch, [g], reps, args.warmup, stream)
+    us = t / reps / copies * 1e6
+    nb = algo_bytes(N, K, 1)
+    gbs = nb / (us * 1e-6) / 1e9
+    kern = KERNEL_NAMES.get(base.query(1)["kernel"], "?")
+    for h in hs:
+        h.close()
+    return {"workload": "one 4096x4096 projection, M=1, d=2 (64 device copies cycled: 268 MB, L2-cold)",
+            "us_per_call": round(us, 3), "GB/s": round(gbs, 1), "frac_of_measured_hbm": round(gbs / peaks["hbm_gbs"], 4),
+            "roofline_us": round(nb / (peaks["hbm_gbs"] * 1e9) * 1e6, 3), "kernel": kern,
+            "timing": "CUDA graph of 64 calls, CUDA events on the launching stream"}
+
+
+def run_70b(torch, binding, peaks, args, stream):
+    """The Llama-2-70B-shaped stack: args.layers_70b layers x {q, o: 8192^2;
+    k, v: 1024x8192; gate, up: 28672x8192; down: 8192x28672} (17.1 GB of codes
+    at 80 layers), decode batches M in {1, 8, 32}. Returns (result, stack)."""
+    shapes = synth.LLAMA2_70B
+    nl = args.layers_70b
+    stack = build_stack(binding, shapes, nl, 3)
+    out = []
+    for M in (1, 8, 32):
+        xs, ys = make_io(torch, shapes, M)
+        g = capture(torch, stack_pass(binding, stack, shapes, GROUPS_7B, xs, ys, M), stream)
+        reps = max(3, args.steps // 40)
+        t = time_graphs(torch, [g], reps, args.warmup, stream)
+        nb = sum(group_bytes(shapes, grp, M) for grp in GROUPS_7B) * nl
+        gbs = nb * reps / t / 1e9
+        kerns = {"+".join(shapes[i][0] for i in grp):
+                 KERNEL_NAMES.get(binding.query_group([stack[0][i] for i in grp], M)["kernel"], "?") for grp in GROUPS_7B}
+        out.append({"M": M, "GB/s": round(gbs, 1), "frac_of_measured_hbm": round(gbs / peaks["hbm_gbs"], 4),
+                    "ms_per_pass": round(t / reps * 1e3, 3), "kernels": kerns})
+        del g
+    st = binding.sync_status(stream)
+    if st != 0:
+        raise RuntimeError(f"device status {binding.status_string(st)}")
+    code_gb = sum(N * K // 4 for _, N, K in shapes) * nl / 1e9
+    return ({"workload": f"Llama-2-70B-shaped projection set x {nl} layers ({code_gb:.1f} GB of 2-bit codes), d=2",
+             "per_M": out, "calls": "q/k/v and gate/up as one group call each, o and down alone",
+             "l2": "inputs larger than L2"}, stack)
+
+
+CROSSOVER_M = (1, 2, 4, 8, 16, 32, 64, 128, 512, 2048)
+
+
+def run_crossover(torch, binding, peaks, args, stream, stack70):
+    """GEMV-to-GEMM crossover on the 70B shapes: for d = 2 (the first 16 layers
+    of the 70B stack) and d = 4 (16 fresh layers), every M of CROSSOVER_M
+    through unisvq_linear_group's own pick; per M the kernel of each call,
+    time per layer and the fraction of the roofline max(bytes / HBM, flops /
+    bf16 peak)."""
+    shapes = synth.LLAMA2_70B
+    nl = min(16, len(stack70))
+    rows = []
+    for d in (2, 4):
+        stack = stack70[:nl] if d == 2 else build_stack(binding, shapes, nl, 4, d=4)
+        for M in CROSSOVER_M:
+            xs, ys = make_io(torch, shapes, M)
+            g = capture(torch, stack_pass(binding, stack, shapes, GROUPS_7B, xs, ys, M), stream)
+            reps = 3 if M >= 512 else max(3, args.steps // 40)
+            t = time_graphs(torch, [g], reps, 2, stream) / reps
+            nb = sum(group_bytes(shapes, grp, M, d) for grp in GROUPS_7B) * nl
+            fl = sum(2.0 * M * N * K for _, N, K in shapes) * nl
+            t_hbm = nb / (peaks["hbm_gbs"] * 1e9)
+            t_tc = fl / (peaks["bf16_tflops"] * 1e12)
+            kerns = {"+".join(shapes[i][0] for i in grp):
+                     KERNEL_NAMES.get(binding.query_group([stack[0][i] for i in grp], M)["kernel"], "?")
+                     for grp in GROUPS_7B}
+            rows.append({"d": d, "M": M, "kernels": kerns, "us_per_layer": round(t / nl * 1e6, 2),
+                         "GB/s": round(nb / t / 1e9, 1), "TFLOP/s": round(fl / t / 1e12, 1),
+                         "bound": "hbm" if t_hbm >= t_tc else "tensor",
+                         "frac_of_roofline": round(max(t_hbm, t_tc) / t, 4)})
+            del g, xs, ys
+        if d == 4:
+            for layer in stack:
+                for h in layer:
+                    h.close()
+    st = binding.sync_status(stream)
+    if st != 0:
+        raise RuntimeError(f"device status {binding.status_string(st)}")
+    return {"workload": f"Llama-2-70B-shaped projection set x {nl} layers per d, M in {list(CROSSOVER_M)}",
+            "roofline": "max(algorithmic bytes / measured HBM, 2MNK / measured bf16 burst)", "rows": rows}
+
+
+def run_cublas_decode(torch, peaks, args, stream, ours_sweep):
+    """cuBLAS bf16 dense GEMM (torch.matmul) on the decode shapes of the
+    Llama-2-7B set, 8 layers of dense weights (1.6 GB, larger than L2), per M of
+    the sweep: the speed a dense fp16/bf16 layer has on this GPU."""
+    shapes = synth.LLAMA2_7B
+    nl = 8
+    W = [[torch.randn(N, K, device="cuda", dtype=torch.bfloat16) for _, N, K in shapes] for _ in range(nl)]
+    out = []
+    for M, ours in zip(M_SWEEP, ours_sweep):
+        xs, ys = make_io(torch, shapes, M)
+
+        def fn():
+            for layer in W:
+                for pi, (_, N, K) in enumerate(shapes):
+                    torch.matmul(xs[K], layer[pi].t(), out=ys[pi])
+        g = capture(torch, fn, stream)
+        reps = max(5, args.steps // 20)
+        t = time_graphs(torch, [g], reps, args.warmup, stream) / reps
+        dense_bytes = sum(2 * N * K + 2 * M * K + 2 * M * N for _, N, K in shapes) * nl
+        us_layer = t / nl * 1e6
+        ours_us = ours["us_per_projection"] * len(shapes)
+        out.append({"M": M, "dense_us_per_layer": round(us_layer, 2), "dense_GB/s": round(dense_bytes / t / 1e9, 1),
+                    "unisvq_us_per_layer": round(ours_us, 2), "speedup_vs_dense": round(us_layer / ours_us, 3)})
+        del g
+    del W
+    return {"workload": "Llama-2-7B projection shapes, dense bf16 weights, 8 layers, torch.matmul (cuBLAS)",
+            "per_M": out}
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -892,6 +1126,9 @@ def main():
     ap.add_argument("--ungrouped", action="store_true",
                     help="one unisvq_linear call per projection instead of grouped calls for q/k/v and gate/up")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--layers-70b", type=int, default=80)
+    ap.add_argument("--no-70b", action="store_true", help="skip config 3 (70B stack) and the crossover table")
+    ap.add_argument("--no-dense", action="store_true", help="skip the cuBLAS dense decode reference")
     ap.add_argument("--only", choices=["decode", "prefill", "grouped", "rht", "bits3"], default=None,
                     help="profiling aid: run only the decode sweep (no e2e/cpu/secondary sweeps), only the "
                          "prefill set, or only one secondary sweep (with --layers layers)")

@@ -111,14 +111,13 @@ def test_3bit_dispatch_groups_and_entry_points():
 
 
 @pytest.mark.parametrize("N,K", [(4096, 11008), (11008, 4096)])
-def test_3bit_full_size_sampled_rows(N, K):
+def test_3bit_full_size_all_rows(N, K):
     codes, A, B, layer = make(N, K, 2, 5)
-    rows = np.sort(np.random.default_rng(N).choice(N, size=48, replace=False))
     for M in (1, 16):
         xb = synth.activations(5, 60, M, M, K)
         y = run(layer, xb)
-        yr, S = oracle.linear(xb, codes[rows], A, B)
-        assert oracle.compare(y[:, rows], yr, S)["ok"]
+        yr, S = oracle.linear(xb, codes, A, B)
+        assert oracle.compare(y, yr, S)["ok"]
     layer.close()
 
 

@@ -135,12 +135,11 @@ def test_grouped_group_call_matches_oracle(M):
 
 
 @pytest.mark.parametrize("N,K", [(4096, 4096), (11008, 4096), (4096, 11008)])
-def test_grouped_full_size_sampled_rows(N, K):
+def test_grouped_full_size_all_rows(N, K):
     codes, A, B, layer = make(N, K, 2, seed=5)
-    rows = np.sort(np.random.default_rng(N + K).choice(N, size=48, replace=False))
     for M in (1, 16):
         xb = synth.activations(5, 40, M, M, K)
-        check(run(layer, xb), xb, codes, A, B, rows=rows)
+        check(run(layer, xb), xb, codes, A, B)
     layer.close()
 
 

@@ -184,19 +184,20 @@ def test_clone_matches_original():
 FULL_SHAPES = [(4096, 4096), (11008, 4096), (4096, 11008), (28672, 8192), (8192, 28672)]
 
 
-@pytest.mark.parametrize("N,K", FULL_SHAPES)
-def test_full_size_decode_sampled_rows(N, K):
-    """Config-sized layers at the decode batch sizes, checked on sampled rows."""
-    d = 2
+@pytest.mark.parametrize("N,K,d", [(N, K, 2) for N, K in FULL_SHAPES] + [(28672, 8192, 4), (8192, 28672, 4)])
+def test_full_size_decode_all_rows(N, K, d):
+    """Config-sized layers (the Llama-2-7B and -70B projections, and the d = 4
+    variant of the 70B crossover workload) at the decode batch sizes: every
+    output row of every kernel that runs them against the oracle."""
     codes, A, B = synth.layer_inputs(0, 3, 0, N, N, K, d)
     layer = binding.UniSVQLinear(codes, A, B)
-    rows = np.sort(synth.rng(0, N, K).choice(N, size=48, replace=False))
-    rows = np.unique(np.concatenate([rows, [0, N - 1]]))
     for M in (1, 8, 16, 32):
         xb = synth.activations(0, 3, M, M, K)
-        check(run(layer, xb), xb, codes, A, B, rows=rows)
+        check(run(layer, xb), xb, codes, A, B)
         if M <= 16:
-            check(run(layer, xb, binding.KERNEL_SKINNY), xb, codes, A, B, rows=rows)
+            check(run(layer, xb, binding.KERNEL_SKINNY), xb, codes, A, B)
+        if M <= 8:
+            check(run(layer, xb, binding.KERNEL_STREAM), xb, codes, A, B)
     layer.close()
 
 
@@ -386,18 +387,26 @@ def test_dispatch_picks_tcgen05_decode_for_large_launches():
 
 
 @pytest.mark.parametrize("N,K", [(4096, 4096), (1024, 4096), (14336, 4096), (4096, 14336)])
-def test_full_size_prefill_sampled_rows(N, K):
-    """Llama-3-8B-shaped projections at M = 2048 (the prefill workload)."""
+def test_full_size_prefill_all_rows(N, K):
+    """Llama-3-8B-shaped projections at M = 2048 (the prefill workload), every row."""
     d = 2
     codes, A, B = synth.layer_inputs(0, 2, 0, N + K, N, K, d)
     layer = binding.UniSVQLinear(codes, A, B)
-    rows = np.unique(np.concatenate([np.sort(synth.rng(1, N, K).choice(N, size=24, replace=False)), [0, N - 1]]))
     M = 2048
     xb = synth.activations(0, 2, K, M, K)
-    yg = run(layer, xb)
-    yr, S = oracle.linear(xb, codes[rows], A, B)
-    res = oracle.compare(yg[:, rows], yr, S)
-    assert res["ok"], res
+    check(run(layer, xb), xb, codes, A, B)
+    layer.close()
+
+
+@pytest.mark.parametrize("N,K,d", [(8192, 28672, 2), (28672, 8192, 2), (28672, 8192, 4)])
+def test_full_size_prefill_70b_shapes(N, K, d):
+    """Llama-2-70B down and gate/up shapes on the crossover sweep's prefill
+    sizes (the d = 4 row is that sweep's variant), every row."""
+    codes, A, B = synth.layer_inputs(0, 4, d, N + K, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    for M in (64, 128, 512, 2048):
+        xb = synth.activations(0, 4, K + M, M, K)
+        check(run(layer, xb), xb, codes, A, B)
     layer.close()
 
 
