@@ -48,7 +48,7 @@ enum {
   UNISVQ_KERNEL_DECODE = 1,   /* the decode kernel auto would pick for this M (a GEMV)  */
   UNISVQ_KERNEL_PREFILL = 2,  /* tcgen05 GEMM, bf16 weight tiles in smem (exact codewords for d <= 4) */
   UNISVQ_KERNEL_GEMV = 3,     /* fold + register-operand tensor-core GEMV, M <= 32/launch */
-  UNISVQ_KERNEL_SKINNY = 4,   /* fold + tcgen05 with codes as 8-bit TMEM operand, M <= 16/launch */
+  UNISVQ_KERNEL_SKINNY = 4,   /* fold + tcgen05 with codes as 8-bit TMEM operand, M <= 32/launch */
   UNISVQ_KERNEL_GEMV_ROWS = 5, /* GEMV with whole-K row slices per CTA (no cluster), M <= 4/launch */
   UNISVQ_KERNEL_GROUPED = 6,   /* per-(row, group) affine GEMV (layers of unisvq_pack_grouped), M <= 32/d per launch */
   UNISVQ_KERNEL_STREAM = 7     /* streaming GEMV: one launch per call, codes prefetched before the previous
@@ -114,7 +114,7 @@ typedef struct {
  * Errors: INVALID_ARG (null pointer, bad shape, code > 3, non-finite A/B),
  * UNSUPPORTED (d not in {1,2,4,8}), OOM, CUDA.
  * The handle owns all device memory: the packed codes, the tables of the
- * prefill kernel and a fold workspace of 1 KB + (Kp/128) * 6 KB that the
+ * prefill kernel and a fold workspace of 2 KB + (Kp/128) * 12 KB that the
  * decode kernels rewrite on every call (the folded activations of Eq.
  * col:matmul). Calls that use the same handle must therefore be ordered on
  * the GPU (one stream, or events between streams); calls on different
@@ -224,20 +224,27 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
                                         int M, void* stream);
 
 /*
- * y = x W_hat^T with the tcgen05 decode kernels (UNISVQ_KERNEL_SKINNY) and
- * their fold workspace in a static device array of the library (2 MiB per
- * device: Kp <= 43648) instead of the handle's workspace. The paper has no
- * counterpart: it is a deployment variant of unisvq_linear for callers that
- * may not allocate on the call path (a server that fixed its device-memory
- * budget at start-up, or code that must not enter the allocator while other
- * work runs, since cudaMalloc and cudaFree can synchronise the device); it
- * calls no allocating routine.
+ * y = x W_hat^T as unisvq_linear computes it (same kernel choice), with one
+ * difference: where that choice is the tcgen05 decode pair
+ * (UNISVQ_KERNEL_SKINNY), its fold workspace is a static device array of the
+ * library (2 MiB per device) instead of the handle's workspace. The paper has
+ * no counterpart: it is a deployment variant of unisvq_linear for callers
+ * that may not allocate on the call path (a server that fixed its
+ * device-memory budget at start-up, or code that must not enter the
+ * allocator while other work runs, since cudaMalloc and cudaFree can
+ * synchronise the device); it calls no allocating routine.
+ * The decode pair runs 32 tokens per launch where their folded activations
+ * fit the array (Kp <= 21760), else 16 (Kp <= 43648); a layer whose fold does
+ * not fit even then runs the register-operand GEMV, which needs no
+ * workspace. Larger M repeat the launches (ceil(M / 32) or ceil(M / 16) fold
+ * + decode pairs), up to 64 tokens; above that the prefill GEMM runs as in
+ * unisvq_linear.
  * The first call on a device looks up the array's device address
  * (cudaGetSymbolAddress, with that device current); make it before any
- * stream capture. All calls on a device share the one array, so calls that
- * overlap on the GPU race: order them on one stream. Arguments as
- * unisvq_linear. Errors: INVALID_ARG (as unisvq_linear), UNSUPPORTED (the
- * layer's fold needs more than the array: Kp > 43648), CUDA.
+ * stream capture. A cudaDeviceReset invalidates that address: reload the
+ * library after one. All calls on a device share the one array, so calls
+ * that overlap on the GPU race: order them on one stream. Arguments and
+ * errors as unisvq_linear.
  */
 unisvq_status unisvq_linear_noalloc(unisvq_handle h, const void* x, void* y, int M, void* stream);
 

@@ -1,4 +1,4 @@
-// Skinny GEMM for decode batches (M <= 16 tokens per launch): tcgen05 tensor
+// Skinny GEMM for decode batches (M <= 32 tokens per launch): tcgen05 tensor
 // cores with the 2-bit codes as an 8-bit operand resident in tensor memory.
 //
 // Computes y = x W_hat^T through the fold of Eq. (col:matmul):
@@ -19,7 +19,7 @@
 // activations, scaled per token and K slice by 2^P (|x' 2^P| < 256), are
 // split into three e4m3 terms h + m + l (about 12 significant bits, the
 // precision of fp16); the terms of token m are B rows 3m, 3m+1, 3m+2, so one
-// MMA of N = 16/32/48 columns covers every term of up to 5/10/16 tokens and a
+// MMA of N = 16/32/48/96 columns covers every term of up to 5/10/16/32 tokens and a
 // 128 x 128 k-tile takes four tcgen05.mma.kind::f8f6f4 (K = 32). The epilogue
 // adds the three term columns of a token and multiplies by 2^(9 - P).
 //
@@ -43,6 +43,8 @@
 // after it, so codes stream while the fold kernel runs. Layers that share x
 // (same K) run in one launch of each kernel: their row blocks are stacked
 // along grid.y of decode_kernel, their folds along grid.z of fold_kernel.
+#include <atomic>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -53,15 +55,16 @@ constexpr int kWarps = 10;
 constexpr int kThreads = kWarps * 32;
 constexpr int kConvWarp0 = 2;
 constexpr int kConvWarps = 8;
-constexpr int kMaxTokPerLaunch = 16;
+constexpr int kMaxTokPerLaunch = 32;
 constexpr int kMaxSplit = 8;                        // K slices (cluster size)
 constexpr int kMaxGroup = UNISVQ_MAX_GROUP;
 constexpr int kFoldThreads = 256;
 
 // Fold workspace of a handle (unisvq_layer::fold_ws): a table of per-(slice,
 // token) scale exponents and bias sums, then the B tiles of every k-tile.
-constexpr int kWsTableBytes = 1024;                 // int pexp[8][16], float cpart[8][16]
-constexpr int kWsTileStride = 48 * 128;             // B tile bytes per k-tile at the widest N
+constexpr int kWsTableBytes = 2048;                 // int pexp[8][32] at 0, float cpart[8][32] at kWsCpart
+constexpr int kWsCpart = 1024;
+constexpr int kWsTileStride = 96 * 128;             // B tile bytes per k-tile at the widest N
 
 struct SkLayer {
   const uint8_t* codes;
@@ -102,21 +105,23 @@ struct FoldArgs {
 };
 
 // Geometry: T k-tiles per pipeline stage. T = 2: 256 TMEM columns (accumulator
-// in [0, 64), three A slots of 64), two CTAs per SM. T = 1: 128 TMEM columns
-// (accumulator in [0, 32), three A slots of 32), N <= 32, three CTAs per SM.
+// in [0, 64), three A slots of 64), two CTAs per SM; for N = 96 (up to 32
+// tokens) 512 columns (accumulator in [0, 128)), one CTA per SM. T = 1: 128
+// TMEM columns (accumulator in [0, 32), three A slots of 32), N <= 32, three
+// CTAs per SM.
 // (One-tile stages for N = 48 would leave room for two A slots only; measured
 // slower than two-tile stages on every Llama shape.)
 template <int NCOL, int T>
 struct Cfg {
   static constexpr int kT = T;
-  static constexpr int kMinBlocks = T == 1 ? 3 : 2;
+  static constexpr int kMinBlocks = T == 1 ? 3 : (NCOL > 64 ? 1 : 2);
   static constexpr int kCodeBytes = T * kTileBytes;
-  static constexpr int kAColBase = T == 1 ? 32 : 64;
+  static constexpr int kAColBase = T == 1 ? 32 : (NCOL > 64 ? 128 : 64);
   static constexpr int kASlots = 3;                              // TMEM A slots (one stage each)
   static constexpr int kASlotCols = 32 * T;
-  static constexpr int kTmemCols = T == 1 ? 128 : 256;
+  static constexpr int kTmemCols = T == 1 ? 128 : (NCOL > 64 ? 512 : 256);
   static constexpr int kMaxTok = NCOL / 3;
-  static constexpr int kStages = NCOL == 48 ? 4 : 6;
+  static constexpr int kStages = NCOL >= 48 ? 4 : 6;
   static constexpr int kBTile = NCOL * 128;                      // one k-tile of B (NCOL rows x 128 bytes)
   static constexpr int kBBytes = T * kBTile;
   static constexpr int kStageBytes = kCodeBytes + kBBytes;       // [codes | B tiles]
@@ -124,8 +129,8 @@ struct Cfg {
   static constexpr int kRedBytes = (kTileRows + 8) * kMaxTok * 4;
   static constexpr int kOffBars = kOffRed + (kRedBytes + 15) / 16 * 16;
   static constexpr int kNumBars = 4 * kStages + 2 * kASlots + 3;
-  static constexpr int kOffTok = kOffBars + kNumBars * 8;        // pexp[16], cpart[16]
-  static constexpr int kOffMisc = kOffTok + 128;                 // tmem ptr, abort flag
+  static constexpr int kOffTok = kOffBars + kNumBars * 8;        // pexp[32], cpart[32]
+  static constexpr int kOffMisc = kOffTok + 256;                 // tmem ptr, abort flag
   static constexpr int kSmem = kOffMisc + 64 + 1024;             // + alignment slack
   // kind::f8f6f4: D f32, A and B e4m3, both K-major, N = NCOL, M = 128.
   static constexpr uint32_t kIdesc =
@@ -373,8 +378,8 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
     if (bound > 0.f) frexpf(bound, &e2);
     const int P = bound > 0.f ? max(-100, min(100, 8 - e2)) : 0;
     sp = P;
-    reinterpret_cast<int*>(ws)[s * 16 + tok] = P;
-    reinterpret_cast<float*>(ws + 512)[s * 16 + tok] = tcs;
+    reinterpret_cast<int*>(ws)[s * kMaxTokPerLaunch + tok] = P;
+    reinterpret_cast<float*>(ws + kWsCpart)[s * kMaxTokPerLaunch + tok] = tcs;
   }
   __syncthreads();
   const int P = sp;
@@ -476,7 +481,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
   const uint32_t bar_tail = bar0 + 8u * (4 * S + 2 * kASlots);
   const uint32_t d_full = bar_tail, tmem_ready = bar_tail + 8, drain = bar_tail + 16;
   int* pexp = reinterpret_cast<int*>(smem + C::kOffTok);
-  float* cpart = reinterpret_cast<float*>(smem + C::kOffTok + 64);
+  float* cpart = reinterpret_cast<float*>(smem + C::kOffTok + 128);
   uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 8);
   float* red = reinterpret_cast<float*>(smem + C::kOffRed);
@@ -644,8 +649,8 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
       if (!ok) *abort_flag = 1;
       pdl_wait();   // the scale table comes from the fold kernel
       if (q == 0 && lane < M) {
-        pexp[lane] = reinterpret_cast<const int*>(lws)[blockIdx.x * 16 + lane];
-        cpart[lane] = reinterpret_cast<const float*>(lws + 512)[blockIdx.x * 16 + lane];
+        pexp[lane] = reinterpret_cast<const int*>(lws)[blockIdx.x * kMaxTokPerLaunch + lane];
+        cpart[lane] = reinterpret_cast<const float*>(lws + kWsCpart)[blockIdx.x * kMaxTokPerLaunch + lane];
       }
       named_barrier_sync(1, 4 * 32);
       const int rows_per = (kTileRows + KS - 1) / KS;
@@ -704,7 +709,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
   }
 }
 
-int ncol_for(int M) { return M <= 5 ? 16 : (M <= 10 ? 32 : 48); }
+int ncol_for(int M) { return M <= 5 ? 16 : (M <= 10 ? 32 : (M <= 16 ? 48 : 96)); }
 
 template <int NCOL, int T>
 bool set_attrs(int dev) {
@@ -735,19 +740,20 @@ bool set_fold_attrs(int dev) {
 
 template <int T>
 size_t smem_of(int ncol) {
-  return ncol == 16 ? Cfg<16, T>::kSmem : (ncol == 32 ? Cfg<32, T>::kSmem : Cfg<48, 2>::kSmem);
+  return ncol == 16 ? Cfg<16, T>::kSmem
+                    : (ncol == 32 ? Cfg<32, T>::kSmem : (ncol == 48 ? Cfg<48, 2>::kSmem : Cfg<96, 2>::kSmem));
 }
 
 // Resident CTAs per SM: as many as the shared memory, the TMEM columns
 // (512 / kTmemCols) and the registers of 320 threads allow (two for T = 2,
-// three for T = 1). The occupancy query of the runtime reports one for this
+// one for the 96-column accumulator, three for T = 1). The occupancy query of the runtime reports one for this
 // kernel although two or three run side by side (measured), so the count is
 // derived here.
 int resident_for(int ncol, int T) {
   const size_t smem = T == 1 ? smem_of<1>(ncol) : smem_of<2>(ncol);
   const int by_smem = static_cast<int>((static_cast<size_t>(228) * 1024) / (smem + 1024));
-  const int by_tmem = T == 1 ? 4 : 2;
-  const int by_regs = T == 1 ? 3 : 2;
+  const int by_tmem = T == 1 ? 4 : (ncol > 64 ? 1 : 2);
+  const int by_regs = T == 1 ? 3 : (ncol > 64 ? 1 : 2);
   return max(1, min(by_smem, min(by_tmem, by_regs)));
 }
 
@@ -820,6 +826,12 @@ unisvq_status launch_ncol(const SkArgs& a, const DecodePlan& p, int dev, cudaStr
 
 size_t fold_workspace_bytes(int KT) { return kWsTableBytes + static_cast<size_t>(KT) * kWsTileStride; }
 
+// Fold workspace a launch of at most max_tok tokens writes (B tiles of the
+// launch's N only).
+static size_t fold_workspace_bytes_for(int KT, int max_tok) {
+  return kWsTableBytes + static_cast<size_t>(KT) * ncol_for(max_tok) * 128;
+}
+
 DecodePlan plan_skinny(const unisvq_layer* L, int M) {
   return plan_rows_split(L->Np / kTileRows, L->KT, L->num_sms, M > kMaxTokPerLaunch ? kMaxTokPerLaunch : M);
 }
@@ -859,9 +871,10 @@ unisvq_status launch_fold(const unisvq_layer* const* Ls, int n, const void* x, i
   return cudaLaunchKernelEx(&fc, fold_kernel<DV>, f) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
-// Fold and stream, the fold workspace of layer i at ws[i].
+// Fold and stream, the fold workspace of layer i at ws[i], at most max_tok
+// tokens per launch.
 unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
-                               cudaStream_t s, uint8_t* const* ws) {
+                               cudaStream_t s, uint8_t* const* ws, int max_tok = kMaxTokPerLaunch) {
   if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
   const unisvq_layer* L0 = Ls[0];
   if (!set_fold_attrs(L0->device)) return UNISVQ_ERR_CUDA;
@@ -871,8 +884,8 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
     nb += Ls[i]->Np / kTileRows;
     d8 = d8 || Ls[i]->d == 8;
   }
-  for (int m0 = 0; m0 < M; m0 += kMaxTokPerLaunch) {
-    const int mc = M - m0 < kMaxTokPerLaunch ? M - m0 : kMaxTokPerLaunch;
+  for (int m0 = 0; m0 < M; m0 += max_tok) {
+    const int mc = M - m0 < max_tok ? M - m0 : max_tok;
     const DecodePlan p = plan_rows_split(nb, L0->KT, L0->num_sms, mc);
     if (p.ks > kMaxSplit) return UNISVQ_ERR_UNSUPPORTED;
     SkArgs a{};
@@ -896,7 +909,8 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
     if (st != UNISVQ_OK) return st;
     if (p.nt == 16) st = p.geom == 1 ? launch_ncol<16, 1>(a, p, L0->device, s) : launch_ncol<16, 2>(a, p, L0->device, s);
     else if (p.nt == 32) st = p.geom == 1 ? launch_ncol<32, 1>(a, p, L0->device, s) : launch_ncol<32, 2>(a, p, L0->device, s);
-    else st = launch_ncol<48, 2>(a, p, L0->device, s);
+    else if (p.nt == 48) st = launch_ncol<48, 2>(a, p, L0->device, s);
+    else st = launch_ncol<96, 2>(a, p, L0->device, s);
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;
@@ -930,19 +944,25 @@ __device__ __align__(256) uint8_t g_static_fold_ws[kStaticWsBytes];
 size_t static_fold_workspace_bytes() { return kStaticWsBytes; }
 
 unisvq_status launch_skinny_static(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
-  if (fold_workspace_bytes(L->KT) > kStaticWsBytes) return UNISVQ_ERR_UNSUPPORTED;
+  // 32 tokens per launch where their B tiles fit the array, else 16
+  const int max_tok = fold_workspace_bytes_for(L->KT, kMaxTokPerLaunch) <= kStaticWsBytes ? kMaxTokPerLaunch : 16;
+  if (fold_workspace_bytes_for(L->KT, max_tok) > kStaticWsBytes) return UNISVQ_ERR_UNSUPPORTED;
   // In host code g_static_fold_ws only names the symbol; its device address
-  // is looked up once per device (the device of L is current here).
-  static uint8_t* dev_ptr[64] = {};
+  // is looked up once per device (the device of L is current here) and kept
+  // in an atomic slot, so concurrent first calls store the same value. A
+  // cudaDeviceReset unloads the module: the library must then be reloaded.
+  static std::atomic<uint8_t*> dev_ptr[64] = {};
   if (L->device < 0 || L->device >= 64) return UNISVQ_ERR_INVALID_ARG;
-  if (!dev_ptr[L->device]) {
+  uint8_t* wsp = dev_ptr[L->device].load(std::memory_order_acquire);
+  if (!wsp) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_static_fold_ws) != cudaSuccess || !p) return UNISVQ_ERR_CUDA;
-    dev_ptr[L->device] = static_cast<uint8_t*>(p);
+    wsp = static_cast<uint8_t*>(p);
+    dev_ptr[L->device].store(wsp, std::memory_order_release);
   }
-  uint8_t* ws[1] = {dev_ptr[L->device]};
+  uint8_t* ws[1] = {wsp};
   void* ys[1] = {y};
-  return launch_skinny_ws(&L, 1, x, ys, M, s, ws);
+  return launch_skinny_ws(&L, 1, x, ys, M, s, ws, max_tok);
 }
 
 }  // namespace unisvq

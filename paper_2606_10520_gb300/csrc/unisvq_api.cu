@@ -1,5 +1,6 @@
 // C-ABI entry points of libunisvq: argument validation, the layer handle,
 // kernel dispatch and the device error word.
+#include <atomic>
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
@@ -14,8 +15,9 @@ namespace unisvq {
 namespace {
 __device__ int g_error_word;
 
-// Per-device cache of the error word's device address.
-int* g_err_ptr[64] = {};
+// Per-device cache of the error word's device address (atomic: concurrent
+// first calls from several host threads store the same value).
+std::atomic<int*> g_err_ptr[64] = {};
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
@@ -35,12 +37,14 @@ unisvq_status cuda_status(cudaError_t e) {
 int* device_error_word() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-  if (!g_err_ptr[dev]) {
+  int* cached = g_err_ptr[dev].load(std::memory_order_acquire);
+  if (!cached) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
-    g_err_ptr[dev] = static_cast<int*>(p);
+    cached = static_cast<int*>(p);
+    g_err_ptr[dev].store(cached, std::memory_order_release);
   }
-  return g_err_ptr[dev];
+  return cached;
 }
 
 }  // namespace unisvq
@@ -442,7 +446,15 @@ static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, vo
       void* ys[1] = {y};
       return launch_grouped_group(Ls, 1, x, ys, M, s);
     }
-    return launch_skinny_static(h, x, y, M, s);
+    // unisvq_linear's own pick; only the tcgen05 decode kernels use a fold
+    // workspace, here the static one, or the GEMV where the fold does not fit it
+    const int k = auto_kernel(h, M);
+    if (k == UNISVQ_KERNEL_PREFILL) return launch_prefill(h, x, y, M, s);
+    if (k == UNISVQ_KERNEL_SKINNY) {
+      const unisvq_status st = launch_skinny_static(h, x, y, M, s);
+      if (st != UNISVQ_ERR_UNSUPPORTED) return st;
+    }
+    return launch_gemv(h, x, y, M, s);
   }
   if (h->grouped) {   // per-group maps: the prefill GEMM (d = 2, 4) for M > 64, else the per-group GEMV
     if ((kernel == UNISVQ_KERNEL_AUTO && M > 64 && prefill_supported(h, M)) || kernel == UNISVQ_KERNEL_PREFILL)
@@ -761,12 +773,12 @@ static void describe_launch(const unisvq_layer* const* Ls, int n, int kernel, in
     info->launches = (m + 31) / 32;
     info->grid_ctas = p.ks * nb * info->launches;
   } else if (kernel == UNISVQ_KERNEL_SKINNY) {
-    const DecodePlan p = plan_skinny(h, m > 16 ? 16 : m);
+    const DecodePlan p = plan_skinny(h, m > 32 ? 32 : m);
     int nb = 0;
     for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
     info->split_k = p.ks;
-    const int chunks = (m + 15) / 16;
-    info->launches = 2 * chunks;   // fold kernel + streaming kernel per 16 tokens
+    const int chunks = (m + 31) / 32;
+    info->launches = 2 * chunks;   // fold kernel + streaming kernel per 32 tokens
     info->grid_ctas = p.ks * nb * chunks;
   } else if (prefill_group_supported(Ls, n, m)) {   // one launch over every layer's tiles
     const PrefillPlan p = plan_prefill_group(Ls, n, m);

@@ -159,6 +159,7 @@ def test_grouped_entry_points():
         assert layer.forward_ptr(x.data_ptr(), y.data_ptr(), 5, stream, kern) == binding.ERR_UNSUPPORTED
     for kern in (binding.KERNEL_AUTO, binding.KERNEL_DECODE, binding.KERNEL_GROUPED, binding.KERNEL_PREFILL):
         assert layer.forward_ptr(x.data_ptr(), y.data_ptr(), 5, stream, kern) == binding.OK
+    y.fill_(float("nan"))   # the results of the calls above must not survive
     assert layer.forward_noalloc_ptr(x.data_ptr(), y.data_ptr(), 5, stream) == binding.OK
     assert binding.sync_status() == binding.OK
     check(y.float().cpu().numpy().astype(np.float64), xb, codes, A, B)

@@ -364,7 +364,7 @@ def test_dispatch_picks_tcgen05_decode_for_large_launches():
     big = binding.UniSVQLinear(*synth.layer_inputs(9, 91, 0, 0, 16384, 4096, 2))
     q = big.query(1)
     assert q["kernel"] == binding.KERNEL_SKINNY and q["launches"] == 2
-    assert big.query(17)["launches"] == 4
+    assert big.query(17)["launches"] == 2 and big.query(33)["launches"] == 4   # 32 tokens per pair
     small = binding.UniSVQLinear(*synth.layer_inputs(9, 91, 1, 0, 4096, 4096, 2))
     assert small.query(16)["kernel"] == binding.KERNEL_GEMV and small.query(16)["launches"] == 1
     tall = binding.UniSVQLinear(*synth.layer_inputs(9, 91, 2, 0, 4096, 11008, 2))   # 2^25.4 weights, 32 row blocks
