@@ -37,6 +37,7 @@ constexpr int kBK = 64;                  // bf16 columns per stage (one 128B swi
 constexpr int kATileBytes = kBM * 128;   // 16 KB
 constexpr int kConvWarp0 = 2;
 constexpr int kEpiWarp0 = 10;
+constexpr int kCodeAhead = 8;   // stages of codes in flight per converter lane (8: 1081 vs 1066 TFLOP/s for 3)
 
 // Layers of one launch (several only for 2-bit layers with one d <= 4 that
 // read the same x, all per-matrix or all per-group): their tiles are numbered
@@ -527,7 +528,8 @@ __global__ void __launch_bounds__(kPfThreads, 1)
           const uint8_t* rbase =
               pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
           const uint32_t lut_s = lut_base + 2048u * static_cast<uint32_t>(li);
-          // Code words of stage kb live at tile kb/2, half kb%2; prefetched 3 stages ahead.
+          // Code words of stage kb live at tile kb/2, half kb%2; prefetched
+          // kCodeAhead stages ahead (a register ring).
           auto load = [&](int kb) -> uint2 {
             return kb < a.nkb ? __ldg(reinterpret_cast<const uint2*>(rbase + (kb >> 1) * kTileBytes + (kb & 1) * 8))
                               : make_uint2(0, 0);
@@ -543,21 +545,27 @@ __global__ void __launch_bounds__(kPfThreads, 1)
                          : 0u;
             return 0u;
           };
-          uint2 q0 = load(0), q1 = load(1), q2 = load(2);
-          uint32_t h0 = load_hi(0), h1 = load_hi(1), h2 = load_hi(2);
+          uint2 qr[kCodeAhead];
+          uint32_t hr[kCodeAhead];
+#pragma unroll
+          for (int j = 0; j < kCodeAhead; ++j) {
+            qr[j] = load(j);
+            hr[j] = load_hi(j);
+          }
+          // The stage loop is unrolled by the ring depth so that slot j is read
+          // and refilled in place: shifting a register ring would read slots
+          // whose loads are still in flight and wait for them every stage.
           bool ok = !*abort_flag;
-          for (int kb = 0; kb < a.nkb; ++kb, ++it) {
+          for (int kb0 = 0; kb0 < a.nkb; kb0 += kCodeAhead) {
+#pragma unroll
+          for (int j = 0; j < kCodeAhead; ++j) {
+            const int kb = kb0 + j;
+            if (kb >= a.nkb) break;
             const int s = it % STAGES;
-            const uint2 cw = q0;
-            q0 = q1;
-            q1 = q2;
-            q2 = load(kb + 3);
-            const uint32_t hw = h0;
-            if constexpr (HI) {
-              h0 = h1;
-              h1 = h2;
-              h2 = load_hi(kb + 3);
-            }
+            const uint2 cw = qr[j];
+            const uint32_t hw = hr[j];
+            qr[j] = load(kb + kCodeAhead);
+            if constexpr (HI) hr[j] = load_hi(kb + kCodeAhead);
             if (ok && it >= STAGES) {
               ok = !*abort_flag && mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty);
               if (!ok) *abort_flag = 1;
@@ -632,6 +640,8 @@ __global__ void __launch_bounds__(kPfThreads, 1)
             }
             __syncwarp();
             if (lane == 0 && ok) mbar_arrive(afull(s));
+            ++it;
+          }
           }
         }
       };
