@@ -43,8 +43,11 @@ identity of Eq. (col:matmul); for the per-group functions, the hand-worked
 example in tests/golden/grouped_hand_worked.json, group-wise uniform scalar
 quantisation (A = s I), reduction to the per-matrix oracle when all groups
 share one map, and the exchange-of-sums identity; for the RHT functions,
-H H^T = n I for every order built, Sylvester's matrix against SciPy's, and the
-undo identity: the RHT layer applied to W_hat = R(W) returns x W^T; for the
+H H^T = n I for every order built, Sylvester's matrix against SciPy's and
+against its closed form (-1)^popcount(p & p'), the field axioms of GF(343)
+and the multiplicativity of its quadratic character (with planted mistakes
+caught: a reducible modulus, the ring Z/343, a dropped reduction term), and
+the undo identity: the RHT layer applied to W_hat = R(W) returns x W^T; for the
 bf16 widening that every activation passes through, hand-chosen bit patterns
 (signed zero, subnormals, the largest finite value, infinities) against the
 IEEE bfloat16 definition. No function here is "parity unpinned".
@@ -240,18 +243,75 @@ def _quadratic_character(q: int) -> np.ndarray:
     return chi
 
 
-def paley_hadamard(m: int) -> np.ndarray:
-    """A +-1 Hadamard matrix of order m in {12, 20, 28} (Paley's constructions).
+# GF(343) = GF(7)[t] / (t^3 - c(t)): t^3 is replaced by the coefficients below
+# (c0, c1, c2), here t^3 = 2. t^3 - 2 is irreducible over GF(7) because it has
+# no root there (2 is not a cube mod 7), so the quotient is a field.
+_GF343_T3 = (2, 0, 0)
 
-    Order q + 1 with q = 11, 19 (q = 3 mod 4, prime): with the Jacobsthal matrix
-    Q[i][j] = chi(j - i), H = I + [[0, 1^T], [-1, Q]].
+
+def gf343_digits(e):
+    """Element e in 0..342 of GF(343) as its coefficients (c0, c1, c2) of
+    c0 + c1 t + c2 t^2, with e = c0 + 7 c1 + 49 c2 (works elementwise on arrays)."""
+    e = np.asarray(e)
+    return e % 7, (e // 7) % 7, e // 49
+
+
+def gf343_index(c0, c1, c2):
+    return (np.asarray(c0) % 7) + 7 * (np.asarray(c1) % 7) + 49 * (np.asarray(c2) % 7)
+
+
+def gf343_sub(a, b):
+    """a - b in GF(343): coefficient-wise mod 7."""
+    a0, a1, a2 = gf343_digits(a)
+    b0, b1, b2 = gf343_digits(b)
+    return gf343_index(a0 - b0, a1 - b1, a2 - b2)
+
+
+def gf343_mul(a, b):
+    """a b in GF(343): the polynomial product, with t^3 and t^4 = t t^3 reduced
+    through _GF343_T3."""
+    a = gf343_digits(a)
+    b = gf343_digits(b)
+    p = [0, 0, 0, 0, 0]
+    for i in range(3):
+        for j in range(3):
+            p[i + j] = p[i + j] + a[i] * b[j]
+    r0, r1, r2 = _GF343_T3
+    # t^3 = r0 + r1 t + r2 t^2; t^4 = r0 t + r1 t^2 + r2 t^3
+    c = [p[0], p[1], p[2]]
+    t4 = [0, r0, r1]            # t^4 without its t^3 term r2 t^3
+    for k in range(3):
+        c[k] = c[k] + p[3] * (r0, r1, r2)[k] + p[4] * t4[k]
+    c = [c[k] + p[4] * r2 * (r0, r1, r2)[k] for k in range(3)]
+    return gf343_index(c[0], c[1], c[2])
+
+
+def gf343_quadratic_character() -> np.ndarray:
+    """chi(e) for e in 0..342: 0 at 0, +1 on the nonzero squares of GF(343), -1 otherwise."""
+    e = np.arange(1, 343)
+    chi = -np.ones(343, dtype=np.int64)
+    chi[0] = 0
+    chi[gf343_mul(e, e)] = 1
+    return chi
+
+
+def paley_hadamard(m: int) -> np.ndarray:
+    """A +-1 Hadamard matrix of order m in {12, 20, 28, 344} (Paley's constructions).
+
+    Order q + 1 with q = 11, 19 (prime) or 343 = 7^3 (q = 3 mod 4): with the
+    Jacobsthal matrix Q[i][j] = chi(e_j - e_i) over the field of order q (for
+    343, e_i is the field element of index i, `gf343_digits`),
+    H = I + [[0, 1^T], [-1, Q]].
     Order 2(q + 1) with q = 13 (q = 1 mod 4, prime): with the symmetric
     conference matrix C = [[0, 1^T], [1, Q]], H = [[C + I, C - I], [C - I, -C - I]].
     """
-    if m in (12, 20):
+    if m in (12, 20, 344):
         q = m - 1
-        chi = _quadratic_character(q)
-        Q = chi[(np.arange(q)[None, :] - np.arange(q)[:, None]) % q]
+        idx = np.arange(q)
+        if q == 343:
+            Q = gf343_quadratic_character()[gf343_sub(idx[None, :], idx[:, None])]
+        else:
+            Q = _quadratic_character(q)[(idx[None, :] - idx[:, None]) % q]
         S = np.zeros((m, m), dtype=np.int64)
         S[0, 1:] = 1
         S[1:, 0] = -1
@@ -267,12 +327,12 @@ def paley_hadamard(m: int) -> np.ndarray:
         C[1:, 1:] = Q
         I = np.eye(q + 1, dtype=np.int64)
         return np.block([[C + I, C - I], [C - I, -C - I]])
-    raise ValueError("Paley order must be 12, 20 or 28")
+    raise ValueError("Paley order must be 12, 20, 28 or 344")
 
 
 def hadamard_factor(n: int):
-    """(2^a, m) with n = 2^a m and m in {1, 12, 20, 28} (the largest such m), or None."""
-    for m in (28, 20, 12, 1):
+    """(2^a, m) with n = 2^a m and m in {1, 12, 20, 28, 344} (the largest such m), or None."""
+    for m in (344, 28, 20, 12, 1):
         if n % m == 0:
             p = n // m
             if p & (p - 1) == 0:
@@ -286,7 +346,7 @@ def hadamard(n: int) -> np.ndarray:
     [(p, q), (p', q')] at index p m + q is H_{2^a}[p][p'] H_m[q][q']."""
     f = hadamard_factor(n)
     if f is None:
-        raise ValueError(f"no Hadamard matrix of order {n} is built (n = 2^a m, m in 1, 12, 20, 28)")
+        raise ValueError(f"no Hadamard matrix of order {n} is built (n = 2^a m, m in 1, 12, 20, 28, 344)")
     p, m = f
     H = np.ones((1, 1), dtype=np.int64)
     while H.shape[0] < p:

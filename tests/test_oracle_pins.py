@@ -379,7 +379,7 @@ def test_grouped_linearity_and_row_chunks():
 # randomized Hadamard transform, Eq. (def:hadamard)
 # --------------------------------------------------------------------------
 
-@pytest.mark.parametrize("n", [1, 2, 8, 12, 20, 28, 64, 96, 112, 160, 448, 1024])
+@pytest.mark.parametrize("n", [1, 2, 8, 12, 20, 28, 64, 96, 112, 160, 344, 448, 688, 1024])
 def test_hadamard_is_orthogonal_pm1(n):
     H = oracle.hadamard(n)
     assert H.shape == (n, n) and set(np.unique(H)) <= {-1, 1}
@@ -396,12 +396,102 @@ def test_hadamard_factor_of_model_widths():
     assert oracle.hadamard_factor(4096) == (4096, 1)
     assert oracle.hadamard_factor(14336) == (512, 28)
     assert oracle.hadamard_factor(28672) == (1024, 28)
-    assert oracle.hadamard_factor(11008) is None        # 64 * 172: no order-172 matrix is built
+    assert oracle.hadamard_factor(11008) == (32, 344)   # 2^5 * (7^3 + 1)
+    assert oracle.hadamard_factor(11008 // 2 * 3) is None
     with pytest.raises(ValueError):
-        oracle.hadamard(11008)
+        oracle.hadamard(172)
 
 
-@pytest.mark.parametrize("N,K", [(24, 64), (56, 40), (16, 112)])
+# GF(343) and the order-344 Paley matrix: pinned to the field axioms, the
+# character's defining property and H H^T = n I, not to the oracle's own output.
+
+def gf343_field_ok(o) -> bool:
+    """The modulus has no root in GF(7), and the multiplication table of the
+    343 elements is that of a field: commutative, associative on a sample,
+    distributive over the coefficient-wise sum, every nonzero row a
+    permutation of the nonzero elements (inverses exist and are unique)."""
+    r0, r1, r2 = o._GF343_T3
+    if any((t ** 3 - (r0 + r1 * t + r2 * t * t)) % 7 == 0 for t in range(7)):
+        return False
+    e = np.arange(343)
+    T = o.gf343_mul(e[:, None], e[None, :])
+    if not np.array_equal(T, T.T) or np.any(T[0] != 0) or np.any(T[1] != e):
+        return False
+    if any(sorted(T[a, 1:]) != list(range(1, 343)) for a in range(1, 343)):
+        return False
+    g = np.random.default_rng(343)
+    a, b, c = (g.integers(0, 343, size=2000) for _ in range(3))
+    if not np.array_equal(T[T[a, b], c], T[a, T[b, c]]):
+        return False
+    add = lambda u, v: o.gf343_sub(u, o.gf343_sub(0, v))
+    return bool(np.array_equal(T[a, add(b, c)], add(T[a, b], T[a, c])))
+
+
+def paley344_ok(o) -> bool:
+    """chi is multiplicative with 171 squares and chi(-1) = -1 (343 = 3 mod 4);
+    the matrix is +-1, of Paley form (first row all +1, H - I antisymmetric)
+    and H H^T = 344 I."""
+    chi = o.gf343_quadratic_character()
+    e = np.arange(343)
+    T = o.gf343_mul(e[:, None], e[None, :])
+    if not np.array_equal(chi[T], chi[:, None] * chi[None, :]):
+        return False
+    if (chi == 1).sum() != 171 or chi[o.gf343_sub(0, 1)] != -1:
+        return False
+    H = o.paley_hadamard(344)
+    S = H - np.eye(344, dtype=np.int64)
+    return bool(set(np.unique(H)) <= {-1, 1} and np.all(H[0] == 1) and np.array_equal(S, -S.T)
+                and np.array_equal(H @ H.T, 344 * np.eye(344, dtype=np.int64)))
+
+
+def test_gf343_is_a_field():
+    assert gf343_field_ok(oracle)
+
+
+def test_paley_344_is_hadamard():
+    assert paley344_ok(oracle)
+
+
+def test_hadamard_11008_is_sylvester_32_kron_paley_344():
+    """Entries and orthogonality of sampled rows of the order-11008 matrix."""
+    H = oracle.hadamard(11008)
+    H344 = oracle.paley_hadamard(344)
+    g = np.random.default_rng(11008)
+    i, j = g.integers(0, 11008, size=(2, 3000))
+    p, q, pp, qq = i // 344, i % 344, j // 344, j % 344
+    syl = np.where(np.bitwise_count(p & pp) % 2 == 1, -1, 1)   # Sylvester: (-1)^popcount(p & p')
+    assert np.array_equal(H[i, j], syl * H344[q, qq])
+    rows = g.choice(11008, size=12, replace=False)
+    G = H[rows] @ H[rows].T
+    assert np.array_equal(G, 11008 * np.eye(12, dtype=np.int64))
+
+
+def test_gf343_pins_catch_planted_mistakes(monkeypatch):
+    # a reducible modulus (t^3 - t - 1 has the root 5 mod 7): a ring, not a field
+    monkeypatch.setattr(oracle, "_GF343_T3", (1, 1, 0))
+    assert not gf343_field_ok(oracle)
+    assert not paley344_ok(oracle)
+    monkeypatch.undo()
+    # the integers mod 343 in place of the field: chi of Z/343 is no character
+    monkeypatch.setattr(oracle, "gf343_mul", lambda a, b: (np.asarray(a) * np.asarray(b)) % 343)
+    monkeypatch.setattr(oracle, "gf343_sub", lambda a, b: (np.asarray(a) - np.asarray(b)) % 343)
+    assert not paley344_ok(oracle)
+    monkeypatch.undo()
+    # the t^4 reduction dropped (t^4 read as 0)
+    real = oracle.gf343_mul
+
+    def no_t4(a, b):
+        a0, a1, a2 = oracle.gf343_digits(a)
+        b0, b1, b2 = oracle.gf343_digits(b)
+        p0, p1, p2, p3 = a0 * b0, a0 * b1 + a1 * b0, a0 * b2 + a1 * b1 + a2 * b0, a1 * b2 + a2 * b1
+        return oracle.gf343_index(p0 + 2 * p3, p1, p2)
+    monkeypatch.setattr(oracle, "gf343_mul", no_t4)
+    assert not gf343_field_ok(oracle)
+    monkeypatch.setattr(oracle, "gf343_mul", real)
+    assert gf343_field_ok(oracle) and paley344_ok(oracle)
+
+
+@pytest.mark.parametrize("N,K", [(24, 64), (56, 40), (16, 112), (344, 64), (24, 688)])
 def test_rht_layer_undoes_the_weight_rotation(N, K):
     """Eq. (def:hadamard): if W_hat is exactly R(W) = U S_U W S_V V, the layer
     with the inverse transform around it returns x W^T. Checked with a dense W
