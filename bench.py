@@ -349,7 +349,8 @@ def run_ours(args, rank, world, local_rank):
         side = torch.cuda.Stream()
         print(json.dumps({"prefill": run_prefill(torch, binding, peaks, args, side)}), flush=True)
         return
-    variants = {"grouped": ("per_group_affine", run_grouped), "rht": ("rht", run_rht), "bits3": ("bits3", run_bits3)}
+    variants = {"grouped": ("per_group_affine", run_grouped), "rht": ("rht", run_rht), "bits3": ("bits3", run_bits3),
+                "rht7": ("rht_llama2_7b", lambda *a: run_rht(*a, which="llama2_7b"))}
     if args.only in variants:
         key, fn = variants[args.only]
         print(json.dumps({key: fn(torch, binding, peaks, args, torch.cuda.Stream())}), flush=True)
@@ -548,9 +549,10 @@ def run_ours(args, rank, world, local_rank):
         bits3 = run_bits3(torch, binding, peaks, args, side)
 
     # ---- inverse RHT around the layers -------------------------------------
-    rht = None
+    rht = rht7 = None
     if not args.no_rht:
         rht = run_rht(torch, binding, peaks, args, side)
+        rht7 = run_rht(torch, binding, peaks, args, side, "llama2_7b")
 
     # ---- prefill (tcgen05 GEMM), Llama-3-8B-shaped set at M = 2048 -------
     prefill = None
@@ -601,6 +603,7 @@ def run_ours(args, rank, world, local_rank):
         "cublas_dense_decode": dense,
         "per_group_affine": grouped,
         "rht": rht,
+        "rht_llama2_7b": rht7,
         "bits3": bits3,
     }
     if rank == 0:
@@ -695,17 +698,21 @@ def run_bits3(torch, binding, peaks, args, stream):
             "timing": "CUDA graphs of the layer stack per M, CUDA events on the capture stream"}
 
 
-def run_rht(torch, binding, peaks, args, stream):
-    """The decode sweep on Llama-3-8B-shaped layers (every width 2^a m with a
-    Hadamard order here) with and without the inverse randomized Hadamard
-    transform around each layer (Eq. def:hadamard): q/k/v and gate/up share
-    their input rotation S_V V, every layer has its own output rotation U S_U.
-    GB/s counts the layers' algorithmic bytes only."""
-    shapes = synth.LLAMA3_8B
+RHT_SETS = {"llama3_8b": ("Llama-3-8B", synth.LLAMA3_8B, 2), "llama2_7b": ("Llama-2-7B", synth.LLAMA2_7B, 1)}
+
+
+def run_rht(torch, binding, peaks, args, stream, which="llama3_8b"):
+    """The decode sweep on Llama-3-8B- or Llama-2-7B-shaped layers with and
+    without the inverse randomized Hadamard transform around each layer (Eq.
+    def:hadamard): q/k/v and gate/up share their input rotation S_V V, every
+    layer has its own output rotation U S_U. Widths: 4096 = 2^12, 14336 =
+    2^9 * 28, 11008 = 2^5 * 344. GB/s counts the layers' algorithmic bytes
+    only (a group call's shared x once)."""
+    label, shapes, config_id = RHT_SETS[which]
     g = np.random.default_rng(5)
     base = []
     for pi, (_, N, K) in enumerate(shapes):
-        codes, A, B = synth.layer_inputs(0, 2, 0, pi, N, K, 2)
+        codes, A, B = synth.layer_inputs(0, config_id, 0, pi, N, K, 2)
         base.append(binding.UniSVQLinear(codes, A, B))
     s_in = {K: g.choice([-1.0, 1.0], K) for K in sorted({K for _, _, K in shapes})}
     s_out = [g.choice([-1.0, 1.0], N) for _, N, _ in shapes]
@@ -715,10 +722,10 @@ def run_rht(torch, binding, peaks, args, stream):
     for M in M_SWEEP:
         for pi, (_, N, K) in enumerate(shapes):
             if (M, K) not in xs:
-                xb = synth.activations(0, 2, 100 + M, M, K)
+                xb = synth.activations(0, config_id, 100 + M, M, K)
                 xs[(M, K)] = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).cuda()
             ys[(M, pi)] = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
-    step_bytes = sum(algo_bytes(N, K, M) for M in M_SWEEP for _, N, K in shapes) * nl
+    step_bytes = sum(group_bytes(shapes, grp, M) for M in M_SWEEP for grp in GROUPS_7B) * nl
     steps = max(5, args.steps // 4)
     out = {}
     for rht in (False, True):
@@ -754,11 +761,11 @@ def run_rht(torch, binding, peaks, args, stream):
     for layer in stack:
         for b in layer:
             b.close()
-    return {"workload": f"Llama-3-8B-shaped projection set x {nl} layers, decode sweep M in "
+    return {"workload": f"{label}-shaped projection set x {nl} layers, decode sweep M in "
                         f"{list(M_SWEEP)}, d=2, per-matrix fp16 affine, inverse RHT around every layer",
             "GB/s": out["with_rht"], "GB/s_without_rht": out["without_rht"],
             "frac_of_measured_hbm": out["with_rht"] / peaks["hbm_gbs"],
-            "kernels": "rht_kernel (input and output rotations, cluster of 8 CTAs per row) + the layers' kernels",
+            "kernels": "rht_kernel (input and output rotations, a cluster of 8 or 16 CTAs per row) + the layers' kernels",
             "bytes": "the layers' algorithmic bytes (codes + affine + x + y); the rotations are overhead",
             "timing": "CUDA graphs of the layer stack per M, CUDA events on the capture stream"}
 
@@ -1129,7 +1136,7 @@ def main():
     ap.add_argument("--layers-70b", type=int, default=80)
     ap.add_argument("--no-70b", action="store_true", help="skip config 3 (70B stack) and the crossover table")
     ap.add_argument("--no-dense", action="store_true", help="skip the cuBLAS dense decode reference")
-    ap.add_argument("--only", choices=["decode", "prefill", "grouped", "rht", "bits3"], default=None,
+    ap.add_argument("--only", choices=["decode", "prefill", "grouped", "rht", "rht7", "bits3"], default=None,
                     help="profiling aid: run only the decode sweep (no e2e/cpu/secondary sweeps), only the "
                          "prefill set, or only one secondary sweep (with --layers layers)")
     args = ap.parse_args()

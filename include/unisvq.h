@@ -258,9 +258,15 @@ unisvq_status unisvq_linear_noalloc(unisvq_handle h, const void* x, void* y, int
  * (row vectors): a rotation kernel on the way in, the layer's kernel, a
  * rotation kernel on the way out, per chunk of max_tokens tokens.
  * H_n is Sylvester's H_{2^a} Kronecker a Paley matrix H_m for n = 2^a m,
- * m in {1, 12, 20, 28} (entry [(p,q),(p',q')] = H_{2^a}[p][p'] H_m[q][q'],
- * index p m + q; H_12 and H_20 from Paley's first construction with q = 11
- * and 19, H_28 from the second with q = 13); n <= 58112 (n floats in shared memory).
+ * m in {1, 12, 20, 28, 344} (entry [(p,q),(p',q')] = H_{2^a}[p][p'] H_m[q][q'],
+ * index p m + q; H_12, H_20 and H_344 from Paley's first construction with
+ * q = 11, 19 and 343, H_28 from the second with q = 13). For q = 343 the
+ * field is GF(7)[t] / (t^3 - 2), element e = e0 + 7 e1 + 49 e2 standing for
+ * e0 + e1 t + e2 t^2, and H_344 = I + [[0, 1^T], [-1, Q]] with
+ * Q[i][j] = chi(e_j - e_i), chi the quadratic character. So 11008 = 32 * 344
+ * is supported. n <= 58112 (n floats in shared memory). The first call for a
+ * width with m = 344 on a device writes a 16 KB sign table to that device
+ * (a synchronous copy): make it outside stream capture.
  *   sign_in  : host, K bytes, 1 = -1 (the diagonal of S_V), 0 = +1
  *   sign_out : host, N bytes (S_U)
  *   max_tokens : rows of the rotated-activation buffer the handle allocates
@@ -279,7 +285,9 @@ unisvq_status unisvq_set_rht(unisvq_handle h, const uint8_t* sign_in, const uint
  * allowed, otherwise no overlap): signs_first = 1 gives y = (x S) H_n /
  * sqrt(n), signs_first = 0 gives y = ((x H_n) / sqrt(n)) S, S the diagonal
  * of `signs` (device, n bytes, 1 = -1; NULL = identity). fp32 inside, bf16
- * rounding once at the end. Errors: INVALID_ARG, UNSUPPORTED (n), CUDA. */
+ * rounding once at the end. H_n as for unisvq_set_rht; the first call with
+ * m = 344 on a device writes its sign table (outside stream capture).
+ * Errors: INVALID_ARG, UNSUPPORTED (n), CUDA. */
 unisvq_status unisvq_hadamard(const void* x, void* y, int M, int n, const uint8_t* signs, int signs_first,
                               void* stream);
 

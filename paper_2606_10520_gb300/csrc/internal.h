@@ -129,8 +129,12 @@ unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s);
 
 // Randomized Hadamard transform of M rows of n bf16 values (rht.cu):
 // signs_first = 1: out = (s x) H / sqrt(n); 0: out = s ((x H) / sqrt(n)).
-// n = 2^a m, m in {1, 12, 20, 28}; in and out may be the same rows.
+// n = 2^a m, m in {1, 12, 20, 28, 344}; in and out may be the same rows.
+// rht_prepare(n) writes the device's H_344 sign table when n needs it (a
+// synchronous copy, made once per device): call it outside stream capture
+// before the first launch_rht of such an n.
 bool rht_factor(int n, int* p2, int* m);
+unisvq_status rht_prepare(int n);
 size_t rht_smem_bytes(int n);
 unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_stride, int M, int n,
                          const uint8_t* signs, int signs_first, cudaStream_t s);

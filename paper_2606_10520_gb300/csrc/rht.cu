@@ -5,8 +5,9 @@
 // the way in (signs, then V) and the rows of the output on the way out (U,
 // then signs). U and V are normalised Hadamard matrices H_n / sqrt(n) of order
 // n = 2^a m: Sylvester's H_{2^a} Kronecker a Paley matrix H_m, m in
-// {1, 12, 20, 28}; entry [(p, q), (p', q')] (index p m + q) is
-// H_{2^a}[p][p'] H_m[q][q'].
+// {1, 12, 20, 28, 344}; entry [(p, q), (p', q')] (index p m + q) is
+// H_{2^a}[p][p'] H_m[q][q']. m = 344 (Paley I over the field of 7^3
+// elements) makes widths such as 11008 = 2^5 * 344 rotatable.
 //
 // A row is split over a cluster of G CTAs (rht_ctas: 8 or 16), CTA j
 // holding the 2^a / G consecutive m-blocks j 2^a / G .. in shared memory
@@ -19,7 +20,9 @@
 // position from the G CTAs' shared memory, transforms them in registers and
 // writes the scaled (and, on the way out, signed) bf16 results. A second
 // cluster barrier keeps every CTA's shared memory alive until all reads end.
+#include <atomic>
 #include <cmath>
+#include <mutex>
 #include <vector>
 
 #include "common.cuh"
@@ -29,7 +32,13 @@ namespace unisvq {
 namespace {
 
 constexpr int kRThreads = 256;
-constexpr int kMaxPaley = 28;
+constexpr int kMaxPaley = 28;     // largest order whose column masks fit one word
+constexpr int kP344 = 344;        // 7^3 + 1
+constexpr int kP344Words = 12;    // words per column mask of H_344 (11 used)
+
+// Column c of H_344 at words [12 c, 12 c + 11): bit q % 32 of word q / 32 set
+// where H_344[q][c] = -1. Written once per device from the host.
+__device__ __align__(16) uint32_t g_h344_neg[kP344 * kP344Words];
 
 struct RhtArgs {
   const uint16_t* in;       // bf16 [M][in_stride]
@@ -40,7 +49,8 @@ struct RhtArgs {
   int in_stride, out_stride;
   int signs_first;          // 1: x -> (s x) H; 0: x -> (x H) s
   float scale;              // 1 / sqrt(n)
-  uint32_t hm_neg[kMaxPaley];   // bit q of column q': H_m[q][q'] = -1
+  uint32_t hm_neg[kMaxPaley];   // bit q of column q': H_m[q][q'] = -1 (m <= 28)
+  const uint32_t* h344_neg;     // g_h344_neg of this device (m = 344)
 };
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float(static_cast<uint32_t>(b) << 16); }
@@ -64,6 +74,37 @@ __device__ __forceinline__ void paley_blocks(const float* src, float* dst, int n
       for (int q = 0; q < M_; ++q) acc += ((mask >> q) & 1u) ? -v[q] : v[q];
       dst[p * M_ + c0 + c] = acc;
     }
+  }
+}
+
+__device__ __forceinline__ float neg_if_bit(float v, uint32_t w, int b) {
+  return __uint_as_float(__float_as_uint(v) ^ ((w << (31 - b)) & 0x80000000u));
+}
+
+// Row vector times H_344 for every block of 344 consecutive entries of src,
+// into dst: one thread per output entry (block p, column c) with its column's
+// sign bits in registers; the block is read as 86 float4 from shared memory
+// (lanes working on one block read the same addresses: broadcasts). Two
+// accumulation chains per entry.
+__device__ __forceinline__ void paley344_blocks(const float* src, float* dst, int nblk, const uint32_t* neg) {
+  for (int it = threadIdx.x; it < nblk * kP344; it += kRThreads) {
+    const int p = it / kP344, c = it - p * kP344;
+    const uint4* col = reinterpret_cast<const uint4*>(neg + c * kP344Words);
+    const uint4 u0 = __ldg(col), u1 = __ldg(col + 1), u2 = __ldg(col + 2);
+    const uint32_t w[kP344Words] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w, u2.x, u2.y, u2.z, u2.w};
+    const float4* blk = reinterpret_cast<const float4*>(src + p * kP344);
+    float acc0 = 0.f, acc1 = 0.f;
+#pragma unroll
+    for (int q4 = 0; q4 < kP344 / 4; ++q4) {
+      const float4 v = blk[q4];
+      const uint32_t ww = w[q4 >> 3];   // entries 4 q4 .. 4 q4 + 3 sit in word q4 / 8
+      const int b = (q4 & 7) * 4;
+      acc0 += neg_if_bit(v.x, ww, b);
+      acc1 += neg_if_bit(v.y, ww, b + 1);
+      acc0 += neg_if_bit(v.z, ww, b + 2);
+      acc1 += neg_if_bit(v.w, ww, b + 3);
+    }
+    dst[it] = acc0 + acc1;
   }
 }
 
@@ -157,7 +198,8 @@ __global__ void __launch_bounds__(kRThreads) rht_kernel(const __grid_constant__ 
     float* out2 = smem_f + chunk;
     if (a.m == 12) paley_blocks<12>(buf, out2, pl, a.hm_neg);
     else if (a.m == 20) paley_blocks<20>(buf, out2, pl, a.hm_neg);
-    else paley_blocks<28>(buf, out2, pl, a.hm_neg);
+    else if (a.m == 28) paley_blocks<28>(buf, out2, pl, a.hm_neg);
+    else paley344_blocks(buf, out2, pl, a.h344_neg);
     buf = out2;
     __syncthreads();
   }
@@ -243,12 +285,91 @@ std::vector<int> paley_signs(int m) {
   return H;
 }
 
+// The field of 343 elements as GF(7)[t] / (t^3 - 2). t^3 - 2 has no root mod 7
+// (the cubes mod 7 are 0, 1 and 6), so it is irreducible and the quotient is
+// a field. Element e = e0 + 7 e1 + 49 e2 stands for e0 + e1 t + e2 t^2.
+int f343_mul(int x, int y) {
+  const int a[3] = {x % 7, x / 7 % 7, x / 49}, b[3] = {y % 7, y / 7 % 7, y / 49};
+  int p[5] = {0, 0, 0, 0, 0};
+  for (int i = 0; i < 3; ++i)
+    for (int j = 0; j < 3; ++j) p[i + j] += a[i] * b[j];
+  // t^3 = 2 and t^4 = 2 t
+  return (p[0] + 2 * p[3]) % 7 + 7 * ((p[1] + 2 * p[4]) % 7) + 49 * (p[2] % 7);
+}
+
+int f343_sub(int x, int y) {
+  int r = 0, w = 1;
+  for (int i = 0; i < 3; ++i, x /= 7, y /= 7, w *= 7) r += ((x % 7 - y % 7 + 7) % 7) * w;
+  return r;
+}
+
+// Quadratic character by Euler's criterion: e^((343 - 1) / 2) is 1 on the
+// nonzero squares and -1 (element 6) on the other nonzero elements.
+int f343_chi(int e) {
+  if (e == 0) return 0;
+  int r = 1, b = e;
+  for (int k = 171; k; k >>= 1) {
+    if (k & 1) r = f343_mul(r, b);
+    b = f343_mul(b, b);
+  }
+  return r == 1 ? 1 : -1;
+}
+
+// Column masks of the Paley I matrix of order 344: H = I + [[0, 1^T], [-1, Q]],
+// Q[i][j] = chi(e_j - e_i) (row and column 0 the point at infinity, row i >= 1
+// the field element i - 1).
+std::vector<uint32_t> h344_column_masks() {
+  std::vector<int> chi(343);
+  for (int e = 0; e < 343; ++e) chi[e] = f343_chi(e);
+  std::vector<uint32_t> masks(static_cast<size_t>(kP344) * kP344Words, 0u);
+  for (int c = 0; c < kP344; ++c)
+    for (int q = 0; q < kP344; ++q) {
+      int h;
+      if (q == c) h = 1;
+      else if (q == 0) h = 1;
+      else if (c == 0) h = -1;
+      else h = chi[f343_sub(c - 1, q - 1)];
+      if (h < 0) masks[static_cast<size_t>(c) * kP344Words + q / 32] |= 1u << (q % 32);
+    }
+  return masks;
+}
+
+std::atomic<const uint32_t*> g_h344_addr[64];
+std::mutex g_h344_mu;
+
+// Device address of g_h344_neg on device `dev`, written from the host on the
+// first request (a synchronous copy, so it must not run under stream capture).
+const uint32_t* h344_table(int dev) {
+  const uint32_t* t = g_h344_addr[dev].load(std::memory_order_acquire);
+  if (t) return t;
+  std::lock_guard<std::mutex> lk(g_h344_mu);
+  t = g_h344_addr[dev].load(std::memory_order_acquire);
+  if (t) return t;
+  static const std::vector<uint32_t> host = h344_column_masks();
+  void* addr = nullptr;
+  if (cudaMemcpyToSymbol(g_h344_neg, host.data(), host.size() * sizeof(uint32_t)) != cudaSuccess ||
+      cudaGetSymbolAddress(&addr, g_h344_neg) != cudaSuccess)
+    return nullptr;
+  t = static_cast<const uint32_t*>(addr);
+  g_h344_addr[dev].store(t, std::memory_order_release);
+  return t;
+}
+
 }  // namespace
+
+unisvq_status rht_prepare(int n) {
+  int p2 = 0, m = 0;
+  if (!rht_factor(n, &p2, &m)) return UNISVQ_ERR_UNSUPPORTED;
+  if (m != kP344) return UNISVQ_OK;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
+  return h344_table(dev) ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+}
 
 bool rht_factor(int n, int* p2, int* m) {
   if (n <= 0) return false;
-  const int ms[4] = {28, 20, 12, 1};
-  for (int k = 0; k < 4; ++k) {
+  const int ms[5] = {kP344, 28, 20, 12, 1};
+  for (int k = 0; k < 5; ++k) {
     if (n % ms[k]) continue;
     const int p = n / ms[k];
     if ((p & (p - 1)) == 0) {
@@ -265,12 +386,17 @@ bool rht_factor(int n, int* p2, int* m) {
 // CTAs per row: 16 (a non-portable cluster) for rows of 16384 values or more,
 // else min(8, 2^a). Measured on GB300 at n = 28672: 6.8 us against 9.0 us with
 // 8 CTAs; at n = 14336 eight CTAs are faster.
-static int rht_ctas(int n, int p2) { return (n >= 16384 && p2 >= 16) ? 16 : (p2 >= 8 ? 8 : p2); }
+// For m = 344 (11008 = 32 * 344), 16 CTAs hold two blocks each: the dense
+// block product is most of the work there.
+static int rht_ctas(int n, int p2, int m) {
+  if ((n >= 16384 || m == kP344) && p2 >= 16) return 16;
+  return p2 >= 8 ? 8 : p2;
+}
 
 size_t rht_smem_bytes(int n) {
   int p2 = 0, m = 0;
   if (!rht_factor(n, &p2, &m)) return static_cast<size_t>(n) * sizeof(float);
-  return static_cast<size_t>(n / rht_ctas(n, p2)) * sizeof(float) * (m > 1 ? 2 : 1);
+  return static_cast<size_t>(n / rht_ctas(n, p2, m)) * sizeof(float) * (m > 1 ? 2 : 1);
 }
 
 unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_stride, int M, int n,
@@ -295,12 +421,15 @@ unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_strid
   a.n = n;
   a.p2 = p2;
   a.m = m;
-  a.G = rht_ctas(n, p2);
+  a.G = rht_ctas(n, p2, m);
   a.in_stride = in_stride;
   a.out_stride = out_stride;
   a.signs_first = signs_first;
   a.scale = static_cast<float>(1.0 / std::sqrt(static_cast<double>(n)));
-  if (m > 1) {
+  if (m == kP344) {
+    a.h344_neg = h344_table(dev);
+    if (!a.h344_neg) return UNISVQ_ERR_CUDA;
+  } else if (m > 1) {
     const std::vector<int> H = paley_signs(m);
     for (int c = 0; c < m; ++c) {
       uint32_t mask = 0;

@@ -556,6 +556,10 @@ unisvq_status unisvq_set_rht(unisvq_handle h, const uint8_t* sign_in, const uint
   int p2 = 0, m = 0;
   if (!rht_factor(h->K, &p2, &m) || !rht_factor(h->N, &p2, &m)) return UNISVQ_ERR_UNSUPPORTED;
   if (rht_smem_bytes(h->K) > 227 * 1024 || rht_smem_bytes(h->N) > 227 * 1024) return UNISVQ_ERR_UNSUPPORTED;
+  for (const int n : {h->K, h->N}) {
+    const unisvq_status st = rht_prepare(n);
+    if (st != UNISVQ_OK) return st;
+  }
   std::vector<uint8_t> signs(static_cast<size_t>(h->K) + h->N);
   std::memcpy(signs.data(), sign_in, h->K);
   std::memcpy(signs.data() + h->K, sign_out, h->N);
@@ -589,6 +593,8 @@ unisvq_status unisvq_hadamard(const void* x, void* y, int M, int n, const uint8_
   if (x != y && overlaps(x, bytes, y, bytes)) return UNISVQ_ERR_INVALID_ARG;
   int p2 = 0, m = 0;
   if (!rht_factor(n, &p2, &m)) return UNISVQ_ERR_UNSUPPORTED;
+  const unisvq_status st = rht_prepare(n);
+  if (st != UNISVQ_OK) return st;
   return launch_rht(x, n, y, n, M, n, signs, signs_first, static_cast<cudaStream_t>(stream));
 }
 

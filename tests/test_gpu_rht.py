@@ -1,6 +1,7 @@
 """The randomized Hadamard transform (Eq. def:hadamard) on the GPU against the
-fp64 oracle: the rotation alone (every supported order family, both sign
-placements, in place and out of place), and the layer with the inverse
+fp64 oracle: the rotation alone (every supported order family, including
+the order-344 Paley factor of 11008 = 2^5 * 344, both sign placements, in
+place and out of place), and the layer with the inverse
 rotation around it (per-matrix and per-group layers, chunked token counts,
 forced kernels, grouped calls)."""
 import numpy as np
@@ -30,7 +31,7 @@ def signs(n, seed):
     return np.random.default_rng(seed).choice([-1.0, 1.0], size=n)
 
 
-@pytest.mark.parametrize("n", [12, 20, 28, 64, 96, 448, 4096, 5120, 14336, 28672])
+@pytest.mark.parametrize("n", [12, 20, 28, 64, 96, 344, 448, 688, 4096, 5120, 5504, 11008, 14336, 28672])
 @pytest.mark.parametrize("signs_first", [1, 0])
 def test_rotation_matches_oracle(n, signs_first):
     M = 3
@@ -65,14 +66,15 @@ def test_rotation_without_signs_and_bad_orders():
     assert binding.sync_status() == binding.OK
     ref = oracle.bf16_bits_to_f64(xb) @ (oracle.hadamard(n) / 16.0)
     assert np.allclose(host(y), ref, rtol=2.0 ** -8, atol=1e-5)
-    for bad in (11008, 36, 100):
+    for bad in (36, 100, 172, 6880):
         xb2 = torch.zeros((1, bad), dtype=torch.bfloat16, device="cuda")
         yb2 = torch.zeros((1, bad), dtype=torch.bfloat16, device="cuda")
         assert binding.hadamard_ptr(xb2.data_ptr(), yb2.data_ptr(), 1, bad, 0, 1, stream) == binding.ERR_UNSUPPORTED
     assert binding.hadamard_ptr(x.data_ptr(), y.data_ptr(), 1, n, 0, 2, stream) == binding.ERR_INVALID_ARG
 
 
-@pytest.mark.parametrize("N,K,d", [(4096, 4096, 2), (1792, 3584, 2), (640, 1280, 4), (768, 2560, 1)])
+@pytest.mark.parametrize("N,K,d", [(4096, 4096, 2), (1792, 3584, 2), (640, 1280, 4), (768, 2560, 1),
+                                   (11008, 4096, 2), (4096, 11008, 2)])
 def test_layer_with_inverse_rht(N, K, d):
     codes, A, B = synth.layer_inputs(7, 52, N, K, N, K, d)
     layer = binding.UniSVQLinear(codes, A, B)
@@ -128,7 +130,7 @@ def test_grouped_layer_and_group_call_with_rht():
 
 
 def test_set_rht_rejects_unsupported_widths_and_bad_signs():
-    N, K = 11008, 4096
+    N, K = 4608, 4096      # 4608 = 2^9 * 9: no Hadamard order here
     codes = np.zeros((N, K), dtype=np.uint8)
     layer = binding.UniSVQLinear(codes, np.eye(2, dtype=np.float16), np.zeros(2, dtype=np.float16))
     with pytest.raises(binding.UnisvqError) as e:
