@@ -136,8 +136,10 @@ unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s);
 bool rht_factor(int n, int* p2, int* m);
 unisvq_status rht_prepare(int n);
 size_t rht_smem_bytes(int n);
+// signs_const: the sign bytes never change between launches (a handle's own
+// buffer), so the kernel reads them before waiting for the previous kernel.
 unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_stride, int M, int n,
-                         const uint8_t* signs, int signs_first, cudaStream_t s);
+                         const uint8_t* signs, int signs_first, bool signs_const, cudaStream_t s);
 
 // Per-(row, group) affine layers (gemv_grouped.cu): every M, at most 32 / d
 // tokens per launch; all layers of one call must be grouped with the same d.

@@ -33,12 +33,22 @@ namespace {
 
 constexpr int kRThreads = 256;
 constexpr int kMaxPaley = 28;     // largest order whose column masks fit one word
-constexpr int kP344 = 344;        // 7^3 + 1
-constexpr int kP344Words = 12;    // words per column mask of H_344 (11 used)
+constexpr int kP344 = 344;                        // 7^3 + 1
+constexpr int kP344Steps = (kP344 + 15) / 16;     // 22 steps of 16 (mma M over columns, mma K over rows)
+constexpr int kP344Blocks = 8;                    // blocks per mma column tile (mma N)
+constexpr int kP344Words = 6;                     // 22 steps x 8 bits per lane
+constexpr int kP344TilesPerWarp = (kP344Steps + kRThreads / 32 - 1) / (kRThreads / 32);   // 3
 
-// Column c of H_344 at words [12 c, 12 c + 11): bit q % 32 of word q / 32 set
-// where H_344[q][c] = -1. Written once per device from the host.
-__device__ __align__(16) uint32_t g_h344_neg[kP344 * kP344Words];
+// Sign bits of H_344 in the A-fragment order of mma.m16n8k16 with
+// A[c][q] = H_344[q][c] (the transpose): for column tile mt and lane l
+// (c0 = 16 mt + l / 4, c1 = c0 + 8, t = l % 4), bits 8 ks .. 8 ks + 7 of the
+// 176-bit string at words [6 (32 mt + l), 6 (32 mt + l) + 6) are set where
+// H_344[q][c] = -1 for (q, c) = (16 ks + 2t, c0), (16 ks + 2t + 1, c0),
+// (16 ks + 2t, c1), (16 ks + 2t + 1, c1), then the same four with q + 8:
+// A registers a0 .. a3 in that order, two bits each. Entries with q or c
+// past 343 are +1 (they meet zero activations or produce discarded outputs).
+// Written once per device from the host.
+__device__ __align__(16) uint32_t g_h344_bits[kP344Steps * 32 * kP344Words];
 
 struct RhtArgs {
   const uint16_t* in;       // bf16 [M][in_stride]
@@ -49,8 +59,9 @@ struct RhtArgs {
   int in_stride, out_stride;
   int signs_first;          // 1: x -> (s x) H; 0: x -> (x H) s
   float scale;              // 1 / sqrt(n)
+  int sign_off;                 // byte offset of the staged sign bytes in shared memory
   uint32_t hm_neg[kMaxPaley];   // bit q of column q': H_m[q][q'] = -1 (m <= 28)
-  const uint32_t* h344_neg;     // g_h344_neg of this device (m = 344)
+  const uint32_t* h344_bits;    // g_h344_bits of this device (m = 344)
 };
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float(static_cast<uint32_t>(b) << 16); }
@@ -77,34 +88,76 @@ __device__ __forceinline__ void paley_blocks(const float* src, float* dst, int n
   }
 }
 
-__device__ __forceinline__ float neg_if_bit(float v, uint32_t w, int b) {
-  return __uint_as_float(__float_as_uint(v) ^ ((w << (31 - b)) & 0x80000000u));
+// Row vector times H_344 for every block of 344 consecutive entries, on the
+// tensor cores as D^T = H_344^T X^T: D^T[c][b] = sum_q H_344[q][c] X[b][q]
+// with mma.sync m16n8k16 (bf16 operands, fp32 accumulation). M runs over the
+// 344 output columns (22 tiles of 16), N over 8 blocks, K over the 344
+// positions (22 steps). The B operand is the blocks in bf16 (the rotation's
+// input values, exact in bf16, so every product is exact), loaded by
+// ldmatrix; blocks past nblk and positions past 343 read a zeroed 16-byte
+// line. The A operand is +-1 in bf16, made per lane from 8 sign bits through
+// a 16-entry table (lut: the two A registers for each 4-bit pattern). Warp w
+// computes column tiles w, w + 8, w + 16 as independent accumulator chains.
+// This lane's sign bits of its warp's column tiles (read before the
+// programmatic-launch wait: the table never depends on the previous kernel).
+__device__ __forceinline__ void load_h344_bits(const uint32_t* bits, uint32_t (&w)[kP344TilesPerWarp][kP344Words]) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll
+  for (int i = 0; i < kP344TilesPerWarp; ++i) {
+    const int mt = warp + i * (kRThreads / 32);
+#pragma unroll
+    for (int k = 0; k < kP344Words; ++k)
+      w[i][k] = mt < kP344Steps ? __ldg(bits + (mt * 32 + lane) * kP344Words + k) : 0u;
+  }
 }
 
-// Row vector times H_344 for every block of 344 consecutive entries of src,
-// into dst: one thread per output entry (block p, column c) with its column's
-// sign bits in registers; the block is read as 86 float4 from shared memory
-// (lanes working on one block read the same addresses: broadcasts). Two
-// accumulation chains per entry.
-__device__ __forceinline__ void paley344_blocks(const float* src, float* dst, int nblk, const uint32_t* neg) {
-  for (int it = threadIdx.x; it < nblk * kP344; it += kRThreads) {
-    const int p = it / kP344, c = it - p * kP344;
-    const uint4* col = reinterpret_cast<const uint4*>(neg + c * kP344Words);
-    const uint4 u0 = __ldg(col), u1 = __ldg(col + 1), u2 = __ldg(col + 2);
-    const uint32_t w[kP344Words] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w, u2.x, u2.y, u2.z, u2.w};
-    const float4* blk = reinterpret_cast<const float4*>(src + p * kP344);
-    float acc0 = 0.f, acc1 = 0.f;
+__device__ __forceinline__ void paley344_mma(const uint16_t* x_bf16, float* dst, int nblk,
+                                             const uint32_t (&w)[kP344TilesPerWarp][kP344Words], const uint2* lut,
+                                             const uint16_t* zero16) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+  const uint32_t x_base = smem_u32(x_bf16), z_addr = smem_u32(zero16);
+  // ldmatrix.x2 row addresses: lanes 0..7 the 8 blocks at k 0..7 of the
+  // step, lanes 8..15 the same blocks at k 8..15 (lanes 16..31 unused)
+  const int bsel = lane & 7, bkoff = ((lane >> 3) & 1) * 8;
+  for (int nb = 0; nb < nblk; nb += kP344Blocks) {
+    const int b = nb + bsel;
+    const bool blk_ok = b < nblk;
+    const uint32_t row_addr = x_base + static_cast<uint32_t>(b * kP344 + bkoff) * 2u;
+    float acc[kP344TilesPerWarp][4] = {};
 #pragma unroll
-    for (int q4 = 0; q4 < kP344 / 4; ++q4) {
-      const float4 v = blk[q4];
-      const uint32_t ww = w[q4 >> 3];   // entries 4 q4 .. 4 q4 + 3 sit in word q4 / 8
-      const int b = (q4 & 7) * 4;
-      acc0 += neg_if_bit(v.x, ww, b);
-      acc1 += neg_if_bit(v.y, ww, b + 1);
-      acc0 += neg_if_bit(v.z, ww, b + 2);
-      acc1 += neg_if_bit(v.w, ww, b + 3);
+    for (int ks = 0; ks < kP344Steps; ++ks) {
+      // the last step's second 8 positions (q = 344 .. 351) are zeros
+      const bool ok = blk_ok && (16 * ks + bkoff < kP344);
+      const uint32_t addr = ok ? row_addr + 32u * ks : z_addr;
+      uint32_t b0, b1;
+      asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];" : "=r"(b0), "=r"(b1) : "r"(addr));
+#pragma unroll
+      for (int i = 0; i < kP344TilesPerWarp; ++i) {
+        if (warp + i * (kRThreads / 32) < kP344Steps) {
+          const uint32_t byte = (w[i][(8 * ks) >> 5] >> ((8 * ks) & 31)) & 0xffu;
+          const uint2 lo = lut[byte & 15u], hi = lut[byte >> 4];
+          asm volatile(
+              "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+              "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+              : "+f"(acc[i][0]), "+f"(acc[i][1]), "+f"(acc[i][2]), "+f"(acc[i][3])
+              : "r"(lo.x), "r"(lo.y), "r"(hi.x), "r"(hi.y), "r"(b0), "r"(b1));
+        }
+      }
     }
-    dst[it] = acc0 + acc1;
+    // D^T fragment: rows c = 16 mt + g (+ 8), columns blocks nb + 2t, + 1
+#pragma unroll
+    for (int i = 0; i < kP344TilesPerWarp; ++i) {
+      const int mt = warp + i * (kRThreads / 32);
+      if (mt >= kP344Steps) continue;
+      const int c = 16 * mt + g, b0 = nb + 2 * t;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int cc = c + 8 * h;
+        if (cc >= kP344) continue;
+        if (b0 < nblk) dst[b0 * kP344 + cc] = acc[i][2 * h];
+        if (b0 + 1 < nblk) dst[(b0 + 1) * kP344 + cc] = acc[i][2 * h + 1];
+      }
+    }
   }
 }
 
@@ -138,8 +191,9 @@ __device__ __forceinline__ void sylvester_pass(float* buf, int p2, int m, int s0
 }
 
 // G-point Sylvester transform of position e of the chunk across the cluster.
-template <int G>
-__device__ __forceinline__ void cross_chunk(const RhtArgs& a, const float* buf, uint16_t* dst, int chunk, int e) {
+template <int G, bool kStaged>
+__device__ __forceinline__ void cross_chunk(const RhtArgs& a, const float* buf, uint16_t* dst, int chunk, int e,
+                                            const uint8_t* osg, int sgi) {
   float v[G];
   const uint32_t local = smem_u32(buf + e);
 #pragma unroll
@@ -157,12 +211,54 @@ __device__ __forceinline__ void cross_chunk(const RhtArgs& a, const float* buf, 
   for (int r = 0; r < G; ++r) {
     const int i = r * chunk + e;
     float o = v[r] * a.scale;
-    if (!a.signs_first && a.signs && a.signs[i]) o = -o;
+    if constexpr (kStaged) {
+      if (osg && osg[sgi + r * ((chunk + G - 1) / G)]) o = -o;
+    } else {
+      if (!a.signs_first && a.signs && a.signs[i]) o = -o;
+    }
     dst[i] = f32_to_bf16_rn(o);
   }
 }
 
-__global__ void __launch_bounds__(kRThreads) rht_kernel(const __grid_constant__ RhtArgs a) {
+// The sign bytes a CTA applies, into shared memory (sg): on the way in those
+// of its chunk, on the way out those of the positions it writes (its chunk
+// when G == 1, else G segments of span positions, segment r at
+// r * chunk + rank * span). Loads are issued eight per thread before their
+// stores, so the copy costs about one memory latency.
+__device__ __forceinline__ void stage_signs(const RhtArgs& a, uint8_t* sg, int nsg, int base, int chunk, int span,
+                                            int rank) {
+  for (int i0 = threadIdx.x; i0 < nsg; i0 += kRThreads * 8) {
+    uint8_t v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int i = i0 + k * kRThreads;
+      int pos = -1;
+      if (i < nsg) {
+        if (a.signs_first) {
+          pos = base + i;
+        } else if (a.G == 1) {
+          pos = i;
+        } else {
+          const int r = i / span, e = rank * span + (i - r * span);
+          pos = e < chunk ? r * chunk + e : -1;
+        }
+      }
+      v[k] = pos >= 0 ? a.signs[pos] : 0;
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (i0 + k * kRThreads < nsg) sg[i0 + k * kRThreads] = v[k];
+  }
+}
+
+// kP344Path: the instance for m = 344 (tensor-core block product; its
+// registers do not limit the residency of the others). kStaged: the sign
+// bytes never change between launches (a handle's own), so they are copied to
+// shared memory before the dependency wait; otherwise (the standalone
+// rotation's signs, which the previous kernel may write) they are read from
+// global memory where they are applied.
+template <bool kP344Path, bool kStaged>
+__global__ void __launch_bounds__(kRThreads, kP344Path ? 1 : 3) rht_kernel(const __grid_constant__ RhtArgs a) {
   extern __shared__ __align__(16) float smem_f[];
   float* buf = smem_f;   // the chunk; a second chunk-sized buffer follows when m > 1
   const int G = a.G;
@@ -171,37 +267,88 @@ __global__ void __launch_bounds__(kRThreads) rht_kernel(const __grid_constant__ 
   const int pl = a.p2 / G;             // m-blocks per CTA
   const int chunk = pl * a.m;          // values per CTA
   const int base = rank * chunk;
+  const int span = (chunk + G - 1) / G;   // positions per CTA in the cross-chunk stage
+  uint8_t* sg = reinterpret_cast<uint8_t*>(smem_f) + a.sign_off;
+  const int nsg = !a.signs ? 0 : (a.signs_first || G == 1 ? chunk : G * span);
   pdl_launch_dependents();
+  uint32_t h344w[kP344Path ? kP344TilesPerWarp : 1][kP344Words];
+  if constexpr (kP344Path) load_h344_bits(a.h344_bits, h344w);
+  if constexpr (kStaged) stage_signs(a, sg, nsg, base, chunk, span, rank);
   pdl_wait();   // the row may be the previous kernel's output
+  if constexpr (kStaged) __syncthreads();
+  // input sign byte i of the chunk
+  const uint8_t* sg_in = kStaged ? sg : a.signs + base;
   const uint16_t* src = a.in + static_cast<size_t>(row) * a.in_stride + base;
   const bool sgn_in = a.signs_first && a.signs;
-  if ((chunk & 7) == 0 && (a.in_stride & 7) == 0) {   // 16-byte loads of 8 values
+  // 16-byte loads where every row's chunk starts on a 16-byte boundary
+  const bool vec_ok = (reinterpret_cast<uintptr_t>(a.in) & 15) == 0 && (a.in_stride & 7) == 0;
+  if constexpr (kP344Path) {
+    // bf16 operand copy of the chunk (signs applied: a bf16 sign flip is
+    // exact), the zeroed line and the B-register table; the fp32 region at
+    // the start of shared memory receives the block products.
+    uint16_t* ab = reinterpret_cast<uint16_t*>(smem_f + chunk);
+    uint16_t* zero16 = ab + chunk;
+    uint2* lut = reinterpret_cast<uint2*>(zero16 + 8);
+    if (threadIdx.x < 16) {
+      const uint32_t nib = threadIdx.x;
+      lut[nib] = make_uint2(0x3f803f80u | ((nib & 1u) << 15) | ((nib & 2u) << 30),
+                            0x3f803f80u | ((nib & 4u) << 13) | ((nib & 8u) << 28));
+    } else if (threadIdx.x == 16) {
+      *reinterpret_cast<uint4*>(zero16) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    if (vec_ok) {   // chunk is a multiple of 344, so of 8
+      for (int i8 = threadIdx.x; i8 < chunk / 8; i8 += kRThreads) {
+        uint4 w = ldg_v4(src + 8 * i8);
+        if (sgn_in) {
+          uint32_t f[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            if (sg_in[8 * i8 + k]) f[k >> 1] |= (k & 1) ? 0x80000000u : 0x8000u;
+          w.x ^= f[0];
+          w.y ^= f[1];
+          w.z ^= f[2];
+          w.w ^= f[3];
+        }
+        *reinterpret_cast<uint4*>(ab + 8 * i8) = w;
+      }
+    } else {
+      for (int i = threadIdx.x; i < chunk; i += kRThreads) {
+        uint16_t v = src[i];
+        if (sgn_in && sg_in[i]) v ^= 0x8000u;
+        ab[i] = v;
+      }
+    }
+    __syncthreads();
+    paley344_mma(ab, buf, pl, h344w, lut, zero16);
+    __syncthreads();
+  } else if ((chunk & 7) == 0 && vec_ok) {   // 16-byte loads of 8 values
     for (int i8 = threadIdx.x; i8 < chunk / 8; i8 += kRThreads) {
       const uint4 w = ldg_v4(src + 8 * i8);
       const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
         float v = (k & 1) ? bf16_hi(ws[k >> 1]) : bf16_lo(ws[k >> 1]);
-        if (sgn_in && a.signs[base + 8 * i8 + k]) v = -v;
+        if (sgn_in && sg_in[8 * i8 + k]) v = -v;
         buf[8 * i8 + k] = v;
       }
     }
   } else {
     for (int i = threadIdx.x; i < chunk; i += kRThreads) {
       float v = bf16_to_f32(src[i]);
-      if (sgn_in && a.signs[base + i]) v = -v;
+      if (sgn_in && sg_in[i]) v = -v;
       buf[i] = v;
     }
   }
-  __syncthreads();
-  if (a.m > 1) {
-    float* out2 = smem_f + chunk;
-    if (a.m == 12) paley_blocks<12>(buf, out2, pl, a.hm_neg);
-    else if (a.m == 20) paley_blocks<20>(buf, out2, pl, a.hm_neg);
-    else if (a.m == 28) paley_blocks<28>(buf, out2, pl, a.hm_neg);
-    else paley344_blocks(buf, out2, pl, a.h344_neg);
-    buf = out2;
+  if constexpr (!kP344Path) {
     __syncthreads();
+    if (a.m > 1) {
+      float* out2 = smem_f + chunk;
+      if (a.m == 12) paley_blocks<12>(buf, out2, pl, a.hm_neg);
+      else if (a.m == 20) paley_blocks<20>(buf, out2, pl, a.hm_neg);
+      else paley_blocks<28>(buf, out2, pl, a.hm_neg);
+      buf = out2;
+      __syncthreads();
+    }
   }
   int lg = 0;
   while ((1 << lg) < pl) ++lg;
@@ -215,22 +362,26 @@ __global__ void __launch_bounds__(kRThreads) rht_kernel(const __grid_constant__ 
   }
   uint16_t* dst = a.out + static_cast<size_t>(row) * a.out_stride;
   if (G == 1) {
+    const bool sgn_out = !a.signs_first && a.signs;
     for (int i = threadIdx.x; i < chunk; i += kRThreads) {
       float v = buf[i] * a.scale;
-      if (!a.signs_first && a.signs && a.signs[i]) v = -v;
+      if (sgn_out && (kStaged ? sg[i] : a.signs[i])) v = -v;
       dst[i] = f32_to_bf16_rn(v);
     }
     return;
   }
   cluster_sync();   // every chunk is transformed locally
-  // CTA `rank` finishes positions [rank span, (rank + 1) span) of all G chunks
-  const int span = (chunk + G - 1) / G;
+  // CTA `rank` finishes positions [rank span, (rank + 1) span) of all G
+  // chunks; the output signs of position e of chunk r are staged at
+  // sg[r span + e - rank span]
+  const uint8_t* osg = !a.signs_first && a.signs ? sg : nullptr;
   const int e1 = min(chunk, (rank + 1) * span);
   for (int e = rank * span + static_cast<int>(threadIdx.x); e < e1; e += kRThreads) {
-    if (G == 16) cross_chunk<16>(a, buf, dst, chunk, e);
-    else if (G == 8) cross_chunk<8>(a, buf, dst, chunk, e);
-    else if (G == 4) cross_chunk<4>(a, buf, dst, chunk, e);
-    else cross_chunk<2>(a, buf, dst, chunk, e);
+    const int sgi = e - rank * span;
+    if (G == 16) cross_chunk<16, kStaged>(a, buf, dst, chunk, e, osg, sgi);
+    else if (G == 8) cross_chunk<8, kStaged>(a, buf, dst, chunk, e, osg, sgi);
+    else if (G == 4) cross_chunk<4, kStaged>(a, buf, dst, chunk, e, osg, sgi);
+    else cross_chunk<2, kStaged>(a, buf, dst, chunk, e, osg, sgi);
   }
   cluster_sync();   // no CTA leaves while another still reads its shared memory
 }
@@ -315,29 +466,41 @@ int f343_chi(int e) {
   return r == 1 ? 1 : -1;
 }
 
-// Column masks of the Paley I matrix of order 344: H = I + [[0, 1^T], [-1, Q]],
-// Q[i][j] = chi(e_j - e_i) (row and column 0 the point at infinity, row i >= 1
-// the field element i - 1).
-std::vector<uint32_t> h344_column_masks() {
+// The Paley I matrix of order 344, H = I + [[0, 1^T], [-1, Q]] with
+// Q[i][j] = chi(e_j - e_i) (row and column 0 the point at infinity, row
+// i >= 1 the field element i - 1): true where H[r][c] = -1.
+bool h344_negative(const std::vector<int>& chi, int r, int c) {
+  if (r == c || r == 0) return false;
+  if (c == 0) return true;
+  return chi[f343_sub(c - 1, r - 1)] < 0;
+}
+
+// g_h344_bits: the sign bits of H_344 in A-fragment order (see its declaration).
+std::vector<uint32_t> h344_fragment_bits() {
   std::vector<int> chi(343);
   for (int e = 0; e < 343; ++e) chi[e] = f343_chi(e);
-  std::vector<uint32_t> masks(static_cast<size_t>(kP344) * kP344Words, 0u);
-  for (int c = 0; c < kP344; ++c)
-    for (int q = 0; q < kP344; ++q) {
-      int h;
-      if (q == c) h = 1;
-      else if (q == 0) h = 1;
-      else if (c == 0) h = -1;
-      else h = chi[f343_sub(c - 1, q - 1)];
-      if (h < 0) masks[static_cast<size_t>(c) * kP344Words + q / 32] |= 1u << (q % 32);
+  std::vector<uint32_t> bits(static_cast<size_t>(kP344Steps) * 32 * kP344Words, 0u);
+  for (int mt = 0; mt < kP344Steps; ++mt)
+    for (int l = 0; l < 32; ++l) {
+      const int c0 = 16 * mt + l / 4, t = l % 4;
+      for (int ks = 0; ks < kP344Steps; ++ks)
+        for (int e = 0; e < 8; ++e) {
+          // e: bit 0 -> q + 1, bit 1 -> column c0 + 8, bit 2 -> q + 8
+          const int q = 16 * ks + 2 * t + (e & 1) + 8 * (e >> 2);
+          const int c = c0 + 8 * ((e >> 1) & 1);
+          if (q < kP344 && c < kP344 && h344_negative(chi, q, c)) {
+            const int b = 8 * ks + e;
+            bits[static_cast<size_t>(mt * 32 + l) * kP344Words + b / 32] |= 1u << (b % 32);
+          }
+        }
     }
-  return masks;
+  return bits;
 }
 
 std::atomic<const uint32_t*> g_h344_addr[64];
 std::mutex g_h344_mu;
 
-// Device address of g_h344_neg on device `dev`, written from the host on the
+// Device address of g_h344_bits on device `dev`, written from the host on the
 // first request (a synchronous copy, so it must not run under stream capture).
 const uint32_t* h344_table(int dev) {
   const uint32_t* t = g_h344_addr[dev].load(std::memory_order_acquire);
@@ -345,10 +508,10 @@ const uint32_t* h344_table(int dev) {
   std::lock_guard<std::mutex> lk(g_h344_mu);
   t = g_h344_addr[dev].load(std::memory_order_acquire);
   if (t) return t;
-  static const std::vector<uint32_t> host = h344_column_masks();
+  static const std::vector<uint32_t> host = h344_fragment_bits();
   void* addr = nullptr;
-  if (cudaMemcpyToSymbol(g_h344_neg, host.data(), host.size() * sizeof(uint32_t)) != cudaSuccess ||
-      cudaGetSymbolAddress(&addr, g_h344_neg) != cudaSuccess)
+  if (cudaMemcpyToSymbol(g_h344_bits, host.data(), host.size() * sizeof(uint32_t)) != cudaSuccess ||
+      cudaGetSymbolAddress(&addr, g_h344_bits) != cudaSuccess)
     return nullptr;
   t = static_cast<const uint32_t*>(addr);
   g_h344_addr[dev].store(t, std::memory_order_release);
@@ -386,33 +549,50 @@ bool rht_factor(int n, int* p2, int* m) {
 // CTAs per row: 16 (a non-portable cluster) for rows of 16384 values or more,
 // else min(8, 2^a). Measured on GB300 at n = 28672: 6.8 us against 9.0 us with
 // 8 CTAs; at n = 14336 eight CTAs are faster.
-// For m = 344 (11008 = 32 * 344), 16 CTAs hold two blocks each: the dense
-// block product is most of the work there.
+// For m = 344 a CTA takes 8 blocks where there are that many (one mma column
+// tile: the block product costs the same 484 MMAs for 1 to 8 blocks), so
+// 11008 = 32 * 344 runs on 4 CTAs per row.
 static int rht_ctas(int n, int p2, int m) {
-  if ((n >= 16384 || m == kP344) && p2 >= 16) return 16;
+  if (m == kP344) return p2 <= kP344Blocks ? 1 : (p2 / kP344Blocks < 16 ? p2 / kP344Blocks : 16);
+  if (n >= 16384 && p2 >= 16) return 16;
   return p2 >= 8 ? 8 : p2;
+}
+
+// Shared memory of one CTA, in this order: the fp32 chunk (m = 1), or two
+// fp32 chunks (m in 12, 20, 28: the block product writes the second), or for
+// m = 344 the fp32 block products, the bf16 operand copy, a zeroed 16-byte
+// line and the 16-entry register table; then the staged sign bytes (at most
+// chunk + 16).
+static size_t rht_sign_offset(int n, int p2, int m) {
+  const size_t chunk = static_cast<size_t>(n / rht_ctas(n, p2, m));
+  if (m == kP344) return chunk * sizeof(float) + chunk * sizeof(uint16_t) + 16 + 16 * sizeof(uint2);
+  return chunk * sizeof(float) * (m > 1 ? 2 : 1);
 }
 
 size_t rht_smem_bytes(int n) {
   int p2 = 0, m = 0;
   if (!rht_factor(n, &p2, &m)) return static_cast<size_t>(n) * sizeof(float);
-  return static_cast<size_t>(n / rht_ctas(n, p2, m)) * sizeof(float) * (m > 1 ? 2 : 1);
+  const size_t chunk = static_cast<size_t>(n / rht_ctas(n, p2, m));
+  return rht_sign_offset(n, p2, m) + ((chunk + 16 + 15) / 16) * 16;
 }
 
 unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_stride, int M, int n,
-                         const uint8_t* signs, int signs_first, cudaStream_t s) {
+                         const uint8_t* signs, int signs_first, bool signs_const, cudaStream_t s) {
   int p2 = 0, m = 0;
   if (!rht_factor(n, &p2, &m)) return UNISVQ_ERR_UNSUPPORTED;
   if (rht_smem_bytes(n) > 227 * 1024) return UNISVQ_ERR_UNSUPPORTED;
   if (M <= 0) return UNISVQ_OK;
-  static bool attr_set[64] = {};
+  static std::atomic<bool> attr_set[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
-  if (!attr_set[dev]) {
-    if (cudaFuncSetAttribute(rht_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess ||
-        cudaFuncSetAttribute(rht_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024) != cudaSuccess)
+  if (!attr_set[dev].load(std::memory_order_acquire)) {
+    bool ok = true;
+    for (auto k : {rht_kernel<false, false>, rht_kernel<false, true>, rht_kernel<true, false>, rht_kernel<true, true>})
+      ok = ok && cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess &&
+           cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024) == cudaSuccess;
+    if (!ok)
       return UNISVQ_ERR_CUDA;
-    attr_set[dev] = true;
+    attr_set[dev].store(true, std::memory_order_release);
   }
   RhtArgs a{};
   a.in = static_cast<const uint16_t*>(in);
@@ -425,10 +605,11 @@ unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_strid
   a.in_stride = in_stride;
   a.out_stride = out_stride;
   a.signs_first = signs_first;
+  a.sign_off = static_cast<int>(rht_sign_offset(n, p2, m));
   a.scale = static_cast<float>(1.0 / std::sqrt(static_cast<double>(n)));
   if (m == kP344) {
-    a.h344_neg = h344_table(dev);
-    if (!a.h344_neg) return UNISVQ_ERR_CUDA;
+    a.h344_bits = h344_table(dev);
+    if (!a.h344_bits) return UNISVQ_ERR_CUDA;
   } else if (m > 1) {
     const std::vector<int> H = paley_signs(m);
     for (int c = 0; c < m; ++c) {
@@ -452,7 +633,10 @@ unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_strid
   attrs[1].val.clusterDim.z = 1;
   cfg.attrs = attrs;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, rht_kernel, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+  void (*kern)(RhtArgs) = m == kP344 ? (signs_const ? rht_kernel<true, true> : rht_kernel<true, false>)
+                                     : (signs_const ? rht_kernel<false, true> : rht_kernel<false, false>);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, a);
+  return e == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
 }  // namespace unisvq

@@ -502,9 +502,9 @@ static unisvq_status linear_rht(unisvq_handle h, int kernel, const void* x, void
     const int mc = M - m0 < h->rht_tokens ? M - m0 : h->rht_tokens;
     const uint16_t* xc = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * h->K;
     uint16_t* yc = static_cast<uint16_t*>(y) + static_cast<size_t>(m0) * h->N;
-    unisvq_status st = launch_rht(xc, h->K, h->rht_x, h->K, mc, h->K, s_in, 1, s);
+    unisvq_status st = launch_rht(xc, h->K, h->rht_x, h->K, mc, h->K, s_in, 1, true, s);
     if (st == UNISVQ_OK) st = linear_inner(h, kernel, h->rht_x, yc, mc, s, noalloc);
-    if (st == UNISVQ_OK) st = launch_rht(yc, h->N, yc, h->N, mc, h->N, s_out, 0, s);
+    if (st == UNISVQ_OK) st = launch_rht(yc, h->N, yc, h->N, mc, h->N, s_out, 0, true, s);
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;
@@ -595,7 +595,7 @@ unisvq_status unisvq_hadamard(const void* x, void* y, int M, int n, const uint8_
   if (!rht_factor(n, &p2, &m)) return UNISVQ_ERR_UNSUPPORTED;
   const unisvq_status st = rht_prepare(n);
   if (st != UNISVQ_OK) return st;
-  return launch_rht(x, n, y, n, M, n, signs, signs_first, static_cast<cudaStream_t>(stream));
+  return launch_rht(x, n, y, n, M, n, signs, signs_first, false, static_cast<cudaStream_t>(stream));
 }
 
 static unisvq_status group_inner(const unisvq_handle* hs, int n, int kernel, const void* x, void* const* ys, int M,
@@ -641,10 +641,10 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
     void* yc[UNISVQ_MAX_GROUP];
     for (int i = 0; i < n; ++i) yc[i] = static_cast<uint16_t*>(ys[i]) + static_cast<size_t>(m0) * hs[i]->N;
     unisvq_status st = launch_rht(static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * K, K, hs[0]->rht_x, K,
-                                  mc, K, hs[0]->rht_signs, 1, s);
+                                  mc, K, hs[0]->rht_signs, 1, true, s);
     if (st == UNISVQ_OK) st = group_inner(hs, n, kernel, hs[0]->rht_x, yc, mc, s);
     for (int i = 0; i < n && st == UNISVQ_OK; ++i)
-      st = launch_rht(yc[i], hs[i]->N, yc[i], hs[i]->N, mc, hs[i]->N, hs[i]->rht_signs + K, 0, s);
+      st = launch_rht(yc[i], hs[i]->N, yc[i], hs[i]->N, mc, hs[i]->N, hs[i]->rht_signs + K, 0, true, s);
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;

@@ -56,6 +56,26 @@ def test_rotation_matches_oracle(n, signs_first):
     assert torch.equal(z, y)
 
 
+@pytest.mark.parametrize("n", [448, 11008])
+def test_rotation_of_rows_not_16_byte_aligned(n):
+    """Rows that start 2 bytes past a 16-byte boundary take the element-wise
+    load path and give the same values as aligned rows."""
+    M = 2
+    xb = synth.activations(7, 55, n, M, n)
+    buf = torch.zeros(M * n + 8, dtype=torch.bfloat16, device="cuda")
+    x = buf[1:1 + M * n].view(M, n)
+    x.copy_(to_dev(xb))
+    s = signs(n, n + 1)
+    sd = torch.from_numpy((s < 0).astype(np.uint8)).cuda()
+    stream = torch.cuda.current_stream().cuda_stream
+    y_al = torch.empty((M, n), dtype=torch.bfloat16, device="cuda")
+    xa = to_dev(xb)
+    assert binding.hadamard_ptr(xa.data_ptr(), y_al.data_ptr(), M, n, sd.data_ptr(), 1, stream) == binding.OK
+    assert binding.hadamard_ptr(x.data_ptr(), x.data_ptr(), M, n, sd.data_ptr(), 1, stream) == binding.OK
+    assert binding.sync_status() == binding.OK
+    assert torch.equal(x, y_al)
+
+
 def test_rotation_without_signs_and_bad_orders():
     n, M = 256, 2
     xb = synth.activations(7, 51, 0, M, n)
