@@ -140,6 +140,19 @@ size_t rht_smem_bytes(int n);
 // buffer), so the kernel reads them before waiting for the previous kernel.
 unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_stride, int M, int n,
                          const uint8_t* signs, int signs_first, bool signs_const, cudaStream_t s);
+// Several row sets (e.g. the outputs of a group call), M rows each: one
+// launch when every width has the same H_m and cluster size, else one per
+// set. At most UNISVQ_MAX_GROUP sets.
+struct RhtSetDesc {
+  const void* in;
+  int in_stride;
+  void* out;
+  int out_stride;
+  int n;
+  const uint8_t* signs;
+};
+unisvq_status launch_rht_sets(const RhtSetDesc* sets, int nsets, int M, int signs_first, bool signs_const,
+                              cudaStream_t s);
 
 // Per-(row, group) affine layers (gemv_grouped.cu): every M, at most 32 / d
 // tokens per launch; all layers of one call must be grouped with the same d.

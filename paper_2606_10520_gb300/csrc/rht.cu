@@ -21,7 +21,9 @@
 // writes the scaled (and, on the way out, signed) bf16 results. A second
 // cluster barrier keeps every CTA's shared memory alive until all reads end.
 #include <atomic>
+#include <algorithm>
 #include <cmath>
+#include <cstring>
 #include <mutex>
 #include <vector>
 
@@ -50,18 +52,30 @@ constexpr int kP344TilesPerWarp = (kP344Steps + kRThreads / 32 - 1) / (kRThreads
 // Written once per device from the host.
 __device__ __align__(16) uint32_t g_h344_bits[kP344Steps * 32 * kP344Words];
 
-struct RhtArgs {
+constexpr int kMaxRowSets = UNISVQ_MAX_GROUP;
+
+// One set of rows of one width (a layer's output rows in a group call).
+struct RhtRows {
   const uint16_t* in;       // bf16 [M][in_stride]
   uint16_t* out;            // bf16 [M][out_stride] (may equal in)
   const uint8_t* signs;     // [n], 1 = negate; null = all +1
-  int n, p2, m;             // n = p2 * m
-  int G;                    // CTAs per row (cluster size), a power of 2 <= min(16, p2)
+  int p2;                   // n = p2 * m
   int in_stride, out_stride;
-  int signs_first;          // 1: x -> (s x) H; 0: x -> (x H) s
   float scale;              // 1 / sqrt(n)
-  int sign_off;                 // byte offset of the staged sign bytes in shared memory
+  int sign_off;             // byte offset of the staged sign bytes in shared memory
+  int cta_end;              // CTAs of sets 0 .. this one (M G each)
+};
+
+// A launch rotates M rows of every set; all sets share m (so H_m) and the
+// cluster size G.
+struct RhtArgs {
+  int m;                        // Paley order: 1, 12, 20, 28 or 344
+  int G;                        // CTAs per row (cluster size), a power of 2 <= min(16, p2)
+  int signs_first;              // 1: x -> (s x) H; 0: x -> (x H) s
+  int nsets;
   uint32_t hm_neg[kMaxPaley];   // bit q of column q': H_m[q][q'] = -1 (m <= 28)
   const uint32_t* h344_bits;    // g_h344_bits of this device (m = 344)
+  RhtRows set[kMaxRowSets];
 };
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float(static_cast<uint32_t>(b) << 16); }
@@ -192,8 +206,8 @@ __device__ __forceinline__ void sylvester_pass(float* buf, int p2, int m, int s0
 
 // G-point Sylvester transform of position e of the chunk across the cluster.
 template <int G, bool kStaged>
-__device__ __forceinline__ void cross_chunk(const RhtArgs& a, const float* buf, uint16_t* dst, int chunk, int e,
-                                            const uint8_t* osg, int sgi) {
+__device__ __forceinline__ void cross_chunk(const float* buf, uint16_t* dst, int chunk, int e, float scale,
+                                            const uint8_t* gsigns, const uint8_t* osg, int sgi) {
   float v[G];
   const uint32_t local = smem_u32(buf + e);
 #pragma unroll
@@ -210,11 +224,11 @@ __device__ __forceinline__ void cross_chunk(const RhtArgs& a, const float* buf, 
 #pragma unroll
   for (int r = 0; r < G; ++r) {
     const int i = r * chunk + e;
-    float o = v[r] * a.scale;
+    float o = v[r] * scale;
     if constexpr (kStaged) {
       if (osg && osg[sgi + r * ((chunk + G - 1) / G)]) o = -o;
     } else {
-      if (!a.signs_first && a.signs && a.signs[i]) o = -o;
+      if (gsigns && gsigns[i]) o = -o;
     }
     dst[i] = f32_to_bf16_rn(o);
   }
@@ -225,8 +239,8 @@ __device__ __forceinline__ void cross_chunk(const RhtArgs& a, const float* buf, 
 // when G == 1, else G segments of span positions, segment r at
 // r * chunk + rank * span). Loads are issued eight per thread before their
 // stores, so the copy costs about one memory latency.
-__device__ __forceinline__ void stage_signs(const RhtArgs& a, uint8_t* sg, int nsg, int base, int chunk, int span,
-                                            int rank) {
+__device__ __forceinline__ void stage_signs(const RhtArgs& a, const uint8_t* signs, uint8_t* sg, int nsg, int base,
+                                            int chunk, int span, int rank) {
   for (int i0 = threadIdx.x; i0 < nsg; i0 += kRThreads * 8) {
     uint8_t v[8];
 #pragma unroll
@@ -243,7 +257,7 @@ __device__ __forceinline__ void stage_signs(const RhtArgs& a, uint8_t* sg, int n
           pos = e < chunk ? r * chunk + e : -1;
         }
       }
-      v[k] = pos >= 0 ? a.signs[pos] : 0;
+      v[k] = pos >= 0 ? signs[pos] : 0;
     }
 #pragma unroll
     for (int k = 0; k < 8; ++k)
@@ -263,25 +277,45 @@ __global__ void __launch_bounds__(kRThreads, kP344Path ? 1 : 3) rht_kernel(const
   float* buf = smem_f;   // the chunk; a second chunk-sized buffer follows when m > 1
   const int G = a.G;
   const int rank = G > 1 ? static_cast<int>(cluster_ctarank()) : 0;
-  const int row = blockIdx.x / G;
-  const int pl = a.p2 / G;             // m-blocks per CTA
+  // this CTA's row set, its fields read with constant parameter offsets only
+  const uint16_t* s_in = a.set[0].in;
+  uint16_t* s_out = a.set[0].out;
+  const uint8_t* s_signs = a.set[0].signs;
+  int s_p2 = a.set[0].p2, s_in_stride = a.set[0].in_stride, s_out_stride = a.set[0].out_stride;
+  int s_sign_off = a.set[0].sign_off, cta0 = 0;
+  float s_scale = a.set[0].scale;
+#pragma unroll
+  for (int l = 1; l < kMaxRowSets; ++l)
+    if (l < a.nsets && static_cast<int>(blockIdx.x) >= a.set[l - 1].cta_end) {
+      s_in = a.set[l].in;
+      s_out = a.set[l].out;
+      s_signs = a.set[l].signs;
+      s_p2 = a.set[l].p2;
+      s_in_stride = a.set[l].in_stride;
+      s_out_stride = a.set[l].out_stride;
+      s_sign_off = a.set[l].sign_off;
+      s_scale = a.set[l].scale;
+      cta0 = a.set[l - 1].cta_end;
+    }
+  const int row = (static_cast<int>(blockIdx.x) - cta0) / G;
+  const int pl = s_p2 / G;             // m-blocks per CTA
   const int chunk = pl * a.m;          // values per CTA
   const int base = rank * chunk;
   const int span = (chunk + G - 1) / G;   // positions per CTA in the cross-chunk stage
-  uint8_t* sg = reinterpret_cast<uint8_t*>(smem_f) + a.sign_off;
-  const int nsg = !a.signs ? 0 : (a.signs_first || G == 1 ? chunk : G * span);
+  uint8_t* sg = reinterpret_cast<uint8_t*>(smem_f) + s_sign_off;
+  const int nsg = !s_signs ? 0 : (a.signs_first || G == 1 ? chunk : G * span);
   pdl_launch_dependents();
   uint32_t h344w[kP344Path ? kP344TilesPerWarp : 1][kP344Words];
   if constexpr (kP344Path) load_h344_bits(a.h344_bits, h344w);
-  if constexpr (kStaged) stage_signs(a, sg, nsg, base, chunk, span, rank);
+  if constexpr (kStaged) stage_signs(a, s_signs, sg, nsg, base, chunk, span, rank);
   pdl_wait();   // the row may be the previous kernel's output
   if constexpr (kStaged) __syncthreads();
   // input sign byte i of the chunk
-  const uint8_t* sg_in = kStaged ? sg : a.signs + base;
-  const uint16_t* src = a.in + static_cast<size_t>(row) * a.in_stride + base;
-  const bool sgn_in = a.signs_first && a.signs;
+  const uint8_t* sg_in = kStaged ? sg : s_signs + base;
+  const uint16_t* src = s_in + static_cast<size_t>(row) * s_in_stride + base;
+  const bool sgn_in = a.signs_first && s_signs;
   // 16-byte loads where every row's chunk starts on a 16-byte boundary
-  const bool vec_ok = (reinterpret_cast<uintptr_t>(a.in) & 15) == 0 && (a.in_stride & 7) == 0;
+  const bool vec_ok = (reinterpret_cast<uintptr_t>(s_in) & 15) == 0 && (s_in_stride & 7) == 0;
   if constexpr (kP344Path) {
     // bf16 operand copy of the chunk (signs applied: a bf16 sign flip is
     // exact), the zeroed line and the B-register table; the fp32 region at
@@ -360,12 +394,12 @@ __global__ void __launch_bounds__(kRThreads, kP344Path ? 1 : 3) rht_kernel(const
     s0 += r;
     __syncthreads();
   }
-  uint16_t* dst = a.out + static_cast<size_t>(row) * a.out_stride;
+  uint16_t* dst = s_out + static_cast<size_t>(row) * s_out_stride;
   if (G == 1) {
-    const bool sgn_out = !a.signs_first && a.signs;
+    const bool sgn_out = !a.signs_first && s_signs;
     for (int i = threadIdx.x; i < chunk; i += kRThreads) {
-      float v = buf[i] * a.scale;
-      if (sgn_out && (kStaged ? sg[i] : a.signs[i])) v = -v;
+      float v = buf[i] * s_scale;
+      if (sgn_out && (kStaged ? sg[i] : s_signs[i])) v = -v;
       dst[i] = f32_to_bf16_rn(v);
     }
     return;
@@ -374,14 +408,15 @@ __global__ void __launch_bounds__(kRThreads, kP344Path ? 1 : 3) rht_kernel(const
   // CTA `rank` finishes positions [rank span, (rank + 1) span) of all G
   // chunks; the output signs of position e of chunk r are staged at
   // sg[r span + e - rank span]
-  const uint8_t* osg = !a.signs_first && a.signs ? sg : nullptr;
+  const uint8_t* osg = !a.signs_first && s_signs ? sg : nullptr;
+  const uint8_t* gsg = !a.signs_first ? s_signs : nullptr;
   const int e1 = min(chunk, (rank + 1) * span);
   for (int e = rank * span + static_cast<int>(threadIdx.x); e < e1; e += kRThreads) {
     const int sgi = e - rank * span;
-    if (G == 16) cross_chunk<16, kStaged>(a, buf, dst, chunk, e, osg, sgi);
-    else if (G == 8) cross_chunk<8, kStaged>(a, buf, dst, chunk, e, osg, sgi);
-    else if (G == 4) cross_chunk<4, kStaged>(a, buf, dst, chunk, e, osg, sgi);
-    else cross_chunk<2, kStaged>(a, buf, dst, chunk, e, osg, sgi);
+    if (G == 16) cross_chunk<16, kStaged>(buf, dst, chunk, e, s_scale, gsg, osg, sgi);
+    else if (G == 8) cross_chunk<8, kStaged>(buf, dst, chunk, e, s_scale, gsg, osg, sgi);
+    else if (G == 4) cross_chunk<4, kStaged>(buf, dst, chunk, e, s_scale, gsg, osg, sgi);
+    else cross_chunk<2, kStaged>(buf, dst, chunk, e, s_scale, gsg, osg, sgi);
   }
   cluster_sync();   // no CTA leaves while another still reads its shared memory
 }
@@ -576,12 +611,45 @@ size_t rht_smem_bytes(int n) {
   return rht_sign_offset(n, p2, m) + ((chunk + 16 + 15) / 16) * 16;
 }
 
-unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_stride, int M, int n,
-                         const uint8_t* signs, int signs_first, bool signs_const, cudaStream_t s) {
-  int p2 = 0, m = 0;
-  if (!rht_factor(n, &p2, &m)) return UNISVQ_ERR_UNSUPPORTED;
-  if (rht_smem_bytes(n) > 227 * 1024) return UNISVQ_ERR_UNSUPPORTED;
+// Column sign masks of H_m for m in {12, 20, 28} (kMaxPaley words each, bit q
+// of word c set where H_m[q][c] = -1), built once.
+static const uint32_t* paley_masks(int m) {
+  static const std::vector<uint32_t> table = [] {
+    std::vector<uint32_t> t(3 * kMaxPaley, 0u);
+    const int orders[3] = {12, 20, 28};
+    for (int k = 0; k < 3; ++k) {
+      const int mm = orders[k];
+      const std::vector<int> H = paley_signs(mm);
+      for (int c = 0; c < mm; ++c)
+        for (int q = 0; q < mm; ++q)
+          if (H[static_cast<size_t>(q) * mm + c] < 0) t[k * kMaxPaley + c] |= 1u << q;
+    }
+    return t;
+  }();
+  return table.data() + (m == 12 ? 0 : (m == 20 ? 1 : 2)) * kMaxPaley;
+}
+
+unisvq_status launch_rht_sets(const RhtSetDesc* sets, int nsets, int M, int signs_first, bool signs_const,
+                              cudaStream_t s) {
+  if (nsets < 1 || nsets > kMaxRowSets) return UNISVQ_ERR_INVALID_ARG;
+  int p2[kMaxRowSets], mm[kMaxRowSets], gg[kMaxRowSets];
+  size_t smem = 0;
+  bool one_launch = true;
+  for (int i = 0; i < nsets; ++i) {
+    if (!rht_factor(sets[i].n, &p2[i], &mm[i])) return UNISVQ_ERR_UNSUPPORTED;
+    if (rht_smem_bytes(sets[i].n) > 227 * 1024) return UNISVQ_ERR_UNSUPPORTED;
+    gg[i] = rht_ctas(sets[i].n, p2[i], mm[i]);
+    smem = std::max(smem, rht_smem_bytes(sets[i].n));
+    one_launch = one_launch && mm[i] == mm[0] && gg[i] == gg[0];
+  }
   if (M <= 0) return UNISVQ_OK;
+  if (!one_launch) {   // widths with different H_m or cluster sizes: one launch per set
+    for (int i = 0; i < nsets; ++i) {
+      const unisvq_status st = launch_rht_sets(sets + i, 1, M, signs_first, signs_const, s);
+      if (st != UNISVQ_OK) return st;
+    }
+    return UNISVQ_OK;
+  }
   static std::atomic<bool> attr_set[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
@@ -590,45 +658,43 @@ unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_strid
     for (auto k : {rht_kernel<false, false>, rht_kernel<false, true>, rht_kernel<true, false>, rht_kernel<true, true>})
       ok = ok && cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess &&
            cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024) == cudaSuccess;
-    if (!ok)
-      return UNISVQ_ERR_CUDA;
+    if (!ok) return UNISVQ_ERR_CUDA;
     attr_set[dev].store(true, std::memory_order_release);
   }
+  const int m = mm[0], G = gg[0];
   RhtArgs a{};
-  a.in = static_cast<const uint16_t*>(in);
-  a.out = static_cast<uint16_t*>(out);
-  a.signs = signs;
-  a.n = n;
-  a.p2 = p2;
   a.m = m;
-  a.G = rht_ctas(n, p2, m);
-  a.in_stride = in_stride;
-  a.out_stride = out_stride;
+  a.G = G;
   a.signs_first = signs_first;
-  a.sign_off = static_cast<int>(rht_sign_offset(n, p2, m));
-  a.scale = static_cast<float>(1.0 / std::sqrt(static_cast<double>(n)));
+  a.nsets = nsets;
+  for (int i = 0; i < nsets; ++i) {
+    RhtRows& r = a.set[i];
+    r.in = static_cast<const uint16_t*>(sets[i].in);
+    r.out = static_cast<uint16_t*>(sets[i].out);
+    r.signs = sets[i].signs;
+    r.p2 = p2[i];
+    r.in_stride = sets[i].in_stride;
+    r.out_stride = sets[i].out_stride;
+    r.scale = static_cast<float>(1.0 / std::sqrt(static_cast<double>(sets[i].n)));
+    r.sign_off = static_cast<int>(rht_sign_offset(sets[i].n, p2[i], m));
+    r.cta_end = (i + 1) * M * G;
+  }
   if (m == kP344) {
     a.h344_bits = h344_table(dev);
     if (!a.h344_bits) return UNISVQ_ERR_CUDA;
   } else if (m > 1) {
-    const std::vector<int> H = paley_signs(m);
-    for (int c = 0; c < m; ++c) {
-      uint32_t mask = 0;
-      for (int q = 0; q < m; ++q)
-        if (H[static_cast<size_t>(q) * m + c] < 0) mask |= 1u << q;
-      a.hm_neg[c] = mask;
-    }
+    std::memcpy(a.hm_neg, paley_masks(m), sizeof(a.hm_neg));
   }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(M * a.G, 1, 1);
+  cfg.gridDim = dim3(nsets * M * G, 1, 1);
   cfg.blockDim = dim3(kRThreads, 1, 1);
-  cfg.dynamicSmemBytes = rht_smem_bytes(n);
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attrs[2];
   attrs[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attrs[0].val.programmaticStreamSerializationAllowed = 1;
   attrs[1].id = cudaLaunchAttributeClusterDimension;
-  attrs[1].val.clusterDim.x = a.G;
+  attrs[1].val.clusterDim.x = G;
   attrs[1].val.clusterDim.y = 1;
   attrs[1].val.clusterDim.z = 1;
   cfg.attrs = attrs;
@@ -637,6 +703,12 @@ unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_strid
                                      : (signs_const ? rht_kernel<false, true> : rht_kernel<false, false>);
   const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, a);
   return e == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+}
+
+unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_stride, int M, int n,
+                         const uint8_t* signs, int signs_first, bool signs_const, cudaStream_t s) {
+  const RhtSetDesc d{in, in_stride, out, out_stride, n, signs};
+  return launch_rht_sets(&d, 1, M, signs_first, signs_const, s);
 }
 
 }  // namespace unisvq

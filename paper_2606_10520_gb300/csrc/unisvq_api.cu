@@ -643,8 +643,11 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
     unisvq_status st = launch_rht(static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * K, K, hs[0]->rht_x, K,
                                   mc, K, hs[0]->rht_signs, 1, true, s);
     if (st == UNISVQ_OK) st = group_inner(hs, n, kernel, hs[0]->rht_x, yc, mc, s);
-    for (int i = 0; i < n && st == UNISVQ_OK; ++i)
-      st = launch_rht(yc[i], hs[i]->N, yc[i], hs[i]->N, mc, hs[i]->N, hs[i]->rht_signs + K, 0, true, s);
+    if (st == UNISVQ_OK) {   // the output rotations of all layers, one launch where the widths allow
+      RhtSetDesc sets[UNISVQ_MAX_GROUP];
+      for (int i = 0; i < n; ++i) sets[i] = RhtSetDesc{yc[i], hs[i]->N, yc[i], hs[i]->N, hs[i]->N, hs[i]->rht_signs + K};
+      st = launch_rht_sets(sets, n, mc, 0, true, s);
+    }
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;

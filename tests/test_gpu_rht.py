@@ -167,12 +167,17 @@ def test_set_rht_rejects_unsupported_widths_and_bad_signs():
     layer.close()
 
 
-@pytest.mark.parametrize("M", [1, 16, 40])
-def test_group_call_sharing_the_input_rotation(M):
+@pytest.mark.parametrize("M,Ns", [(1, (4096, 1024, 1024)), (16, (4096, 1024, 1024)), (40, (4096, 1024, 1024)),
+                                  (5, (11008, 11008)), (16, (11008, 11008)), (3, (4096, 14336)),
+                                  (7, (1024, 11008, 4096))])
+def test_group_call_sharing_the_input_rotation(M, Ns):
     """Layers that share S_V (same input space) rotate x once and run as one
-    group; each output still gets its own U S_U."""
+    group; each output still gets its own U S_U. The output rotations of
+    widths with one H_m and cluster size run as one launch (4096 and 1024,
+    11008 twice), the others one launch per width (4096 with 14336 = 2^9 * 28,
+    11008 = 2^5 * 344 with powers of two)."""
     K, d = 4096, 2
-    shapes = [(4096, K), (1024, K), (1024, K)]
+    shapes = [(N, K) for N in Ns]
     made = [synth.layer_inputs(7, 54, i, 0, N, K_, d) for i, (N, K_) in enumerate(shapes)]
     layers = [binding.UniSVQLinear(c, A, B) for c, A, B in made]
     s_V = signs(K, 99)
