@@ -44,8 +44,11 @@
 // (same K) run in one launch of each kernel: their row blocks are stacked
 // along grid.y of decode_kernel, their folds along grid.z of fold_kernel.
 #include <atomic>
+#include <cstring>
+#include <cmath>
 
 #include "common.cuh"
+#include "hadamard.cuh"
 #include "internal.h"
 
 namespace unisvq {
@@ -101,6 +104,12 @@ struct FoldArgs {
   int kt_per_cta;
   int ncol;            // B rows (16, 32, 48)
   int nlayers;
+  // Fused input rotation of the inverse RHT (x -> (x S_V) H_K / sqrt(K)):
+  // S_V as sign bytes [K] (1 = -1), or null for none.
+  const uint8_t* rht_sv;
+  int rht_m;                   // Paley order m of K = p2 m (1, 12, 20 or 28)
+  float rht_scale;             // 1 / sqrt(K)
+  uint32_t rht_neg[28];        // column masks of H_m (m > 1)
   FoldLayer<DV> layer[kMaxGroup];
 };
 
@@ -252,12 +261,59 @@ __device__ __forceinline__ void fold4(int d, const float (&A)[16], const float (
   }
 }
 
+// The rotated activations of slice s (positions [s L, (s + 1) L) of the
+// row, L = K / KS with KS = gridDim.x slices) for the fused inverse RHT, into
+// xs as bf16. With H_K = H_{2^a} (Sylvester) Kronecker H_m and KS dividing
+// 2^a, Sylvester's matrix splits over the high and low bits of the block
+// index, so the slice needs (1) the signed sum over the KS slices of the row,
+// term h with sign (-1)^popcount(h & s), of S_V x; (2) H_m on each of its
+// L / m blocks; (3) Sylvester's transform over those blocks; then the scale
+// 1 / sqrt(K). r0, r1: two fp32 buffers of L values in shared memory.
+template <int DV>
+__device__ __forceinline__ void fold_rotate_slice(const FoldArgs<DV>& a, const uint16_t* row, int s, int L,
+                                                  uint16_t* xs, float* r0, float* r1) {
+  const int KS = static_cast<int>(gridDim.x);
+  for (int j8 = threadIdx.x; j8 < L / 8; j8 += kFoldThreads) {
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int h = 0; h < KS; ++h) {
+      const int k = h * L + 8 * j8;
+      const uint4 u = ldg_v4(row + k);
+      const uint2 sb = __ldg(reinterpret_cast<const uint2*>(a.rht_sv + k));
+      const uint32_t flip_h = (__popc(h & s) & 1) ? 0x80000000u : 0u;
+      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int t = 0; t < 8; ++t) {
+        const float v = (t & 1) ? bf16_hi(w[t >> 1]) : bf16_lo(w[t >> 1]);
+        const uint32_t sbyte = (((t >> 2) ? sb.y : sb.x) >> (8 * (t & 3))) & 0xffu;
+        acc[t] += __uint_as_float(__float_as_uint(v) ^ flip_h ^ (sbyte ? 0x80000000u : 0u));
+      }
+    }
+#pragma unroll
+    for (int t = 0; t < 8; ++t) r0[8 * j8 + t] = acc[t];
+  }
+  __syncthreads();
+  const int m = a.rht_m, nblk = L / m;
+  float* buf = r0;
+  if (m > 1) {
+    if (m == 12) paley_blocks<kFoldThreads, 12>(r0, r1, nblk, a.rht_neg);
+    else if (m == 20) paley_blocks<kFoldThreads, 20>(r0, r1, nblk, a.rht_neg);
+    else paley_blocks<kFoldThreads, 28>(r0, r1, nblk, a.rht_neg);
+    buf = r1;
+    __syncthreads();
+  }
+  sylvester_all<kFoldThreads>(buf, nblk, m);
+  for (int j = threadIdx.x; j < L; j += kFoldThreads) xs[j] = f32_to_bf16_rn(buf[j] * a.rht_scale);
+  __syncthreads();
+}
+
 // Fold of one K slice for one token of one layer: the scale 2^P and the bias
 // sum c over the slice, then the slice's B tiles (rows 3 tok .. 3 tok + 2) in
 // the layer's workspace. Rows of absent tokens are never written: an MMA
 // column depends on its own B row only, and the epilogue never reads those
 // columns.
-template <int DV>
+// kRht: the instance with the fused input rotation (its registers do not
+// limit the residency of the plain instance).
+template <int DV, bool kRht>
 __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constant__ FoldArgs<DV> a) {
   extern __shared__ __align__(16) uint8_t fsm[];
   uint16_t* xs = reinterpret_cast<uint16_t*>(fsm);   // the token's x slice, zero past K
@@ -322,7 +378,27 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
   const bool vec8 = (a.K & 7) == 0;
   const uint16_t* row = a.x + static_cast<size_t>(tok) * a.K;
   float mx = 0.f, cs = 0.f;
-  for (int c0 = tid * 8; c0 < span; c0 += kFoldThreads * 8 * 4) {
+  if constexpr (kRht) {   // the slice of the rotated row (every slice full: K = KS span)
+    float* r0 = reinterpret_cast<float*>(fsm + static_cast<size_t>(span) * 2);
+    fold_rotate_slice(a, row, s, span, xs, r0, r0 + span);
+    for (int c = tid * 8; c < span; c += kFoldThreads * 8) {
+      const uint4 u = *reinterpret_cast<const uint4*>(xs + c);
+      const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {   // c is a multiple of 8: (k + i) mod d = i mod d
+        const float v0 = bf16_lo(w4[t]), v1 = bf16_hi(w4[t]);
+        mx = fmaxf(mx, fmaxf(fabsf(v0), fabsf(v1)));
+        if constexpr (DV == 8) {
+          cs = fmaf(v0, Bv[2 * t], cs);
+          cs = fmaf(v1, Bv[2 * t + 1], cs);
+        } else {
+          cs = fmaf(v0, Bv[(2 * t) & (d - 1)], cs);
+          cs = fmaf(v1, Bv[(2 * t + 1) & (d - 1)], cs);
+        }
+      }
+    }
+  }
+  for (int c0 = tid * 8; !kRht && c0 < span; c0 += kFoldThreads * 8 * 4) {
     uint4 u[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
@@ -731,8 +807,14 @@ bool set_fold_attrs(int dev) {
   static bool done[64] = {};
   if (dev < 0 || dev >= 64) return false;
   if (done[dev]) return true;
-  if (cudaFuncSetAttribute(fold_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFoldMaxSmem) != cudaSuccess ||
-      cudaFuncSetAttribute(fold_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFoldMaxSmem) != cudaSuccess)
+  if (cudaFuncSetAttribute(fold_kernel<4, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFoldMaxSmem) !=
+          cudaSuccess ||
+      cudaFuncSetAttribute(fold_kernel<8, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFoldMaxSmem) !=
+          cudaSuccess ||
+      cudaFuncSetAttribute(fold_kernel<4, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFoldMaxSmem) !=
+          cudaSuccess ||
+      cudaFuncSetAttribute(fold_kernel<8, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFoldMaxSmem) !=
+          cudaSuccess)
     return false;
   done[dev] = true;
   return true;
@@ -796,6 +878,18 @@ DecodePlan plan_rows_split(int nb, int KT, int num_sms, int M) {
   return p2;
 }
 
+// The plan of a launch whose fold kernel also rotates x (K = p2 m): the K
+// split reduced to the largest power of 2 that divides both KT and p2, so
+// every slice is full and a union of whole m-blocks.
+DecodePlan plan_rht(int nb, int KT, int num_sms, int M, int p2) {
+  DecodePlan p = plan_rows_split(nb, KT, num_sms, M);
+  int ks = 1;
+  while (ks * 2 <= p.ks && KT % (ks * 2) == 0 && p2 % (ks * 2) == 0) ks *= 2;
+  p.ks = ks;
+  p.kt_per_cta = KT / ks;
+  return p;
+}
+
 cudaLaunchAttribute pdl_attr() {
   cudaLaunchAttribute at;
   at.id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -838,10 +932,10 @@ DecodePlan plan_skinny(const unisvq_layer* L, int M) {
 
 namespace {
 
-// The fold of tokens m0 .. m0 + mc - 1 for plan p (fold_kernel<DV>).
+// The fold of tokens m0 .. m0 + mc - 1 for plan p (fold_kernel<DV, rht_sv != null>).
 template <int DV>
 unisvq_status launch_fold(const unisvq_layer* const* Ls, int n, const void* x, int m0, int mc, const DecodePlan& p,
-                          cudaStream_t s, uint8_t* const* ws) {
+                          cudaStream_t s, uint8_t* const* ws, const uint8_t* rht_sv) {
   const unisvq_layer* L0 = Ls[0];
   FoldArgs<DV> f{};
   f.x = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * L0->K;
@@ -851,6 +945,16 @@ unisvq_status launch_fold(const unisvq_layer* const* Ls, int n, const void* x, i
   f.kt_per_cta = p.kt_per_cta;
   f.ncol = p.nt;
   f.nlayers = n;
+  size_t smem = static_cast<size_t>(p.kt_per_cta) * kTileCols * 2;
+  if (rht_sv) {   // fused input rotation: two fp32 copies of the slice besides the bf16 one
+    int p2 = 0, m = 0;
+    if (!rht_factor(L0->K, &p2, &m) || m > 28) return UNISVQ_ERR_UNSUPPORTED;
+    f.rht_sv = rht_sv;
+    f.rht_m = m;
+    f.rht_scale = static_cast<float>(1.0 / std::sqrt(static_cast<double>(L0->K)));
+    if (m > 1) std::memcpy(f.rht_neg, rht_paley_masks(m), sizeof(f.rht_neg));
+    smem *= 5;
+  }
   for (int i = 0; i < n; ++i) {
     const unisvq_layer* L = Ls[i];
     FoldLayer<DV>& fl = f.layer[i];
@@ -863,18 +967,21 @@ unisvq_status launch_fold(const unisvq_layer* const* Ls, int n, const void* x, i
   cudaLaunchConfig_t fc = {};
   fc.gridDim = dim3(p.ks, mc, n);
   fc.blockDim = dim3(kFoldThreads, 1, 1);
-  fc.dynamicSmemBytes = static_cast<size_t>(p.kt_per_cta) * kTileCols * 2;
+  fc.dynamicSmemBytes = smem;
   fc.stream = s;
   cudaLaunchAttribute fat[1] = {pdl_attr()};
   fc.attrs = fat;
   fc.numAttrs = 1;
-  return cudaLaunchKernelEx(&fc, fold_kernel<DV>, f) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+  const cudaError_t e = rht_sv ? cudaLaunchKernelEx(&fc, fold_kernel<DV, true>, f)
+                               : cudaLaunchKernelEx(&fc, fold_kernel<DV, false>, f);
+  return e == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
 // Fold and stream, the fold workspace of layer i at ws[i], at most max_tok
 // tokens per launch.
 unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
-                               cudaStream_t s, uint8_t* const* ws, int max_tok = kMaxTokPerLaunch) {
+                               cudaStream_t s, uint8_t* const* ws, int max_tok = kMaxTokPerLaunch,
+                               const uint8_t* rht_sv = nullptr) {
   if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
   const unisvq_layer* L0 = Ls[0];
   if (!set_fold_attrs(L0->device)) return UNISVQ_ERR_CUDA;
@@ -884,9 +991,12 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
     nb += Ls[i]->Np / kTileRows;
     d8 = d8 || Ls[i]->d == 8;
   }
+  int rht_p2 = 0, rht_m = 0;
+  if (rht_sv && !rht_factor(L0->K, &rht_p2, &rht_m)) return UNISVQ_ERR_UNSUPPORTED;
   for (int m0 = 0; m0 < M; m0 += max_tok) {
     const int mc = M - m0 < max_tok ? M - m0 : max_tok;
-    const DecodePlan p = plan_rows_split(nb, L0->KT, L0->num_sms, mc);
+    const DecodePlan p = rht_sv ? plan_rht(nb, L0->KT, L0->num_sms, mc, rht_p2)
+                                : plan_rows_split(nb, L0->KT, L0->num_sms, mc);
     if (p.ks > kMaxSplit) return UNISVQ_ERR_UNSUPPORTED;
     SkArgs a{};
     a.M = mc;
@@ -905,7 +1015,8 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
       l.rb0 = rb0;
       rb0 += L->Np / kTileRows;
     }
-    unisvq_status st = d8 ? launch_fold<8>(Ls, n, x, m0, mc, p, s, ws) : launch_fold<4>(Ls, n, x, m0, mc, p, s, ws);
+    unisvq_status st = d8 ? launch_fold<8>(Ls, n, x, m0, mc, p, s, ws, rht_sv)
+                          : launch_fold<4>(Ls, n, x, m0, mc, p, s, ws, rht_sv);
     if (st != UNISVQ_OK) return st;
     if (p.nt == 16) st = p.geom == 1 ? launch_ncol<16, 1>(a, p, L0->device, s) : launch_ncol<16, 2>(a, p, L0->device, s);
     else if (p.nt == 32) st = p.geom == 1 ? launch_ncol<32, 1>(a, p, L0->device, s) : launch_ncol<32, 2>(a, p, L0->device, s);
@@ -929,6 +1040,36 @@ unisvq_status launch_skinny_group(const unisvq_layer* const* Ls, int n, const vo
 unisvq_status launch_skinny(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
   void* ys[1] = {y};
   return launch_skinny_group(&L, 1, x, ys, M, s);
+}
+
+bool skinny_rht_foldable(const unisvq_layer* const* Ls, int n, int M) {
+  if (n < 1 || n > kMaxGroup || M < 1) return false;
+  const unisvq_layer* L0 = Ls[0];
+  int p2 = 0, m = 0;
+  if (!rht_factor(L0->K, &p2, &m) || m > 28 || L0->K != L0->KT * kTileCols) return false;
+  int nb = 0;
+  for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
+  // every launch size of the call: full launches and the remainder
+  const int sizes[2] = {M < kMaxTokPerLaunch ? M : kMaxTokPerLaunch, M > kMaxTokPerLaunch ? M % kMaxTokPerLaunch : 0};
+  for (const int mc : sizes) {
+    if (mc == 0) continue;
+    // a K split of 1 would leave one CTA per token and layer to transform the
+    // whole row: measured slower than the separate rotation kernel (cluster
+    // of CTAs) whose latency the decode kernel's code prefetch hides
+    const DecodePlan p = plan_rht(nb, L0->KT, L0->num_sms, mc, p2);
+    if (p.ks < 2 || p.ks * p.kt_per_cta != L0->KT || p2 % p.ks != 0) return false;
+    if (static_cast<size_t>(p.kt_per_cta) * kTileCols * 10 > static_cast<size_t>(kFoldMaxSmem)) return false;
+  }
+  return true;
+}
+
+unisvq_status launch_skinny_group_rht(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                                      const uint8_t* rht_sv, cudaStream_t s) {
+  if (n < 1 || n > kMaxGroup || !rht_sv) return UNISVQ_ERR_INVALID_ARG;
+  if (!skinny_rht_foldable(Ls, n, M)) return UNISVQ_ERR_UNSUPPORTED;
+  uint8_t* ws[kMaxGroup];
+  for (int i = 0; i < n; ++i) ws[i] = Ls[i]->fold_ws;
+  return launch_skinny_ws(Ls, n, x, ys, M, s, ws, kMaxTokPerLaunch, rht_sv);
 }
 
 // ---- allocation-free variant (unisvq_linear_noalloc) -------------------------

@@ -99,9 +99,19 @@ DecodePlan plan_skinny(const unisvq_layer* L, int M);
 unisvq_status launch_skinny(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
 // Device bytes of a handle's fold workspace for the skinny decode kernel.
 size_t fold_workspace_bytes(int KT);
-// Several layers with the same K that read the same x, in one launch per 16 tokens.
+// Several layers with the same K that read the same x, in one launch pair per 32 tokens.
 unisvq_status launch_skinny_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
                                   cudaStream_t s);
+// The same with the input rotation of the inverse RHT, x -> (x S_V) H_K /
+// sqrt(K), done by the fold kernel (rht_sv: S_V sign bytes on the device,
+// 8-byte aligned). Possible where skinny_rht_foldable holds: K = 2^a m with
+// m in {1, 12, 20, 28}; the launches then split K into KS full slices, KS the
+// largest power of 2 up to the usual split that divides both K / 128 and
+// 2^a, at least 2, each slice's bf16 and two fp32 copies within the fold
+// kernel's shared memory.
+bool skinny_rht_foldable(const unisvq_layer* const* Ls, int n, int M);
+unisvq_status launch_skinny_group_rht(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
+                                      const uint8_t* rht_sv, cudaStream_t s);
 // As launch_skinny with the fold workspace in a static device array of
 // static_fold_workspace_bytes() (UNSUPPORTED if the layer needs more).
 unisvq_status launch_skinny_static(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
@@ -135,6 +145,9 @@ unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s);
 // before the first launch_rht of such an n.
 bool rht_factor(int n, int* p2, int* m);
 unisvq_status rht_prepare(int n);
+// Column sign masks of H_m for m in {12, 20, 28}: 28 words, bit q of word c
+// set where H_m[q][c] = -1.
+const uint32_t* rht_paley_masks(int m);
 size_t rht_smem_bytes(int n);
 // signs_const: the sign bytes never change between launches (a handle's own
 // buffer), so the kernel reads them before waiting for the previous kernel.
@@ -153,6 +166,8 @@ struct RhtSetDesc {
 };
 unisvq_status launch_rht_sets(const RhtSetDesc* sets, int nsets, int M, int signs_first, bool signs_const,
                               cudaStream_t s);
+// Launches launch_rht_sets makes for row sets of these widths (1 or nsets).
+int rht_set_launches(const int* ns, int nsets);
 
 // Per-(row, group) affine layers (gemv_grouped.cu): every M, at most 32 / d
 // tokens per launch; all layers of one call must be grouped with the same d.

@@ -28,6 +28,7 @@
 #include <vector>
 
 #include "common.cuh"
+#include "hadamard.cuh"
 #include "internal.h"
 
 namespace unisvq {
@@ -79,28 +80,6 @@ struct RhtArgs {
 };
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float(static_cast<uint32_t>(b) << 16); }
-
-// Row vector times H_m for every block of M_ consecutive entries of src,
-// into dst: four threads per block, each forming M_/4 of its outputs.
-template <int M_>
-__device__ __forceinline__ void paley_blocks(const float* src, float* dst, int nblk, const uint32_t* neg) {
-  constexpr int C = M_ / 4;
-  for (int it = threadIdx.x; it < nblk * 4; it += kRThreads) {
-    const int p = it >> 2, c0 = (it & 3) * C;
-    const float* blk = src + p * M_;
-    float v[M_];
-#pragma unroll
-    for (int q = 0; q < M_; ++q) v[q] = blk[q];
-#pragma unroll
-    for (int c = 0; c < C; ++c) {
-      const uint32_t mask = neg[c0 + c];
-      float acc = 0.f;
-#pragma unroll
-      for (int q = 0; q < M_; ++q) acc += ((mask >> q) & 1u) ? -v[q] : v[q];
-      dst[p * M_ + c0 + c] = acc;
-    }
-  }
-}
 
 // Row vector times H_344 for every block of 344 consecutive entries, on the
 // tensor cores as D^T = H_344^T X^T: D^T[c][b] = sum_q H_344[q][c] X[b][q]
@@ -172,35 +151,6 @@ __device__ __forceinline__ void paley344_mma(const uint16_t* x_bf16, float* dst,
         if (b0 + 1 < nblk) dst[(b0 + 1) * kP344 + cc] = acc[i][2 * h + 1];
       }
     }
-  }
-}
-
-// Sylvester stages s0 .. s0 + R - 1 (butterfly distances 2^s0 .. 2^(s0+R-1)
-// blocks) for every column of the p2 x m view, R stages per pass in registers.
-template <int R>
-__device__ __forceinline__ void sylvester_pass(float* buf, int p2, int m, int s0) {
-  constexpr int G = 1 << R;
-  const int h = 1 << s0;
-  const int groups = (p2 >> R) * m;
-  for (int gi = threadIdx.x; gi < groups; gi += kRThreads) {
-    const int col = gi % m, rest = gi / m;
-    const int lo = (rest & (h - 1)) | ((rest >> s0) << (s0 + R));   // R zero bits inserted at s0
-    float v[G];
-#pragma unroll
-    for (int j = 0; j < G; ++j) v[j] = buf[(lo + j * h) * m + col];
-#pragma unroll
-    for (int st = 0; st < R; ++st) {
-      const int d = 1 << st;
-#pragma unroll
-      for (int j = 0; j < G; ++j)
-        if (!(j & d)) {
-          const float a = v[j], b = v[j + d];
-          v[j] = a + b;
-          v[j + d] = a - b;
-        }
-    }
-#pragma unroll
-    for (int j = 0; j < G; ++j) buf[(lo + j * h) * m + col] = v[j];
   }
 }
 
@@ -377,23 +327,14 @@ __global__ void __launch_bounds__(kRThreads, kP344Path ? 1 : 3) rht_kernel(const
     __syncthreads();
     if (a.m > 1) {
       float* out2 = smem_f + chunk;
-      if (a.m == 12) paley_blocks<12>(buf, out2, pl, a.hm_neg);
-      else if (a.m == 20) paley_blocks<20>(buf, out2, pl, a.hm_neg);
-      else paley_blocks<28>(buf, out2, pl, a.hm_neg);
+      if (a.m == 12) paley_blocks<kRThreads, 12>(buf, out2, pl, a.hm_neg);
+      else if (a.m == 20) paley_blocks<kRThreads, 20>(buf, out2, pl, a.hm_neg);
+      else paley_blocks<kRThreads, 28>(buf, out2, pl, a.hm_neg);
       buf = out2;
       __syncthreads();
     }
   }
-  int lg = 0;
-  while ((1 << lg) < pl) ++lg;
-  for (int s0 = 0; s0 < lg;) {
-    const int r = min(3, lg - s0);
-    if (r == 3) sylvester_pass<3>(buf, pl, a.m, s0);
-    else if (r == 2) sylvester_pass<2>(buf, pl, a.m, s0);
-    else sylvester_pass<1>(buf, pl, a.m, s0);
-    s0 += r;
-    __syncthreads();
-  }
+  sylvester_all<kRThreads>(buf, pl, a.m);
   uint16_t* dst = s_out + static_cast<size_t>(row) * s_out_stride;
   if (G == 1) {
     const bool sgn_out = !a.signs_first && s_signs;
@@ -613,7 +554,7 @@ size_t rht_smem_bytes(int n) {
 
 // Column sign masks of H_m for m in {12, 20, 28} (kMaxPaley words each, bit q
 // of word c set where H_m[q][c] = -1), built once.
-static const uint32_t* paley_masks(int m) {
+const uint32_t* rht_paley_masks(int m) {
   static const std::vector<uint32_t> table = [] {
     std::vector<uint32_t> t(3 * kMaxPaley, 0u);
     const int orders[3] = {12, 20, 28};
@@ -683,7 +624,7 @@ unisvq_status launch_rht_sets(const RhtSetDesc* sets, int nsets, int M, int sign
     a.h344_bits = h344_table(dev);
     if (!a.h344_bits) return UNISVQ_ERR_CUDA;
   } else if (m > 1) {
-    std::memcpy(a.hm_neg, paley_masks(m), sizeof(a.hm_neg));
+    std::memcpy(a.hm_neg, rht_paley_masks(m), sizeof(a.hm_neg));
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(nsets * M * G, 1, 1);
@@ -703,6 +644,16 @@ unisvq_status launch_rht_sets(const RhtSetDesc* sets, int nsets, int M, int sign
                                      : (signs_const ? rht_kernel<false, true> : rht_kernel<false, false>);
   const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, a);
   return e == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+}
+
+int rht_set_launches(const int* ns, int nsets) {
+  int p0 = 0, m0 = 0;
+  if (nsets < 1 || !rht_factor(ns[0], &p0, &m0)) return nsets;
+  for (int i = 1; i < nsets; ++i) {
+    int p = 0, m = 0;
+    if (!rht_factor(ns[i], &p, &m) || m != m0 || rht_ctas(ns[i], p, m) != rht_ctas(ns[0], p0, m0)) return nsets;
+  }
+  return 1;
 }
 
 unisvq_status launch_rht(const void* in, int in_stride, void* out, int out_stride, int M, int n,

@@ -489,15 +489,45 @@ static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, vo
   return UNISVQ_ERR_INVALID_ARG;
 }
 
+// Whether the layers of a call with the inverse RHT (one S_V) run the tcgen05
+// decode path with the input rotation fused into its fold kernel: 2-bit
+// per-matrix layers whose call resolves to UNISVQ_KERNEL_SKINNY, K foldable.
+static bool rht_fused(const unisvq_handle* hs, int n, int kernel, int M) {
+  long long weights = 0;
+  int nb = 0;
+  for (int i = 0; i < n; ++i) {
+    if (hs[i]->bits != 2 || hs[i]->grouped) return false;
+    weights += static_cast<long long>(hs[i]->N) * hs[i]->K;
+    nb += hs[i]->Np / kTileRows;
+  }
+  if (kernel == UNISVQ_KERNEL_AUTO)
+    kernel = M > 64 && prefill_supported(hs[0], M) ? UNISVQ_KERNEL_PREFILL : decode_kernel_for(weights, nb, M);
+  else if (kernel == UNISVQ_KERNEL_DECODE)
+    kernel = decode_kernel_for(weights, nb, M);
+  if (kernel != UNISVQ_KERNEL_SKINNY) return false;
+  const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
+  for (int i = 0; i < n; ++i) Ls[i] = hs[i];
+  return skinny_rht_foldable(Ls, n, M);
+}
+
 // The layer with the inverse RHT around it when the handle has one (Eq.
-// def:hadamard: y = ((x S_V V) W_hat^T) U S_U), in chunks of the handle's
-// rotated-activation buffer; else the layer alone.
+// def:hadamard: y = ((x S_V V) W_hat^T) U S_U): on the tcgen05 decode path
+// the fold kernel rotates x itself and one kernel rotates y; otherwise a
+// rotation kernel, the layer and a rotation kernel per chunk of the handle's
+// rotated-activation buffer. Without the RHT, the layer alone.
 static unisvq_status linear_rht(unisvq_handle h, int kernel, const void* x, void* y, int M, cudaStream_t s,
                                 bool noalloc) {
   if (!h->rht) return linear_inner(h, kernel, x, y, M, s, noalloc);
   if (kernel < UNISVQ_KERNEL_AUTO || kernel > UNISVQ_KERNEL_STREAM) return UNISVQ_ERR_INVALID_ARG;
   const uint8_t* s_in = h->rht_signs;
   const uint8_t* s_out = h->rht_signs + h->K;
+  if (!noalloc && rht_fused(&h, 1, kernel, M)) {
+    const unisvq_layer* Ls[1] = {h};
+    void* ys[1] = {y};
+    unisvq_status st = launch_skinny_group_rht(Ls, 1, x, ys, M, s_in, s);
+    if (st == UNISVQ_OK) st = launch_rht(y, h->N, y, h->N, M, h->N, s_out, 0, true, s);
+    return st;
+  }
   for (int m0 = 0; m0 < M; m0 += h->rht_tokens) {
     const int mc = M - m0 < h->rht_tokens ? M - m0 : h->rht_tokens;
     const uint16_t* xc = static_cast<const uint16_t*>(x) + static_cast<size_t>(m0) * h->K;
@@ -633,9 +663,20 @@ unisvq_status unisvq_linear_group_force(const unisvq_handle* hs, int n, int kern
   // One S_V for every layer: rotate x once (into the first handle's buffer),
   // run the layers as one group, rotate each output with its own U S_U.
   if (kernel < UNISVQ_KERNEL_AUTO || kernel > UNISVQ_KERNEL_STREAM) return UNISVQ_ERR_INVALID_ARG;
+  const int K = hs[0]->K;
+  if (rht_fused(hs, n, kernel, M)) {   // the fold kernel rotates x; one launch rotates the outputs
+    const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
+    RhtSetDesc sets[UNISVQ_MAX_GROUP];
+    for (int i = 0; i < n; ++i) {
+      Ls[i] = hs[i];
+      sets[i] = RhtSetDesc{ys[i], hs[i]->N, ys[i], hs[i]->N, hs[i]->N, hs[i]->rht_signs + K};
+    }
+    unisvq_status st = launch_skinny_group_rht(Ls, n, x, ys, M, hs[0]->rht_signs, s);
+    if (st == UNISVQ_OK) st = launch_rht_sets(sets, n, M, 0, true, s);
+    return st;
+  }
   int cap = hs[0]->rht_tokens;
   for (int i = 1; i < n; ++i) cap = hs[i]->rht_tokens < cap ? hs[i]->rht_tokens : cap;
-  const int K = hs[0]->K;
   for (int m0 = 0; m0 < M; m0 += cap) {
     const int mc = M - m0 < cap ? M - m0 : cap;
     void* yc[UNISVQ_MAX_GROUP];
@@ -821,9 +862,13 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
                  : h->bits == 3 ? (mq > 64 && prefill_supported(h, mq) ? UNISVQ_KERNEL_PREFILL : UNISVQ_KERNEL_GEMV)
                                 : auto_kernel(h, mq);
   describe_launch(Ls, 1, kq, M, info);
-  if (h->rht) {   // an input and an output rotation per chunk of the rotated-activation buffer
-    const int m = M > 0 ? M : 1;
-    info->launches += 2 * ((m + h->rht_tokens - 1) / h->rht_tokens);
+  if (h->rht) {
+    // fused: one output rotation; else an input and an output rotation per
+    // chunk of the rotated-activation buffer
+    if (rht_fused(&h, 1, UNISVQ_KERNEL_AUTO, mq))
+      info->launches += 1;
+    else
+      info->launches += 2 * ((mq + h->rht_tokens - 1) / h->rht_tokens);
   }
   return UNISVQ_OK;
 }
@@ -860,6 +905,31 @@ unisvq_status unisvq_query_group(const unisvq_handle* hs, int n, int M, unisvq_i
   const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
   for (int i = 0; i < n; ++i) Ls[i] = hs[i];
   describe_launch(Ls, n, kernel, M, info);
+  int nrht = 0;
+  for (int i = 0; i < n; ++i) nrht += hs[i]->rht ? 1 : 0;
+  if (nrht) {   // the rotations of unisvq_linear_group_force's RHT paths
+    bool shared = nrht == n;
+    for (int i = 1; i < n && shared; ++i) shared = hs[i]->rht_in_host == hs[0]->rht_in_host;
+    if (!shared) {   // one unisvq_linear per layer: count each layer's own launches
+      info->launches = 0;
+      for (int i = 0; i < n; ++i) {
+        unisvq_info one;
+        unisvq_query(hs[i], M, &one);
+        info->launches += one.launches;
+      }
+    } else {
+      int ns[UNISVQ_MAX_GROUP], cap = hs[0]->rht_tokens;
+      for (int i = 0; i < n; ++i) {
+        ns[i] = hs[i]->N;
+        cap = hs[i]->rht_tokens < cap ? hs[i]->rht_tokens : cap;
+      }
+      const int outs = rht_set_launches(ns, n);
+      if (rht_fused(hs, n, UNISVQ_KERNEL_AUTO, m))
+        info->launches += outs;
+      else
+        info->launches += (1 + outs) * ((m + cap - 1) / cap);
+    }
+  }
   return UNISVQ_OK;
 }
 

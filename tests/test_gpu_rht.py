@@ -193,3 +193,66 @@ def test_group_call_sharing_the_input_rotation(M, Ns):
         assert res["ok"], res
     for layer in layers:
         layer.close()
+
+
+@pytest.mark.parametrize("N,K,d", [(4096, 4096, 2), (4096, 14336, 2), (1024, 5120, 4), (1024, 3072, 2),
+                                   (1024, 2048, 8), (1792, 3584, 2), (512, 1536, 1)])
+def test_input_rotation_fused_into_the_fold(N, K, d):
+    """The tcgen05 decode path rotates x inside its fold kernel where K = 2^a m
+    (m in 1, 12, 20, 28) splits into full slices of whole blocks (4096, 14336
+    = 2^9 * 28, 5120 = 2^8 * 20, 3072 = 2^8 * 12, 2048 with d = 8); K = 3584
+    and 1536 split into 7 and 6 slices and take the separate rotation. The
+    layer matches the oracle for token counts inside one launch and across
+    two."""
+    codes, A, B = synth.layer_inputs(7, 56, N, K, N, K, d)
+    layer = binding.UniSVQLinear(codes, A, B)
+    s_U, s_V = signs(N, 3 + N), signs(K, 4 + K)
+    layer.set_rht(s_V, s_U, max_tokens=8)
+    Ms = (1, 7, 16, 33)
+    xall = synth.activations(7, 56, N + K, sum(Ms), K)
+    yr, S = oracle.linear_rht(xall, codes, A, B, s_U, s_V)
+    o = 0
+    for M in Ms:
+        y = layer.forward(to_dev(xall[o:o + M]), kernel=binding.KERNEL_SKINNY)
+        assert binding.sync_status() == binding.OK
+        res = oracle.compare(host(y), yr[o:o + M], S[o:o + M])
+        assert res["ok"], (M, res)
+        o += M
+    layer.close()
+
+
+def test_fused_rotation_launch_counts():
+    """Where the call resolves to the tcgen05 path, the RHT adds one launch
+    (the output rotation): the fold kernel rotates the input."""
+    K = 4096
+    big = binding.UniSVQLinear(*synth.layer_inputs(7, 57, 0, 0, 14336, K, 2))
+    big.set_rht(signs(K, 5), signs(14336, 6), max_tokens=8)
+    assert big.query(5)["kernel"] == binding.KERNEL_SKINNY
+    assert big.query(5)["launches"] == 2 + 1       # K split 2 or more: fused
+    # 40 tokens: the 32-token launch does not split K (one CTA per row block
+    # fills the GPU), so the separate rotations run, per chunk of 8 tokens
+    assert big.query(40)["launches"] == 4 + 2 * 5
+    xb = synth.activations(7, 57, 0, 5, K)
+    y = big.forward(to_dev(xb))
+    assert binding.sync_status() == binding.OK
+    c, A, B = synth.layer_inputs(7, 57, 0, 0, 14336, K, 2)
+    ref, S = oracle.linear_rht(xb, c, A, B, signs(14336, 6), signs(K, 5))
+    assert oracle.compare(host(y), ref, S)["ok"]
+    big.close()
+    # a Llama-2-7B q/k/v group (3 x 4096 x 4096) sharing S_V: fold + decode + one output launch
+    made = [synth.layer_inputs(7, 58, i, 0, 4096, K, 2) for i in range(3)]
+    layers = [binding.UniSVQLinear(c, A, B) for c, A, B in made]
+    s_V = signs(K, 7)
+    s_Us = [signs(4096, 8 + i) for i in range(3)]
+    for layer, s_U in zip(layers, s_Us):
+        layer.set_rht(s_V, s_U, max_tokens=8)
+    info = binding.query_group(layers, 16)
+    assert info["kernel"] == binding.KERNEL_SKINNY and info["launches"] == 2 + 1
+    xb = synth.activations(7, 58, 0, 16, K)
+    ys = binding.linear_group(layers, to_dev(xb))
+    assert binding.sync_status() == binding.OK
+    for (c, A, B), s_U, y in zip(made, s_Us, ys):
+        ref, S = oracle.linear_rht(xb, c, A, B, s_U, s_V)
+        assert oracle.compare(host(y), ref, S)["ok"]
+    for layer in layers:
+        layer.close()
