@@ -926,8 +926,22 @@ static size_t fold_workspace_bytes_for(int KT, int max_tok) {
   return kWsTableBytes + static_cast<size_t>(KT) * ncol_for(max_tok) * 128;
 }
 
-DecodePlan plan_skinny(const unisvq_layer* L, int M) {
-  return plan_rows_split(L->Np / kTileRows, L->KT, L->num_sms, M > kMaxTokPerLaunch ? kMaxTokPerLaunch : M);
+// Tokens per launch pair: 32 (the 96-column accumulator, one CTA per SM)
+// where the row blocks of the call fit one wave of the SMs, else 16 (two CTAs
+// per SM). Measured on GB300 at M = 32: the Llama-2-7B gate/up pair (172 row
+// blocks) takes 35.5 us in one 32-token launch, 32.3 in two 16-token
+// launches; q/k/v (96 row blocks) 19.1 against 24.6.
+int skinny_tokens_per_launch(const unisvq_layer* const* Ls, int n) {
+  int nb = 0;
+  for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
+  return nb <= Ls[0]->num_sms ? kMaxTokPerLaunch : 16;
+}
+
+DecodePlan plan_skinny(const unisvq_layer* const* Ls, int n, int M) {
+  int nb = 0;
+  for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
+  const int per = skinny_tokens_per_launch(Ls, n);
+  return plan_rows_split(nb, Ls[0]->KT, Ls[0]->num_sms, M > per ? per : M);
 }
 
 namespace {
@@ -1034,7 +1048,7 @@ unisvq_status launch_skinny_group(const unisvq_layer* const* Ls, int n, const vo
   if (n < 1 || n > kMaxGroup) return UNISVQ_ERR_INVALID_ARG;
   uint8_t* ws[kMaxGroup];
   for (int i = 0; i < n; ++i) ws[i] = Ls[i]->fold_ws;
-  return launch_skinny_ws(Ls, n, x, ys, M, s, ws);
+  return launch_skinny_ws(Ls, n, x, ys, M, s, ws, skinny_tokens_per_launch(Ls, n));
 }
 
 unisvq_status launch_skinny(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
@@ -1050,7 +1064,8 @@ bool skinny_rht_foldable(const unisvq_layer* const* Ls, int n, int M) {
   int nb = 0;
   for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
   // every launch size of the call: full launches and the remainder
-  const int sizes[2] = {M < kMaxTokPerLaunch ? M : kMaxTokPerLaunch, M > kMaxTokPerLaunch ? M % kMaxTokPerLaunch : 0};
+  const int per = skinny_tokens_per_launch(Ls, n);
+  const int sizes[2] = {M < per ? M : per, M > per ? M % per : 0};
   for (const int mc : sizes) {
     if (mc == 0) continue;
     // a K split of 1 would leave one CTA per token and layer to transform the
@@ -1069,7 +1084,7 @@ unisvq_status launch_skinny_group_rht(const unisvq_layer* const* Ls, int n, cons
   if (!skinny_rht_foldable(Ls, n, M)) return UNISVQ_ERR_UNSUPPORTED;
   uint8_t* ws[kMaxGroup];
   for (int i = 0; i < n; ++i) ws[i] = Ls[i]->fold_ws;
-  return launch_skinny_ws(Ls, n, x, ys, M, s, ws, kMaxTokPerLaunch, rht_sv);
+  return launch_skinny_ws(Ls, n, x, ys, M, s, ws, skinny_tokens_per_launch(Ls, n), rht_sv);
 }
 
 // ---- allocation-free variant (unisvq_linear_noalloc) -------------------------
@@ -1085,8 +1100,9 @@ __device__ __align__(256) uint8_t g_static_fold_ws[kStaticWsBytes];
 size_t static_fold_workspace_bytes() { return kStaticWsBytes; }
 
 unisvq_status launch_skinny_static(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
-  // 32 tokens per launch where their B tiles fit the array, else 16
-  const int max_tok = fold_workspace_bytes_for(L->KT, kMaxTokPerLaunch) <= kStaticWsBytes ? kMaxTokPerLaunch : 16;
+  // unisvq_linear's tokens per launch where their B tiles fit the array, else 16
+  const int per = skinny_tokens_per_launch(&L, 1);
+  const int max_tok = fold_workspace_bytes_for(L->KT, per) <= kStaticWsBytes ? per : 16;
   if (fold_workspace_bytes_for(L->KT, max_tok) > kStaticWsBytes) return UNISVQ_ERR_UNSUPPORTED;
   // In host code g_static_fold_ws only names the symbol; its device address
   // is looked up once per device (the device of L is current here) and kept

@@ -95,7 +95,10 @@ unisvq_status launch_gemv_rows_group(const unisvq_layer* const* Ls, int n, const
 unisvq_status launch_gemv_group(const unisvq_layer* const* Ls, int n, const void* x, void* const* ys, int M,
                                 cudaStream_t s);
 // tcgen05 skinny GEMM with the codes as 8-bit TMEM operand (decode.cu), M <= 16 per launch.
-DecodePlan plan_skinny(const unisvq_layer* L, int M);
+// The plan of the call's launch pairs and their tokens per launch (32 where
+// the call's row blocks fit one wave at one CTA per SM, else 16).
+DecodePlan plan_skinny(const unisvq_layer* const* Ls, int n, int M);
+int skinny_tokens_per_launch(const unisvq_layer* const* Ls, int n);
 unisvq_status launch_skinny(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);
 // Device bytes of a handle's fold workspace for the skinny decode kernel.
 size_t fold_workspace_bytes(int KT);

@@ -403,13 +403,14 @@ unisvq_status unisvq_destroy(unisvq_handle h) {
 // of one launch and `nb` = their 128-row blocks (measured crossovers on
 // GB300, Llama-shaped layers): the tcgen05 skinny kernel (fold + streaming
 // kernel, cost nearly independent of M) for launches of at least 2^26
-// weights, or of at least 2^25 weights over 64 or more row blocks; the K-split
-// cluster GEMV (lower fixed latency, better for few row blocks) otherwise.
+// weights, or of at least 2^25 weights over 64 or more row blocks or above 16
+// tokens (Llama-2-7B down, 4096 x 11008, at M = 32: 16.4 us against 22.5 on
+// the GEMV); the K-split cluster GEMV (lower fixed latency, better for few
+// row blocks) otherwise.
 // The whole-K row-slice GEMV is reachable through the force calls only.
 static int decode_kernel_for(long long weights, int nb, int M) {
-  (void)M;
   if (weights >= (1ll << 26)) return UNISVQ_KERNEL_SKINNY;
-  if (weights >= (1ll << 25) && nb >= 64) return UNISVQ_KERNEL_SKINNY;
+  if (weights >= (1ll << 25) && (nb >= 64 || M > 16)) return UNISVQ_KERNEL_SKINNY;
   return UNISVQ_KERNEL_GEMV;
 }
 
@@ -823,12 +824,13 @@ static void describe_launch(const unisvq_layer* const* Ls, int n, int kernel, in
     info->launches = (m + 31) / 32;
     info->grid_ctas = p.ks * nb * info->launches;
   } else if (kernel == UNISVQ_KERNEL_SKINNY) {
-    const DecodePlan p = plan_skinny(h, m > 32 ? 32 : m);
+    const DecodePlan p = plan_skinny(Ls, n, m);
+    const int per = skinny_tokens_per_launch(Ls, n);
     int nb = 0;
     for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
     info->split_k = p.ks;
-    const int chunks = (m + 31) / 32;
-    info->launches = 2 * chunks;   // fold kernel + streaming kernel per 32 tokens
+    const int chunks = (m + per - 1) / per;
+    info->launches = 2 * chunks;   // fold kernel + streaming kernel per 32 (or 16) tokens
     info->grid_ctas = p.ks * nb * chunks;
   } else if (prefill_group_supported(Ls, n, m)) {   // one launch over every layer's tiles
     const PrefillPlan p = plan_prefill_group(Ls, n, m);
