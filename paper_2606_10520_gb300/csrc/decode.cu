@@ -927,14 +927,17 @@ static size_t fold_workspace_bytes_for(int KT, int max_tok) {
 }
 
 // Tokens per launch pair: 32 (the 96-column accumulator, one CTA per SM)
-// where the row blocks of the call fit one wave of the SMs, else 16 (two CTAs
-// per SM). Measured on GB300 at M = 32: the Llama-2-7B gate/up pair (172 row
-// blocks) takes 35.5 us in one 32-token launch, 32.3 in two 16-token
-// launches; q/k/v (96 row blocks) 19.1 against 24.6.
+// where that takes fewer waves of row blocks than two 16-token launches (two
+// CTAs per SM), else 16. Measured on GB300 at M = 32: Llama-2-7B q/k/v (96
+// row blocks: 1 wave against 2) 19.1 us in one launch, 24.6 in two; the
+// gate/up pair (172: 2 against 2) 35.5 against 32.3; the Llama-2-70B gate/up
+// pair (448: 3 against 4) is faster in one launch.
 int skinny_tokens_per_launch(const unisvq_layer* const* Ls, int n) {
   int nb = 0;
   for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
-  return nb <= Ls[0]->num_sms ? kMaxTokPerLaunch : 16;
+  const int sms = Ls[0]->num_sms > 0 ? Ls[0]->num_sms : 1;
+  const int waves32 = (nb + sms - 1) / sms, waves16 = 2 * ((nb + 2 * sms - 1) / (2 * sms));
+  return waves32 < waves16 ? kMaxTokPerLaunch : 16;
 }
 
 DecodePlan plan_skinny(const unisvq_layer* const* Ls, int n, int M) {

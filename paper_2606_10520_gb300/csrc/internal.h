@@ -96,7 +96,8 @@ unisvq_status launch_gemv_group(const unisvq_layer* const* Ls, int n, const void
                                 cudaStream_t s);
 // tcgen05 skinny GEMM with the codes as 8-bit TMEM operand (decode.cu), M <= 16 per launch.
 // The plan of the call's launch pairs and their tokens per launch (32 where
-// the call's row blocks fit one wave at one CTA per SM, else 16).
+// one 32-token launch at one CTA per SM takes fewer waves of the call's row
+// blocks than two 16-token launches at two per SM, else 16).
 DecodePlan plan_skinny(const unisvq_layer* const* Ls, int n, int M);
 int skinny_tokens_per_launch(const unisvq_layer* const* Ls, int n);
 unisvq_status launch_skinny(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s);

@@ -361,8 +361,9 @@ def test_dispatch_picks_tcgen05_decode_for_large_launches():
     """The library's pick (unisvq_query / unisvq_query_group): the tcgen05
     skinny path (fold + streaming kernel: two launches) from 2^26 weights per
     launch, or from 2^25 weights over >= 64 row blocks or above 16 tokens; the
-    GEMV otherwise. A launch pair takes 32 tokens where the row blocks fit one
-    wave at one CTA per SM, else 16."""
+    GEMV otherwise. A launch pair takes 32 tokens where that needs fewer waves
+    of row blocks (one CTA per SM) than two 16-token pairs (two per SM), else
+    16."""
     big = binding.UniSVQLinear(*synth.layer_inputs(9, 91, 0, 0, 16384, 4096, 2))
     q = big.query(1)
     assert q["kernel"] == binding.KERNEL_SKINNY and q["launches"] == 2
@@ -373,7 +374,7 @@ def test_dispatch_picks_tcgen05_decode_for_large_launches():
     assert tall.query(1)["kernel"] == binding.KERNEL_GEMV and tall.query(16)["kernel"] == binding.KERNEL_GEMV
     assert tall.query(32)["kernel"] == binding.KERNEL_SKINNY and tall.query(32)["launches"] == 2
     wide = binding.UniSVQLinear(*synth.layer_inputs(9, 91, 3, 0, 11008, 4096, 2))
-    pair = [wide, wide.clone()]                                     # 172 row blocks: 16 tokens per pair
+    pair = [wide, wide.clone()]            # 172 row blocks: 2 waves either way, so 16 tokens per pair
     assert binding.query_group(pair, 17)["launches"] == 4 and binding.query_group(pair, 32)["launches"] == 4
     xw = synth.activations(9, 91, 5, 20, 4096)
     cw, Aw, Bw = synth.layer_inputs(9, 91, 3, 0, 11008, 4096, 2)
