@@ -296,6 +296,18 @@ unisvq_status unisvq_hadamard(const void* x, void* y, int M, int n, const uint8_
  * same code-extraction helpers the layer kernels use. */
 unisvq_status unisvq_dequant_debug(unisvq_handle h, float* W, void* stream);
 
+/* Test hook for the unwind path of the kernels' bounded waits (every wait on
+ * the device gives up after 2 s, records a code in the library's error word
+ * and unwinds). One CTA allocates tensor memory, starts a 16-byte bulk copy
+ * from src16 (device, 16-byte aligned) into shared memory and waits on an
+ * mbarrier that nothing arrives at; after 2 s that wait records a timeout,
+ * the CTA waits for its own copy, frees the tensor memory and returns.
+ * out3 (device, 3 ints) receives: whether the first wait succeeded (0), whether
+ * the copy landed (1), and the copy's first byte. unisvq_sync_status on the
+ * stream then returns UNISVQ_ERR_TIMEOUT (and clears the error word); the
+ * context stays usable. Errors: INVALID_ARG, CUDA. */
+unisvq_status unisvq_debug_wait_timeout(const void* src16, int* out3, void* stream);
+
 /* Describe the launch unisvq_linear would make for M tokens (host only). */
 unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info);
 

@@ -24,7 +24,7 @@ EXPORTS = [
     "unisvq_status_string", "unisvq_packed_code_bytes", "unisvq_pack_host", "unisvq_version",
     "unisvq_linear_group", "unisvq_linear_group_force", "unisvq_linear_noalloc", "unisvq_query_group",
     "unisvq_pack_grouped", "unisvq_set_rht", "unisvq_hadamard", "unisvq_pack_bits",
-    "unisvq_prefill_table_host",
+    "unisvq_prefill_table_host", "unisvq_debug_wait_timeout",
 ]
 MAX_GROUP = 4
 
@@ -66,6 +66,7 @@ def load():
     lib.unisvq_linear_group_force.argtypes = [vp, i, i, vp, vp, i, vp]
     lib.unisvq_linear_noalloc.argtypes = [vp, vp, vp, i, vp]
     lib.unisvq_dequant_debug.argtypes = [vp, vp, vp]
+    lib.unisvq_debug_wait_timeout.argtypes = [vp, vp, vp]
     lib.unisvq_query.argtypes = [vp, i, ctypes.POINTER(Info)]
     lib.unisvq_query_group.argtypes = [vp, i, i, ctypes.POINTER(Info)]
     lib.unisvq_sync_status.argtypes = [vp]
@@ -147,6 +148,12 @@ def hadamard_ptr(x_ptr: int, y_ptr: int, M: int, n: int, signs_ptr: int, signs_f
 
 def sync_status(stream=None) -> int:
     return int(load().unisvq_sync_status(_stream_ptr(stream)))
+
+
+def wait_timeout_probe_ptr(src16_ptr: int, out3_ptr: int, stream=None) -> int:
+    """unisvq_debug_wait_timeout: a bounded device wait that runs out (test hook)."""
+    return int(load().unisvq_debug_wait_timeout(ctypes.c_void_p(src16_ptr), ctypes.c_void_p(out3_ptr),
+                                                 _stream_ptr(stream)))
 
 
 class UniSVQLinear:

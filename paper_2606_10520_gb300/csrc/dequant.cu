@@ -87,6 +87,47 @@ __global__ void __launch_bounds__(256) dequant_grouped_kernel(const uint8_t* __r
   W[id] = static_cast<float>(w);
 }
 
+// Test hook for the unwind path of a bounded wait: one CTA allocates 32
+// TMEM columns, starts a bulk copy of `src` (16 bytes) into shared memory
+// counted on one mbarrier, and waits on a second mbarrier that nothing
+// arrives at. That wait runs out after the library's limit and records
+// kErrTimeoutFull; the CTA then waits (bounded) for its own copy, frees TMEM
+// and returns, the steps every kernel of the library takes when a wait runs
+// out.
+__global__ void __launch_bounds__(32) wait_probe_kernel(const uint8_t* src, int* err, int* out) {
+  __shared__ __align__(16) uint8_t buf[16];
+  __shared__ __align__(8) uint64_t bars[2];
+  __shared__ uint32_t tmem_slot;
+  const uint32_t copy_bar = smem_u32(&bars[0]), never = smem_u32(&bars[1]);
+  if (threadIdx.x == 0) {
+    mbar_init(copy_bar, 1);
+    mbar_init(never, 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 32;" ::"r"(smem_u32(&tmem_slot))
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncwarp();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t taddr = tmem_slot;
+  int waited = 0, copied = 0;
+  if (threadIdx.x == 0) {
+    mbar_arrive_expect_tx(copy_bar, 16);
+    bulk_g2s(smem_u32(buf), src, 16, copy_bar, policy_evict_first());
+    waited = mbar_wait(never, 0, err, kErrTimeoutFull) ? 1 : 0;    // runs out: nothing arrives
+    copied = mbar_wait(copy_bar, 0, err, kErrTimeoutFull) ? 1 : 0;  // the own copy still lands
+    out[0] = waited;
+    out[1] = copied;
+    out[2] = copied ? static_cast<int>(buf[0]) : -1;
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncwarp();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 32;" ::"r"(taddr) : "memory");
+}
+
 }  // namespace
 
 unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s) {
@@ -99,6 +140,11 @@ unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s) {
   const int nchunks = (L->Np / kTileRows) * L->KT * 256;
   dequant_kernel<<<(nchunks + 255) / 256, 256, 0, s>>>(L->codes, L->hi, L->lut32, W, L->N, L->K, L->KT, L->d,
                                                        L->bits, nchunks);
+  return cudaGetLastError() == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+}
+
+unisvq_status launch_wait_probe(const void* src16, int* out3, cudaStream_t s) {
+  wait_probe_kernel<<<1, 32, 0, s>>>(static_cast<const uint8_t*>(src16), device_error_word(), out3);
   return cudaGetLastError() == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 

@@ -140,6 +140,9 @@ unisvq_status launch_prefill_group(const unisvq_layer* const* Ls, int n, const v
                                    cudaStream_t s);
 
 unisvq_status launch_dequant(const unisvq_layer* L, float* W, cudaStream_t s);
+// The bounded-wait test hook (dequant.cu): src16 device, 16 bytes, 16-byte
+// aligned; out3 device, three ints.
+unisvq_status launch_wait_probe(const void* src16, int* out3, cudaStream_t s);
 
 // Randomized Hadamard transform of M rows of n bf16 values (rht.cu):
 // signs_first = 1: out = (s x) H / sqrt(n); 0: out = s ((x H) / sqrt(n)).

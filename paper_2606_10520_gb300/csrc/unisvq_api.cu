@@ -781,6 +781,11 @@ unisvq_status unisvq_linear_group(const unisvq_handle* hs, int n, const void* x,
   return unisvq_linear_group_force(hs, n, UNISVQ_KERNEL_AUTO, x, ys, M, stream);
 }
 
+unisvq_status unisvq_debug_wait_timeout(const void* src16, int* out3, void* stream) {
+  if (!src16 || !out3 || !aligned(src16, 16) || !aligned(out3, 4)) return UNISVQ_ERR_INVALID_ARG;
+  return launch_wait_probe(src16, out3, static_cast<cudaStream_t>(stream));
+}
+
 unisvq_status unisvq_dequant_debug(unisvq_handle h, float* W, void* stream) {
   if (!h || !W || !aligned(W, 4)) return UNISVQ_ERR_INVALID_ARG;
   return launch_dequant(h, W, static_cast<cudaStream_t>(stream));
