@@ -855,9 +855,9 @@ def run_prefill(torch, binding, peaks, args, stream):
     td = time_graphs(torch, [gd], reps, 3, stream)
     for l in layers:
         l.close()
-    # the same set with one affine map per (row, 128-column group), d = 2 and d = 4
+    # the same set with one affine map per (row, 128-column group), d = 1, 2 and 4
     per_group = {}
-    for dg in (2, 4):
+    for dg in (1, 2, 4):
         glayers = []
         for pi, (_, N, K) in enumerate(shapes):
             codes, A, B = synth.layer_inputs_grouped(0, 2, 0, pi, N, K, dg)
@@ -898,6 +898,7 @@ def run_prefill(torch, binding, peaks, args, stream):
             "per_group_maps_TFLOP/s": flops * reps / per_group[2] / 1e12,
             "per_group_maps_group_calls_TFLOP/s": flops * reps / per_group["calls"] / 1e12,
             "per_group_maps_d4_TFLOP/s": flops * reps / per_group[4] / 1e12,
+            "per_group_maps_d1_TFLOP/s": flops * reps / per_group[1] / 1e12,
             "bits3_TFLOP/s": flops * reps / t3 / 1e12,
             "bits3_d4_TFLOP/s": flops * reps / t34 / 1e12,
             "d8_TFLOP/s": flops * reps / t8 / 1e12,

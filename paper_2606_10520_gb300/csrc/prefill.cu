@@ -180,6 +180,9 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
 __device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
+__device__ __forceinline__ void sts64(uint32_t addr, uint32_t a, uint32_t b) {
+  asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
+}
 __device__ __forceinline__ uint32_t lds32(uint32_t addr) {
   uint32_t v;
   asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(addr));
@@ -417,6 +420,85 @@ __global__ void __launch_bounds__(kPfThreads, 1)
                   o[2 * vv + 1] = pack_bf16x2(w[2], w[3]);
                 }
                 sts128(row_addr + ((cc ^ g) << 4), o[0], o[1], o[2], o[3]);
+              }
+            }
+            fence_proxy_async_smem();
+          }
+          __syncwarp();
+          if (lane == 0 && ok) mbar_arrive(afull(s));
+        }
+      }
+    } else if (a.meta[0] && a.d == 1) {
+      // Per-(row, 128-column group) maps, d = 1, codes permuted within each group
+      // (pack_codes_grouped_host): packed position (h, t, s, b) holds group
+      // column 64 h + 16 s + 4 t + e(b). So stage half h needs the words of half
+      // h only, and lane t's word of a row gives, for each s, the natural
+      // columns 16 s + 4 t + j (j = e(b); e swaps b = 1 and 2) of the stage:
+      // 8 bytes of the 16-byte chunk 2 s + t/2. Per k-tile the warp builds, for
+      // each of its 16 rows, the 16 bf16 pairs (a z0 + b, a z1 + b) of the
+      // row's map (four entries per lane and row); the columns j, j + 1 (bytes
+      // e(j), e(j + 1)) index it.
+      const uint32_t tab_s = sbase + C::kOffGrp + c * 1024;   // [16 rows][16 entries] bf16x2
+      for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
+        const int li = tile_layer(a, tile);
+        const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
+        const uint8_t* rbase =
+            pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
+        const uint16_t* mbase = pick_layer(a.meta, li) + static_cast<size_t>(n_blk) * a.KT * kBM * 2;
+        const int nkt = (a.nkb + 1) >> 1;
+        auto load_codes = [&](int kt) -> uint4 {
+          return kt < nkt ? __ldg(reinterpret_cast<const uint4*>(rbase + static_cast<size_t>(kt) * kTileBytes))
+                          : make_uint4(0, 0, 0, 0);
+        };
+        // a row's map (a, b) as one word
+        auto load_map = [&](int kt, int row) -> uint32_t {
+          return kt < nkt ? __ldg(reinterpret_cast<const uint32_t*>(mbase + (static_cast<size_t>(kt) * kBM + row) * 2))
+                          : 0u;
+        };
+        uint4 cn = load_codes(0), cur = cn;
+        uint32_t mn0 = load_map(0, r0), mn1 = load_map(0, r1);
+        bool ok = !*abort_flag;
+        for (int kb = 0; kb < a.nkb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const int hs = kb & 1;
+          if (hs == 0) {
+            cur = cn;
+            const uint32_t m0 = mn0, m1 = mn1;
+            cn = load_codes((kb >> 1) + 1);
+            mn0 = load_map((kb >> 1) + 1, r0);
+            mn1 = load_map((kb >> 1) + 1, r1);
+            __syncwarp();   // every lane is done with the previous group's table
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const uint32_t m = q ? m1 : m0;
+              const float am = f16_lo(m), bm = f16_hi(m);
+              const int rr = g + 8 * q;
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const int idx = 4 * t + k;
+                const float z0 = static_cast<float>(idx & 3), z1 = static_cast<float>(idx >> 2);
+                sts32(tab_s + (rr * 16 + idx) * 4, pack_bf16x2(fmaf(am, z0, bm), fmaf(am, z1, bm)));
+              }
+            }
+            __syncwarp();
+          }
+          if (ok && it >= STAGES) {
+            ok = !*abort_flag && mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty);
+            if (!ok) *abort_flag = 1;
+          }
+          if (ok) {
+            const uint32_t tile_addr = sbase + C::kOffA + s * kATileBytes;
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const uint32_t w = hs ? (q ? cur.w : cur.z) : (q ? cur.y : cur.x);   // half hs of the row
+              const uint32_t row_addr = tile_addr + (q ? r1 : r0) * 128;
+              const uint32_t trow = tab_s + (g + 8 * q) * 64;
+#pragma unroll
+              for (int sq = 0; sq < 4; ++sq) {
+                const uint32_t i0 = ((w >> (2 * sq)) & 3u) | (((w >> (16 + 2 * sq)) & 3u) << 2);       // columns j = 0, 1
+                const uint32_t i1 = ((w >> (8 + 2 * sq)) & 3u) | (((w >> (24 + 2 * sq)) & 3u) << 2);  // j = 2, 3
+                const int cc = 2 * sq + (t >> 1);
+                sts64(row_addr + ((cc ^ g) << 4) + ((t & 1) << 3), lds32(trow + i0 * 4), lds32(trow + i1 * 4));
               }
             }
             fence_proxy_async_smem();
@@ -766,11 +848,11 @@ int pick_bn(int M) { return M <= 64 ? 64 : (M <= 128 ? 128 : 256); }
 }  // namespace
 
 bool prefill_supported(const unisvq_layer* L, int M) {
-  // per-group layers: d = 2 (a 16-pair table per row and group) or d = 4 (direct
-  // sums); 3-bit layers: d <= 4 (a 64-pair codeword table for d <= 2, two
+  // per-group layers: d = 1 or 2 (a 16-pair table per row and group) or d = 4
+  // (direct sums); 3-bit layers: d <= 4 (a 64-pair codeword table for d <= 2, two
   // 64-row pair tables for d = 4); per-matrix 2-bit layers: every d (d = 8
   // through two quad tables)
-  const bool maps_ok = L->grouped ? (L->d == 2 || L->d == 4) : (L->bits == 3 ? L->d <= 4 : true);
+  const bool maps_ok = L->grouped ? (L->d <= 4) : (L->bits == 3 ? L->d <= 4 : true);
   return M > 0 && maps_ok && (L->K % 8) == 0 && get_encode() != nullptr;
 }
 

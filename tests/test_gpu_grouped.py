@@ -177,11 +177,12 @@ def test_grouped_entry_points():
         h.close()
 
 
-@pytest.mark.parametrize("d", [2, 4])
+@pytest.mark.parametrize("d", [1, 2, 4])
 @pytest.mark.parametrize("N,K", [(256, 1024), (520, 1000), (1000, 2048), (384, 640)])
 def test_grouped_prefill_parity(N, K, d):
-    """d = 2 and d = 4 per-group layers run the tcgen05 prefill GEMM above 64
-    tokens (d = 2: per-(row, group) codeword tables; d = 4: direct sums)."""
+    """d = 1, 2 and 4 per-group layers run the tcgen05 prefill GEMM above 64
+    tokens (d = 1, 2: per-(row, group) codeword-pair tables; d = 4: direct
+    sums)."""
     codes, A, B, layer = make(N, K, d, seed=7)
     assert layer.query(65)["kernel"] == binding.KERNEL_PREFILL
     assert layer.query(64)["kernel"] == binding.KERNEL_GROUPED
@@ -199,7 +200,7 @@ def test_grouped_prefill_parity(N, K, d):
     layer.close()
 
 
-@pytest.mark.parametrize("d", [2, 4])
+@pytest.mark.parametrize("d", [1, 2, 4])
 def test_grouped_prefill_integer_case_bit_exact(d):
     g = np.random.default_rng(77 + d)
     N, K = 256, 640
@@ -216,8 +217,8 @@ def test_grouped_prefill_integer_case_bit_exact(d):
     layer.close()
 
 
-@pytest.mark.parametrize("d", [1, 8])
-def test_grouped_prefill_only_for_d2_and_d4(d):
+@pytest.mark.parametrize("d", [8])
+def test_grouped_prefill_not_for_d8(d):
     codes, A, B, layer = make(256, 512, d, seed=8)
     assert layer.query(200)["kernel"] == binding.KERNEL_GROUPED
     x = torch.zeros((100, 512), dtype=torch.bfloat16, device="cuda")
@@ -229,7 +230,7 @@ def test_grouped_prefill_only_for_d2_and_d4(d):
     layer.close()
 
 
-@pytest.mark.parametrize("d", [2, 4])
+@pytest.mark.parametrize("d", [1, 2, 4])
 def test_grouped_group_call_at_prefill_sizes(d):
     """Per-group layers that share x run one persistent prefill launch (each
     converter reading its tile's layer's maps): bit-identical to per-layer
