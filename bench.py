@@ -855,14 +855,19 @@ def run_prefill(torch, binding, peaks, args, stream):
     td = time_graphs(torch, [gd], reps, 3, stream)
     for l in layers:
         l.close()
-    # the same set with one affine map per (row, 128-column group), d = 1, 2 and 4
+    # the same set with one affine map per (row, 128-column group), d = 1, 2, 4 and 8
+    # (d = 8: without down, whose 4096 x 14336 maps do not fit the per-group
+    # GEMV's shared memory, so that it does not pack)
     per_group = {}
-    for dg in (1, 2, 4):
+    shapes_d8 = [sh for sh in shapes if sh[2] <= 4096]
+    flops_d8 = sum(2.0 * M * N * K for _, N, K in shapes_d8)
+    for dg in (1, 2, 4, 8):
+        sset = shapes_d8 if dg == 8 else shapes
         glayers = []
-        for pi, (_, N, K) in enumerate(shapes):
+        for pi, (_, N, K) in enumerate(sset):
             codes, A, B = synth.layer_inputs_grouped(0, 2, 0, pi, N, K, dg)
             glayers.append(b.UniSVQLinear(codes, A, B, group_cols=128))
-        per_group[dg] = time_prefill_layers(torch, b, shapes, glayers, xs, ys, M, reps, stream)
+        per_group[dg] = time_prefill_layers(torch, b, sset, glayers, xs, ys, M, reps, stream)
         if dg == 2:
             per_group["calls"] = time_prefill_groups(torch, b, shapes, glayers, xs, M, reps, stream)
         for l in glayers:
@@ -899,6 +904,7 @@ def run_prefill(torch, binding, peaks, args, stream):
             "per_group_maps_group_calls_TFLOP/s": flops * reps / per_group["calls"] / 1e12,
             "per_group_maps_d4_TFLOP/s": flops * reps / per_group[4] / 1e12,
             "per_group_maps_d1_TFLOP/s": flops * reps / per_group[1] / 1e12,
+            "per_group_maps_d8_without_down_TFLOP/s": flops_d8 * reps / per_group[8] / 1e12,
             "bits3_TFLOP/s": flops * reps / t3 / 1e12,
             "bits3_d4_TFLOP/s": flops * reps / t34 / 1e12,
             "d8_TFLOP/s": flops * reps / t8 / 1e12,

@@ -89,7 +89,7 @@ struct PfCfg {
   static constexpr int kOffB = STAGES * kATileBytes;
   static constexpr int kOffLut = STAGES * kStageBytes;            // 2 KB (d = 8: the 16 KB region)
   static constexpr int kOffGrp = kOffLut + 2048;                   // 8 x 1 KB: per-group tables
-  static constexpr int kOffBars = kOffLut + 16 * 1024;
+  static constexpr int kOffBars = kOffLut + 20 * 1024;            // per-group d = 8: 8 x 2304 B of maps
   // bars: bfull[S], afull[S], empty[S], accfull[2], accempty[2]
   static constexpr int kOffTmemPtr = kOffBars + (3 * STAGES + 5) * 8;   // + drain barrier
   static constexpr int kOffFlag = kOffTmemPtr + 8;
@@ -328,7 +328,115 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     const int r0 = 16 * c + g, r1 = r0 + 8;
     const uint32_t lut_base = sbase + C::kOffLut;   // layer i's table at + 2 KB i
     int it = 0;
-    if (a.meta[0] && a.d == 4) {
+    if (a.meta[0] && a.d == 8) {
+      // Per-(row, 128-column group) maps, d = 8, codes permuted within each group
+      // (pack_codes_grouped_host): packed position (h, t, s, b) holds coordinate
+      // 4 h + s of vector v = 4 t + e(b), natural columns 8 v .. 8 v + 7. So a
+      // lane's 16-byte load holds every coordinate of four vectors of rows g and
+      // g + 8, all in stage half t / 2. Lanes t and t ^ 2 share the work: in
+      // stage half hs the lane with t / 2 == hs forms the vectors of bytes
+      // b = 0, 1 from its own words, its partner those of b = 2, 3 from the
+      // same words (one shuffle per word and k-tile). Each output is
+      // sum_c' A[c][c'] z_c' + B[c] in fp32 (one 16-byte store per vector); the
+      // warp stages its 16 rows' maps (72 fp16 each) in shared memory per k-tile.
+      const uint32_t map_s = sbase + C::kOffLut + c * 2304;   // [16 rows][72] fp16
+      for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
+        const int li = tile_layer(a, tile);
+        const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
+        const uint8_t* rbase =
+            pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
+        const uint32_t* mbase = reinterpret_cast<const uint32_t*>(pick_layer(a.meta, li) +
+                                                                  static_cast<size_t>(n_blk) * a.KT * kBM * 72 +
+                                                                  static_cast<size_t>(16 * c) * 72);
+        const int nkt = (a.nkb + 1) >> 1;
+        auto load_codes = [&](int kt) -> uint4 {
+          return kt < nkt ? __ldg(reinterpret_cast<const uint4*>(rbase + static_cast<size_t>(kt) * kTileBytes))
+                          : make_uint4(0, 0, 0, 0);
+        };
+        // this lane's 18 of the 576 words of the warp's 16 row maps of group kt
+        auto load_maps = [&](int kt, uint32_t (&w)[18]) {
+#pragma unroll
+          for (int i = 0; i < 18; ++i)
+            w[i] = kt < nkt ? __ldg(mbase + static_cast<size_t>(kt) * kBM * 36 + lane + 32 * i) : 0u;
+        };
+        uint4 cn = load_codes(0), own = cn, par = cn;
+        uint32_t mw[18];
+        load_maps(0, mw);
+        bool ok = !*abort_flag;
+        for (int kb = 0; kb < a.nkb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const int hs = kb & 1;
+          if (hs == 0) {
+            own = cn;
+            par.x = __shfl_xor_sync(0xffffffffu, own.x, 2);
+            par.y = __shfl_xor_sync(0xffffffffu, own.y, 2);
+            par.z = __shfl_xor_sync(0xffffffffu, own.z, 2);
+            par.w = __shfl_xor_sync(0xffffffffu, own.w, 2);
+            __syncwarp();   // every lane is done with the previous group's maps
+#pragma unroll
+            for (int i = 0; i < 18; ++i) sts32(map_s + (lane + 32 * i) * 4, mw[i]);
+            __syncwarp();
+            cn = load_codes((kb >> 1) + 1);
+            load_maps((kb >> 1) + 1, mw);
+          }
+          if (ok && it >= STAGES) {
+            ok = !*abort_flag && mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty);
+            if (!ok) *abort_flag = 1;
+          }
+          if (ok) {
+            const uint32_t tile_addr = sbase + C::kOffA + s * kATileBytes;
+            const bool mine = (t >> 1) == hs;                    // own words, bytes 0, 1; else the partner's, 2, 3
+            const int tq = mine ? t : (t ^ 2);                   // the quarter whose vectors this lane forms
+            const uint4 src = mine ? own : par;
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const uint32_t wh[2] = {q ? src.y : src.x, q ? src.w : src.z};   // halves 0 and 1 of the row
+              const uint32_t row_addr = tile_addr + (q ? r1 : r0) * 128;
+              const uint32_t rec = map_s + (g + 8 * q) * 144;
+              float z[2][8];
+#pragma unroll
+              for (int jb = 0; jb < 2; ++jb) {
+                const int bb = mine ? jb : 2 + jb;
+#pragma unroll
+                for (int cc2 = 0; cc2 < 8; ++cc2)
+                  z[jb][cc2] = static_cast<float>((wh[cc2 >> 2] >> (8 * bb + 2 * (cc2 & 3))) & 3u);
+              }
+              float w[2][8];
+#pragma unroll
+              for (int cr = 0; cr < 8; ++cr) {
+                const uint32_t bw = lds32(rec + 128 + 4 * (cr >> 1));
+                const float bc = (cr & 1) ? f16_hi(bw) : f16_lo(bw);
+                float ar[8];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                  const uint32_t aw = lds32(rec + 16 * cr + 4 * i);
+                  ar[2 * i] = f16_lo(aw);
+                  ar[2 * i + 1] = f16_hi(aw);
+                }
+#pragma unroll
+                for (int jb = 0; jb < 2; ++jb) {
+                  float acc = bc;
+#pragma unroll
+                  for (int c2 = 0; c2 < 8; ++c2) acc = fmaf(ar[c2], z[jb][c2], acc);
+                  w[jb][cr] = acc;
+                }
+              }
+#pragma unroll
+              for (int jb = 0; jb < 2; ++jb) {
+                const int bb = mine ? jb : 2 + jb;
+                const int ev = (bb >> 1) | ((bb & 1) << 1);     // vector 4 tq + e(b): chunk 4 (tq & 1) + e(b)
+                const int cc = 4 * (tq & 1) + ev;
+                sts128(row_addr + ((cc ^ g) << 4), pack_bf16x2(w[jb][0], w[jb][1]), pack_bf16x2(w[jb][2], w[jb][3]),
+                       pack_bf16x2(w[jb][4], w[jb][5]), pack_bf16x2(w[jb][6], w[jb][7]));
+              }
+            }
+            fence_proxy_async_smem();
+          }
+          __syncwarp();
+          if (lane == 0 && ok) mbar_arrive(afull(s));
+        }
+      }
+    } else if (a.meta[0] && a.d == 4) {
       // Per-(row, 128-column group) maps, d = 4: 256 codewords per row and group
       // are too many to tabulate per k-tile, so each output is formed directly,
       // sum_c' A[c][c'] z_c' + B[c] in fp32. Natural columns 64 h + 8 cc + j
@@ -849,10 +957,10 @@ int pick_bn(int M) { return M <= 64 ? 64 : (M <= 128 ? 128 : 256); }
 
 bool prefill_supported(const unisvq_layer* L, int M) {
   // per-group layers: d = 1 or 2 (a 16-pair table per row and group) or d = 4
-  // (direct sums); 3-bit layers: d <= 4 (a 64-pair codeword table for d <= 2, two
+  // and 8 (direct sums); 3-bit layers: d <= 4 (a 64-pair codeword table for d <= 2, two
   // 64-row pair tables for d = 4); per-matrix 2-bit layers: every d (d = 8
   // through two quad tables)
-  const bool maps_ok = L->grouped ? (L->d <= 4) : (L->bits == 3 ? L->d <= 4 : true);
+  const bool maps_ok = L->grouped ? true : (L->bits == 3 ? L->d <= 4 : true);
   return M > 0 && maps_ok && (L->K % 8) == 0 && get_encode() != nullptr;
 }
 

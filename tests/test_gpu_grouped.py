@@ -177,12 +177,11 @@ def test_grouped_entry_points():
         h.close()
 
 
-@pytest.mark.parametrize("d", [1, 2, 4])
+@pytest.mark.parametrize("d", [1, 2, 4, 8])
 @pytest.mark.parametrize("N,K", [(256, 1024), (520, 1000), (1000, 2048), (384, 640)])
 def test_grouped_prefill_parity(N, K, d):
-    """d = 1, 2 and 4 per-group layers run the tcgen05 prefill GEMM above 64
-    tokens (d = 1, 2: per-(row, group) codeword-pair tables; d = 4: direct
-    sums)."""
+    """Per-group layers run the tcgen05 prefill GEMM above 64 tokens (d = 1, 2:
+    per-(row, group) codeword-pair tables; d = 4, 8: direct sums)."""
     codes, A, B, layer = make(N, K, d, seed=7)
     assert layer.query(65)["kernel"] == binding.KERNEL_PREFILL
     assert layer.query(64)["kernel"] == binding.KERNEL_GROUPED
@@ -200,7 +199,7 @@ def test_grouped_prefill_parity(N, K, d):
     layer.close()
 
 
-@pytest.mark.parametrize("d", [1, 2, 4])
+@pytest.mark.parametrize("d", [1, 2, 4, 8])
 def test_grouped_prefill_integer_case_bit_exact(d):
     g = np.random.default_rng(77 + d)
     N, K = 256, 640
@@ -217,17 +216,23 @@ def test_grouped_prefill_integer_case_bit_exact(d):
     layer.close()
 
 
-@pytest.mark.parametrize("d", [8])
-def test_grouped_prefill_not_for_d8(d):
-    codes, A, B, layer = make(256, 512, d, seed=8)
-    assert layer.query(200)["kernel"] == binding.KERNEL_GROUPED
-    x = torch.zeros((100, 512), dtype=torch.bfloat16, device="cuda")
-    y = torch.zeros((100, 256), dtype=torch.bfloat16, device="cuda")
-    stream = torch.cuda.current_stream().cuda_stream
-    assert layer.forward_ptr(x.data_ptr(), y.data_ptr(), 100, stream, binding.KERNEL_PREFILL) == binding.ERR_UNSUPPORTED
-    xb = synth.activations(8, 40, d, 100, 512)
-    check(run(layer, xb), xb, codes, A, B)
-    layer.close()
+def test_grouped_d8_group_call_runs_one_prefill_launch_per_layer():
+    """d = 8 per-group layers run the prefill GEMM, but a group call of them
+    takes one launch per layer (their maps fill the converters' shared
+    memory); the outputs meet the oracle."""
+    K = 512
+    made = [synth.layer_inputs_grouped(8, 41, i, 0, N, K, 8) for i, N in enumerate((256, 128))]
+    layers = [binding.UniSVQLinear(c, A, B, group_cols=GC) for c, A, B in made]
+    assert layers[0].query(200)["kernel"] == binding.KERNEL_PREFILL
+    q = binding.query_group(layers, 200)
+    assert q["kernel"] == binding.KERNEL_PREFILL and q["launches"] == 2
+    xb = synth.activations(8, 41, 200, 200, K)
+    ys = binding.linear_group(layers, to_dev(xb))
+    assert binding.sync_status() == binding.OK
+    for (c, A, B), y in zip(made, ys):
+        check(y.float().cpu().numpy().astype(np.float64), xb, c, A, B)
+    for l in layers:
+        l.close()
 
 
 @pytest.mark.parametrize("d", [1, 2, 4])
