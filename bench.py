@@ -613,7 +613,9 @@ def run_ours(args, rank, world, local_rank):
 def sweep_variant(torch, binding, args, stream, base, kernel_id):
     """The Llama-2-7B decode sweep (GROUPED_LAYERS layers: `base` and device
     copies) for one layer variant; returns (GB/s over the sweep, per-M list,
-    launches per step). Bytes are the library's algorithmic bytes per call."""
+    launches per step). Bytes are the library's algorithmic bytes per call.
+    kernel_id: the kernel every call must resolve to, or None for the
+    library's own pick (then reported per M and call)."""
     shapes = synth.LLAMA2_7B
     nl = variant_layers(args)
     stack = [base] + [[b.clone() for b in base] for _ in range(nl - 1)]
@@ -624,7 +626,7 @@ def sweep_variant(torch, binding, args, stream, base, kernel_id):
                 xb = synth.activations(0, 1, 100 + M, M, K)
                 xs[(M, K)] = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).cuda()
             ys[(M, pi)] = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
-    graphs, sweep_bytes, launches = [], [], 0
+    graphs, sweep_bytes, launches, kernels = [], [], 0, []
     for M in M_SWEEP:
         def one_pass(M=M):
             sp = torch.cuda.current_stream().cuda_stream
@@ -643,22 +645,25 @@ def sweep_variant(torch, binding, args, stream, base, kernel_id):
             one_pass()
         graphs.append(g)
         nbytes = 0
+        kern_m = {}
         for grp in GROUPS_7B:
             info = binding.query_group([base[i] for i in grp], M)
-            assert info["kernel"] == kernel_id
+            assert kernel_id is None or info["kernel"] == kernel_id
+            kern_m["+".join(shapes[i][0] for i in grp)] = KERNEL_NAMES.get(info["kernel"], "?")
             nbytes += info["algo_bytes"] * nl
             launches += info["launches"] * nl
         sweep_bytes.append(nbytes)
+        kernels.append(kern_m)
     st = binding.sync_status(stream)
     if st != 0:
         raise RuntimeError(f"device status {binding.status_string(st)}")
     steps = max(5, args.steps // 4)
     t = time_graphs(torch, graphs, steps, args.warmup, stream)
     per_m = []
-    for M, g, nb in zip(M_SWEEP, graphs, sweep_bytes):
+    for M, g, nb, km in zip(M_SWEEP, graphs, sweep_bytes, kernels):
         tm = time_graphs(torch, [g], steps, 2, stream)
         per_m.append({"M": M, "GB/s": round(nb * steps / tm / 1e9, 1),
-                      "us_per_layer": round(tm / steps / nl * 1e6, 3)})
+                      "us_per_layer": round(tm / steps / nl * 1e6, 3), "kernels": km})
     for layer in stack:
         for b in layer:
             b.close()
@@ -684,16 +689,19 @@ def run_grouped(torch, binding, peaks, args, stream):
 
 def run_bits3(torch, binding, peaks, args, stream):
     """The decode sweep on Llama-2-7B-shaped layers with 3-bit codes (z in
-    0..7, Sec. 5.2): the GEMV with the high-bit plane (gemv_kernel, BITS = 3)."""
+    0..7, Sec. 5.2) through the library's own pick: the tcgen05 decode path
+    (decode_kernel, 3-bit instance) for q/k/v and gate/up, the GEMV with the
+    high-bit plane (gemv_kernel, BITS = 3) for o and down."""
     base = []
     for pi, (_, N, K) in enumerate(synth.LLAMA2_7B):
         codes, A, B = synth.layer_inputs_bits(0, 1, 0, pi, N, K, 2, 3)
         base.append(binding.UniSVQLinear(codes, A, B, bits=3))
-    gbs, per_m, launches = sweep_variant(torch, binding, args, stream, base, binding.KERNEL_GEMV)
+    gbs, per_m, launches = sweep_variant(torch, binding, args, stream, base, None)
     return {"workload": f"Llama-2-7B-shaped projection set x {variant_layers(args)} layers, decode sweep M in "
                         f"{list(M_SWEEP)}, 3-bit codes d=2, per-matrix fp16 affine",
             "GB/s": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"], "sweep": per_m,
-            "kernel": "gemv_kernel (3-bit instance)", "launches_per_step": launches,
+            "kernel": "decode_kernel / gemv_kernel (3-bit instances), per call as listed in sweep",
+            "launches_per_step": launches,
             "bytes": "codes 3*N*K/8 + affine + x + y per call",
             "timing": "CUDA graphs of the layer stack per M, CUDA events on the capture stream"}
 

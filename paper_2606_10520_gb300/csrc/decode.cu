@@ -71,6 +71,7 @@ constexpr int kWsTileStride = 96 * 128;             // B tile bytes per k-tile a
 
 struct SkLayer {
   const uint8_t* codes;
+  const uint8_t* hi;   // 3-bit codes: the high-bit plane (2048 bytes per tile), else null
   const uint8_t* ws;   // fold workspace (B tiles at kWsTableBytes)
   uint16_t* y;         // bf16 [M][N]
   int N;
@@ -92,6 +93,7 @@ template <int DV>
 struct FoldLayer {
   uint8_t* ws;
   int d;
+  int odd_exp;         // exponent of the B columns of odd s: -2 (2-bit codes, bytes 4 z), 0 (3-bit, bytes z)
   float colnorm;       // max_c sum_r |A[r][c]|
   float A[DV * DV];    // row-major d x d (d <= DV)
   float B[DV];
@@ -120,11 +122,12 @@ struct FoldArgs {
 // CTAs per SM.
 // (One-tile stages for N = 48 would leave room for two A slots only; measured
 // slower than two-tile stages on every Llama shape.)
-template <int NCOL, int T>
+template <int NCOL, int T, int BITS = 2>
 struct Cfg {
   static constexpr int kT = T;
   static constexpr int kMinBlocks = T == 1 ? 3 : (NCOL > 64 ? 1 : 2);
   static constexpr int kCodeBytes = T * kTileBytes;
+  static constexpr int kHiBytes = BITS == 3 ? T * (kTileBytes / 2) : 0;   // the stage's high-bit plane
   static constexpr int kAColBase = T == 1 ? 32 : (NCOL > 64 ? 128 : 64);
   static constexpr int kASlots = 3;                              // TMEM A slots (one stage each)
   static constexpr int kASlotCols = 32 * T;
@@ -133,7 +136,8 @@ struct Cfg {
   static constexpr int kStages = NCOL >= 48 ? 4 : 6;
   static constexpr int kBTile = NCOL * 128;                      // one k-tile of B (NCOL rows x 128 bytes)
   static constexpr int kBBytes = T * kBTile;
-  static constexpr int kStageBytes = kCodeBytes + kBBytes;       // [codes | B tiles]
+  static constexpr int kStageBytes = kCodeBytes + kHiBytes + kBBytes;   // [codes | high bits | B tiles]
+  static constexpr int kOffBStage = kCodeBytes + kHiBytes;
   static constexpr int kOffRed = kStages * kStageBytes;
   static constexpr int kRedBytes = (kTileRows + 8) * kMaxTok * 4;
   static constexpr int kOffBars = kOffRed + (kRedBytes + 15) / 16 * 16;
@@ -215,6 +219,31 @@ __device__ __forceinline__ void expand_unit(uint4 c, uint32_t (&v)[16]) {
     v[8 * h + 5] = sg & 0x0c0c0c0cu;    // k = 2h + 1, e = 1: s = 3
     v[8 * h + 6] = sg8 & 0x03030303u;
     v[8 * h + 7] = sg8 & 0x0c0c0c0cu;
+  }
+}
+
+// 3-bit codes: the same slot placement with the whole code z = z_lo + 4 z_hi in
+// every byte (e4m3 z * 2^-9, exact for z <= 7; odd s get no factor 4, so the
+// fold leaves their B columns unscaled). hw holds the chunk's four high-bit
+// halfwords (halfword i for word i; bit 4b + s is z_hi of byte b, shift s).
+__device__ __forceinline__ uint32_t spread_nibbles(uint32_t h16) {   // nibble b -> byte b
+  return (h16 & 0xFu) | ((h16 & 0xF0u) << 4) | ((h16 & 0xF00u) << 8) | ((h16 & 0xF000u) << 12);
+}
+__device__ __forceinline__ void expand_unit3(uint4 c, uint2 hw, uint32_t (&v)[16]) {
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const uint32_t wg = h ? c.z : c.x, wg8 = h ? c.w : c.y;
+    const uint32_t hh = h ? hw.y : hw.x;   // halfwords 2h (row g) and 2h + 1 (row g + 8)
+    const uint32_t Hg = spread_nibbles(hh & 0xFFFFu), Hg8 = spread_nibbles(hh >> 16);
+#pragma unroll
+    for (int sq = 0; sq < 4; ++sq) {
+      const int k = 2 * h + (sq >> 1), e = sq & 1;
+      // bit s of each nibble-byte to bit 2 of the byte
+      const uint32_t hig = (sq <= 2 ? (Hg << (2 - sq)) : (Hg >> 1)) & 0x04040404u;
+      const uint32_t hig8 = (sq <= 2 ? (Hg8 << (2 - sq)) : (Hg8 >> 1)) & 0x04040404u;
+      v[4 * k + e] = ((wg >> (2 * sq)) & 0x03030303u) | hig;
+      v[4 * k + 2 + e] = ((wg8 >> (2 * sq)) & 0x03030303u) | hig8;
+    }
   }
 }
 
@@ -328,6 +357,7 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
   uint8_t* ws = a.layer[0].ws;
   int d = a.layer[0].d;
   float colnorm = a.layer[0].colnorm;
+  int odd_exp = a.layer[0].odd_exp;
   float A4[16], Bv[DV == 8 ? 8 : 4];
   if constexpr (DV == 4) {
 #pragma unroll
@@ -341,6 +371,7 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
       ws = a.layer[l].ws;
       d = a.layer[l].d;
       colnorm = a.layer[l].colnorm;
+      odd_exp = a.layer[l].odd_exp;
       if constexpr (DV == 4) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) A4[i] = a.layer[l].A[i];
@@ -492,7 +523,7 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
       const float v[4] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y)};
       fold4(d, A4, v, o);
     }
-    const float sc = exp2i(P + ((g & 1) ? -2 : 0));
+    const float sc = exp2i(P + ((g & 1) ? odd_exp : 0));
     uint16_t h0, m0, l0, h1, m1, l1;
     split3(pack_half2(o[0] * sc, o[1] * sc), h0, m0, l0);
     split3(pack_half2(o[2] * sc, o[3] * sc), h1, m1, l1);
@@ -506,9 +537,10 @@ __global__ void __launch_bounds__(kFoldThreads) fold_kernel(const __grid_constan
   }
 }
 
-template <int NCOL, int T>
-__global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_kernel(const __grid_constant__ SkArgs a) {
-  using C = Cfg<NCOL, T>;
+template <int NCOL, int T, int BITS>
+__global__ void __launch_bounds__(kThreads, Cfg<NCOL, T, BITS>::kMinBlocks)
+    decode_kernel(const __grid_constant__ SkArgs a) {
+  using C = Cfg<NCOL, T, BITS>;
   constexpr int kStageTiles = C::kT;
   constexpr int kCodeBytes = C::kCodeBytes;
   constexpr int kAColBase = C::kAColBase;
@@ -533,6 +565,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
   for (int i = 1; i < kMaxGroup; ++i)
     if (i < a.nlayers && static_cast<int>(blockIdx.y) >= a.layer[i].rb0) li = i;
   const uint8_t* lcodes = a.layer[0].codes;
+  const uint8_t* lhi = a.layer[0].hi;
   const uint8_t* lws = a.layer[0].ws;
   uint16_t* ly = a.layer[0].y;
   int lN = a.layer[0].N, lrb0 = a.layer[0].rb0;
@@ -540,6 +573,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
   for (int i = 1; i < kMaxGroup; ++i)
     if (i == li) {
       lcodes = a.layer[i].codes;
+      lhi = a.layer[i].hi;
       lws = a.layer[i].ws;
       ly = a.layer[i].y;
       lN = a.layer[i].N;
@@ -590,20 +624,24 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
     if (lane == 0 && !*abort_flag) {
       const uint64_t pol = policy_evict_first();
       const uint8_t* csrc = lcodes + (static_cast<size_t>(rb) * a.KT + kt0) * kTileBytes;
+      const uint8_t* hsrc = BITS == 3 ? lhi + (static_cast<size_t>(rb) * a.KT + kt0) * (kTileBytes / 2) : nullptr;
       const uint8_t* bsrc = lws + kWsTableBytes + static_cast<size_t>(kt0) * C::kBTile;
       const int pre = min(S, n_st);
       // Codes of the first stages do not depend on the previous kernels.
       for (int st = 0; st < pre; ++st) {
         const uint32_t nt = static_cast<uint32_t>(min(kStageTiles, n_kt - st * kStageTiles));
-        mbar_arrive_expect_tx(cfull(st), nt * kTileBytes);
+        mbar_arrive_expect_tx(cfull(st), nt * (kTileBytes + C::kHiBytes / kStageTiles));
         bulk_g2s(sbase + st * C::kStageBytes, csrc + static_cast<size_t>(st) * kCodeBytes, nt * kTileBytes,
                  cfull(st), pol);
+        if constexpr (BITS == 3)
+          bulk_g2s(sbase + st * C::kStageBytes + kCodeBytes, hsrc + static_cast<size_t>(st) * C::kHiBytes,
+                   nt * (kTileBytes / 2), cfull(st), pol);
       }
       pdl_wait();   // the B tiles come from the fold kernel
       for (int st = 0; st < pre; ++st) {
         const uint32_t nt = static_cast<uint32_t>(min(kStageTiles, n_kt - st * kStageTiles));
         mbar_arrive_expect_tx(bfull(st), nt * C::kBTile);
-        bulk_g2s(sbase + st * C::kStageBytes + kCodeBytes, bsrc + static_cast<size_t>(st) * C::kBBytes,
+        bulk_g2s(sbase + st * C::kStageBytes + C::kOffBStage, bsrc + static_cast<size_t>(st) * C::kBBytes,
                  nt * C::kBTile, bfull(st), pol);
       }
       int st = pre;
@@ -616,11 +654,14 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
         }
         if (*abort_flag) break;
         const uint32_t nt = static_cast<uint32_t>(min(kStageTiles, n_kt - st * kStageTiles));
-        mbar_arrive_expect_tx(cfull(s), nt * kTileBytes);
+        mbar_arrive_expect_tx(cfull(s), nt * (kTileBytes + C::kHiBytes / kStageTiles));
         bulk_g2s(sbase + s * C::kStageBytes, csrc + static_cast<size_t>(st) * kCodeBytes, nt * kTileBytes, cfull(s),
                  pol);
+        if constexpr (BITS == 3)
+          bulk_g2s(sbase + s * C::kStageBytes + kCodeBytes, hsrc + static_cast<size_t>(st) * C::kHiBytes,
+                   nt * (kTileBytes / 2), cfull(s), pol);
         mbar_arrive_expect_tx(bfull(s), nt * C::kBTile);
-        bulk_g2s(sbase + s * C::kStageBytes + kCodeBytes, bsrc + static_cast<size_t>(st) * C::kBBytes,
+        bulk_g2s(sbase + s * C::kStageBytes + C::kOffBStage, bsrc + static_cast<size_t>(st) * C::kBBytes,
                  nt * C::kBTile, bfull(s), pol);
       }
       if (*abort_flag)   // copies nobody consumed must land before exit
@@ -652,7 +693,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
         tc_fence_after();
         const int nt = min(kStageTiles, n_kt - st * kStageTiles);
         const uint32_t acol = tbase + kAColBase + kASlotCols * sa;
-        const uint32_t bst = sbase + s * C::kStageBytes + kCodeBytes;
+        const uint32_t bst = sbase + s * C::kStageBytes + C::kOffBStage;
         for (int j = 0; j < nt; ++j) {
           const uint64_t bd = sw128_desc(bst + j * C::kBTile);
 #pragma unroll
@@ -682,14 +723,22 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
       if (ok) ok = !*abort_flag && mbar_wait(cfull(s), (st / S) & 1, a.err, kErrTimeoutFull);
       const int nt = min(kStageTiles, n_kt - st * kStageTiles);
       uint4 cu[kStageTiles][2];
+      uint2 hu[kStageTiles][2];
 #pragma unroll
       for (int j = 0; j < kStageTiles; ++j) {
         cu[j][0] = make_uint4(0, 0, 0, 0);
         cu[j][1] = cu[j][0];
+        hu[j][0] = make_uint2(0, 0);
+        hu[j][1] = hu[j][0];
         if (ok && j < nt) {
           const uint8_t* tile = smem + s * C::kStageBytes + j * kTileBytes + (2 * q) * kUnitBytes + lane * 16;
           cu[j][0] = *reinterpret_cast<const uint4*>(tile);
           cu[j][1] = *reinterpret_cast<const uint4*>(tile + kUnitBytes);
+          if constexpr (BITS == 3) {   // unit u's halfwords at 256 u + 8 lane of the tile's 2 KB
+            const uint8_t* ht = smem + s * C::kStageBytes + kCodeBytes + j * (kTileBytes / 2) + (2 * q) * 256 + lane * 8;
+            hu[j][0] = *reinterpret_cast<const uint2*>(ht);
+            hu[j][1] = *reinterpret_cast<const uint2*>(ht + 256);
+          }
         }
       }
       __syncwarp();
@@ -703,9 +752,11 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
         for (int j = 0; j < kStageTiles; ++j) {
           if (j < nt) {
             uint32_t v[16];
-            expand_unit(cu[j][0], v);
+            if constexpr (BITS == 3) expand_unit3(cu[j][0], hu[j][0], v);
+            else expand_unit(cu[j][0], v);
             tmem_st16x256b_x4(tq + col + 32 * j, v);
-            expand_unit(cu[j][1], v);
+            if constexpr (BITS == 3) expand_unit3(cu[j][1], hu[j][1], v);
+            else expand_unit(cu[j][1], v);
             tmem_st16x256b_x4(tq + (16u << 16) + col + 32 * j, v);
           }
         }
@@ -787,17 +838,17 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T>::kMinBlocks) decode_ker
 
 int ncol_for(int M) { return M <= 5 ? 16 : (M <= 10 ? 32 : (M <= 16 ? 48 : 96)); }
 
-template <int NCOL, int T>
+template <int NCOL, int T, int BITS>
 bool set_attrs(int dev) {
-  static bool done[64] = {};
+  static std::atomic<bool> done[64];
   if (dev < 0 || dev >= 64) return false;
-  if (done[dev]) return true;
-  if (cudaFuncSetAttribute(decode_kernel<NCOL, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           Cfg<NCOL, T>::kSmem) != cudaSuccess ||
-      cudaFuncSetAttribute(decode_kernel<NCOL, T>, cudaFuncAttributePreferredSharedMemoryCarveout,
+  if (done[dev].load(std::memory_order_acquire)) return true;
+  if (cudaFuncSetAttribute(decode_kernel<NCOL, T, BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           Cfg<NCOL, T, BITS>::kSmem) != cudaSuccess ||
+      cudaFuncSetAttribute(decode_kernel<NCOL, T, BITS>, cudaFuncAttributePreferredSharedMemoryCarveout,
                            cudaSharedmemCarveoutMaxShared) != cudaSuccess)
     return false;
-  done[dev] = true;
+  done[dev].store(true, std::memory_order_release);
   return true;
 }
 
@@ -820,10 +871,15 @@ bool set_fold_attrs(int dev) {
   return true;
 }
 
-template <int T>
-size_t smem_of(int ncol) {
-  return ncol == 16 ? Cfg<16, T>::kSmem
-                    : (ncol == 32 ? Cfg<32, T>::kSmem : (ncol == 48 ? Cfg<48, 2>::kSmem : Cfg<96, 2>::kSmem));
+template <int T, int BITS>
+size_t smem_of_b(int ncol) {
+  return ncol == 16 ? Cfg<16, T, BITS>::kSmem
+                    : (ncol == 32 ? Cfg<32, T, BITS>::kSmem
+                                  : (ncol == 48 ? Cfg<48, 2, BITS>::kSmem : Cfg<96, 2, BITS>::kSmem));
+}
+size_t smem_of(int ncol, int T, int bits) {
+  if (bits == 3) return T == 1 ? smem_of_b<1, 3>(ncol) : smem_of_b<2, 3>(ncol);
+  return T == 1 ? smem_of_b<1, 2>(ncol) : smem_of_b<2, 2>(ncol);
 }
 
 // Resident CTAs per SM: as many as the shared memory, the TMEM columns
@@ -831,8 +887,8 @@ size_t smem_of(int ncol) {
 // one for the 96-column accumulator, three for T = 1). The occupancy query of the runtime reports one for this
 // kernel although two or three run side by side (measured), so the count is
 // derived here.
-int resident_for(int ncol, int T) {
-  const size_t smem = T == 1 ? smem_of<1>(ncol) : smem_of<2>(ncol);
+int resident_for(int ncol, int T, int bits) {
+  const size_t smem = smem_of(ncol, T, bits);
   const int by_smem = static_cast<int>((static_cast<size_t>(228) * 1024) / (smem + 1024));
   const int by_tmem = T == 1 ? 4 : (ncol > 64 ? 1 : 2);
   const int by_regs = T == 1 ? 3 : (ncol > 64 ? 1 : 2);
@@ -842,12 +898,12 @@ int resident_for(int ncol, int T) {
 // Largest K split (cluster size <= 8, >= 1 k-tile per CTA) whose grid fits in
 // one wave of resident CTAs of geometry T; at least enough slices for the
 // fold kernel's shared memory.
-DecodePlan plan_with(int nb, int KT, int num_sms, int ncol, int T) {
+DecodePlan plan_with(int nb, int KT, int num_sms, int ncol, int T, int bits) {
   DecodePlan p{};
   p.nt = ncol;
   p.nb = nb;
   p.geom = T;
-  const int slots = resident_for(ncol, T) * num_sms;
+  const int slots = resident_for(ncol, T, bits) * num_sms;
   const int min_ks = (KT * kTileCols * 2 + kFoldMaxSmem - 1) / kFoldMaxSmem;
   int ks = 0;
   for (int c = kMaxSplit; c >= 1; --c)
@@ -859,7 +915,7 @@ DecodePlan plan_with(int nb, int KT, int num_sms, int ncol, int T) {
   if (ks < 1) ks = 1;
   p.kt_per_cta = (KT + ks - 1) / ks;
   p.ks = (KT + p.kt_per_cta - 1) / p.kt_per_cta;
-  p.smem = T == 1 ? smem_of<1>(ncol) : smem_of<2>(ncol);
+  p.smem = smem_of(ncol, T, bits);
   return p;
 }
 
@@ -868,11 +924,11 @@ DecodePlan plan_with(int nb, int KT, int num_sms, int ncol, int T) {
 // stages are cheaper, but more slices spread a launch over more CTAs
 // (measured on GB300: 4096 x 11008 prefers two-tile stages at K split 8;
 // 3 x 4096 x 4096 and 28672 x 8192 prefer one-tile stages).
-DecodePlan plan_rows_split(int nb, int KT, int num_sms, int M) {
+DecodePlan plan_rows_split(int nb, int KT, int num_sms, int M, int bits = 2) {
   const int ncol = ncol_for(M);
-  const DecodePlan p2 = plan_with(nb, KT, num_sms, ncol, 2);
+  const DecodePlan p2 = plan_with(nb, KT, num_sms, ncol, 2, bits);
   if (ncol <= 32) {
-    const DecodePlan p1 = plan_with(nb, KT, num_sms, ncol, 1);
+    const DecodePlan p1 = plan_with(nb, KT, num_sms, ncol, 1, bits);
     if (p1.ks > p2.ks) return p1;
   }
   return p2;
@@ -897,13 +953,13 @@ cudaLaunchAttribute pdl_attr() {
   return at;
 }
 
-template <int NCOL, int T>
+template <int NCOL, int T, int BITS>
 unisvq_status launch_ncol(const SkArgs& a, const DecodePlan& p, int dev, cudaStream_t s) {
-  if (!set_attrs<NCOL, T>(dev)) return UNISVQ_ERR_CUDA;
+  if (!set_attrs<NCOL, T, BITS>(dev)) return UNISVQ_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.ks, p.nb, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = Cfg<NCOL, T>::kSmem;
+  cfg.dynamicSmemBytes = Cfg<NCOL, T, BITS>::kSmem;
   cfg.stream = s;
   cudaLaunchAttribute attrs[2];
   attrs[0].id = cudaLaunchAttributeClusterDimension;
@@ -913,7 +969,7 @@ unisvq_status launch_ncol(const SkArgs& a, const DecodePlan& p, int dev, cudaStr
   attrs[1] = pdl_attr();
   cfg.attrs = attrs;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, decode_kernel<NCOL, T>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
+  return cudaLaunchKernelEx(&cfg, decode_kernel<NCOL, T, BITS>, a) == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
 }  // namespace
@@ -944,7 +1000,7 @@ DecodePlan plan_skinny(const unisvq_layer* const* Ls, int n, int M) {
   int nb = 0;
   for (int i = 0; i < n; ++i) nb += Ls[i]->Np / kTileRows;
   const int per = skinny_tokens_per_launch(Ls, n);
-  return plan_rows_split(nb, Ls[0]->KT, Ls[0]->num_sms, M > per ? per : M);
+  return plan_rows_split(nb, Ls[0]->KT, Ls[0]->num_sms, M > per ? per : M, Ls[0]->bits);
 }
 
 namespace {
@@ -978,6 +1034,7 @@ unisvq_status launch_fold(const unisvq_layer* const* Ls, int n, const void* x, i
     fl.ws = ws[i];
     fl.d = L->d;
     fl.colnorm = L->colnorm;
+    fl.odd_exp = L->bits == 3 ? 0 : -2;
     for (int j = 0; j < DV * DV; ++j) fl.A[j] = L->A[j];
     for (int j = 0; j < DV; ++j) fl.B[j] = L->B[j];
   }
@@ -1007,13 +1064,16 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
   for (int i = 0; i < n; ++i) {
     nb += Ls[i]->Np / kTileRows;
     d8 = d8 || Ls[i]->d == 8;
+    // one code width per launch (the kernel instance); 3-bit codes have d <= 4
+    if (Ls[i]->bits != L0->bits || Ls[i]->grouped || (Ls[i]->bits == 3 && Ls[i]->d > 4))
+      return UNISVQ_ERR_UNSUPPORTED;
   }
   int rht_p2 = 0, rht_m = 0;
-  if (rht_sv && !rht_factor(L0->K, &rht_p2, &rht_m)) return UNISVQ_ERR_UNSUPPORTED;
+  if (rht_sv && (L0->bits != 2 || !rht_factor(L0->K, &rht_p2, &rht_m))) return UNISVQ_ERR_UNSUPPORTED;
   for (int m0 = 0; m0 < M; m0 += max_tok) {
     const int mc = M - m0 < max_tok ? M - m0 : max_tok;
     const DecodePlan p = rht_sv ? plan_rht(nb, L0->KT, L0->num_sms, mc, rht_p2)
-                                : plan_rows_split(nb, L0->KT, L0->num_sms, mc);
+                                : plan_rows_split(nb, L0->KT, L0->num_sms, mc, L0->bits);
     if (p.ks > kMaxSplit) return UNISVQ_ERR_UNSUPPORTED;
     SkArgs a{};
     a.M = mc;
@@ -1026,6 +1086,7 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
       const unisvq_layer* L = Ls[i];
       SkLayer& l = a.layer[i];
       l.codes = L->codes;
+      l.hi = L->bits == 3 ? L->hi : nullptr;
       l.ws = ws[i];
       l.y = static_cast<uint16_t*>(ys[i]) + static_cast<size_t>(m0) * L->N;
       l.N = L->N;
@@ -1035,10 +1096,17 @@ unisvq_status launch_skinny_ws(const unisvq_layer* const* Ls, int n, const void*
     unisvq_status st = d8 ? launch_fold<8>(Ls, n, x, m0, mc, p, s, ws, rht_sv)
                           : launch_fold<4>(Ls, n, x, m0, mc, p, s, ws, rht_sv);
     if (st != UNISVQ_OK) return st;
-    if (p.nt == 16) st = p.geom == 1 ? launch_ncol<16, 1>(a, p, L0->device, s) : launch_ncol<16, 2>(a, p, L0->device, s);
-    else if (p.nt == 32) st = p.geom == 1 ? launch_ncol<32, 1>(a, p, L0->device, s) : launch_ncol<32, 2>(a, p, L0->device, s);
-    else if (p.nt == 48) st = launch_ncol<48, 2>(a, p, L0->device, s);
-    else st = launch_ncol<96, 2>(a, p, L0->device, s);
+    if (L0->bits == 3) {
+      if (p.nt == 16) st = p.geom == 1 ? launch_ncol<16, 1, 3>(a, p, L0->device, s) : launch_ncol<16, 2, 3>(a, p, L0->device, s);
+      else if (p.nt == 32) st = p.geom == 1 ? launch_ncol<32, 1, 3>(a, p, L0->device, s) : launch_ncol<32, 2, 3>(a, p, L0->device, s);
+      else if (p.nt == 48) st = launch_ncol<48, 2, 3>(a, p, L0->device, s);
+      else st = launch_ncol<96, 2, 3>(a, p, L0->device, s);
+    } else {
+      if (p.nt == 16) st = p.geom == 1 ? launch_ncol<16, 1, 2>(a, p, L0->device, s) : launch_ncol<16, 2, 2>(a, p, L0->device, s);
+      else if (p.nt == 32) st = p.geom == 1 ? launch_ncol<32, 1, 2>(a, p, L0->device, s) : launch_ncol<32, 2, 2>(a, p, L0->device, s);
+      else if (p.nt == 48) st = launch_ncol<48, 2, 2>(a, p, L0->device, s);
+      else st = launch_ncol<96, 2, 2>(a, p, L0->device, s);
+    }
     if (st != UNISVQ_OK) return st;
   }
   return UNISVQ_OK;

@@ -433,12 +433,18 @@ static unisvq_status check_io(unisvq_handle h, const void* x, void* y, int M) {
 // decode path with the library's static fold workspace.
 static unisvq_status linear_inner(unisvq_handle h, int kernel, const void* x, void* y, int M, cudaStream_t s,
                                   bool noalloc) {
-  if (h->bits == 3) {   // 3-bit codes: the prefill GEMM (d <= 2) above 64 tokens, else the GEMV
+  if (h->bits == 3) {   // 3-bit codes: the prefill GEMM (d <= 4) above 64 tokens, else the tcgen05
+                        // decode path (large layers) or the GEMV, as for 2-bit codes
     if (!noalloc && ((kernel == UNISVQ_KERNEL_AUTO && M > 64 && prefill_supported(h, M)) ||
                      kernel == UNISVQ_KERNEL_PREFILL))
       return prefill_supported(h, M) ? launch_prefill(h, x, y, M, s) : UNISVQ_ERR_UNSUPPORTED;
-    if (!noalloc && kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GEMV)
+    if (noalloc) return launch_gemv(h, x, y, M, s);
+    if (kernel != UNISVQ_KERNEL_AUTO && kernel != UNISVQ_KERNEL_DECODE && kernel != UNISVQ_KERNEL_GEMV &&
+        kernel != UNISVQ_KERNEL_SKINNY)
       return kernel >= 0 && kernel <= UNISVQ_KERNEL_STREAM ? UNISVQ_ERR_UNSUPPORTED : UNISVQ_ERR_INVALID_ARG;
+    if (kernel == UNISVQ_KERNEL_AUTO || kernel == UNISVQ_KERNEL_DECODE)
+      kernel = decode_kernel_for(static_cast<long long>(h->N) * h->K, h->Np / kTileRows, M);
+    if (kernel == UNISVQ_KERNEL_SKINNY) return h->d <= 4 ? launch_skinny(h, x, y, M, s) : UNISVQ_ERR_UNSUPPORTED;
     return launch_gemv(h, x, y, M, s);
   }
   if (noalloc) {
@@ -701,13 +707,25 @@ static unisvq_status group_inner(const unisvq_handle* hs, int n, int kernel, con
                                  cudaStream_t s) {
   int n3 = 0;
   for (int i = 0; i < n; ++i) n3 += hs[i]->bits == 3 ? 1 : 0;
-  if (n3) {   // 3-bit layers: one GEMV launch when every layer is 3-bit, else layer by layer
+  if (n3) {   // 3-bit layers: one decode launch (tcgen05 or GEMV) when every layer is 3-bit, else layer by layer
     bool pf = kernel == UNISVQ_KERNEL_AUTO && M > 64;
     for (int i = 0; i < n && pf; ++i) pf = prefill_supported(hs[i], M);
     if (!pf && n3 == n &&
-        (kernel == UNISVQ_KERNEL_AUTO || kernel == UNISVQ_KERNEL_DECODE || kernel == UNISVQ_KERNEL_GEMV)) {
+        (kernel == UNISVQ_KERNEL_AUTO || kernel == UNISVQ_KERNEL_DECODE || kernel == UNISVQ_KERNEL_GEMV ||
+         kernel == UNISVQ_KERNEL_SKINNY)) {
       const unisvq_layer* Ls[UNISVQ_MAX_GROUP];
-      for (int i = 0; i < n; ++i) Ls[i] = hs[i];
+      long long w3 = 0;
+      int nb3 = 0;
+      bool d_ok = true;
+      for (int i = 0; i < n; ++i) {
+        Ls[i] = hs[i];
+        w3 += static_cast<long long>(hs[i]->N) * hs[i]->K;
+        nb3 += hs[i]->Np / kTileRows;
+        d_ok = d_ok && hs[i]->d <= 4;
+      }
+      int k = kernel;
+      if (k == UNISVQ_KERNEL_AUTO || k == UNISVQ_KERNEL_DECODE) k = decode_kernel_for(w3, nb3, M);
+      if (k == UNISVQ_KERNEL_SKINNY) return d_ok ? launch_skinny_group(Ls, n, x, ys, M, s) : UNISVQ_ERR_UNSUPPORTED;
       return launch_gemv_group(Ls, n, x, ys, M, s);
     }
     for (int i = 0; i < n; ++i) {
@@ -866,8 +884,7 @@ unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info) {
   const unisvq_layer* Ls[1] = {h};
   const int mq = M > 0 ? M : 1;
   const int kq = h->grouped ? (mq > 64 && prefill_supported(h, mq) ? UNISVQ_KERNEL_PREFILL : UNISVQ_KERNEL_GROUPED)
-                 : h->bits == 3 ? (mq > 64 && prefill_supported(h, mq) ? UNISVQ_KERNEL_PREFILL : UNISVQ_KERNEL_GEMV)
-                                : auto_kernel(h, mq);
+                             : auto_kernel(h, mq);
   describe_launch(Ls, 1, kq, M, info);
   if (h->rht) {
     // fused: one output rotation; else an input and an output rotation per
@@ -905,8 +922,6 @@ unisvq_status unisvq_query_group(const unisvq_handle* hs, int n, int M, unisvq_i
   const int m = M > 0 ? M : 1;
   const int kernel = hs[0]->grouped ? (m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL
                                                                             : UNISVQ_KERNEL_GROUPED)
-                     : hs[0]->bits == 3 ? (m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL
-                                                                                 : UNISVQ_KERNEL_GEMV)
                      : m > 64 && prefill_supported(hs[0], m) ? UNISVQ_KERNEL_PREFILL
                                                              : decode_kernel_for(weights, nb, m);
   const unisvq_layer* Ls[UNISVQ_MAX_GROUP];

@@ -1,6 +1,8 @@
 """3-bit codes (z in {0..7}, Sec. 5.2) against the fp64 oracle: dequantised
 weights bit-exact, layer outputs within the tolerance, integer cases bit-exact,
-d in {1, 2, 4}, ragged shapes, token chunking, grouped calls and dispatch."""
+d in {1, 2, 4}, ragged shapes, token chunking, grouped calls and dispatch, on
+the GEMV, the tcgen05 decode path (codes z as e4m3 bytes with the high bit
+from the bit plane) and the prefill GEMM."""
 import numpy as np
 import pytest
 
@@ -88,7 +90,7 @@ def test_3bit_dispatch_groups_and_entry_points():
     x = to_dev(xb)
     stream = torch.cuda.current_stream().cuda_stream
     y = torch.zeros((5, N), dtype=torch.bfloat16, device="cuda")
-    for kern in (binding.KERNEL_SKINNY, binding.KERNEL_GEMV_ROWS, binding.KERNEL_GROUPED):
+    for kern in (binding.KERNEL_GEMV_ROWS, binding.KERNEL_GROUPED):
         assert layer.forward_ptr(x.data_ptr(), y.data_ptr(), 5, stream, kern) == binding.ERR_UNSUPPORTED
     assert layer.forward_noalloc_ptr(x.data_ptr(), y.data_ptr(), 5, stream) == binding.OK
     assert binding.sync_status() == binding.OK
@@ -168,3 +170,59 @@ def test_3bit_d4_dispatch():
     assert oracle.compare(run(layer, xb), yr, S)["ok"]
     assert oracle.compare(run(layer, xb, binding.KERNEL_GEMV), yr, S)["ok"]
     layer.close()
+
+
+@pytest.mark.parametrize("d", [1, 2, 4])
+@pytest.mark.parametrize("N,K", [(256, 1024), (520, 1000), (130, 4096), (1024, 8192)])
+def test_3bit_tcgen05_decode_parity(d, N, K):
+    """The tcgen05 decode path on 3-bit codes: each byte of the tensor-memory
+    A operand is the whole code z (z_lo from the code words, z_hi from the
+    bit plane), forced at every token count of one and two launch pairs."""
+    if K % d:
+        pytest.skip("K must be a multiple of d")
+    codes, A, B, layer = make(N, K, d, 8)
+    Ms = (1, 3, 8, 16, 17, 33, 40)
+    xall = synth.activations(8, 60, 100 * d + N, sum(Ms), K)
+    yr, S = oracle.linear(xall, codes, A, B)
+    o = 0
+    for M in Ms:
+        res = oracle.compare(run(layer, xall[o:o + M], binding.KERNEL_SKINNY), yr[o:o + M], S[o:o + M])
+        assert res["ok"], (M, res)
+        o += M
+    layer.close()
+
+
+@pytest.mark.parametrize("d", [1, 2, 4])
+def test_3bit_tcgen05_decode_integer_case_bit_exact(d):
+    g = np.random.default_rng(60 + d)
+    N, K = 384, 1024
+    codes = g.integers(0, 8, size=(N, K), dtype=np.uint8)
+    A = (np.eye(d) - np.eye(d, k=1)).astype(np.float16)
+    B = g.integers(-3, 4, size=d).astype(np.float16)
+    layer = binding.UniSVQLinear(codes, A, B, bits=3)
+    for M in (1, 7, 33):
+        x = g.integers(-1, 2, size=(M, K)).astype(np.float32) * (g.random((M, K)) < 0.03)
+        xb = synth.f32_to_bf16_bits(x)
+        yr, _ = oracle.linear(xb, codes, A, B)
+        assert np.abs(yr).max() <= 256
+        assert np.array_equal(run(layer, xb, binding.KERNEL_SKINNY), yr)
+    layer.close()
+
+
+def test_3bit_large_layers_dispatch_to_tcgen05_decode():
+    """Large 3-bit layers and groups take the tcgen05 decode path up to 64
+    tokens, as 2-bit ones do; a group of them runs one launch pair."""
+    K = 4096
+    made = [synth.layer_inputs_bits(9, 61, i, 0, 4096, K, 2, 3) for i in range(3)]
+    layers = [binding.UniSVQLinear(c, A, B, bits=3) for c, A, B in made]
+    assert layers[0].query(4)["kernel"] == binding.KERNEL_GEMV          # 2^24 weights
+    q = binding.query_group(layers, 4)
+    assert q["kernel"] == binding.KERNEL_SKINNY and q["launches"] == 2
+    xb = synth.activations(9, 61, 0, 12, K)
+    ys = binding.linear_group(layers, to_dev(xb))
+    assert binding.sync_status() == binding.OK
+    for (c, A, B), y in zip(made, ys):
+        yr, S = oracle.linear(xb, c, A, B)
+        assert oracle.compare(y.float().cpu().numpy().astype(np.float64), yr, S)["ok"]
+    for l in layers:
+        l.close()
