@@ -31,12 +31,14 @@
 namespace unisvq {
 namespace {
 
-constexpr int kPfThreads = 14 * 32;
+// Warps: TMA producer, MMA issuer, NCONV converters (8, or 16 for per-matrix
+// 2-bit layers with d <= 4), four epilogue warps.
+__host__ __device__ constexpr int pf_threads(int nconv) { return (2 + nconv + 4) * 32; }
+constexpr int kPfThreads = pf_threads(8);
 constexpr int kBM = 128;
 constexpr int kBK = 64;                  // bf16 columns per stage (one 128B swizzle row)
 constexpr int kATileBytes = kBM * 128;   // 16 KB
 constexpr int kConvWarp0 = 2;
-constexpr int kEpiWarp0 = 10;
 constexpr int kCodeAhead = 8;   // stages of codes in flight per converter lane (8: 1081 vs 1066 TFLOP/s for 3)
 
 // Layers of one launch (several only for 2-bit layers with one d <= 4 that
@@ -202,10 +204,11 @@ __device__ __forceinline__ float4 lds128f(uint32_t addr) {
   return v;
 }
 
-template <int BN, int STAGES>
-__global__ void __launch_bounds__(kPfThreads, 1)
+template <int BN, int STAGES, int NCONV>
+__global__ void __launch_bounds__(pf_threads(NCONV), 1)
     prefill_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ PrefillArgs a) {
   using C = PfCfg<BN, STAGES>;
+  constexpr int kEpiWarp0 = kConvWarp0 + NCONV;
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the 128B-swizzled tiles.
   const uint32_t raw_addr = smem_u32(smem_raw);
@@ -227,7 +230,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(bfull(s), 1);
-      mbar_init(afull(s), 8);
+      mbar_init(afull(s), NCONV);
       mbar_init(empty(s), 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -248,7 +251,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       if (l < a.nlayers) {
         uint32_t* lut_s = reinterpret_cast<uint32_t*>(smem + C::kOffLut + 2048 * l);
         const uint32_t* src = a.lut[l];
-        for (int i = threadIdx.x; i < words; i += kPfThreads) lut_s[i] = src[i];
+        for (int i = threadIdx.x; i < words; i += pf_threads(NCONV)) lut_s[i] = src[i];
       }
     }
   }
@@ -318,7 +321,73 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       mma_commit(drain);
       mbar_wait(drain, 0, a.err, kErrTimeoutMma);
     }
-  } else if (warp < kEpiWarp0) {
+  } else if (NCONV == 16 && warp < kEpiWarp0) {
+    // ---------------- converters, 16 warps (per-matrix maps, 2-bit, d <= 4) ----------------
+    // Warp c covers row half hr = c / 8 of unit u = c % 8: lane 4g + t converts
+    // row 16u + g + 8hr, column quarter t of the stage's half, i.e. the chunks
+    // 2t and 2t + 1 of that row (one code word per stage).
+    const int c = warp - kConvWarp0, u = c & 7, hr = c >> 3;
+    const int g = lane >> 2, t = lane & 3;
+    const int r = 16 * u + g + 8 * hr;
+    const uint32_t lut_base = sbase + C::kOffLut;   // layer i's table at + 2 KB i
+    int it = 0;
+    for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
+      const int li = tile_layer(a, tile);
+      const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
+      // word (h, hr) of the lane's 16-byte chunk: byte 4 (2h + hr)
+      const uint8_t* rbase = pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes +
+                             u * kUnitBytes + lane * 16 + 4 * hr;
+      const uint32_t lut_s = lut_base + 2048u * static_cast<uint32_t>(li);
+      auto load = [&](int kb) -> uint32_t {
+        return kb < a.nkb ? __ldg(reinterpret_cast<const uint32_t*>(rbase + (kb >> 1) * kTileBytes + (kb & 1) * 8))
+                          : 0u;
+      };
+      uint32_t qr[kCodeAhead];
+#pragma unroll
+      for (int j = 0; j < kCodeAhead; ++j) qr[j] = load(j);
+      bool ok = !*abort_flag;
+      for (int kb0 = 0; kb0 < a.nkb; kb0 += kCodeAhead) {
+#pragma unroll
+        for (int j = 0; j < kCodeAhead; ++j) {
+          const int kb = kb0 + j;
+          if (kb >= a.nkb) break;
+          const int s = it % STAGES;
+          const uint32_t w = qr[j];
+          qr[j] = load(kb + kCodeAhead);   // refill the slot just read
+          if (ok && it >= STAGES) {
+            ok = !*abort_flag && mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty);
+            if (!ok) *abort_flag = 1;
+          }
+          if (ok) {
+            const uint32_t row_addr = sbase + C::kOffA + s * kATileBytes + r * 128;
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const int cc = 2 * t + e;                       // chunk: stage columns 8cc .. 8cc+7
+              const uint32_t e0 = extract4(w, 2 * e);         // columns 8cc .. 8cc+3
+              const uint32_t e1 = extract4(w, 2 * e + 1);     // columns 8cc+4 .. 8cc+7
+              uint32_t o0, o1, o2, o3;
+              if (a.d == 4) {
+                const uint32_t i0 = (e0 & 3u) | ((e0 >> 6) & 0xCu) | ((e0 >> 12) & 0x30u) | ((e0 >> 18) & 0xC0u);
+                const uint32_t i1 = (e1 & 3u) | ((e1 >> 6) & 0xCu) | ((e1 >> 12) & 0x30u) | ((e1 >> 18) & 0xC0u);
+                const uint2 v0 = lds64(lut_s + i0 * 8), v1 = lds64(lut_s + i1 * 8);
+                o0 = v0.x; o1 = v0.y; o2 = v1.x; o3 = v1.y;
+              } else {
+                o0 = lds32(lut_s + (((e0 & 3u) | ((e0 >> 6) & 0xCu)) << 2));
+                o1 = lds32(lut_s + ((((e0 >> 16) & 3u) | ((e0 >> 22) & 0xCu)) << 2));
+                o2 = lds32(lut_s + (((e1 & 3u) | ((e1 >> 6) & 0xCu)) << 2));
+                o3 = lds32(lut_s + ((((e1 >> 16) & 3u) | ((e1 >> 22) & 0xCu)) << 2));
+              }
+              sts128(row_addr + ((cc ^ g) << 4), o0, o1, o2, o3);
+            }
+            fence_proxy_async_smem();
+          }
+          __syncwarp();
+          if (lane == 0 && ok) mbar_arrive(afull(s));
+          ++it;
+        }
+      }
+    }
+  } else if (NCONV == 8 && warp < kEpiWarp0) {
     // ---------------- converters: codes -> bf16 codeword tile ----------------
     // Warp c covers unit c (rows 16c .. 16c+15): lane 4g + t reads the 8-byte
     // pair of words of rows 16c + g and 16c + g + 8 for column quarter t of the
@@ -899,7 +968,7 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, int NCONV>
 unisvq_status launch_bn(const unisvq_layer* const* Ls, int n, const PrefillPlan& p, const void* x,
                         void* const* ys, int M, cudaStream_t s) {
   using C = PfCfg<BN, STAGES>;
@@ -908,7 +977,7 @@ unisvq_status launch_bn(const unisvq_layer* const* Ls, int n, const PrefillPlan&
   const int dev = L->device;
   if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
   if (!attr_set[dev]) {
-    if (cudaFuncSetAttribute(prefill_kernel<BN, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(prefill_kernel<BN, STAGES, NCONV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              C::kSmem) != cudaSuccess)
       return UNISVQ_ERR_CUDA;
     attr_set[dev] = true;
@@ -947,7 +1016,7 @@ unisvq_status launch_bn(const unisvq_layer* const* Ls, int n, const PrefillPlan&
   a.tiles = p.tiles;
   a.err = device_error_word();
   if (tile != p.tiles) return UNISVQ_ERR_INVALID_ARG;
-  prefill_kernel<BN, STAGES><<<p.grid, kPfThreads, C::kSmem, s>>>(map, a);
+  prefill_kernel<BN, STAGES, NCONV><<<p.grid, pf_threads(NCONV), C::kSmem, s>>>(map, a);
   return cudaGetLastError() == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
@@ -995,9 +1064,18 @@ unisvq_status launch_prefill_group(const unisvq_layer* const* Ls, int n, const v
                                    cudaStream_t s) {
   if (!prefill_group_supported(Ls, n, M)) return UNISVQ_ERR_UNSUPPORTED;
   const PrefillPlan p = plan_prefill_group(Ls, n, M);
-  if (p.bn == 64) return launch_bn<64, 8>(Ls, n, p, x, ys, M, s);
-  if (p.bn == 128) return launch_bn<128, 6>(Ls, n, p, x, ys, M, s);
-  return launch_bn<256, 4>(Ls, n, p, x, ys, M, s);
+  // per-matrix 2-bit layers with d <= 4: sixteen converter warps (a row each
+  // per unit), else eight
+  bool pm = true;
+  for (int i = 0; i < n; ++i) pm = pm && !Ls[i]->grouped && Ls[i]->bits == 2 && Ls[i]->d <= 4;
+  if (pm) {
+    if (p.bn == 64) return launch_bn<64, 8, 16>(Ls, n, p, x, ys, M, s);
+    if (p.bn == 128) return launch_bn<128, 6, 16>(Ls, n, p, x, ys, M, s);
+    return launch_bn<256, 4, 16>(Ls, n, p, x, ys, M, s);
+  }
+  if (p.bn == 64) return launch_bn<64, 8, 8>(Ls, n, p, x, ys, M, s);
+  if (p.bn == 128) return launch_bn<128, 6, 8>(Ls, n, p, x, ys, M, s);
+  return launch_bn<256, 4, 8>(Ls, n, p, x, ys, M, s);
 }
 
 unisvq_status launch_prefill(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
