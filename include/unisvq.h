@@ -95,10 +95,6 @@ typedef struct {
   long long algo_bytes;   /* N*K/4 + meta + 2*M*K (x) + 2*M*N (y)               */
   double flops;           /* 2*M*N*K                                            */
   int launches;           /* kernel launches the call makes                     */
-  int cta_group;          /* prefill GEMM: CTAs per 128*cta_group-row MMA tile,
-                             1, or 2 (a cta_group::2 pair: 256-token tiles of
-                             layers whose padded rows are a multiple of 256);
-                             0 for the decode kernels                           */
 } unisvq_info;
 
 /*
@@ -311,15 +307,6 @@ unisvq_status unisvq_dequant_debug(unisvq_handle h, float* W, void* stream);
  * stream then returns UNISVQ_ERR_TIMEOUT (and clears the error word); the
  * context stays usable. Errors: INVALID_ARG, CUDA. */
 unisvq_status unisvq_debug_wait_timeout(const void* src16, int* out3, void* stream);
-
-/* Test hook (process-wide): with enable != 0, prefill launches of 256-token
- * tiles whose layers' padded rows are multiples of 256 run the GEMM on CTA
- * pairs (tcgen05 cta_group::2: a 256-row tile, each CTA converting its 128
- * weight rows and staging half of the tokens); with 0 (the default) on single
- * CTAs. The pair kernel computes the same outputs but measured slower on
- * GB300, so the library does not pick it by itself. Returns the previous
- * setting (0 or 1). */
-int unisvq_debug_prefill_pairs(int enable);
 
 /* Describe the launch unisvq_linear would make for M tokens (host only). */
 unisvq_status unisvq_query(unisvq_handle h, int M, unisvq_info* info);

@@ -24,7 +24,7 @@ EXPORTS = [
     "unisvq_status_string", "unisvq_packed_code_bytes", "unisvq_pack_host", "unisvq_version",
     "unisvq_linear_group", "unisvq_linear_group_force", "unisvq_linear_noalloc", "unisvq_query_group",
     "unisvq_pack_grouped", "unisvq_set_rht", "unisvq_hadamard", "unisvq_pack_bits",
-    "unisvq_prefill_table_host", "unisvq_debug_wait_timeout", "unisvq_debug_prefill_pairs",
+    "unisvq_prefill_table_host", "unisvq_debug_wait_timeout",
 ]
 MAX_GROUP = 4
 
@@ -40,8 +40,7 @@ class Info(ctypes.Structure):
                 ("Np", ctypes.c_int), ("Kp", ctypes.c_int), ("kernel", ctypes.c_int),
                 ("split_k", ctypes.c_int), ("grid_ctas", ctypes.c_int),
                 ("code_bytes", ctypes.c_longlong), ("meta_bytes", ctypes.c_longlong),
-                ("algo_bytes", ctypes.c_longlong), ("flops", ctypes.c_double), ("launches", ctypes.c_int),
-                ("cta_group", ctypes.c_int)]
+                ("algo_bytes", ctypes.c_longlong), ("flops", ctypes.c_double), ("launches", ctypes.c_int)]
 
 
 _lib = None
@@ -68,8 +67,6 @@ def load():
     lib.unisvq_linear_noalloc.argtypes = [vp, vp, vp, i, vp]
     lib.unisvq_dequant_debug.argtypes = [vp, vp, vp]
     lib.unisvq_debug_wait_timeout.argtypes = [vp, vp, vp]
-    lib.unisvq_debug_prefill_pairs.argtypes = [ctypes.c_int]
-    lib.unisvq_debug_prefill_pairs.restype = ctypes.c_int
     lib.unisvq_query.argtypes = [vp, i, ctypes.POINTER(Info)]
     lib.unisvq_query_group.argtypes = [vp, i, i, ctypes.POINTER(Info)]
     lib.unisvq_sync_status.argtypes = [vp]
@@ -157,12 +154,6 @@ def wait_timeout_probe_ptr(src16_ptr: int, out3_ptr: int, stream=None) -> int:
     """unisvq_debug_wait_timeout: a bounded device wait that runs out (test hook)."""
     return int(load().unisvq_debug_wait_timeout(ctypes.c_void_p(src16_ptr), ctypes.c_void_p(out3_ptr),
                                                  _stream_ptr(stream)))
-
-
-def prefill_pairs(enable: bool) -> bool:
-    """unisvq_debug_prefill_pairs: run 256-token prefill tiles on CTA pairs
-    (cta_group::2) or not (the default); returns the previous setting."""
-    return bool(load().unisvq_debug_prefill_pairs(1 if enable else 0))
 
 
 class UniSVQLinear:

@@ -77,7 +77,6 @@ struct StreamPlan {
 
 struct PrefillPlan {
   int bn;          // tokens per tile
-  int cg;          // CTAs per tile: 1, or 2 (a cta_group::2 pair, 256 weight rows)
   int tiles;
   int grid;
   size_t smem;

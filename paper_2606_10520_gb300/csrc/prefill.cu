@@ -22,7 +22,6 @@
 // under the main loop of the next.
 #include <cudaTypedefs.h>
 
-#include <atomic>
 #include <type_traits>
 
 #include "common.cuh"
@@ -84,19 +83,17 @@ __device__ __forceinline__ T pick_layer(const T (&v)[kPfMaxLayers], int li) {
   return r;
 }
 
-// CG = 2: a CTA pair computes a 256-row tile with cta_group::2 MMAs; each CTA
-// holds its 128 weight rows (A) and half of the BN tokens (B) of every stage.
-template <int BN, int STAGES, int CG = 1>
+template <int BN, int STAGES>
 struct PfCfg {
-  static constexpr int kBTileBytes = (BN / CG) * 128;
+  static constexpr int kBTileBytes = BN * 128;
   static constexpr int kStageBytes = kATileBytes + kBTileBytes;
   static constexpr int kOffA = 0;
   static constexpr int kOffB = STAGES * kATileBytes;
   static constexpr int kOffLut = STAGES * kStageBytes;            // 2 KB (d = 8: the 16 KB region)
   static constexpr int kOffGrp = kOffLut + 2048;                   // 8 x 1 KB: per-group tables
   static constexpr int kOffBars = kOffLut + 20 * 1024;            // per-group d = 8: 8 x 2304 B of maps
-  // bars: bfull[S], afull[S], empty[S], accfull[2], accempty[2], drain
-  static constexpr int kOffTmemPtr = kOffBars + (3 * STAGES + 5) * 8;
+  // bars: bfull[S], afull[S], empty[S], accfull[2], accempty[2]
+  static constexpr int kOffTmemPtr = kOffBars + (3 * STAGES + 5) * 8;   // + drain barrier
   static constexpr int kOffFlag = kOffTmemPtr + 8;
   static constexpr int kSmem = kOffFlag + 8 + 1024;                // + alignment slack
   static constexpr uint32_t kTmemCols = 2 * BN < 32 ? 32 : 2 * BN;
@@ -104,36 +101,17 @@ struct PfCfg {
 
 // ---- tcgen05 / TMA wrappers --------------------------------------------------
 
-// Arrive on an mbarrier of another CTA of the cluster (address from
-// map_shared_rank), releasing this thread's prior writes at cluster scope.
-__device__ __forceinline__ void mbar_arrive_remote(uint32_t remote_bar) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote_bar) : "memory");
-}
-
-// Every tcgen05 instruction of a kernel names the same CTA group; with
-// cta_group::2 one warp of each CTA of the pair allocates and frees together.
-template <int CG>
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
-  if constexpr (CG == 2)
-    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
-                 : "memory");
-  else
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
-                 : "memory");
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+               "r"(ncols)
+               : "memory");
 }
-template <int CG>
 __device__ __forceinline__ void tmem_relinquish() {
-  if constexpr (CG == 2)
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
-  else
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
 }
-template <int CG>
 __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-  if constexpr (CG == 2)
-    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
-  else
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
 }
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -157,45 +135,26 @@ __device__ __forceinline__ uint64_t make_sw128_desc(uint32_t saddr) {
   return d;
 }
 
-// Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major,
-// M = 128 per CTA of the group, N = BN.
-template <int BN, int CG>
+// Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major, M = 128.
+template <int BN>
 __device__ __forceinline__ uint32_t make_idesc() {
   return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
-         (static_cast<uint32_t>((CG * kBM) >> 4) << 24);
+         (static_cast<uint32_t>(kBM >> 4) << 24);
 }
 
-template <int CG>
-__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                         uint32_t accumulate) {
-  if constexpr (CG == 2)
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-        : "memory");
-  else
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-        : "memory");
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
 }
 
-// Arrive on `bar` once the MMAs issued so far have completed; with CG = 2 on
-// the barrier at the same offset in both CTAs of the pair.
-template <int CG>
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
-  if constexpr (CG == 2)
-    asm volatile(
-        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
-        "h"(static_cast<uint16_t>(3))
-        : "memory");
-  else
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-                 : "memory");
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
 }
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int c0, int c1,
@@ -245,10 +204,10 @@ __device__ __forceinline__ float4 lds128f(uint32_t addr) {
   return v;
 }
 
-template <int BN, int STAGES, int NCONV, int CG>
+template <int BN, int STAGES, int NCONV>
 __global__ void __launch_bounds__(pf_threads(NCONV), 1)
     prefill_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ PrefillArgs a) {
-  using C = PfCfg<BN, STAGES, CG>;
+  using C = PfCfg<BN, STAGES>;
   constexpr int kEpiWarp0 = kConvWarp0 + NCONV;
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the 128B-swizzled tiles.
@@ -267,31 +226,16 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
   const uint32_t drain = bar0 + 8u * (3 * STAGES + 4);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffFlag);
   uint32_t* tmem_ptr = reinterpret_cast<uint32_t*>(smem + C::kOffTmemPtr);
-  // Tiles: a.tiles tiles of CG x 128 rows x BN tokens; CTA `rank` of a group
-  // holds the 128-row block CG * (tile's row tile) + rank.
-  const int rank = CG == 2 ? static_cast<int>(cluster_ctarank()) : 0;
-  const int tile_first = static_cast<int>(blockIdx.x) / CG, tile_step = static_cast<int>(gridDim.x) / CG;
-  auto row_block = [&](int tile, int li) { return CG * ((tile - pick_layer(a.tile0, li)) / a.mtiles) + rank; };
-  // A converter warp has stored its rows of stage s (lane 0, after the proxy
-  // fence); with CG = 2 the second CTA's warps arrive on the first CTA's
-  // barrier, releasing their stores at cluster scope.
-  auto conv_arrive = [&](int s) {
-    if (CG == 2 && rank != 0) mbar_arrive_remote(map_shared_rank(afull(s), 0));
-    else mbar_arrive(afull(s));
-  };
-
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(bfull(s), 1);
-      // the converter warps of every CTA of the group, and (CG = 2) the
-      // second CTA's forwarder once its B half has landed
-      mbar_init(afull(s), NCONV * CG + (CG - 1));
+      mbar_init(afull(s), NCONV);
       mbar_init(empty(s), 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(accfull(b), 1);
-      mbar_init(accempty(b), 4 * CG);   // the epilogue warps of every CTA of the group
+      mbar_init(accempty(b), 4);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -312,12 +256,11 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
     }
   }
   if (warp == 0) {
-    tmem_alloc<CG>(sbase + C::kOffTmemPtr, C::kTmemCols);
-    tmem_relinquish<CG>();
+    tmem_alloc(sbase + C::kOffTmemPtr, C::kTmemCols);
+    tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
-  if (CG == 2) cluster_sync();   // both CTAs' barriers initialised before any remote arrive or commit
   tc_fence_after();
   const uint32_t tmem_base = *tmem_ptr;
 
@@ -325,9 +268,8 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
     // ---------------- TMA producer: activations ----------------
     if (lane == 0) {
       int it = 0;
-      for (int tile = tile_first; tile < a.tiles && !*abort_flag; tile += tile_step) {
-        // this CTA's half of the tile's tokens (CG = 2)
-        const int m0 = ((tile - pick_layer(a.tile0, tile_layer(a, tile))) % a.mtiles) * BN + rank * (BN / CG);
+      for (int tile = blockIdx.x; tile < a.tiles && !*abort_flag; tile += gridDim.x) {
+        const int m0 = ((tile - pick_layer(a.tile0, tile_layer(a, tile))) % a.mtiles) * BN;
         for (int kb = 0; kb < a.nkb; ++kb, ++it) {
           const int s = it % STAGES;
           if (it >= STAGES && !mbar_wait(empty(s), ((it / STAGES) - 1) & 1, a.err, kErrTimeoutEmpty)) {
@@ -344,17 +286,15 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
           mbar_wait(bfull(j % STAGES), (j / STAGES) & 1, a.err, kErrTimeoutFull);
     }
   } else if (warp == 1) {
-    if (CG == 1 || rank == 0) {
-    // ---------------- MMA issuer (CG = 2: the pair's first CTA) ----------------
+    // ---------------- MMA issuer ----------------
     if (lane == 0) {
-      const uint32_t idesc = make_idesc<BN, CG>();
+      const uint32_t idesc = make_idesc<BN>();
       int it = 0, lt = 0;
       bool ok = true;
-      for (int tile = tile_first; tile < a.tiles && ok; tile += tile_step, ++lt) {
+      for (int tile = blockIdx.x; tile < a.tiles && ok; tile += gridDim.x, ++lt) {
         const int b = lt & 1;
         if (lt >= 2) {
-          ok = CG == 2 ? mbar_wait_cluster(accempty(b), ((lt >> 1) - 1) & 1, a.err, kErrTimeoutAcc)
-                       : mbar_wait(accempty(b), ((lt >> 1) - 1) & 1, a.err, kErrTimeoutAcc);
+          ok = mbar_wait(accempty(b), ((lt >> 1) - 1) & 1, a.err, kErrTimeoutAcc);
           if (!ok) break;
         }
         tc_fence_after();
@@ -362,44 +302,23 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
         for (int kb = 0; kb < a.nkb; ++kb, ++it) {
           const int s = it % STAGES;
           const uint32_t ph = (it / STAGES) & 1;
-          // this CTA's B tile, and the A rows of every CTA of the group (with
-          // CG = 2 also the second CTA's B half) have landed
           ok = !*abort_flag && mbar_wait(bfull(s), ph, a.err, kErrTimeoutFull) &&
-               (CG == 2 ? mbar_wait_cluster(afull(s), ph, a.err, kErrTimeoutFull)
-                        : mbar_wait(afull(s), ph, a.err, kErrTimeoutFull));
+               mbar_wait(afull(s), ph, a.err, kErrTimeoutFull);
           if (!ok) break;
           tc_fence_after();
-          // CG = 2: the same offsets in the peer hold its 128 rows of A and its half of B
           const uint64_t ad = make_sw128_desc(sbase + C::kOffA + s * kATileBytes);
           const uint64_t bd = make_sw128_desc(sbase + C::kOffB + s * C::kBTileBytes);
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k)   // +32 bytes per K=16 step inside the swizzle row
-            mma_bf16<CG>(dcol, ad + 2 * k, bd + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
-          mma_commit<CG>(empty(s));
+            mma_bf16(dcol, ad + 2 * k, bd + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          mma_commit(empty(s));
         }
         if (!ok) break;
-        mma_commit<CG>(accfull(b));
+        mma_commit(accfull(b));
       }
       if (!ok) *abort_flag = 1;
       // Everything issued so far must retire before TMEM is released.
-      mma_commit<CG>(drain);
-      mbar_wait(drain, 0, a.err, kErrTimeoutMma);
-    }
-    } else if (lane == 0) {
-      // ---------------- forwarder (CG = 2, second CTA) ----------------
-      // Arrives on the first CTA's afull(s) once this CTA's B half of stage s
-      // has landed (the release at cluster scope carries the TMA's bytes).
-      int it = 0;
-      bool ok = true;
-      for (int tile = tile_first; tile < a.tiles && ok; tile += tile_step)
-        for (int kb = 0; kb < a.nkb; ++kb, ++it) {
-          const int s = it % STAGES;
-          ok = !*abort_flag && mbar_wait(bfull(s), (it / STAGES) & 1, a.err, kErrTimeoutFull);
-          if (!ok) break;
-          mbar_arrive_remote(map_shared_rank(afull(s), 0));
-        }
-      if (!ok) *abort_flag = 1;
-      // the first CTA's drain commit also arrives here
+      mma_commit(drain);
       mbar_wait(drain, 0, a.err, kErrTimeoutMma);
     }
   } else if (NCONV == 16 && warp < kEpiWarp0) {
@@ -412,9 +331,9 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
     const int r = 16 * u + g + 8 * hr;
     const uint32_t lut_base = sbase + C::kOffLut;   // layer i's table at + 2 KB i
     int it = 0;
-    for (int tile = tile_first; tile < a.tiles; tile += tile_step) {
+    for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
       const int li = tile_layer(a, tile);
-      const int n_blk = row_block(tile, li);
+      const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
       // word (h, hr) of the lane's 16-byte chunk: byte 4 (2h + hr)
       const uint8_t* rbase = pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes +
                              u * kUnitBytes + lane * 16 + 4 * hr;
@@ -463,7 +382,7 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
             fence_proxy_async_smem();
           }
           __syncwarp();
-          if (lane == 0 && ok) conv_arrive(s);
+          if (lane == 0 && ok) mbar_arrive(afull(s));
           ++it;
         }
       }
@@ -490,9 +409,9 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
       // sum_c' A[c][c'] z_c' + B[c] in fp32 (one 16-byte store per vector); the
       // warp stages its 16 rows' maps (72 fp16 each) in shared memory per k-tile.
       const uint32_t map_s = sbase + C::kOffLut + c * 2304;   // [16 rows][72] fp16
-      for (int tile = tile_first; tile < a.tiles; tile += tile_step) {
+      for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
         const int li = tile_layer(a, tile);
-        const int n_blk = row_block(tile, li);
+        const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
         const uint8_t* rbase =
             pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
         const uint32_t* mbase = reinterpret_cast<const uint32_t*>(pick_layer(a.meta, li) +
@@ -583,7 +502,7 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
             fence_proxy_async_smem();
           }
           __syncwarp();
-          if (lane == 0 && ok) conv_arrive(s);
+          if (lane == 0 && ok) mbar_arrive(afull(s));
         }
       }
     } else if (a.meta[0] && a.d == 4) {
@@ -596,9 +515,9 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
       // warp stages its 16 rows' maps (20 fp16 each, 640 contiguous bytes) in
       // shared memory once per k-tile.
       const uint32_t map_s = sbase + C::kOffGrp + c * 1024;   // [16 rows][20] fp16
-      for (int tile = tile_first; tile < a.tiles; tile += tile_step) {
+      for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
         const int li = tile_layer(a, tile);
-        const int n_blk = row_block(tile, li);
+        const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
         const uint8_t* rbase =
             pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
         const uint32_t* mbase = reinterpret_cast<const uint32_t*>(pick_layer(a.meta, li) + static_cast<size_t>(n_blk) * a.KT * kBM * 20 +
@@ -683,7 +602,7 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
             fence_proxy_async_smem();
           }
           __syncwarp();
-          if (lane == 0 && ok) conv_arrive(s);
+          if (lane == 0 && ok) mbar_arrive(afull(s));
         }
       }
     } else if (a.meta[0] && a.d == 1) {
@@ -697,9 +616,9 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
       // row's map (four entries per lane and row); the columns j, j + 1 (bytes
       // e(j), e(j + 1)) index it.
       const uint32_t tab_s = sbase + C::kOffGrp + c * 1024;   // [16 rows][16 entries] bf16x2
-      for (int tile = tile_first; tile < a.tiles; tile += tile_step) {
+      for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
         const int li = tile_layer(a, tile);
-        const int n_blk = row_block(tile, li);
+        const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
         const uint8_t* rbase =
             pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
         const uint16_t* mbase = pick_layer(a.meta, li) + static_cast<size_t>(n_blk) * a.KT * kBM * 2;
@@ -762,7 +681,7 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
             fence_proxy_async_smem();
           }
           __syncwarp();
-          if (lane == 0 && ok) conv_arrive(s);
+          if (lane == 0 && ok) mbar_arrive(afull(s));
         }
       }
     } else if (a.meta[0]) {
@@ -775,9 +694,9 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
       // 16-byte load. Per k-tile the warp builds, for each of its 16 rows, the 16
       // bf16 pairs RN(A z + B) of the row's map (four entries per lane and row).
       const uint32_t tab_s = sbase + C::kOffGrp + c * 1024;   // [16 rows][16 entries] bf16x2
-      for (int tile = tile_first; tile < a.tiles; tile += tile_step) {
+      for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
         const int li = tile_layer(a, tile);
-        const int n_blk = row_block(tile, li);
+        const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
         const uint8_t* rbase =
             pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
         const uint16_t* mbase = pick_layer(a.meta, li) + static_cast<size_t>(n_blk) * a.KT * kBM * 6;
@@ -850,7 +769,7 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
             fence_proxy_async_smem();
           }
           __syncwarp();
-          if (lane == 0 && ok) conv_arrive(s);
+          if (lane == 0 && ok) mbar_arrive(afull(s));
         }
       }
     } else {
@@ -862,9 +781,9 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
         constexpr bool HI = decltype(hi_tag)::value;
         constexpr bool D8 = decltype(d8_tag)::value;
         constexpr bool P4 = decltype(p4_tag)::value;
-        for (int tile = tile_first; tile < a.tiles; tile += tile_step) {
+        for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
           const int li = tile_layer(a, tile);
-          const int n_blk = row_block(tile, li);
+          const int n_blk = (tile - pick_layer(a.tile0, li)) / a.mtiles;
           const uint8_t* rbase =
               pick_layer(a.codes, li) + static_cast<size_t>(n_blk) * a.KT * kTileBytes + c * kUnitBytes + lane * 16;
           const uint32_t lut_s = lut_base + 2048u * static_cast<uint32_t>(li);
@@ -979,7 +898,7 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
               fence_proxy_async_smem();
             }
             __syncwarp();
-            if (lane == 0 && ok) conv_arrive(s);
+            if (lane == 0 && ok) mbar_arrive(afull(s));
             ++it;
           }
           }
@@ -995,11 +914,11 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
     const int q = warp & 3;                      // TMEM lane quarter of this warp
     int lt = 0;
     bool ok = true;
-    for (int tile = tile_first; tile < a.tiles && ok; tile += tile_step, ++lt) {
+    for (int tile = blockIdx.x; tile < a.tiles && ok; tile += gridDim.x, ++lt) {
       const int b = lt & 1;
       const int li = tile_layer(a, tile);
       const int local = tile - pick_layer(a.tile0, li);
-      const int n0 = row_block(tile, li) * kBM;   // this CTA's 128 rows; its TMEM holds all BN tokens
+      const int n0 = (local / a.mtiles) * kBM;
       const int m0 = (local % a.mtiles) * BN;
       uint16_t* const yl = pick_layer(a.y, li);
       const int Nl = pick_layer(a.N, li);
@@ -1024,21 +943,15 @@ __global__ void __launch_bounds__(pf_threads(NCONV), 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) {
-        if (CG == 2 && rank != 0) mbar_arrive_remote(map_shared_rank(accempty(b), 0));
-        else mbar_arrive(accempty(b));
-      }
+      if (lane == 0) mbar_arrive(accempty(b));
     }
   }
 
   tc_fence_before();
   __syncthreads();
-  // CG = 2: no CTA leaves (or frees TMEM) while the other may still arrive on
-  // its barriers or the pair's MMAs may still read its shared memory.
-  if (CG == 2) cluster_sync();
   if (warp == 0) {
     tc_fence_after();
-    tmem_dealloc<CG>(tmem_base, C::kTmemCols);
+    tmem_dealloc(tmem_base, C::kTmemCols);
   }
 }
 
@@ -1055,68 +968,26 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
-// Shared-memory attribute of one kernel instance, set once per device.
-template <int BN, int STAGES, int NCONV, int CG>
-bool set_smem_attr(int dev) {
-  static std::atomic<bool> done[64];
-  if (dev < 0 || dev >= 64) return false;
-  if (done[dev].load()) return true;
-  if (cudaFuncSetAttribute(prefill_kernel<BN, STAGES, NCONV, CG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           PfCfg<BN, STAGES, CG>::kSmem) != cudaSuccess)
-    return false;
-  done[dev].store(true);
-  return true;
-}
-
-constexpr int kPairStages = 6;   // CG = 2, BN = 256: 16 KB of A + 16 KB of B per stage
-
-// CTA pairs of the cta_group::2 kernel that can be resident at once (one CTA
-// per SM; a pair sits on two SMs of one cluster slot), per device and
-// converter count; 0 if the query fails.
-int pair_slots(int dev, int nconv) {
-  static std::atomic<int> slots[64][2];
-  if (dev < 0 || dev >= 64) return 0;
-  const int ci = nconv == 16 ? 1 : 0;
-  int v = slots[dev][ci].load();
-  if (v > 0) return v;
-  const bool attr = nconv == 16 ? set_smem_attr<256, kPairStages, 16, 2>(dev) : set_smem_attr<256, kPairStages, 8, 2>(dev);
-  if (!attr) return 0;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(2, 1, 1);
-  cfg.blockDim = dim3(pf_threads(nconv), 1, 1);
-  cfg.dynamicSmemBytes = PfCfg<256, kPairStages, 2>::kSmem;
-  cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeClusterDimension;
-  at[0].val.clusterDim.x = 2;
-  at[0].val.clusterDim.y = 1;
-  at[0].val.clusterDim.z = 1;
-  cfg.attrs = at;
-  cfg.numAttrs = 1;
-  int n = 0;
-  const cudaError_t e = nconv == 16
-                            ? cudaOccupancyMaxActiveClusters(&n, prefill_kernel<256, kPairStages, 16, 2>, &cfg)
-                            : cudaOccupancyMaxActiveClusters(&n, prefill_kernel<256, kPairStages, 8, 2>, &cfg);
-  if (e != cudaSuccess || n < 1) {
-    (void)cudaGetLastError();
-    return 0;
-  }
-  slots[dev][ci].store(n);
-  return n;
-}
-
-template <int BN, int STAGES, int NCONV, int CG>
+template <int BN, int STAGES, int NCONV>
 unisvq_status launch_bn(const unisvq_layer* const* Ls, int n, const PrefillPlan& p, const void* x,
                         void* const* ys, int M, cudaStream_t s) {
-  using C = PfCfg<BN, STAGES, CG>;
+  using C = PfCfg<BN, STAGES>;
   const unisvq_layer* L = Ls[0];
+  static bool attr_set[64] = {};
   const int dev = L->device;
-  if (p.cg != CG || !set_smem_attr<BN, STAGES, NCONV, CG>(dev)) return UNISVQ_ERR_CUDA;
+  if (dev < 0 || dev >= 64) return UNISVQ_ERR_CUDA;
+  if (!attr_set[dev]) {
+    if (cudaFuncSetAttribute(prefill_kernel<BN, STAGES, NCONV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::kSmem) != cudaSuccess)
+      return UNISVQ_ERR_CUDA;
+    attr_set[dev] = true;
+  }
   PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode();
   if (!enc) return UNISVQ_ERR_CUDA;
   CUtensorMap map;
   const cuuint64_t dims[2] = {static_cast<cuuint64_t>(L->K), static_cast<cuuint64_t>(M)};
   const cuuint64_t strides[1] = {static_cast<cuuint64_t>(L->K) * 2};
-  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), static_cast<cuuint32_t>(BN / CG)};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), static_cast<cuuint32_t>(BN)};
   const cuuint32_t estr[2] = {1, 1};
   if (enc(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(x), dims, strides, box, estr,
           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -1133,7 +1004,7 @@ unisvq_status launch_bn(const unisvq_layer* const* Ls, int n, const PrefillPlan&
     a.N[i] = Ls[i]->N;
     a.meta[i] = Ls[i]->grouped ? Ls[i]->meta : nullptr;
     a.tile0[i] = tile;
-    tile += (Ls[i]->Np / (CG * kBM)) * a.mtiles;
+    tile += (Ls[i]->Np / kBM) * a.mtiles;
   }
   a.nlayers = n;
   a.hi = L->bits == 3 ? L->hi : nullptr;
@@ -1145,24 +1016,8 @@ unisvq_status launch_bn(const unisvq_layer* const* Ls, int n, const PrefillPlan&
   a.tiles = p.tiles;
   a.err = device_error_word();
   if (tile != p.tiles) return UNISVQ_ERR_INVALID_ARG;
-  if constexpr (CG == 1) {
-    prefill_kernel<BN, STAGES, NCONV, 1><<<p.grid, pf_threads(NCONV), C::kSmem, s>>>(map, a);
-    return cudaGetLastError() == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
-  }
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.grid, 1, 1);
-  cfg.blockDim = dim3(pf_threads(NCONV), 1, 1);
-  cfg.dynamicSmemBytes = C::kSmem;
-  cfg.stream = s;
-  cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeClusterDimension;
-  at[0].val.clusterDim.x = CG;
-  at[0].val.clusterDim.y = 1;
-  at[0].val.clusterDim.z = 1;
-  cfg.attrs = at;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, prefill_kernel<BN, STAGES, NCONV, CG>, map, a) == cudaSuccess ? UNISVQ_OK
-                                                                                                 : UNISVQ_ERR_CUDA;
+  prefill_kernel<BN, STAGES, NCONV><<<p.grid, pf_threads(NCONV), C::kSmem, s>>>(map, a);
+  return cudaGetLastError() == cudaSuccess ? UNISVQ_OK : UNISVQ_ERR_CUDA;
 }
 
 int pick_bn(int M) { return M <= 64 ? 64 : (M <= 128 ? 128 : 256); }
@@ -1191,35 +1046,15 @@ bool prefill_group_supported(const unisvq_layer* const* Ls, int n, int M) {
   return true;
 }
 
-// CTA pairs for 256-token tiles: off unless a test turns them on (measured
-// slower than single CTAs on GB300).
-std::atomic<int> g_prefill_pairs{0};
-
-// Converter warps: sixteen (a row each per unit) for per-matrix 2-bit layers
-// with d <= 4, else eight.
-int pick_nconv(const unisvq_layer* const* Ls, int n) {
-  bool pm = true;
-  for (int i = 0; i < n; ++i) pm = pm && !Ls[i]->grouped && Ls[i]->bits == 2 && Ls[i]->d <= 4;
-  return pm ? 16 : 8;
-}
-
 PrefillPlan plan_prefill_group(const unisvq_layer* const* Ls, int n, int M) {
   PrefillPlan p{};
   p.bn = pick_bn(M);
-  // 256-token tiles of layers whose padded rows fill 256-row tiles run on CTA
-  // pairs (cta_group::2): each CTA stages half of the tokens' B tiles
-  bool rows256 = true;
-  for (int i = 0; i < n; ++i) rows256 = rows256 && Ls[i]->Np % 256 == 0;
-  const int pairs = g_prefill_pairs.load() && p.bn == 256 && rows256 ? pair_slots(Ls[0]->device, pick_nconv(Ls, n)) : 0;
-  p.cg = pairs > 0 ? 2 : 1;
   const int mtiles = (M + p.bn - 1) / p.bn;
   p.tiles = 0;
-  for (int i = 0; i < n; ++i) p.tiles += (Ls[i]->Np / (p.cg * kBM)) * mtiles;
-  const int slots = p.cg == 2 ? pairs : Ls[0]->num_sms;
-  p.grid = p.cg * (p.tiles < slots ? p.tiles : slots);
-  if (p.grid < p.cg) p.grid = p.cg;
-  p.smem = p.cg == 2 ? PfCfg<256, kPairStages, 2>::kSmem
-                     : (p.bn == 64 ? PfCfg<64, 8>::kSmem : (p.bn == 128 ? PfCfg<128, 6>::kSmem : PfCfg<256, 4>::kSmem));
+  for (int i = 0; i < n; ++i) p.tiles += (Ls[i]->Np / kBM) * mtiles;
+  p.grid = p.tiles < Ls[0]->num_sms ? p.tiles : Ls[0]->num_sms;
+  if (p.grid < 1) p.grid = 1;
+  p.smem = p.bn == 64 ? PfCfg<64, 8>::kSmem : (p.bn == 128 ? PfCfg<128, 6>::kSmem : PfCfg<256, 4>::kSmem);
   return p;
 }
 
@@ -1229,16 +1064,18 @@ unisvq_status launch_prefill_group(const unisvq_layer* const* Ls, int n, const v
                                    cudaStream_t s) {
   if (!prefill_group_supported(Ls, n, M)) return UNISVQ_ERR_UNSUPPORTED;
   const PrefillPlan p = plan_prefill_group(Ls, n, M);
-  if (pick_nconv(Ls, n) == 16) {
-    if (p.cg == 2) return launch_bn<256, kPairStages, 16, 2>(Ls, n, p, x, ys, M, s);
-    if (p.bn == 64) return launch_bn<64, 8, 16, 1>(Ls, n, p, x, ys, M, s);
-    if (p.bn == 128) return launch_bn<128, 6, 16, 1>(Ls, n, p, x, ys, M, s);
-    return launch_bn<256, 4, 16, 1>(Ls, n, p, x, ys, M, s);
+  // per-matrix 2-bit layers with d <= 4: sixteen converter warps (a row each
+  // per unit), else eight
+  bool pm = true;
+  for (int i = 0; i < n; ++i) pm = pm && !Ls[i]->grouped && Ls[i]->bits == 2 && Ls[i]->d <= 4;
+  if (pm) {
+    if (p.bn == 64) return launch_bn<64, 8, 16>(Ls, n, p, x, ys, M, s);
+    if (p.bn == 128) return launch_bn<128, 6, 16>(Ls, n, p, x, ys, M, s);
+    return launch_bn<256, 4, 16>(Ls, n, p, x, ys, M, s);
   }
-  if (p.cg == 2) return launch_bn<256, kPairStages, 8, 2>(Ls, n, p, x, ys, M, s);
-  if (p.bn == 64) return launch_bn<64, 8, 8, 1>(Ls, n, p, x, ys, M, s);
-  if (p.bn == 128) return launch_bn<128, 6, 8, 1>(Ls, n, p, x, ys, M, s);
-  return launch_bn<256, 4, 8, 1>(Ls, n, p, x, ys, M, s);
+  if (p.bn == 64) return launch_bn<64, 8, 8>(Ls, n, p, x, ys, M, s);
+  if (p.bn == 128) return launch_bn<128, 6, 8>(Ls, n, p, x, ys, M, s);
+  return launch_bn<256, 4, 8>(Ls, n, p, x, ys, M, s);
 }
 
 unisvq_status launch_prefill(const unisvq_layer* L, const void* x, void* y, int M, cudaStream_t s) {
@@ -1247,7 +1084,3 @@ unisvq_status launch_prefill(const unisvq_layer* L, const void* x, void* y, int 
 }
 
 }  // namespace unisvq
-
-extern "C" int unisvq_debug_prefill_pairs(int enable) {
-  return unisvq::g_prefill_pairs.exchange(enable ? 1 : 0);
-}

@@ -860,16 +860,10 @@ static void describe_launch(const unisvq_layer* const* Ls, int n, int kernel, in
     info->split_k = 1;
     info->grid_ctas = p.grid;
     info->launches = 1;
-    info->cta_group = p.cg;
   } else {
     info->split_k = 1;
     info->grid_ctas = 0;
-    info->cta_group = 2;
-    for (int i = 0; i < n; ++i) {
-      const PrefillPlan p = plan_prefill(Ls[i], m);
-      info->grid_ctas += p.grid;
-      if (p.cg < info->cta_group) info->cta_group = p.cg;
-    }
+    for (int i = 0; i < n; ++i) info->grid_ctas += plan_prefill(Ls[i], m).grid;
     info->launches = n;
   }
 }

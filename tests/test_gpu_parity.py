@@ -248,96 +248,6 @@ def test_prefill_group_one_launch(d):
         l.close()
 
 
-@pytest.fixture
-def cta_pairs():
-    """Turn the prefill's CTA-pair path (a test hook, off by default) on for
-    one test."""
-    prev = binding.prefill_pairs(True)
-    assert prev is False
-    yield
-    binding.prefill_pairs(False)
-
-
-def test_prefill_cta_pairs_off_by_default():
-    codes, A, B = synth.layer_inputs(8, 94, 2, 0, 512, 256, 2)
-    layer = binding.UniSVQLinear(codes, A, B)
-    assert layer.query(300)["cta_group"] == 1
-    layer.close()
-
-
-@pytest.mark.parametrize("d", [2, 4, 8])
-def test_prefill_cta_pairs(d, cta_pairs):
-    """With the hook on, 256-token tiles of layers whose padded rows are a
-    multiple of 256 run on cta_group::2 CTA pairs (each CTA converts its 128
-    rows and stages half of the tokens); other row counts, and 64/128-token
-    tiles, on single CTAs. A group call of pair layers equals the per-layer
-    calls bit for bit, and every output meets the oracle, ragged token tails
-    included."""
-    K = 1024
-    shapes = [512, 256, 768]
-    layers, data = [], []
-    for i, N in enumerate(shapes):
-        c, A, B = synth.layer_inputs(8, 95 + i, d, 0, N, K, d)
-        layers.append(binding.UniSVQLinear(c, A, B))
-        data.append((c, A, B))
-    odd_c, odd_A, odd_B = synth.layer_inputs(8, 99, d, 0, 384, K, d)
-    odd = binding.UniSVQLinear(odd_c, odd_A, odd_B)
-    for M in (129, 300, 777):
-        q = binding.query_group(layers, M)
-        assert q["kernel"] == binding.KERNEL_PREFILL and q["launches"] == (1 if d <= 4 else 3)
-        assert q["cta_group"] == 2 and q["grid_ctas"] % 2 == 0, q
-        assert layers[0].query(M)["cta_group"] == 2
-        assert odd.query(M)["cta_group"] == 1
-        assert binding.query_group([layers[0], odd], M)["cta_group"] == 1
-    assert layers[0].query(128)["cta_group"] == 1
-    assert layers[0].query(65)["cta_group"] == 1
-    for M in (129, 300, 777):
-        xb = synth.activations(8, 95, M, M, K)
-        x = to_dev(xb)
-        got = binding.linear_group(layers, x, kernel=binding.KERNEL_PREFILL)
-        assert binding.sync_status() == binding.OK
-        for l, y, (c, A, B) in zip(layers, got, data):
-            yl = l.forward(x, kernel=binding.KERNEL_PREFILL)
-            assert binding.sync_status() == binding.OK
-            assert np.array_equal(y.view(torch.int16).cpu().numpy(), yl.view(torch.int16).cpu().numpy())
-            check(y.float().cpu().numpy().astype(np.float64), xb, c, A, B)
-        check(run(odd, xb, binding.KERNEL_PREFILL), xb, odd_c, odd_A, odd_B)
-    for l in layers + [odd]:
-        l.close()
-
-
-def test_prefill_cta_pairs_integer_case_bit_exact(cta_pairs):
-    """Integer codewords and activations on the CTA-pair path (N = 512, two
-    pair tiles of rows; M = 300: a full and a ragged token tile)."""
-    d = 2
-    A = np.array([[1, -1], [1, 1]], dtype=np.float16)
-    B = np.array([-1, 2], dtype=np.float16)
-    N, K = 512, 768
-    g = np.random.default_rng(21)
-    codes = g.integers(0, 4, size=(N, K), dtype=np.uint8)
-    layer = binding.UniSVQLinear(codes, A, B)
-    M = 300
-    assert layer.query(M)["cta_group"] == 2
-    x = g.integers(-1, 2, size=(M, K)).astype(np.float32) * (g.random((M, K)) < 0.05)
-    xb = synth.f32_to_bf16_bits(x)
-    yr, _ = oracle.linear(xb, codes, A, B)
-    assert np.abs(yr).max() <= 256
-    yg = run(layer, xb, binding.KERNEL_PREFILL)
-    assert np.array_equal(yg, yr), np.abs(yg - yr).max()
-    layer.close()
-
-
-def test_prefill_cta_pairs_full_size(cta_pairs):
-    """The Llama-3-8B gate shape at M = 2048 on CTA pairs, every row."""
-    N, K, d = 14336, 4096, 2
-    codes, A, B = synth.layer_inputs(0, 2, 0, N + K, N, K, d)
-    layer = binding.UniSVQLinear(codes, A, B)
-    assert layer.query(2048)["cta_group"] == 2
-    xb = synth.activations(0, 2, K, 2048, K)
-    check(run(layer, xb), xb, codes, A, B)
-    layer.close()
-
-
 def test_prefill_group_falls_back_per_layer():
     """Mixed d (2 and 4) or a d = 8 layer: one prefill launch per layer."""
     K = 512
