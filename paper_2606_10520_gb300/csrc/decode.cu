@@ -791,15 +791,43 @@ __global__ void __launch_bounds__(kThreads, Cfg<NCOL, T, BITS>::kMinBlocks)
 #pragma unroll
       for (int c0 = 0; c0 < NCOL; c0 += 16) tmem_ld16(tq + c0, dv + c0);
       asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+      bool done_v4 = false;
+      if constexpr (C::kMaxTok % 4 == 0) {
+        if (KS > 1) {
+          // 16-byte stores into the owner's slots (kMaxTok floats per row,
+          // 16-byte aligned): a quarter of the cluster transactions of scalar
+          // stores; slots past M get zeros the reduction never reads
+          done_v4 = true;
+          const uint32_t dst = map_shared_rank(red_addr + slot_off, owner);
 #pragma unroll
-      for (int tok = 0; tok < C::kMaxTok; ++tok) {
-        if (ok && tok < M) {
-          const float acc = __uint_as_float(dv[3 * tok]) + __uint_as_float(dv[3 * tok + 1]) +
-                            __uint_as_float(dv[3 * tok + 2]);
-          const float val = fmaf(acc, exp2i(9 - pexp[tok]), cpart[tok]);
-          const uint32_t off = slot_off + tok * 4u;
-          if (KS > 1) st_shared_cluster_f32(map_shared_rank(red_addr + off, owner), val);
-          else red[off / 4] = val;
+          for (int t4 = 0; t4 < C::kMaxTok; t4 += 4) {
+            if (ok && t4 < M) {
+              float v[4];
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {
+                const int tok = t4 + j;
+                const float acc = __uint_as_float(dv[3 * tok]) + __uint_as_float(dv[3 * tok + 1]) +
+                                  __uint_as_float(dv[3 * tok + 2]);
+                v[j] = tok < M ? fmaf(acc, exp2i(9 - pexp[tok]), cpart[tok]) : 0.f;
+              }
+              asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(dst + 4u * t4), "f"(v[0]),
+                           "f"(v[1]), "f"(v[2]), "f"(v[3])
+                           : "memory");
+            }
+          }
+        }
+      }
+      if (!done_v4) {
+#pragma unroll
+        for (int tok = 0; tok < C::kMaxTok; ++tok) {
+          if (ok && tok < M) {
+            const float acc = __uint_as_float(dv[3 * tok]) + __uint_as_float(dv[3 * tok + 1]) +
+                              __uint_as_float(dv[3 * tok + 2]);
+            const float val = fmaf(acc, exp2i(9 - pexp[tok]), cpart[tok]);
+            const uint32_t off = slot_off + tok * 4u;
+            if (KS > 1) st_shared_cluster_f32(map_shared_rank(red_addr + off, owner), val);
+            else red[off / 4] = val;
+          }
         }
       }
       tc_fence_before();
